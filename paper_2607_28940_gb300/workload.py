@@ -1,0 +1,226 @@
+"""Seeded synthetic workloads for the TransX serving path.
+
+This module only draws numbers: model weights, behavior encodings, serving
+context tokens, candidate tokens and appended behavior rows.  It contains none
+of the method's arithmetic, so both the fp64 oracle (via the tests) and the
+CUDA path consume exactly the same arrays.
+
+Shapes follow the workloads the paper serves (Sec. 4.3: ~500 candidates per
+request on average, long behavior histories, L_local = 10 from Sec. 5.1), with
+distributions stated for the synthetic stand-ins: inputs ~ N(0, 1), weights and
+biases ~ N(0, 0.02), LayerNorm gain 1 + N(0, 0.02) and bias N(0, 0.02).
+
+Random streams.  ``np.random.SeedSequence(seed)`` is split into three
+independent PCG64 streams: one for per-request sizes, one for weights, and one
+parent from which request ``r`` gets its own child stream.  Request ``r``'s data
+therefore depends only on (seed, r, its sizes), which lets a test regenerate a
+subset of requests of a large workload.
+
+Storage rounding.  For bf16 workloads every drawn value is rounded to the
+nearest bf16 (ties to even) and kept as float32, so the oracle sees exactly the
+values the GPU receives.
+
+Weight names follow the paper's notation (Sec. 4.1.2, Sec. 4.1.3, App. B):
+per decoder layer ``l`` the serving-stream attention (``W_qkv``, ``b_qkv``,
+``W_os``, ``b_os``, ``ln1_g``, ``ln1_b``), the cross-attention (``W_Q``,
+``b_Q``, ``W_K``, ``b_K``, ``W_V``, ``b_V``, ``W_oc``, ``b_oc``, ``ln2_g``,
+``ln2_b``) and the FFN (``W_1``, ``b_1``, ``W_2``, ``b_2``, ``ln3_g``,
+``ln3_b``); then the head: ``w_pool``, ``W_dec``, ``b_dec``, ``Q_dec``.
+Matrices are stored in the row-vector convention ``y = x W + b`` with ``W`` of
+shape ``[d_in, d_out]``.
+"""
+from __future__ import annotations
+
+from dataclasses import dataclass, field, replace
+from typing import Dict, List, Optional, Sequence, Tuple, Union
+
+import numpy as np
+
+LAYER_WEIGHTS: Tuple[Tuple[str, str], ...] = (
+    # (name, shape code) in draw order; shape codes resolved by _shape()
+    ("W_qkv", "d,3d"), ("b_qkv", "3d"), ("W_os", "d,d"), ("b_os", "d"),
+    ("ln1_g", "d"), ("ln1_b", "d"),
+    ("W_Q", "d,d"), ("b_Q", "d"), ("W_K", "d,d"), ("b_K", "d"),
+    ("W_V", "d,d"), ("b_V", "d"), ("W_oc", "d,d"), ("b_oc", "d"),
+    ("ln2_g", "d"), ("ln2_b", "d"),
+    ("W_1", "d,F"), ("b_1", "F"), ("W_2", "F,d"), ("b_2", "d"),
+    ("ln3_g", "d"), ("ln3_b", "d"),
+)
+HEAD_WEIGHTS: Tuple[Tuple[str, str], ...] = (
+    ("w_pool", "d"), ("W_dec", "2d,d"), ("b_dec", "d"), ("Q_dec", "k,d"),
+)
+
+SizeSpec = Union[int, Tuple[str, int, int], Sequence[int]]
+
+
+@dataclass(frozen=True)
+class Workload:
+    name: str
+    dtype: str              # "fp32" or "bf16": storage and transfer type
+    n_req: int              # R
+    n_layers: int           # nL decoder layers
+    d_model: int            # d
+    n_heads: int            # H (d_h = d / H)
+    d_ff: int               # F
+    L: SizeSpec             # behavior length per request
+    M: SizeSpec             # candidates per request
+    seed: int
+    n_ctx: int = 2          # S shared serving-context tokens per request
+    n_actions: int = 4      # k action tokens
+    l_local: int = 10       # L_local (Sec. 5.1)
+    ln_eps: float = 1e-5
+    dL: SizeSpec = 0        # appended behavior rows per request
+    capacity_extra: int = 64
+
+    @property
+    def d_head(self) -> int:
+        return self.d_model // self.n_heads
+
+
+# The five workloads: shapes of the paper's serving setting at growing scale.
+WORKLOADS: Dict[str, Workload] = {
+    "tiny_fp32": Workload("tiny_fp32", "fp32", 1, 1, 64, 2, 256, 64, 16, 20261, dL=4),
+    "small_bf16": Workload("small_bf16", "bf16", 32, 2, 256, 8, 1024, 1024, 256, 20262, dL=8),
+    "mid_bf16": Workload("mid_bf16", "bf16", 64, 4, 512, 8, 2048, 4096, 512, 20263, dL=8),
+    "ragged_bf16": Workload("ragged_bf16", "bf16", 64, 4, 512, 8, 2048,
+                            ("uniform", 1024, 16384), 1000, 20264, dL=8),
+    "sweep_bf16": Workload("sweep_bf16", "bf16", 16, 4, 512, 8, 2048, 8192, 1024, 20265,
+                           dL=("uniform", 1, 64)),
+}
+
+
+def _streams(seed: int):
+    ss = np.random.SeedSequence(seed)
+    s_sizes, s_weights, s_data = ss.spawn(3)
+    return s_sizes, s_weights, s_data
+
+
+def round_bf16(x: np.ndarray) -> np.ndarray:
+    """Round float32 values to the nearest bf16 (ties to even), as float32."""
+    x = np.ascontiguousarray(x, dtype=np.float32)
+    u = x.view(np.uint32).astype(np.uint64)
+    lsb = (u >> 16) & 1
+    r = ((u + 0x7FFF + lsb) >> 16) << 16
+    out = (r & 0xFFFFFFFF).astype(np.uint32).view(np.float32)
+    nan = np.isnan(x)
+    if nan.any():
+        out = out.copy()
+        out[nan] = np.float32("nan")
+    return out
+
+
+def _store(wl: Workload, x: np.ndarray) -> np.ndarray:
+    x = np.asarray(x, dtype=np.float32)
+    return round_bf16(x) if wl.dtype == "bf16" else x
+
+
+def _draw_sizes(spec: SizeSpec, n: int, rng: np.random.Generator) -> np.ndarray:
+    if isinstance(spec, (int, np.integer)):
+        return np.full(n, int(spec), dtype=np.int64)
+    if isinstance(spec, tuple) and len(spec) == 3 and spec[0] == "uniform":
+        lo, hi = int(spec[1]), int(spec[2])
+        return rng.integers(lo, hi + 1, size=n).astype(np.int64)  # inclusive bounds
+    arr = np.asarray(spec, dtype=np.int64)
+    if arr.shape != (n,):
+        raise ValueError(f"size list has shape {arr.shape}, expected ({n},)")
+    return arr
+
+
+def sizes(wl: Workload) -> Tuple[np.ndarray, np.ndarray, np.ndarray]:
+    """Per-request (L_r, M_r, dL_r), drawn from the size stream in that order."""
+    s_sizes, _, _ = _streams(wl.seed)
+    rng = np.random.default_rng(s_sizes)
+    L = _draw_sizes(wl.L, wl.n_req, rng)
+    M = _draw_sizes(wl.M, wl.n_req, rng)
+    dL = _draw_sizes(wl.dL, wl.n_req, rng)
+    return L, M, dL
+
+
+def _shape(code: str, wl: Workload) -> Tuple[int, ...]:
+    env = {"d": wl.d_model, "3d": 3 * wl.d_model, "2d": 2 * wl.d_model,
+           "F": wl.d_ff, "k": wl.n_actions}
+    return tuple(env[c] for c in code.split(","))
+
+
+def weights(wl: Workload) -> Dict[str, np.ndarray]:
+    """All model weights.  Per-layer names get the suffix ``.<l>``."""
+    _, s_weights, _ = _streams(wl.seed)
+    rng = np.random.default_rng(s_weights)
+    out: Dict[str, np.ndarray] = {}
+    for l in range(wl.n_layers):
+        for name, code in LAYER_WEIGHTS:
+            shp = _shape(code, wl)
+            x = rng.standard_normal(shp) * 0.02
+            if name.endswith("_g"):
+                x = 1.0 + x
+            out[f"{name}.{l}"] = _store(wl, x)
+    for name, code in HEAD_WEIGHTS:
+        out[name] = _store(wl, rng.standard_normal(_shape(code, wl)) * 0.02)
+    return out
+
+
+@dataclass
+class Batch:
+    """One synthetic serving batch, packed request after request.
+
+    ``beh``  [sum L_r, d]  encoded behavior rows Phi_b (Sec. 4.1.2)
+    ``ctx``  [R, S, d]     serving-context tokens (App. B)
+    ``cand`` [sum M_r, d]  candidate tokens Phi_c rows (Sec. 4.1.2)
+    ``app``  [sum dL_r, d] behavior rows appended after the cache build (App. D)
+    Offsets are exclusive prefix sums with a leading 0.
+    """
+    beh: np.ndarray
+    beh_off: np.ndarray
+    ctx: np.ndarray
+    cand: np.ndarray
+    cand_off: np.ndarray
+    app: np.ndarray
+    app_off: np.ndarray
+    L: np.ndarray
+    M: np.ndarray
+    dL: np.ndarray
+    requests: np.ndarray = field(default_factory=lambda: np.zeros(0, np.int64))
+
+
+def _offsets(n: np.ndarray) -> np.ndarray:
+    off = np.zeros(len(n) + 1, dtype=np.int32)
+    off[1:] = np.cumsum(n)
+    return off
+
+
+def batch(wl: Workload, requests: Optional[Sequence[int]] = None,
+          M_override: Optional[int] = None) -> Batch:
+    """Draw the batch, or only the listed ``requests`` (same values as in the full batch).
+
+    Per request ``r`` the draw order is: Phi_b rows, context rows, candidate
+    rows, appended rows.  ``M_override`` replaces every M_r (used by the
+    candidate-count sweep; the drawn values then differ from the default M).
+    """
+    Ls, Ms, dLs = sizes(wl)
+    if M_override is not None:
+        Ms = np.full_like(Ms, int(M_override))
+    reqs = np.arange(wl.n_req) if requests is None else np.asarray(requests, dtype=np.int64)
+    _, _, s_data = _streams(wl.seed)
+    children = s_data.spawn(wl.n_req)
+    d, S = wl.d_model, wl.n_ctx
+    beh, ctx, cand, app = [], [], [], []
+    for r in reqs:
+        rng = np.random.default_rng(children[int(r)])
+        beh.append(rng.standard_normal((int(Ls[r]), d), dtype=np.float32))
+        ctx.append(rng.standard_normal((S, d), dtype=np.float32))
+        cand.append(rng.standard_normal((int(Ms[r]), d), dtype=np.float32))
+        app.append(rng.standard_normal((int(dLs[r]), d), dtype=np.float32))
+    L, M, dL = Ls[reqs], Ms[reqs], dLs[reqs]
+    cat = lambda xs: _store(wl, np.concatenate(xs, axis=0)) if xs else np.zeros((0, d), np.float32)
+    return Batch(
+        beh=cat(beh), beh_off=_offsets(L),
+        ctx=_store(wl, np.stack(ctx, 0)) if ctx else np.zeros((0, S, d), np.float32),
+        cand=cat(cand), cand_off=_offsets(M),
+        app=cat(app), app_off=_offsets(dL),
+        L=L, M=M, dL=dL, requests=reqs,
+    )
+
+
+def with_sizes(wl: Workload, **kw) -> Workload:
+    """A copy of ``wl`` with some fields replaced (e.g. a smaller L or M)."""
+    return replace(wl, **kw)
