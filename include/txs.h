@@ -1,0 +1,213 @@
+/*
+ * txs.h — C ABI of libtxs, the GB300 (sm_103a) serving path of TransX:
+ * amortised behavior K/V caching and multi-candidate next-action decoding.
+ *
+ * Paper: "TransX: Scaling Transformer-based Recommendation via Behavioral and
+ * Serving Stream Crossings" (KDD '26), arXiv 2607.28940.
+ *
+ * Conventions for every entry point
+ * ---------------------------------
+ * - Row-vector convention y = x W + b; matrices are row-major.
+ * - "device" pointers are CUDA device (or managed) memory owned by the caller;
+ *   the library never frees them.  "host" pointers are ordinary host memory,
+ *   read before the call returns.
+ * - Floating-point storage type of weights, behavior rows and tokens is the
+ *   model's dtype (TXS_FP32: float, TXS_BF16: bfloat16).  Outputs of scores are
+ *   always float.
+ * - `stream` is a cudaStream_t passed as void* (NULL = legacy default stream).
+ *   Every call enqueues its work on that stream and returns without waiting;
+ *   argument errors are detected on the host and returned before anything is
+ *   enqueued.  Errors found by kernels (bounds, timeouts) are latched in a
+ *   per-model device status word read by txs_device_status().
+ * - No entry point throws; all return txs_status.
+ * - Handles (txs_model, txs_kv_cache) own the device memory they allocate at
+ *   create/build time and free it in the matching destroy call.
+ * - Calls on the same handle must be ordered by the caller (same stream, or
+ *   events); the library does not lock.
+ */
+#ifndef TXS_H
+#define TXS_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  TXS_OK = 0,
+  TXS_ERR_INVALID_ARG = 1,    /* bad pointer, size, offset array or config      */
+  TXS_ERR_COLD_START = 2,     /* a request has no behavior rows (App. D)         */
+  TXS_ERR_CAPACITY = 3,       /* append exceeds the cache's spare capacity       */
+  TXS_ERR_STALE_CACHE = 4,    /* cache built by a model with other weights/config*/
+  TXS_ERR_CUDA = 5,           /* a CUDA runtime/driver call failed               */
+  TXS_ERR_DEVICE_TIMEOUT = 6, /* a bounded device-side wait gave up              */
+  TXS_ERR_BOUNDS = 7,         /* a kernel saw an index outside its buffers       */
+  TXS_ERR_UNSUPPORTED = 8     /* shape outside what the kernels implement        */
+} txs_status;
+
+typedef enum { TXS_FP32 = 0, TXS_BF16 = 1 } txs_dtype;
+
+/* Key set of the cross-attention (Sec. 4.1.2 local-global sparse set):
+ * LOCAL_GLOBAL = the l_local most recent behavior rows plus the attention-pooled
+ * global anchor; FULL = every cached row, no anchor (the -sparseAttn ablation,
+ * Sec. 5.2). */
+typedef enum { TXS_ATTN_LOCAL_GLOBAL = 0, TXS_ATTN_FULL = 1 } txs_attn_mode;
+
+typedef struct {
+  int32_t d_model;   /* d; multiple of 64 for TXS_BF16, of 32 for TXS_FP32; <= 512 */
+  int32_t n_heads;   /* H; d_head = d_model / n_heads must be 32 or 64             */
+  int32_t d_ff;      /* F; multiple of 64                                         */
+  int32_t n_layers;  /* decoder layers, >= 1                                      */
+  int32_t n_actions; /* k action tokens (Sec. 4.1.3), 1..16                       */
+  int32_t n_ctx;     /* S serving-context tokens per request (App. B), 0..8       */
+  int32_t l_local;   /* L_local (Sec. 4.1.2), >= 1                                */
+  int32_t attn_mode; /* txs_attn_mode                                             */
+  int32_t dtype;     /* txs_dtype                                                 */
+  float ln_eps;      /* LayerNorm epsilon (> 0)                                   */
+} txs_config;
+
+typedef struct txs_model txs_model;       /* opaque */
+typedef struct txs_kv_cache txs_kv_cache; /* opaque */
+
+/* Number of per-layer weight tensors and of head tensors in the `weights`
+ * array of txs_model_create. */
+#define TXS_WEIGHTS_PER_LAYER 22
+#define TXS_HEAD_WEIGHTS 4
+
+/*
+ * txs_model_create — copy the decoder weights into the library's device layout.
+ *
+ * `weights` (host array of device pointers) holds n_layers * 22 + 4 pointers,
+ * layer by layer, then the head, in this order and with these shapes
+ * (d = d_model, F = d_ff, k = n_actions), all in the config's dtype:
+ *   per layer l (Sec. 4.1.2 crossAttend block; App. B serving-stream attention):
+ *     0 W_qkv [d,3d]  1 b_qkv [3d]   2 W_os [d,d]  3 b_os [d]  4 ln1_g [d] 5 ln1_b [d]
+ *     6 W_Q  [d,d]    7 b_Q  [d]     8 W_K [d,d]   9 b_K [d]  10 W_V [d,d] 11 b_V [d]
+ *    12 W_oc [d,d]   13 b_oc [d]    14 ln2_g [d]  15 ln2_b [d]
+ *    16 W_1  [d,F]   17 b_1  [F]    18 W_2 [F,d]  19 b_2 [d]  20 ln3_g [d] 21 ln3_b [d]
+ *   head (Sec. 4.1.3; attention pooling Sec. 5.1):
+ *     w_pool [d], W_dec [2d,d], b_dec [d], Q_dec [k,d]
+ * The call synchronises the device first (the weights may still be in flight
+ * on any stream) and returns after the copies are done; the inputs may be
+ * freed afterwards.  The model keeps a 64-bit content hash of config and weights.
+ * Errors: TXS_ERR_INVALID_ARG, TXS_ERR_UNSUPPORTED, TXS_ERR_CUDA.
+ */
+txs_status txs_model_create(const txs_config* cfg, const void* const* weights, txs_model** out);
+void txs_model_destroy(txs_model* model);
+/* Content hash of config + weights (identical weights give identical hashes). */
+uint64_t txs_model_hash(const txs_model* model);
+
+/*
+ * txs_build_kv_cache — nearline cache build (Sec. 4.3, amortised encoding and
+ * KV caching; Sec. 4.1.2 K = Phi_b W_K, V = Phi_b W_V).
+ *
+ * For each request r the rows beh_enc[beh_offsets[r] .. beh_offsets[r+1]) are
+ * the encoded behavior stream Phi_b (row-major [sum L_r, d_model], device).
+ * For every layer l the cache stores K_l = Phi_b W_K^l + b_K^l and
+ * V_l = Phi_b W_V^l + b_V^l in the model dtype, plus the attention-pooled
+ * anchor g = softmax(Phi_b w_pool / sqrt(d))^T Phi_b and its projections.
+ * `beh_offsets` is a host int32 array [n_req + 1], offsets[0] == 0, strictly
+ * increasing (every request needs >= 1 row, else TXS_ERR_COLD_START).
+ * `capacity_extra` >= 0 spare rows per request are reserved for appends.
+ * Allocates the cache (device memory) and returns it in *out.
+ */
+txs_status txs_build_kv_cache(txs_model* model, int32_t n_req, const int32_t* beh_offsets,
+                              const void* beh_enc, int32_t capacity_extra, void* stream,
+                              txs_kv_cache** out);
+void txs_cache_destroy(txs_kv_cache* cache);
+
+/*
+ * txs_append_behavior — incremental update (App. D, incremental-encoding
+ * remark): rows new_enc[new_offsets[r] .. new_offsets[r+1]) (device, model
+ * dtype, [sum dL_r, d_model]) are projected into the free slots after request
+ * r's current rows; existing rows are untouched; the pooled anchor is merged
+ * with the new rows (online softmax) and re-projected.  dL_r may be 0.
+ * `new_offsets` host int32 [n_req + 1]; n_req must equal the cache's.
+ * Errors: TXS_ERR_CAPACITY if any request would exceed its capacity (nothing
+ * is changed), TXS_ERR_STALE_CACHE, TXS_ERR_INVALID_ARG.
+ */
+txs_status txs_append_behavior(txs_model* model, txs_kv_cache* cache, int32_t n_req,
+                               const int32_t* new_offsets, const void* new_enc, void* stream);
+
+/* Copy rows row0 .. row0+n_rows-1 of request `req`'s cached K (which = 0) or
+ * V (which = 1) of layer `layer` into dst (device, model dtype, [n_rows, d]),
+ * asynchronously on `stream`.  Rows must be < the request's current length. */
+txs_status txs_cache_read_rows(const txs_kv_cache* cache, int32_t layer, int32_t which, int32_t req, int32_t row0,
+                               int32_t n_rows, void* dst, void* stream);
+/* Copy the anchor's projected key (which = 0) or value (which = 1) of `layer`
+ * for all requests, or the pooled anchor g itself (which = 2, layer ignored),
+ * into dst (device, float, [n_req, d]). */
+txs_status txs_cache_read_anchor(const txs_kv_cache* cache, int32_t layer, int32_t which, float* dst, void* stream);
+
+/* Current per-request lengths L_r (host int32 [n_req]) and request count. */
+txs_status txs_cache_lengths(const txs_kv_cache* cache, int32_t* out_len);
+int32_t txs_cache_n_req(const txs_kv_cache* cache);
+
+/*
+ * txs_score_workspace_size — bytes of device scratch txs_score_candidates needs
+ * for n_req requests with total_cand candidates in all (256-byte aligned start).
+ */
+txs_status txs_score_workspace_size(const txs_model* model, int32_t n_req, int64_t total_cand,
+                                    size_t* bytes);
+
+/*
+ * txs_score_candidates — multi-candidate next-action decoding against the
+ * cache (Sec. 4.1.2 multi-query cross-attention sharing K/V across the m
+ * candidates; Sec. 4.1.3 parallel grouped decoding and the action softmax).
+ *
+ * Request r has candidates cand_tok[cand_offsets[r] .. cand_offsets[r+1])
+ * (device, model dtype, [sum M_r, d_model]; M_r >= 0) and n_ctx context tokens
+ * ctx_tok[r] (device, [n_req, n_ctx, d_model]; may be NULL iff n_ctx == 0).
+ * Every decoder layer runs serving-stream attention (context rows attend to
+ * the context rows, a candidate to the context rows and itself), cross-
+ * attention to the cached key set, and the FFN, each post-LN with a residual.
+ * Outputs (device, float, [sum M_r, n_actions]): out_logits = Q_dec k_dec with
+ * k_dec = [z, x] W_dec + b_dec, and out_probs = softmax(out_logits) (may be NULL).
+ * `workspace` (device, >= txs_score_workspace_size bytes, 256-byte aligned)
+ * is scratch owned by the caller; its contents are overwritten.
+ * `cand_offsets` host int32 [n_req + 1]; n_req must equal the cache's.
+ * Errors: TXS_ERR_STALE_CACHE if the cache came from a model with another hash.
+ */
+txs_status txs_score_candidates(txs_model* model, const txs_kv_cache* cache, int32_t n_req,
+                                const int32_t* cand_offsets, const void* cand_tok,
+                                const void* ctx_tok, void* workspace, size_t workspace_bytes,
+                                float* out_logits, float* out_probs, void* stream);
+
+/*
+ * txs_rank_candidates — per request, candidate indices (local to the request)
+ * sorted by descending probs[:, action]; ties go to the lower index and NaN
+ * scores rank last.  `probs` device float [sum M_r, n_actions].
+ * top_k == 0: out_idx is device int32 [sum M_r], request r's ranking at
+ * out_idx[cand_offsets[r] ...].  top_k > 0: out_idx is [n_req, top_k], padded
+ * with -1 when M_r < top_k.  Requires M_r <= 32768.
+ */
+txs_status txs_rank_candidates(int32_t n_req, const int32_t* cand_offsets, const float* probs,
+                               int32_t n_actions, int32_t action, int32_t top_k, int32_t* out_idx,
+                               void* stream);
+
+/* Synchronise the device, read and clear the model's latched device status. */
+txs_status txs_device_status(txs_model* model);
+
+/* Process-wide per-kernel-class timing with CUDA events on the launching
+ * stream (off by default).  While enabled, every library launch is bracketed
+ * by two events; txs_profile_collect synchronises, writes per-class total
+ * milliseconds and launch counts (host arrays of length n >=
+ * TXS_N_KERNEL_CLASSES) and clears the record.  Not thread-safe; not for use
+ * during CUDA-graph capture. */
+#define TXS_N_KERNEL_CLASSES 16
+txs_status txs_profile_enable(int32_t enable);
+txs_status txs_profile_collect(double* total_ms, int64_t* launches, int32_t n);
+const char* txs_kernel_class_name(int32_t cls);
+
+const char* txs_status_string(txs_status s);
+/* Text of the last host-side failure of this thread (a CUDA error string or
+ * the config field that was rejected); empty if none. */
+const char* txs_last_error(void);
+const char* txs_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* TXS_H */

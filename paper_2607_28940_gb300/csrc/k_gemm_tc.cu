@@ -1,0 +1,539 @@
+// Tensor-core GEMM for sm_103a with fused epilogues: C = A B^T (+ epilogue).
+//
+// A [M, K] bf16 row-major (activations or behavior rows), B [N, K] bf16
+// row-major (a transposed weight, K-major), fp32 accumulation in TMEM.
+// Used by every dense projection of the path: the cache build K/V projection
+// (Sec. 4.1.2, K = Phi_b W_K, V = Phi_b W_V), the serving-attention QKV, the
+// cross-attention query, the output projections with residual + LayerNorm
+// (Sec. 4.1.2 crossAttend equation) and the FFN with GELU.
+//
+// One CTA computes a 128 x BN tile: warp 0 streams A/B tiles with TMA into a
+// STAGES-deep ring of 128-byte-swizzled shared-memory buffers, warp 1 issues
+// tcgen05.mma (M=128, N<=256 per instruction, K=16) into TMEM, warps 2-5 read
+// the accumulator back with tcgen05.ld (one row per thread) and run the
+// epilogue.  All waits are bounded; a timeout latches TXS_ERR_DEVICE_TIMEOUT.
+#include <cstdio>
+
+#include "txs_internal.cuh"
+
+namespace txs {
+namespace tc {
+
+constexpr int BM = 128;
+constexpr int BK = 64;                        // 64 bf16 = one 128-byte swizzle row
+constexpr int A_STAGE_BYTES = BM * BK * 2;    // 16 KB
+constexpr int NUM_THREADS = 192;
+
+// ------------------------------------------------------------------ PTX wrappers
+
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count) : "memory");
+}
+
+__device__ __forceinline__ void mbar_expect_tx(uint64_t* bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)), "r"(bytes)
+               : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(smem_u32(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+
+// Wait for the phase of `parity` to complete; gives up (returning false) when
+// another role raised *abort or after kSpinCycles, raising *abort itself.
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort) {
+  const long long t0 = clock64();
+  while (!mbar_try_wait(bar, parity)) {
+    if (*abort) return false;
+    if (clock64() - t0 > kSpinCycles) {
+      *abort = 1;
+      return false;
+    }
+  }
+  return true;
+}
+
+__device__ __forceinline__ bool mbar_wait_plain(uint64_t* bar, uint32_t parity) {
+  const long long t0 = clock64();
+  while (!mbar_try_wait(bar, parity))
+    if (clock64() - t0 > kSpinCycles) return false;
+  return true;
+}
+
+__device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* tm, uint64_t* bar, int x, int y) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%3, %4}], [%2];" ::"r"(
+          smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(tm)), "r"(smem_u32(bar)), "r"(x), "r"(y)
+      : "memory");
+}
+
+__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
+
+__device__ __forceinline__ void tmem_alloc(uint32_t* holder, uint32_t ncols) {
+  asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(holder)), "r"(ncols)
+               : "memory");
+  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+}
+
+__device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
+  asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols) : "memory");
+}
+
+// Shared-memory matrix descriptor: K-major tile written by TMA with 128-byte
+// swizzle; 8-row core-matrix groups 1024 bytes apart (SBO); LBO unused for this
+// layout (set to 16 bytes); descriptor version 1; layout code 2 = SWIZZLE_128B.
+__device__ __forceinline__ uint64_t sdesc_sw128(uint32_t saddr) {
+  uint64_t d = 0;
+  d |= static_cast<uint64_t>((saddr & 0x3FFFFu) >> 4);
+  d |= static_cast<uint64_t>(16 >> 4) << 16;
+  d |= static_cast<uint64_t>(1024 >> 4) << 32;
+  d |= 1ull << 46;
+  d |= 2ull << 61;
+  return d;
+}
+
+// Instruction descriptor, kind::f16: D fp32, A and B bf16, both K-major.
+__host__ __device__ constexpr uint32_t idesc_bf16(int m, int n) {
+  return (1u << 4) | (1u << 7) | (1u << 10) | (static_cast<uint32_t>(n >> 3) << 17) |
+         (static_cast<uint32_t>(m >> 4) << 24);
+}
+
+__device__ __forceinline__ void mma_bf16(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
+                                         uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+
+__device__ __forceinline__ void mma_commit(uint64_t* bar) {
+  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(smem_u32(bar))
+               : "memory");
+}
+
+// 32 consecutive fp32 accumulator columns of this thread's TMEM lane.
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, float* v) {
+  uint32_t r[32];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
+      "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
+      "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];\n\t"
+      "tcgen05.wait::ld.sync.aligned;"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+        "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]),
+        "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]),
+        "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+      : "r"(taddr)
+      : "memory");
+#pragma unroll
+  for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+__device__ __forceinline__ void tmem_st32(uint32_t taddr, const float* v) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], "
+      "{%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,"
+      "%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,%32};\n\t"
+      "tcgen05.wait::st.sync.aligned;" ::"r"(taddr),
+      "r"(__float_as_uint(v[0])), "r"(__float_as_uint(v[1])), "r"(__float_as_uint(v[2])),
+      "r"(__float_as_uint(v[3])), "r"(__float_as_uint(v[4])), "r"(__float_as_uint(v[5])),
+      "r"(__float_as_uint(v[6])), "r"(__float_as_uint(v[7])), "r"(__float_as_uint(v[8])),
+      "r"(__float_as_uint(v[9])), "r"(__float_as_uint(v[10])), "r"(__float_as_uint(v[11])),
+      "r"(__float_as_uint(v[12])), "r"(__float_as_uint(v[13])), "r"(__float_as_uint(v[14])),
+      "r"(__float_as_uint(v[15])), "r"(__float_as_uint(v[16])), "r"(__float_as_uint(v[17])),
+      "r"(__float_as_uint(v[18])), "r"(__float_as_uint(v[19])), "r"(__float_as_uint(v[20])),
+      "r"(__float_as_uint(v[21])), "r"(__float_as_uint(v[22])), "r"(__float_as_uint(v[23])),
+      "r"(__float_as_uint(v[24])), "r"(__float_as_uint(v[25])), "r"(__float_as_uint(v[26])),
+      "r"(__float_as_uint(v[27])), "r"(__float_as_uint(v[28])), "r"(__float_as_uint(v[29])),
+      "r"(__float_as_uint(v[30])), "r"(__float_as_uint(v[31]))
+      : "memory");
+}
+
+// ------------------------------------------------------------------ epilogues
+
+__device__ __forceinline__ void load_bias32(const float* bias, int n, float* b) {
+  const float4* p = reinterpret_cast<const float4*>(bias + n);
+#pragma unroll
+  for (int j = 0; j < 8; ++j) {
+    float4 t = __ldg(p + j);
+    b[4 * j] = t.x; b[4 * j + 1] = t.y; b[4 * j + 2] = t.z; b[4 * j + 3] = t.w;
+  }
+}
+
+__device__ __forceinline__ void store_bf16x32(__nv_bfloat16* p, const float* v) {
+#pragma unroll
+  for (int j = 0; j < 4; ++j) Vec16<__nv_bfloat16>::store(p + 8 * j, v + 8 * j);
+}
+
+__device__ __forceinline__ void load_bf16x32(const __nv_bfloat16* p, float* v) {
+#pragma unroll
+  for (int j = 0; j < 4; ++j) Vec16<__nv_bfloat16>::load(p + 8 * j, v + 8 * j);
+}
+
+template <int BN, int EPI>
+__device__ __forceinline__ void epilogue(const EpiArgs& e, uint32_t tlane, int row, int n0) {
+  const bool valid = row < e.M;
+  float v[32];
+  if constexpr (EPI == EPI_BIAS || EPI == EPI_BIAS_GELU || EPI == EPI_KV) {
+    __nv_bfloat16* out = nullptr;
+    if (valid) {
+      long long orow = row;
+      long long ocol = n0;
+      if constexpr (EPI == EPI_KV) {
+        const int r = find_segment(e.seg_off, e.n_seg, row);
+        orow = static_cast<long long>(__ldg(e.dst_row0 + r)) + (row - __ldg(e.seg_off + r));
+        const int blk = n0 / e.col_blk;
+        ocol = static_cast<long long>(blk) * e.col_blk_stride + (n0 - blk * e.col_blk);
+      }
+      out = static_cast<__nv_bfloat16*>(e.out) + orow * e.ldo + ocol;
+    }
+#pragma unroll 1
+    for (int c = 0; c < BN; c += 32) {
+      tmem_ld32(tlane + c, v);
+      if (valid) {
+        float b[32];
+        load_bias32(e.bias, n0 + c, b);
+#pragma unroll
+        for (int i = 0; i < 32; ++i) {
+          float x = v[i] + b[i];
+          if constexpr (EPI == EPI_BIAS_GELU) x = gelu_erf(x);
+          v[i] = x;
+        }
+        store_bf16x32(out + c, v);
+      }
+    }
+  } else {
+    // Row-wise LayerNorm over the full row (BN == N): two passes over TMEM,
+    // the pre-norm values written back in place by the first pass.
+    const __nv_bfloat16* res = valid ? static_cast<const __nv_bfloat16*>(e.res) + row * e.ldr : nullptr;
+    float sum = 0.f;
+#pragma unroll 1
+    for (int c = 0; c < BN; c += 32) {
+      tmem_ld32(tlane + c, v);
+      float b[32], r[32];
+      load_bias32(e.bias, c, b);
+      if (valid) load_bf16x32(res + c, r);
+      else {
+#pragma unroll
+        for (int i = 0; i < 32; ++i) r[i] = 0.f;
+      }
+#pragma unroll
+      for (int i = 0; i < 32; ++i) {
+        v[i] += b[i] + r[i];
+        sum += v[i];
+      }
+      tmem_st32(tlane + c, v);
+    }
+    const float mean = sum / static_cast<float>(BN);
+    float sq = 0.f;
+#pragma unroll 1
+    for (int c = 0; c < BN; c += 32) {
+      tmem_ld32(tlane + c, v);
+#pragma unroll
+      for (int i = 0; i < 32; ++i) {
+        const float t = v[i] - mean;
+        sq += t * t;
+      }
+    }
+    const float rstd = rsqrtf(sq / static_cast<float>(BN) + e.ln_eps);
+    float lg[16];
+#pragma unroll
+    for (int a = 0; a < 16; ++a) lg[a] = 0.f;
+    __nv_bfloat16* out = nullptr;
+    if constexpr (EPI == EPI_LN) {
+      if (valid) out = static_cast<__nv_bfloat16*>(e.out) + row * e.ldo;
+    }
+#pragma unroll 1
+    for (int c = 0; c < BN; c += 32) {
+      tmem_ld32(tlane + c, v);
+      float g[32], bt[32];
+      load_bias32(e.gamma, c, g);
+      load_bias32(e.beta, c, bt);
+#pragma unroll
+      for (int i = 0; i < 32; ++i) v[i] = (v[i] - mean) * rstd * g[i] + bt[i];
+      if constexpr (EPI == EPI_LN) {
+        if (valid) store_bf16x32(out + c, v);
+      } else {
+        const int na = e.n_act;
+#pragma unroll 4
+        for (int i = 0; i < 32; ++i) {
+          const float* w = e.weff_z + static_cast<long long>(c + i) * na;
+#pragma unroll
+          for (int a = 0; a < 16; ++a)
+            if (a < na) lg[a] = fmaf(v[i], __ldg(w + a), lg[a]);
+        }
+      }
+    }
+    if constexpr (EPI == EPI_LN_HEAD) {
+      if (valid && row < e.n_cand_rows) {
+        const int na = e.n_act;
+        float mx = -INFINITY;
+#pragma unroll
+        for (int a = 0; a < 16; ++a)
+          if (a < na) {
+            lg[a] += __ldg(e.xlog + static_cast<long long>(row) * na + a);
+            mx = fmaxf(mx, lg[a]);
+          }
+        float s = 0.f, p[16];
+#pragma unroll
+        for (int a = 0; a < 16; ++a)
+          if (a < na) {
+            p[a] = expf(lg[a] - mx);
+            s += p[a];
+          }
+        const float inv = 1.f / s;
+#pragma unroll
+        for (int a = 0; a < 16; ++a)
+          if (a < na) {
+            e.logits[static_cast<long long>(row) * na + a] = lg[a];
+            if (e.probs) e.probs[static_cast<long long>(row) * na + a] = p[a] * inv;
+          }
+      }
+    }
+  }
+}
+
+// ------------------------------------------------------------------ kernel
+
+template <int BN>
+struct Shape {
+  static constexpr int BN_MMA = BN < 256 ? BN : 256;     // N of one tcgen05.mma
+  static constexpr int B_BOX = BN_MMA;                    // rows of one TMA box of B
+  static constexpr int B_STAGE_BYTES = BN * BK * 2;
+  static constexpr int STAGE_BYTES = A_STAGE_BYTES + B_STAGE_BYTES;
+  static constexpr int STAGES = (BN >= 512) ? 2 : (196608 / STAGE_BYTES);
+  static constexpr int TMEM_COLS = BN < 32 ? 32 : BN;
+  static constexpr int SMEM_BYTES = STAGES * STAGE_BYTES + 1024 + 256;
+  static_assert(SMEM_BYTES <= 232448, "shared memory");
+  static_assert((TMEM_COLS & (TMEM_COLS - 1)) == 0 && TMEM_COLS <= 512, "TMEM columns");
+};
+
+template <int BN, int EPI>
+__global__ void __launch_bounds__(NUM_THREADS, 1)
+    gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                   const EpiArgs e) {
+  using S = Shape<BN>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint8_t* sA = smem;
+  uint8_t* sB = smem + S::STAGES * A_STAGE_BYTES;
+  uint64_t* full = reinterpret_cast<uint64_t*>(sB + S::STAGES * S::B_STAGE_BYTES);
+  uint64_t* empty = full + S::STAGES;
+  uint64_t* accum = empty + S::STAGES;
+  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(accum + 1);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_holder + 1);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int m0 = blockIdx.x * BM;
+  const int n0 = blockIdx.y * BN;
+  const int num_kb = e.K / BK;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < S::STAGES; ++s) {
+      mbar_init(full + s, 1);
+      mbar_init(empty + s, 1);
+    }
+    mbar_init(accum, 1);
+    *abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == 1) tmem_alloc(tmem_holder, S::TMEM_COLS);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_holder;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmA)) : "memory");
+      asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmB)) : "memory");
+      int issued = 0;
+      for (int kb = 0; kb < num_kb; ++kb) {
+        const int s = kb % S::STAGES;
+        const uint32_t ph = (kb / S::STAGES) & 1;
+        if (!mbar_wait(empty + s, ph ^ 1, abort_flag)) break;
+        mbar_expect_tx(full + s, S::STAGE_BYTES);
+        tma_load_2d(sA + s * A_STAGE_BYTES, &tmA, full + s, kb * BK, m0);
+#pragma unroll
+        for (int j = 0; j < BN; j += S::B_BOX)
+          tma_load_2d(sB + s * S::B_STAGE_BYTES + j * (BK * 2), &tmB, full + s, kb * BK, n0 + j);
+        issued = kb + 1;
+      }
+      if (*abort_flag) {
+        // let the copies already in flight land before shared memory is released
+        for (int kb = issued > S::STAGES ? issued - S::STAGES : 0; kb < issued; ++kb)
+          mbar_wait_plain(full + kb % S::STAGES, (kb / S::STAGES) & 1);
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      constexpr uint32_t idesc = idesc_bf16(BM, S::BN_MMA);
+      for (int kb = 0; kb < num_kb; ++kb) {
+        const int s = kb % S::STAGES;
+        const uint32_t ph = (kb / S::STAGES) & 1;
+        if (!mbar_wait(full + s, ph, abort_flag)) break;
+        tc_fence_after();
+        const uint64_t adesc = sdesc_sw128(smem_u32(sA + s * A_STAGE_BYTES));
+        const uint64_t bdesc = sdesc_sw128(smem_u32(sB + s * S::B_STAGE_BYTES));
+#pragma unroll
+        for (int k = 0; k < BK / 16; ++k) {
+#pragma unroll
+          for (int j = 0; j < BN / S::BN_MMA; ++j) {
+            // advance 32 bytes along K inside the swizzle row; N halves are
+            // S::BN_MMA rows (x 128 bytes) apart
+            const uint64_t boff = static_cast<uint64_t>((j * S::BN_MMA * BK * 2) >> 4);
+            mma_bf16(tmem + j * S::BN_MMA, adesc + 2 * k, bdesc + boff + 2 * k, idesc,
+                     (kb > 0 || k > 0) ? 1u : 0u);
+          }
+        }
+        mma_commit(empty + s);
+      }
+      mma_commit(accum);
+    }
+  } else {
+    const int q = warp & 3;
+    const int row = m0 + q * 32 + lane;
+    bool go = mbar_wait(accum, 0, abort_flag);
+    go = go && !*abort_flag;
+    go = __shfl_sync(0xffffffffu, go ? 1 : 0, 0) != 0;  // warp-uniform: tcgen05.ld is .sync.aligned
+    tc_fence_after();
+    if (go) epilogue<BN, EPI>(e, tmem + (static_cast<uint32_t>(q * 32) << 16), row, n0);
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, S::TMEM_COLS);
+  }
+  if (threadIdx.x == 0 && *abort_flag) latch_status(e.status, TXS_ERR_DEVICE_TIMEOUT);
+}
+
+// ------------------------------------------------------------------ host side
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                  const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+static EncodeTiledFn encode_fn() {
+  static EncodeTiledFn fn = nullptr;
+  if (!fn) {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(p);
+  }
+  return fn;
+}
+
+// 2-D bf16 tensor map over a row-major [rows, cols] matrix with leading
+// dimension ld (elements), box {64 columns, box_rows rows}, 128-byte swizzle.
+static bool make_tmap(CUtensorMap* tm, const void* base, long long rows, long long cols, long long ld,
+                      int box_rows) {
+  EncodeTiledFn fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[2] = {static_cast<cuuint64_t>(cols), static_cast<cuuint64_t>(rows)};
+  cuuint64_t strides[1] = {static_cast<cuuint64_t>(ld) * 2};
+  cuuint32_t box[2] = {static_cast<cuuint32_t>(BK), static_cast<cuuint32_t>(box_rows)};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = fn(tm, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
+template <int BN, int EPI>
+static cudaError_t launch_bn(const __nv_bfloat16* A, long long lda, const __nv_bfloat16* B, const EpiArgs& e,
+                             cudaStream_t s, int cls) {
+  using Sh = Shape<BN>;
+  static bool attr_set = false;
+  if (!attr_set) {
+    cudaError_t err = cudaFuncSetAttribute(gemm_tc_kernel<BN, EPI>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                           Sh::SMEM_BYTES);
+    if (err != cudaSuccess) return err;
+    attr_set = true;
+  }
+  CUtensorMap ta, tb;
+  if (!make_tmap(&ta, A, e.M, e.K, lda, BM)) return cudaErrorInvalidValue;
+  if (!make_tmap(&tb, B, e.N, e.K, e.K, Sh::B_BOX)) return cudaErrorInvalidValue;
+  dim3 grid((e.M + BM - 1) / BM, e.N / BN);
+  prof_begin(cls, s);
+  gemm_tc_kernel<BN, EPI><<<grid, NUM_THREADS, Sh::SMEM_BYTES, s>>>(ta, tb, e);
+  cudaError_t err = cudaGetLastError();
+  prof_end(cls, s);
+  return err;
+}
+
+bool tc_gemm_supported(int N, int K, int epi) {
+  if (K <= 0 || K % BK != 0 || N <= 0) return false;
+  if (epi == EPI_LN || epi == EPI_LN_HEAD) return N == 64 || N == 128 || N == 256 || N == 512;
+  return N % 64 == 0;
+}
+
+template <int EPI>
+static cudaError_t launch_plain(const __nv_bfloat16* A, long long lda, const __nv_bfloat16* B, const EpiArgs& e,
+                                cudaStream_t s, int cls) {
+  // widest tile that divides N (and the cache's column blocks) while the grid
+  // still fills the machine; narrower tiles otherwise
+  const long long m_tiles = (e.M + BM - 1) / BM;
+  auto fits = [&](int bn) {
+    if (e.N % bn) return false;
+    if (EPI == EPI_KV && e.col_blk % bn) return false;
+    return true;
+  };
+  if (fits(256) && m_tiles * (e.N / 256) >= 148) return launch_bn<256, EPI>(A, lda, B, e, s, cls);
+  if (fits(128)) return launch_bn<128, EPI>(A, lda, B, e, s, cls);
+  if (fits(64)) return launch_bn<64, EPI>(A, lda, B, e, s, cls);
+  return cudaErrorInvalidValue;
+}
+
+cudaError_t launch_gemm_tc(const __nv_bfloat16* A, long long lda, const __nv_bfloat16* B, const EpiArgs& e,
+                           cudaStream_t s, int cls) {
+  if (e.M == 0) return cudaSuccess;
+  if (!tc_gemm_supported(e.N, e.K, e.epi)) return cudaErrorInvalidValue;
+  if ((reinterpret_cast<uintptr_t>(A) & 15) || (reinterpret_cast<uintptr_t>(B) & 15) || (lda % 8))
+    return cudaErrorInvalidValue;
+  switch (e.epi) {
+    case EPI_LN:
+    case EPI_LN_HEAD: {
+      const bool head = e.epi == EPI_LN_HEAD;
+      switch (e.N) {
+        case 64: return head ? launch_bn<64, EPI_LN_HEAD>(A, lda, B, e, s, cls) : launch_bn<64, EPI_LN>(A, lda, B, e, s, cls);
+        case 128: return head ? launch_bn<128, EPI_LN_HEAD>(A, lda, B, e, s, cls) : launch_bn<128, EPI_LN>(A, lda, B, e, s, cls);
+        case 256: return head ? launch_bn<256, EPI_LN_HEAD>(A, lda, B, e, s, cls) : launch_bn<256, EPI_LN>(A, lda, B, e, s, cls);
+        default: return head ? launch_bn<512, EPI_LN_HEAD>(A, lda, B, e, s, cls) : launch_bn<512, EPI_LN>(A, lda, B, e, s, cls);
+      }
+    }
+    case EPI_BIAS: return launch_plain<EPI_BIAS>(A, lda, B, e, s, cls);
+    case EPI_BIAS_GELU: return launch_plain<EPI_BIAS_GELU>(A, lda, B, e, s, cls);
+    case EPI_KV: return launch_plain<EPI_KV>(A, lda, B, e, s, cls);
+    default: return cudaErrorInvalidValue;
+  }
+}
+
+}  // namespace tc
+
+cudaError_t launch_gemm_tc(const __nv_bfloat16* A, long long lda, const __nv_bfloat16* B, const EpiArgs& e,
+                           cudaStream_t s, int cls) {
+  return tc::launch_gemm_tc(A, lda, B, e, s, cls);
+}
+bool tc_gemm_supported(int N, int K, int epi) { return tc::tc_gemm_supported(N, K, epi); }
+
+}  // namespace txs

@@ -1,0 +1,177 @@
+// Per-call batch kernels of the scoring path: ragged packing and ranking.
+//
+// pack: builds the decoder input X = [candidate rows of all requests; context
+// rows of all requests] (App. B token sequence, per request [ctx; cand]),
+// the row -> request map used by the attention kernels, and the part of the
+// action logits that depends only on the raw candidate token x
+// (Sec. 4.1.3 with linear f_dec: logits = z Weff_z + x Weff_x + b_dec Q_dec^T).
+// The host passes the candidate offsets by value (no host->device copy).
+//
+// rank: per request, candidate indices by descending probability of one
+// action, ties to the lower index, NaN last (an exact counting rank).
+#include "txs_internal.cuh"
+
+namespace txs {
+
+constexpr int kMaxReqParamV = 4096;
+extern const int kMaxReqParam = kMaxReqParamV;
+
+struct PackArgs {
+  int n_req, n_cand, S, d, na;
+  int cand_off[kMaxReqParamV + 1];
+};
+
+struct RankArgs {
+  int n_req, na, action, top_k;
+  int cand_off[kMaxReqParamV + 1];
+};
+
+namespace {
+
+__device__ __forceinline__ int find_segment_param(const int* off, int n, int row) {
+  int lo = 0, hi = n - 1;
+  while (lo < hi) {
+    const int mid = (lo + hi + 1) >> 1;
+    if (off[mid] <= row) lo = mid; else hi = mid - 1;
+  }
+  return lo;
+}
+
+template <typename T>
+__global__ void __launch_bounds__(256) pack_kernel(const __grid_constant__ PackArgs a, const T* __restrict__ cand,
+                                                   const T* __restrict__ ctx, T* __restrict__ X,
+                                                   int* __restrict__ row_req, const float* __restrict__ weff_x,
+                                                   const float* __restrict__ cdec, float* __restrict__ xlog) {
+  constexpr int VEC = Vec16<T>::N;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const long long p = static_cast<long long>(blockIdx.x) * 8 + warp;
+  const long long n_rows = a.n_cand + static_cast<long long>(a.n_req) * a.S;
+  if (p >= n_rows) return;
+  const int d = a.d;
+  int r;
+  const T* src;
+  if (p < a.n_cand) {
+    r = find_segment_param(a.cand_off, a.n_req, static_cast<int>(p));
+    src = cand + p * d;
+  } else {
+    const long long q = p - a.n_cand;
+    r = static_cast<int>(q / a.S);
+    src = ctx + q * d;
+  }
+  T* dst = X + p * d;
+  float lg[16];
+#pragma unroll
+  for (int i = 0; i < 16; ++i) lg[i] = 0.f;
+  for (int c = lane * VEC; c < d; c += 32 * VEC) {
+    float v[VEC];
+    Vec16<T>::load(src + c, v);
+    Vec16<T>::store(dst + c, v);
+    if (p < a.n_cand) {
+#pragma unroll
+      for (int i = 0; i < VEC; ++i)
+#pragma unroll
+        for (int k = 0; k < 16; ++k)
+          if (k < a.na) lg[k] = fmaf(v[i], __ldg(weff_x + static_cast<long long>(c + i) * a.na + k), lg[k]);
+    }
+  }
+  if (lane == 0) row_req[p] = r;
+  if (p < a.n_cand) {
+#pragma unroll
+    for (int k = 0; k < 16; ++k) {
+      float x = lg[k];
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
+      if (lane == 0 && k < a.na) xlog[p * a.na + k] = x + __ldg(cdec + k);
+    }
+  }
+}
+
+// Monotone map of a float to uint32 for descending comparison; NaN -> 0
+// (after every number), -0 -> +0.
+__device__ __forceinline__ uint32_t order_key(float f) {
+  if (f != f) return 0u;
+  uint32_t u = __float_as_uint(f);
+  if ((u & 0x7FFFFFFFu) == 0) u = 0;
+  return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+}
+
+__global__ void __launch_bounds__(1024) rank_kernel(const __grid_constant__ RankArgs a, const float* __restrict__ probs,
+                                                    int* __restrict__ out) {
+  extern __shared__ uint32_t keys[];
+  const int r = blockIdx.x;
+  const int c0 = a.cand_off[r];
+  const int M = a.cand_off[r + 1] - c0;
+  for (int i = threadIdx.x; i < M; i += blockDim.x)
+    keys[i] = order_key(probs[static_cast<long long>(c0 + i) * a.na + a.action]);
+  __syncthreads();
+  for (int i = threadIdx.x; i < M; i += blockDim.x) {
+    const uint32_t ki = keys[i];
+    int rank = 0;
+    for (int j = 0; j < M; ++j) {
+      const uint32_t kj = keys[j];
+      rank += (kj > ki) | ((kj == ki) & (j < i));
+    }
+    if (a.top_k == 0) out[c0 + rank] = i;
+    else if (rank < a.top_k) out[static_cast<long long>(r) * a.top_k + rank] = i;
+  }
+  if (a.top_k > 0)
+    for (int t = M + threadIdx.x; t < a.top_k; t += blockDim.x) out[static_cast<long long>(r) * a.top_k + t] = -1;
+}
+
+}  // namespace
+
+template <typename T>
+cudaError_t launch_pack(int n_req, const int* cand_off_host, int S, int d, int na, const T* cand, const T* ctx, T* X,
+                        int* row_req, const float* weff_x, const float* cdec, float* xlog, cudaStream_t s) {
+  if (n_req > kMaxReqParam || na > 16) return cudaErrorInvalidValue;
+  PackArgs a;
+  a.n_req = n_req;
+  a.n_cand = cand_off_host[n_req];
+  a.S = S;
+  a.d = d;
+  a.na = na;
+  for (int i = 0; i <= n_req; ++i) a.cand_off[i] = cand_off_host[i];
+  const long long n_rows = a.n_cand + static_cast<long long>(n_req) * S;
+  if (n_rows == 0) return cudaSuccess;
+  prof_begin(KC_PACK, s);
+  pack_kernel<T><<<static_cast<int>((n_rows + 7) / 8), 256, 0, s>>>(a, cand, ctx, X, row_req, weff_x, cdec, xlog);
+  cudaError_t err = cudaGetLastError();
+  prof_end(KC_PACK, s);
+  return err;
+}
+
+cudaError_t launch_rank(int n_req, const int* cand_off_host, const float* probs, int na, int action, int top_k,
+                        int* out, cudaStream_t s) {
+  if (n_req > kMaxReqParam) return cudaErrorInvalidValue;
+  RankArgs a;
+  a.n_req = n_req;
+  a.na = na;
+  a.action = action;
+  a.top_k = top_k;
+  int max_m = 0;
+  for (int i = 0; i <= n_req; ++i) {
+    a.cand_off[i] = cand_off_host[i];
+    if (i > 0) max_m = max_m > cand_off_host[i] - cand_off_host[i - 1] ? max_m : cand_off_host[i] - cand_off_host[i - 1];
+  }
+  if (max_m > 32768) return cudaErrorInvalidValue;
+  const size_t smem = static_cast<size_t>(max_m > 0 ? max_m : 1) * sizeof(uint32_t);
+  static bool attr = false;
+  if (!attr) {
+    cudaError_t e = cudaFuncSetAttribute(rank_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, 32768 * 4);
+    if (e != cudaSuccess) return e;
+    attr = true;
+  }
+  prof_begin(KC_RANK, s);
+  rank_kernel<<<n_req, 1024, smem, s>>>(a, probs, out);
+  cudaError_t err = cudaGetLastError();
+  prof_end(KC_RANK, s);
+  return err;
+}
+
+template cudaError_t launch_pack<float>(int, const int*, int, int, int, const float*, const float*, float*, int*,
+                                        const float*, const float*, float*, cudaStream_t);
+template cudaError_t launch_pack<__nv_bfloat16>(int, const int*, int, int, int, const __nv_bfloat16*,
+                                                const __nv_bfloat16*, __nv_bfloat16*, int*, const float*,
+                                                const float*, float*, cudaStream_t);
+
+}  // namespace txs

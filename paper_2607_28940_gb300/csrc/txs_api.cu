@@ -1,0 +1,716 @@
+// C ABI of libtxs: host-side validation, handle management and the order of
+// kernel launches for the cache build, the incremental append, candidate
+// scoring and ranking.  Every step of the path runs in the kernels of this
+// library; the host only checks arguments, sizes buffers and enqueues work.
+#include <algorithm>
+#include <cmath>
+#include <cstdio>
+#include <cstring>
+#include <string>
+#include <vector>
+
+#include "txs_internal.cuh"
+
+namespace txs {
+
+// ------------------------------------------------------------------ profiler
+
+namespace {
+struct ProfRec {
+  cudaEvent_t a, b;
+  int cls;
+};
+struct Profiler {
+  bool on = false;
+  std::vector<ProfRec> recs;
+  std::vector<cudaEvent_t> pool;
+  int open_cls = -1;
+  cudaEvent_t ev() {
+    if (!pool.empty()) {
+      cudaEvent_t e = pool.back();
+      pool.pop_back();
+      return e;
+    }
+    cudaEvent_t e;
+    cudaEventCreate(&e);
+    return e;
+  }
+};
+Profiler g_prof;
+thread_local std::string g_last_error;
+
+void set_error(const char* where, cudaError_t e) {
+  g_last_error = std::string(where) + ": " + cudaGetErrorString(e);
+}
+void set_error(const char* msg) { g_last_error = msg; }
+}  // namespace
+
+void prof_begin(int cls, cudaStream_t s) {
+  if (!g_prof.on) return;
+  ProfRec r{g_prof.ev(), g_prof.ev(), cls};
+  cudaEventRecord(r.a, s);
+  g_prof.recs.push_back(r);
+}
+
+void prof_end(int cls, cudaStream_t s) {
+  if (!g_prof.on || g_prof.recs.empty()) return;
+  cudaEventRecord(g_prof.recs.back().b, s);
+  (void)cls;
+}
+
+// ------------------------------------------------------------------ handles
+
+struct LayerW {
+  void *Wt_qkv, *Wt_os, *Wt_q, *Wt_oc, *Wt_1, *Wt_2;  // transposed weights [d_out, d_in]
+  float *b_qkv, *b_os, *g1, *be1, *b_q, *b_oc, *g2, *be2, *b_1, *b_2, *g3, *be3;
+};
+
+}  // namespace txs
+
+struct txs_model {
+  txs_config cfg;
+  int es = 0;                    // bytes per stored element
+  std::vector<void*> allocs;
+  std::vector<txs::LayerW> layers;
+  void* Wt_kv = nullptr;         // [2 nL d, d]: rows (l, K|V, c)
+  float* b_kv = nullptr;         // [2 nL d]
+  float* w_pool = nullptr;       // [d]
+  float* weff = nullptr;         // [2d, k]
+  float* cdec = nullptr;         // [k]
+  int* status = nullptr;         // device status word
+  uint64_t hash = 0;
+};
+
+struct txs_kv_cache {
+  int n_req = 0, n_layers = 0, d = 0, es = 0, cap_extra = 0;
+  uint64_t model_hash = 0;
+  long long cap_total = 0;
+  std::vector<int> h_off, h_len, h_cap;  // capacity offsets [R+1], lengths, capacities
+  std::vector<int> h_stage;              // host staging for offset uploads
+  int* d_off = nullptr;                  // [R+1]
+  int* d_len = nullptr;                  // [R]
+  int* d_in_off = nullptr;               // [R+1] offsets of the rows being projected
+  int* d_dst0 = nullptr;                 // [R]   first cache row they go to
+  void* kv = nullptr;                    // [nL][2][cap_total][d] model dtype
+  float *pool_m = nullptr, *pool_s = nullptr, *pool_acc = nullptr, *g = nullptr;
+  float* gkv = nullptr;                  // [nL][2][R][d] fp32
+  float* part = nullptr;                 // pooling chunk states
+  int max_chunks = 0;
+  std::vector<void*> allocs;
+};
+
+namespace txs {
+namespace {
+
+bool cfg_ok(const txs_config& c, std::string* why) {
+  auto bad = [&](const char* m) {
+    *why = m;
+    return false;
+  };
+  if (c.dtype != TXS_FP32 && c.dtype != TXS_BF16) return bad("dtype");
+  if (c.attn_mode != TXS_ATTN_LOCAL_GLOBAL && c.attn_mode != TXS_ATTN_FULL) return bad("attn_mode");
+  if (c.n_layers < 1 || c.n_layers > 64) return bad("n_layers");
+  if (c.n_heads < 1 || c.d_model % c.n_heads) return bad("n_heads");
+  const int dh = c.d_model / c.n_heads;
+  if (dh != 32 && dh != 64) return bad("d_head must be 32 or 64");
+  if (c.dtype == TXS_BF16) {
+    if (c.d_model != 64 && c.d_model != 128 && c.d_model != 256 && c.d_model != 512) return bad("d_model (bf16)");
+  } else if (c.d_model % 32 || c.d_model > 512 || c.d_model < 32) {
+    return bad("d_model (fp32)");
+  }
+  if (c.d_ff < 64 || c.d_ff % 64 || c.d_ff > 16384) return bad("d_ff");
+  if (c.n_actions < 1 || c.n_actions > 16) return bad("n_actions");
+  if (c.n_ctx < 0 || c.n_ctx > 8) return bad("n_ctx");
+  if (c.l_local < 1) return bad("l_local");
+  if (!(c.ln_eps > 0.f) || !std::isfinite(c.ln_eps)) return bad("ln_eps");
+  return true;
+}
+
+// offsets[0] == 0, non-decreasing (strictly if `strict`), last <= INT32_MAX
+bool offsets_ok(const int32_t* off, int n, bool strict) {
+  if (!off || n < 0 || off[0] != 0) return false;
+  for (int i = 0; i < n; ++i) {
+    if (off[i + 1] < off[i]) return false;
+    if (strict && off[i + 1] == off[i]) return false;
+  }
+  return true;
+}
+
+template <typename T>
+T* dalloc(std::vector<void*>& list, size_t bytes, cudaError_t* err) {
+  void* p = nullptr;
+  if (bytes == 0) bytes = 16;
+  *err = cudaMalloc(&p, bytes);
+  if (*err != cudaSuccess) return nullptr;
+  list.push_back(p);
+  return static_cast<T*>(p);
+}
+
+size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
+
+struct ScoreLayout {
+  size_t row_req, X, QKV, A, X1, X2, Hf, xlog, tmp, total;
+};
+
+ScoreLayout score_layout(const txs_config& c, int es, int n_req, long long n_cand) {
+  const long long N = n_cand + static_cast<long long>(n_req) * c.n_ctx;
+  const size_t d = c.d_model, F = c.d_ff;
+  ScoreLayout L{};
+  size_t o = 0;
+  auto take = [&](size_t bytes) {
+    size_t at = o;
+    o = align256(o + bytes);
+    return at;
+  };
+  L.row_req = take(N * 4);
+  L.X = take(N * d * es);
+  L.QKV = take(N * 3 * d * es);
+  L.A = take(N * d * es);
+  L.X1 = take(N * d * es);
+  L.X2 = take(N * d * es);
+  L.Hf = take(N * F * es);
+  L.xlog = take(n_cand * c.n_actions * 4);
+  L.tmp = take(c.dtype == TXS_FP32 ? N * d * 4 : 0);
+  L.total = o;
+  return L;
+}
+
+// One dense projection C = A W (+ epilogue) in the model's dtype: bf16 on the
+// tensor cores, fp32 on the CUDA cores.
+cudaError_t gemm(const txs_model* m, const void* A, long long lda, const void* Bt, EpiArgs e, float* tmp,
+                 cudaStream_t s, int cls) {
+  e.status = m->status;
+  if (m->cfg.dtype == TXS_BF16)
+    return launch_gemm_tc(static_cast<const __nv_bfloat16*>(A), lda, static_cast<const __nv_bfloat16*>(Bt), e, s, cls);
+  return launch_gemm_simt(static_cast<const float*>(A), lda, static_cast<const float*>(Bt), e, tmp, s, cls);
+}
+
+EpiArgs epi_base(int epi, long long M, int N, int K) {
+  EpiArgs e;
+  std::memset(&e, 0, sizeof(e));
+  e.epi = epi;
+  e.M = static_cast<int>(M);
+  e.N = N;
+  e.K = K;
+  return e;
+}
+
+txs_status fail_cuda(const char* where, cudaError_t e) {
+  set_error(where, e);
+  return TXS_ERR_CUDA;
+}
+
+#define TXS_CK(call)                                      \
+  do {                                                    \
+    cudaError_t e_ = (call);                              \
+    if (e_ != cudaSuccess) return fail_cuda(#call, e_);   \
+  } while (0)
+
+template <typename T>
+txs_status model_prepare(txs_model* m, const void* const* w, cudaStream_t s) {
+  const txs_config& c = m->cfg;
+  const int d = c.d_model, F = c.d_ff, nL = c.n_layers, k = c.n_actions;
+  cudaError_t err;
+  auto wt = [&](int rows, int cols) { return dalloc<T>(m->allocs, size_t(rows) * cols * sizeof(T), &err); };
+  auto vf = [&](int n) { return dalloc<float>(m->allocs, size_t(n) * 4, &err); };
+  auto W = [&](int l, int i) { return static_cast<const T*>(w[l * TXS_WEIGHTS_PER_LAYER + i]); };
+  m->Wt_kv = wt(2 * nL * d, d);
+  if (!m->Wt_kv) return fail_cuda("cudaMalloc", err);
+  m->b_kv = vf(2 * nL * d);
+  if (!m->b_kv) return fail_cuda("cudaMalloc", err);
+  for (int l = 0; l < nL; ++l) {
+    LayerW L;
+    T* p;
+    // transposed weights (K-major B operands)
+    if (!(p = wt(3 * d, d))) return fail_cuda("cudaMalloc", err);
+    TXS_CK(launch_transpose<T>(W(l, 0), p, d, 3 * d, s));
+    L.Wt_qkv = p;
+    if (!(p = wt(d, d))) return fail_cuda("cudaMalloc", err);
+    TXS_CK(launch_transpose<T>(W(l, 2), p, d, d, s));
+    L.Wt_os = p;
+    if (!(p = wt(d, d))) return fail_cuda("cudaMalloc", err);
+    TXS_CK(launch_transpose<T>(W(l, 6), p, d, d, s));
+    L.Wt_q = p;
+    if (!(p = wt(d, d))) return fail_cuda("cudaMalloc", err);
+    TXS_CK(launch_transpose<T>(W(l, 12), p, d, d, s));
+    L.Wt_oc = p;
+    if (!(p = wt(F, d))) return fail_cuda("cudaMalloc", err);
+    TXS_CK(launch_transpose<T>(W(l, 16), p, d, F, s));
+    L.Wt_1 = p;
+    if (!(p = wt(d, F))) return fail_cuda("cudaMalloc", err);
+    TXS_CK(launch_transpose<T>(W(l, 18), p, F, d, s));
+    L.Wt_2 = p;
+    T* kv = static_cast<T*>(m->Wt_kv);
+    TXS_CK(launch_transpose<T>(W(l, 8), kv + size_t(2 * l) * d * d, d, d, s));
+    TXS_CK(launch_transpose<T>(W(l, 10), kv + size_t(2 * l + 1) * d * d, d, d, s));
+    // vectors in fp32
+    float** dst[] = {&L.b_qkv, &L.b_os, &L.g1, &L.be1, &L.b_q, &L.b_oc, &L.g2, &L.be2,
+                     &L.b_1, &L.b_2, &L.g3, &L.be3};
+    const int idx[] = {1, 3, 4, 5, 7, 13, 14, 15, 17, 19, 20, 21};
+    const int len[] = {3 * d, d, d, d, d, d, d, d, F, d, d, d};
+    for (int i = 0; i < 12; ++i) {
+      float* v = vf(len[i]);
+      if (!v) return fail_cuda("cudaMalloc", err);
+      TXS_CK(launch_to_f32<T>(W(l, idx[i]), v, len[i], s));
+      *dst[i] = v;
+    }
+    TXS_CK(launch_to_f32<T>(W(l, 9), m->b_kv + size_t(2 * l) * d, d, s));
+    TXS_CK(launch_to_f32<T>(W(l, 11), m->b_kv + size_t(2 * l + 1) * d, d, s));
+    m->layers.push_back(L);
+  }
+  const void* const* head = w + nL * TXS_WEIGHTS_PER_LAYER;
+  if (!(m->w_pool = vf(d))) return fail_cuda("cudaMalloc", err);
+  TXS_CK(launch_to_f32<T>(static_cast<const T*>(head[0]), m->w_pool, d, s));
+  if (!(m->weff = vf(2 * d * k))) return fail_cuda("cudaMalloc", err);
+  if (!(m->cdec = vf(k))) return fail_cuda("cudaMalloc", err);
+  TXS_CK(launch_fold_head<T>(static_cast<const T*>(head[1]), static_cast<const T*>(head[2]),
+                             static_cast<const T*>(head[3]), m->weff, m->cdec, d, k, s));
+  // content hash of config and every input tensor
+  unsigned long long* dh = dalloc<unsigned long long>(m->allocs, 8, &err);
+  if (!dh) return fail_cuda("cudaMalloc", err);
+  TXS_CK(cudaMemsetAsync(dh, 0, 8, s));
+  const size_t es = sizeof(T);
+  for (int l = 0; l < nL; ++l) {
+    const size_t n[TXS_WEIGHTS_PER_LAYER] = {size_t(d) * 3 * d, 3 * size_t(d), size_t(d) * d, size_t(d), size_t(d),
+                                             size_t(d), size_t(d) * d, size_t(d), size_t(d) * d, size_t(d),
+                                             size_t(d) * d, size_t(d), size_t(d) * d, size_t(d), size_t(d), size_t(d),
+                                             size_t(d) * F, size_t(F), size_t(F) * d, size_t(d), size_t(d), size_t(d)};
+    for (int i = 0; i < TXS_WEIGHTS_PER_LAYER; ++i)
+      TXS_CK(launch_hash(W(l, i), static_cast<long long>(n[i] * es), uint64_t(l) * 64 + i + 1, dh, s));
+  }
+  const size_t nh[TXS_HEAD_WEIGHTS] = {size_t(d), 2 * size_t(d) * d, size_t(d), size_t(k) * d};
+  for (int i = 0; i < TXS_HEAD_WEIGHTS; ++i)
+    TXS_CK(launch_hash(head[i], static_cast<long long>(nh[i] * es), 100000 + i, dh, s));
+  unsigned long long hv = 0;
+  TXS_CK(cudaMemcpyAsync(&hv, dh, 8, cudaMemcpyDeviceToHost, s));
+  TXS_CK(cudaStreamSynchronize(s));
+  uint64_t h = hv;
+  const int32_t cf[] = {c.d_model, c.n_heads, c.d_ff, c.n_layers, c.n_actions, c.n_ctx, c.l_local, c.attn_mode,
+                        c.dtype};
+  for (int32_t v : cf) h = (h ^ static_cast<uint64_t>(static_cast<uint32_t>(v))) * 0x100000001B3ull;
+  uint32_t eps_bits;
+  std::memcpy(&eps_bits, &c.ln_eps, 4);
+  h = (h ^ eps_bits) * 0x100000001B3ull;
+  m->hash = h;
+  return TXS_OK;
+}
+
+template <typename T>
+txs_status project_rows(txs_model* m, txs_kv_cache* c, int n_req, const int32_t* in_off, const void* rows,
+                        bool append, cudaStream_t s) {
+  const txs_config& cf = m->cfg;
+  const int d = cf.d_model, nL = cf.n_layers;
+  const long long total = in_off[n_req];
+  // stage [in_off (R+1) | dst0 (R)] and upload in one copy
+  c->h_stage.assign(2 * n_req + 1, 0);
+  int max_rows = 0;
+  for (int r = 0; r <= n_req; ++r) c->h_stage[r] = in_off[r];
+  for (int r = 0; r < n_req; ++r) {
+    c->h_stage[n_req + 1 + r] = c->h_off[r] + (append ? c->h_len[r] : 0);
+    max_rows = std::max(max_rows, in_off[r + 1] - in_off[r]);
+  }
+  TXS_CK(cudaMemcpyAsync(c->d_in_off, c->h_stage.data(), sizeof(int) * (2 * n_req + 1), cudaMemcpyHostToDevice, s));
+  if (total > 0) {
+    EpiArgs e = epi_base(EPI_KV, total, 2 * nL * d, d);
+    e.bias = m->b_kv;
+    e.out = c->kv;
+    e.ldo = d;
+    e.seg_off = c->d_in_off;
+    e.dst_row0 = c->d_dst0;
+    e.n_seg = n_req;
+    e.col_blk = d;
+    e.col_blk_stride = c->cap_total * d;
+    TXS_CK(gemm(m, rows, d, m->Wt_kv, e, nullptr, s, KC_GEMM_KV));
+  }
+  TXS_CK(launch_pool<T>(static_cast<const T*>(rows), c->d_in_off, n_req, max_rows, m->w_pool, d, c->max_chunks,
+                        c->part, append ? 1 : 0, c->pool_m, c->pool_s, c->pool_acc, c->g, s));
+  TXS_CK(launch_global_kv<T>(c->g, static_cast<const T*>(m->Wt_kv), m->b_kv, c->gkv, n_req, d, nL, s));
+  return TXS_OK;
+}
+
+template <typename T>
+txs_status score_impl(txs_model* m, const txs_kv_cache* c, int n_req, const int32_t* cand_off, const void* cand_tok,
+                      const void* ctx_tok, void* ws, float* logits, float* probs, cudaStream_t s) {
+  const txs_config& cf = m->cfg;
+  const int d = cf.d_model, F = cf.d_ff, H = cf.n_heads, S = cf.n_ctx, k = cf.n_actions;
+  const long long n_cand = cand_off[n_req];
+  const long long N = n_cand + static_cast<long long>(n_req) * S;
+  const ScoreLayout L = score_layout(cf, sizeof(T), n_req, n_cand);
+  uint8_t* base = static_cast<uint8_t*>(ws);
+  int* row_req = reinterpret_cast<int*>(base + L.row_req);
+  T* X = reinterpret_cast<T*>(base + L.X);
+  T* QKV = reinterpret_cast<T*>(base + L.QKV);
+  T* A = reinterpret_cast<T*>(base + L.A);
+  T* X1 = reinterpret_cast<T*>(base + L.X1);
+  T* X2 = reinterpret_cast<T*>(base + L.X2);
+  T* Hf = reinterpret_cast<T*>(base + L.Hf);
+  float* xlog = reinterpret_cast<float*>(base + L.xlog);
+  float* tmp = reinterpret_cast<float*>(base + L.tmp);
+
+  TXS_CK(launch_pack<T>(n_req, cand_off, S, d, k, static_cast<const T*>(cand_tok), static_cast<const T*>(ctx_tok), X,
+                        row_req, m->weff + size_t(d) * k, m->cdec, xlog, s));
+  const T* kv = static_cast<const T*>(c->kv);
+  for (int l = 0; l < cf.n_layers; ++l) {
+    const LayerW& W = m->layers[l];
+    // serving-stream attention (App. B mask), O-projection + residual + LN1
+    EpiArgs e = epi_base(EPI_BIAS, N, 3 * d, d);
+    e.bias = W.b_qkv;
+    e.out = QKV;
+    e.ldo = 3 * d;
+    TXS_CK(gemm(m, X, d, W.Wt_qkv, e, tmp, s, KC_GEMM_QKV));
+    TXS_CK(launch_serving_attn<T>(QKV, A, row_req, static_cast<int>(N), static_cast<int>(n_cand), S, H, d, s));
+    e = epi_base(EPI_LN, N, d, d);
+    e.bias = W.b_os;
+    e.res = X;
+    e.ldr = d;
+    e.gamma = W.g1;
+    e.beta = W.be1;
+    e.ln_eps = cf.ln_eps;
+    e.out = X1;
+    e.ldo = d;
+    TXS_CK(gemm(m, A, d, W.Wt_os, e, tmp, s, KC_GEMM_OPROJ));
+    // multi-query cross-attention against the shared cache (Sec. 4.1.2)
+    e = epi_base(EPI_BIAS, N, d, d);
+    e.bias = W.b_q;
+    e.out = QKV;
+    e.ldo = d;
+    TXS_CK(gemm(m, X1, d, W.Wt_q, e, tmp, s, KC_GEMM_Q));
+    const T* Kc = kv + (size_t(2 * l) * c->cap_total) * d;
+    const T* Vc = kv + (size_t(2 * l + 1) * c->cap_total) * d;
+    const float* Kg = c->gkv + size_t(2 * l) * n_req * d;
+    const float* Vg = c->gkv + size_t(2 * l + 1) * n_req * d;
+    TXS_CK(launch_cross_attn<T>(QKV, A, Kc, Vc, row_req, static_cast<int>(N), c->d_off, c->d_len, Kg, Vg,
+                                cf.l_local, cf.attn_mode, H, d, s));
+    e = epi_base(EPI_LN, N, d, d);
+    e.bias = W.b_oc;
+    e.res = X1;
+    e.ldr = d;
+    e.gamma = W.g2;
+    e.beta = W.be2;
+    e.ln_eps = cf.ln_eps;
+    e.out = X2;
+    e.ldo = d;
+    TXS_CK(gemm(m, A, d, W.Wt_oc, e, tmp, s, KC_GEMM_OPROJ));
+    // FFN with GELU, then residual + LN3 (the last layer also runs the head)
+    e = epi_base(EPI_BIAS_GELU, N, F, d);
+    e.bias = W.b_1;
+    e.out = Hf;
+    e.ldo = F;
+    TXS_CK(gemm(m, X2, d, W.Wt_1, e, tmp, s, KC_GEMM_FFN1));
+    const bool last = l == cf.n_layers - 1;
+    e = epi_base(last ? EPI_LN_HEAD : EPI_LN, N, d, F);
+    e.bias = W.b_2;
+    e.res = X2;
+    e.ldr = d;
+    e.gamma = W.g3;
+    e.beta = W.be3;
+    e.ln_eps = cf.ln_eps;
+    e.out = X;
+    e.ldo = d;
+    if (last) {
+      e.weff_z = m->weff;
+      e.xlog = xlog;
+      e.n_act = k;
+      e.n_cand_rows = static_cast<int>(n_cand);
+      e.logits = logits;
+      e.probs = probs;
+    }
+    TXS_CK(gemm(m, Hf, F, W.Wt_2, e, tmp, s, KC_GEMM_FFN2));
+  }
+  return TXS_OK;
+}
+
+}  // namespace
+}  // namespace txs
+
+using namespace txs;
+
+// ------------------------------------------------------------------ C ABI
+
+TXS_API const char* txs_version(void) { return "txs 0.1 (sm_103a)"; }
+
+TXS_API const char* txs_status_string(txs_status s) {
+  switch (s) {
+    case TXS_OK: return "ok";
+    case TXS_ERR_INVALID_ARG: return "invalid argument";
+    case TXS_ERR_COLD_START: return "cold start: request without behavior rows";
+    case TXS_ERR_CAPACITY: return "append exceeds cache capacity";
+    case TXS_ERR_STALE_CACHE: return "cache built by another model";
+    case TXS_ERR_CUDA: return "CUDA error";
+    case TXS_ERR_DEVICE_TIMEOUT: return "device-side wait timed out";
+    case TXS_ERR_BOUNDS: return "device-side bounds check failed";
+    case TXS_ERR_UNSUPPORTED: return "unsupported shape";
+  }
+  return "unknown status";
+}
+
+TXS_API const char* txs_last_error(void) { return g_last_error.c_str(); }
+
+TXS_API txs_status txs_model_create(const txs_config* cfg, const void* const* weights, txs_model** out) {
+  if (!cfg || !weights || !out) return TXS_ERR_INVALID_ARG;
+  *out = nullptr;
+  std::string why;
+  if (!cfg_ok(*cfg, &why)) {
+    set_error(why.c_str());
+    return TXS_ERR_UNSUPPORTED;
+  }
+  const int n_w = cfg->n_layers * TXS_WEIGHTS_PER_LAYER + TXS_HEAD_WEIGHTS;
+  for (int i = 0; i < n_w; ++i)
+    if (!weights[i]) return TXS_ERR_INVALID_ARG;
+  // the weight tensors may still be in flight on any stream of the caller
+  cudaError_t pre = cudaDeviceSynchronize();
+  if (pre != cudaSuccess) return fail_cuda("cudaDeviceSynchronize", pre);
+  txs_model* m = new txs_model();
+  m->cfg = *cfg;
+  m->es = cfg->dtype == TXS_BF16 ? 2 : 4;
+  cudaError_t err;
+  m->status = dalloc<int>(m->allocs, 4, &err);
+  txs_status st = TXS_OK;
+  if (!m->status) st = fail_cuda("cudaMalloc", err);
+  if (st == TXS_OK && cudaMemset(m->status, 0, 4) != cudaSuccess) st = TXS_ERR_CUDA;
+  cudaStream_t s = nullptr;
+  if (st == TXS_OK && cudaStreamCreateWithFlags(&s, cudaStreamNonBlocking) != cudaSuccess) st = TXS_ERR_CUDA;
+  if (st == TXS_OK)
+    st = cfg->dtype == TXS_BF16 ? model_prepare<__nv_bfloat16>(m, weights, s) : model_prepare<float>(m, weights, s);
+  if (s) {
+    if (cudaStreamSynchronize(s) != cudaSuccess && st == TXS_OK) st = TXS_ERR_CUDA;
+    cudaStreamDestroy(s);
+  }
+  if (st != TXS_OK) {
+    txs_model_destroy(m);
+    return st;
+  }
+  *out = m;
+  return TXS_OK;
+}
+
+TXS_API void txs_model_destroy(txs_model* m) {
+  if (!m) return;
+  for (void* p : m->allocs) cudaFree(p);
+  delete m;
+}
+
+TXS_API uint64_t txs_model_hash(const txs_model* m) { return m ? m->hash : 0; }
+
+TXS_API txs_status txs_build_kv_cache(txs_model* m, int32_t n_req, const int32_t* beh_offsets, const void* beh_enc,
+                                      int32_t capacity_extra, void* stream, txs_kv_cache** out) {
+  if (!m || !out || n_req < 1 || capacity_extra < 0 || !beh_offsets) return TXS_ERR_INVALID_ARG;
+  *out = nullptr;
+  if (!offsets_ok(beh_offsets, n_req, false)) return TXS_ERR_INVALID_ARG;
+  for (int r = 0; r < n_req; ++r)
+    if (beh_offsets[r + 1] == beh_offsets[r]) return TXS_ERR_COLD_START;
+  if (!beh_enc) return TXS_ERR_INVALID_ARG;
+  if (n_req > kMaxReqParam) return TXS_ERR_UNSUPPORTED;
+  const txs_config& cf = m->cfg;
+  const int d = cf.d_model, nL = cf.n_layers;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  txs_kv_cache* c = new txs_kv_cache();
+  c->n_req = n_req;
+  c->n_layers = nL;
+  c->d = d;
+  c->es = m->es;
+  c->cap_extra = capacity_extra;
+  c->model_hash = m->hash;
+  c->h_off.assign(n_req + 1, 0);
+  c->h_len.assign(n_req, 0);
+  c->h_cap.assign(n_req, 0);
+  long long tot = 0;
+  int max_cap = 0;
+  for (int r = 0; r < n_req; ++r) {
+    c->h_len[r] = beh_offsets[r + 1] - beh_offsets[r];
+    c->h_cap[r] = c->h_len[r] + capacity_extra;
+    max_cap = std::max(max_cap, std::max(c->h_len[r], capacity_extra));
+    c->h_off[r] = static_cast<int>(tot);
+    tot += c->h_cap[r];
+    if (tot > 0x7FFFFFFFLL) {
+      delete c;
+      return TXS_ERR_UNSUPPORTED;
+    }
+  }
+  c->h_off[n_req] = static_cast<int>(tot);
+  c->cap_total = tot;
+  c->max_chunks = (max_cap + kPoolChunk - 1) / kPoolChunk;
+  cudaError_t err = cudaSuccess;
+  txs_status st = TXS_OK;
+  auto A = [&](size_t bytes) -> void* {
+    if (st != TXS_OK) return nullptr;
+    void* p = dalloc<void>(c->allocs, bytes, &err);
+    if (!p) st = fail_cuda("cudaMalloc", err);
+    return p;
+  };
+  c->kv = A(size_t(nL) * 2 * tot * d * m->es);
+  c->d_off = static_cast<int*>(A(4 * (n_req + 1)));
+  c->d_len = static_cast<int*>(A(4 * n_req));
+  c->d_in_off = static_cast<int*>(A(4 * (2 * n_req + 1)));
+  if (st == TXS_OK) c->d_dst0 = c->d_in_off + n_req + 1;
+  c->pool_m = static_cast<float*>(A(4 * n_req));
+  c->pool_s = static_cast<float*>(A(4 * n_req));
+  c->pool_acc = static_cast<float*>(A(size_t(4) * n_req * d));
+  c->g = static_cast<float*>(A(size_t(4) * n_req * d));
+  c->gkv = static_cast<float*>(A(size_t(4) * nL * 2 * n_req * d));
+  c->part = static_cast<float*>(A(size_t(4) * n_req * c->max_chunks * (d + 2)));
+  if (st == TXS_OK) {
+    if ((err = cudaMemcpyAsync(c->d_off, c->h_off.data(), 4 * (n_req + 1), cudaMemcpyHostToDevice, s)) != cudaSuccess ||
+        (err = cudaMemcpyAsync(c->d_len, c->h_len.data(), 4 * n_req, cudaMemcpyHostToDevice, s)) != cudaSuccess)
+      st = fail_cuda("upload", err);
+  }
+  if (st == TXS_OK)
+    st = cf.dtype == TXS_BF16 ? project_rows<__nv_bfloat16>(m, c, n_req, beh_offsets, beh_enc, false, s)
+                              : project_rows<float>(m, c, n_req, beh_offsets, beh_enc, false, s);
+  if (st != TXS_OK) {
+    cudaStreamSynchronize(s);
+    txs_cache_destroy(c);
+    return st;
+  }
+  *out = c;
+  return TXS_OK;
+}
+
+TXS_API void txs_cache_destroy(txs_kv_cache* c) {
+  if (!c) return;
+  for (void* p : c->allocs) cudaFree(p);
+  delete c;
+}
+
+TXS_API txs_status txs_append_behavior(txs_model* m, txs_kv_cache* c, int32_t n_req, const int32_t* new_offsets,
+                                       const void* new_enc, void* stream) {
+  if (!m || !c || !new_offsets) return TXS_ERR_INVALID_ARG;
+  if (c->model_hash != m->hash) return TXS_ERR_STALE_CACHE;
+  if (n_req != c->n_req || !offsets_ok(new_offsets, n_req, false)) return TXS_ERR_INVALID_ARG;
+  for (int r = 0; r < n_req; ++r)
+    if (static_cast<long long>(c->h_len[r]) + (new_offsets[r + 1] - new_offsets[r]) > c->h_cap[r])
+      return TXS_ERR_CAPACITY;
+  if (new_offsets[n_req] == 0) return TXS_OK;
+  if (!new_enc) return TXS_ERR_INVALID_ARG;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  txs_status st = m->cfg.dtype == TXS_BF16 ? project_rows<__nv_bfloat16>(m, c, n_req, new_offsets, new_enc, true, s)
+                                           : project_rows<float>(m, c, n_req, new_offsets, new_enc, true, s);
+  if (st != TXS_OK) return st;
+  for (int r = 0; r < n_req; ++r) c->h_len[r] += new_offsets[r + 1] - new_offsets[r];
+  cudaError_t err = cudaMemcpyAsync(c->d_len, c->h_len.data(), 4 * n_req, cudaMemcpyHostToDevice, s);
+  if (err != cudaSuccess) return fail_cuda("upload lengths", err);
+  return TXS_OK;
+}
+
+TXS_API txs_status txs_cache_lengths(const txs_kv_cache* c, int32_t* out_len) {
+  if (!c || !out_len) return TXS_ERR_INVALID_ARG;
+  for (int r = 0; r < c->n_req; ++r) out_len[r] = c->h_len[r];
+  return TXS_OK;
+}
+
+TXS_API int32_t txs_cache_n_req(const txs_kv_cache* c) { return c ? c->n_req : 0; }
+
+TXS_API txs_status txs_cache_read_rows(const txs_kv_cache* c, int32_t layer, int32_t which, int32_t req, int32_t row0,
+                                       int32_t n_rows, void* dst, void* stream) {
+  if (!c || !dst || layer < 0 || layer >= c->n_layers || which < 0 || which > 1 || req < 0 || req >= c->n_req ||
+      row0 < 0 || n_rows < 0 || static_cast<long long>(row0) + n_rows > c->h_len[req])
+    return TXS_ERR_INVALID_ARG;
+  if (n_rows == 0) return TXS_OK;
+  const size_t row_bytes = size_t(c->d) * c->es;
+  const size_t blk = size_t(2 * layer + which) * c->cap_total;
+  const uint8_t* src = static_cast<const uint8_t*>(c->kv) + (blk + c->h_off[req] + row0) * row_bytes;
+  cudaError_t err = cudaMemcpyAsync(dst, src, n_rows * row_bytes, cudaMemcpyDeviceToDevice,
+                                    static_cast<cudaStream_t>(stream));
+  return err == cudaSuccess ? TXS_OK : fail_cuda("read rows", err);
+}
+
+TXS_API txs_status txs_cache_read_anchor(const txs_kv_cache* c, int32_t layer, int32_t which, float* dst,
+                                         void* stream) {
+  if (!c || !dst || which < 0 || which > 2 || (which < 2 && (layer < 0 || layer >= c->n_layers)))
+    return TXS_ERR_INVALID_ARG;
+  const size_t bytes = size_t(c->n_req) * c->d * 4;
+  const float* src = which == 2 ? c->g : c->gkv + size_t(2 * layer + which) * c->n_req * c->d;
+  cudaError_t err = cudaMemcpyAsync(dst, src, bytes, cudaMemcpyDeviceToDevice, static_cast<cudaStream_t>(stream));
+  return err == cudaSuccess ? TXS_OK : fail_cuda("read anchor", err);
+}
+
+TXS_API txs_status txs_score_workspace_size(const txs_model* m, int32_t n_req, int64_t total_cand, size_t* bytes) {
+  if (!m || !bytes || n_req < 0 || total_cand < 0) return TXS_ERR_INVALID_ARG;
+  *bytes = score_layout(m->cfg, m->es, n_req, total_cand).total;
+  return TXS_OK;
+}
+
+TXS_API txs_status txs_score_candidates(txs_model* m, const txs_kv_cache* c, int32_t n_req,
+                                        const int32_t* cand_offsets, const void* cand_tok, const void* ctx_tok,
+                                        void* workspace, size_t workspace_bytes, float* out_logits, float* out_probs,
+                                        void* stream) {
+  if (!m || !c || !cand_offsets) return TXS_ERR_INVALID_ARG;
+  if (c->model_hash != m->hash) return TXS_ERR_STALE_CACHE;
+  if (n_req != c->n_req || !offsets_ok(cand_offsets, n_req, false)) return TXS_ERR_INVALID_ARG;
+  if (n_req > kMaxReqParam) return TXS_ERR_UNSUPPORTED;
+  const txs_config& cf = m->cfg;
+  const long long n_cand = cand_offsets[n_req];
+  if (n_cand + static_cast<long long>(n_req) * cf.n_ctx > 0x7FFFFFFFLL) return TXS_ERR_UNSUPPORTED;
+  if (n_cand == 0) return TXS_OK;
+  if (!cand_tok || !out_logits || (cf.n_ctx > 0 && !ctx_tok) || !workspace) return TXS_ERR_INVALID_ARG;
+  if (reinterpret_cast<uintptr_t>(workspace) & 255) return TXS_ERR_INVALID_ARG;
+  if ((reinterpret_cast<uintptr_t>(cand_tok) & 15) || (ctx_tok && (reinterpret_cast<uintptr_t>(ctx_tok) & 15)))
+    return TXS_ERR_INVALID_ARG;
+  if (workspace_bytes < score_layout(cf, m->es, n_req, n_cand).total) return TXS_ERR_INVALID_ARG;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  return cf.dtype == TXS_BF16
+             ? score_impl<__nv_bfloat16>(m, c, n_req, cand_offsets, cand_tok, ctx_tok, workspace, out_logits,
+                                         out_probs, s)
+             : score_impl<float>(m, c, n_req, cand_offsets, cand_tok, ctx_tok, workspace, out_logits, out_probs, s);
+}
+
+TXS_API txs_status txs_rank_candidates(int32_t n_req, const int32_t* cand_offsets, const float* probs,
+                                       int32_t n_actions, int32_t action, int32_t top_k, int32_t* out_idx,
+                                       void* stream) {
+  if (n_req < 0 || !cand_offsets || n_actions < 1 || action < 0 || action >= n_actions || top_k < 0)
+    return TXS_ERR_INVALID_ARG;
+  if (n_req == 0) return TXS_OK;
+  if (!offsets_ok(cand_offsets, n_req, false)) return TXS_ERR_INVALID_ARG;
+  if (n_req > kMaxReqParam) return TXS_ERR_UNSUPPORTED;
+  for (int r = 0; r < n_req; ++r)
+    if (cand_offsets[r + 1] - cand_offsets[r] > 32768) return TXS_ERR_UNSUPPORTED;
+  if (cand_offsets[n_req] == 0 && top_k == 0) return TXS_OK;
+  if (!out_idx || (!probs && cand_offsets[n_req] > 0)) return TXS_ERR_INVALID_ARG;
+  cudaError_t err = launch_rank(n_req, cand_offsets, probs, n_actions, action, top_k, out_idx,
+                                static_cast<cudaStream_t>(stream));
+  if (err != cudaSuccess) return fail_cuda("rank", err);
+  return TXS_OK;
+}
+
+TXS_API txs_status txs_device_status(txs_model* m) {
+  if (!m) return TXS_ERR_INVALID_ARG;
+  cudaError_t err = cudaDeviceSynchronize();
+  if (err != cudaSuccess) return fail_cuda("cudaDeviceSynchronize", err);
+  int v = 0;
+  if ((err = cudaMemcpy(&v, m->status, 4, cudaMemcpyDeviceToHost)) != cudaSuccess) return fail_cuda("status", err);
+  if (v != 0 && (err = cudaMemset(m->status, 0, 4)) != cudaSuccess) return fail_cuda("status reset", err);
+  return static_cast<txs_status>(v);
+}
+
+TXS_API txs_status txs_profile_enable(int32_t enable) {
+  g_prof.on = enable != 0;
+  return TXS_OK;
+}
+
+TXS_API txs_status txs_profile_collect(double* total_ms, int64_t* launches, int32_t n) {
+  if (!total_ms || !launches || n < TXS_N_KERNEL_CLASSES) return TXS_ERR_INVALID_ARG;
+  for (int i = 0; i < n; ++i) {
+    total_ms[i] = 0;
+    launches[i] = 0;
+  }
+  txs_status st = TXS_OK;
+  for (ProfRec& r : g_prof.recs) {
+    float ms = 0.f;
+    if (cudaEventSynchronize(r.b) != cudaSuccess || cudaEventElapsedTime(&ms, r.a, r.b) != cudaSuccess)
+      st = TXS_ERR_CUDA;
+    total_ms[r.cls] += ms;
+    launches[r.cls] += 1;
+    g_prof.pool.push_back(r.a);
+    g_prof.pool.push_back(r.b);
+  }
+  g_prof.recs.clear();
+  return st;
+}
+
+TXS_API const char* txs_kernel_class_name(int32_t cls) {
+  static const char* names[] = {"pack", "gemm_qkv", "attn_serving", "gemm_oproj_ln", "gemm_q", "attn_cross",
+                                "gemm_ffn1_gelu", "gemm_ffn2_ln", "gemm_kv_build", "pool", "global_kv", "rank",
+                                "misc", "row_ln"};
+  if (cls < 0 || cls >= KC_COUNT_) return "";
+  return names[cls];
+}

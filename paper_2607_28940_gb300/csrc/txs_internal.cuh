@@ -1,0 +1,174 @@
+// Internal declarations shared by the libtxs translation units (not installed).
+#pragma once
+
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "../../include/txs.h"
+
+#define TXS_API extern "C" __attribute__((visibility("default")))
+
+namespace txs {
+
+// Device-side bounded waits give up after this many SM clock cycles (~1 s at
+// 2 GHz), latch TXS_ERR_DEVICE_TIMEOUT and let the kernel wind down.
+constexpr long long kSpinCycles = 2000000000LL;
+
+// Kernel classes for the event profiler (txs_profile_*).
+enum KernelClass : int {
+  KC_PACK = 0, KC_GEMM_QKV, KC_ATTN_SERVING, KC_GEMM_OPROJ, KC_GEMM_Q, KC_ATTN_CROSS,
+  KC_GEMM_FFN1, KC_GEMM_FFN2, KC_GEMM_KV, KC_POOL, KC_GLOBAL_KV, KC_RANK, KC_MISC,
+  KC_ROW_LN, KC_COUNT_
+};
+static_assert(KC_COUNT_ <= TXS_N_KERNEL_CLASSES, "profiler classes");
+
+// ------------------------------------------------------------------ device helpers
+
+__device__ __forceinline__ void latch_status(int* status, int code) {
+  if (status) atomicCAS(status, 0, code);
+}
+
+template <typename T> struct Elem;
+template <> struct Elem<float> {
+  static __device__ __forceinline__ float load(const float* p) { return *p; }
+  static __device__ __forceinline__ void store(float* p, float v) { *p = v; }
+};
+template <> struct Elem<__nv_bfloat16> {
+  static __device__ __forceinline__ float load(const __nv_bfloat16* p) { return __bfloat162float(*p); }
+  static __device__ __forceinline__ void store(__nv_bfloat16* p, float v) { *p = __float2bfloat16_rn(v); }
+};
+
+// 16-byte vectors of T converted to/from float.
+template <typename T> struct Vec16;
+template <> struct Vec16<float> {
+  static constexpr int N = 4;
+  static __device__ __forceinline__ void load(const float* p, float* v) {
+    float4 a = *reinterpret_cast<const float4*>(p);
+    v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w;
+  }
+  static __device__ __forceinline__ void store(float* p, const float* v) {
+    *reinterpret_cast<float4*>(p) = make_float4(v[0], v[1], v[2], v[3]);
+  }
+};
+template <> struct Vec16<__nv_bfloat16> {
+  static constexpr int N = 8;
+  static __device__ __forceinline__ void load(const __nv_bfloat16* p, float* v) {
+    uint4 a = *reinterpret_cast<const uint4*>(p);
+    const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&a);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      float2 f = __bfloat1622float2(h[i]);
+      v[2 * i] = f.x; v[2 * i + 1] = f.y;
+    }
+  }
+  static __device__ __forceinline__ void store(__nv_bfloat16* p, const float* v) {
+    uint4 a;
+    __nv_bfloat162* h = reinterpret_cast<__nv_bfloat162*>(&a);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) h[i] = __floats2bfloat162_rn(v[2 * i], v[2 * i + 1]);
+    *reinterpret_cast<uint4*>(p) = a;
+  }
+};
+
+__device__ __forceinline__ float gelu_erf(float x) {
+  return 0.5f * x * (1.0f + erff(x * 0.70710678118654752f));
+}
+
+// Index of the segment that contains `row` in an exclusive-offset array
+// off[0..n] (off[0] == 0, non-decreasing): largest r with off[r] <= row.
+__device__ __forceinline__ int find_segment(const int* off, int n, int row) {
+  int lo = 0, hi = n - 1;
+  while (lo < hi) {
+    int mid = (lo + hi + 1) >> 1;
+    if (__ldg(off + mid) <= row) lo = mid; else hi = mid - 1;
+  }
+  return lo;
+}
+
+// ------------------------------------------------------------------ host side
+
+struct Prof;  // event profiler (txs_api.cu)
+void prof_begin(int cls, cudaStream_t s);
+void prof_end(int cls, cudaStream_t s);
+
+// Epilogue kinds shared by the SIMT and tensor-core GEMMs.
+enum Epi : int {
+  EPI_BIAS = 0,       // out = acc + bias
+  EPI_BIAS_GELU = 1,  // out = GELU(acc + bias)
+  EPI_KV = 2,         // out = acc + bias, rows remapped into the cache, cols into [l][K|V]
+  EPI_LN = 3,         // out = LN(acc + bias + res) over the full row (N == d)
+  EPI_LN_HEAD = 4,    // z = LN(...); logits = z Weff_z + xlog; probs = softmax(logits)
+};
+
+// Arguments of every GEMM epilogue; unused fields are ignored.
+struct EpiArgs {
+  int epi;
+  int M, N, K;
+  const float* bias;      // [N]
+  void* out;              // row-major, leading dimension ldo (elements)
+  long long ldo;
+  const void* res;        // residual, leading dimension ldr (EPI_LN*)
+  long long ldr;
+  const float* gamma;     // LN gain/bias [N]
+  const float* beta;
+  float ln_eps;
+  // EPI_KV: row remap (request of row from seg_off[0..n_seg]; out row =
+  // dst_row0[r] + row - seg_off[r]) and column blocks of width col_blk placed
+  // col_blk_stride elements apart.
+  const int* seg_off;
+  const int* dst_row0;
+  int n_seg;
+  int col_blk;
+  long long col_blk_stride;
+  // EPI_LN_HEAD
+  const float* weff_z;    // [N, n_act]  (W_dec[:d] Q_dec^T)
+  const float* xlog;      // [n_cand_rows, n_act] (x W_dec[d:] Q_dec^T + b_dec Q_dec^T)
+  int n_act;
+  int n_cand_rows;        // rows >= this are context rows (no head output)
+  float* logits;
+  float* probs;
+  int* status;
+};
+
+// Launchers (return cudaError_t of the launch).
+cudaError_t launch_gemm_simt(const float* A, long long lda, const float* B, const EpiArgs& e,
+                             float* tmp, cudaStream_t s, int cls);
+cudaError_t launch_gemm_tc(const __nv_bfloat16* A, long long lda, const __nv_bfloat16* B,
+                           const EpiArgs& e, cudaStream_t s, int cls);
+bool tc_gemm_supported(int N, int K, int epi);
+
+template <typename T>
+cudaError_t launch_serving_attn(const T* qkv, T* out, const int* row_req, int n_rows, int n_cand_rows, int S, int H,
+                                int d, cudaStream_t s);
+template <typename T>
+cudaError_t launch_cross_attn(const T* q, T* out, const T* Kc, const T* Vc, const int* row_req, int n_rows,
+                              const int* kv_off, const int* kv_len, const float* Kg, const float* Vg, int l_local,
+                              int mode, int H, int d, cudaStream_t s);
+
+extern const int kPoolChunk;
+template <typename T>
+cudaError_t launch_pool(const T* phi, const int* seg_off, int R, int max_rows, const float* w_pool, int d,
+                        int max_chunks, float* part, int merge_existing, float* st_m, float* st_s, float* st_acc,
+                        float* g, cudaStream_t s);
+template <typename T>
+cudaError_t launch_global_kv(const float* g, const T* Wt_kv, const float* b_kv, float* gkv, int R, int d, int n_layers,
+                             cudaStream_t s);
+template <typename T>
+cudaError_t launch_transpose(const T* W, T* Wt, int rows, int cols, cudaStream_t s);
+template <typename T>
+cudaError_t launch_to_f32(const T* src, float* dst, long long n, cudaStream_t s);
+template <typename T>
+cudaError_t launch_fold_head(const T* W_dec, const T* b_dec, const T* Q_dec, float* weff, float* cdec, int d, int k,
+                             cudaStream_t s);
+cudaError_t launch_hash(const void* p, long long bytes, uint64_t salt, unsigned long long* out, cudaStream_t s);
+
+extern const int kMaxReqParam;
+template <typename T>
+cudaError_t launch_pack(int n_req, const int* cand_off_host, int S, int d, int na, const T* cand, const T* ctx, T* X,
+                        int* row_req, const float* weff_x, const float* cdec, float* xlog, cudaStream_t s);
+cudaError_t launch_rank(int n_req, const int* cand_off_host, const float* probs, int na, int action, int top_k,
+                        int* out, cudaStream_t s);
+
+}  // namespace txs
