@@ -1,0 +1,492 @@
+#!/usr/bin/env python
+"""Throughput benchmark of the TransX serving hot path on GB300.
+
+One step = one pass of the whole path over one synthetic serving batch:
+refresh the behavior K/V cache of every request in place (projection of all
+rows + attention-pooled anchor), append new behavior rows, score every
+candidate through the decoder stack and the action head, and rank each
+request's candidates.  `value` is candidates per second over the K timed steps
+(inputs resident in HBM); `e2e` is the same through the public API with host
+buffers (pinned host -> device copies of the step's inputs and the device ->
+host read of probabilities and rankings inside the timed region).
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl txs|reference]
+
+Under torchrun every rank runs its own batch (requests shard across GPUs with
+no collective on the data path); rank 0 prints one JSON line.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+from paper_2607_28940_gb300 import workload as W  # noqa: E402
+
+METRIC = "candidates scored/sec per GB300 and p50 request latency vs behavior length L"
+HEADLINE = "small_bf16"
+LAT_WORKLOAD = "ragged_bf16"          # the long-history model for the latency-vs-L sweep
+LAT_LENGTHS = (1024, 2048, 4096, 8192, 16384)
+LAT_M = 1000
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0}
+
+# DRAM traffic per launch measured with ncu (dram__bytes_read.sum +
+# dram__bytes_write.sum) for the kernel classes that can be dominant, with the
+# sha256 prefix of the kernel source at capture time; a source change voids it.
+NCU_TRAFFIC = {}
+
+
+def parse():
+    p = argparse.ArgumentParser()
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=300)
+    p.add_argument("--warmup", type=int, default=20)
+    p.add_argument("--impl", default="txs", choices=["txs", "reference"])
+    p.add_argument("--workload", default=HEADLINE, choices=sorted(W.WORKLOADS))
+    p.add_argument("--mode", default="local_global", choices=["local_global", "full"])
+    p.add_argument("--no-extras", action="store_true", help="skip latency sweep, e2e and CPU baseline")
+    return p.parse_args()
+
+
+def describe(wl: W.Workload, mode: str) -> str:
+    return (f"{wl.name}: R={wl.n_req} requests, {wl.n_layers} layers, d={wl.d_model}, {wl.n_heads} heads, "
+            f"FFN {wl.d_ff}, L={wl.L}, M={wl.M}, +{wl.dL} appended rows/request, S={wl.n_ctx}, k={wl.n_actions}, "
+            f"L_local={wl.l_local}, {mode.upper()} cross-attention")
+
+
+def load_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            p = json.load(f)
+        return {"hbm_gbs": float(p["hbm_gbs"]), "bf16_tflops": float(p["bf16_tflops"]),
+                "bf16_tflops_sustained": float(p.get("bf16_tflops_sustained", p["bf16_tflops"]))}, "measured"
+    except Exception:
+        return dict(FALLBACK_PEAKS, bf16_tflops_sustained=1700.0), "fallback"
+
+
+# ---------------------------------------------------------------- algorithmic work per class
+
+def algorithmic(wl: W.Workload, mode: int, L: np.ndarray, M: np.ndarray, dL: np.ndarray):
+    """Per-step algorithmic (flops, bytes) of each kernel class: what the method
+    must compute and move (bf16 operands, fp32 vectors), independent of how the
+    kernels tile it."""
+    es = 2 if wl.dtype == "bf16" else 4
+    d, F, nL, H, S, k = wl.d_model, wl.d_ff, wl.n_layers, wl.n_heads, wl.n_ctx, wl.n_actions
+    R = wl.n_req
+    n_cand = int(M.sum())
+    N = n_cand + R * S
+    sumL, sumdL = int(L.sum()), int(dL.sum())
+
+    def gemm(m, n, kk, res=False, out_es=es):
+        flops = 2.0 * m * n * kk
+        byt = es * (m * kk + n * kk) + out_es * m * n + (es * m * n if res else 0) + 4 * n
+        return flops, byt
+
+    out = {}
+
+    def add(name, fb):
+        f0, b0 = out.get(name, (0.0, 0.0))
+        out[name] = (f0 + fb[0], b0 + fb[1])
+
+    for rows in (sumL, sumdL):   # rebuild, append
+        add("gemm_kv_build", gemm(rows, 2 * nL * d, d))
+        add("pool", (4.0 * rows * d, es * rows * d + 4 * R * (d + 2)))
+        add("global_kv", (2.0 * R * 2 * nL * d * d, es * 2 * nL * d * d + 4 * R * d * (1 + 2 * nL)))
+    add("pack", (2.0 * n_cand * d * k, es * 2 * N * d + 4 * n_cand * k))
+    L_after = L + dL
+    W_keys = np.minimum(L_after, wl.l_local) + 1 if mode == 0 else L_after
+    rows_per_req = M + S
+    for l in range(nL):
+        add("gemm_qkv", gemm(N, 3 * d, d))
+        add("attn_serving", (4.0 * d * (n_cand * (S + 1) + R * S * S), es * (N * 3 * d + N * d)))
+        add("gemm_oproj_ln", gemm(N, d, d, res=True))
+        add("gemm_q", gemm(N, d, d))
+        kv_bytes = float((W_keys * 2 * d * es).sum())
+        add("attn_cross", (float((4.0 * d * rows_per_req * W_keys).sum()), es * 2 * N * d + kv_bytes))
+        add("gemm_oproj_ln", gemm(N, d, d, res=True))
+        add("gemm_ffn1_gelu", gemm(N, F, d))
+        add("gemm_ffn2_ln", gemm(N, d, F, res=True))
+    add("rank", (float((M.astype(np.float64) ** 2).sum()), 4.0 * n_cand * (k + 1)))
+    return out
+
+
+# ---------------------------------------------------------------- clocks
+
+CLOCK_FIELDS = ("timestamp,index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+                "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+                "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+
+class ClockSampler:
+    """nvidia-smi sampling in the background while the GPU works."""
+
+    def __init__(self, index: int):
+        self.path = tempfile.mktemp(suffix=".csv")
+        self.proc = None
+        self.index = index
+
+    def start(self):
+        try:
+            self.f = open(self.path, "w")
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.index), f"--query-gpu={CLOCK_FIELDS}",
+                                          "--format=csv,noheader,nounits", "-lms", "100"],
+                                         stdout=self.f, stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+        self.t0 = time.time()
+
+    def stop(self):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except Exception:
+                self.proc.kill()
+            self.f.close()
+
+    def summary(self):
+        rows = []
+        try:
+            with open(self.path) as f:
+                for line in f:
+                    parts = [p.strip() for p in line.split(",")]
+                    if len(parts) >= 10:
+                        rows.append(parts)
+        except Exception:
+            pass
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"], "samples": 0}
+        sm = [float(r[2]) for r in rows if r[2].replace(".", "").isdigit()]
+        mx = [float(r[3]) for r in rows if r[3].replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in rows for i in range(4) if r[6 + i].lower() == "active"})
+        pw = [float(r[4]) for r in rows if r[4].replace(".", "").isdigit()]
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(mx) if mx else None,
+                "reasons": reasons, "samples": len(rows), "power_w_max": max(pw) if pw else None}
+
+
+# ---------------------------------------------------------------- the GPU arm
+
+def run_txs(args, rank, world):
+    import torch
+    from paper_2607_28940_gb300 import build as B
+    from paper_2607_28940_gb300 import txs
+
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    if not os.path.exists(txs.LIB_PATH):
+        B.build()
+    mode = txs.LOCAL_GLOBAL if args.mode == "local_global" else txs.FULL
+    base = W.WORKLOADS[args.workload]
+    wl = W.with_sizes(base, seed=base.seed + 1000 * rank)   # each rank: its own shard of requests
+    weights = W.weights(base)                               # one model, replicated
+    b = W.batch(wl)
+    dt = txs.torch_dtype(wl.dtype)
+    n_cand = int(b.cand_off[-1])
+    full_off = b.beh_off
+
+    model = txs.Model(wl, weights, mode)
+    beh = txs.to_device(b.beh, dt)
+    app = txs.to_device(b.app, dt)
+    cand = txs.to_device(b.cand, dt)
+    ctx = txs.to_device(b.ctx.reshape(-1, wl.d_model), dt) if wl.n_ctx else None
+    cache = txs.KVCache(model, full_off, beh, capacity_extra=wl.capacity_extra)
+    ws = torch.empty(txs.workspace_bytes(model, wl.n_req, n_cand), dtype=torch.uint8, device="cuda")
+    logits = torch.empty((n_cand, wl.n_actions), dtype=torch.float32, device="cuda")
+    probs = torch.empty_like(logits)
+    ranks = torch.empty(n_cand, dtype=torch.int32, device="cuda")
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device="cuda")
+    stream = torch.cuda.current_stream()
+
+    def step(beh_t=beh, app_t=app, cand_t=cand, ctx_t=ctx):
+        cache.rebuild(full_off, beh_t)
+        cache.append(b.app_off, app_t)
+        txs.score(model, cache, b.cand_off, cand_t, ctx_t, workspace=ws, out_logits=logits, out_probs=probs)
+        txs.rank(b.cand_off, probs, wl.n_actions, 0, 0, out=ranks)
+
+    def barrier():
+        torch.cuda.synchronize()
+        if world > 1:
+            torch.distributed.barrier()
+
+    def timed(fn, steps, do_flush=True):
+        evs = []
+        for _ in range(steps):
+            if do_flush:
+                flush.zero_()
+            e0 = torch.cuda.Event(enable_timing=True)
+            e1 = torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            fn()
+            e1.record(stream)
+            evs.append((e0, e1))
+        torch.cuda.synchronize()
+        return [a.elapsed_time(c) for a, c in evs]
+
+    clocks = ClockSampler(local)
+    clocks.start()
+    for _ in range(max(args.warmup, 3)):
+        step()
+    barrier()
+    wall0 = time.perf_counter()
+    ms = timed(step, args.steps)
+    barrier()
+    wall = time.perf_counter() - wall0
+    clocks.stop()
+    st = model.device_status()
+    if st != txs.TXS_OK:
+        raise RuntimeError(f"device status {st} after timed region")
+
+    total_ms = float(sum(ms))
+    t = torch.tensor([total_ms], dtype=torch.float64, device="cuda")
+    if world > 1:
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+    total_ms_max = float(t.item())
+    value = world * n_cand * args.steps / (total_ms_max / 1e3)
+
+    # per-kernel breakdown: the same K steps again with event pairs around every launch
+    txs.profile_enable(True)
+    timed(step, args.steps)
+    prof = txs.profile_collect()
+    txs.profile_enable(False)
+    launches_per_step = sum(c for _, c in prof.values()) / args.steps
+
+    out = {"metric": METRIC, "value": value, "unit": "candidates/s", "n_gpus": world, "steps": args.steps,
+           "warmup": args.warmup, "ms_per_step": total_ms_max / args.steps, "higher_is_better": True,
+           "scaling": "weak", "vs_baseline": None, "dtype": "bf16" if wl.dtype == "bf16" else "f32",
+           "data": "synthetic (seeded N(0,1) inputs, N(0,0.02) weights; shapes of the paper's serving setting)"}
+    out["config"] = {"workload": describe(wl, args.mode), "global_batch": n_cand * world,
+                     "requests_per_gpu": wl.n_req, "seq_len": int(b.L.max()),
+                     "step": "in-place cache rebuild + append + score + rank",
+                     "l2": "flushed before every timed step (256 MiB device write, untimed)",
+                     "parallelism": f"request-sharded replicas x{world} (no data-path collective)"}
+    out["wall_s_timed_region"] = wall
+    out["gpu_launches"] = int(round(launches_per_step * args.steps))
+    out["clocks"] = clocks.summary()
+
+    peaks, peak_src = load_peaks()
+    alg = algorithmic(wl, mode, b.L, b.M, b.dL)
+    kern = {}
+    for name, (tot, cnt) in prof.items():
+        per_step_ms = tot / args.steps
+        f, by = alg.get(name, (0.0, 0.0))
+        t_s = per_step_ms / 1e3
+        kern[name] = {"ms_per_step": per_step_ms, "launches_per_step": cnt / args.steps,
+                      "share": tot / max(sum(v[0] for v in prof.values()), 1e-12),
+                      "tflops": f / t_s / 1e12 if t_s > 0 else None, "gbs": by / t_s / 1e9 if t_s > 0 else None}
+    out["kernels"] = kern
+    dom = max(prof.items(), key=lambda kv: kv[1][0])[0]
+    f, by = alg[dom]
+    per_launch_ms = prof[dom][0] / prof[dom][1]
+    launches = prof[dom][1] / args.steps
+    t_tensor = f / (peaks["bf16_tflops"] * 1e12)
+    t_hbm = by / (peaks["hbm_gbs"] * 1e9)
+    if t_tensor >= t_hbm:
+        achieved = f / launches / (per_launch_ms / 1e3) / 1e12
+        roof = {"bound": "tensor", "achieved": achieved, "peak": peaks["bf16_tflops"], "unit": "TFLOP/s"}
+    else:
+        achieved = by / launches / (per_launch_ms / 1e3) / 1e9
+        roof = {"bound": "hbm", "achieved": achieved, "peak": peaks["hbm_gbs"], "unit": "GB/s"}
+    roof["frac"] = roof["achieved"] / roof["peak"]
+    tr = NCU_TRAFFIC.get((args.workload, args.mode, dom))
+    src_sha = hashlib.sha256(open(os.path.join(ROOT, "paper_2607_28940_gb300", "csrc",
+                                               "k_gemm_tc.cu" if dom.startswith("gemm") else "k_attn.cu"),
+                                  "rb").read()).hexdigest()[:12]
+    roof["traffic"] = tr[0] if tr and tr[1] == src_sha else None
+    roof["kernel"] = dom
+    roof["peak_source"] = f"{peak_src} ({'burst' if roof['bound'] == 'tensor' else 'copy'})"
+    roof["algorithmic_per_launch"] = {"flops": f / launches, "bytes": by / launches}
+    out["roofline"] = roof
+
+    if not args.no_extras:
+        out["score_only"] = score_only(txs, torch, model, cache, b, cand, ctx, ws, logits, probs, ranks, wl,
+                                       timed, args.steps)
+        out["e2e"] = e2e(txs, torch, model, cache, b, wl, args, dt, logits, probs, ranks, ws, world)
+        if rank == 0:
+            out["latency_vs_L"] = latency_sweep(txs, torch)
+            out["cpu_baseline"] = cpu_baseline(args.workload, budget_s=12.0)
+    return out
+
+
+def score_only(txs, torch, model, cache, b, cand, ctx, ws, logits, probs, ranks, wl, timed, steps):
+    def fn():
+        txs.score(model, cache, b.cand_off, cand, ctx, workspace=ws, out_logits=logits, out_probs=probs)
+        txs.rank(b.cand_off, probs, wl.n_actions, 0, 0, out=ranks)
+    ms = timed(fn, steps)
+    n = int(b.cand_off[-1])
+    return {"value": n * steps / (sum(ms) / 1e3), "unit": "candidates/s", "ms_per_call": sum(ms) / steps,
+            "what": "score + rank against the prebuilt cache (the online part of the path), L2 flushed"}
+
+
+def e2e(txs, torch, model, cache, b, wl, args, dt, logits, probs, ranks, ws, world):
+    """The step through the public API from pinned host buffers, reading results back."""
+    pin = lambda a: torch.from_numpy(np.ascontiguousarray(a, np.float32)).to(dt).pin_memory()
+    h_beh, h_app, h_cand = pin(b.beh), pin(b.app), pin(b.cand)
+    h_ctx = pin(b.ctx.reshape(-1, wl.d_model)) if wl.n_ctx else None
+    d_beh = torch.empty(h_beh.shape, dtype=dt, device="cuda")
+    d_app = torch.empty(h_app.shape, dtype=dt, device="cuda")
+    d_cand = torch.empty(h_cand.shape, dtype=dt, device="cuda")
+    d_ctx = torch.empty(h_ctx.shape, dtype=dt, device="cuda") if h_ctx is not None else None
+    h_probs = torch.empty(probs.shape, dtype=torch.float32).pin_memory()
+    h_ranks = torch.empty(ranks.shape, dtype=torch.int32).pin_memory()
+    n = int(b.cand_off[-1])
+
+    def one():
+        d_beh.copy_(h_beh, non_blocking=True)
+        d_app.copy_(h_app, non_blocking=True)
+        d_cand.copy_(h_cand, non_blocking=True)
+        if d_ctx is not None:
+            d_ctx.copy_(h_ctx, non_blocking=True)
+        cache.rebuild(b.beh_off, d_beh)
+        cache.append(b.app_off, d_app)
+        txs.score(model, cache, b.cand_off, d_cand, d_ctx, workspace=ws, out_logits=logits, out_probs=probs)
+        txs.rank(b.cand_off, probs, wl.n_actions, 0, 0, out=ranks)
+        h_probs.copy_(probs, non_blocking=True)
+        h_ranks.copy_(ranks, non_blocking=True)
+        torch.cuda.current_stream().synchronize()
+
+    for _ in range(3):
+        one()
+    steps = max(args.steps // 2, 10)
+    t0 = time.perf_counter()
+    for _ in range(steps):
+        one()
+    dt_s = time.perf_counter() - t0
+    t = torch.tensor([dt_s], dtype=torch.float64, device="cuda")
+    if world > 1:
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+    h2d = sum(x.numel() * x.element_size() for x in (h_beh, h_app, h_cand) + ((h_ctx,) if h_ctx is not None else ()))
+    d2h = h_probs.numel() * 4 + h_ranks.numel() * 4
+    return {"value": world * n * steps / float(t.item()), "unit": "candidates/s", "h2d_bytes_per_step": int(h2d),
+            "d2h_bytes_per_step": int(d2h), "steps": steps,
+            "what": "pinned host -> device inputs, full step, device -> host probs and ranks, synchronised per step"}
+
+
+def latency_sweep(txs, torch):
+    """p50 latency of one request (score + rank of M candidates) against prebuilt
+    caches of growing behavior length L, both key-set modes."""
+    base = W.WORKLOADS[LAT_WORKLOAD]
+    weights = W.weights(base)
+    res = {"model": f"{LAT_WORKLOAD} layers/width (d={base.d_model}, {base.n_layers} layers), R=1, M={LAT_M}",
+           "unit": "ms", "note": "CUDA events, weights L2-warm as in steady serving"}
+    for mode_name, mode in (("local_global", txs.LOCAL_GLOBAL), ("full", txs.FULL)):
+        model = txs.Model(base, weights, mode)
+        p50 = {}
+        for L in LAT_LENGTHS:
+            wl = W.with_sizes(base, n_req=1, L=L, M=LAT_M, dL=0)
+            b = W.batch(wl)
+            dt = txs.torch_dtype(wl.dtype)
+            cache = txs.KVCache(model, b.beh_off, txs.to_device(b.beh, dt))
+            cand = txs.to_device(b.cand, dt)
+            ctx = txs.to_device(b.ctx.reshape(-1, wl.d_model), dt)
+            ws = torch.empty(txs.workspace_bytes(model, 1, LAT_M), dtype=torch.uint8, device="cuda")
+            lg = torch.empty((LAT_M, wl.n_actions), dtype=torch.float32, device="cuda")
+            pr = torch.empty_like(lg)
+            rk = torch.empty(LAT_M, dtype=torch.int32, device="cuda")
+            times = []
+            for i in range(40):
+                e0 = torch.cuda.Event(enable_timing=True)
+                e1 = torch.cuda.Event(enable_timing=True)
+                e0.record()
+                txs.score(model, cache, b.cand_off, cand, ctx, workspace=ws, out_logits=lg, out_probs=pr)
+                txs.rank(b.cand_off, pr, wl.n_actions, 0, 0, out=rk)
+                e1.record()
+                e1.synchronize()
+                if i >= 10:
+                    times.append(e0.elapsed_time(e1))
+            p50[str(L)] = statistics.median(times)
+            cache.close()
+        res[mode_name] = p50
+        res[f"{mode_name}_ratio_16384_over_1024"] = p50["16384"] / p50["1024"]
+        model.close()
+    return res
+
+
+# ---------------------------------------------------------------- the oracle (CPU) arm
+
+def oracle_step(O, model, wl, b, r):
+    """One request through the oracle: cache build, append, scoring, ranking."""
+    phi = b.beh[b.beh_off[r]:b.beh_off[r + 1]]
+    c = O.build_cache(model, phi)
+    c = O.append_cache(model, c, b.app[b.app_off[r]:b.app_off[r + 1]])
+    _, pr = O.score_request(model, c, b.ctx[r], b.cand[b.cand_off[r]:b.cand_off[r + 1]])
+    O.rank(pr[:, 0], [0, pr.shape[0]])
+    return pr.shape[0]
+
+
+def cpu_baseline(workload: str, budget_s: float):
+    from oracle import txs_oracle as O
+    wl = W.WORKLOADS[workload]
+    model = O.Model.from_arrays(W.weights(wl), wl)
+    n_done, cands, t_tot = 0, 0, 0.0
+    while n_done < wl.n_req and (t_tot < budget_s or n_done == 0):
+        b = W.batch(wl, requests=[n_done])
+        t0 = time.perf_counter()
+        cands += oracle_step(O, model, wl, b, 0)
+        t_tot += time.perf_counter() - t0
+        n_done += 1
+    return {"value": cands / t_tot, "unit": "candidates/s", "cores": os.cpu_count(), "kind": "oracle",
+            "sample": f"{n_done} of {wl.n_req} requests of {workload}, each cache build + append + score + rank "
+                      f"in float64 NumPy ({t_tot:.1f} s)"}
+
+
+def run_reference(args, rank, world):
+    """The oracle, as it stands, timed on the host cores: each step one request
+    of the same workload (bounded sample), same metric and unit."""
+    from oracle import txs_oracle as O
+    wl = W.WORKLOADS[args.workload]
+    model = O.Model.from_arrays(W.weights(wl), wl)
+    batches = [W.batch(wl, requests=[r]) for r in range(min(wl.n_req, 4))]
+    for i in range(min(max(args.warmup, 1), 2)):
+        oracle_step(O, model, wl, batches[i % len(batches)], 0)
+    cands, t_tot = 0, 0.0
+    for i in range(args.steps):
+        t0 = time.perf_counter()
+        cands += oracle_step(O, model, wl, batches[i % len(batches)], 0)
+        t_tot += time.perf_counter() - t0
+    value = cands / t_tot
+    sample = (f"{args.steps} steps, each one request (M={int(batches[0].M[0])} candidates) of {args.workload}: "
+              f"cache build + append + score + rank in float64 NumPy")
+    return {"impl": "reference", "metric": METRIC, "value": value, "unit": "candidates/s", "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * t_tot / args.steps,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic", "config": {"workload": describe(wl, args.mode), "host": "CPU cores of the GPU box"},
+            "cpu_baseline": {"value": value, "unit": "candidates/s", "cores": os.cpu_count(), "kind": "oracle",
+                             "sample": sample},
+            "e2e": {"value": value, "unit": "candidates/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+
+
+def main():
+    args = parse()
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    if args.impl == "reference":
+        if rank == 0:
+            print(json.dumps(run_reference(args, rank, world)), flush=True)
+        return
+    if world > 1:
+        import torch
+        torch.cuda.set_device(int(os.environ.get("LOCAL_RANK", "0")))
+        torch.distributed.init_process_group("nccl")
+    out = run_txs(args, rank, world)
+    if rank == 0:
+        print(json.dumps(out), flush=True)
+    if world > 1:
+        import torch
+        torch.distributed.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

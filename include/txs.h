@@ -119,6 +119,17 @@ txs_status txs_build_kv_cache(txs_model* model, int32_t n_req, const int32_t* be
 void txs_cache_destroy(txs_kv_cache* cache);
 
 /*
+ * txs_rebuild_kv_cache — nearline refresh in place (App. D, time-based batch
+ * re-encoding): recompute every request of an existing cache from new rows,
+ * exactly as txs_build_kv_cache would, reusing its memory (no allocation).
+ * n_req must equal the cache's; each new L_r must be >= 1 (else
+ * TXS_ERR_COLD_START) and fit the request's capacity from the original build
+ * (else TXS_ERR_CAPACITY; nothing is changed).
+ */
+txs_status txs_rebuild_kv_cache(txs_model* model, txs_kv_cache* cache, int32_t n_req, const int32_t* beh_offsets,
+                                const void* beh_enc, void* stream);
+
+/*
  * txs_append_behavior — incremental update (App. D, incremental-encoding
  * remark): rows new_enc[new_offsets[r] .. new_offsets[r+1]) (device, model
  * dtype, [sum dL_r, d_model]) are projected into the free slots after request

@@ -86,7 +86,10 @@ struct txs_kv_cache {
   uint64_t model_hash = 0;
   long long cap_total = 0;
   std::vector<int> h_off, h_len, h_cap;  // capacity offsets [R+1], lengths, capacities
-  std::vector<int> h_stage;              // host staging for offset uploads
+  int* h_stage = nullptr;                // pinned staging ring for offset uploads
+  int stage_ints = 0;                    // ints per ring slot
+  int stage_next = 0;
+  cudaEvent_t stage_ev[4] = {nullptr, nullptr, nullptr, nullptr};
   int* d_off = nullptr;                  // [R+1]
   int* d_len = nullptr;                  // [R]
   int* d_in_off = nullptr;               // [R+1] offsets of the rows being projected
@@ -295,21 +298,42 @@ txs_status model_prepare(txs_model* m, const void* const* w, cudaStream_t s) {
   return TXS_OK;
 }
 
+// Next slot of the cache's pinned staging ring, once the copy that last used it
+// has run (copies from pinned memory are asynchronous, so a slot is reused
+// only after its event has completed).
+int* stage_slot(txs_kv_cache* c, cudaStream_t s, cudaEvent_t** ev) {
+  const int i = c->stage_next;
+  c->stage_next = (i + 1) & 3;
+  cudaEventSynchronize(c->stage_ev[i]);
+  *ev = &c->stage_ev[i];
+  return c->h_stage + static_cast<size_t>(i) * c->stage_ints;
+}
+
+// Upload n ints from a staging slot to dst on stream s.
+cudaError_t stage_upload(txs_kv_cache* c, int* dst, const int* src, int n, cudaStream_t s) {
+  cudaEvent_t* ev;
+  int* slot = stage_slot(c, s, &ev);
+  std::memcpy(slot, src, sizeof(int) * n);
+  cudaError_t err = cudaMemcpyAsync(dst, slot, sizeof(int) * n, cudaMemcpyHostToDevice, s);
+  if (err != cudaSuccess) return err;
+  return cudaEventRecord(*ev, s);
+}
+
 template <typename T>
 txs_status project_rows(txs_model* m, txs_kv_cache* c, int n_req, const int32_t* in_off, const void* rows,
                         bool append, cudaStream_t s) {
   const txs_config& cf = m->cfg;
   const int d = cf.d_model, nL = cf.n_layers;
   const long long total = in_off[n_req];
-  // stage [in_off (R+1) | dst0 (R)] and upload in one copy
-  c->h_stage.assign(2 * n_req + 1, 0);
+  // [in_off (R+1) | dst0 (R)] in one upload
+  std::vector<int> up(2 * n_req + 1);
   int max_rows = 0;
-  for (int r = 0; r <= n_req; ++r) c->h_stage[r] = in_off[r];
+  for (int r = 0; r <= n_req; ++r) up[r] = in_off[r];
   for (int r = 0; r < n_req; ++r) {
-    c->h_stage[n_req + 1 + r] = c->h_off[r] + (append ? c->h_len[r] : 0);
+    up[n_req + 1 + r] = c->h_off[r] + (append ? c->h_len[r] : 0);
     max_rows = std::max(max_rows, in_off[r + 1] - in_off[r]);
   }
-  TXS_CK(cudaMemcpyAsync(c->d_in_off, c->h_stage.data(), sizeof(int) * (2 * n_req + 1), cudaMemcpyHostToDevice, s));
+  TXS_CK(stage_upload(c, c->d_in_off, up.data(), 2 * n_req + 1, s));
   if (total > 0) {
     EpiArgs e = epi_base(EPI_KV, total, 2 * nL * d, d);
     e.bias = m->b_kv;
@@ -519,7 +543,7 @@ TXS_API txs_status txs_build_kv_cache(txs_model* m, int32_t n_req, const int32_t
   for (int r = 0; r < n_req; ++r) {
     c->h_len[r] = beh_offsets[r + 1] - beh_offsets[r];
     c->h_cap[r] = c->h_len[r] + capacity_extra;
-    max_cap = std::max(max_cap, std::max(c->h_len[r], capacity_extra));
+    max_cap = std::max(max_cap, c->h_cap[r]);
     c->h_off[r] = static_cast<int>(tot);
     tot += c->h_cap[r];
     if (tot > 0x7FFFFFFFLL) {
@@ -550,8 +574,18 @@ TXS_API txs_status txs_build_kv_cache(txs_model* m, int32_t n_req, const int32_t
   c->gkv = static_cast<float*>(A(size_t(4) * nL * 2 * n_req * d));
   c->part = static_cast<float*>(A(size_t(4) * n_req * c->max_chunks * (d + 2)));
   if (st == TXS_OK) {
-    if ((err = cudaMemcpyAsync(c->d_off, c->h_off.data(), 4 * (n_req + 1), cudaMemcpyHostToDevice, s)) != cudaSuccess ||
-        (err = cudaMemcpyAsync(c->d_len, c->h_len.data(), 4 * n_req, cudaMemcpyHostToDevice, s)) != cudaSuccess)
+    c->stage_ints = 2 * n_req + 1;
+    if ((err = cudaMallocHost(&c->h_stage, sizeof(int) * 4 * c->stage_ints)) != cudaSuccess) {
+      c->h_stage = nullptr;
+      st = fail_cuda("cudaMallocHost", err);
+    }
+    for (int i = 0; i < 4 && st == TXS_OK; ++i)
+      if ((err = cudaEventCreateWithFlags(&c->stage_ev[i], cudaEventDisableTiming)) != cudaSuccess)
+        st = fail_cuda("cudaEventCreate", err);
+  }
+  if (st == TXS_OK) {
+    if ((err = stage_upload(c, c->d_off, c->h_off.data(), n_req + 1, s)) != cudaSuccess ||
+        (err = stage_upload(c, c->d_len, c->h_len.data(), n_req, s)) != cudaSuccess)
       st = fail_cuda("upload", err);
   }
   if (st == TXS_OK)
@@ -568,8 +602,33 @@ TXS_API txs_status txs_build_kv_cache(txs_model* m, int32_t n_req, const int32_t
 
 TXS_API void txs_cache_destroy(txs_kv_cache* c) {
   if (!c) return;
+  for (cudaEvent_t e : c->stage_ev)
+    if (e) cudaEventSynchronize(e);
   for (void* p : c->allocs) cudaFree(p);
+  for (cudaEvent_t e : c->stage_ev)
+    if (e) cudaEventDestroy(e);
+  if (c->h_stage) cudaFreeHost(c->h_stage);
   delete c;
+}
+
+TXS_API txs_status txs_rebuild_kv_cache(txs_model* m, txs_kv_cache* c, int32_t n_req, const int32_t* beh_offsets,
+                                        const void* beh_enc, void* stream) {
+  if (!m || !c || !beh_offsets) return TXS_ERR_INVALID_ARG;
+  if (c->model_hash != m->hash) return TXS_ERR_STALE_CACHE;
+  if (n_req != c->n_req || !offsets_ok(beh_offsets, n_req, false)) return TXS_ERR_INVALID_ARG;
+  for (int r = 0; r < n_req; ++r) {
+    if (beh_offsets[r + 1] == beh_offsets[r]) return TXS_ERR_COLD_START;
+    if (beh_offsets[r + 1] - beh_offsets[r] > c->h_cap[r]) return TXS_ERR_CAPACITY;
+  }
+  if (!beh_enc) return TXS_ERR_INVALID_ARG;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  txs_status st = m->cfg.dtype == TXS_BF16 ? project_rows<__nv_bfloat16>(m, c, n_req, beh_offsets, beh_enc, false, s)
+                                           : project_rows<float>(m, c, n_req, beh_offsets, beh_enc, false, s);
+  if (st != TXS_OK) return st;
+  for (int r = 0; r < n_req; ++r) c->h_len[r] = beh_offsets[r + 1] - beh_offsets[r];
+  cudaError_t err = stage_upload(c, c->d_len, c->h_len.data(), n_req, s);
+  if (err != cudaSuccess) return fail_cuda("upload lengths", err);
+  return TXS_OK;
 }
 
 TXS_API txs_status txs_append_behavior(txs_model* m, txs_kv_cache* c, int32_t n_req, const int32_t* new_offsets,
@@ -587,7 +646,7 @@ TXS_API txs_status txs_append_behavior(txs_model* m, txs_kv_cache* c, int32_t n_
                                            : project_rows<float>(m, c, n_req, new_offsets, new_enc, true, s);
   if (st != TXS_OK) return st;
   for (int r = 0; r < n_req; ++r) c->h_len[r] += new_offsets[r + 1] - new_offsets[r];
-  cudaError_t err = cudaMemcpyAsync(c->d_len, c->h_len.data(), 4 * n_req, cudaMemcpyHostToDevice, s);
+  cudaError_t err = stage_upload(c, c->d_len, c->h_len.data(), n_req, s);
   if (err != cudaSuccess) return fail_cuda("upload lengths", err);
   return TXS_OK;
 }

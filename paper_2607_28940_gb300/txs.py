@@ -62,6 +62,7 @@ _SIGS = {
     "txs_model_hash": (ctypes.c_uint64, [_P]),
     "txs_build_kv_cache": (_I32, [_P, _I32, _I32P, _P, _I32, _P, ctypes.POINTER(_P)]),
     "txs_cache_destroy": (None, [_P]),
+    "txs_rebuild_kv_cache": (_I32, [_P, _P, _I32, _I32P, _P, _P]),
     "txs_append_behavior": (_I32, [_P, _P, _I32, _I32P, _P, _P]),
     "txs_cache_read_rows": (_I32, [_P, _I32, _I32, _I32, _I32, _I32, _P, _P]),
     "txs_cache_read_anchor": (_I32, [_P, _I32, _I32, _P, _P]),
@@ -191,6 +192,11 @@ class KVCache:
         _check(lib().txs_build_kv_cache(model.handle, self.n_req, p, _ptr(beh_enc), int(capacity_extra),
                                         _stream(stream), ctypes.byref(h)), "txs_build_kv_cache")
         self.handle = h
+
+    def rebuild(self, beh_offsets, beh_enc: torch.Tensor, stream=None):
+        off, p = _offsets(beh_offsets)
+        _check(lib().txs_rebuild_kv_cache(self.model.handle, self.handle, len(off) - 1, p, _ptr(beh_enc),
+                                          _stream(stream)), "txs_rebuild_kv_cache")
 
     def append(self, new_offsets, new_enc: Optional[torch.Tensor], stream=None, model: Optional[Model] = None):
         off, p = _offsets(new_offsets)
