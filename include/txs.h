@@ -198,6 +198,35 @@ txs_status txs_rank_candidates(int32_t n_req, const int32_t* cand_offsets, const
                                int32_t n_actions, int32_t action, int32_t top_k, int32_t* out_idx,
                                void* stream);
 
+/*
+ * txs_pool_anchor_static — the attention-pooled anchor g of each request (the
+ * value txs_build_kv_cache keeps and txs_cache_read_anchor returns with
+ * which = 2), computed without allocating any memory.  The paper has no
+ * counterpart: this entry point is for callers that cannot allocate device
+ * memory while serving (a process that reserves its GPU memory up front and
+ * forbids driver allocations afterwards, a plugin inside another runtime with
+ * no allocator of its own, a path that cannot take the implicit device
+ * synchronisation of cudaMalloc/cudaFree).
+ *
+ * Inputs as for txs_build_kv_cache: `beh_offsets` host int32 [n_req + 1],
+ * strictly increasing from 0 (an empty request returns TXS_ERR_COLD_START),
+ * `beh_enc` device rows [sum L_r, d_model] in the model dtype.  Output:
+ * `out_g` device float [n_req, d_model].  The call itself never calls
+ * cudaMalloc, cudaFree or any allocating routine.
+ *
+ * Scratch: a 4 MiB file-scope device array of the library (held on every GPU
+ * that loads it until the process exits) — n_req * 16 * (d_model + 2) floats
+ * must fit in 1,048,576 (d_model = 512: up to 127 requests), and n_req <= 1024;
+ * larger calls return TXS_ERR_UNSUPPORTED (txs_last_error says why) before
+ * anything is enqueued.  Every call overwrites all scratch it reads, and all
+ * calls share that one array: calls that overlap on the GPU (other streams,
+ * other threads) race and must be serialised by the caller.  The first call
+ * on each device looks up the array's device address with that device
+ * current; make that first call before any stream capture.
+ */
+txs_status txs_pool_anchor_static(const txs_model* model, int32_t n_req, const int32_t* beh_offsets,
+                                  const void* beh_enc, float* out_g, void* stream);
+
 /* Synchronise the device, read and clear the model's latched device status. */
 txs_status txs_device_status(txs_model* model);
 

@@ -470,6 +470,13 @@ TXS_API const char* txs_status_string(txs_status s) {
 
 TXS_API const char* txs_last_error(void) { return g_last_error.c_str(); }
 
+namespace txs {
+void set_last_error(const char* msg) { set_error(msg); }
+int model_d(const txs_model* m) { return m->cfg.d_model; }
+int model_dtype(const txs_model* m) { return m->cfg.dtype; }
+const float* model_w_pool(const txs_model* m) { return m->w_pool; }
+}  // namespace txs
+
 TXS_API txs_status txs_model_create(const txs_config* cfg, const void* const* weights, txs_model** out) {
   if (!cfg || !weights || !out) return TXS_ERR_INVALID_ARG;
   *out = nullptr;

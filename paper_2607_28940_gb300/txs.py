@@ -72,6 +72,7 @@ _SIGS = {
     "txs_score_candidates": (_I32, [_P, _P, _I32, _I32P, _P, _P, _P, ctypes.c_size_t, _P, _P, _P]),
     "txs_rank_candidates": (_I32, [_I32, _I32P, _P, _I32, _I32, _I32, _P, _P]),
     "txs_device_status": (_I32, [_P]),
+    "txs_pool_anchor_static": (_I32, [_P, _I32, _I32P, _P, _P, _P]),
     "txs_profile_enable": (_I32, [_I32]),
     "txs_profile_collect": (_I32, [ctypes.POINTER(ctypes.c_double), ctypes.POINTER(ctypes.c_int64), _I32]),
     "txs_kernel_class_name": (ctypes.c_char_p, [_I32]),
@@ -268,6 +269,20 @@ def rank(cand_offsets, probs: torch.Tensor, n_actions: int, action: int = 0, top
         out = torch.empty(max(n, 1), dtype=torch.int32, device="cuda")
     _check(lib().txs_rank_candidates(n_req, p, _ptr(probs) if probs is not None and probs.numel() else None,
                                      n_actions, action, top_k, _ptr(out), _stream(stream)), "txs_rank_candidates")
+    return out
+
+
+def pool_anchor_static(model: Model, beh_offsets, beh_enc: torch.Tensor, out: Optional[torch.Tensor] = None,
+                       stream=None) -> torch.Tensor:
+    """Pooled anchor g [n_req, d] without any device allocation inside the
+    library (for callers that cannot allocate while serving; `out` may be
+    preallocated by the caller)."""
+    off, p = _offsets(beh_offsets)
+    n_req = len(off) - 1
+    if out is None:
+        out = torch.empty((n_req, model.wl.d_model), dtype=torch.float32, device="cuda")
+    _check(lib().txs_pool_anchor_static(model.handle, n_req, p, _ptr(beh_enc), _ptr(out), _stream(stream)),
+           "txs_pool_anchor_static")
     return out
 
 
