@@ -189,10 +189,11 @@ def run_txs(args, rank, world):
     if not os.path.exists(txs.LIB_PATH):
         B.build()
     mode = txs.LOCAL_GLOBAL if args.mode == "local_global" else txs.FULL
-    base = W.WORKLOADS[args.workload]
-    wl = W.with_sizes(base, seed=base.seed + 1000 * rank)   # each rank: its own shard of requests
-    weights = W.weights(base)                               # one model, replicated
-    b = W.batch(wl)
+    from paper_2607_28940_gb300 import shard
+    wl = W.WORKLOADS[args.workload]                          # per-rank batch shape
+    # the job is world * R requests; each rank takes its own contiguous block
+    b = W.batch(shard.global_workload(wl, world), requests=shard.shard_requests(wl.n_req, rank, world))
+    weights = W.weights(wl)                                  # one model, replicated
     dt = txs.torch_dtype(wl.dtype)
     n_cand = int(b.cand_off[-1])
     full_off = b.beh_off
@@ -249,11 +250,7 @@ def run_txs(args, rank, world):
     if st != txs.TXS_OK:
         raise RuntimeError(f"device status {st} after timed region")
 
-    total_ms = float(sum(ms))
-    t = torch.tensor([total_ms], dtype=torch.float64, device="cuda")
-    if world > 1:
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-    total_ms_max = float(t.item())
+    total_ms_max = shard.reduce_max(float(sum(ms)), device="cuda")
     value = world * n_cand * args.steps / (total_ms_max / 1e3)
 
     # per-kernel breakdown: the same K steps again with event pairs around every launch
@@ -363,13 +360,11 @@ def e2e(txs, torch, model, cache, b, wl, args, dt, logits, probs, ranks, ws, wor
     t0 = time.perf_counter()
     for _ in range(steps):
         one()
-    dt_s = time.perf_counter() - t0
-    t = torch.tensor([dt_s], dtype=torch.float64, device="cuda")
-    if world > 1:
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+    from paper_2607_28940_gb300 import shard
+    dt_s = shard.reduce_max(time.perf_counter() - t0, device="cuda")
     h2d = sum(x.numel() * x.element_size() for x in (h_beh, h_app, h_cand) + ((h_ctx,) if h_ctx is not None else ()))
     d2h = h_probs.numel() * 4 + h_ranks.numel() * 4
-    return {"value": world * n * steps / float(t.item()), "unit": "candidates/s", "h2d_bytes_per_step": int(h2d),
+    return {"value": world * n * steps / dt_s, "unit": "candidates/s", "h2d_bytes_per_step": int(h2d),
             "d2h_bytes_per_step": int(d2h), "steps": steps,
             "what": "pinned host -> device inputs, full step, device -> host probs and ranks, synchronised per step"}
 
