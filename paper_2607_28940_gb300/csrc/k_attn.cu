@@ -18,6 +18,10 @@ namespace txs {
 
 namespace {
 
+}  // namespace
+
+namespace {
+
 template <typename T, int DH>
 struct Group {
   static constexpr int VEC = Vec16<T>::N;
@@ -49,6 +53,36 @@ struct OnlineSoftmax {
   }
 };
 
+
+// Online softmax over n_keys keys whose rows are `key_row(t)` (element
+// pointers of width d in global memory; this thread's slice at `col`), one key
+// per step (measured faster than batching keys: fewer registers, more warps).
+template <typename T, typename G, typename KeyRow>
+__device__ __forceinline__ void attend_rows(const float* q, int n_keys, int col, unsigned gmask, float scale,
+                                            OnlineSoftmax& smx, float* acc, KeyRow key_row) {
+  constexpr int VEC = G::VEC;
+  for (int t = 0; t < n_keys; ++t) {
+    const T* kr;
+    const T* vr;
+    key_row(t, kr, vr);
+    float k[VEC], v[VEC];
+    Vec16<T>::load(kr + col, k);
+    Vec16<T>::load(vr + col, v);
+    float dot = 0.f;
+#pragma unroll
+    for (int i = 0; i < VEC; ++i) dot = fmaf(q[i], k[i], dot);
+    dot = G::reduce(dot, gmask) * scale;
+    float corr, w;
+    smx.push(dot, corr, w);
+#pragma unroll
+    for (int i = 0; i < VEC; ++i) acc[i] = acc[i] * corr + w * v[i];
+  }
+}
+
+// Serving-stream attention: thread group per (row, head); a candidate row
+// attends to the S context rows of its request and to itself, a context row to
+// the S context rows.  The context rows' K/V are read by every row of the
+// request and stay in L1.
 template <typename T, int DH>
 __global__ void __launch_bounds__(256) serving_attn_kernel(const T* __restrict__ qkv, T* __restrict__ out,
                                                            const int* __restrict__ row_req, int n_rows,
@@ -58,9 +92,9 @@ __global__ void __launch_bounds__(256) serving_attn_kernel(const T* __restrict__
   const long long gid = static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x;
   const long long pair = gid / G::TPH;
   const int sub = static_cast<int>(gid % G::TPH);
-  const bool active = pair < static_cast<long long>(n_rows) * H;
-  const int row = active ? static_cast<int>(pair / H) : 0;
-  const int h = active ? static_cast<int>(pair % H) : 0;
+  if (pair >= static_cast<long long>(n_rows) * H) return;   // whole group
+  const int row = static_cast<int>(pair / H);
+  const int h = static_cast<int>(pair % H);
   const long long ld = 3LL * d;
   const int col = h * DH + sub * VEC;
   const unsigned gmask = G::mask();
@@ -68,30 +102,19 @@ __global__ void __launch_bounds__(256) serving_attn_kernel(const T* __restrict__
   Vec16<T>::load(qkv + row * ld + col, q);
 #pragma unroll
   for (int i = 0; i < VEC; ++i) acc[i] = 0.f;
-  OnlineSoftmax sm;
+  OnlineSoftmax smx;
   const int r = __ldg(row_req + row);
-  const int c0 = n_cand_rows + r * S;
+  const long long c0 = n_cand_rows + static_cast<long long>(r) * S;
   const int n_keys = S + (row < n_cand_rows ? 1 : 0);
-  for (int j = 0; j < n_keys; ++j) {
-    const int krow = j < S ? c0 + j : row;
-    float k[VEC], v[VEC];
-    Vec16<T>::load(qkv + krow * ld + d + col, k);
-    Vec16<T>::load(qkv + krow * ld + 2 * d + col, v);
-    float dot = 0.f;
+  attend_rows<T, G>(q, n_keys, col, gmask, scale, smx, acc, [&](int t, const T*& kr, const T*& vr) {
+    const long long krow = t < S ? c0 + t : row;
+    kr = qkv + krow * ld + d;
+    vr = qkv + krow * ld + 2 * d;
+  });
+  const float inv = 1.f / smx.l;
 #pragma unroll
-    for (int i = 0; i < VEC; ++i) dot = fmaf(q[i], k[i], dot);
-    dot = G::reduce(dot, gmask) * scale;
-    float corr, w;
-    sm.push(dot, corr, w);
-#pragma unroll
-    for (int i = 0; i < VEC; ++i) acc[i] = acc[i] * corr + w * v[i];
-  }
-  if (active) {
-    const float inv = 1.f / sm.l;
-#pragma unroll
-    for (int i = 0; i < VEC; ++i) acc[i] *= inv;
-    Vec16<T>::store(out + static_cast<long long>(row) * d + col, acc);
-  }
+  for (int i = 0; i < VEC; ++i) acc[i] *= inv;
+  Vec16<T>::store(out + static_cast<long long>(row) * d + col, acc);
 }
 
 struct CrossArgs {
@@ -116,9 +139,9 @@ __global__ void __launch_bounds__(256) cross_attn_kernel(const T* __restrict__ q
   const long long gid = static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x;
   const long long pair = gid / G::TPH;
   const int sub = static_cast<int>(gid % G::TPH);
-  const bool active = pair < static_cast<long long>(a.n_rows) * a.H;
-  const int row = active ? static_cast<int>(pair / a.H) : 0;
-  const int h = active ? static_cast<int>(pair % a.H) : 0;
+  if (pair >= static_cast<long long>(a.n_rows) * a.H) return;   // whole group
+  const int row = static_cast<int>(pair / a.H);
+  const int h = static_cast<int>(pair % a.H);
   const int col = h * DH + sub * VEC;
   const int d = a.d;
   const unsigned gmask = G::mask();
@@ -131,19 +154,10 @@ __global__ void __launch_bounds__(256) cross_attn_kernel(const T* __restrict__ q
   const int len = __ldg(a.kv_len + r);
   const long long base = __ldg(a.kv_off + r);
   const int lo = (a.mode == TXS_ATTN_LOCAL_GLOBAL) ? max(0, len - a.l_local) : 0;
-  for (int j = lo; j < len; ++j) {
-    float k[VEC], v[VEC];
-    Vec16<T>::load(Kc + (base + j) * d + col, k);
-    Vec16<T>::load(Vc + (base + j) * d + col, v);
-    float dot = 0.f;
-#pragma unroll
-    for (int i = 0; i < VEC; ++i) dot = fmaf(q[i], k[i], dot);
-    dot = G::reduce(dot, gmask) * a.scale;
-    float corr, w;
-    sm.push(dot, corr, w);
-#pragma unroll
-    for (int i = 0; i < VEC; ++i) acc[i] = acc[i] * corr + w * v[i];
-  }
+  attend_rows<T, G>(q, len - lo, col, gmask, a.scale, sm, acc, [&](int t, const T*& kr, const T*& vr) {
+    kr = Kc + (base + lo + t) * d;
+    vr = Vc + (base + lo + t) * d;
+  });
   if (a.mode == TXS_ATTN_LOCAL_GLOBAL) {
     const float* kg = a.Kg + static_cast<long long>(r) * d + col;
     const float* vg = a.Vg + static_cast<long long>(r) * d + col;
@@ -156,22 +170,10 @@ __global__ void __launch_bounds__(256) cross_attn_kernel(const T* __restrict__ q
 #pragma unroll
     for (int i = 0; i < VEC; ++i) acc[i] = acc[i] * corr + w * __ldg(vg + i);
   }
-  if (active) {
-    const float inv = 1.f / sm.l;
+  const float inv = 1.f / sm.l;
 #pragma unroll
-    for (int i = 0; i < VEC; ++i) acc[i] *= inv;
-    Vec16<T>::store(out + static_cast<long long>(row) * d + col, acc);
-  }
-}
-
-template <typename T, int DH>
-cudaError_t serving_launch(const T* qkv, T* out, const int* row_req, int n_rows, int n_cand_rows, int S, int H, int d,
-                           cudaStream_t s) {
-  const long long threads = static_cast<long long>(n_rows) * H * Group<T, DH>::TPH;
-  const int blocks = static_cast<int>((threads + 255) / 256);
-  serving_attn_kernel<T, DH><<<blocks, 256, 0, s>>>(qkv, out, row_req, n_rows, n_cand_rows, S, H, d,
-                                                    (1.0f / sqrtf(static_cast<float>(DH))));
-  return cudaGetLastError();
+  for (int i = 0; i < VEC; ++i) acc[i] *= inv;
+  Vec16<T>::store(out + static_cast<long long>(row) * d + col, acc);
 }
 
 template <typename T, int DH>
@@ -184,6 +186,16 @@ cudaError_t cross_launch(const T* q, T* out, const T* Kc, const T* Vc, CrossArgs
 }
 
 }  // namespace
+
+template <typename T, int DH>
+static cudaError_t serving_launch(const T* qkv, T* out, const int* row_req, int n_rows, int n_cand_rows, int S, int H,
+                                  int d, cudaStream_t s) {
+  const long long threads = static_cast<long long>(n_rows) * H * Group<T, DH>::TPH;
+  const int blocks = static_cast<int>((threads + 255) / 256);
+  serving_attn_kernel<T, DH><<<blocks, 256, 0, s>>>(qkv, out, row_req, n_rows, n_cand_rows, S, H, d,
+                                                    1.0f / sqrtf(static_cast<float>(DH)));
+  return cudaGetLastError();
+}
 
 template <typename T>
 cudaError_t launch_serving_attn(const T* qkv, T* out, const int* row_req, int n_rows, int n_cand_rows, int S, int H,

@@ -12,17 +12,27 @@
 
 namespace txs {
 
-constexpr int kPoolChunkV = 128;
+constexpr int kPoolChunkV = 64;
 extern const int kPoolChunk = kPoolChunkV;
 
 namespace {
 
-template <typename T>
+constexpr int kPoolWarps = 8;
+constexpr int kPoolRowsPerWarp = kPoolChunkV / kPoolWarps;
+
+// One CTA per (chunk of kPoolChunk rows, request).  Each warp loads its rows
+// (all loads issued before any arithmetic), computes the pooling logits with a
+// warp reduction and folds the rows into an online-softmax state; the CTA then
+// merges its warps' states.  One coalesced read of the behavior rows.
+template <typename T, int MAXC>
 __global__ void __launch_bounds__(256) pool_partial_kernel(const T* __restrict__ phi, const int* __restrict__ seg_off,
                                                            const float* __restrict__ w_pool, int d, float inv_sqrt_d,
-                                                           int max_chunks, float* __restrict__ part) {
-  __shared__ float z[kPoolChunkV];
-  __shared__ float red[8];
+                                                           int max_chunks, float* __restrict__ part,
+                                                           int merge_existing, float* st_m, float* st_s,
+                                                           float* st_acc, float* __restrict__ g, int* counter) {
+  constexpr int VEC = Vec16<T>::N;               // MAXC: 16-byte chunks per lane, ceil(d / (32 VEC))
+  __shared__ float sm_m[kPoolWarps], sm_s[kPoolWarps];
+  __shared__ float sm_acc[kPoolWarps][512];
   const int r = blockIdx.y, c = blockIdx.x;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int seg_beg = seg_off[r], seg_end = seg_off[r + 1];
@@ -37,103 +47,192 @@ __global__ void __launch_bounds__(256) pool_partial_kernel(const T* __restrict__
     }
     return;
   }
-  for (int i = warp; i < nrows; i += 8) {
-    const T* row = phi + static_cast<long long>(beg + i) * d;
-    float dot = 0.f;
-    for (int k = lane; k < d; k += 32) dot = fmaf(Elem<T>::load(row + k), __ldg(w_pool + k), dot);
+  constexpr int nch = MAXC;
+  float w[MAXC][VEC];
 #pragma unroll
-    for (int o = 16; o > 0; o >>= 1) dot += __shfl_xor_sync(0xffffffffu, dot, o);
-    if (lane == 0) z[i] = dot * inv_sqrt_d;
+  for (int j = 0; j < MAXC; ++j) {
+    const int col = (j * 32 + lane) * VEC;
+#pragma unroll
+    for (int i = 0; i < VEC; ++i) w[j][i] = (j < nch && col + i < d) ? __ldg(w_pool + col + i) : 0.f;
+  }
+  // this warp's rows: beg + warp + 8 t, loaded RB at a time (all loads of a
+  // batch issued before its arithmetic)
+  constexpr int RB = MAXC >= 4 ? 2 : (MAXC == 2 ? 4 : kPoolRowsPerWarp);
+  float m = -INFINITY, s = 0.f;
+  float acc[MAXC][VEC];
+#pragma unroll
+  for (int j = 0; j < MAXC; ++j)
+#pragma unroll
+    for (int q = 0; q < VEC; ++q) acc[j][q] = 0.f;
+#pragma unroll
+  for (int t0 = 0; t0 < kPoolRowsPerWarp; t0 += RB) {
+    float v[RB][MAXC][VEC];
+#pragma unroll
+    for (int t = 0; t < RB; ++t) {
+      const int i = warp + kPoolWarps * (t0 + t);
+#pragma unroll
+      for (int j = 0; j < MAXC; ++j) {
+        const int col = (j * 32 + lane) * VEC;
+        if (i < nrows && col < d) Vec16<T>::load(phi + static_cast<long long>(beg + i) * d + col, v[t][j]);
+        else {
+#pragma unroll
+          for (int q = 0; q < VEC; ++q) v[t][j][q] = 0.f;
+        }
+      }
+    }
+#pragma unroll
+    for (int t = 0; t < RB; ++t) {
+      if (warp + kPoolWarps * (t0 + t) >= nrows) break;
+      float dot = 0.f;
+#pragma unroll
+      for (int j = 0; j < MAXC; ++j)
+#pragma unroll
+        for (int q = 0; q < VEC; ++q) dot = fmaf(v[t][j][q], w[j][q], dot);
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) dot += __shfl_xor_sync(0xffffffffu, dot, o);
+      const float z = dot * inv_sqrt_d;
+      const float mn = fmaxf(m, z);
+      const float corr = expf(m - mn);
+      const float e = expf(z - mn);
+      s = s * corr + e;
+#pragma unroll
+      for (int j = 0; j < MAXC; ++j)
+#pragma unroll
+        for (int q = 0; q < VEC; ++q) acc[j][q] = fmaf(acc[j][q], corr, e * v[t][j][q]);
+      m = mn;
+    }
+  }
+#pragma unroll
+  for (int j = 0; j < MAXC; ++j) {
+    const int col = (j * 32 + lane) * VEC;
+#pragma unroll
+    for (int q = 0; q < VEC; ++q)
+      if (j < nch && col + q < d) sm_acc[warp][col + q] = acc[j][q];
+  }
+  if (lane == 0) {
+    sm_m[warp] = m;
+    sm_s[warp] = s;
   }
   __syncthreads();
-  float m = -INFINITY;
-  for (int i = tid; i < nrows; i += 256) m = fmaxf(m, z[i]);
+  float M = -INFINITY;
 #pragma unroll
-  for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
-  if (lane == 0) red[warp] = m;
-  __syncthreads();
-  m = red[0];
+  for (int w8 = 0; w8 < kPoolWarps; ++w8) M = fmaxf(M, sm_m[w8]);
+  float scale[kPoolWarps];
+  float S = 0.f;
 #pragma unroll
-  for (int w = 1; w < 8; ++w) m = fmaxf(m, red[w]);
-  __syncthreads();
-  for (int i = tid; i < nrows; i += 256) z[i] = expf(z[i] - m);
-  __syncthreads();
+  for (int w8 = 0; w8 < kPoolWarps; ++w8) {
+    scale[w8] = sm_s[w8] > 0.f ? expf(sm_m[w8] - M) : 0.f;
+    S += sm_s[w8] * scale[w8];
+  }
   for (int k = tid; k < d; k += 256) {
     float a = 0.f;
-    for (int i = 0; i < nrows; ++i) a = fmaf(z[i], Elem<T>::load(phi + static_cast<long long>(beg + i) * d + k), a);
+#pragma unroll
+    for (int w8 = 0; w8 < kPoolWarps; ++w8) a = fmaf(sm_acc[w8][k], scale[w8], a);
     out[2 + k] = a;
   }
   if (tid == 0) {
-    float s = 0.f;
-    for (int i = 0; i < nrows; ++i) s += z[i];
-    out[0] = m;
-    out[1] = s;
+    out[0] = M;
+    out[1] = S;
   }
-}
-
-// Per request: merge the chunk states (and, for an append, the stored state)
-// into the stored state and write g = acc / s.
-__global__ void __launch_bounds__(256) pool_merge_kernel(const float* __restrict__ part, const int* __restrict__ seg_off,
-                                                         int max_chunks, int d, int merge_existing, float* st_m,
-                                                         float* st_s, float* st_acc, float* __restrict__ g) {
-  const int r = blockIdx.x;
-  const int rows = seg_off[r + 1] - seg_off[r];
-  const int nch = (rows + kPoolChunkV - 1) / kPoolChunkV;
-  const float* p = part + static_cast<long long>(r) * max_chunks * (d + 2);
+  // The last chunk CTA of request r to finish merges the request's chunk states
+  // (and, for an append, the stored state) and writes g = acc / s.
+  __shared__ int is_last;
+  __threadfence();
+  __syncthreads();
+  const int nch_r = (seg_end - seg_beg + kPoolChunkV - 1) / kPoolChunkV;
+  if (tid == 0) is_last = atomicAdd(counter + r, 1) == nch_r - 1;
+  __syncthreads();
+  if (!is_last) return;
+  __threadfence();
+  const float* pr = part + static_cast<long long>(r) * max_chunks * (d + 2);
   const float old_m = merge_existing ? st_m[r] : -INFINITY;
   const float old_s = merge_existing ? st_s[r] : 0.f;
-  float M = old_m;
-  for (int c = 0; c < nch; ++c) M = fmaxf(M, p[static_cast<long long>(c) * (d + 2)]);
-  const float w_old = merge_existing ? expf(old_m - M) : 0.f;
-  float S = old_s * w_old;
-  for (int c = 0; c < nch; ++c) {
-    const float* pc = p + static_cast<long long>(c) * (d + 2);
-    S += pc[1] * expf(pc[0] - M);
+  float Mr = old_m;
+  for (int ch = 0; ch < nch_r; ++ch) Mr = fmaxf(Mr, __ldcg(pr + static_cast<long long>(ch) * (d + 2)));
+  const float w_old = merge_existing ? expf(old_m - Mr) : 0.f;
+  float Sr = old_s * w_old;
+  for (int ch = 0; ch < nch_r; ++ch) {
+    const float* pc = pr + static_cast<long long>(ch) * (d + 2);
+    Sr += __ldcg(pc + 1) * expf(__ldcg(pc) - Mr);
   }
-  for (int k = threadIdx.x; k < d; k += blockDim.x) {
+  for (int k = tid; k < d; k += 256) {
     float a = merge_existing ? st_acc[static_cast<long long>(r) * d + k] * w_old : 0.f;
-    for (int c = 0; c < nch; ++c) {
-      const float* pc = p + static_cast<long long>(c) * (d + 2);
-      a = fmaf(pc[2 + k], expf(pc[0] - M), a);
+    for (int ch = 0; ch < nch_r; ++ch) {
+      const float* pc = pr + static_cast<long long>(ch) * (d + 2);
+      a = fmaf(__ldcg(pc + 2 + k), expf(__ldcg(pc) - Mr), a);
     }
     st_acc[static_cast<long long>(r) * d + k] = a;
-    g[static_cast<long long>(r) * d + k] = a / S;
+    g[static_cast<long long>(r) * d + k] = a / Sr;
   }
   __syncthreads();
-  if (threadIdx.x == 0) {
-    st_m[r] = M;
-    st_s[r] = S;
+  if (tid == 0) {
+    st_m[r] = Mr;
+    st_s[r] = Sr;
+    counter[r] = 0;   // ready for the next call
   }
 }
 
-// Anchor projections for every layer: gkv[blk][r][c] = g[r] . Wt[n] + b[n],
-// n = blk * d + c, blk = 2 l + {0: K, 1: V}.  One warp per output column n.
-template <typename T>
-__global__ void __launch_bounds__(256) global_kv_kernel(const float* __restrict__ g, const T* __restrict__ Wt,
-                                                        const float* __restrict__ b, float* __restrict__ gkv, int R,
-                                                        int d, int n_total) {
+// Anchor projections of every layer: gkv[blk][r][c] = g[r] . Wt[n] + b[n] with
+// n = blk * d + c, blk = 2 l + {0: K, 1: V}.  One warp per (column n, group of
+// 8 requests): the weight row is read once per warp (coalesced), the 8 dot
+// products are reduced with shuffles.
+constexpr int kAnchorReqPerWarp = 8;
+
+template <typename T, int NCH>
+__global__ void __launch_bounds__(256) anchor_proj_kernel(const float* __restrict__ g, const T* __restrict__ Wt,
+                                                          const float* __restrict__ b, float* __restrict__ gkv,
+                                                          int R, int d, int n_total) {
+  constexpr int VEC = Vec16<T>::N;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int n = blockIdx.x * 8 + warp;
-  if (n >= n_total) return;
-  float w[16];
+  const long long wid = static_cast<long long>(blockIdx.x) * 8 + warp;
+  const int r_groups = (R + kAnchorReqPerWarp - 1) / kAnchorReqPerWarp;
+  if (wid >= static_cast<long long>(n_total) * r_groups) return;
+  const int n = static_cast<int>(wid / r_groups);
+  const int r0 = static_cast<int>(wid % r_groups) * kAnchorReqPerWarp;
+  float w[NCH][VEC];
 #pragma unroll
-  for (int i = 0; i < 16; ++i) {
-    const int k = lane + 32 * i;
-    w[i] = k < d ? Elem<T>::load(Wt + static_cast<long long>(n) * d + k) : 0.f;
-  }
-  const int blk = n / d, c = n - blk * d;
-  const float bias = b[n];
-  for (int r = 0; r < R; ++r) {
-    const float* gr = g + static_cast<long long>(r) * d;
-    float dot = 0.f;
+  for (int j = 0; j < NCH; ++j) {
+    const int col = (j * 32 + lane) * VEC;
+    if (col < d) Vec16<T>::load(Wt + static_cast<long long>(n) * d + col, w[j]);
+    else {
 #pragma unroll
-    for (int i = 0; i < 16; ++i) {
-      const int k = lane + 32 * i;
-      if (k < d) dot = fmaf(w[i], gr[k], dot);
+      for (int q = 0; q < VEC; ++q) w[j][q] = 0.f;
     }
+  }
+  float dot[kAnchorReqPerWarp];
 #pragma unroll
-    for (int o = 16; o > 0; o >>= 1) dot += __shfl_xor_sync(0xffffffffu, dot, o);
-    if (lane == 0) gkv[(static_cast<long long>(blk) * R + r) * d + c] = dot + bias;
+  for (int t = 0; t < kAnchorReqPerWarp; ++t) {
+    dot[t] = 0.f;
+    const int r = r0 + t;
+    if (r < R) {
+#pragma unroll
+      for (int j = 0; j < NCH; ++j) {
+        const int col = (j * 32 + lane) * VEC;
+        if (col < d) {
+          const float4* gp = reinterpret_cast<const float4*>(g + static_cast<long long>(r) * d + col);
+#pragma unroll
+          for (int q4 = 0; q4 < VEC / 4; ++q4) {
+            const float4 x = __ldg(gp + q4);
+            dot[t] = fmaf(w[j][4 * q4], x.x, dot[t]);
+            dot[t] = fmaf(w[j][4 * q4 + 1], x.y, dot[t]);
+            dot[t] = fmaf(w[j][4 * q4 + 2], x.z, dot[t]);
+            dot[t] = fmaf(w[j][4 * q4 + 3], x.w, dot[t]);
+          }
+        }
+      }
+    }
+  }
+#pragma unroll
+  for (int t = 0; t < kAnchorReqPerWarp; ++t)
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) dot[t] += __shfl_xor_sync(0xffffffffu, dot[t], o);
+  if (lane < kAnchorReqPerWarp && r0 + lane < R) {
+    float v = 0.f;
+#pragma unroll
+    for (int t = 0; t < kAnchorReqPerWarp; ++t)
+      if (t == lane) v = dot[t];
+    const int blk = n / d, c = n - blk * d;
+    gkv[(static_cast<long long>(blk) * R + r0 + lane) * d + c] = v + __ldg(b + n);
   }
 }
 
@@ -198,29 +297,44 @@ __global__ void hash_kernel(const uint32_t* __restrict__ p, long long n_words, u
 template <typename T>
 cudaError_t launch_pool(const T* phi, const int* seg_off, int R, int max_rows, const float* w_pool, int d,
                         int max_chunks, float* part, int merge_existing, float* st_m, float* st_s, float* st_acc,
-                        float* g, cudaStream_t s) {
+                        float* g, int* counter, cudaStream_t s) {
   const int chunks = (max_rows + kPoolChunkV - 1) / kPoolChunkV;
   if (chunks > max_chunks) return cudaErrorInvalidValue;
+  if (chunks == 0) return cudaSuccess;   // no new rows: the stored state and g stay as they are
+  constexpr int VEC = Vec16<T>::N;
+  const int nch = (d + 32 * VEC - 1) / (32 * VEC);
+  const float isd = 1.0f / sqrtf(static_cast<float>(d));
+  const dim3 grid(chunks, R);
   prof_begin(KC_POOL, s);
-  if (chunks > 0) {
-    pool_partial_kernel<T><<<dim3(chunks, R), 256, 0, s>>>(phi, seg_off, w_pool, d, 1.0f / sqrtf(static_cast<float>(d)),
-                                                          max_chunks, part);
-    cudaError_t err = cudaGetLastError();
-    if (err != cudaSuccess) return err;
-  }
-  pool_merge_kernel<<<R, 256, 0, s>>>(part, seg_off, max_chunks, d, merge_existing, st_m, st_s, st_acc, g);
+  if (nch == 1)
+    pool_partial_kernel<T, 1><<<grid, 256, 0, s>>>(phi, seg_off, w_pool, d, isd, max_chunks, part, merge_existing,
+                                                   st_m, st_s, st_acc, g, counter);
+  else if (nch == 2)
+    pool_partial_kernel<T, 2><<<grid, 256, 0, s>>>(phi, seg_off, w_pool, d, isd, max_chunks, part, merge_existing,
+                                                   st_m, st_s, st_acc, g, counter);
+  else if (nch <= 4)
+    pool_partial_kernel<T, 4><<<grid, 256, 0, s>>>(phi, seg_off, w_pool, d, isd, max_chunks, part, merge_existing,
+                                                   st_m, st_s, st_acc, g, counter);
+  else
+    return cudaErrorInvalidValue;
   cudaError_t err = cudaGetLastError();
   prof_end(KC_POOL, s);
   return err;
 }
 
 template <typename T>
-cudaError_t launch_global_kv(const float* g, const T* Wt_kv, const float* b_kv, float* gkv, int R, int d, int n_layers,
-                             cudaStream_t s) {
-  if (d > 512) return cudaErrorInvalidValue;
+cudaError_t launch_anchor_proj(const float* g, const T* Wt_kv, const float* b_kv, float* gkv, int R, int d,
+                               int n_layers, cudaStream_t s) {
+  constexpr int VEC = Vec16<T>::N;
+  const int nch = (d + 32 * VEC - 1) / (32 * VEC);
   const int n_total = 2 * n_layers * d;
+  const long long warps = static_cast<long long>(n_total) * ((R + kAnchorReqPerWarp - 1) / kAnchorReqPerWarp);
+  const int blocks = static_cast<int>((warps + 7) / 8);
   prof_begin(KC_GLOBAL_KV, s);
-  global_kv_kernel<T><<<(n_total + 7) / 8, 256, 0, s>>>(g, Wt_kv, b_kv, gkv, R, d, n_total);
+  if (nch == 1) anchor_proj_kernel<T, 1><<<blocks, 256, 0, s>>>(g, Wt_kv, b_kv, gkv, R, d, n_total);
+  else if (nch == 2) anchor_proj_kernel<T, 2><<<blocks, 256, 0, s>>>(g, Wt_kv, b_kv, gkv, R, d, n_total);
+  else if (nch <= 4) anchor_proj_kernel<T, 4><<<blocks, 256, 0, s>>>(g, Wt_kv, b_kv, gkv, R, d, n_total);
+  else return cudaErrorInvalidValue;
   cudaError_t err = cudaGetLastError();
   prof_end(KC_GLOBAL_KV, s);
   return err;
@@ -260,9 +374,9 @@ cudaError_t launch_hash(const void* p, long long bytes, uint64_t salt, unsigned 
 
 #define TXS_INST(T)                                                                                                 \
   template cudaError_t launch_pool<T>(const T*, const int*, int, int, const float*, int, int, float*, int, float*, \
-                                      float*, float*, float*, cudaStream_t);                                        \
-  template cudaError_t launch_global_kv<T>(const float*, const T*, const float*, float*, int, int, int,            \
-                                           cudaStream_t);                                                           \
+                                      float*, float*, float*, int*, cudaStream_t);                                  \
+  template cudaError_t launch_anchor_proj<T>(const float*, const T*, const float*, float*, int, int, int,          \
+                                             cudaStream_t);                                                         \
   template cudaError_t launch_transpose<T>(const T*, T*, int, int, cudaStream_t);                                  \
   template cudaError_t launch_to_f32<T>(const T*, float*, long long, cudaStream_t);                                \
   template cudaError_t launch_fold_head<T>(const T*, const T*, const T*, float*, float*, int, int, cudaStream_t);

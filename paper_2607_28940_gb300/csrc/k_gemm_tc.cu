@@ -7,11 +7,13 @@
 // cross-attention query, the output projections with residual + LayerNorm
 // (Sec. 4.1.2 crossAttend equation) and the FFN with GELU.
 //
-// One CTA computes a 128 x BN tile: warp 0 streams A/B tiles with TMA into a
-// STAGES-deep ring of 128-byte-swizzled shared-memory buffers, warp 1 issues
-// tcgen05.mma (M=128, N<=256 per instruction, K=16) into TMEM, warps 2-5 read
-// the accumulator back with tcgen05.ld (one row per thread) and run the
-// epilogue.  All waits are bounded; a timeout latches TXS_ERR_DEVICE_TIMEOUT.
+// Persistent kernel, one CTA per SM, 128 x BN output tiles: warp 0 streams A/B
+// tiles with TMA into a STAGES-deep ring of 128-byte-swizzled shared-memory
+// buffers, warp 1 issues tcgen05.mma (M=128, N<=256 per instruction, K=16)
+// into one of two TMEM accumulators, warps 2-9 read the accumulator back with
+// tcgen05.ld (one row per thread, two warps per row block, each half of the
+// columns) and run the epilogue while the next tile accumulates into the other
+// buffer.  All waits are bounded; a timeout latches TXS_ERR_DEVICE_TIMEOUT.
 #include <cstdio>
 
 #include "txs_internal.cuh"
@@ -22,7 +24,6 @@ namespace tc {
 constexpr int BM = 128;
 constexpr int BK = 64;                        // 64 bf16 = one 128-byte swizzle row
 constexpr int A_STAGE_BYTES = BM * BK * 2;    // 16 KB
-constexpr int NUM_THREADS = 192;
 
 // ------------------------------------------------------------------ PTX wrappers
 
@@ -165,13 +166,21 @@ __device__ __forceinline__ void tmem_st32(uint32_t taddr, const float* v) {
       : "memory");
 }
 
+__device__ __forceinline__ void named_bar(int id, int count) {
+  asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(count) : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
+
 // ------------------------------------------------------------------ epilogues
 
-__device__ __forceinline__ void load_bias32(const float* bias, int n, float* b) {
-  const float4* p = reinterpret_cast<const float4*>(bias + n);
+__device__ __forceinline__ void load_f32x32(const float* p, float* b) {
+  const float4* q = reinterpret_cast<const float4*>(p);
 #pragma unroll
   for (int j = 0; j < 8; ++j) {
-    float4 t = __ldg(p + j);
+    float4 t = __ldg(q + j);
     b[4 * j] = t.x; b[4 * j + 1] = t.y; b[4 * j + 2] = t.z; b[4 * j + 3] = t.w;
   }
 }
@@ -186,29 +195,39 @@ __device__ __forceinline__ void load_bf16x32(const __nv_bfloat16* p, float* v) {
   for (int j = 0; j < 4; ++j) Vec16<__nv_bfloat16>::load(p + 8 * j, v + 8 * j);
 }
 
-template <int BN, int EPI>
-__device__ __forceinline__ void epilogue(const EpiArgs& e, uint32_t tlane, int row, int n0) {
+constexpr int kEpiWarps = 8;                  // two warps per TMEM lane quarter
+constexpr int NUM_THREADS = 64 + 32 * kEpiWarps;
+constexpr int kRedStride = 17;                // per-row exchange slots: sum + 16 logits
+
+// Epilogue of one 128 x BN tile for one warp: TMEM lanes `tlane` (32 rows of
+// the tile), columns [c0, c0 + BN/2) of the accumulator.  The two warps that
+// share a lane quarter exchange row sums (and head logits) through `red`.
+template <int BN, int EPI, int NAP>
+__device__ __forceinline__ void epilogue(const EpiArgs& e, uint32_t tacc, int row, int n0, int c0, int q, int h,
+                                         float* red, const float* s_weff) {
+  constexpr int HALF = BN / 2;
   const bool valid = row < e.M;
+  const int lane = threadIdx.x & 31;
   float v[32];
   if constexpr (EPI == EPI_BIAS || EPI == EPI_BIAS_GELU || EPI == EPI_KV) {
     __nv_bfloat16* out = nullptr;
     if (valid) {
       long long orow = row;
-      long long ocol = n0;
+      long long ocol = n0 + c0;
       if constexpr (EPI == EPI_KV) {
         const int r = find_segment(e.seg_off, e.n_seg, row);
         orow = static_cast<long long>(__ldg(e.dst_row0 + r)) + (row - __ldg(e.seg_off + r));
         const int blk = n0 / e.col_blk;
-        ocol = static_cast<long long>(blk) * e.col_blk_stride + (n0 - blk * e.col_blk);
+        ocol = static_cast<long long>(blk) * e.col_blk_stride + (n0 - blk * e.col_blk) + c0;
       }
       out = static_cast<__nv_bfloat16*>(e.out) + orow * e.ldo + ocol;
     }
 #pragma unroll 1
-    for (int c = 0; c < BN; c += 32) {
-      tmem_ld32(tlane + c, v);
+    for (int c = 0; c < HALF; c += 32) {
+      tmem_ld32(tacc + c0 + c, v);
       if (valid) {
         float b[32];
-        load_bias32(e.bias, n0 + c, b);
+        load_f32x32(e.bias + n0 + c0 + c, b);
 #pragma unroll
         for (int i = 0; i < 32; ++i) {
           float x = v[i] + b[i];
@@ -219,16 +238,19 @@ __device__ __forceinline__ void epilogue(const EpiArgs& e, uint32_t tlane, int r
       }
     }
   } else {
-    // Row-wise LayerNorm over the full row (BN == N): two passes over TMEM,
-    // the pre-norm values written back in place by the first pass.
+    // Row LayerNorm over the full row (BN == N): two passes over TMEM, the
+    // pre-norm values written back in place; halves combined through `red`.
+    const int trow = q * 32 + lane;              // row within the tile
+    float* my = red + (h * 128 + trow) * kRedStride;
+    const float* other = red + ((1 - h) * 128 + trow) * kRedStride;
     const __nv_bfloat16* res = valid ? static_cast<const __nv_bfloat16*>(e.res) + row * e.ldr : nullptr;
     float sum = 0.f;
 #pragma unroll 1
-    for (int c = 0; c < BN; c += 32) {
-      tmem_ld32(tlane + c, v);
+    for (int c = 0; c < HALF; c += 32) {
+      tmem_ld32(tacc + c0 + c, v);
       float b[32], r[32];
-      load_bias32(e.bias, c, b);
-      if (valid) load_bf16x32(res + c, r);
+      load_f32x32(e.bias + c0 + c, b);
+      if (valid) load_bf16x32(res + c0 + c, r);
       else {
 #pragma unroll
         for (int i = 0; i < 32; ++i) r[i] = 0.f;
@@ -238,110 +260,139 @@ __device__ __forceinline__ void epilogue(const EpiArgs& e, uint32_t tlane, int r
         v[i] += b[i] + r[i];
         sum += v[i];
       }
-      tmem_st32(tlane + c, v);
+      tmem_st32(tacc + c0 + c, v);
     }
-    const float mean = sum / static_cast<float>(BN);
+    my[0] = sum;
+    named_bar(1 + q, 64);
+    const float mean = (sum + other[0]) / static_cast<float>(BN);
+    named_bar(1 + q, 64);                        // both read before the slot is reused
     float sq = 0.f;
 #pragma unroll 1
-    for (int c = 0; c < BN; c += 32) {
-      tmem_ld32(tlane + c, v);
+    for (int c = 0; c < HALF; c += 32) {
+      tmem_ld32(tacc + c0 + c, v);
 #pragma unroll
       for (int i = 0; i < 32; ++i) {
         const float t = v[i] - mean;
         sq += t * t;
       }
     }
-    const float rstd = rsqrtf(sq / static_cast<float>(BN) + e.ln_eps);
-    float lg[16];
+    my[0] = sq;
+    named_bar(1 + q, 64);
+    const float rstd = rsqrtf((sq + other[0]) / static_cast<float>(BN) + e.ln_eps);
+    float lg[NAP];
 #pragma unroll
-    for (int a = 0; a < 16; ++a) lg[a] = 0.f;
+    for (int a = 0; a < NAP; ++a) lg[a] = 0.f;
     __nv_bfloat16* out = nullptr;
     if constexpr (EPI == EPI_LN) {
-      if (valid) out = static_cast<__nv_bfloat16*>(e.out) + row * e.ldo;
+      if (valid) out = static_cast<__nv_bfloat16*>(e.out) + row * e.ldo + c0;
     }
 #pragma unroll 1
-    for (int c = 0; c < BN; c += 32) {
-      tmem_ld32(tlane + c, v);
+    for (int c = 0; c < HALF; c += 32) {
+      tmem_ld32(tacc + c0 + c, v);
       float g[32], bt[32];
-      load_bias32(e.gamma, c, g);
-      load_bias32(e.beta, c, bt);
+      load_f32x32(e.gamma + c0 + c, g);
+      load_f32x32(e.beta + c0 + c, bt);
 #pragma unroll
       for (int i = 0; i < 32; ++i) v[i] = (v[i] - mean) * rstd * g[i] + bt[i];
       if constexpr (EPI == EPI_LN) {
         if (valid) store_bf16x32(out + c, v);
       } else {
-        const int na = e.n_act;
-#pragma unroll 4
-        for (int i = 0; i < 32; ++i) {
-          const float* w = e.weff_z + static_cast<long long>(c + i) * na;
+        // head: z . W_eff_z, weights zero-padded to NAP actions in shared memory
+        const float4* w4 = reinterpret_cast<const float4*>(s_weff + (c0 + c) * NAP);
 #pragma unroll
-          for (int a = 0; a < 16; ++a)
-            if (a < na) lg[a] = fmaf(v[i], __ldg(w + a), lg[a]);
+        for (int i = 0; i < 32; ++i) {
+#pragma unroll
+          for (int a4 = 0; a4 < NAP / 4; ++a4) {
+            const float4 w = w4[i * (NAP / 4) + a4];
+            lg[4 * a4] = fmaf(v[i], w.x, lg[4 * a4]);
+            lg[4 * a4 + 1] = fmaf(v[i], w.y, lg[4 * a4 + 1]);
+            lg[4 * a4 + 2] = fmaf(v[i], w.z, lg[4 * a4 + 2]);
+            lg[4 * a4 + 3] = fmaf(v[i], w.w, lg[4 * a4 + 3]);
+          }
         }
       }
     }
     if constexpr (EPI == EPI_LN_HEAD) {
-      if (valid && row < e.n_cand_rows) {
-        const int na = e.n_act;
+      const int na = e.n_act;
+      named_bar(1 + q, 64);                      // partner has read `sq`
+#pragma unroll
+      for (int a = 0; a < NAP; ++a) my[1 + a] = lg[a];
+      named_bar(1 + q, 64);
+      if (h == 0 && valid && row < e.n_cand_rows) {
         float mx = -INFINITY;
 #pragma unroll
-        for (int a = 0; a < 16; ++a)
+        for (int a = 0; a < NAP; ++a)
           if (a < na) {
-            lg[a] += __ldg(e.xlog + static_cast<long long>(row) * na + a);
+            lg[a] += other[1 + a] + __ldg(e.xlog + static_cast<long long>(row) * na + a);
             mx = fmaxf(mx, lg[a]);
           }
-        float s = 0.f, p[16];
+        float s = 0.f, p[NAP];
 #pragma unroll
-        for (int a = 0; a < 16; ++a)
-          if (a < na) {
-            p[a] = expf(lg[a] - mx);
-            s += p[a];
-          }
+        for (int a = 0; a < NAP; ++a) {
+          p[a] = a < na ? expf(lg[a] - mx) : 0.f;
+          s += p[a];
+        }
         const float inv = 1.f / s;
 #pragma unroll
-        for (int a = 0; a < 16; ++a)
+        for (int a = 0; a < NAP; ++a)
           if (a < na) {
             e.logits[static_cast<long long>(row) * na + a] = lg[a];
             if (e.probs) e.probs[static_cast<long long>(row) * na + a] = p[a] * inv;
           }
       }
     }
+    named_bar(1 + q, 64);                        // `red` free for the next tile
   }
 }
 
 // ------------------------------------------------------------------ kernel
 
-template <int BN>
+template <int BN, int EPI, int NAP = 4>
 struct Shape {
   static constexpr int BN_MMA = BN < 256 ? BN : 256;     // N of one tcgen05.mma
   static constexpr int B_BOX = BN_MMA;                    // rows of one TMA box of B
   static constexpr int B_STAGE_BYTES = BN * BK * 2;
   static constexpr int STAGE_BYTES = A_STAGE_BYTES + B_STAGE_BYTES;
-  static constexpr int STAGES = (BN >= 512) ? 2 : (196608 / STAGE_BYTES);
-  static constexpr int TMEM_COLS = BN < 32 ? 32 : BN;
-  static constexpr int SMEM_BYTES = STAGES * STAGE_BYTES + 1024 + 256;
+  static constexpr bool LN = EPI == EPI_LN || EPI == EPI_LN_HEAD;
+  static constexpr int RED_BYTES = LN ? 2 * 128 * kRedStride * 4 : 0;
+  static constexpr int WEFF_BYTES = EPI == EPI_LN_HEAD ? BN * NAP * 4 : 0;
+  static constexpr int EXTRA = RED_BYTES + WEFF_BYTES + 1024 + 256;
+  static constexpr int STAGES_FIT = (227 * 1024 - EXTRA) / STAGE_BYTES;
+  static constexpr int STAGES = STAGES_FIT > 8 ? 8 : STAGES_FIT;
+  static constexpr int ACC_BUFS = BN <= 256 ? 2 : 1;      // TMEM double buffer
+  static constexpr int TMEM_COLS = BN * ACC_BUFS < 32 ? 32 : BN * ACC_BUFS;
+  static constexpr int SMEM_BYTES = STAGES * STAGE_BYTES + EXTRA;
+  static_assert(STAGES >= 2, "pipeline depth");
   static_assert(SMEM_BYTES <= 232448, "shared memory");
   static_assert((TMEM_COLS & (TMEM_COLS - 1)) == 0 && TMEM_COLS <= 512, "TMEM columns");
 };
 
-template <int BN, int EPI>
+// Persistent: CTA b processes tiles b, b + gridDim.x, ... (tile t -> n tile
+// t % n_tiles, m tile t / n_tiles).  Warp 0: TMA producer over all tiles and
+// K blocks; warp 1: MMA issuer, accumulating tile i into TMEM buffer i % 2;
+// warps 2..9: epilogue, releasing the buffer as soon as its last TMEM read is
+// done so the next tile's MMAs overlap this tile's stores.
+template <int BN, int EPI, int NAP>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                    const EpiArgs e) {
-  using S = Shape<BN>;
+  using S = Shape<BN, EPI, NAP>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* sA = smem;
   uint8_t* sB = smem + S::STAGES * A_STAGE_BYTES;
-  uint64_t* full = reinterpret_cast<uint64_t*>(sB + S::STAGES * S::B_STAGE_BYTES);
+  float* red = reinterpret_cast<float*>(sB + S::STAGES * S::B_STAGE_BYTES);
+  float* s_weff = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(red) + S::RED_BYTES);
+  uint64_t* full = reinterpret_cast<uint64_t*>(reinterpret_cast<uint8_t*>(s_weff) + S::WEFF_BYTES);
   uint64_t* empty = full + S::STAGES;
-  uint64_t* accum = empty + S::STAGES;
-  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(accum + 1);
+  uint64_t* acc_full = empty + S::STAGES;
+  uint64_t* acc_empty = acc_full + 2;
+  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(acc_empty + 2);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_holder + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int m0 = blockIdx.x * BM;
-  const int n0 = blockIdx.y * BN;
+  const int n_tiles = e.N / BN;
+  const int num_tiles = ((e.M + BM - 1) / BM) * n_tiles;
   const int num_kb = e.K / BK;
 
   if (threadIdx.x == 0) {
@@ -349,9 +400,18 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       mbar_init(full + s, 1);
       mbar_init(empty + s, 1);
     }
-    mbar_init(accum, 1);
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(acc_full + b, 1);
+      mbar_init(acc_empty + b, kEpiWarps);
+    }
     *abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if constexpr (EPI == EPI_LN_HEAD) {
+    for (int i = threadIdx.x; i < e.N * NAP; i += NUM_THREADS) {
+      const int c = i / NAP, a = i - c * NAP;
+      s_weff[i] = a < e.n_act ? e.weff_z[c * e.n_act + a] : 0.f;
+    }
   }
   if (warp == 1) tmem_alloc(tmem_holder, S::TMEM_COLS);
   tc_fence_before();
@@ -363,57 +423,90 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     if (lane == 0) {
       asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmA)) : "memory");
       asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmB)) : "memory");
-      int issued = 0;
-      for (int kb = 0; kb < num_kb; ++kb) {
-        const int s = kb % S::STAGES;
-        const uint32_t ph = (kb / S::STAGES) & 1;
-        if (!mbar_wait(empty + s, ph ^ 1, abort_flag)) break;
-        mbar_expect_tx(full + s, S::STAGE_BYTES);
-        tma_load_2d(sA + s * A_STAGE_BYTES, &tmA, full + s, kb * BK, m0);
+      int it = 0;  // global k-block counter (ring position)
+      bool ok = true;
+      for (int t = blockIdx.x; t < num_tiles && ok; t += gridDim.x) {
+        const int m0 = (t / n_tiles) * BM, n0 = (t % n_tiles) * BN;
+        for (int kb = 0; kb < num_kb; ++kb, ++it) {
+          const int s = it % S::STAGES;
+          const uint32_t ph = (it / S::STAGES) & 1;
+          if (!mbar_wait(empty + s, ph ^ 1, abort_flag)) {
+            ok = false;
+            break;
+          }
+          mbar_expect_tx(full + s, S::STAGE_BYTES);
+          tma_load_2d(sA + s * A_STAGE_BYTES, &tmA, full + s, kb * BK, m0);
 #pragma unroll
-        for (int j = 0; j < BN; j += S::B_BOX)
-          tma_load_2d(sB + s * S::B_STAGE_BYTES + j * (BK * 2), &tmB, full + s, kb * BK, n0 + j);
-        issued = kb + 1;
+          for (int j = 0; j < BN; j += S::B_BOX)
+            tma_load_2d(sB + s * S::B_STAGE_BYTES + j * (BK * 2), &tmB, full + s, kb * BK, n0 + j);
+        }
       }
       if (*abort_flag) {
         // let the copies already in flight land before shared memory is released
-        for (int kb = issued > S::STAGES ? issued - S::STAGES : 0; kb < issued; ++kb)
-          mbar_wait_plain(full + kb % S::STAGES, (kb / S::STAGES) & 1);
+        for (int k = it > S::STAGES ? it - S::STAGES : 0; k < it; ++k)
+          mbar_wait_plain(full + k % S::STAGES, (k / S::STAGES) & 1);
       }
     }
   } else if (warp == 1) {
     if (lane == 0) {
       constexpr uint32_t idesc = idesc_bf16(BM, S::BN_MMA);
-      for (int kb = 0; kb < num_kb; ++kb) {
-        const int s = kb % S::STAGES;
-        const uint32_t ph = (kb / S::STAGES) & 1;
-        if (!mbar_wait(full + s, ph, abort_flag)) break;
+      int it = 0, i = 0;
+      bool ok = true;
+      for (int t = blockIdx.x; t < num_tiles && ok; t += gridDim.x, ++i) {
+        const int buf = i % S::ACC_BUFS;
+        const uint32_t use = i / S::ACC_BUFS;
+        if (!mbar_wait(acc_empty + buf, (use & 1) ^ 1, abort_flag)) break;
         tc_fence_after();
-        const uint64_t adesc = sdesc_sw128(smem_u32(sA + s * A_STAGE_BYTES));
-        const uint64_t bdesc = sdesc_sw128(smem_u32(sB + s * S::B_STAGE_BYTES));
-#pragma unroll
-        for (int k = 0; k < BK / 16; ++k) {
-#pragma unroll
-          for (int j = 0; j < BN / S::BN_MMA; ++j) {
-            // advance 32 bytes along K inside the swizzle row; N halves are
-            // S::BN_MMA rows (x 128 bytes) apart
-            const uint64_t boff = static_cast<uint64_t>((j * S::BN_MMA * BK * 2) >> 4);
-            mma_bf16(tmem + j * S::BN_MMA, adesc + 2 * k, bdesc + boff + 2 * k, idesc,
-                     (kb > 0 || k > 0) ? 1u : 0u);
+        const uint32_t dacc = tmem + buf * BN;
+        for (int kb = 0; kb < num_kb; ++kb, ++it) {
+          const int s = it % S::STAGES;
+          const uint32_t ph = (it / S::STAGES) & 1;
+          if (!mbar_wait(full + s, ph, abort_flag)) {
+            ok = false;
+            break;
           }
+          tc_fence_after();
+          const uint64_t adesc = sdesc_sw128(smem_u32(sA + s * A_STAGE_BYTES));
+          const uint64_t bdesc = sdesc_sw128(smem_u32(sB + s * S::B_STAGE_BYTES));
+#pragma unroll
+          for (int k = 0; k < BK / 16; ++k) {
+#pragma unroll
+            for (int j = 0; j < BN / S::BN_MMA; ++j) {
+              // 32 bytes along K per step inside the swizzle row; N halves are
+              // S::BN_MMA rows (x 128 bytes) apart
+              const uint64_t boff = static_cast<uint64_t>((j * S::BN_MMA * BK * 2) >> 4);
+              mma_bf16(dacc + j * S::BN_MMA, adesc + 2 * k, bdesc + boff + 2 * k, idesc,
+                       (kb > 0 || k > 0) ? 1u : 0u);
+            }
+          }
+          mma_commit(empty + s);
         }
-        mma_commit(empty + s);
+        mma_commit(acc_full + buf);   // also on abort: the epilogue waits on every issued MMA
       }
-      mma_commit(accum);
     }
   } else {
-    const int q = warp & 3;
-    const int row = m0 + q * 32 + lane;
-    bool go = mbar_wait(accum, 0, abort_flag);
-    go = go && !*abort_flag;
-    go = __shfl_sync(0xffffffffu, go ? 1 : 0, 0) != 0;  // warp-uniform: tcgen05.ld is .sync.aligned
-    tc_fence_after();
-    if (go) epilogue<BN, EPI>(e, tmem + (static_cast<uint32_t>(q * 32) << 16), row, n0);
+    const int ew = warp - 2;
+    const int q = warp & 3;           // TMEM lane quarter this warp may access
+    const int h = ew / 4;             // column half
+    int i = 0;
+    for (int t = blockIdx.x; t < num_tiles; t += gridDim.x, ++i) {
+      const int buf = i % S::ACC_BUFS;
+      const uint32_t use = i / S::ACC_BUFS;
+      // Go on exactly when the accumulator is complete: both warps of a lane
+      // quarter see the same barrier phase, so they agree (they meet at named
+      // barriers inside the LayerNorm epilogues).  Warp-uniform because
+      // tcgen05.ld is .sync.aligned.
+      bool go = mbar_wait(acc_full + buf, use & 1, abort_flag);
+      go = __shfl_sync(0xffffffffu, go ? 1 : 0, 0) != 0;
+      if (!go) break;
+      tc_fence_after();
+      const int m0 = (t / n_tiles) * BM, n0 = (t % n_tiles) * BN;
+      epilogue<BN, EPI, NAP>(e, tmem + buf * BN + (static_cast<uint32_t>(q * 32) << 16), m0 + q * 32 + lane, n0,
+                        h * (BN / 2), q, h, red, s_weff);
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(acc_empty + buf);
+    }
   }
   tc_fence_before();
   __syncthreads();
@@ -459,13 +552,23 @@ static bool make_tmap(CUtensorMap* tm, const void* base, long long rows, long lo
   return r == CUDA_SUCCESS;
 }
 
-template <int BN, int EPI>
+static int num_sms() {
+  static int n = 0;
+  if (!n) {
+    int dev = 0;
+    cudaGetDevice(&dev);
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0) n = 148;
+  }
+  return n;
+}
+
+template <int BN, int EPI, int NAP = 4>
 static cudaError_t launch_bn(const __nv_bfloat16* A, long long lda, const __nv_bfloat16* B, const EpiArgs& e,
                              cudaStream_t s, int cls) {
-  using Sh = Shape<BN>;
+  using Sh = Shape<BN, EPI, NAP>;
   static bool attr_set = false;
   if (!attr_set) {
-    cudaError_t err = cudaFuncSetAttribute(gemm_tc_kernel<BN, EPI>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    cudaError_t err = cudaFuncSetAttribute(gemm_tc_kernel<BN, EPI, NAP>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                            Sh::SMEM_BYTES);
     if (err != cudaSuccess) return err;
     attr_set = true;
@@ -473,9 +576,10 @@ static cudaError_t launch_bn(const __nv_bfloat16* A, long long lda, const __nv_b
   CUtensorMap ta, tb;
   if (!make_tmap(&ta, A, e.M, e.K, lda, BM)) return cudaErrorInvalidValue;
   if (!make_tmap(&tb, B, e.N, e.K, e.K, Sh::B_BOX)) return cudaErrorInvalidValue;
-  dim3 grid((e.M + BM - 1) / BM, e.N / BN);
+  const long long tiles = static_cast<long long>((e.M + BM - 1) / BM) * (e.N / BN);
+  const int grid = static_cast<int>(tiles < num_sms() ? tiles : num_sms());
   prof_begin(cls, s);
-  gemm_tc_kernel<BN, EPI><<<grid, NUM_THREADS, Sh::SMEM_BYTES, s>>>(ta, tb, e);
+  gemm_tc_kernel<BN, EPI, NAP><<<grid, NUM_THREADS, Sh::SMEM_BYTES, s>>>(ta, tb, e);
   cudaError_t err = cudaGetLastError();
   prof_end(cls, s);
   return err;
@@ -490,15 +594,15 @@ bool tc_gemm_supported(int N, int K, int epi) {
 template <int EPI>
 static cudaError_t launch_plain(const __nv_bfloat16* A, long long lda, const __nv_bfloat16* B, const EpiArgs& e,
                                 cudaStream_t s, int cls) {
-  // widest tile that divides N (and the cache's column blocks) while the grid
-  // still fills the machine; narrower tiles otherwise
+  // the widest tile that divides N (and the cache's column blocks) while there
+  // are still at least as many tiles as SMs; narrower tiles otherwise
   const long long m_tiles = (e.M + BM - 1) / BM;
   auto fits = [&](int bn) {
     if (e.N % bn) return false;
     if (EPI == EPI_KV && e.col_blk % bn) return false;
     return true;
   };
-  if (fits(256) && m_tiles * (e.N / 256) >= 148) return launch_bn<256, EPI>(A, lda, B, e, s, cls);
+  if (fits(256) && m_tiles * (e.N / 256) >= num_sms()) return launch_bn<256, EPI>(A, lda, B, e, s, cls);
   if (fits(128)) return launch_bn<128, EPI>(A, lda, B, e, s, cls);
   if (fits(64)) return launch_bn<64, EPI>(A, lda, B, e, s, cls);
   return cudaErrorInvalidValue;
@@ -510,17 +614,30 @@ cudaError_t launch_gemm_tc(const __nv_bfloat16* A, long long lda, const __nv_bfl
   if (!tc_gemm_supported(e.N, e.K, e.epi)) return cudaErrorInvalidValue;
   if ((reinterpret_cast<uintptr_t>(A) & 15) || (reinterpret_cast<uintptr_t>(B) & 15) || (lda % 8))
     return cudaErrorInvalidValue;
+  if (e.epi == EPI_LN_HEAD && (e.n_act < 1 || e.n_act > 16)) return cudaErrorInvalidValue;
   switch (e.epi) {
     case EPI_LN:
-    case EPI_LN_HEAD: {
-      const bool head = e.epi == EPI_LN_HEAD;
       switch (e.N) {
-        case 64: return head ? launch_bn<64, EPI_LN_HEAD>(A, lda, B, e, s, cls) : launch_bn<64, EPI_LN>(A, lda, B, e, s, cls);
-        case 128: return head ? launch_bn<128, EPI_LN_HEAD>(A, lda, B, e, s, cls) : launch_bn<128, EPI_LN>(A, lda, B, e, s, cls);
-        case 256: return head ? launch_bn<256, EPI_LN_HEAD>(A, lda, B, e, s, cls) : launch_bn<256, EPI_LN>(A, lda, B, e, s, cls);
-        default: return head ? launch_bn<512, EPI_LN_HEAD>(A, lda, B, e, s, cls) : launch_bn<512, EPI_LN>(A, lda, B, e, s, cls);
+        case 64: return launch_bn<64, EPI_LN>(A, lda, B, e, s, cls);
+        case 128: return launch_bn<128, EPI_LN>(A, lda, B, e, s, cls);
+        case 256: return launch_bn<256, EPI_LN>(A, lda, B, e, s, cls);
+        default: return launch_bn<512, EPI_LN>(A, lda, B, e, s, cls);
       }
-    }
+    case EPI_LN_HEAD:
+      if (e.n_act <= 4) {
+        switch (e.N) {
+          case 64: return launch_bn<64, EPI_LN_HEAD, 4>(A, lda, B, e, s, cls);
+          case 128: return launch_bn<128, EPI_LN_HEAD, 4>(A, lda, B, e, s, cls);
+          case 256: return launch_bn<256, EPI_LN_HEAD, 4>(A, lda, B, e, s, cls);
+          default: return launch_bn<512, EPI_LN_HEAD, 4>(A, lda, B, e, s, cls);
+        }
+      }
+      switch (e.N) {
+        case 64: return launch_bn<64, EPI_LN_HEAD, 16>(A, lda, B, e, s, cls);
+        case 128: return launch_bn<128, EPI_LN_HEAD, 16>(A, lda, B, e, s, cls);
+        case 256: return launch_bn<256, EPI_LN_HEAD, 16>(A, lda, B, e, s, cls);
+        default: return launch_bn<512, EPI_LN_HEAD, 16>(A, lda, B, e, s, cls);
+      }
     case EPI_BIAS: return launch_plain<EPI_BIAS>(A, lda, B, e, s, cls);
     case EPI_BIAS_GELU: return launch_plain<EPI_BIAS_GELU>(A, lda, B, e, s, cls);
     case EPI_KV: return launch_plain<EPI_KV>(A, lda, B, e, s, cls);

@@ -37,51 +37,76 @@ __device__ __forceinline__ int find_segment_param(const int* off, int n, int row
   return lo;
 }
 
+constexpr int kPackRowsPerWarp = 2;
+
+// 8 warps per CTA, kPackRowsPerWarp rows per warp.  W_eff_x is staged once per
+// CTA in shared memory as [action][column] so that a lane's 16-byte slice of a
+// row meets contiguous weights.
 template <typename T>
 __global__ void __launch_bounds__(256) pack_kernel(const __grid_constant__ PackArgs a, const T* __restrict__ cand,
                                                    const T* __restrict__ ctx, T* __restrict__ X,
-                                                   int* __restrict__ row_req, const float* __restrict__ weff_x,
+                                                   int* __restrict__ row_req, int* __restrict__ cand_off_dev,
+                                                   const float* __restrict__ weff_x,
                                                    const float* __restrict__ cdec, float* __restrict__ xlog) {
   constexpr int VEC = Vec16<T>::N;
+  extern __shared__ float sw[];                 // [na][d]
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const long long p = static_cast<long long>(blockIdx.x) * 8 + warp;
+  const int d = a.d, na = a.na;
+  if (blockIdx.x == 0)
+    for (int i = threadIdx.x; i <= a.n_req; i += 256) cand_off_dev[i] = a.cand_off[i];
+  for (int i = threadIdx.x; i < d * na; i += 256) {
+    const int c = i / na, k = i - c * na;       // weff_x is [d][na]
+    sw[k * d + c] = weff_x[i];
+  }
+  __syncthreads();
   const long long n_rows = a.n_cand + static_cast<long long>(a.n_req) * a.S;
-  if (p >= n_rows) return;
-  const int d = a.d;
-  int r;
-  const T* src;
-  if (p < a.n_cand) {
-    r = find_segment_param(a.cand_off, a.n_req, static_cast<int>(p));
-    src = cand + p * d;
-  } else {
-    const long long q = p - a.n_cand;
-    r = static_cast<int>(q / a.S);
-    src = ctx + q * d;
-  }
-  T* dst = X + p * d;
-  float lg[16];
-#pragma unroll
-  for (int i = 0; i < 16; ++i) lg[i] = 0.f;
-  for (int c = lane * VEC; c < d; c += 32 * VEC) {
-    float v[VEC];
-    Vec16<T>::load(src + c, v);
-    Vec16<T>::store(dst + c, v);
-    if (p < a.n_cand) {
-#pragma unroll
-      for (int i = 0; i < VEC; ++i)
-#pragma unroll
-        for (int k = 0; k < 16; ++k)
-          if (k < a.na) lg[k] = fmaf(v[i], __ldg(weff_x + static_cast<long long>(c + i) * a.na + k), lg[k]);
+  const long long p0 = (static_cast<long long>(blockIdx.x) * 8 + warp) * kPackRowsPerWarp;
+  for (int t = 0; t < kPackRowsPerWarp; ++t) {
+    const long long p = p0 + t;
+    if (p >= n_rows) return;
+    int r;
+    const T* src;
+    const bool is_cand = p < a.n_cand;
+    if (is_cand) {
+      r = find_segment_param(a.cand_off, a.n_req, static_cast<int>(p));
+      src = cand + p * d;
+    } else {
+      const long long q = p - a.n_cand;
+      r = static_cast<int>(q / a.S);
+      src = ctx + q * d;
     }
-  }
-  if (lane == 0) row_req[p] = r;
-  if (p < a.n_cand) {
+    T* dst = X + p * d;
+    float lg[16];
 #pragma unroll
-    for (int k = 0; k < 16; ++k) {
-      float x = lg[k];
+    for (int k = 0; k < 16; ++k) lg[k] = 0.f;
+    for (int c = lane * VEC; c < d; c += 32 * VEC) {
+      float v[VEC];
+      Vec16<T>::load(src + c, v);
+      Vec16<T>::store(dst + c, v);
+      if (is_cand) {
 #pragma unroll
-      for (int o = 16; o > 0; o >>= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
-      if (lane == 0 && k < a.na) xlog[p * a.na + k] = x + __ldg(cdec + k);
+        for (int k = 0; k < 16; ++k) {
+          if (k < na) {
+            const float* w = sw + k * d + c;
+            float acc = 0.f;
+#pragma unroll
+            for (int i = 0; i < VEC; ++i) acc = fmaf(v[i], w[i], acc);
+            lg[k] += acc;
+          }
+        }
+      }
+    }
+    if (lane == 0) row_req[p] = r;
+    if (is_cand) {
+#pragma unroll
+      for (int k = 0; k < 16; ++k) {
+        if (k < na) {
+          float x = lg[k];
+#pragma unroll
+          for (int o = 16; o > 0; o >>= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
+          if (lane == 0) xlog[p * na + k] = x + __ldg(cdec + k);
+        }
+      }
     }
   }
 }
@@ -122,7 +147,8 @@ __global__ void __launch_bounds__(1024) rank_kernel(const __grid_constant__ Rank
 
 template <typename T>
 cudaError_t launch_pack(int n_req, const int* cand_off_host, int S, int d, int na, const T* cand, const T* ctx, T* X,
-                        int* row_req, const float* weff_x, const float* cdec, float* xlog, cudaStream_t s) {
+                        int* row_req, int* cand_off_dev, const float* weff_x, const float* cdec, float* xlog,
+                        cudaStream_t s) {
   if (n_req > kMaxReqParam || na > 16) return cudaErrorInvalidValue;
   PackArgs a;
   a.n_req = n_req;
@@ -133,8 +159,17 @@ cudaError_t launch_pack(int n_req, const int* cand_off_host, int S, int d, int n
   for (int i = 0; i <= n_req; ++i) a.cand_off[i] = cand_off_host[i];
   const long long n_rows = a.n_cand + static_cast<long long>(n_req) * S;
   if (n_rows == 0) return cudaSuccess;
+  const size_t smem = sizeof(float) * d * na;
+  static bool attr = false;
+  if (!attr) {
+    cudaError_t e = cudaFuncSetAttribute(pack_kernel<T>, cudaFuncAttributeMaxDynamicSharedMemorySize, 512 * 16 * 4);
+    if (e != cudaSuccess) return e;
+    attr = true;
+  }
+  const long long rows_per_cta = 8LL * kPackRowsPerWarp;
   prof_begin(KC_PACK, s);
-  pack_kernel<T><<<static_cast<int>((n_rows + 7) / 8), 256, 0, s>>>(a, cand, ctx, X, row_req, weff_x, cdec, xlog);
+  pack_kernel<T><<<static_cast<int>((n_rows + rows_per_cta - 1) / rows_per_cta), 256, smem, s>>>(
+      a, cand, ctx, X, row_req, cand_off_dev, weff_x, cdec, xlog);
   cudaError_t err = cudaGetLastError();
   prof_end(KC_PACK, s);
   return err;
@@ -169,9 +204,9 @@ cudaError_t launch_rank(int n_req, const int* cand_off_host, const float* probs,
 }
 
 template cudaError_t launch_pack<float>(int, const int*, int, int, int, const float*, const float*, float*, int*,
-                                        const float*, const float*, float*, cudaStream_t);
+                                        int*, const float*, const float*, float*, cudaStream_t);
 template cudaError_t launch_pack<__nv_bfloat16>(int, const int*, int, int, int, const __nv_bfloat16*,
-                                                const __nv_bfloat16*, __nv_bfloat16*, int*, const float*,
+                                                const __nv_bfloat16*, __nv_bfloat16*, int*, int*, const float*,
                                                 const float*, float*, cudaStream_t);
 
 }  // namespace txs

@@ -15,9 +15,9 @@ namespace {
 
 constexpr int TM = 64, TN = 64, TK = 16;
 
-template <int EPI>
+template <int EPI, typename TB>
 __global__ void __launch_bounds__(256) gemm_simt_kernel(const float* __restrict__ A, long long lda,
-                                                        const float* __restrict__ B, const EpiArgs e,
+                                                        const TB* __restrict__ B, const EpiArgs e,
                                                         float* __restrict__ tmp) {
   __shared__ float As[TK][TM + 4];
   __shared__ float Bs[TK][TN + 4];
@@ -35,7 +35,7 @@ __global__ void __launch_bounds__(256) gemm_simt_kernel(const float* __restrict_
       const int gm = m0 + mm, gk = k0 + kk;
       As[kk][mm] = (gm < e.M && gk < e.K) ? A[static_cast<long long>(gm) * lda + gk] : 0.f;
       const int gn = n0 + mm;
-      Bs[kk][mm] = (gn < e.N && gk < e.K) ? B[static_cast<long long>(gn) * e.K + gk] : 0.f;
+      Bs[kk][mm] = (gn < e.N && gk < e.K) ? Elem<TB>::load(B + static_cast<long long>(gn) * e.K + gk) : 0.f;
     }
     __syncthreads();
 #pragma unroll
@@ -59,8 +59,10 @@ __global__ void __launch_bounds__(256) gemm_simt_kernel(const float* __restrict_
     if (m >= e.M) continue;
     long long orow = m;
     if constexpr (EPI == EPI_KV) {
-      const int r = find_segment(e.seg_off, e.n_seg, m);
-      orow = static_cast<long long>(e.dst_row0[r]) + (m - e.seg_off[r]);
+      if (e.seg_off) {   // rows remapped into cache slots; identity otherwise
+        const int r = find_segment(e.seg_off, e.n_seg, m);
+        orow = static_cast<long long>(e.dst_row0[r]) + (m - e.seg_off[r]);
+      }
     }
 #pragma unroll
     for (int j = 0; j < 4; ++j) {
@@ -157,19 +159,20 @@ __global__ void __launch_bounds__(256) row_ln_kernel(const float* __restrict__ t
 
 }  // namespace
 
-cudaError_t launch_gemm_simt(const float* A, long long lda, const float* B, const EpiArgs& e, float* tmp,
+template <typename TB>
+cudaError_t launch_gemm_simt(const float* A, long long lda, const TB* B, const EpiArgs& e, float* tmp,
                              cudaStream_t s, int cls) {
   if (e.M == 0) return cudaSuccess;
-  if (e.N > 1024) return cudaErrorInvalidValue;
+  if ((e.epi == EPI_LN || e.epi == EPI_LN_HEAD) && e.N > 1024) return cudaErrorInvalidValue;
   dim3 grid((e.M + TM - 1) / TM, (e.N + TN - 1) / TN);
   prof_begin(cls, s);
   switch (e.epi) {
-    case EPI_BIAS: gemm_simt_kernel<EPI_BIAS><<<grid, 256, 0, s>>>(A, lda, B, e, tmp); break;
-    case EPI_BIAS_GELU: gemm_simt_kernel<EPI_BIAS_GELU><<<grid, 256, 0, s>>>(A, lda, B, e, tmp); break;
-    case EPI_KV: gemm_simt_kernel<EPI_KV><<<grid, 256, 0, s>>>(A, lda, B, e, tmp); break;
+    case EPI_BIAS: gemm_simt_kernel<EPI_BIAS, TB><<<grid, 256, 0, s>>>(A, lda, B, e, tmp); break;
+    case EPI_BIAS_GELU: gemm_simt_kernel<EPI_BIAS_GELU, TB><<<grid, 256, 0, s>>>(A, lda, B, e, tmp); break;
+    case EPI_KV: gemm_simt_kernel<EPI_KV, TB><<<grid, 256, 0, s>>>(A, lda, B, e, tmp); break;
     case EPI_LN:
     case EPI_LN_HEAD:
-      gemm_simt_kernel<EPI_LN><<<grid, 256, 0, s>>>(A, lda, B, e, tmp);
+      gemm_simt_kernel<EPI_LN, TB><<<grid, 256, 0, s>>>(A, lda, B, e, tmp);
       break;
     default: return cudaErrorInvalidValue;
   }
@@ -186,5 +189,10 @@ cudaError_t launch_gemm_simt(const float* A, long long lda, const float* B, cons
   }
   return err;
 }
+
+template cudaError_t launch_gemm_simt<float>(const float*, long long, const float*, const EpiArgs&, float*,
+                                             cudaStream_t, int);
+template cudaError_t launch_gemm_simt<__nv_bfloat16>(const float*, long long, const __nv_bfloat16*, const EpiArgs&,
+                                                     float*, cudaStream_t, int);
 
 }  // namespace txs

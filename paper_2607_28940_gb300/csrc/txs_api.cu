@@ -98,6 +98,7 @@ struct txs_kv_cache {
   float *pool_m = nullptr, *pool_s = nullptr, *pool_acc = nullptr, *g = nullptr;
   float* gkv = nullptr;                  // [nL][2][R][d] fp32
   float* part = nullptr;                 // pooling chunk states
+  int* pool_cnt = nullptr;               // [R] chunk arrivals (zero between calls)
   int max_chunks = 0;
   std::vector<void*> allocs;
 };
@@ -152,7 +153,7 @@ T* dalloc(std::vector<void*>& list, size_t bytes, cudaError_t* err) {
 size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
 
 struct ScoreLayout {
-  size_t row_req, X, QKV, A, X1, X2, Hf, xlog, tmp, total;
+  size_t row_req, cand_off, X, QKV, A, X1, X2, Hf, xlog, tmp, total;
 };
 
 ScoreLayout score_layout(const txs_config& c, int es, int n_req, long long n_cand) {
@@ -166,6 +167,7 @@ ScoreLayout score_layout(const txs_config& c, int es, int n_req, long long n_can
     return at;
   };
   L.row_req = take(N * 4);
+  L.cand_off = take((n_req + 1) * 4);
   L.X = take(N * d * es);
   L.QKV = take(N * 3 * d * es);
   L.A = take(N * d * es);
@@ -185,7 +187,7 @@ cudaError_t gemm(const txs_model* m, const void* A, long long lda, const void* B
   e.status = m->status;
   if (m->cfg.dtype == TXS_BF16)
     return launch_gemm_tc(static_cast<const __nv_bfloat16*>(A), lda, static_cast<const __nv_bfloat16*>(Bt), e, s, cls);
-  return launch_gemm_simt(static_cast<const float*>(A), lda, static_cast<const float*>(Bt), e, tmp, s, cls);
+  return launch_gemm_simt<float>(static_cast<const float*>(A), lda, static_cast<const float*>(Bt), e, tmp, s, cls);
 }
 
 EpiArgs epi_base(int epi, long long M, int N, int K) {
@@ -347,8 +349,8 @@ txs_status project_rows(txs_model* m, txs_kv_cache* c, int n_req, const int32_t*
     TXS_CK(gemm(m, rows, d, m->Wt_kv, e, nullptr, s, KC_GEMM_KV));
   }
   TXS_CK(launch_pool<T>(static_cast<const T*>(rows), c->d_in_off, n_req, max_rows, m->w_pool, d, c->max_chunks,
-                        c->part, append ? 1 : 0, c->pool_m, c->pool_s, c->pool_acc, c->g, s));
-  TXS_CK(launch_global_kv<T>(c->g, static_cast<const T*>(m->Wt_kv), m->b_kv, c->gkv, n_req, d, nL, s));
+                        c->part, append ? 1 : 0, c->pool_m, c->pool_s, c->pool_acc, c->g, c->pool_cnt, s));
+  TXS_CK(launch_anchor_proj<T>(c->g, static_cast<const T*>(m->Wt_kv), m->b_kv, c->gkv, n_req, d, nL, s));
   return TXS_OK;
 }
 
@@ -362,6 +364,7 @@ txs_status score_impl(txs_model* m, const txs_kv_cache* c, int n_req, const int3
   const ScoreLayout L = score_layout(cf, sizeof(T), n_req, n_cand);
   uint8_t* base = static_cast<uint8_t*>(ws);
   int* row_req = reinterpret_cast<int*>(base + L.row_req);
+  int* cand_off_dev = reinterpret_cast<int*>(base + L.cand_off);
   T* X = reinterpret_cast<T*>(base + L.X);
   T* QKV = reinterpret_cast<T*>(base + L.QKV);
   T* A = reinterpret_cast<T*>(base + L.A);
@@ -372,7 +375,7 @@ txs_status score_impl(txs_model* m, const txs_kv_cache* c, int n_req, const int3
   float* tmp = reinterpret_cast<float*>(base + L.tmp);
 
   TXS_CK(launch_pack<T>(n_req, cand_off, S, d, k, static_cast<const T*>(cand_tok), static_cast<const T*>(ctx_tok), X,
-                        row_req, m->weff + size_t(d) * k, m->cdec, xlog, s));
+                        row_req, cand_off_dev, m->weff + size_t(d) * k, m->cdec, xlog, s));
   const T* kv = static_cast<const T*>(c->kv);
   for (int l = 0; l < cf.n_layers; ++l) {
     const LayerW& W = m->layers[l];
@@ -580,6 +583,9 @@ TXS_API txs_status txs_build_kv_cache(txs_model* m, int32_t n_req, const int32_t
   c->g = static_cast<float*>(A(size_t(4) * n_req * d));
   c->gkv = static_cast<float*>(A(size_t(4) * nL * 2 * n_req * d));
   c->part = static_cast<float*>(A(size_t(4) * n_req * c->max_chunks * (d + 2)));
+  c->pool_cnt = static_cast<int*>(A(size_t(4) * n_req));
+  if (st == TXS_OK && (err = cudaMemsetAsync(c->pool_cnt, 0, size_t(4) * n_req, s)) != cudaSuccess)
+    st = fail_cuda("cudaMemsetAsync", err);
   if (st == TXS_OK) {
     c->stage_ints = 2 * n_req + 1;
     if ((err = cudaMallocHost(&c->h_stage, sizeof(int) * 4 * c->stage_ints)) != cudaSuccess) {

@@ -133,7 +133,9 @@ struct EpiArgs {
 };
 
 // Launchers (return cudaError_t of the launch).
-cudaError_t launch_gemm_simt(const float* A, long long lda, const float* B, const EpiArgs& e,
+// fp32 A; B float or bf16; fp32 output (EPI_KV with seg_off == nullptr keeps rows)
+template <typename TB>
+cudaError_t launch_gemm_simt(const float* A, long long lda, const TB* B, const EpiArgs& e,
                              float* tmp, cudaStream_t s, int cls);
 cudaError_t launch_gemm_tc(const __nv_bfloat16* A, long long lda, const __nv_bfloat16* B,
                            const EpiArgs& e, cudaStream_t s, int cls);
@@ -151,10 +153,10 @@ extern const int kPoolChunk;
 template <typename T>
 cudaError_t launch_pool(const T* phi, const int* seg_off, int R, int max_rows, const float* w_pool, int d,
                         int max_chunks, float* part, int merge_existing, float* st_m, float* st_s, float* st_acc,
-                        float* g, cudaStream_t s);
+                        float* g, int* counter, cudaStream_t s);
 template <typename T>
-cudaError_t launch_global_kv(const float* g, const T* Wt_kv, const float* b_kv, float* gkv, int R, int d, int n_layers,
-                             cudaStream_t s);
+cudaError_t launch_anchor_proj(const float* g, const T* Wt_kv, const float* b_kv, float* gkv, int R, int d,
+                               int n_layers, cudaStream_t s);
 template <typename T>
 cudaError_t launch_transpose(const T* W, T* Wt, int rows, int cols, cudaStream_t s);
 template <typename T>
@@ -167,7 +169,8 @@ cudaError_t launch_hash(const void* p, long long bytes, uint64_t salt, unsigned 
 extern const int kMaxReqParam;
 template <typename T>
 cudaError_t launch_pack(int n_req, const int* cand_off_host, int S, int d, int na, const T* cand, const T* ctx, T* X,
-                        int* row_req, const float* weff_x, const float* cdec, float* xlog, cudaStream_t s);
+                        int* row_req, int* cand_off_dev, const float* weff_x, const float* cdec, float* xlog,
+                        cudaStream_t s);
 cudaError_t launch_rank(int n_req, const int* cand_off_host, const float* probs, int na, int action, int top_k,
                         int* out, cudaStream_t s);
 
