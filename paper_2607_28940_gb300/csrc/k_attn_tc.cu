@@ -1,0 +1,497 @@
+// Multi-query cross-attention over all cached rows of a request on the tensor
+// cores (FULL key set: the -sparseAttn variant of Sec. 5.2; sparse
+// cross-attention equation of Sec. 4.1.2 with I = every behavior row).
+//
+// One CTA per (query tile of 128 rows, request r, head h).  All M_r + S query
+// rows of request r share the request's K/V (Sec. 4.1.2 multi-query
+// formulation), so each 128-key K/V tile is staged once per CTA by TMA and
+// serves all 128 queries:
+//   warp 0     TMA producer: K_j, V_j tiles of the request (head h columns)
+//              into a STG-deep shared-memory ring;
+//   warp 1     MMA issuer: S_j = Q K_j^T into one of two TMEM buffers, then
+//              O_j = P_j V_j into a TMEM tile (V used MN-major: no transpose);
+//   warps 2-5  softmax: one query row per thread straight out of TMEM (row
+//              max, exp2, row sum need no shuffles), P_j written to shared
+//              memory in the 128-byte-swizzled layout the MMA reads, and the
+//              running output O = O * exp(m_old - m_new) + O_j kept in registers.
+// All waits are bounded; a timeout latches TXS_ERR_DEVICE_TIMEOUT.
+#include <algorithm>
+
+#include "txs_internal.cuh"
+
+namespace txs {
+namespace fa {
+
+constexpr int BQ = 128;            // queries per CTA (TMEM lanes)
+constexpr int BKV = 128;           // keys per K/V tile
+constexpr int STG = 3;             // K/V ring depth
+constexpr int NUM_THREADS = 192;   // producer, MMA, 4 softmax warps
+
+// ------------------------------------------------------------------ PTX wrappers
+
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count) : "memory");
+}
+__device__ __forceinline__ void mbar_expect_tx(uint64_t* bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)), "r"(bytes)
+               : "memory");
+}
+__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(smem_u32(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort) {
+  const long long t0 = clock64();
+  while (!mbar_try_wait(bar, parity)) {
+    if (*abort) return false;
+    if (clock64() - t0 > kSpinCycles) {
+      *abort = 1;
+      return false;
+    }
+  }
+  return true;
+}
+__device__ __forceinline__ bool mbar_wait_plain(uint64_t* bar, uint32_t parity) {
+  const long long t0 = clock64();
+  while (!mbar_try_wait(bar, parity))
+    if (clock64() - t0 > kSpinCycles) return false;
+  return true;
+}
+__device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* tm, uint64_t* bar, int x, int y) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%3, %4}], [%2];" ::"r"(
+          smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(tm)), "r"(smem_u32(bar)), "r"(x), "r"(y)
+      : "memory");
+}
+__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void fence_async_smem() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
+__device__ __forceinline__ void tmem_alloc(uint32_t* holder, uint32_t ncols) {
+  asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(holder)), "r"(ncols)
+               : "memory");
+  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
+  asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols) : "memory");
+}
+__device__ __forceinline__ void mma_bf16(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
+                                         uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+__device__ __forceinline__ void mma_commit(uint64_t* bar) {
+  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(smem_u32(bar))
+               : "memory");
+}
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, float* v) {
+  uint32_t r[32];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
+      "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
+      "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];\n\t"
+      "tcgen05.wait::ld.sync.aligned;"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+        "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]),
+        "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]),
+        "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+      : "r"(taddr)
+      : "memory");
+#pragma unroll
+  for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+// Shared-memory matrix descriptor (tcgen05): start address, leading/stride
+// byte offsets, descriptor version 1, layout code (2 = 128-byte swizzle,
+// 4 = 64-byte swizzle).
+__device__ __forceinline__ uint64_t sdesc(uint32_t saddr, uint32_t lbo, uint32_t sbo, uint32_t layout) {
+  uint64_t d = 0;
+  d |= static_cast<uint64_t>((saddr & 0x3FFFFu) >> 4);
+  d |= static_cast<uint64_t>((lbo >> 4) & 0x3FFFu) << 16;
+  d |= static_cast<uint64_t>((sbo >> 4) & 0x3FFFu) << 32;
+  d |= 1ull << 46;
+  d |= static_cast<uint64_t>(layout) << 61;
+  return d;
+}
+
+// kind::f16 instruction descriptor: D fp32, A/B bf16, A K-major; B K-major or
+// MN-major (bit 16).
+__host__ __device__ constexpr uint32_t idesc_bf16(int m, int n, bool b_mn_major) {
+  return (1u << 4) | (1u << 7) | (1u << 10) | (b_mn_major ? (1u << 16) : 0u) |
+         (static_cast<uint32_t>(n >> 3) << 17) | (static_cast<uint32_t>(m >> 4) << 24);
+}
+
+// ------------------------------------------------------------------ kernel
+
+struct FaArgs {
+  const __nv_bfloat16* q;     // [N_rows, d] packed query rows
+  __nv_bfloat16* out;         // [N_rows, d]
+  const int* cand_off;        // device [R + 1]
+  const int* kv_off;          // device [R + 1] cache row offsets
+  const int* kv_len;          // device [R]
+  int n_cand, S, d;
+  float scale_log2;           // log2(e) / sqrt(d_h)
+  int* status;
+};
+
+template <int DH>
+struct FaShape {
+  static constexpr int ROW_BYTES = DH * 2;                  // 64 or 128: one swizzle row
+  static constexpr uint32_t SW = DH == 64 ? 2u : 4u;        // 128-byte or 64-byte swizzle
+  static constexpr int ATOM = 8 * ROW_BYTES;                // 8 rows
+  static constexpr int Q_BYTES = BQ * ROW_BYTES;
+  static constexpr int KV_BYTES = BKV * ROW_BYTES;
+  static constexpr int P_BYTES = BQ * BKV * 2;              // two 64-key blocks, 128-byte swizzle
+  static constexpr int SMEM = Q_BYTES + P_BYTES + 2 * STG * KV_BYTES + 1024 + 256;
+  static constexpr int TMEM_COLS = 512;                     // S x2 (256) + O tile (DH)
+};
+
+// byte offset of 16-byte chunk c of row m in a swizzled K-major tile whose rows
+// are ROW_BYTES long (Swizzle: chunk index XOR row bits above the 128-byte line)
+template <int ROW_BYTES>
+__device__ __forceinline__ int swz(int m, int c) {
+  if constexpr (ROW_BYTES == 128) return m * 128 + ((c ^ (m & 7)) << 4);
+  else return m * 64 + ((c ^ ((m >> 1) & 3)) << 4);
+}
+
+template <int DH>
+__global__ void __launch_bounds__(NUM_THREADS, 1)
+    fa_full_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV, const FaArgs a) {
+  using Sh = FaShape<DH>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint8_t* sQ = smem;
+  uint8_t* sP = sQ + Sh::Q_BYTES;
+  uint8_t* sK = sP + Sh::P_BYTES;
+  uint8_t* sV = sK + STG * Sh::KV_BYTES;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(sV + STG * Sh::KV_BYTES);
+  uint64_t* kv_full = bars;
+  uint64_t* kv_empty = kv_full + STG;
+  uint64_t* s_full = kv_empty + STG;
+  uint64_t* s_free = s_full + 2;
+  uint64_t* q_ready = s_free + 2;
+  uint64_t* p_full = q_ready + 1;
+  uint64_t* o_full = p_full + 1;
+  uint64_t* o_free = o_full + 1;
+  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(o_free + 1);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_holder + 1);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int qt = blockIdx.x, r = blockIdx.y, h = blockIdx.z;
+  const int c0 = a.cand_off[r];
+  const int M = a.cand_off[r + 1] - c0;
+  const int n_q = M + a.S;
+  if (qt * BQ >= n_q) return;                       // uniform: no tile here
+  const int len = a.kv_len[r];
+  const int kv0 = a.kv_off[r];
+  const int nkv = (len + BKV - 1) / BKV;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < STG; ++s) {
+      mbar_init(kv_full + s, 1);
+      mbar_init(kv_empty + s, 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(s_full + b, 1);
+      mbar_init(s_free + b, 4);
+    }
+    mbar_init(q_ready, 4);
+    mbar_init(p_full, 4);
+    mbar_init(o_full, 1);
+    mbar_init(o_free, 4);
+    *abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == 1) tmem_alloc(tmem_holder, Sh::TMEM_COLS);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_holder;
+  const uint32_t t_s = tmem;            // S buffers at columns 0 and 128
+  const uint32_t t_o = tmem + 256;      // O tile
+
+  if (warp == 0) {
+    if (lane == 0) {
+      asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmK)) : "memory");
+      asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmV)) : "memory");
+      int issued = 0;
+      for (int j = 0; j < nkv; ++j) {
+        const int st = j % STG;
+        if (!mbar_wait(kv_empty + st, ((j / STG) & 1) ^ 1, abort_flag)) break;
+        mbar_expect_tx(kv_full + st, 2 * Sh::KV_BYTES);
+        tma_load_2d(sK + st * Sh::KV_BYTES, &tmK, kv_full + st, h * DH, kv0 + j * BKV);
+        tma_load_2d(sV + st * Sh::KV_BYTES, &tmV, kv_full + st, h * DH, kv0 + j * BKV);
+        issued = j + 1;
+      }
+      if (*abort_flag)
+        for (int k = issued > STG ? issued - STG : 0; k < issued; ++k)
+          mbar_wait_plain(kv_full + k % STG, (k / STG) & 1);
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      constexpr uint32_t id_s = idesc_bf16(BQ, BKV, false);
+      constexpr uint32_t id_pv = idesc_bf16(BQ, DH, true);
+      const uint32_t q_addr = smem_u32(sQ), p_addr = smem_u32(sP);
+      bool ok = mbar_wait(q_ready, 0, abort_flag);
+      tc_fence_after();
+      auto pv = [&](int t) -> bool {
+        if (!mbar_wait(p_full, t & 1, abort_flag)) return false;
+        if (!mbar_wait(o_free, (t & 1) ^ 1, abort_flag)) return false;
+        tc_fence_after();
+        const int st = t % STG;
+        const uint32_t v_addr = smem_u32(sV + st * Sh::KV_BYTES);
+#pragma unroll
+        for (int k = 0; k < BKV / 16; ++k) {
+          // P: 64-key blocks of 16 KB, 32 bytes per 16-key step inside a block
+          const uint64_t pd = sdesc(p_addr + (k / 4) * (BQ * 128) + (k % 4) * 32, 16, 1024, 2);
+          // V (MN-major): 16 keys = two 8-row atoms of the tile
+          const uint64_t vd = sdesc(v_addr + k * 16 * Sh::ROW_BYTES, Sh::ATOM, Sh::ATOM, Sh::SW);
+          mma_bf16(t_o, pd, vd, id_pv, k > 0 ? 1u : 0u);
+        }
+        mma_commit(o_full);
+        mma_commit(kv_empty + st);
+        return true;
+      };
+      for (int j = 0; j < nkv && ok; ++j) {
+        const int st = j % STG, b = j & 1;
+        if (!mbar_wait(kv_full + st, (j / STG) & 1, abort_flag)) break;
+        if (!mbar_wait(s_free + b, ((j >> 1) & 1) ^ 1, abort_flag)) break;
+        tc_fence_after();
+        const uint32_t k_addr = smem_u32(sK + st * Sh::KV_BYTES);
+#pragma unroll
+        for (int k = 0; k < DH / 16; ++k) {
+          const uint64_t qd = sdesc(q_addr + k * 32, 16, Sh::ATOM, Sh::SW);
+          const uint64_t kd = sdesc(k_addr + k * 32, 16, Sh::ATOM, Sh::SW);
+          mma_bf16(t_s + b * BKV, qd, kd, id_s, k > 0 ? 1u : 0u);
+        }
+        mma_commit(s_full + b);
+        if (j >= 1) ok = pv(j - 1);
+      }
+      if (ok && !*abort_flag) pv(nkv - 1);
+    }
+  } else {
+    // ---------------- softmax warps: one query row per thread
+    const int qw = warp & 3;                  // TMEM lane quarter
+    const int m = qw * 32 + lane;             // row of the tile
+    const int j_q = qt * BQ + m;              // query index within the request
+    const bool valid = j_q < n_q;
+    const long long grow = j_q < M ? static_cast<long long>(c0) + j_q
+                                   : a.n_cand + static_cast<long long>(r) * a.S + (j_q - M);
+    // gather this row's head slice of Q into the swizzled tile
+    {
+      constexpr int CH = Sh::ROW_BYTES / 16;
+      const uint4* src = reinterpret_cast<const uint4*>(a.q + grow * a.d + h * DH);
+#pragma unroll
+      for (int c = 0; c < CH; ++c) {
+        uint4 v = valid ? src[c] : make_uint4(0, 0, 0, 0);
+        *reinterpret_cast<uint4*>(sQ + swz<Sh::ROW_BYTES>(m, c)) = v;
+      }
+      fence_async_smem();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(q_ready);
+    }
+    const uint32_t lane_off = static_cast<uint32_t>(qw * 32) << 16;
+    float o[DH];
+#pragma unroll
+    for (int i = 0; i < DH; ++i) o[i] = 0.f;
+    float m_run = -INFINITY, l_run = 0.f, corr_prev = 1.f;
+    bool ok = true;
+    for (int j = 0; j < nkv && ok; ++j) {
+      const int b = j & 1;
+      ok = mbar_wait(s_full + b, (j >> 1) & 1, abort_flag);
+      ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
+      if (!ok) break;
+      tc_fence_after();
+      const int kbase = j * BKV;
+      // pass 1: row max of the scaled scores (keys past the history masked)
+      float mx = m_run;
+#pragma unroll 1
+      for (int cc = 0; cc < BKV; cc += 32) {
+        float sv[32];
+        tmem_ld32(t_s + b * BKV + cc + lane_off, sv);
+#pragma unroll
+        for (int i = 0; i < 32; ++i)
+          if (kbase + cc + i < len) mx = fmaxf(mx, sv[i] * a.scale_log2);
+      }
+      const float corr = exp2f(m_run - mx);
+      // the O tile of the previous K/V tile is complete: fold it in
+      if (j >= 1) {
+        ok = mbar_wait(o_full, (j - 1) & 1, abort_flag);
+        ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
+        if (!ok) break;
+        tc_fence_after();
+#pragma unroll
+        for (int cc = 0; cc < DH; cc += 32) {
+          float ov[32];
+          tmem_ld32(t_o + cc + lane_off, ov);
+#pragma unroll
+          for (int i = 0; i < 32; ++i) o[cc + i] = fmaf(o[cc + i], corr_prev, ov[i]);
+        }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(o_free);
+      }
+      // pass 2: P = exp2(s - max) into the swizzled P tile (bf16), row sum
+      float psum = 0.f;
+#pragma unroll 1
+      for (int cc = 0; cc < BKV; cc += 32) {
+        float sv[32];
+        tmem_ld32(t_s + b * BKV + cc + lane_off, sv);
+#pragma unroll
+        for (int g8 = 0; g8 < 4; ++g8) {
+          float p[8];
+#pragma unroll
+          for (int i = 0; i < 8; ++i) {
+            const int kk = cc + 8 * g8 + i;
+            p[i] = (kbase + kk < len) ? exp2f(sv[8 * g8 + i] * a.scale_log2 - mx) : 0.f;
+            psum += p[i];
+          }
+          uint4 pk;
+          __nv_bfloat162* h2 = reinterpret_cast<__nv_bfloat162*>(&pk);
+#pragma unroll
+          for (int i = 0; i < 4; ++i) h2[i] = __floats2bfloat162_rn(p[2 * i], p[2 * i + 1]);
+          const int key16 = (cc + 8 * g8) / 8;          // 16-byte chunk index within the 128 keys
+          const int blk = key16 / 8, c = key16 % 8;     // 64-key block, chunk within its 128-byte row
+          *reinterpret_cast<uint4*>(sP + blk * (BQ * 128) + swz<128>(m, c)) = pk;
+        }
+      }
+      tc_fence_before();
+      fence_async_smem();
+      __syncwarp();
+      if (lane == 0) {
+        mbar_arrive(s_free + b);
+        mbar_arrive(p_full);
+      }
+      l_run = l_run * corr + psum;
+      m_run = mx;
+      corr_prev = corr;
+    }
+    if (ok) {
+      ok = mbar_wait(o_full, (nkv - 1) & 1, abort_flag);
+      ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
+    }
+    if (ok) {
+      tc_fence_after();
+#pragma unroll
+      for (int cc = 0; cc < DH; cc += 32) {
+        float ov[32];
+        tmem_ld32(t_o + cc + lane_off, ov);
+#pragma unroll
+        for (int i = 0; i < 32; ++i) o[cc + i] = fmaf(o[cc + i], corr_prev, ov[i]);
+      }
+      if (valid) {
+        const float inv = 1.f / l_run;
+        __nv_bfloat16* dst = a.out + grow * a.d + h * DH;
+#pragma unroll
+        for (int c = 0; c < DH; c += 8) {
+          float t[8];
+#pragma unroll
+          for (int i = 0; i < 8; ++i) t[i] = o[c + i] * inv;
+          Vec16<__nv_bfloat16>::store(dst + c, t);
+        }
+      }
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, Sh::TMEM_COLS);
+  }
+  if (threadIdx.x == 0 && *abort_flag) latch_status(a.status, TXS_ERR_DEVICE_TIMEOUT);
+}
+
+// ------------------------------------------------------------------ host side
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                  const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+static EncodeTiledFn encode_fn() {
+  static EncodeTiledFn fn = nullptr;
+  if (!fn) {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(p);
+  }
+  return fn;
+}
+
+// K or V of one layer: [rows, d] bf16, box {DH columns, 128 rows}.
+template <int DH>
+static bool make_kv_map(CUtensorMap* tm, const void* base, long long rows, int d) {
+  EncodeTiledFn fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[2] = {static_cast<cuuint64_t>(d), static_cast<cuuint64_t>(rows)};
+  cuuint64_t strides[1] = {static_cast<cuuint64_t>(d) * 2};
+  cuuint32_t box[2] = {static_cast<cuuint32_t>(DH), static_cast<cuuint32_t>(BKV)};
+  cuuint32_t estr[2] = {1, 1};
+  return fn(tm, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, DH == 64 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_64B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+template <int DH>
+static cudaError_t launch_dh(const FaArgs& a, const void* Kc, const void* Vc, long long cap_total, int n_req,
+                             int max_q_tiles, int H, cudaStream_t s) {
+  using Sh = FaShape<DH>;
+  static bool attr = false;
+  if (!attr) {
+    cudaError_t e = cudaFuncSetAttribute(fa_full_kernel<DH>, cudaFuncAttributeMaxDynamicSharedMemorySize, Sh::SMEM);
+    if (e != cudaSuccess) return e;
+    attr = true;
+  }
+  CUtensorMap tk, tv;
+  if (!make_kv_map<DH>(&tk, Kc, cap_total, a.d) || !make_kv_map<DH>(&tv, Vc, cap_total, a.d))
+    return cudaErrorInvalidValue;
+  const dim3 grid(max_q_tiles, n_req, H);
+  fa_full_kernel<DH><<<grid, NUM_THREADS, Sh::SMEM, s>>>(tk, tv, a);
+  return cudaGetLastError();
+}
+
+}  // namespace fa
+
+bool fa_full_supported(int d, int H, long long cap_total) {
+  const int dh = d / H;
+  return (dh == 32 || dh == 64) && cap_total >= fa::BKV && d % 8 == 0;
+}
+
+cudaError_t launch_fa_full(const __nv_bfloat16* q, __nv_bfloat16* out, const __nv_bfloat16* Kc,
+                           const __nv_bfloat16* Vc, long long cap_total, const int* cand_off_dev,
+                           const int* cand_off_host, const int* kv_off, const int* kv_len, int n_req, int n_cand,
+                           int S, int H, int d, int* status, cudaStream_t s) {
+  int max_q = 0;
+  for (int r = 0; r < n_req; ++r) max_q = std::max(max_q, cand_off_host[r + 1] - cand_off_host[r] + S);
+  if (max_q == 0) return cudaSuccess;
+  const int dh = d / H;
+  fa::FaArgs a{q, out, cand_off_dev, kv_off, kv_len, n_cand, S, d,
+               1.4426950408889634f / sqrtf(static_cast<float>(dh)), status};
+  const int tiles = (max_q + fa::BQ - 1) / fa::BQ;
+  prof_begin(KC_ATTN_CROSS, s);
+  cudaError_t err = dh == 64 ? fa::launch_dh<64>(a, Kc, Vc, cap_total, n_req, tiles, H, s)
+                             : fa::launch_dh<32>(a, Kc, Vc, cap_total, n_req, tiles, H, s);
+  prof_end(KC_ATTN_CROSS, s);
+  return err;
+}
+
+}  // namespace txs

@@ -7,6 +7,7 @@
 #include <cstdio>
 #include <cstring>
 #include <string>
+#include <type_traits>
 #include <vector>
 
 #include "txs_internal.cuh"
@@ -406,8 +407,18 @@ txs_status score_impl(txs_model* m, const txs_kv_cache* c, int n_req, const int3
     const T* Vc = kv + (size_t(2 * l + 1) * c->cap_total) * d;
     const float* Kg = c->gkv + size_t(2 * l) * n_req * d;
     const float* Vg = c->gkv + size_t(2 * l + 1) * n_req * d;
-    TXS_CK(launch_cross_attn<T>(QKV, A, Kc, Vc, row_req, static_cast<int>(N), c->d_off, c->d_len, Kg, Vg,
-                                cf.l_local, cf.attn_mode, H, d, s));
+    if constexpr (std::is_same<T, __nv_bfloat16>::value) {
+      if (cf.attn_mode == TXS_ATTN_FULL && fa_full_supported(d, H, c->cap_total)) {
+        TXS_CK(launch_fa_full(QKV, A, Kc, Vc, c->cap_total, cand_off_dev, cand_off, c->d_off, c->d_len, n_req,
+                              static_cast<int>(n_cand), S, H, d, m->status, s));
+      } else {
+        TXS_CK(launch_cross_attn<T>(QKV, A, Kc, Vc, row_req, static_cast<int>(N), c->d_off, c->d_len, Kg, Vg,
+                                    cf.l_local, cf.attn_mode, H, d, s));
+      }
+    } else {
+      TXS_CK(launch_cross_attn<T>(QKV, A, Kc, Vc, row_req, static_cast<int>(N), c->d_off, c->d_len, Kg, Vg,
+                                  cf.l_local, cf.attn_mode, H, d, s));
+    }
     e = epi_base(EPI_LN, N, d, d);
     e.bias = W.b_oc;
     e.res = X1;

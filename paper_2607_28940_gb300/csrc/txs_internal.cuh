@@ -149,6 +149,14 @@ cudaError_t launch_cross_attn(const T* q, T* out, const T* Kc, const T* Vc, cons
                               const int* kv_off, const int* kv_len, const float* Kg, const float* Vg, int l_local,
                               int mode, int H, int d, cudaStream_t s);
 
+// FULL-mode cross-attention on the tensor cores (bf16): one CTA per
+// (128-query tile, request, head).
+bool fa_full_supported(int d, int H, long long cap_total);
+cudaError_t launch_fa_full(const __nv_bfloat16* q, __nv_bfloat16* out, const __nv_bfloat16* Kc,
+                           const __nv_bfloat16* Vc, long long cap_total, const int* cand_off_dev,
+                           const int* cand_off_host, const int* kv_off, const int* kv_len, int n_req, int n_cand,
+                           int S, int H, int d, int* status, cudaStream_t s);
+
 extern const int kPoolChunk;
 template <typename T>
 cudaError_t launch_pool(const T* phi, const int* seg_off, int R, int max_rows, const float* w_pool, int d,
