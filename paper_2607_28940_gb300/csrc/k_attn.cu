@@ -87,6 +87,8 @@ template <typename T, int DH>
 __global__ void __launch_bounds__(256) serving_attn_kernel(const T* __restrict__ qkv, T* __restrict__ out,
                                                            const int* __restrict__ row_req, int n_rows,
                                                            int n_cand_rows, int S, int H, int d, float scale) {
+  pdl_launch_dependents();
+  pdl_wait();
   using G = Group<T, DH>;
   constexpr int VEC = G::VEC;
   const long long gid = static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x;
@@ -134,6 +136,8 @@ template <typename T, int DH>
 __global__ void __launch_bounds__(256) cross_attn_kernel(const T* __restrict__ q_in, T* __restrict__ out,
                                                          const T* __restrict__ Kc, const T* __restrict__ Vc,
                                                          const CrossArgs a) {
+  pdl_launch_dependents();
+  pdl_wait();
   using G = Group<T, DH>;
   constexpr int VEC = G::VEC;
   const long long gid = static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x;
@@ -181,8 +185,7 @@ cudaError_t cross_launch(const T* q, T* out, const T* Kc, const T* Vc, CrossArgs
   const long long threads = static_cast<long long>(a.n_rows) * a.H * Group<T, DH>::TPH;
   const int blocks = static_cast<int>((threads + 255) / 256);
   a.scale = (1.0f / sqrtf(static_cast<float>(DH)));
-  cross_attn_kernel<T, DH><<<blocks, 256, 0, s>>>(q, out, Kc, Vc, a);
-  return cudaGetLastError();
+  return launch_pdl(cross_attn_kernel<T, DH>, dim3(blocks), dim3(256), 0, s, q, out, Kc, Vc, a);
 }
 
 }  // namespace
@@ -192,9 +195,8 @@ static cudaError_t serving_launch(const T* qkv, T* out, const int* row_req, int 
                                   int d, cudaStream_t s) {
   const long long threads = static_cast<long long>(n_rows) * H * Group<T, DH>::TPH;
   const int blocks = static_cast<int>((threads + 255) / 256);
-  serving_attn_kernel<T, DH><<<blocks, 256, 0, s>>>(qkv, out, row_req, n_rows, n_cand_rows, S, H, d,
-                                                    1.0f / sqrtf(static_cast<float>(DH)));
-  return cudaGetLastError();
+  return launch_pdl(serving_attn_kernel<T, DH>, dim3(blocks), dim3(256), 0, s, qkv, out, row_req, n_rows,
+                    n_cand_rows, S, H, d, 1.0f / sqrtf(static_cast<float>(DH)));
 }
 
 template <typename T>

@@ -193,6 +193,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(o_free + 1);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_holder + 1);
 
+  pdl_launch_dependents();
+  pdl_wait();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int qt = blockIdx.x, r = blockIdx.y, h = blockIdx.z;
   const int c0 = a.cand_off[r];
@@ -465,8 +467,7 @@ static cudaError_t launch_dh(const FaArgs& a, const void* Kc, const void* Vc, lo
   if (!make_kv_map<DH>(&tk, Kc, cap_total, a.d) || !make_kv_map<DH>(&tv, Vc, cap_total, a.d))
     return cudaErrorInvalidValue;
   const dim3 grid(max_q_tiles, n_req, H);
-  fa_full_kernel<DH><<<grid, NUM_THREADS, Sh::SMEM, s>>>(tk, tv, a);
-  return cudaGetLastError();
+  return launch_pdl(fa_full_kernel<DH>, grid, dim3(NUM_THREADS), Sh::SMEM, s, tk, tv, a);
 }
 
 }  // namespace fa

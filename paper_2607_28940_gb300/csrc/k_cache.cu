@@ -30,6 +30,8 @@ __global__ void __launch_bounds__(256) pool_partial_kernel(const T* __restrict__
                                                            int max_chunks, float* __restrict__ part,
                                                            int merge_existing, float* st_m, float* st_s,
                                                            float* st_acc, float* __restrict__ g, int* counter) {
+  pdl_launch_dependents();
+  pdl_wait();
   constexpr int VEC = Vec16<T>::N;               // MAXC: 16-byte chunks per lane, ceil(d / (32 VEC))
   __shared__ float sm_m[kPoolWarps], sm_s[kPoolWarps];
   __shared__ float sm_acc[kPoolWarps][512];
@@ -182,6 +184,8 @@ template <typename T, int NCH>
 __global__ void __launch_bounds__(256) anchor_proj_kernel(const float* __restrict__ g, const T* __restrict__ Wt,
                                                           const float* __restrict__ b, float* __restrict__ gkv,
                                                           int R, int d, int n_total) {
+  pdl_launch_dependents();
+  pdl_wait();
   constexpr int VEC = Vec16<T>::N;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const long long wid = static_cast<long long>(blockIdx.x) * 8 + warp;
@@ -305,19 +309,20 @@ cudaError_t launch_pool(const T* phi, const int* seg_off, int R, int max_rows, c
   const int nch = (d + 32 * VEC - 1) / (32 * VEC);
   const float isd = 1.0f / sqrtf(static_cast<float>(d));
   const dim3 grid(chunks, R);
+  cudaError_t err0 = cudaSuccess;
   prof_begin(KC_POOL, s);
   if (nch == 1)
-    pool_partial_kernel<T, 1><<<grid, 256, 0, s>>>(phi, seg_off, w_pool, d, isd, max_chunks, part, merge_existing,
-                                                   st_m, st_s, st_acc, g, counter);
+    err0 = launch_pdl(pool_partial_kernel<T, 1>, grid, dim3(256), 0, s, phi, seg_off, w_pool, d, isd, max_chunks,
+                      part, merge_existing, st_m, st_s, st_acc, g, counter);
   else if (nch == 2)
-    pool_partial_kernel<T, 2><<<grid, 256, 0, s>>>(phi, seg_off, w_pool, d, isd, max_chunks, part, merge_existing,
-                                                   st_m, st_s, st_acc, g, counter);
+    err0 = launch_pdl(pool_partial_kernel<T, 2>, grid, dim3(256), 0, s, phi, seg_off, w_pool, d, isd, max_chunks,
+                      part, merge_existing, st_m, st_s, st_acc, g, counter);
   else if (nch <= 4)
-    pool_partial_kernel<T, 4><<<grid, 256, 0, s>>>(phi, seg_off, w_pool, d, isd, max_chunks, part, merge_existing,
-                                                   st_m, st_s, st_acc, g, counter);
+    err0 = launch_pdl(pool_partial_kernel<T, 4>, grid, dim3(256), 0, s, phi, seg_off, w_pool, d, isd, max_chunks,
+                      part, merge_existing, st_m, st_s, st_acc, g, counter);
   else
     return cudaErrorInvalidValue;
-  cudaError_t err = cudaGetLastError();
+  cudaError_t err = err0 != cudaSuccess ? err0 : cudaGetLastError();
   prof_end(KC_POOL, s);
   return err;
 }
@@ -331,11 +336,11 @@ cudaError_t launch_anchor_proj(const float* g, const T* Wt_kv, const float* b_kv
   const long long warps = static_cast<long long>(n_total) * ((R + kAnchorReqPerWarp - 1) / kAnchorReqPerWarp);
   const int blocks = static_cast<int>((warps + 7) / 8);
   prof_begin(KC_GLOBAL_KV, s);
-  if (nch == 1) anchor_proj_kernel<T, 1><<<blocks, 256, 0, s>>>(g, Wt_kv, b_kv, gkv, R, d, n_total);
-  else if (nch == 2) anchor_proj_kernel<T, 2><<<blocks, 256, 0, s>>>(g, Wt_kv, b_kv, gkv, R, d, n_total);
-  else if (nch <= 4) anchor_proj_kernel<T, 4><<<blocks, 256, 0, s>>>(g, Wt_kv, b_kv, gkv, R, d, n_total);
+  cudaError_t err;
+  if (nch == 1) err = launch_pdl(anchor_proj_kernel<T, 1>, dim3(blocks), dim3(256), 0, s, g, Wt_kv, b_kv, gkv, R, d, n_total);
+  else if (nch == 2) err = launch_pdl(anchor_proj_kernel<T, 2>, dim3(blocks), dim3(256), 0, s, g, Wt_kv, b_kv, gkv, R, d, n_total);
+  else if (nch <= 4) err = launch_pdl(anchor_proj_kernel<T, 4>, dim3(blocks), dim3(256), 0, s, g, Wt_kv, b_kv, gkv, R, d, n_total);
   else return cudaErrorInvalidValue;
-  cudaError_t err = cudaGetLastError();
   prof_end(KC_GLOBAL_KV, s);
   return err;
 }

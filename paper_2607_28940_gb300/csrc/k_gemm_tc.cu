@@ -407,17 +407,21 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     *abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
-  if constexpr (EPI == EPI_LN_HEAD) {
-    for (int i = threadIdx.x; i < e.N * NAP; i += NUM_THREADS) {
-      const int c = i / NAP, a = i - c * NAP;
-      s_weff[i] = a < e.n_act ? e.weff_z[c * e.n_act + a] : 0.f;
-    }
-  }
   if (warp == 1) tmem_alloc(tmem_holder, S::TMEM_COLS);
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_holder;
+  // the set-up above overlaps the previous kernel's tail; its outputs are read below
+  pdl_launch_dependents();
+  pdl_wait();
+  if constexpr (EPI == EPI_LN_HEAD) {
+    for (int i = threadIdx.x; i < e.N * NAP; i += NUM_THREADS) {
+      const int c = i / NAP, a = i - c * NAP;
+      s_weff[i] = a < e.n_act ? e.weff_z[c * e.n_act + a] : 0.f;
+    }
+    __syncthreads();
+  }
 
   if (warp == 0) {
     if (lane == 0) {
@@ -579,8 +583,7 @@ static cudaError_t launch_bn(const __nv_bfloat16* A, long long lda, const __nv_b
   const long long tiles = static_cast<long long>((e.M + BM - 1) / BM) * (e.N / BN);
   const int grid = static_cast<int>(tiles < num_sms() ? tiles : num_sms());
   prof_begin(cls, s);
-  gemm_tc_kernel<BN, EPI, NAP><<<grid, NUM_THREADS, Sh::SMEM_BYTES, s>>>(ta, tb, e);
-  cudaError_t err = cudaGetLastError();
+  cudaError_t err = launch_pdl(gemm_tc_kernel<BN, EPI, NAP>, dim3(grid), dim3(NUM_THREADS), Sh::SMEM_BYTES, s, ta, tb, e);
   prof_end(cls, s);
   return err;
 }

@@ -48,6 +48,8 @@ __global__ void __launch_bounds__(256) pack_kernel(const __grid_constant__ PackA
                                                    int* __restrict__ row_req, int* __restrict__ cand_off_dev,
                                                    const float* __restrict__ weff_x,
                                                    const float* __restrict__ cdec, float* __restrict__ xlog) {
+  pdl_launch_dependents();
+  pdl_wait();
   constexpr int VEC = Vec16<T>::N;
   extern __shared__ float sw[];                 // [na][d]
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -122,6 +124,8 @@ __device__ __forceinline__ uint32_t order_key(float f) {
 
 __global__ void __launch_bounds__(1024) rank_kernel(const __grid_constant__ RankArgs a, const float* __restrict__ probs,
                                                     int* __restrict__ out) {
+  pdl_launch_dependents();
+  pdl_wait();
   extern __shared__ uint32_t keys[];
   const int r = blockIdx.x;
   const int c0 = a.cand_off[r];
@@ -168,9 +172,8 @@ cudaError_t launch_pack(int n_req, const int* cand_off_host, int S, int d, int n
   }
   const long long rows_per_cta = 8LL * kPackRowsPerWarp;
   prof_begin(KC_PACK, s);
-  pack_kernel<T><<<static_cast<int>((n_rows + rows_per_cta - 1) / rows_per_cta), 256, smem, s>>>(
-      a, cand, ctx, X, row_req, cand_off_dev, weff_x, cdec, xlog);
-  cudaError_t err = cudaGetLastError();
+  cudaError_t err = launch_pdl(pack_kernel<T>, dim3(static_cast<int>((n_rows + rows_per_cta - 1) / rows_per_cta)),
+                               dim3(256), smem, s, a, cand, ctx, X, row_req, cand_off_dev, weff_x, cdec, xlog);
   prof_end(KC_PACK, s);
   return err;
 }
@@ -197,8 +200,7 @@ cudaError_t launch_rank(int n_req, const int* cand_off_host, const float* probs,
     attr = true;
   }
   prof_begin(KC_RANK, s);
-  rank_kernel<<<n_req, 1024, smem, s>>>(a, probs, out);
-  cudaError_t err = cudaGetLastError();
+  cudaError_t err = launch_pdl(rank_kernel, dim3(n_req), dim3(1024), smem, s, a, probs, out);
   prof_end(KC_RANK, s);
   return err;
 }

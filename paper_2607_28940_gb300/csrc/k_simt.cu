@@ -19,6 +19,8 @@ template <int EPI, typename TB>
 __global__ void __launch_bounds__(256) gemm_simt_kernel(const float* __restrict__ A, long long lda,
                                                         const TB* __restrict__ B, const EpiArgs e,
                                                         float* __restrict__ tmp) {
+  pdl_launch_dependents();
+  pdl_wait();
   __shared__ float As[TK][TM + 4];
   __shared__ float Bs[TK][TN + 4];
   const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
@@ -89,6 +91,8 @@ __global__ void __launch_bounds__(256) gemm_simt_kernel(const float* __restrict_
 // variance), then either store (EPI_LN) or the action head (EPI_LN_HEAD).
 template <int EPI>
 __global__ void __launch_bounds__(256) row_ln_kernel(const float* __restrict__ tmp, const EpiArgs e) {
+  pdl_launch_dependents();
+  pdl_wait();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int row = blockIdx.x * 8 + warp;
   if (row >= e.M) return;
@@ -165,26 +169,26 @@ cudaError_t launch_gemm_simt(const float* A, long long lda, const TB* B, const E
   if (e.M == 0) return cudaSuccess;
   if ((e.epi == EPI_LN || e.epi == EPI_LN_HEAD) && e.N > 1024) return cudaErrorInvalidValue;
   dim3 grid((e.M + TM - 1) / TM, (e.N + TN - 1) / TN);
+  cudaError_t err0 = cudaSuccess;
   prof_begin(cls, s);
   switch (e.epi) {
-    case EPI_BIAS: gemm_simt_kernel<EPI_BIAS, TB><<<grid, 256, 0, s>>>(A, lda, B, e, tmp); break;
-    case EPI_BIAS_GELU: gemm_simt_kernel<EPI_BIAS_GELU, TB><<<grid, 256, 0, s>>>(A, lda, B, e, tmp); break;
-    case EPI_KV: gemm_simt_kernel<EPI_KV, TB><<<grid, 256, 0, s>>>(A, lda, B, e, tmp); break;
+    case EPI_BIAS: err0 = launch_pdl(gemm_simt_kernel<EPI_BIAS, TB>, grid, dim3(256), 0, s, A, lda, B, e, tmp); break;
+    case EPI_BIAS_GELU: err0 = launch_pdl(gemm_simt_kernel<EPI_BIAS_GELU, TB>, grid, dim3(256), 0, s, A, lda, B, e, tmp); break;
+    case EPI_KV: err0 = launch_pdl(gemm_simt_kernel<EPI_KV, TB>, grid, dim3(256), 0, s, A, lda, B, e, tmp); break;
     case EPI_LN:
     case EPI_LN_HEAD:
-      gemm_simt_kernel<EPI_LN, TB><<<grid, 256, 0, s>>>(A, lda, B, e, tmp);
+      err0 = launch_pdl(gemm_simt_kernel<EPI_LN, TB>, grid, dim3(256), 0, s, A, lda, B, e, tmp);
       break;
     default: return cudaErrorInvalidValue;
   }
-  cudaError_t err = cudaGetLastError();
+  cudaError_t err = err0 != cudaSuccess ? err0 : cudaGetLastError();
   prof_end(cls, s);
   if (err != cudaSuccess) return err;
   if (e.epi == EPI_LN || e.epi == EPI_LN_HEAD) {
     prof_begin(KC_ROW_LN, s);
     const int blocks = (e.M + 7) / 8;
-    if (e.epi == EPI_LN) row_ln_kernel<EPI_LN><<<blocks, 256, 0, s>>>(tmp, e);
-    else row_ln_kernel<EPI_LN_HEAD><<<blocks, 256, 0, s>>>(tmp, e);
-    err = cudaGetLastError();
+    if (e.epi == EPI_LN) err = launch_pdl(row_ln_kernel<EPI_LN>, dim3(blocks), dim3(256), 0, s, tmp, e);
+    else err = launch_pdl(row_ln_kernel<EPI_LN_HEAD>, dim3(blocks), dim3(256), 0, s, tmp, e);
     prof_end(KC_ROW_LN, s);
   }
   return err;

@@ -26,6 +26,12 @@ static_assert(KC_COUNT_ <= TXS_N_KERNEL_CLASSES, "profiler classes");
 
 // ------------------------------------------------------------------ device helpers
 
+// Programmatic dependent launch: every hot-path kernel lets its successor
+// launch early (its prologue then overlaps this kernel's tail) and waits for
+// its predecessor's completion before touching global memory.
+__device__ __forceinline__ void pdl_launch_dependents() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
 __device__ __forceinline__ void latch_status(int* status, int code) {
   if (status) atomicCAS(status, 0, code);
 }
@@ -88,6 +94,23 @@ __device__ __forceinline__ int find_segment(const int* off, int n, int row) {
 }
 
 // ------------------------------------------------------------------ host side
+
+// Launch with programmatic stream serialization (see pdl_wait).
+template <typename... KArgs, typename... Args>
+inline cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t s,
+                              Args&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kernel, static_cast<KArgs>(args)...);
+}
 
 struct Prof;  // event profiler (txs_api.cu)
 void prof_begin(int cls, cudaStream_t s);
