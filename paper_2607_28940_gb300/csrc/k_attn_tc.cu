@@ -118,6 +118,13 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float* v) {
   for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
 }
 
+// 2^x on the special-function unit (PTX ex2.approx, flush-to-zero).
+__device__ __forceinline__ float ex2(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
 // Shared-memory matrix descriptor (tcgen05): start address, leading/stride
 // byte offsets, descriptor version 1, layout code (2 = 128-byte swizzle,
 // 4 = 64-byte swizzle).
@@ -313,7 +320,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     float o[DH];
 #pragma unroll
     for (int i = 0; i < DH; ++i) o[i] = 0.f;
-    float m_run = -INFINITY, l_run = 0.f, corr_prev = 1.f;
+    float m_run = -INFINITY, l_run = 0.f, corr_prev = 0.f;
     bool ok = true;
     for (int j = 0; j < nkv && ok; ++j) {
       const int b = j & 1;
@@ -322,17 +329,21 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       if (!ok) break;
       tc_fence_after();
       const int kbase = j * BKV;
-      // pass 1: row max of the scaled scores (keys past the history masked)
-      float mx = m_run;
-#pragma unroll 1
-      for (int cc = 0; cc < BKV; cc += 32) {
-        float sv[32];
-        tmem_ld32(t_s + b * BKV + cc + lane_off, sv);
+      const bool full_tile = kbase + BKV <= len;       // no masking needed (uniform)
+      // the whole score row of this tile: one pass over TMEM
+      float sv[BKV];
 #pragma unroll
-        for (int i = 0; i < 32; ++i)
-          if (kbase + cc + i < len) mx = fmaxf(mx, sv[i] * a.scale_log2);
+      for (int cc = 0; cc < BKV; cc += 32) tmem_ld32(t_s + b * BKV + cc + lane_off, sv + cc);
+      if (!full_tile) {
+#pragma unroll
+        for (int i = 0; i < BKV; ++i)
+          if (kbase + i >= len) sv[i] = -INFINITY;
       }
-      const float corr = exp2f(m_run - mx);
+      float mraw = sv[0];
+#pragma unroll
+      for (int i = 1; i < BKV; ++i) mraw = fmaxf(mraw, sv[i]);
+      const float mx = fmaxf(m_run, mraw * a.scale_log2);
+      const float corr = ex2(m_run - mx);
       // the O tile of the previous K/V tile is complete: fold it in
       if (j >= 1) {
         ok = mbar_wait(o_full, (j - 1) & 1, abort_flag);
@@ -350,29 +361,22 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         __syncwarp();
         if (lane == 0) mbar_arrive(o_free);
       }
-      // pass 2: P = exp2(s - max) into the swizzled P tile (bf16), row sum
+      // P = 2^(s * scale - max) into the swizzled P tile (bf16), row sum
       float psum = 0.f;
-#pragma unroll 1
-      for (int cc = 0; cc < BKV; cc += 32) {
-        float sv[32];
-        tmem_ld32(t_s + b * BKV + cc + lane_off, sv);
 #pragma unroll
-        for (int g8 = 0; g8 < 4; ++g8) {
-          float p[8];
+      for (int key16 = 0; key16 < BKV / 8; ++key16) {
+        float p[8];
 #pragma unroll
-          for (int i = 0; i < 8; ++i) {
-            const int kk = cc + 8 * g8 + i;
-            p[i] = (kbase + kk < len) ? exp2f(sv[8 * g8 + i] * a.scale_log2 - mx) : 0.f;
-            psum += p[i];
-          }
-          uint4 pk;
-          __nv_bfloat162* h2 = reinterpret_cast<__nv_bfloat162*>(&pk);
-#pragma unroll
-          for (int i = 0; i < 4; ++i) h2[i] = __floats2bfloat162_rn(p[2 * i], p[2 * i + 1]);
-          const int key16 = (cc + 8 * g8) / 8;          // 16-byte chunk index within the 128 keys
-          const int blk = key16 / 8, c = key16 % 8;     // 64-key block, chunk within its 128-byte row
-          *reinterpret_cast<uint4*>(sP + blk * (BQ * 128) + swz<128>(m, c)) = pk;
+        for (int i = 0; i < 8; ++i) {
+          p[i] = ex2(fmaf(sv[8 * key16 + i], a.scale_log2, -mx));
+          psum += p[i];
         }
+        uint4 pk;
+        __nv_bfloat162* h2 = reinterpret_cast<__nv_bfloat162*>(&pk);
+#pragma unroll
+        for (int i = 0; i < 4; ++i) h2[i] = __floats2bfloat162_rn(p[2 * i], p[2 * i + 1]);
+        const int blk = key16 / 8, c = key16 % 8;       // 64-key block, 16-byte chunk within its row
+        *reinterpret_cast<uint4*>(sP + blk * (BQ * 128) + swz<128>(m, c)) = pk;
       }
       tc_fence_before();
       fence_async_smem();

@@ -185,6 +185,29 @@ __device__ __forceinline__ void load_f32x32(const float* p, float* b) {
   }
 }
 
+// Same, from a generic pointer (shared or global memory).
+__device__ __forceinline__ void load_f32x32_gen(const float* p, float* b) {
+  const float4* q = reinterpret_cast<const float4*>(p);
+#pragma unroll
+  for (int j = 0; j < 8; ++j) {
+    float4 t = q[j];
+    b[4 * j] = t.x; b[4 * j + 1] = t.y; b[4 * j + 2] = t.z; b[4 * j + 3] = t.w;
+  }
+}
+
+// largest r with off[r] <= row, off[0..n] non-decreasing (generic pointer)
+__device__ __forceinline__ int find_seg_gen(const int* off, int n, int row) {
+  int lo = 0, hi = n - 1;
+  while (lo < hi) {
+    const int mid = (lo + hi + 1) >> 1;
+    if (off[mid] <= row) lo = mid; else hi = mid - 1;
+  }
+  return lo;
+}
+
+constexpr int kStageN = 4096;     // bias entries staged in shared memory
+constexpr int kStageSeg = 1024;   // request offsets staged in shared memory (cache-row remap)
+
 __device__ __forceinline__ void store_bf16x32(__nv_bfloat16* p, const float* v) {
 #pragma unroll
   for (int j = 0; j < 4; ++j) Vec16<__nv_bfloat16>::store(p + 8 * j, v + 8 * j);
@@ -204,7 +227,8 @@ constexpr int kRedStride = 17;                // per-row exchange slots: sum + 1
 // share a lane quarter exchange row sums (and head logits) through `red`.
 template <int BN, int EPI, int NAP>
 __device__ __forceinline__ void epilogue(const EpiArgs& e, uint32_t tacc, int row, int n0, int c0, int q, int h,
-                                         float* red, const float* s_weff) {
+                                         float* red, const float* s_weff, const float* bias,
+                                         const int* seg_off, const int* dst_row0) {
   constexpr int HALF = BN / 2;
   const bool valid = row < e.M;
   const int lane = threadIdx.x & 31;
@@ -215,8 +239,8 @@ __device__ __forceinline__ void epilogue(const EpiArgs& e, uint32_t tacc, int ro
       long long orow = row;
       long long ocol = n0 + c0;
       if constexpr (EPI == EPI_KV) {
-        const int r = find_segment(e.seg_off, e.n_seg, row);
-        orow = static_cast<long long>(__ldg(e.dst_row0 + r)) + (row - __ldg(e.seg_off + r));
+        const int r = find_seg_gen(seg_off, e.n_seg, row);
+        orow = static_cast<long long>(dst_row0[r]) + (row - seg_off[r]);
         const int blk = n0 / e.col_blk;
         ocol = static_cast<long long>(blk) * e.col_blk_stride + (n0 - blk * e.col_blk) + c0;
       }
@@ -227,7 +251,7 @@ __device__ __forceinline__ void epilogue(const EpiArgs& e, uint32_t tacc, int ro
       tmem_ld32(tacc + c0 + c, v);
       if (valid) {
         float b[32];
-        load_f32x32(e.bias + n0 + c0 + c, b);
+        load_f32x32_gen(bias + n0 + c0 + c, b);
 #pragma unroll
         for (int i = 0; i < 32; ++i) {
           float x = v[i] + b[i];
@@ -356,13 +380,18 @@ struct Shape {
   static constexpr bool LN = EPI == EPI_LN || EPI == EPI_LN_HEAD;
   static constexpr int RED_BYTES = LN ? 2 * 128 * kRedStride * 4 : 0;
   static constexpr int WEFF_BYTES = EPI == EPI_LN_HEAD ? BN * NAP * 4 : 0;
-  static constexpr int EXTRA = RED_BYTES + WEFF_BYTES + 1024 + 256;
+  // bias [kStageN] floats, then (cache-row remap) offsets and first rows; the
+  // mbarriers after this region need 8-byte alignment, so round to 16 bytes
+  static constexpr int AUX_BYTES =
+      LN ? 0 : ((kStageN * 4 + (EPI == EPI_KV ? (2 * kStageSeg + 1) * 4 : 0) + 15) / 16) * 16;
+  static constexpr int EXTRA = RED_BYTES + WEFF_BYTES + AUX_BYTES + 1024 + 256;
   static constexpr int STAGES_FIT = (227 * 1024 - EXTRA) / STAGE_BYTES;
   static constexpr int STAGES = STAGES_FIT > 8 ? 8 : STAGES_FIT;
   static constexpr int ACC_BUFS = BN <= 256 ? 2 : 1;      // TMEM double buffer
   static constexpr int TMEM_COLS = BN * ACC_BUFS < 32 ? 32 : BN * ACC_BUFS;
   static constexpr int SMEM_BYTES = STAGES * STAGE_BYTES + EXTRA;
   static_assert(STAGES >= 2, "pipeline depth");
+  static_assert((RED_BYTES + WEFF_BYTES + AUX_BYTES) % 16 == 0, "mbarriers must stay 8-byte aligned");
   static_assert(SMEM_BYTES <= 232448, "shared memory");
   static_assert((TMEM_COLS & (TMEM_COLS - 1)) == 0 && TMEM_COLS <= 512, "TMEM columns");
 };
@@ -383,7 +412,10 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   uint8_t* sB = smem + S::STAGES * A_STAGE_BYTES;
   float* red = reinterpret_cast<float*>(sB + S::STAGES * S::B_STAGE_BYTES);
   float* s_weff = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(red) + S::RED_BYTES);
-  uint64_t* full = reinterpret_cast<uint64_t*>(reinterpret_cast<uint8_t*>(s_weff) + S::WEFF_BYTES);
+  float* s_bias = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(s_weff) + S::WEFF_BYTES);
+  int* s_seg = reinterpret_cast<int*>(s_bias + kStageN);
+  int* s_dst = s_seg + kStageSeg + 1;
+  uint64_t* full = reinterpret_cast<uint64_t*>(reinterpret_cast<uint8_t*>(s_bias) + S::AUX_BYTES);
   uint64_t* empty = full + S::STAGES;
   uint64_t* acc_full = empty + S::STAGES;
   uint64_t* acc_empty = acc_full + 2;
@@ -419,6 +451,26 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     for (int i = threadIdx.x; i < e.N * NAP; i += NUM_THREADS) {
       const int c = i / NAP, a = i - c * NAP;
       s_weff[i] = a < e.n_act ? e.weff_z[c * e.n_act + a] : 0.f;
+    }
+    __syncthreads();
+  }
+  // epilogue operands read by every tile: bias (and the cache-row remap) in
+  // shared memory when they fit
+  const float* bias = e.bias;
+  const int* seg_off = e.seg_off;
+  const int* dst_row0 = e.dst_row0;
+  if constexpr (!S::LN) {
+    if (e.N <= kStageN) {
+      for (int i = threadIdx.x; i < e.N; i += NUM_THREADS) s_bias[i] = e.bias[i];
+      bias = s_bias;
+    }
+    if constexpr (EPI == EPI_KV) {
+      if (e.n_seg <= kStageSeg) {
+        for (int i = threadIdx.x; i <= e.n_seg; i += NUM_THREADS) s_seg[i] = e.seg_off[i];
+        for (int i = threadIdx.x; i < e.n_seg; i += NUM_THREADS) s_dst[i] = e.dst_row0[i];
+        seg_off = s_seg;
+        dst_row0 = s_dst;
+      }
     }
     __syncthreads();
   }
@@ -506,7 +558,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       tc_fence_after();
       const int m0 = (t / n_tiles) * BM, n0 = (t % n_tiles) * BN;
       epilogue<BN, EPI, NAP>(e, tmem + buf * BN + (static_cast<uint32_t>(q * 32) << 16), m0 + q * 32 + lane, n0,
-                        h * (BN / 2), q, h, red, s_weff);
+                             h * (BN / 2), q, h, red, s_weff, bias, seg_off, dst_row0);
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(acc_empty + buf);
