@@ -44,7 +44,11 @@ FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0}
 # DRAM traffic per launch measured with ncu (dram__bytes_read.sum +
 # dram__bytes_write.sum) for the kernel classes that can be dominant, with the
 # sha256 prefix of the kernel source at capture time; a source change voids it.
-NCU_TRAFFIC = {}
+# (workload, mode, class) -> (bytes per launch, source sha256[:12]); from
+# profiles/gemm_tc_small_bf16.md.
+NCU_TRAFFIC = {
+    ("small_bf16", "local_global", "gemm_oproj_ln"): (8.61e6, "40a69cd3f2dd"),
+}
 
 
 def parse():
@@ -141,7 +145,7 @@ class ClockSampler:
         try:
             self.f = open(self.path, "w")
             self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.index), f"--query-gpu={CLOCK_FIELDS}",
-                                          "--format=csv,noheader,nounits", "-lms", "100"],
+                                          "--format=csv,noheader,nounits", "-lms", "50"],
                                          stdout=self.f, stderr=subprocess.DEVNULL)
         except Exception:
             self.proc = None
@@ -298,8 +302,11 @@ def run_txs(args, rank, world):
         roof = {"bound": "hbm", "achieved": achieved, "peak": peaks["hbm_gbs"], "unit": "GB/s"}
     roof["frac"] = roof["achieved"] / roof["peak"]
     tr = NCU_TRAFFIC.get((args.workload, args.mode, dom))
-    src_sha = hashlib.sha256(open(os.path.join(ROOT, "paper_2607_28940_gb300", "csrc",
-                                               "k_gemm_tc.cu" if dom.startswith("gemm") else "k_attn.cu"),
+    src_file = ("k_gemm_tc.cu" if dom.startswith("gemm") else
+                "k_attn_tc.cu" if (dom == "attn_cross" and args.mode == "full" and wl.dtype == "bf16") else
+                "k_score.cu" if dom in ("pack", "rank") else
+                "k_cache.cu" if dom in ("pool", "global_kv") else "k_attn.cu")
+    src_sha = hashlib.sha256(open(os.path.join(ROOT, "paper_2607_28940_gb300", "csrc", src_file),
                                   "rb").read()).hexdigest()[:12]
     roof["traffic"] = tr[0] if tr and tr[1] == src_sha else None
     roof["kernel"] = dom
@@ -426,15 +433,20 @@ def cpu_baseline(workload: str, budget_s: float):
     wl = W.WORKLOADS[workload]
     model = O.Model.from_arrays(W.weights(wl), wl)
     n_done, cands, t_tot = 0, 0, 0.0
-    while n_done < wl.n_req and (t_tot < budget_s or n_done == 0):
-        b = W.batch(wl, requests=[n_done])
+    batches = {}
+    while t_tot < budget_s or n_done == 0:
+        r = n_done % wl.n_req
+        if r not in batches:
+            batches[r] = W.batch(wl, requests=[r])
         t0 = time.perf_counter()
-        cands += oracle_step(O, model, wl, b, 0)
+        cands += oracle_step(O, model, wl, batches[r], 0)
         t_tot += time.perf_counter() - t0
         n_done += 1
+        if n_done >= 50 * wl.n_req:
+            break
     return {"value": cands / t_tot, "unit": "candidates/s", "cores": os.cpu_count(), "kind": "oracle",
-            "sample": f"{n_done} of {wl.n_req} requests of {workload}, each cache build + append + score + rank "
-                      f"in float64 NumPy ({t_tot:.1f} s)"}
+            "sample": f"{n_done} request-steps cycling over the {wl.n_req} requests of {workload}, each cache build "
+                      f"+ append + score + rank in float64 NumPy ({t_tot:.1f} s)"}
 
 
 def run_reference(args, rank, world):
