@@ -81,6 +81,23 @@ __device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* tm, ui
       : "memory");
 }
 
+// Bulk tensor store shared -> global (one thread), tracked in a per-thread bulk group.
+__device__ __forceinline__ void tma_store_2d(const CUtensorMap* tm, const void* src, int x, int y) {
+  asm volatile("cp.async.bulk.tensor.2d.global.shared::cta.bulk_group [%0, {%2, %3}], [%1];" ::"l"(
+                   reinterpret_cast<uint64_t>(tm)),
+               "r"(smem_u32(src)), "r"(x), "r"(y)
+               : "memory");
+}
+__device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
+// Wait until at most N of this thread's bulk groups still read shared memory.
+template <int N>
+__device__ __forceinline__ void bulk_wait_read() {
+  asm volatile("cp.async.bulk.wait_group.read %0;" ::"n"(N) : "memory");
+}
+// Wait until all of this thread's bulk groups have completed.
+__device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
+__device__ __forceinline__ void fence_async_smem() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
+
 __device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
 __device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
 
@@ -213,6 +230,37 @@ __device__ __forceinline__ void store_bf16x32(__nv_bfloat16* p, const float* v) 
   for (int j = 0; j < 4; ++j) Vec16<__nv_bfloat16>::store(p + 8 * j, v + 8 * j);
 }
 
+// Store this warp's 32 rows x 32 bf16 columns.  With `tma_ok` the lanes write
+// their rows into a 2 KB staging buffer (64-byte swizzle, matching the output
+// tensor map) and lane 0 issues one bulk tensor store at (x, y): full 32-byte
+// sectors instead of 32 row-strided 16-byte stores.  Otherwise each valid lane
+// stores its own 64 bytes at `direct`.  `k` counts the warp's chunks so that
+// each of the two staging buffers is reused only after its store has read it.
+__device__ __forceinline__ void store_chunk(const float* v, __nv_bfloat16* direct, bool valid, bool tma_ok,
+                                            const CUtensorMap* tmO, int x, int y, uint8_t* stage, int k, int lane) {
+  if (tma_ok) {
+    uint8_t* buf = stage + (k & 1) * 2048;
+    if (lane == 0) bulk_wait_read<1>();
+    __syncwarp();
+#pragma unroll
+    for (int c = 0; c < 4; ++c) {
+      uint4 pk;
+      __nv_bfloat162* h2 = reinterpret_cast<__nv_bfloat162*>(&pk);
+#pragma unroll
+      for (int i = 0; i < 4; ++i) h2[i] = __floats2bfloat162_rn(v[8 * c + 2 * i], v[8 * c + 2 * i + 1]);
+      *reinterpret_cast<uint4*>(buf + lane * 64 + ((c ^ ((lane >> 1) & 3)) << 4)) = pk;
+    }
+    fence_async_smem();
+    __syncwarp();
+    if (lane == 0) {
+      tma_store_2d(tmO, buf, x, y);
+      bulk_commit();
+    }
+  } else if (valid) {
+    store_bf16x32(direct, v);
+  }
+}
+
 __device__ __forceinline__ void load_bf16x32(const __nv_bfloat16* p, float* v) {
 #pragma unroll
   for (int j = 0; j < 4; ++j) Vec16<__nv_bfloat16>::load(p + 8 * j, v + 8 * j);
@@ -228,38 +276,51 @@ constexpr int kRedStride = 17;                // per-row exchange slots: sum + 1
 template <int BN, int EPI, int NAP>
 __device__ __forceinline__ void epilogue(const EpiArgs& e, uint32_t tacc, int row, int n0, int c0, int q, int h,
                                          float* red, const float* s_weff, const float* bias,
-                                         const int* seg_off, const int* dst_row0) {
+                                         const int* seg_off, const int* dst_row0, const CUtensorMap* tmO,
+                                         uint8_t* stage, int& kchunk) {
   constexpr int HALF = BN / 2;
   const bool valid = row < e.M;
   const int lane = threadIdx.x & 31;
   float v[32];
   if constexpr (EPI == EPI_BIAS || EPI == EPI_BIAS_GELU || EPI == EPI_KV) {
     __nv_bfloat16* out = nullptr;
-    if (valid) {
-      long long orow = row;
-      long long ocol = n0 + c0;
-      if constexpr (EPI == EPI_KV) {
-        const int r = find_seg_gen(seg_off, e.n_seg, row);
+    // bulk-store coordinates of this warp's 32 rows: plain outputs are a
+    // [M, N] tensor (rows past M are dropped by the store); the cache is a
+    // [blocks * cap_total, d] tensor and takes the bulk path only when all 32
+    // rows are valid and belong to one request (consecutive cache rows)
+    bool tma_ok = true;
+    int tx = n0 + c0, ty = row - lane;
+    long long orow = row;
+    long long ocol = n0 + c0;
+    int r = 0;
+    if constexpr (EPI == EPI_KV) {
+      const int blk = n0 / e.col_blk;
+      if (valid) {
+        r = find_seg_gen(seg_off, e.n_seg, row);
         orow = static_cast<long long>(dst_row0[r]) + (row - seg_off[r]);
-        const int blk = n0 / e.col_blk;
-        ocol = static_cast<long long>(blk) * e.col_blk_stride + (n0 - blk * e.col_blk) + c0;
       }
-      out = static_cast<__nv_bfloat16*>(e.out) + orow * e.ldo + ocol;
+      ocol = static_cast<long long>(blk) * e.col_blk_stride + (n0 - blk * e.col_blk) + c0;
+      // lane 0 holds the warp's first row: if it is invalid, so are all
+      const int r_first = __shfl_sync(0xffffffffu, r, 0);
+      const long long y0 = static_cast<long long>(blk) * (e.col_blk_stride / e.col_blk) + orow;
+      tx = (n0 - blk * e.col_blk) + c0;
+      ty = static_cast<int>(__shfl_sync(0xffffffffu, y0, 0));
+      tma_ok = valid && r == r_first;
     }
+    if (valid) out = static_cast<__nv_bfloat16*>(e.out) + orow * e.ldo + ocol;
+    tma_ok = __all_sync(0xffffffffu, tma_ok);
 #pragma unroll 1
     for (int c = 0; c < HALF; c += 32) {
       tmem_ld32(tacc + c0 + c, v);
-      if (valid) {
-        float b[32];
-        load_f32x32_gen(bias + n0 + c0 + c, b);
+      float b[32];
+      load_f32x32_gen(bias + n0 + c0 + c, b);
 #pragma unroll
-        for (int i = 0; i < 32; ++i) {
-          float x = v[i] + b[i];
-          if constexpr (EPI == EPI_BIAS_GELU) x = gelu_erf(x);
-          v[i] = x;
-        }
-        store_bf16x32(out + c, v);
+      for (int i = 0; i < 32; ++i) {
+        float x = v[i] + b[i];
+        if constexpr (EPI == EPI_BIAS_GELU) x = gelu_erf(x);
+        v[i] = x;
       }
+      store_chunk(v, out + c, valid, tma_ok, tmO, tx + c, ty, stage, kchunk++, lane);
     }
   } else {
     // Row LayerNorm over the full row (BN == N): two passes over TMEM, the
@@ -310,6 +371,7 @@ __device__ __forceinline__ void epilogue(const EpiArgs& e, uint32_t tacc, int ro
     if constexpr (EPI == EPI_LN) {
       if (valid) out = static_cast<__nv_bfloat16*>(e.out) + row * e.ldo + c0;
     }
+    const int ty = row - lane;
 #pragma unroll 1
     for (int c = 0; c < HALF; c += 32) {
       tmem_ld32(tacc + c0 + c, v);
@@ -319,7 +381,7 @@ __device__ __forceinline__ void epilogue(const EpiArgs& e, uint32_t tacc, int ro
 #pragma unroll
       for (int i = 0; i < 32; ++i) v[i] = (v[i] - mean) * rstd * g[i] + bt[i];
       if constexpr (EPI == EPI_LN) {
-        if (valid) store_bf16x32(out + c, v);
+        store_chunk(v, out + c, valid, true, tmO, c0 + c, ty, stage, kchunk++, lane);
       } else {
         // head: z . W_eff_z, weights zero-padded to NAP actions in shared memory
         const float4* w4 = reinterpret_cast<const float4*>(s_weff + (c0 + c) * NAP);
@@ -380,18 +442,23 @@ struct Shape {
   static constexpr bool LN = EPI == EPI_LN || EPI == EPI_LN_HEAD;
   static constexpr int RED_BYTES = LN ? 2 * 128 * kRedStride * 4 : 0;
   static constexpr int WEFF_BYTES = EPI == EPI_LN_HEAD ? BN * NAP * 4 : 0;
-  // bias [kStageN] floats, then (cache-row remap) offsets and first rows; the
-  // mbarriers after this region need 8-byte alignment, so round to 16 bytes
+  // bias [kStageN] floats, then (cache-row remap) offsets and first rows;
+  // rounded to 1 KB so that the staging buffers after it start on a
+  // swizzle-atom boundary
   static constexpr int AUX_BYTES =
-      LN ? 0 : ((kStageN * 4 + (EPI == EPI_KV ? (2 * kStageSeg + 1) * 4 : 0) + 15) / 16) * 16;
-  static constexpr int EXTRA = RED_BYTES + WEFF_BYTES + AUX_BYTES + 1024 + 256;
+      LN ? 0 : ((kStageN * 4 + (EPI == EPI_KV ? (2 * kStageSeg + 1) * 4 : 0) + 1023) / 1024) * 1024;
+  // bulk-store staging: two 2 KB buffers per epilogue warp (bf16 outputs)
+  static constexpr int STG_BYTES = EPI == EPI_LN_HEAD ? 0 : kEpiWarps * 2 * 2048;
+  static constexpr int EXTRA = RED_BYTES + WEFF_BYTES + AUX_BYTES + STG_BYTES + 1024 + 256;
   static constexpr int STAGES_FIT = (227 * 1024 - EXTRA) / STAGE_BYTES;
   static constexpr int STAGES = STAGES_FIT > 8 ? 8 : STAGES_FIT;
   static constexpr int ACC_BUFS = BN <= 256 ? 2 : 1;      // TMEM double buffer
   static constexpr int TMEM_COLS = BN * ACC_BUFS < 32 ? 32 : BN * ACC_BUFS;
   static constexpr int SMEM_BYTES = STAGES * STAGE_BYTES + EXTRA;
   static_assert(STAGES >= 2, "pipeline depth");
-  static_assert((RED_BYTES + WEFF_BYTES + AUX_BYTES) % 16 == 0, "mbarriers must stay 8-byte aligned");
+  static_assert((RED_BYTES + WEFF_BYTES + AUX_BYTES) % 1024 == 0 || STG_BYTES == 0,
+                "staging buffers need 512-byte alignment (64-byte swizzle atoms)");
+  static_assert((RED_BYTES + WEFF_BYTES + AUX_BYTES + STG_BYTES) % 16 == 0, "mbarriers must stay 8-byte aligned");
   static_assert(SMEM_BYTES <= 232448, "shared memory");
   static_assert((TMEM_COLS & (TMEM_COLS - 1)) == 0 && TMEM_COLS <= 512, "TMEM columns");
 };
@@ -404,7 +471,7 @@ struct Shape {
 template <int BN, int EPI, int NAP>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
-                   const EpiArgs e) {
+                   const __grid_constant__ CUtensorMap tmO, const EpiArgs e) {
   using S = Shape<BN, EPI, NAP>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -415,7 +482,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   float* s_bias = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(s_weff) + S::WEFF_BYTES);
   int* s_seg = reinterpret_cast<int*>(s_bias + kStageN);
   int* s_dst = s_seg + kStageSeg + 1;
-  uint64_t* full = reinterpret_cast<uint64_t*>(reinterpret_cast<uint8_t*>(s_bias) + S::AUX_BYTES);
+  uint8_t* s_stage = reinterpret_cast<uint8_t*>(s_bias) + S::AUX_BYTES;
+  uint64_t* full = reinterpret_cast<uint64_t*>(s_stage + S::STG_BYTES);
   uint64_t* empty = full + S::STAGES;
   uint64_t* acc_full = empty + S::STAGES;
   uint64_t* acc_empty = acc_full + 2;
@@ -544,6 +612,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     const int ew = warp - 2;
     const int q = warp & 3;           // TMEM lane quarter this warp may access
     const int h = ew / 4;             // column half
+    uint8_t* stage = s_stage + ew * 4096;
+    int kchunk = 0;
     int i = 0;
     for (int t = blockIdx.x; t < num_tiles; t += gridDim.x, ++i) {
       const int buf = i % S::ACC_BUFS;
@@ -558,11 +628,12 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       tc_fence_after();
       const int m0 = (t / n_tiles) * BM, n0 = (t % n_tiles) * BN;
       epilogue<BN, EPI, NAP>(e, tmem + buf * BN + (static_cast<uint32_t>(q * 32) << 16), m0 + q * 32 + lane, n0,
-                             h * (BN / 2), q, h, red, s_weff, bias, seg_off, dst_row0);
+                             h * (BN / 2), q, h, red, s_weff, bias, seg_off, dst_row0, &tmO, stage, kchunk);
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(acc_empty + buf);
     }
+    if (lane == 0) bulk_wait_all();   // this warp's bulk stores are complete before exit
   }
   tc_fence_before();
   __syncthreads();
@@ -608,6 +679,20 @@ static bool make_tmap(CUtensorMap* tm, const void* base, long long rows, long lo
   return r == CUDA_SUCCESS;
 }
 
+// Output map for bulk stores: bf16 [rows, cols] with leading dimension ld,
+// box {32 columns, 32 rows}, 64-byte swizzle.
+static bool make_tmap_out(CUtensorMap* tm, const void* base, long long rows, long long cols, long long ld) {
+  EncodeTiledFn fn = encode_fn();
+  if (!fn || (reinterpret_cast<uintptr_t>(base) & 15) || (ld * 2) % 16) return false;
+  cuuint64_t dims[2] = {static_cast<cuuint64_t>(cols), static_cast<cuuint64_t>(rows)};
+  cuuint64_t strides[1] = {static_cast<cuuint64_t>(ld) * 2};
+  cuuint32_t box[2] = {32, 32};
+  cuuint32_t estr[2] = {1, 1};
+  return fn(tm, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_64B, CU_TENSOR_MAP_L2_PROMOTION_NONE,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 static int num_sms() {
   static int n = 0;
   if (!n) {
@@ -629,13 +714,23 @@ static cudaError_t launch_bn(const __nv_bfloat16* A, long long lda, const __nv_b
     if (err != cudaSuccess) return err;
     attr_set = true;
   }
-  CUtensorMap ta, tb;
+  CUtensorMap ta, tb, to;
   if (!make_tmap(&ta, A, e.M, e.K, lda, BM)) return cudaErrorInvalidValue;
   if (!make_tmap(&tb, B, e.N, e.K, e.K, Sh::B_BOX)) return cudaErrorInvalidValue;
+  if (EPI == EPI_LN_HEAD) {
+    to = ta;   // unused
+  } else if (EPI == EPI_KV) {
+    // the cache viewed as [(N / col_blk) * cap_total rows, col_blk] bf16
+    const long long rows = static_cast<long long>(e.N / e.col_blk) * (e.col_blk_stride / e.col_blk);
+    if (!make_tmap_out(&to, e.out, rows, e.col_blk, e.ldo)) return cudaErrorInvalidValue;
+  } else {
+    if (!make_tmap_out(&to, e.out, e.M, e.N, e.ldo)) return cudaErrorInvalidValue;
+  }
   const long long tiles = static_cast<long long>((e.M + BM - 1) / BM) * (e.N / BN);
   const int grid = static_cast<int>(tiles < num_sms() ? tiles : num_sms());
   prof_begin(cls, s);
-  cudaError_t err = launch_pdl(gemm_tc_kernel<BN, EPI, NAP>, dim3(grid), dim3(NUM_THREADS), Sh::SMEM_BYTES, s, ta, tb, e);
+  cudaError_t err =
+      launch_pdl(gemm_tc_kernel<BN, EPI, NAP>, dim3(grid), dim3(NUM_THREADS), Sh::SMEM_BYTES, s, ta, tb, to, e);
   prof_end(cls, s);
   return err;
 }
