@@ -82,27 +82,45 @@ __global__ void __launch_bounds__(256) pool_partial_kernel(const T* __restrict__
         }
       }
     }
+    // the batch's logits first (independent reductions), then one rescale
+    float z[RB];
 #pragma unroll
     for (int t = 0; t < RB; ++t) {
-      if (warp + kPoolWarps * (t0 + t) >= nrows) break;
       float dot = 0.f;
 #pragma unroll
       for (int j = 0; j < MAXC; ++j)
 #pragma unroll
         for (int q = 0; q < VEC; ++q) dot = fmaf(v[t][j][q], w[j][q], dot);
-#pragma unroll
-      for (int o = 16; o > 0; o >>= 1) dot += __shfl_xor_sync(0xffffffffu, dot, o);
-      const float z = dot * inv_sqrt_d;
-      const float mn = fmaxf(m, z);
-      const float corr = expf(m - mn);
-      const float e = expf(z - mn);
-      s = s * corr + e;
-#pragma unroll
-      for (int j = 0; j < MAXC; ++j)
-#pragma unroll
-        for (int q = 0; q < VEC; ++q) acc[j][q] = fmaf(acc[j][q], corr, e * v[t][j][q]);
-      m = mn;
+      z[t] = dot;
     }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1)
+#pragma unroll
+      for (int t = 0; t < RB; ++t) z[t] += __shfl_xor_sync(0xffffffffu, z[t], o);
+    float mb = m;
+#pragma unroll
+    for (int t = 0; t < RB; ++t) {
+      z[t] *= inv_sqrt_d;
+      if (warp + kPoolWarps * (t0 + t) < nrows) mb = fmaxf(mb, z[t]);
+    }
+    const float corr = mb == -INFINITY ? 1.f : expf(m - mb);   // no valid row yet: nothing to rescale
+    s *= corr;
+#pragma unroll
+    for (int j = 0; j < MAXC; ++j)
+#pragma unroll
+      for (int q = 0; q < VEC; ++q) acc[j][q] *= corr;
+#pragma unroll
+    for (int t = 0; t < RB; ++t) {
+      if (warp + kPoolWarps * (t0 + t) < nrows) {
+        const float e = expf(z[t] - mb);
+        s += e;
+#pragma unroll
+        for (int j = 0; j < MAXC; ++j)
+#pragma unroll
+          for (int q = 0; q < VEC; ++q) acc[j][q] = fmaf(e, v[t][j][q], acc[j][q]);
+      }
+    }
+    m = mb;
   }
 #pragma unroll
   for (int j = 0; j < MAXC; ++j) {
@@ -147,21 +165,27 @@ __global__ void __launch_bounds__(256) pool_partial_kernel(const T* __restrict__
   if (!is_last) return;
   __threadfence();
   const float* pr = part + static_cast<long long>(r) * max_chunks * (d + 2);
+  __shared__ float ch_scale[512];
   const float old_m = merge_existing ? st_m[r] : -INFINITY;
   const float old_s = merge_existing ? st_s[r] : 0.f;
   float Mr = old_m;
   for (int ch = 0; ch < nch_r; ++ch) Mr = fmaxf(Mr, __ldcg(pr + static_cast<long long>(ch) * (d + 2)));
   const float w_old = merge_existing ? expf(old_m - Mr) : 0.f;
+  for (int ch = tid; ch < nch_r && ch < 512; ch += 256)
+    ch_scale[ch] = expf(__ldcg(pr + static_cast<long long>(ch) * (d + 2)) - Mr);
+  __syncthreads();
   float Sr = old_s * w_old;
   for (int ch = 0; ch < nch_r; ++ch) {
     const float* pc = pr + static_cast<long long>(ch) * (d + 2);
-    Sr += __ldcg(pc + 1) * expf(__ldcg(pc) - Mr);
+    const float sc = ch < 512 ? ch_scale[ch] : expf(__ldcg(pc) - Mr);
+    Sr += __ldcg(pc + 1) * sc;
   }
   for (int k = tid; k < d; k += 256) {
     float a = merge_existing ? st_acc[static_cast<long long>(r) * d + k] * w_old : 0.f;
     for (int ch = 0; ch < nch_r; ++ch) {
       const float* pc = pr + static_cast<long long>(ch) * (d + 2);
-      a = fmaf(__ldcg(pc + 2 + k), expf(__ldcg(pc) - Mr), a);
+      const float sc = ch < 512 ? ch_scale[ch] : expf(__ldcg(pc) - Mr);
+      a = fmaf(__ldcg(pc + 2 + k), sc, a);
     }
     st_acc[static_cast<long long>(r) * d + k] = a;
     g[static_cast<long long>(r) * d + k] = a / Sr;
