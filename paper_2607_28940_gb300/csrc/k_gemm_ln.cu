@@ -1,0 +1,385 @@
+// Projections followed by residual + LayerNorm (and, for the last layer, the
+// action head), with the row split across a thread-block cluster.
+//
+// Out = LN(A W + b + residual) needs whole rows (Sec. 4.1.2 crossAttend
+// equation, post-LN).  A 128 x d tile computed by one CTA leaves most SMs idle
+// when there are few rows, so here a cluster of CS = d / 128 CTAs shares each
+// 128-row tile: CTA k computes columns [128 k, 128 k + 128) (tcgen05, TMEM
+// double buffer, persistent over the cluster's row tiles) and the row
+// statistics are combined across the cluster through distributed shared
+// memory: every epilogue warp publishes the mean and the sum of squared
+// deviations of its 64 columns to all CTAs of the cluster, and each row merges
+// the 2 CS partial results (pairwise-update formula for equal counts).  With
+// the head, each CTA's partial logits z . W_eff_z go to rank 0, which adds the
+// x part, applies the softmax and writes logits and probabilities
+// (Sec. 4.1.3 action-decoding equation).
+#include "tc_ptx.cuh"
+
+namespace txs {
+namespace tcln {
+
+using namespace tc;
+
+constexpr int BN = 128;                 // columns per CTA
+constexpr int kWarps = 8;               // epilogue warps: two per TMEM lane quarter
+constexpr int NUM_THREADS = 64 + 32 * kWarps;
+
+template <int CS, bool HEAD>
+struct LnShape {
+  static constexpr int NAP = 4;                                    // head actions padded to 4
+  static constexpr int P = 2 * CS;                                 // partials per row
+  static constexpr int B_STAGE_BYTES = BN * BK * 2;                // 16 KB
+  static constexpr int STAGE_BYTES = A_STAGE_BYTES + B_STAGE_BYTES;
+  static constexpr int STG_BYTES = HEAD ? 0 : kWarps * 2 * 2048;   // bulk-store staging
+  static constexpr int XBUF_BYTES = 2 * P * 128 * 8;               // (mean, M2), two parities
+  static constexpr int HBUF_BYTES = HEAD ? 2 * P * 128 * NAP * 4 : 0;
+  static constexpr int WEFF_BYTES = HEAD ? BN * NAP * 4 : 0;
+  static constexpr int EXTRA = STG_BYTES + XBUF_BYTES + HBUF_BYTES + WEFF_BYTES + 1024 + 512;
+  static constexpr int STAGES_FIT = (227 * 1024 - EXTRA) / STAGE_BYTES;
+  static constexpr int STAGES = STAGES_FIT > 6 ? 6 : STAGES_FIT;
+  static constexpr int SMEM_BYTES = STAGES * STAGE_BYTES + EXTRA;
+  static constexpr int TMEM_COLS = 2 * BN;
+  static_assert(STAGES >= 2 && SMEM_BYTES <= 232448, "shared memory");
+};
+
+template <int CS, bool HEAD>
+__global__ void __launch_bounds__(NUM_THREADS, 1)
+    gemm_ln_cluster_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                           const __grid_constant__ CUtensorMap tmO, const EpiArgs e) {
+  using S = LnShape<CS, HEAD>;
+  constexpr int NAP = S::NAP, P = S::P;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint8_t* sA = smem;
+  uint8_t* sB = sA + S::STAGES * A_STAGE_BYTES;
+  uint8_t* s_stage = sB + S::STAGES * S::B_STAGE_BYTES;
+  float2* xbuf = reinterpret_cast<float2*>(s_stage + S::STG_BYTES);                 // [2][P][128]
+  float* hbuf = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(xbuf) + S::XBUF_BYTES);  // [2][P][128][NAP]
+  float* s_weff = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(hbuf) + S::HBUF_BYTES);
+  uint64_t* full = reinterpret_cast<uint64_t*>(reinterpret_cast<uint8_t*>(s_weff) + S::WEFF_BYTES);
+  uint64_t* empty = full + S::STAGES;
+  uint64_t* acc_full = empty + S::STAGES;
+  uint64_t* acc_empty = acc_full + 2;
+  uint64_t* xfull = acc_empty + 2;    // [2][4]: statistics of lane quarter q have arrived
+  uint64_t* hfull = xfull + 8;        // [2][4]: head partials have arrived (rank 0)
+  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(hfull + 8);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_holder + 1);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint32_t rk = cluster_rank();
+  const int cid = blockIdx.x / CS, ncl = gridDim.x / CS;
+  const int m_tiles = (e.M + BM - 1) / BM;
+  const int my_tiles = m_tiles > cid ? (m_tiles - 1 - cid) / ncl + 1 : 0;   // equal within a cluster
+  const int n0 = static_cast<int>(rk) * BN;
+  const int num_kb = e.K / BK;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < S::STAGES; ++s) {
+      mbar_init(full + s, 1);
+      mbar_init(empty + s, 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(acc_full + b, 1);
+      mbar_init(acc_empty + b, kWarps);
+    }
+    for (int i = 0; i < 8; ++i) {
+      mbar_init(xfull + i, P * 32);
+      mbar_init(hfull + i, P * 32);
+    }
+    *abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == 1) tmem_alloc(tmem_holder, S::TMEM_COLS);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_holder;
+  cluster_sync();                     // every CTA's barriers exist before any peer arrives
+  pdl_launch_dependents();
+  pdl_wait();
+  if constexpr (HEAD) {
+    for (int i = threadIdx.x; i < BN * NAP; i += NUM_THREADS) {
+      const int c = i / NAP, a = i - c * NAP;
+      s_weff[i] = a < e.n_act ? e.weff_z[static_cast<long long>(n0 + c) * e.n_act + a] : 0.f;
+    }
+    __syncthreads();
+  }
+
+  if (warp == 0) {
+    if (lane == 0) {
+      asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmA)) : "memory");
+      asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmB)) : "memory");
+      int it = 0;
+      bool ok = true;
+      for (int i = 0; i < my_tiles && ok; ++i) {
+        const int m0 = (cid + i * ncl) * BM;
+        for (int kb = 0; kb < num_kb; ++kb, ++it) {
+          const int s = it % S::STAGES;
+          if (!mbar_wait(empty + s, ((it / S::STAGES) & 1) ^ 1, abort_flag)) {
+            ok = false;
+            break;
+          }
+          mbar_expect_tx(full + s, S::STAGE_BYTES);
+          tma_load_2d(sA + s * A_STAGE_BYTES, &tmA, full + s, kb * BK, m0);
+          tma_load_2d(sB + s * S::B_STAGE_BYTES, &tmB, full + s, kb * BK, n0);
+        }
+      }
+      if (*abort_flag)
+        for (int k = it > S::STAGES ? it - S::STAGES : 0; k < it; ++k)
+          mbar_wait_plain(full + k % S::STAGES, (k / S::STAGES) & 1);
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      constexpr uint32_t idesc = idesc_bf16(BM, BN);
+      int it = 0;
+      bool ok = true;
+      for (int i = 0; i < my_tiles && ok; ++i) {
+        const int buf = i & 1;
+        if (!mbar_wait(acc_empty + buf, ((i >> 1) & 1) ^ 1, abort_flag)) break;
+        tc_fence_after();
+        for (int kb = 0; kb < num_kb; ++kb, ++it) {
+          const int s = it % S::STAGES;
+          if (!mbar_wait(full + s, (it / S::STAGES) & 1, abort_flag)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint64_t adesc = sdesc_sw128(smem_u32(sA + s * A_STAGE_BYTES));
+          const uint64_t bdesc = sdesc_sw128(smem_u32(sB + s * S::B_STAGE_BYTES));
+#pragma unroll
+          for (int k = 0; k < BK / 16; ++k)
+            mma_bf16(tmem + buf * BN, adesc + 2 * k, bdesc + 2 * k, idesc, (kb > 0 || k > 0) ? 1u : 0u);
+          mma_commit(empty + s);
+        }
+        mma_commit(acc_full + buf);
+      }
+    }
+  } else {
+    const int ew = warp - 2;
+    const int q = warp & 3;            // TMEM lane quarter
+    const int h = ew / 4;              // 64-column half of this CTA's slice
+    const int c0 = h * 64;
+    const int slot = static_cast<int>(rk) * 2 + h;
+    const int trow = q * 32 + lane;
+    uint8_t* stage = s_stage + ew * 4096;
+    int kchunk = 0;
+    float v[32];
+    for (int i = 0; i < my_tiles; ++i) {
+      const int buf = i & 1, pb = i & 1;
+      const uint32_t use = static_cast<uint32_t>(i >> 1) & 1;
+      bool go = mbar_wait(acc_full + buf, use, abort_flag);
+      go = __shfl_sync(0xffffffffu, go ? 1 : 0, 0) != 0;
+      if (!go) break;
+      tc_fence_after();
+      const int m0 = (cid + i * ncl) * BM;
+      const int row = m0 + trow;
+      const bool valid = row < e.M;
+      const uint32_t tacc = tmem + buf * BN + (static_cast<uint32_t>(q * 32) << 16) + c0;
+      const __nv_bfloat16* res = valid ? static_cast<const __nv_bfloat16*>(e.res) + row * e.ldr + n0 + c0 : nullptr;
+      // pass 1: v = acc + bias + residual, written back to TMEM
+      float sum = 0.f;
+#pragma unroll
+      for (int c = 0; c < 64; c += 32) {
+        tmem_ld32(tacc + c, v);
+        float b[32], r[32];
+        load_f32x32(e.bias + n0 + c0 + c, b);
+        if (valid) load_bf16x32(res + c, r);
+        else {
+#pragma unroll
+          for (int k = 0; k < 32; ++k) r[k] = 0.f;
+        }
+#pragma unroll
+        for (int k = 0; k < 32; ++k) {
+          v[k] += b[k] + r[k];
+          sum += v[k];
+        }
+        tmem_st32(tacc + c, v);
+      }
+      const float mean_p = sum * (1.f / 64.f);
+      float m2 = 0.f;
+#pragma unroll
+      for (int c = 0; c < 64; c += 32) {
+        tmem_ld32(tacc + c, v);
+#pragma unroll
+        for (int k = 0; k < 32; ++k) {
+          const float t = v[k] - mean_p;
+          m2 = fmaf(t, t, m2);
+        }
+      }
+      // publish (mean, M2) of these 64 columns to every CTA of the cluster
+      {
+        float2* mine = xbuf + (pb * P + slot) * 128 + trow;
+#pragma unroll
+        for (int pr = 0; pr < CS; ++pr) {
+          st_peer_f32x2(map_peer(mine, pr), mean_p, m2);
+          mbar_arrive_peer(map_peer(xfull + pb * 4 + q, pr));
+        }
+      }
+      bool ok = mbar_wait_cluster(xfull + pb * 4 + q, use, abort_flag);
+      ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
+      if (!ok) break;
+      float mp[P];
+      float mean = 0.f;
+#pragma unroll
+      for (int p = 0; p < P; ++p) {
+        const float2 x = xbuf[(pb * P + p) * 128 + trow];
+        mp[p] = x.x;
+        mean += x.x;
+        m2 = p == 0 ? x.y : m2 + x.y;
+      }
+      mean *= 1.f / P;
+#pragma unroll
+      for (int p = 0; p < P; ++p) {
+        const float t = mp[p] - mean;
+        m2 = fmaf(64.f * t, t, m2);
+      }
+      const float rstd = rsqrtf(m2 / static_cast<float>(BN * CS) + e.ln_eps);
+      // pass 3: normalise; store, or the head's partial logits
+      float lg[NAP];
+#pragma unroll
+      for (int a = 0; a < NAP; ++a) lg[a] = 0.f;
+#pragma unroll
+      for (int c = 0; c < 64; c += 32) {
+        tmem_ld32(tacc + c, v);
+        float g[32], bt[32];
+        load_f32x32(e.gamma + n0 + c0 + c, g);
+        load_f32x32(e.beta + n0 + c0 + c, bt);
+#pragma unroll
+        for (int k = 0; k < 32; ++k) v[k] = (v[k] - mean) * rstd * g[k] + bt[k];
+        if constexpr (!HEAD) {
+          __nv_bfloat16* out = valid ? static_cast<__nv_bfloat16*>(e.out) + row * e.ldo + n0 + c0 + c : nullptr;
+          store_chunk(v, out, valid, true, &tmO, n0 + c0 + c, m0 + q * 32, stage, kchunk++, lane);
+        } else {
+          const float4* w4 = reinterpret_cast<const float4*>(s_weff + (c0 + c) * NAP);
+#pragma unroll
+          for (int k = 0; k < 32; ++k) {
+            const float4 w = w4[k];
+            lg[0] = fmaf(v[k], w.x, lg[0]);
+            lg[1] = fmaf(v[k], w.y, lg[1]);
+            lg[2] = fmaf(v[k], w.z, lg[2]);
+            lg[3] = fmaf(v[k], w.w, lg[3]);
+          }
+        }
+      }
+      if constexpr (HEAD) {
+        // partial logits of these 64 columns -> rank 0
+        float* mine = hbuf + ((pb * P + slot) * 128 + trow) * NAP;
+        st_peer_f32x4(map_peer(mine, 0), lg[0], lg[1], lg[2], lg[3]);
+        mbar_arrive_peer(map_peer(hfull + pb * 4 + q, 0));
+        if (rk == 0 && h == 0) {
+          ok = mbar_wait_cluster(hfull + pb * 4 + q, use, abort_flag);
+          ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
+          if (!ok) break;
+          if (valid && row < e.n_cand_rows) {
+            const int na = e.n_act;
+            float t[NAP];
+#pragma unroll
+            for (int a = 0; a < NAP; ++a) t[a] = 0.f;
+#pragma unroll
+            for (int p = 0; p < P; ++p) {
+              const float4 x = *reinterpret_cast<const float4*>(hbuf + ((pb * P + p) * 128 + trow) * NAP);
+              t[0] += x.x; t[1] += x.y; t[2] += x.z; t[3] += x.w;
+            }
+            float mx = -INFINITY;
+#pragma unroll
+            for (int a = 0; a < NAP; ++a)
+              if (a < na) {
+                t[a] += __ldg(e.xlog + static_cast<long long>(row) * na + a);
+                mx = fmaxf(mx, t[a]);
+              }
+            float ssum = 0.f, pe[NAP];
+#pragma unroll
+            for (int a = 0; a < NAP; ++a) {
+              pe[a] = a < na ? expf(t[a] - mx) : 0.f;
+              ssum += pe[a];
+            }
+            const float inv = 1.f / ssum;
+#pragma unroll
+            for (int a = 0; a < NAP; ++a)
+              if (a < na) {
+                e.logits[static_cast<long long>(row) * na + a] = t[a];
+                if (e.probs) e.probs[static_cast<long long>(row) * na + a] = pe[a] * inv;
+              }
+          }
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(acc_empty + buf);
+    }
+    if (lane == 0) bulk_wait_all();
+  }
+  tc_fence_before();
+  __syncthreads();
+  cluster_sync();                     // no CTA leaves while a peer may still write into it
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, S::TMEM_COLS);
+  }
+  if (threadIdx.x == 0 && *abort_flag) latch_status(e.status, TXS_ERR_DEVICE_TIMEOUT);
+}
+
+template <int CS, bool HEAD>
+static cudaError_t launch_cs(const __nv_bfloat16* A, long long lda, const __nv_bfloat16* B, const EpiArgs& e,
+                             cudaStream_t s, int cls) {
+  using Sh = LnShape<CS, HEAD>;
+  auto kern = gemm_ln_cluster_kernel<CS, HEAD>;
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = CS;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
+  cudaLaunchConfig_t cfg = {};
+  cfg.blockDim = dim3(NUM_THREADS);
+  cfg.dynamicSmemBytes = Sh::SMEM_BYTES;
+  cfg.stream = s;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  // clusters that can be resident at once (one CTA per SM)
+  static int max_clusters = 0;
+  if (!max_clusters) {
+    cudaError_t err = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, Sh::SMEM_BYTES);
+    if (err != cudaSuccess) return err;
+    cfg.gridDim = dim3((num_sms() / CS) * CS);
+    int n = 0;
+    if (cudaOccupancyMaxActiveClusters(&n, kern, &cfg) != cudaSuccess || n <= 0) {
+      (void)cudaGetLastError();
+      n = num_sms() / CS;
+    }
+    max_clusters = n;
+  }
+  CUtensorMap ta, tb, to;
+  if (!make_tmap(&ta, A, e.M, e.K, lda, BM)) return cudaErrorInvalidValue;
+  if (!make_tmap(&tb, B, e.N, e.K, e.K, BN)) return cudaErrorInvalidValue;
+  if (HEAD) to = ta;   // unused
+  else if (!make_tmap_out(&to, e.out, e.M, e.N, e.ldo)) return cudaErrorInvalidValue;
+  const int m_tiles = (e.M + BM - 1) / BM;
+  const int ncl = m_tiles < max_clusters ? m_tiles : max_clusters;
+  cfg.gridDim = dim3(ncl * CS);
+  cfg.numAttrs = 2;
+  prof_begin(cls, s);
+  cudaError_t err = cudaLaunchKernelEx(&cfg, kern, ta, tb, to, e);
+  prof_end(cls, s);
+  return err;
+}
+
+}  // namespace tcln
+
+namespace tc {
+
+cudaError_t launch_gemm_ln_cluster(const __nv_bfloat16* A, long long lda, const __nv_bfloat16* B, const EpiArgs& e,
+                                   cudaStream_t s, int cls) {
+  if (e.epi == EPI_LN_HEAD && (e.n_act < 1 || e.n_act > 4)) return cudaErrorNotSupported;
+  if (e.epi != EPI_LN && e.epi != EPI_LN_HEAD) return cudaErrorNotSupported;
+  const bool head = e.epi == EPI_LN_HEAD;
+  switch (e.N) {
+    case 256: return head ? tcln::launch_cs<2, true>(A, lda, B, e, s, cls) : tcln::launch_cs<2, false>(A, lda, B, e, s, cls);
+    case 512: return head ? tcln::launch_cs<4, true>(A, lda, B, e, s, cls) : tcln::launch_cs<4, false>(A, lda, B, e, s, cls);
+    default: return cudaErrorNotSupported;
+  }
+}
+
+}  // namespace tc
+}  // namespace txs
