@@ -9,11 +9,17 @@
 //   warp 0     TMA producer: K_j, V_j tiles of the request (head h columns)
 //              into a STG-deep shared-memory ring;
 //   warp 1     MMA issuer: S_j = Q K_j^T into one of two TMEM buffers, then
-//              O_j = P_j V_j into a TMEM tile (V used MN-major: no transpose);
+//              O += P_j V_j into the TMEM output tile (V used MN-major: no
+//              transpose);
 //   warps 2-5  softmax: one query row per thread straight out of TMEM (row
-//              max, exp2, row sum need no shuffles), P_j written to shared
-//              memory in the 128-byte-swizzled layout the MMA reads, and the
-//              running output O = O * exp(m_old - m_new) + O_j kept in registers.
+//              max, exp2, row sum need no shuffles); P_j goes to one of two
+//              shared-memory buffers in the 128-byte-swizzled layout the MMA
+//              reads, so the exponentials of tile j overlap the PV product of
+//              tile j - 1.
+// The running maximum is raised only when a tile's maximum exceeds it by more
+// than 2^8 (then O and the row sum are rescaled in place); otherwise the
+// stale maximum is kept, P stays below 256 and no rescale is needed.  Exact
+// softmax is recovered at the end from O / l either way.
 // All waits are bounded; a timeout latches TXS_ERR_DEVICE_TIMEOUT.
 #include <algorithm>
 
@@ -26,6 +32,7 @@ constexpr int BQ = 128;            // queries per CTA (TMEM lanes)
 constexpr int BKV = 128;           // keys per K/V tile
 constexpr int STG = 3;             // K/V ring depth
 constexpr int NUM_THREADS = 192;   // producer, MMA, 4 softmax warps
+constexpr float kRescaleLog2 = 8.f;  // raise the running max only past this (log2 units)
 
 // ------------------------------------------------------------------ PTX wrappers
 
@@ -46,10 +53,10 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
   uint32_t ok;
   asm volatile(
       "{\n\t.reg .pred p;\n\t"
-      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
       "selp.u32 %0, 1, 0, p;\n\t}"
       : "=r"(ok)
-      : "r"(smem_u32(bar)), "r"(parity)
+      : "r"(smem_u32(bar)), "r"(parity), "r"(1000000u)   // suspend up to 1 ms per try
       : "memory");
   return ok != 0;
 }
@@ -118,6 +125,26 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float* v) {
   for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
 }
 
+__device__ __forceinline__ void tmem_st32(uint32_t taddr, const float* v) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], "
+      "{%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,"
+      "%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,%32};\n\t"
+      "tcgen05.wait::st.sync.aligned;" ::"r"(taddr),
+      "r"(__float_as_uint(v[0])), "r"(__float_as_uint(v[1])), "r"(__float_as_uint(v[2])),
+      "r"(__float_as_uint(v[3])), "r"(__float_as_uint(v[4])), "r"(__float_as_uint(v[5])),
+      "r"(__float_as_uint(v[6])), "r"(__float_as_uint(v[7])), "r"(__float_as_uint(v[8])),
+      "r"(__float_as_uint(v[9])), "r"(__float_as_uint(v[10])), "r"(__float_as_uint(v[11])),
+      "r"(__float_as_uint(v[12])), "r"(__float_as_uint(v[13])), "r"(__float_as_uint(v[14])),
+      "r"(__float_as_uint(v[15])), "r"(__float_as_uint(v[16])), "r"(__float_as_uint(v[17])),
+      "r"(__float_as_uint(v[18])), "r"(__float_as_uint(v[19])), "r"(__float_as_uint(v[20])),
+      "r"(__float_as_uint(v[21])), "r"(__float_as_uint(v[22])), "r"(__float_as_uint(v[23])),
+      "r"(__float_as_uint(v[24])), "r"(__float_as_uint(v[25])), "r"(__float_as_uint(v[26])),
+      "r"(__float_as_uint(v[27])), "r"(__float_as_uint(v[28])), "r"(__float_as_uint(v[29])),
+      "r"(__float_as_uint(v[30])), "r"(__float_as_uint(v[31]))
+      : "memory");
+}
+
 // 2^x on the special-function unit (PTX ex2.approx, flush-to-zero).
 __device__ __forceinline__ float ex2(float x) {
   float y;
@@ -165,8 +192,8 @@ struct FaShape {
   static constexpr int ATOM = 8 * ROW_BYTES;                // 8 rows
   static constexpr int Q_BYTES = BQ * ROW_BYTES;
   static constexpr int KV_BYTES = BKV * ROW_BYTES;
-  static constexpr int P_BYTES = BQ * BKV * 2;              // two 64-key blocks, 128-byte swizzle
-  static constexpr int SMEM = Q_BYTES + P_BYTES + 2 * STG * KV_BYTES + 1024 + 256;
+  static constexpr int P_BYTES = BQ * BKV * 2;              // one P buffer: two 64-key blocks, 128-byte swizzle
+  static constexpr int SMEM = Q_BYTES + 2 * P_BYTES + 2 * STG * KV_BYTES + 1024 + 256;
   static constexpr int TMEM_COLS = 512;                     // S x2 (256) + O tile (DH)
 };
 
@@ -185,19 +212,18 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* sQ = smem;
-  uint8_t* sP = sQ + Sh::Q_BYTES;
-  uint8_t* sK = sP + Sh::P_BYTES;
+  uint8_t* sP = sQ + Sh::Q_BYTES;                      // two P buffers
+  uint8_t* sK = sP + 2 * Sh::P_BYTES;
   uint8_t* sV = sK + STG * Sh::KV_BYTES;
   uint64_t* bars = reinterpret_cast<uint64_t*>(sV + STG * Sh::KV_BYTES);
   uint64_t* kv_full = bars;
   uint64_t* kv_empty = kv_full + STG;
-  uint64_t* s_full = kv_empty + STG;
-  uint64_t* s_free = s_full + 2;
-  uint64_t* q_ready = s_free + 2;
-  uint64_t* p_full = q_ready + 1;
-  uint64_t* o_full = p_full + 1;
-  uint64_t* o_free = o_full + 1;
-  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(o_free + 1);
+  uint64_t* s_full = kv_empty + STG;    // [2] S_j in TMEM buffer j % 2
+  uint64_t* s_free = s_full + 2;        // [2] the softmax warps have read it
+  uint64_t* p_full = s_free + 2;        // [2] P_j in shared buffer j % 2
+  uint64_t* pv_done = p_full + 2;       // [2] O += P_j V_j complete
+  uint64_t* q_ready = pv_done + 2;
+  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(q_ready + 1);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_holder + 1);
 
   pdl_launch_dependents();
@@ -211,6 +237,10 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   const int len = a.kv_len[r];
   const int kv0 = a.kv_off[r];
   const int nkv = (len + BKV - 1) / BKV;
+  if (nkv <= 0) {                                   // a built cache never has an empty request
+    if (threadIdx.x == 0) latch_status(a.status, TXS_ERR_BOUNDS);
+    return;
+  }
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < STG; ++s) {
@@ -220,11 +250,10 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     for (int b = 0; b < 2; ++b) {
       mbar_init(s_full + b, 1);
       mbar_init(s_free + b, 4);
+      mbar_init(p_full + b, 4);
+      mbar_init(pv_done + b, 1);
     }
     mbar_init(q_ready, 4);
-    mbar_init(p_full, 4);
-    mbar_init(o_full, 1);
-    mbar_init(o_free, 4);
     *abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
@@ -260,21 +289,23 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       const uint32_t q_addr = smem_u32(sQ), p_addr = smem_u32(sP);
       bool ok = mbar_wait(q_ready, 0, abort_flag);
       tc_fence_after();
+      // O += P_t V_t, after the softmax warps have written P_t (and rescaled O
+      // if they had to)
       auto pv = [&](int t) -> bool {
-        if (!mbar_wait(p_full, t & 1, abort_flag)) return false;
-        if (!mbar_wait(o_free, (t & 1) ^ 1, abort_flag)) return false;
+        const int bt = t & 1, st = t % STG;
+        if (!mbar_wait(p_full + bt, (t >> 1) & 1, abort_flag)) return false;
         tc_fence_after();
-        const int st = t % STG;
         const uint32_t v_addr = smem_u32(sV + st * Sh::KV_BYTES);
+        const uint32_t pb = p_addr + bt * Sh::P_BYTES;
 #pragma unroll
         for (int k = 0; k < BKV / 16; ++k) {
           // P: 64-key blocks of 16 KB, 32 bytes per 16-key step inside a block
-          const uint64_t pd = sdesc(p_addr + (k / 4) * (BQ * 128) + (k % 4) * 32, 16, 1024, 2);
+          const uint64_t pd = sdesc(pb + (k / 4) * (BQ * 128) + (k % 4) * 32, 16, 1024, 2);
           // V (MN-major): 16 keys = two 8-row atoms of the tile
           const uint64_t vd = sdesc(v_addr + k * 16 * Sh::ROW_BYTES, Sh::ATOM, Sh::ATOM, Sh::SW);
-          mma_bf16(t_o, pd, vd, id_pv, k > 0 ? 1u : 0u);
+          mma_bf16(t_o, pd, vd, id_pv, (t > 0 || k > 0) ? 1u : 0u);
         }
-        mma_commit(o_full);
+        mma_commit(pv_done + bt);
         mma_commit(kv_empty + st);
         return true;
       };
@@ -317,10 +348,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       if (lane == 0) mbar_arrive(q_ready);
     }
     const uint32_t lane_off = static_cast<uint32_t>(qw * 32) << 16;
-    float o[DH];
-#pragma unroll
-    for (int i = 0; i < DH; ++i) o[i] = 0.f;
-    float m_run = -INFINITY, l_run = 0.f, corr_prev = 0.f;
+    float m_run = -INFINITY, l_run = 0.f;     // running max (log2 units, scaled), row sum
     bool ok = true;
     for (int j = 0; j < nkv && ok; ++j) {
       const int b = j & 1;
@@ -328,89 +356,108 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
       if (!ok) break;
       tc_fence_after();
-      const int kbase = j * BKV;
-      const bool full_tile = kbase + BKV <= len;       // no masking needed (uniform)
-      // the whole score row of this tile: one pass over TMEM
+      // the whole score row of this tile in one pass over TMEM; the buffer is
+      // free for S_{j+2} as soon as it is in registers
       float sv[BKV];
 #pragma unroll
       for (int cc = 0; cc < BKV; cc += 32) tmem_ld32(t_s + b * BKV + cc + lane_off, sv + cc);
-      if (!full_tile) {
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(s_free + b);
+      const int kbase = j * BKV;
+      if (kbase + BKV > len) {                   // ragged last tile (uniform)
 #pragma unroll
         for (int i = 0; i < BKV; ++i)
           if (kbase + i >= len) sv[i] = -INFINITY;
       }
-      float mraw = sv[0];
+      // row max in 8 independent chains
+      float mx8[8];
 #pragma unroll
-      for (int i = 1; i < BKV; ++i) mraw = fmaxf(mraw, sv[i]);
-      const float mx = fmaxf(m_run, mraw * a.scale_log2);
-      const float corr = ex2(m_run - mx);
-      // the O tile of the previous K/V tile is complete: fold it in
-      if (j >= 1) {
-        ok = mbar_wait(o_full, (j - 1) & 1, abort_flag);
+      for (int i = 0; i < 8; ++i) mx8[i] = sv[i];
+#pragma unroll
+      for (int i = 8; i < BKV; ++i) mx8[i & 7] = fmaxf(mx8[i & 7], sv[i]);
+#pragma unroll
+      for (int w = 4; w >= 1; w >>= 1)
+#pragma unroll
+        for (int i = 0; i < w; ++i) mx8[i] = fmaxf(mx8[i], mx8[i + w]);
+      const float m_tile = mx8[0] * a.scale_log2;
+      if (__any_sync(0xffffffffu, m_tile > m_run + kRescaleLog2)) {
+        const float m_new = fmaxf(m_run, m_tile);
+        const float alpha = ex2(m_run - m_new);  // 0 on the first tile
+        if (j >= 1) {
+          // O holds P_0..P_{j-1} V: rescale it once PV(j-1) is complete
+          ok = mbar_wait(pv_done + ((j - 1) & 1), ((j - 1) >> 1) & 1, abort_flag);
+          ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
+          if (!ok) break;
+          tc_fence_after();
+#pragma unroll
+          for (int cc = 0; cc < DH; cc += 32) {
+            float ov[32];
+            tmem_ld32(t_o + cc + lane_off, ov);
+#pragma unroll
+            for (int i = 0; i < 32; ++i) ov[i] *= alpha;
+            tmem_st32(t_o + cc + lane_off, ov);
+          }
+        }
+        l_run *= alpha;
+        m_run = m_new;
+      }
+      // P buffer b was last read by PV(j - 2)
+      if (j >= 2) {
+        ok = mbar_wait(pv_done + b, ((j - 2) >> 1) & 1, abort_flag);
         ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
         if (!ok) break;
-        tc_fence_after();
-#pragma unroll
-        for (int cc = 0; cc < DH; cc += 32) {
-          float ov[32];
-          tmem_ld32(t_o + cc + lane_off, ov);
-#pragma unroll
-          for (int i = 0; i < 32; ++i) o[cc + i] = fmaf(o[cc + i], corr_prev, ov[i]);
-        }
-        tc_fence_before();
-        __syncwarp();
-        if (lane == 0) mbar_arrive(o_free);
       }
-      // P = 2^(s * scale - max) into the swizzled P tile (bf16), row sum
-      float psum = 0.f;
+      // P = 2^(s * scale - m_run) into the swizzled P buffer (bf16), row sum
+      uint8_t* pbuf = sP + b * Sh::P_BYTES;
+      float ps8[8];
+#pragma unroll
+      for (int i = 0; i < 8; ++i) ps8[i] = 0.f;
 #pragma unroll
       for (int key16 = 0; key16 < BKV / 8; ++key16) {
         float p[8];
 #pragma unroll
         for (int i = 0; i < 8; ++i) {
-          p[i] = ex2(fmaf(sv[8 * key16 + i], a.scale_log2, -mx));
-          psum += p[i];
+          p[i] = ex2(fmaf(sv[8 * key16 + i], a.scale_log2, -m_run));
+          ps8[i] += p[i];
         }
         uint4 pk;
         __nv_bfloat162* h2 = reinterpret_cast<__nv_bfloat162*>(&pk);
 #pragma unroll
         for (int i = 0; i < 4; ++i) h2[i] = __floats2bfloat162_rn(p[2 * i], p[2 * i + 1]);
         const int blk = key16 / 8, c = key16 % 8;       // 64-key block, 16-byte chunk within its row
-        *reinterpret_cast<uint4*>(sP + blk * (BQ * 128) + swz<128>(m, c)) = pk;
+        *reinterpret_cast<uint4*>(pbuf + blk * (BQ * 128) + swz<128>(m, c)) = pk;
       }
-      tc_fence_before();
       fence_async_smem();
+      tc_fence_before();
       __syncwarp();
-      if (lane == 0) {
-        mbar_arrive(s_free + b);
-        mbar_arrive(p_full);
-      }
-      l_run = l_run * corr + psum;
-      m_run = mx;
-      corr_prev = corr;
+      if (lane == 0) mbar_arrive(p_full + b);
+#pragma unroll
+      for (int w = 4; w >= 1; w >>= 1)
+#pragma unroll
+        for (int i = 0; i < w; ++i) ps8[i] += ps8[i + w];
+      l_run += ps8[0];
     }
     if (ok) {
-      ok = mbar_wait(o_full, (nkv - 1) & 1, abort_flag);
+      ok = mbar_wait(pv_done + ((nkv - 1) & 1), ((nkv - 1) >> 1) & 1, abort_flag);
       ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
     }
     if (ok) {
       tc_fence_after();
+      const float inv = 1.f / l_run;
+      __nv_bfloat16* dst = a.out + grow * a.d + h * DH;
 #pragma unroll
       for (int cc = 0; cc < DH; cc += 32) {
         float ov[32];
         tmem_ld32(t_o + cc + lane_off, ov);
+        if (valid) {
 #pragma unroll
-        for (int i = 0; i < 32; ++i) o[cc + i] = fmaf(o[cc + i], corr_prev, ov[i]);
-      }
-      if (valid) {
-        const float inv = 1.f / l_run;
-        __nv_bfloat16* dst = a.out + grow * a.d + h * DH;
+          for (int c = 0; c < 32; c += 8) {
+            float t[8];
 #pragma unroll
-        for (int c = 0; c < DH; c += 8) {
-          float t[8];
-#pragma unroll
-          for (int i = 0; i < 8; ++i) t[i] = o[c + i] * inv;
-          Vec16<__nv_bfloat16>::store(dst + c, t);
+            for (int i = 0; i < 8; ++i) t[i] = ov[c + i] * inv;
+            Vec16<__nv_bfloat16>::store(dst + cc + c, t);
+          }
         }
       }
     }

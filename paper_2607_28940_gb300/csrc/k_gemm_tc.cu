@@ -217,29 +217,35 @@ __device__ __forceinline__ void epilogue(const EpiArgs& e, uint32_t tacc, int ro
 
 // ------------------------------------------------------------------ kernel
 
-template <int BN, int EPI, int NAP = 4>
+// BRES: the CTA's whole B slice (BN x K, K <= KRES) stays resident in shared
+// memory and only A streams through the ring.
+template <int BN, int EPI, int NAP = 4, bool BRES = false>
 struct Shape {
   static constexpr int BN_MMA = BN < 256 ? BN : 256;     // N of one tcgen05.mma
   static constexpr int B_BOX = BN_MMA;                    // rows of one TMA box of B
-  static constexpr int B_STAGE_BYTES = BN * BK * 2;
+  static constexpr int KRES = 256;
+  static constexpr int BRES_BYTES = BRES ? BN * KRES * 2 : 0;
+  static constexpr int B_STAGE_BYTES = BRES ? 0 : BN * BK * 2;
   static constexpr int STAGE_BYTES = A_STAGE_BYTES + B_STAGE_BYTES;
   static constexpr bool LN = EPI == EPI_LN || EPI == EPI_LN_HEAD;
   static constexpr int RED_BYTES = LN ? 2 * 128 * kRedStride * 4 : 0;
   static constexpr int WEFF_BYTES = EPI == EPI_LN_HEAD ? BN * NAP * 4 : 0;
-  // bias [kStageN] floats, then (cache-row remap) offsets and first rows;
-  // rounded to 1 KB so that the staging buffers after it start on a
-  // swizzle-atom boundary
+  // bias [kStageN] floats (not with BRES), then (cache-row remap) offsets and
+  // first rows; rounded to 1 KB so that the staging buffers after it start on
+  // a swizzle-atom boundary
   static constexpr int AUX_BYTES =
-      LN ? 0 : ((kStageN * 4 + (EPI == EPI_KV ? (2 * kStageSeg + 1) * 4 : 0) + 1023) / 1024) * 1024;
+      LN ? 0
+         : (((BRES ? 0 : kStageN * 4) + (EPI == EPI_KV ? (2 * kStageSeg + 1) * 4 : 0) + 1023) / 1024) * 1024;
   // bulk-store staging: two 2 KB buffers per epilogue warp (bf16 outputs)
   static constexpr int STG_BYTES = EPI == EPI_LN_HEAD ? 0 : kEpiWarps * 2 * 2048;
-  static constexpr int EXTRA = RED_BYTES + WEFF_BYTES + AUX_BYTES + STG_BYTES + 1024 + 256;
+  static constexpr int EXTRA = BRES_BYTES + RED_BYTES + WEFF_BYTES + AUX_BYTES + STG_BYTES + 1024 + 256;
   static constexpr int STAGES_FIT = (227 * 1024 - EXTRA) / STAGE_BYTES;
   static constexpr int STAGES = STAGES_FIT > 8 ? 8 : STAGES_FIT;
   static constexpr int ACC_BUFS = BN <= 256 ? 2 : 1;      // TMEM double buffer
   static constexpr int TMEM_COLS = BN * ACC_BUFS < 32 ? 32 : BN * ACC_BUFS;
   static constexpr int SMEM_BYTES = STAGES * STAGE_BYTES + EXTRA;
   static_assert(STAGES >= 2, "pipeline depth");
+  static_assert(!(BRES && LN), "resident B only for the plain epilogues");
   static_assert((RED_BYTES + WEFF_BYTES + AUX_BYTES) % 1024 == 0 || STG_BYTES == 0,
                 "staging buffers need 512-byte alignment (64-byte swizzle atoms)");
   static_assert((RED_BYTES + WEFF_BYTES + AUX_BYTES + STG_BYTES) % 16 == 0, "mbarriers must stay 8-byte aligned");
@@ -248,36 +254,53 @@ struct Shape {
 };
 
 // Persistent: CTA b processes tiles b, b + gridDim.x, ... (tile t -> n tile
-// t % n_tiles, m tile t / n_tiles).  Warp 0: TMA producer over all tiles and
-// K blocks; warp 1: MMA issuer, accumulating tile i into TMEM buffer i % 2;
+// t % n_tiles, m tile t / n_tiles).  With BRES, CTA b instead takes the
+// contiguous range [b T / G, (b + 1) T / G) of the T tiles in n-major order
+// (tile t -> n tile t / m_tiles, m tile t % m_tiles), so it loads one B slice,
+// rarely two; the CTAs of different n slices walk the m tiles in step and
+// share each A tile through L2.  Warp 0: TMA producer over all tiles and K
+// blocks; warp 1: MMA issuer, accumulating tile i into TMEM buffer i % 2;
 // warps 2..9: epilogue, releasing the buffer as soon as its last TMEM read is
 // done so the next tile's MMAs overlap this tile's stores.
-template <int BN, int EPI, int NAP>
+template <int BN, int EPI, int NAP, bool BRES>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                    const __grid_constant__ CUtensorMap tmO, const EpiArgs e) {
-  using S = Shape<BN, EPI, NAP>;
+  using S = Shape<BN, EPI, NAP, BRES>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* sA = smem;
   uint8_t* sB = smem + S::STAGES * A_STAGE_BYTES;
-  float* red = reinterpret_cast<float*>(sB + S::STAGES * S::B_STAGE_BYTES);
+  uint8_t* sBres = sB + S::STAGES * S::B_STAGE_BYTES;
+  float* red = reinterpret_cast<float*>(sBres + S::BRES_BYTES);
   float* s_weff = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(red) + S::RED_BYTES);
   float* s_bias = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(s_weff) + S::WEFF_BYTES);
-  int* s_seg = reinterpret_cast<int*>(s_bias + kStageN);
+  int* s_seg = reinterpret_cast<int*>(s_bias + (BRES ? 0 : kStageN));
   int* s_dst = s_seg + kStageSeg + 1;
   uint8_t* s_stage = reinterpret_cast<uint8_t*>(s_bias) + S::AUX_BYTES;
   uint64_t* full = reinterpret_cast<uint64_t*>(s_stage + S::STG_BYTES);
   uint64_t* empty = full + S::STAGES;
   uint64_t* acc_full = empty + S::STAGES;
   uint64_t* acc_empty = acc_full + 2;
-  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(acc_empty + 2);
+  uint64_t* b_full = acc_empty + 2;     // resident B slice loaded
+  uint64_t* b_empty = b_full + 1;       // last MMA reading the resident B slice done
+  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(b_empty + 1);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_holder + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int n_tiles = e.N / BN;
   const int num_tiles = ((e.M + BM - 1) / BM) * n_tiles;
   const int num_kb = e.K / BK;
+  const int m_tiles = (e.M + BM - 1) / BM;
+  // this CTA's tiles: t_lo, t_lo + t_step, ... < t_hi
+  int t_lo = blockIdx.x, t_hi = num_tiles, t_step = gridDim.x;
+  if constexpr (BRES) {
+    t_lo = static_cast<int>(static_cast<long long>(blockIdx.x) * num_tiles / gridDim.x);
+    t_hi = static_cast<int>(static_cast<long long>(blockIdx.x + 1) * num_tiles / gridDim.x);
+    t_step = 1;
+  }
+  auto tile_n = [&](int t) { return BRES ? t / m_tiles : t % n_tiles; };
+  auto tile_m = [&](int t) { return BRES ? t % m_tiles : t / n_tiles; };
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < S::STAGES; ++s) {
@@ -288,6 +311,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       mbar_init(acc_full + b, 1);
       mbar_init(acc_empty + b, kEpiWarps);
     }
+    mbar_init(b_full, 1);
+    mbar_init(b_empty, 1);
     *abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
@@ -312,7 +337,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   const int* seg_off = e.seg_off;
   const int* dst_row0 = e.dst_row0;
   if constexpr (!S::LN) {
-    if (e.N <= kStageN) {
+    if (!BRES && e.N <= kStageN) {
       for (int i = threadIdx.x; i < e.N; i += NUM_THREADS) s_bias[i] = e.bias[i];
       bias = s_bias;
     }
@@ -332,9 +357,22 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmA)) : "memory");
       asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmB)) : "memory");
       int it = 0;  // global k-block counter (ring position)
+      int nb = 0, cur_n = -1;   // resident B slices loaded, current slice
       bool ok = true;
-      for (int t = blockIdx.x; t < num_tiles && ok; t += gridDim.x) {
-        const int m0 = (t / n_tiles) * BM, n0 = (t % n_tiles) * BN;
+      for (int t = t_lo; t < t_hi && ok; t += t_step) {
+        const int m0 = tile_m(t) * BM, n0 = tile_n(t) * BN;
+        if constexpr (BRES) {
+          if (n0 != cur_n) {
+            if (nb > 0 && !mbar_wait(b_empty, (nb - 1) & 1, abort_flag)) break;
+            mbar_expect_tx(b_full, BN * e.K * 2);
+            for (int kb = 0; kb < num_kb; ++kb)
+#pragma unroll
+              for (int j = 0; j < BN; j += S::B_BOX)
+                tma_load_2d(sBres + kb * (BN * BK * 2) + j * (BK * 2), &tmB, b_full, kb * BK, n0 + j);
+            ++nb;
+            cur_n = n0;
+          }
+        }
         for (int kb = 0; kb < num_kb; ++kb, ++it) {
           const int s = it % S::STAGES;
           const uint32_t ph = (it / S::STAGES) & 1;
@@ -344,23 +382,35 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           }
           mbar_expect_tx(full + s, S::STAGE_BYTES);
           tma_load_2d(sA + s * A_STAGE_BYTES, &tmA, full + s, kb * BK, m0);
+          if constexpr (!BRES) {
 #pragma unroll
-          for (int j = 0; j < BN; j += S::B_BOX)
-            tma_load_2d(sB + s * S::B_STAGE_BYTES + j * (BK * 2), &tmB, full + s, kb * BK, n0 + j);
+            for (int j = 0; j < BN; j += S::B_BOX)
+              tma_load_2d(sB + s * S::B_STAGE_BYTES + j * (BK * 2), &tmB, full + s, kb * BK, n0 + j);
+          }
         }
       }
       if (*abort_flag) {
         // let the copies already in flight land before shared memory is released
         for (int k = it > S::STAGES ? it - S::STAGES : 0; k < it; ++k)
           mbar_wait_plain(full + k % S::STAGES, (k / S::STAGES) & 1);
+        if (BRES && nb > 0) mbar_wait_plain(b_full, (nb - 1) & 1);
       }
     }
   } else if (warp == 1) {
     if (lane == 0) {
       constexpr uint32_t idesc = idesc_bf16(BM, S::BN_MMA);
       int it = 0, i = 0;
+      int nb = 0, cur_n = -1;
       bool ok = true;
-      for (int t = blockIdx.x; t < num_tiles && ok; t += gridDim.x, ++i) {
+      for (int t = t_lo; t < t_hi && ok; t += t_step, ++i) {
+        const int nt = tile_n(t);
+        if constexpr (BRES) {
+          if (nt != cur_n) {
+            if (!mbar_wait(b_full, nb & 1, abort_flag)) break;
+            ++nb;
+            cur_n = nt;
+          }
+        }
         const int buf = i % S::ACC_BUFS;
         const uint32_t use = i / S::ACC_BUFS;
         if (!mbar_wait(acc_empty + buf, (use & 1) ^ 1, abort_flag)) break;
@@ -375,7 +425,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           }
           tc_fence_after();
           const uint64_t adesc = sdesc_sw128(smem_u32(sA + s * A_STAGE_BYTES));
-          const uint64_t bdesc = sdesc_sw128(smem_u32(sB + s * S::B_STAGE_BYTES));
+          const uint64_t bdesc = BRES ? sdesc_sw128(smem_u32(sBres + kb * (BN * BK * 2)))
+                                      : sdesc_sw128(smem_u32(sB + s * S::B_STAGE_BYTES));
 #pragma unroll
           for (int k = 0; k < BK / 16; ++k) {
 #pragma unroll
@@ -390,6 +441,10 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           mma_commit(empty + s);
         }
         mma_commit(acc_full + buf);   // also on abort: the epilogue waits on every issued MMA
+        if constexpr (BRES) {
+          // the resident slice is free once this tile's MMAs are done
+          if (t + 1 >= t_hi || tile_n(t + 1) != nt) mma_commit(b_empty);
+        }
       }
     }
   } else {
@@ -399,7 +454,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     uint8_t* stage = s_stage + ew * 4096;
     int kchunk = 0;
     int i = 0;
-    for (int t = blockIdx.x; t < num_tiles; t += gridDim.x, ++i) {
+    for (int t = t_lo; t < t_hi; t += t_step, ++i) {
       const int buf = i % S::ACC_BUFS;
       const uint32_t use = i / S::ACC_BUFS;
       // Go on exactly when the accumulator is complete: both warps of a lane
@@ -410,7 +465,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       go = __shfl_sync(0xffffffffu, go ? 1 : 0, 0) != 0;
       if (!go) break;
       tc_fence_after();
-      const int m0 = (t / n_tiles) * BM, n0 = (t % n_tiles) * BN;
+      const int m0 = tile_m(t) * BM, n0 = tile_n(t) * BN;
       epilogue<BN, EPI, NAP>(e, tmem + buf * BN + (static_cast<uint32_t>(q * 32) << 16), m0 + q * 32 + lane, n0,
                              h * (BN / 2), q, h, red, s_weff, bias, seg_off, dst_row0, &tmO, stage, kchunk);
       tc_fence_before();
@@ -486,14 +541,15 @@ int num_sms() {
   return n;
 }
 
-template <int BN, int EPI, int NAP = 4>
+template <int BN, int EPI, int NAP = 4, bool BRES = false>
 static cudaError_t launch_bn(const __nv_bfloat16* A, long long lda, const __nv_bfloat16* B, const EpiArgs& e,
                              cudaStream_t s, int cls) {
-  using Sh = Shape<BN, EPI, NAP>;
+  using Sh = Shape<BN, EPI, NAP, BRES>;
+  if (BRES && e.K > Sh::KRES) return cudaErrorInvalidValue;
   static bool attr_set = false;
   if (!attr_set) {
-    cudaError_t err = cudaFuncSetAttribute(gemm_tc_kernel<BN, EPI, NAP>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                           Sh::SMEM_BYTES);
+    cudaError_t err = cudaFuncSetAttribute(gemm_tc_kernel<BN, EPI, NAP, BRES>,
+                                           cudaFuncAttributeMaxDynamicSharedMemorySize, Sh::SMEM_BYTES);
     if (err != cudaSuccess) return err;
     attr_set = true;
   }
@@ -513,7 +569,7 @@ static cudaError_t launch_bn(const __nv_bfloat16* A, long long lda, const __nv_b
   const int grid = static_cast<int>(tiles < num_sms() ? tiles : num_sms());
   prof_begin(cls, s);
   cudaError_t err =
-      launch_pdl(gemm_tc_kernel<BN, EPI, NAP>, dim3(grid), dim3(NUM_THREADS), Sh::SMEM_BYTES, s, ta, tb, to, e);
+      launch_pdl(gemm_tc_kernel<BN, EPI, NAP, BRES>, dim3(grid), dim3(NUM_THREADS), Sh::SMEM_BYTES, s, ta, tb, to, e);
   prof_end(cls, s);
   return err;
 }
@@ -535,6 +591,9 @@ static cudaError_t launch_plain(const __nv_bfloat16* A, long long lda, const __n
     if (EPI == EPI_KV && e.col_blk % bn) return false;
     return true;
   };
+  // short K and at least two tiles per SM: keep each CTA's B slice resident
+  if (fits(256) && e.K <= Shape<256, EPI, 4, true>::KRES && m_tiles * (e.N / 256) >= 2 * num_sms())
+    return launch_bn<256, EPI, 4, true>(A, lda, B, e, s, cls);
   if (fits(256) && m_tiles * (e.N / 256) >= num_sms()) return launch_bn<256, EPI>(A, lda, B, e, s, cls);
   if (fits(128)) return launch_bn<128, EPI>(A, lda, B, e, s, cls);
   if (fits(64)) return launch_bn<64, EPI>(A, lda, B, e, s, cls);
