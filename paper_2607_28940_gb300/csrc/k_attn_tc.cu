@@ -9,13 +9,13 @@
 //   warp 0     TMA producer: K_j, V_j tiles of the request (head h columns)
 //              into a STG-deep shared-memory ring;
 //   warp 1     MMA issuer: S_j = Q K_j^T into one of two TMEM buffers, then
-//              O += P_j V_j into the TMEM output tile (V used MN-major: no
-//              transpose);
+//              O += P_j V_j into the TMEM output tile.  Q and P are the A
+//              operands and are read from TMEM, so the tensor core reads only
+//              K and V from shared memory (V used MN-major: no transpose);
 //   warps 2-5  softmax: one query row per thread straight out of TMEM (row
-//              max, exp2, row sum need no shuffles); P_j goes to one of two
-//              shared-memory buffers in the 128-byte-swizzled layout the MMA
-//              reads, so the exponentials of tile j overlap the PV product of
-//              tile j - 1.
+//              max, exp2, row sum need no shuffles); P_j (bf16) goes back to
+//              one of two TMEM buffers, so the exponentials of tile j overlap
+//              the PV product of tile j - 1.
 // The running maximum is raised only when a tile's maximum exceeds it by more
 // than 2^8 (then O and the row sum are rescaled in place); otherwise the
 // stale maximum is kept, P stays below 256 and no rescale is needed.  Exact
@@ -30,7 +30,7 @@ namespace fa {
 
 constexpr int BQ = 128;            // queries per CTA (TMEM lanes)
 constexpr int BKV = 128;           // keys per K/V tile
-constexpr int STG = 3;             // K/V ring depth
+constexpr int STG = 4;             // K/V ring depth
 constexpr int NUM_THREADS = 192;   // producer, MMA, 4 softmax warps
 constexpr float kRescaleLog2 = 8.f;  // raise the running max only past this (log2 units)
 
@@ -53,10 +53,10 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
   uint32_t ok;
   asm volatile(
       "{\n\t.reg .pred p;\n\t"
-      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
       "selp.u32 %0, 1, 0, p;\n\t}"
       : "=r"(ok)
-      : "r"(smem_u32(bar)), "r"(parity), "r"(1000000u)   // suspend up to 1 ms per try
+      : "r"(smem_u32(bar)), "r"(parity)
       : "memory");
   return ok != 0;
 }
@@ -104,6 +104,27 @@ __device__ __forceinline__ void mma_bf16(uint32_t d_tmem, uint64_t adesc, uint64
       "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
       : "memory");
 }
+// Same, with the A operand (M x 16 bf16, K-major: lane = row, two elements
+// per 32-bit column) read from TMEM at a_tmem.
+__device__ __forceinline__ void mma_bf16_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t bdesc, uint32_t idesc,
+                                            uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "r"(a_tmem), "l"(bdesc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+// 16 columns of this warp's 32 lanes; completion is awaited by tmem_wait_st.
+__device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint32_t* v) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], "
+      "{%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16};" ::"r"(taddr),
+      "r"(v[0]), "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7]), "r"(v[8]), "r"(v[9]),
+      "r"(v[10]), "r"(v[11]), "r"(v[12]), "r"(v[13]), "r"(v[14]), "r"(v[15])
+      : "memory");
+}
+__device__ __forceinline__ void tmem_wait_st() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
 __device__ __forceinline__ void mma_commit(uint64_t* bar) {
   asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(smem_u32(bar))
                : "memory");
@@ -143,6 +164,19 @@ __device__ __forceinline__ void tmem_st32(uint32_t taddr, const float* v) {
       "r"(__float_as_uint(v[27])), "r"(__float_as_uint(v[28])), "r"(__float_as_uint(v[29])),
       "r"(__float_as_uint(v[30])), "r"(__float_as_uint(v[31]))
       : "memory");
+}
+
+// 128 consecutive columns of this warp's 32 lanes: one load, one wait.
+__device__ __forceinline__ void tmem_ld128(uint32_t taddr, float* v) {
+  uint32_t r[128];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x128.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,%32,%33,%34,%35,%36,%37,%38,%39,%40,%41,%42,%43,%44,%45,%46,%47,%48,%49,%50,%51,%52,%53,%54,%55,%56,%57,%58,%59,%60,%61,%62,%63,%64,%65,%66,%67,%68,%69,%70,%71,%72,%73,%74,%75,%76,%77,%78,%79,%80,%81,%82,%83,%84,%85,%86,%87,%88,%89,%90,%91,%92,%93,%94,%95,%96,%97,%98,%99,%100,%101,%102,%103,%104,%105,%106,%107,%108,%109,%110,%111,%112,%113,%114,%115,%116,%117,%118,%119,%120,%121,%122,%123,%124,%125,%126,%127}, [%128];\n\t"
+      "tcgen05.wait::ld.sync.aligned;"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31]), "=r"(r[32]), "=r"(r[33]), "=r"(r[34]), "=r"(r[35]), "=r"(r[36]), "=r"(r[37]), "=r"(r[38]), "=r"(r[39]), "=r"(r[40]), "=r"(r[41]), "=r"(r[42]), "=r"(r[43]), "=r"(r[44]), "=r"(r[45]), "=r"(r[46]), "=r"(r[47]), "=r"(r[48]), "=r"(r[49]), "=r"(r[50]), "=r"(r[51]), "=r"(r[52]), "=r"(r[53]), "=r"(r[54]), "=r"(r[55]), "=r"(r[56]), "=r"(r[57]), "=r"(r[58]), "=r"(r[59]), "=r"(r[60]), "=r"(r[61]), "=r"(r[62]), "=r"(r[63]), "=r"(r[64]), "=r"(r[65]), "=r"(r[66]), "=r"(r[67]), "=r"(r[68]), "=r"(r[69]), "=r"(r[70]), "=r"(r[71]), "=r"(r[72]), "=r"(r[73]), "=r"(r[74]), "=r"(r[75]), "=r"(r[76]), "=r"(r[77]), "=r"(r[78]), "=r"(r[79]), "=r"(r[80]), "=r"(r[81]), "=r"(r[82]), "=r"(r[83]), "=r"(r[84]), "=r"(r[85]), "=r"(r[86]), "=r"(r[87]), "=r"(r[88]), "=r"(r[89]), "=r"(r[90]), "=r"(r[91]), "=r"(r[92]), "=r"(r[93]), "=r"(r[94]), "=r"(r[95]), "=r"(r[96]), "=r"(r[97]), "=r"(r[98]), "=r"(r[99]), "=r"(r[100]), "=r"(r[101]), "=r"(r[102]), "=r"(r[103]), "=r"(r[104]), "=r"(r[105]), "=r"(r[106]), "=r"(r[107]), "=r"(r[108]), "=r"(r[109]), "=r"(r[110]), "=r"(r[111]), "=r"(r[112]), "=r"(r[113]), "=r"(r[114]), "=r"(r[115]), "=r"(r[116]), "=r"(r[117]), "=r"(r[118]), "=r"(r[119]), "=r"(r[120]), "=r"(r[121]), "=r"(r[122]), "=r"(r[123]), "=r"(r[124]), "=r"(r[125]), "=r"(r[126]), "=r"(r[127])
+      : "r"(taddr)
+      : "memory");
+#pragma unroll
+  for (int i = 0; i < 128; ++i) v[i] = __uint_as_float(r[i]);
 }
 
 // 2^x on the special-function unit (PTX ex2.approx, flush-to-zero).
@@ -190,20 +224,14 @@ struct FaShape {
   static constexpr int ROW_BYTES = DH * 2;                  // 64 or 128: one swizzle row
   static constexpr uint32_t SW = DH == 64 ? 2u : 4u;        // 128-byte or 64-byte swizzle
   static constexpr int ATOM = 8 * ROW_BYTES;                // 8 rows
-  static constexpr int Q_BYTES = BQ * ROW_BYTES;
   static constexpr int KV_BYTES = BKV * ROW_BYTES;
-  static constexpr int P_BYTES = BQ * BKV * 2;              // one P buffer: two 64-key blocks, 128-byte swizzle
-  static constexpr int SMEM = Q_BYTES + 2 * P_BYTES + 2 * STG * KV_BYTES + 1024 + 256;
-  static constexpr int TMEM_COLS = 512;                     // S x2 (256) + O tile (DH)
+  static constexpr int SMEM = 2 * STG * KV_BYTES + 1024 + 256;
+  // TMEM columns: S_0, S_1 (fp32, 128 each), O (fp32, DH), P_0, P_1 (bf16
+  // pairs, 64 each), Q (bf16 pairs, DH / 2)
+  static constexpr uint32_t T_S = 0, T_O = 256, T_P = 320, T_Q = 448;
+  static constexpr int TMEM_COLS = 512;
+  static_assert(T_O + DH <= T_P && T_Q + DH / 2 <= TMEM_COLS, "TMEM columns");
 };
-
-// byte offset of 16-byte chunk c of row m in a swizzled K-major tile whose rows
-// are ROW_BYTES long (Swizzle: chunk index XOR row bits above the 128-byte line)
-template <int ROW_BYTES>
-__device__ __forceinline__ int swz(int m, int c) {
-  if constexpr (ROW_BYTES == 128) return m * 128 + ((c ^ (m & 7)) << 4);
-  else return m * 64 + ((c ^ ((m >> 1) & 3)) << 4);
-}
 
 template <int DH>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
@@ -211,16 +239,14 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   using Sh = FaShape<DH>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  uint8_t* sQ = smem;
-  uint8_t* sP = sQ + Sh::Q_BYTES;                      // two P buffers
-  uint8_t* sK = sP + 2 * Sh::P_BYTES;
+  uint8_t* sK = smem;
   uint8_t* sV = sK + STG * Sh::KV_BYTES;
   uint64_t* bars = reinterpret_cast<uint64_t*>(sV + STG * Sh::KV_BYTES);
   uint64_t* kv_full = bars;
   uint64_t* kv_empty = kv_full + STG;
   uint64_t* s_full = kv_empty + STG;    // [2] S_j in TMEM buffer j % 2
   uint64_t* s_free = s_full + 2;        // [2] the softmax warps have read it
-  uint64_t* p_full = s_free + 2;        // [2] P_j in shared buffer j % 2
+  uint64_t* p_full = s_free + 2;        // [2] P_j in TMEM buffer j % 2
   uint64_t* pv_done = p_full + 2;       // [2] O += P_j V_j complete
   uint64_t* q_ready = pv_done + 2;
   uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(q_ready + 1);
@@ -262,8 +288,6 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_holder;
-  const uint32_t t_s = tmem;            // S buffers at columns 0 and 128
-  const uint32_t t_o = tmem + 256;      // O tile
 
   if (warp == 0) {
     if (lane == 0) {
@@ -286,7 +310,6 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     if (lane == 0) {
       constexpr uint32_t id_s = idesc_bf16(BQ, BKV, false);
       constexpr uint32_t id_pv = idesc_bf16(BQ, DH, true);
-      const uint32_t q_addr = smem_u32(sQ), p_addr = smem_u32(sP);
       bool ok = mbar_wait(q_ready, 0, abort_flag);
       tc_fence_after();
       // O += P_t V_t, after the softmax warps have written P_t (and rescaled O
@@ -296,14 +319,11 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         if (!mbar_wait(p_full + bt, (t >> 1) & 1, abort_flag)) return false;
         tc_fence_after();
         const uint32_t v_addr = smem_u32(sV + st * Sh::KV_BYTES);
-        const uint32_t pb = p_addr + bt * Sh::P_BYTES;
 #pragma unroll
         for (int k = 0; k < BKV / 16; ++k) {
-          // P: 64-key blocks of 16 KB, 32 bytes per 16-key step inside a block
-          const uint64_t pd = sdesc(pb + (k / 4) * (BQ * 128) + (k % 4) * 32, 16, 1024, 2);
           // V (MN-major): 16 keys = two 8-row atoms of the tile
           const uint64_t vd = sdesc(v_addr + k * 16 * Sh::ROW_BYTES, Sh::ATOM, Sh::ATOM, Sh::SW);
-          mma_bf16(t_o, pd, vd, id_pv, (t > 0 || k > 0) ? 1u : 0u);
+          mma_bf16_ts(tmem + Sh::T_O, tmem + Sh::T_P + 64 * bt + 8 * k, vd, id_pv, (t > 0 || k > 0) ? 1u : 0u);
         }
         mma_commit(pv_done + bt);
         mma_commit(kv_empty + st);
@@ -317,9 +337,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         const uint32_t k_addr = smem_u32(sK + st * Sh::KV_BYTES);
 #pragma unroll
         for (int k = 0; k < DH / 16; ++k) {
-          const uint64_t qd = sdesc(q_addr + k * 32, 16, Sh::ATOM, Sh::SW);
           const uint64_t kd = sdesc(k_addr + k * 32, 16, Sh::ATOM, Sh::SW);
-          mma_bf16(t_s + b * BKV, qd, kd, id_s, k > 0 ? 1u : 0u);
+          mma_bf16_ts(tmem + Sh::T_S + BKV * b, tmem + Sh::T_Q + 8 * k, kd, id_s, k > 0 ? 1u : 0u);
         }
         mma_commit(s_full + b);
         if (j >= 1) ok = pv(j - 1);
@@ -334,20 +353,24 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     const bool valid = j_q < n_q;
     const long long grow = j_q < M ? static_cast<long long>(c0) + j_q
                                    : a.n_cand + static_cast<long long>(r) * a.S + (j_q - M);
-    // gather this row's head slice of Q into the swizzled tile
+    const uint32_t lane_off = static_cast<uint32_t>(qw * 32) << 16;
+    // this row's head slice of Q into TMEM (bf16 pairs)
     {
-      constexpr int CH = Sh::ROW_BYTES / 16;
-      const uint4* src = reinterpret_cast<const uint4*>(a.q + grow * a.d + h * DH);
+      uint32_t qv[DH / 2];
+      const uint4* src = reinterpret_cast<const uint4*>(a.q + (valid ? grow : 0) * a.d + h * DH);
 #pragma unroll
-      for (int c = 0; c < CH; ++c) {
-        uint4 v = valid ? src[c] : make_uint4(0, 0, 0, 0);
-        *reinterpret_cast<uint4*>(sQ + swz<Sh::ROW_BYTES>(m, c)) = v;
+      for (int c = 0; c < DH / 8; ++c) {
+        const uint4 v = valid ? src[c] : make_uint4(0, 0, 0, 0);
+        qv[4 * c] = v.x; qv[4 * c + 1] = v.y; qv[4 * c + 2] = v.z; qv[4 * c + 3] = v.w;
       }
-      fence_async_smem();
+#pragma unroll
+      for (int c = 0; c < DH / 2; c += 16) tmem_st16(tmem + Sh::T_Q + c + lane_off, qv + c);
+      tmem_wait_st();
+      tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(q_ready);
     }
-    const uint32_t lane_off = static_cast<uint32_t>(qw * 32) << 16;
+    const uint32_t t_o = tmem + Sh::T_O + lane_off;
     float m_run = -INFINITY, l_run = 0.f;     // running max (log2 units, scaled), row sum
     bool ok = true;
     for (int j = 0; j < nkv && ok; ++j) {
@@ -356,11 +379,10 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
       if (!ok) break;
       tc_fence_after();
-      // the whole score row of this tile in one pass over TMEM; the buffer is
-      // free for S_{j+2} as soon as it is in registers
+      // the whole score row of this tile in one TMEM load; the buffer is free
+      // for S_{j+2} as soon as it is in registers
       float sv[BKV];
-#pragma unroll
-      for (int cc = 0; cc < BKV; cc += 32) tmem_ld32(t_s + b * BKV + cc + lane_off, sv + cc);
+      tmem_ld128(tmem + Sh::T_S + BKV * b + lane_off, sv);
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(s_free + b);
@@ -393,10 +415,10 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
 #pragma unroll
           for (int cc = 0; cc < DH; cc += 32) {
             float ov[32];
-            tmem_ld32(t_o + cc + lane_off, ov);
+            tmem_ld32(t_o + cc, ov);
 #pragma unroll
             for (int i = 0; i < 32; ++i) ov[i] *= alpha;
-            tmem_st32(t_o + cc + lane_off, ov);
+            tmem_st32(t_o + cc, ov);
           }
         }
         l_run *= alpha;
@@ -407,28 +429,28 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         ok = mbar_wait(pv_done + b, ((j - 2) >> 1) & 1, abort_flag);
         ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
         if (!ok) break;
+        tc_fence_after();
       }
-      // P = 2^(s * scale - m_run) into the swizzled P buffer (bf16), row sum
-      uint8_t* pbuf = sP + b * Sh::P_BYTES;
+      // P = 2^(s * scale - m_run) as bf16 pairs into TMEM buffer b, row sum
+      const uint32_t t_p = tmem + Sh::T_P + 64 * b + lane_off;
       float ps8[8];
 #pragma unroll
       for (int i = 0; i < 8; ++i) ps8[i] = 0.f;
 #pragma unroll
-      for (int key16 = 0; key16 < BKV / 8; ++key16) {
-        float p[8];
+      for (int c32 = 0; c32 < BKV; c32 += 32) {
+        uint32_t pk[16];
 #pragma unroll
-        for (int i = 0; i < 8; ++i) {
-          p[i] = ex2(fmaf(sv[8 * key16 + i], a.scale_log2, -m_run));
-          ps8[i] += p[i];
+        for (int i = 0; i < 32; i += 2) {
+          const float p0 = ex2(fmaf(sv[c32 + i], a.scale_log2, -m_run));
+          const float p1 = ex2(fmaf(sv[c32 + i + 1], a.scale_log2, -m_run));
+          ps8[i & 7] += p0;
+          ps8[(i + 1) & 7] += p1;
+          __nv_bfloat162 h2 = __floats2bfloat162_rn(p0, p1);      // lower key in the low half
+          pk[i / 2] = *reinterpret_cast<uint32_t*>(&h2);
         }
-        uint4 pk;
-        __nv_bfloat162* h2 = reinterpret_cast<__nv_bfloat162*>(&pk);
-#pragma unroll
-        for (int i = 0; i < 4; ++i) h2[i] = __floats2bfloat162_rn(p[2 * i], p[2 * i + 1]);
-        const int blk = key16 / 8, c = key16 % 8;       // 64-key block, 16-byte chunk within its row
-        *reinterpret_cast<uint4*>(pbuf + blk * (BQ * 128) + swz<128>(m, c)) = pk;
+        tmem_st16(t_p + c32 / 2, pk);
       }
-      fence_async_smem();
+      tmem_wait_st();
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(p_full + b);
@@ -449,7 +471,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
 #pragma unroll
       for (int cc = 0; cc < DH; cc += 32) {
         float ov[32];
-        tmem_ld32(t_o + cc + lane_off, ov);
+        tmem_ld32(t_o + cc, ov);
         if (valid) {
 #pragma unroll
           for (int c = 0; c < 32; c += 8) {
