@@ -44,10 +44,11 @@ FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0}
 # DRAM traffic per launch measured with ncu (dram__bytes_read.sum +
 # dram__bytes_write.sum) for the kernel classes that can be dominant, with the
 # sha256 prefix of the kernel source at capture time; a source change voids it.
-# (workload, mode, class) -> (bytes per launch, source sha256[:12]); from
-# profiles/gemm_tc_small_bf16.md.
+# (workload, mode, class) -> (bytes per launch, source sha256[:12]), each from
+# one --set full capture of that class's kernel on that workload.
 NCU_TRAFFIC = {
-    ("small_bf16", "local_global", "gemm_oproj_ln"): (8.61e6, "40a69cd3f2dd"),
+    ("small_bf16", "local_global", "gemm_oproj_ln"): (8.62e6, "19df9b0ee59c"),
+    ("mid_bf16", "full", "attn_cross"): (830.4e6, "5e48154e4f63"),
 }
 
 
@@ -302,7 +303,9 @@ def run_txs(args, rank, world):
         roof = {"bound": "hbm", "achieved": achieved, "peak": peaks["hbm_gbs"], "unit": "GB/s"}
     roof["frac"] = roof["achieved"] / roof["peak"]
     tr = NCU_TRAFFIC.get((args.workload, args.mode, dom))
-    src_file = ("k_gemm_tc.cu" if dom.startswith("gemm") else
+    src_file = ("k_gemm_ln.cu" if dom in ("gemm_oproj_ln", "gemm_ffn2_ln") and wl.dtype == "bf16" and
+                wl.d_model in (256, 512) else
+                "k_gemm_tc.cu" if dom.startswith("gemm") else
                 "k_attn_tc.cu" if (dom == "attn_cross" and args.mode == "full" and wl.dtype == "bf16") else
                 "k_score.cu" if dom in ("pack", "rank") else
                 "k_cache.cu" if dom in ("pool", "global_kv") else "k_attn.cu")
