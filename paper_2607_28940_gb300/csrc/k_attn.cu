@@ -12,6 +12,8 @@
 // Both: scale 1/sqrt(d_h), per-head online softmax in fp32.  A group of
 // TPH = d_h / VEC threads (VEC = elements per 16-byte vector) owns one
 // (row, head); dot products are reduced with warp shuffles inside the group.
+#include <algorithm>
+
 #include "txs_internal.cuh"
 
 namespace txs {
@@ -180,6 +182,148 @@ __global__ void __launch_bounds__(256) cross_attn_kernel(const T* __restrict__ q
   Vec16<T>::store(out + static_cast<long long>(row) * d + col, acc);
 }
 
+// LOCAL_GLOBAL cross-attention with the request's window staged in shared
+// memory.  One CTA per (32 query rows, request): the window's key and value
+// rows (at most kWin) and the anchor are copied once into shared memory; warp
+// w takes heads w, w + 8, ..., and lane i the query row 32 c + i, so the 32
+// lanes of a warp read the same key/value elements (shared-memory broadcast).
+// Each thread computes all the row's scores for the head, the softmax and the
+// weighted values in registers.
+constexpr int kWin = 16;
+
+struct CrossLgArgs {
+  const int* cand_off;  // [R+1] candidate offsets (device)
+  int n_cand, S;
+  const int* kv_off;    // [R+1] cache row offsets
+  const int* kv_len;    // [R]
+  const float* Kg;      // [R, d] anchor key / value of this layer, fp32
+  const float* Vg;
+  int l_local, H, d;
+  float scale_log2;     // log2(e) / sqrt(d_h)
+};
+
+template <typename T, int DH>
+__global__ void __launch_bounds__(256) cross_lg_kernel(const T* __restrict__ q_in, T* __restrict__ out,
+                                                       const T* __restrict__ Kc, const T* __restrict__ Vc,
+                                                       const CrossLgArgs a) {
+  pdl_launch_dependents();
+  pdl_wait();
+  extern __shared__ __align__(16) uint8_t smem_lg[];
+  const int d = a.d;
+  T* sK = reinterpret_cast<T*>(smem_lg);                      // [kWin][d]
+  T* sV = sK + kWin * d;                                      // [kWin][d]
+  float* sKg = reinterpret_cast<float*>(sV + kWin * d);       // [d]
+  float* sVg = sKg + d;                                       // [d]
+  const int r = blockIdx.y;
+  const int c0 = __ldg(a.cand_off + r);
+  const int M = __ldg(a.cand_off + r + 1) - c0;
+  const int n_q = M + a.S;
+  const int row0 = blockIdx.x * 32;
+  if (row0 >= n_q) return;                                    // uniform
+  const int len = __ldg(a.kv_len + r);
+  const int lo = len > a.l_local ? len - a.l_local : 0;
+  const int W = len - lo;                                     // <= kWin (checked on the host)
+  const long long base = static_cast<long long>(__ldg(a.kv_off + r)) + lo;
+  {
+    constexpr int VE = Vec16<T>::N;                           // elements per 16 bytes
+    const int per_row = d / VE;
+    for (int i = threadIdx.x; i < W * per_row; i += blockDim.x) {
+      const int t = i / per_row, c = (i - t * per_row) * VE;
+      *reinterpret_cast<uint4*>(sK + t * d + c) = *reinterpret_cast<const uint4*>(Kc + (base + t) * d + c);
+      *reinterpret_cast<uint4*>(sV + t * d + c) = *reinterpret_cast<const uint4*>(Vc + (base + t) * d + c);
+    }
+    for (int i = threadIdx.x; i < d; i += blockDim.x) {
+      sKg[i] = __ldg(a.Kg + static_cast<long long>(r) * d + i);
+      sVg[i] = __ldg(a.Vg + static_cast<long long>(r) * d + i);
+    }
+  }
+  __syncthreads();
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int j = row0 + lane;                                  // query row within the request
+  const bool valid = j < n_q;
+  const long long grow = j < M ? static_cast<long long>(c0) + j
+                               : a.n_cand + static_cast<long long>(r) * a.S + (j - M);
+  for (int h = warp; h < a.H; h += (blockDim.x >> 5)) {
+    const int col = h * DH;
+    float q[DH];
+    if (valid) {
+#pragma unroll
+      for (int c = 0; c < DH; c += Vec16<T>::N) Vec16<T>::load(q_in + grow * d + col + c, q + c);
+    } else {
+#pragma unroll
+      for (int c = 0; c < DH; ++c) q[c] = 0.f;
+    }
+#pragma unroll
+    for (int c = 0; c < DH; ++c) q[c] *= a.scale_log2;
+    // scores (log2 units): the window rows, then the anchor
+    float sc[kWin + 1];
+#pragma unroll
+    for (int t = 0; t < kWin; ++t) {
+      float dot = -INFINITY;
+      if (t < W) {
+        dot = 0.f;
+#pragma unroll
+        for (int c = 0; c < DH; c += Vec16<T>::N) {
+          float k[Vec16<T>::N];
+          Vec16<T>::load(sK + t * d + col + c, k);
+#pragma unroll
+          for (int i = 0; i < Vec16<T>::N; ++i) dot = fmaf(q[c + i], k[i], dot);
+        }
+      }
+      sc[t] = dot;
+    }
+    {
+      float dot = 0.f;
+#pragma unroll
+      for (int c = 0; c < DH; c += 4) {
+        const float4 k4 = *reinterpret_cast<const float4*>(sKg + col + c);
+        dot = fmaf(q[c], k4.x, dot);
+        dot = fmaf(q[c + 1], k4.y, dot);
+        dot = fmaf(q[c + 2], k4.z, dot);
+        dot = fmaf(q[c + 3], k4.w, dot);
+      }
+      sc[kWin] = dot;
+    }
+    float mx = sc[kWin];
+#pragma unroll
+    for (int t = 0; t < kWin; ++t) mx = fmaxf(mx, sc[t]);
+    float sum = 0.f;
+#pragma unroll
+    for (int t = 0; t <= kWin; ++t) {
+      sc[t] = exp2f(sc[t] - mx);
+      sum += sc[t];
+    }
+    // weighted values (q reused as the accumulator)
+#pragma unroll
+    for (int c = 0; c < DH; c += 4) {
+      const float4 v4 = *reinterpret_cast<const float4*>(sVg + col + c);
+      q[c] = sc[kWin] * v4.x;
+      q[c + 1] = sc[kWin] * v4.y;
+      q[c + 2] = sc[kWin] * v4.z;
+      q[c + 3] = sc[kWin] * v4.w;
+    }
+#pragma unroll
+    for (int t = 0; t < kWin; ++t) {
+      if (t < W) {
+#pragma unroll
+        for (int c = 0; c < DH; c += Vec16<T>::N) {
+          float v[Vec16<T>::N];
+          Vec16<T>::load(sV + t * d + col + c, v);
+#pragma unroll
+          for (int i = 0; i < Vec16<T>::N; ++i) q[c + i] = fmaf(sc[t], v[i], q[c + i]);
+        }
+      }
+    }
+    if (valid) {
+      const float inv = 1.f / sum;
+#pragma unroll
+      for (int c = 0; c < DH; ++c) q[c] *= inv;
+#pragma unroll
+      for (int c = 0; c < DH; c += Vec16<T>::N) Vec16<T>::store(out + grow * d + col + c, q + c);
+    }
+  }
+}
+
 template <typename T, int DH>
 cudaError_t cross_launch(const T* q, T* out, const T* Kc, const T* Vc, CrossArgs a, cudaStream_t s) {
   const long long threads = static_cast<long long>(a.n_rows) * a.H * Group<T, DH>::TPH;
@@ -230,6 +374,41 @@ cudaError_t launch_cross_attn(const T* q, T* out, const T* Kc, const T* Vc, cons
   prof_end(KC_ATTN_CROSS, s);
   return err;
 }
+
+template <typename T>
+cudaError_t launch_cross_attn_lg(const T* q, T* out, const T* Kc, const T* Vc, const int* cand_off_dev,
+                                 const int* cand_off_host, int n_req, int n_cand, int S, const int* kv_off,
+                                 const int* kv_len, const float* Kg, const float* Vg, int l_local, int H, int d,
+                                 cudaStream_t s) {
+  const int dh = d / H;
+  if (l_local > kWin || (dh != 32 && dh != 64) || d % 8 != 0) return cudaErrorNotSupported;
+  int max_q = 0;
+  for (int r = 0; r < n_req; ++r) max_q = std::max(max_q, cand_off_host[r + 1] - cand_off_host[r] + S);
+  if (max_q == 0 || n_req == 0) return cudaSuccess;
+  CrossLgArgs a{cand_off_dev, n_cand, S, kv_off, kv_len, Kg, Vg, l_local, H, d,
+                1.4426950408889634f / sqrtf(static_cast<float>(dh))};
+  const size_t smem = static_cast<size_t>(2 * kWin * d) * sizeof(T) + 2 * d * sizeof(float);
+  const dim3 grid((max_q + 31) / 32, n_req);
+  prof_begin(KC_ATTN_CROSS, s);
+  cudaError_t err;
+  if (dh == 32) {
+    if (smem > 48 * 1024) cudaFuncSetAttribute(cross_lg_kernel<T, 32>, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
+    err = launch_pdl(cross_lg_kernel<T, 32>, grid, dim3(256), smem, s, q, out, Kc, Vc, a);
+  } else {
+    if (smem > 48 * 1024) cudaFuncSetAttribute(cross_lg_kernel<T, 64>, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
+    err = launch_pdl(cross_lg_kernel<T, 64>, grid, dim3(256), smem, s, q, out, Kc, Vc, a);
+  }
+  prof_end(KC_ATTN_CROSS, s);
+  return err;
+}
+
+template cudaError_t launch_cross_attn_lg<float>(const float*, float*, const float*, const float*, const int*,
+                                                 const int*, int, int, int, const int*, const int*, const float*,
+                                                 const float*, int, int, int, cudaStream_t);
+template cudaError_t launch_cross_attn_lg<__nv_bfloat16>(const __nv_bfloat16*, __nv_bfloat16*, const __nv_bfloat16*,
+                                                         const __nv_bfloat16*, const int*, const int*, int, int, int,
+                                                         const int*, const int*, const float*, const float*, int,
+                                                         int, int, cudaStream_t);
 
 template cudaError_t launch_serving_attn<float>(const float*, float*, const int*, int, int, int, int, int, cudaStream_t);
 template cudaError_t launch_serving_attn<__nv_bfloat16>(const __nv_bfloat16*, __nv_bfloat16*, const int*, int, int,

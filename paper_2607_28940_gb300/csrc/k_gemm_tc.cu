@@ -45,6 +45,7 @@ __device__ __forceinline__ int find_seg_gen(const int* off, int n, int row) {
 }
 
 constexpr int kStageN = 4096;     // bias entries staged in shared memory
+constexpr int kStageNRes = 1024;  // the same with a resident B slice (less room)
 constexpr int kStageSeg = 1024;   // request offsets staged in shared memory (cache-row remap)
 
 
@@ -93,18 +94,39 @@ __device__ __forceinline__ void epilogue(const EpiArgs& e, uint32_t tacc, int ro
     }
     if (valid) out = static_cast<__nv_bfloat16*>(e.out) + orow * e.ldo + ocol;
     tma_ok = __all_sync(0xffffffffu, tma_ok);
+    if constexpr (HALF % 64 == 0) {
+      // 64 columns per TMEM load (one wait), two bulk-stored chunks
 #pragma unroll 1
-    for (int c = 0; c < HALF; c += 32) {
-      tmem_ld32(tacc + c0 + c, v);
-      float b[32];
-      load_f32x32_gen(bias + n0 + c0 + c, b);
+      for (int c = 0; c < HALF; c += 64) {
+        float w[64];
+        tmem_ld64(tacc + c0 + c, w);
 #pragma unroll
-      for (int i = 0; i < 32; ++i) {
-        float x = v[i] + b[i];
-        if constexpr (EPI == EPI_BIAS_GELU) x = gelu_erf(x);
-        v[i] = x;
+        for (int hh = 0; hh < 64; hh += 32) {
+          float b[32];
+          load_f32x32_gen(bias + n0 + c0 + c + hh, b);
+#pragma unroll
+          for (int i = 0; i < 32; ++i) {
+            float x = w[hh + i] + b[i];
+            if constexpr (EPI == EPI_BIAS_GELU) x = gelu_erf(x);
+            w[hh + i] = x;
+          }
+          store_chunk(w + hh, out + c + hh, valid, tma_ok, tmO, tx + c + hh, ty, stage, kchunk++, lane);
+        }
       }
-      store_chunk(v, out + c, valid, tma_ok, tmO, tx + c, ty, stage, kchunk++, lane);
+    } else {
+#pragma unroll 1
+      for (int c = 0; c < HALF; c += 32) {
+        tmem_ld32(tacc + c0 + c, v);
+        float b[32];
+        load_f32x32_gen(bias + n0 + c0 + c, b);
+#pragma unroll
+        for (int i = 0; i < 32; ++i) {
+          float x = v[i] + b[i];
+          if constexpr (EPI == EPI_BIAS_GELU) x = gelu_erf(x);
+          v[i] = x;
+        }
+        store_chunk(v, out + c, valid, tma_ok, tmO, tx + c, ty, stage, kchunk++, lane);
+      }
     }
   } else {
     // Row LayerNorm over the full row (BN == N): two passes over TMEM, the
@@ -230,12 +252,12 @@ struct Shape {
   static constexpr bool LN = EPI == EPI_LN || EPI == EPI_LN_HEAD;
   static constexpr int RED_BYTES = LN ? 2 * 128 * kRedStride * 4 : 0;
   static constexpr int WEFF_BYTES = EPI == EPI_LN_HEAD ? BN * NAP * 4 : 0;
-  // bias [kStageN] floats (not with BRES), then (cache-row remap) offsets and
+  // bias [kStageN] floats ([kStageNRes] with BRES), then (cache-row remap) offsets and
   // first rows; rounded to 1 KB so that the staging buffers after it start on
   // a swizzle-atom boundary
   static constexpr int AUX_BYTES =
       LN ? 0
-         : (((BRES ? 0 : kStageN * 4) + (EPI == EPI_KV ? (2 * kStageSeg + 1) * 4 : 0) + 1023) / 1024) * 1024;
+         : (((BRES ? kStageNRes * 4 : kStageN * 4) + (EPI == EPI_KV ? (2 * kStageSeg + 1) * 4 : 0) + 1023) / 1024) * 1024;
   // bulk-store staging: two 2 KB buffers per epilogue warp (bf16 outputs)
   static constexpr int STG_BYTES = EPI == EPI_LN_HEAD ? 0 : kEpiWarps * 2 * 2048;
   static constexpr int EXTRA = BRES_BYTES + RED_BYTES + WEFF_BYTES + AUX_BYTES + STG_BYTES + 1024 + 256;
@@ -275,7 +297,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   float* red = reinterpret_cast<float*>(sBres + S::BRES_BYTES);
   float* s_weff = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(red) + S::RED_BYTES);
   float* s_bias = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(s_weff) + S::WEFF_BYTES);
-  int* s_seg = reinterpret_cast<int*>(s_bias + (BRES ? 0 : kStageN));
+  int* s_seg = reinterpret_cast<int*>(s_bias + (BRES ? kStageNRes : kStageN));
   int* s_dst = s_seg + kStageSeg + 1;
   uint8_t* s_stage = reinterpret_cast<uint8_t*>(s_bias) + S::AUX_BYTES;
   uint64_t* full = reinterpret_cast<uint64_t*>(s_stage + S::STG_BYTES);
@@ -337,7 +359,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   const int* seg_off = e.seg_off;
   const int* dst_row0 = e.dst_row0;
   if constexpr (!S::LN) {
-    if (!BRES && e.N <= kStageN) {
+    if (e.N <= (BRES ? kStageNRes : kStageN)) {
       for (int i = threadIdx.x; i < e.N; i += NUM_THREADS) s_bias[i] = e.bias[i];
       bias = s_bias;
     }

@@ -407,7 +407,13 @@ txs_status score_impl(txs_model* m, const txs_kv_cache* c, int n_req, const int3
     const T* Vc = kv + (size_t(2 * l + 1) * c->cap_total) * d;
     const float* Kg = c->gkv + size_t(2 * l) * n_req * d;
     const float* Vg = c->gkv + size_t(2 * l + 1) * n_req * d;
-    if constexpr (std::is_same<T, __nv_bfloat16>::value) {
+    cudaError_t lg = cudaErrorNotSupported;
+    if (cf.attn_mode == TXS_ATTN_LOCAL_GLOBAL)
+      lg = launch_cross_attn_lg<T>(QKV, A, Kc, Vc, cand_off_dev, cand_off, n_req, static_cast<int>(n_cand), S,
+                                   c->d_off, c->d_len, Kg, Vg, cf.l_local, H, d, s);
+    if (lg != cudaErrorNotSupported) {
+      if (lg != cudaSuccess) return fail_cuda("cross-attention", lg);
+    } else if constexpr (std::is_same<T, __nv_bfloat16>::value) {
       if (cf.attn_mode == TXS_ATTN_FULL && fa_full_supported(d, H, c->cap_total)) {
         TXS_CK(launch_fa_full(QKV, A, Kc, Vc, c->cap_total, cand_off_dev, cand_off, c->d_off, c->d_len, n_req,
                               static_cast<int>(n_cand), S, H, d, m->status, s));

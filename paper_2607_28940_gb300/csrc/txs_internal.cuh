@@ -167,6 +167,13 @@ bool tc_gemm_supported(int N, int K, int epi);
 template <typename T>
 cudaError_t launch_serving_attn(const T* qkv, T* out, const int* row_req, int n_rows, int n_cand_rows, int S, int H,
                                 int d, cudaStream_t s);
+// LOCAL_GLOBAL cross-attention with the window in shared memory; cudaErrorNotSupported
+// when the window is longer than 16 rows or d_h is not 32 / 64.
+template <typename T>
+cudaError_t launch_cross_attn_lg(const T* q, T* out, const T* Kc, const T* Vc, const int* cand_off_dev,
+                                 const int* cand_off_host, int n_req, int n_cand, int S, const int* kv_off,
+                                 const int* kv_len, const float* Kg, const float* Vg, int l_local, int H, int d,
+                                 cudaStream_t s);
 template <typename T>
 cudaError_t launch_cross_attn(const T* q, T* out, const T* Kc, const T* Vc, const int* row_req, int n_rows,
                               const int* kv_off, const int* kv_len, const float* Kg, const float* Vg, int l_local,
