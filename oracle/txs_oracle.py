@@ -30,6 +30,9 @@ What it computes (row-vector convention ``y = x W + b``):
   ``= Q_dec k_dec`` (no scale), probabilities ``= softmax(logits)``.
 * Ranking: per request, candidates by descending probability of one action,
   ties to the lower candidate index.
+* Streaming multi-event scoring (Sec. 4.2 prefix reuse, Sec. 5.1 per-event
+  global token): event t of a user is scored against the behavior prefix
+  before it, exactly as a request whose history is that prefix.
 
 Readings where the paper is silent (LN eps 1e-5 with biased variance, exact erf
 GELU, k = 4 actions, S = 2 context tokens, the serving-stream mask) are listed
@@ -281,6 +284,33 @@ def score_batch(model: Model, caches: List[RequestCache], ctx: np.ndarray, cand:
     lg, pr = [], []
     for r, c in enumerate(caches):
         a, b = score_request(model, c, ctx[r], cand[cand_off[r]:cand_off[r + 1]], mode, use_global)
+        lg.append(a)
+        pr.append(b)
+    return np.concatenate(lg, axis=0), np.concatenate(pr, axis=0)
+
+
+# ---------------------------------------------------------------- streaming events
+
+def score_events(model: Model, phi: np.ndarray, ends: Sequence[int], ctx: np.ndarray, cand: np.ndarray,
+                 cand_off: Sequence[int], mode: int = LOCAL_GLOBAL, use_global: bool = True):
+    """Multi-event scoring of one user in the streaming form (Sec. 4.2, causal
+    attention and prefix reuse; Sec. 5.1, a global token for each event
+    timestamp).  Event t sees only the behavior prefix ``phi[:ends[t]]``: its
+    key set is the most recent L_local rows of that prefix plus the anchor
+    pooled over that prefix (LOCAL_GLOBAL), or the whole prefix (FULL).  Its
+    slate is ``cand[cand_off[t]:cand_off[t + 1]]`` with context rows
+    ``ctx[t]``.  Written as the definition: one cache per event, built from
+    the prefix alone.  Returns concatenated (logits, probs) over all events."""
+    phi = np.asarray(phi, dtype=np.float64)
+    lg, pr = [], []
+    for t, e in enumerate(ends):
+        e = int(e)
+        if e <= 0:
+            raise ValueError("cold start: an event with no behavior rows before it")
+        if e > phi.shape[0]:
+            raise ValueError("event end beyond the behavior stream")
+        cache = build_cache(model, phi[:e])
+        a, b = score_request(model, cache, ctx[t], cand[cand_off[t]:cand_off[t + 1]], mode, use_global)
         lg.append(a)
         pr.append(b)
     return np.concatenate(lg, axis=0), np.concatenate(pr, axis=0)

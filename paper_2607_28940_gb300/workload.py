@@ -221,6 +221,36 @@ def batch(wl: Workload, requests: Optional[Sequence[int]] = None,
     )
 
 
+@dataclass
+class Events:
+    """One user's behavior stream and T serving events (streaming form).
+
+    ``beh``  [L, d]        encoded behavior rows Phi_b of the whole stream
+    ``ends`` [T]           rows of the stream before each event (1 <= end <= L)
+    ``ctx``  [T, S, d]     each event's context tokens
+    ``cand`` [sum m_t, d]  each event's candidate tokens, packed by ``cand_off``
+    """
+    beh: np.ndarray
+    ends: np.ndarray
+    ctx: np.ndarray
+    cand: np.ndarray
+    cand_off: np.ndarray
+
+
+def events(wl: Workload, L: int, T: int, m: Union[int, Sequence[int]], seed: int) -> Events:
+    """Draw a stream of L rows and T events; event ends are uniform in
+    [1, L] (sorted, the last one L), slates of m_t candidates."""
+    rng = np.random.default_rng(seed)
+    d, S = wl.d_model, wl.n_ctx
+    beh = rng.standard_normal((L, d), dtype=np.float32)
+    ends = np.sort(rng.integers(1, L + 1, size=T)).astype(np.int32)
+    ends[-1] = L
+    ms = np.full(T, int(m), dtype=np.int64) if np.isscalar(m) else np.asarray(m, dtype=np.int64)
+    ctx = rng.standard_normal((T, S, d), dtype=np.float32)
+    cand = rng.standard_normal((int(ms.sum()), d), dtype=np.float32)
+    return Events(_store(wl, beh), ends, _store(wl, ctx), _store(wl, cand), _offsets(ms))
+
+
 def with_sizes(wl: Workload, **kw) -> Workload:
     """A copy of ``wl`` with some fields replaced (e.g. a smaller L or M)."""
     return replace(wl, **kw)

@@ -157,3 +157,40 @@ def test_planted_mistake_is_caught(name, monkeypatch):
     monkeypatch.setattr(O, attr, fn)
     gaps = [_gap(model, phi, ctx, cand, mode) for mode in (O.LOCAL_GLOBAL, O.FULL)]
     assert max(gaps) > 1e-9, f"mutation {name} went unnoticed (gaps {gaps})"
+
+
+# ---------------------------------------------------------------- streaming events
+
+def _events_gap(model, ev, mode=O.LOCAL_GLOBAL):
+    lg, _ = O.score_events(model, ev.beh, ev.ends, ev.ctx, ev.cand, ev.cand_off, mode)
+    gap = 0.0
+    for t, e in enumerate(ev.ends):
+        sl = slice(ev.cand_off[t], ev.cand_off[t + 1])
+        rl, _ = torch_score(model, np.asarray(ev.beh[:e], np.float64), np.asarray(ev.ctx[t], np.float64),
+                            np.asarray(ev.cand[sl], np.float64), mode)
+        gap = max(gap, float(np.abs(lg[sl] - rl).max()))
+    return gap
+
+
+def test_event_mistakes_are_caught(monkeypatch):
+    wl, model, _, _, _ = _setup()
+    ev = W.events(wl, 30, 4, 3, 21)
+    ev.ends[:3] = [4, 12, 19]
+    assert _events_gap(model, ev) < 1e-10
+    orig_build = O.build_cache
+
+    # anchor pooled over the whole stream instead of the event's prefix
+    def build_with_stream_anchor(m, phi):
+        c = orig_build(m, phi)
+        full = orig_build(m, ev.beh)
+        return O.RequestCache(c.K, c.V, full.pool, full.Kg, full.Vg)
+    monkeypatch.setattr(O, "build_cache", build_with_stream_anchor)
+    assert _events_gap(model, ev) > 1e-4
+    monkeypatch.setattr(O, "build_cache", orig_build)
+
+    # window taken from the end of the stream instead of the event's prefix
+    def build_with_stream_rows(m, phi):
+        c = orig_build(m, ev.beh)
+        return O.RequestCache(c.K, c.V, orig_build(m, phi).pool, orig_build(m, phi).Kg, orig_build(m, phi).Vg)
+    monkeypatch.setattr(O, "build_cache", build_with_stream_rows)
+    assert _events_gap(model, ev) > 1e-4
