@@ -323,6 +323,7 @@ def run_txs(args, rank, world):
         out["e2e"] = e2e(txs, torch, model, cache, b, wl, args, dt, logits, probs, ranks, ws, world)
         if rank == 0:
             out["latency_vs_L"] = latency_sweep(txs, torch)
+            out["events"] = events_bench(txs, torch)
             out["cpu_baseline"] = cpu_baseline(args.workload, budget_s=12.0)
     return out
 
@@ -415,6 +416,64 @@ def latency_sweep(txs, torch):
             cache.close()
         res[mode_name] = p50
         res[f"{mode_name}_ratio_16384_over_1024"] = p50["16384"] / p50["1024"]
+        model.close()
+    return res
+
+
+EV_WORKLOAD = "mid_bf16"     # model dims of the streaming multi-event measurement
+EV_L, EV_T, EV_M = 8192, 64, 256
+
+
+def events_bench(txs, torch):
+    """Streaming multi-event scoring (txs_score_events): one user's stream of
+    EV_L rows cached once, EV_T events at sorted prefix ends, EV_M candidates
+    each; candidates/s and events/s over repeated calls, L2 flushed before
+    each call, plus the per-class time of one call."""
+    base = W.WORKLOADS[EV_WORKLOAD]
+    wl = W.with_sizes(base, n_req=1, L=EV_L, M=1, dL=0)
+    res = {"workload": f"{EV_WORKLOAD} model (d={base.d_model}, {base.n_layers} layers), one user with L={EV_L} "
+                       f"rows, T={EV_T} events at uniform sorted prefix ends, {EV_M} candidates per event",
+           "unit": "candidates/s"}
+    ev = W.events(wl, EV_L, EV_T, EV_M, 20267)
+    dt = txs.torch_dtype(wl.dtype)
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device="cuda")
+    for mode_name, mode in (("local_global", txs.LOCAL_GLOBAL), ("full", txs.FULL)):
+        model = txs.Model(wl, W.weights(wl), mode)
+        beh = txs.to_device(ev.beh, dt)
+        cache = txs.KVCache(model, np.array([0, EV_L], dtype=np.int32), beh)
+        cand = txs.to_device(ev.cand, dt)
+        ctx = txs.to_device(ev.ctx.reshape(-1, wl.d_model), dt)
+        n_cand = int(ev.cand_off[-1])
+        ws = torch.empty(txs.events_workspace_bytes(model, EV_T, n_cand, int(ev.ends.max())), dtype=torch.uint8,
+                         device="cuda")
+        lg = torch.empty((n_cand, wl.n_actions), dtype=torch.float32, device="cuda")
+        pr = torch.empty_like(lg)
+        call = lambda: txs.score_events(model, cache, 0, beh, ev.ends, ev.cand_off, cand, ctx, workspace=ws,
+                                        out_logits=lg, out_probs=pr)
+        for _ in range(3):
+            call()
+        times = []
+        for _ in range(10):
+            flush.zero_()
+            e0 = torch.cuda.Event(enable_timing=True)
+            e1 = torch.cuda.Event(enable_timing=True)
+            e0.record()
+            call()
+            e1.record()
+            e1.synchronize()
+            times.append(e0.elapsed_time(e1))
+        txs.profile_enable(True)
+        call()
+        torch.cuda.synchronize()
+        prof = txs.profile_collect()
+        txs.profile_enable(False)
+        ms = statistics.median(times)
+        res[mode_name] = {"ms_per_call": ms, "candidates_per_s": n_cand / (ms / 1e3),
+                          "events_per_s": EV_T / (ms / 1e3),
+                          "kernels_ms": {k: v[0] for k, v in prof.items()}}
+        if model.device_status() != txs.TXS_OK:
+            raise RuntimeError("device status after the events measurement")
+        cache.close()
         model.close()
     return res
 

@@ -187,6 +187,41 @@ txs_status txs_score_candidates(txs_model* model, const txs_kv_cache* cache, int
                                 float* out_logits, float* out_probs, void* stream);
 
 /*
+ * txs_events_workspace_size — bytes of device scratch txs_score_events needs
+ * for n_events events with total_cand candidates in all, the longest event
+ * prefix being max_event_end rows.
+ */
+txs_status txs_events_workspace_size(const txs_model* model, int32_t n_events, int64_t total_cand,
+                                     int32_t max_event_end, size_t* bytes);
+
+/*
+ * txs_score_events — streaming multi-event scoring of one user (Sec. 4.2,
+ * causal attention and prefix reuse: each serving event slices the behavior
+ * prefix before it; Sec. 5.1, a global token pooled for each event timestamp).
+ *
+ * `user` selects a request of `cache` whose rows hold the whole behavior
+ * stream; beh_enc (device, model dtype, [L_user, d_model]) are the encoded
+ * rows the cache was built (and appended) from, in order.  Event t sees the
+ * first event_ends[t] rows only (1 <= event_ends[t] <= L_user, host int32
+ * [n_events], any order): its key set is the most recent l_local of those
+ * rows plus the anchor pooled over them (LOCAL_GLOBAL), or all of them
+ * (FULL).  Event t's candidates are cand_tok[cand_offsets[t] ..
+ * cand_offsets[t+1]) (device, [sum m_t, d_model]) and its context tokens
+ * ctx_tok[t] (device, [n_events, n_ctx, d_model]; NULL iff n_ctx == 0).
+ * Outputs as for txs_score_candidates, packed by cand_offsets (host int32
+ * [n_events + 1]).  The cached K/V rows are reused, not recomputed; the
+ * per-event anchors are pooled from beh_enc into `workspace` (device, >=
+ * txs_events_workspace_size bytes, 256-byte aligned, caller-owned).
+ * Errors: TXS_ERR_COLD_START for an event end of 0, TXS_ERR_INVALID_ARG for
+ * an end beyond the user's rows or a bad argument, TXS_ERR_STALE_CACHE,
+ * TXS_ERR_UNSUPPORTED for more than 4096 events or d_model > 512.
+ */
+txs_status txs_score_events(txs_model* model, const txs_kv_cache* cache, int32_t user, const void* beh_enc,
+                            int32_t n_events, const int32_t* event_ends, const int32_t* cand_offsets,
+                            const void* cand_tok, const void* ctx_tok, void* workspace, size_t workspace_bytes,
+                            float* out_logits, float* out_probs, void* stream);
+
+/*
  * txs_rank_candidates — per request, candidate indices (local to the request)
  * sorted by descending probs[:, action]; ties go to the lower index and NaN
  * scores rank last.  `probs` device float [sum M_r, n_actions].

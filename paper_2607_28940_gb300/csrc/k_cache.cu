@@ -8,6 +8,8 @@
 // acc = sum exp(logit - m) phi) so that an append (App. D incremental-encoding
 // remark) merges new rows without revisiting old ones.  Rows are processed in
 // chunks of kPoolChunk (one CTA each); chunk states are merged per request.
+#include <algorithm>
+
 #include "txs_internal.cuh"
 
 namespace txs {
@@ -24,12 +26,15 @@ constexpr int kPoolRowsPerWarp = kPoolChunkV / kPoolWarps;
 // (all loads issued before any arithmetic), computes the pooling logits with a
 // warp reduction and folds the rows into an online-softmax state; the CTA then
 // merges its warps' states.  One coalesced read of the behavior rows.
-template <typename T, int MAXC>
+// MERGE = false (prefix pooling of a stream): only the chunk states are
+// written; seg_off is then null and the rows are [0, n_fixed).
+template <typename T, int MAXC, bool MERGE = true>
 __global__ void __launch_bounds__(256) pool_partial_kernel(const T* __restrict__ phi, const int* __restrict__ seg_off,
                                                            const float* __restrict__ w_pool, int d, float inv_sqrt_d,
                                                            int max_chunks, float* __restrict__ part,
                                                            int merge_existing, float* st_m, float* st_s,
-                                                           float* st_acc, float* __restrict__ g, int* counter) {
+                                                           float* st_acc, float* __restrict__ g, int* counter,
+                                                           int n_fixed) {
   pdl_launch_dependents();
   pdl_wait();
   constexpr int VEC = Vec16<T>::N;               // MAXC: 16-byte chunks per lane, ceil(d / (32 VEC))
@@ -37,7 +42,7 @@ __global__ void __launch_bounds__(256) pool_partial_kernel(const T* __restrict__
   __shared__ float sm_acc[kPoolWarps][512];
   const int r = blockIdx.y, c = blockIdx.x;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int seg_beg = seg_off[r], seg_end = seg_off[r + 1];
+  const int seg_beg = MERGE ? seg_off[r] : 0, seg_end = MERGE ? seg_off[r + 1] : n_fixed;
   const int beg = seg_beg + c * kPoolChunkV;
   const int nrows = min(seg_end - beg, kPoolChunkV);
   float* out = part + (static_cast<long long>(r) * max_chunks + c) * (d + 2);
@@ -154,6 +159,7 @@ __global__ void __launch_bounds__(256) pool_partial_kernel(const T* __restrict__
     out[0] = M;
     out[1] = S;
   }
+  if constexpr (!MERGE) return;
   // The last chunk CTA of request r to finish merges the request's chunk states
   // (and, for an append, the stored state) and writes g = acc / s.
   __shared__ int is_last;
@@ -337,13 +343,13 @@ cudaError_t launch_pool(const T* phi, const int* seg_off, int R, int max_rows, c
   prof_begin(KC_POOL, s);
   if (nch == 1)
     err0 = launch_pdl(pool_partial_kernel<T, 1>, grid, dim3(256), 0, s, phi, seg_off, w_pool, d, isd, max_chunks,
-                      part, merge_existing, st_m, st_s, st_acc, g, counter);
+                      part, merge_existing, st_m, st_s, st_acc, g, counter, 0);
   else if (nch == 2)
     err0 = launch_pdl(pool_partial_kernel<T, 2>, grid, dim3(256), 0, s, phi, seg_off, w_pool, d, isd, max_chunks,
-                      part, merge_existing, st_m, st_s, st_acc, g, counter);
+                      part, merge_existing, st_m, st_s, st_acc, g, counter, 0);
   else if (nch <= 4)
     err0 = launch_pdl(pool_partial_kernel<T, 4>, grid, dim3(256), 0, s, phi, seg_off, w_pool, d, isd, max_chunks,
-                      part, merge_existing, st_m, st_s, st_acc, g, counter);
+                      part, merge_existing, st_m, st_s, st_acc, g, counter, 0);
   else
     return cudaErrorInvalidValue;
   cudaError_t err = err0 != cudaSuccess ? err0 : cudaGetLastError();
@@ -401,9 +407,184 @@ cudaError_t launch_hash(const void* p, long long bytes, uint64_t salt, unsigned 
   return cudaGetLastError();
 }
 
+// ------------------------------------------------------------------ prefix pooling
+
+// Streaming events (Sec. 4.2 prefix reuse; Sec. 5.1 a global token for each
+// event timestamp): event t's anchor is the attention pooling of the first
+// ends[t] behavior rows of the user.  The stream is pooled once in chunks of
+// kPoolChunkV rows (pool_partial_kernel, no merge); then one CTA per event
+// merges the states of the chunks wholly inside its prefix with the rows of
+// the last, partial chunk (online-softmax merge: every term rescaled to the
+// common maximum).  The CTA also writes the event's cache view: first row
+// off_user, length ends[t].
+constexpr int kEvMax = 4096;
+
+struct PrefixPoolArgs {
+  int n_ev;
+  int off_user;
+  int ends[kEvMax];
+};
+
+template <typename T, int MAXC>
+__global__ void __launch_bounds__(256) prefix_finish_kernel(const T* __restrict__ phi,
+                                                            const float* __restrict__ w_pool, int d,
+                                                            float inv_sqrt_d, const float* __restrict__ part,
+                                                            float* __restrict__ g, int* __restrict__ ev_off,
+                                                            int* __restrict__ ev_len,
+                                                            const __grid_constant__ PrefixPoolArgs a) {
+  pdl_launch_dependents();
+  pdl_wait();
+  constexpr int VEC = Vec16<T>::N;
+  constexpr int W = 8;
+  __shared__ float sm_m[W], sm_s[W];
+  extern __shared__ float sm_acc[];                      // [W][d]
+  const int t = blockIdx.x;
+  const int end = a.ends[t];
+  const int nfull = end / kPoolChunkV;                   // chunks wholly inside the prefix
+  const int beg = nfull * kPoolChunkV;                   // rows [beg, end) pooled here
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (threadIdx.x == 0) {
+    ev_off[t] = a.off_user;
+    ev_len[t] = end;
+  }
+  const int nch = (d + 32 * VEC - 1) / (32 * VEC);      // 16-byte vectors per lane
+  float w[MAXC][VEC], acc[MAXC][VEC];
+#pragma unroll
+  for (int j = 0; j < MAXC; ++j)
+#pragma unroll
+    for (int i = 0; i < VEC; ++i) {
+      const int col = (j * 32 + lane) * VEC + i;
+      w[j][i] = (j < nch && col < d) ? __ldg(w_pool + col) : 0.f;
+      acc[j][i] = 0.f;
+    }
+  float m = -INFINITY, ssum = 0.f;
+  for (int row = beg + warp; row < end; row += W) {
+    const T* pr = phi + static_cast<long long>(row) * d;
+    float x[MAXC][VEC];
+    float dot = 0.f;
+#pragma unroll
+    for (int j = 0; j < MAXC; ++j) {
+      const int col = (j * 32 + lane) * VEC;
+      if (j < nch && col < d) {
+        Vec16<T>::load(pr + col, x[j]);
+      } else {
+#pragma unroll
+        for (int i = 0; i < VEC; ++i) x[j][i] = 0.f;
+      }
+#pragma unroll
+      for (int i = 0; i < VEC; ++i) dot = fmaf(x[j][i], w[j][i], dot);
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) dot += __shfl_xor_sync(0xffffffffu, dot, o);
+    const float lg = dot * inv_sqrt_d;
+    const float mn = fmaxf(m, lg);
+    const float corr = expf(m - mn);                     // 0 on the first row
+    const float p = expf(lg - mn);
+    ssum = ssum * corr + p;
+#pragma unroll
+    for (int j = 0; j < MAXC; ++j)
+#pragma unroll
+      for (int i = 0; i < VEC; ++i) acc[j][i] = fmaf(acc[j][i], corr, p * x[j][i]);
+    m = mn;
+  }
+  if (lane == 0) {
+    sm_m[warp] = m;
+    sm_s[warp] = ssum;
+  }
+#pragma unroll
+  for (int j = 0; j < MAXC; ++j)
+#pragma unroll
+    for (int i = 0; i < VEC; ++i) {
+      const int col = (j * 32 + lane) * VEC + i;
+      if (j < nch && col < d) sm_acc[warp * d + col] = acc[j][i];
+    }
+  __syncthreads();
+  // common maximum over the full chunks and the warps' partial states
+  float M = -INFINITY;
+  for (int c = 0; c < nfull; ++c) M = fmaxf(M, __ldg(part + static_cast<long long>(c) * (d + 2)));
+#pragma unroll
+  for (int k = 0; k < W; ++k) M = fmaxf(M, sm_m[k]);
+  float S = 0.f;
+  for (int c = 0; c < nfull; ++c) {
+    const float* pc = part + static_cast<long long>(c) * (d + 2);
+    S = fmaf(__ldg(pc + 1), expf(__ldg(pc) - M), S);
+  }
+  float scale[W];
+#pragma unroll
+  for (int k = 0; k < W; ++k) {
+    scale[k] = sm_s[k] > 0.f ? expf(sm_m[k] - M) : 0.f;  // a warp with no rows contributes nothing
+    S = fmaf(sm_s[k], scale[k], S);
+  }
+  const float inv = 1.f / S;
+  for (int col = threadIdx.x; col < d; col += blockDim.x) {
+    float v = 0.f;
+#pragma unroll
+    for (int k = 0; k < W; ++k) v = fmaf(sm_acc[k * d + col], scale[k], v);
+    for (int c = 0; c < nfull; ++c) {
+      const float* pc = part + static_cast<long long>(c) * (d + 2);
+      v = fmaf(__ldg(pc + 2 + col), expf(__ldg(pc) - M), v);
+    }
+    g[static_cast<long long>(t) * d + col] = v * inv;
+  }
+}
+
+size_t prefix_pool_scratch_floats(int max_end, int d) {
+  return static_cast<size_t>((max_end + kPoolChunkV - 1) / kPoolChunkV) * (d + 2);
+}
+
+template <typename T>
+cudaError_t launch_prefix_pool(const T* phi, const int* ends, int n_ev, int off_user, const float* w_pool, int d,
+                               float* part, float* g, int* ev_off, int* ev_len, cudaStream_t s) {
+  if (n_ev <= 0) return cudaSuccess;
+  if (n_ev > kEvMax) return cudaErrorInvalidValue;
+  PrefixPoolArgs a;
+  a.n_ev = n_ev;
+  a.off_user = off_user;
+  int max_end = 0;
+  for (int t = 0; t < n_ev; ++t) {
+    a.ends[t] = ends[t];
+    max_end = std::max(max_end, ends[t]);
+  }
+  constexpr int VEC = Vec16<T>::N;
+  const int nch = (d + 32 * VEC - 1) / (32 * VEC);
+  if (nch > 4 || d > 512) return cudaErrorInvalidValue;
+  const float isd = 1.0f / sqrtf(static_cast<float>(d));
+  const size_t smem = static_cast<size_t>(8) * d * sizeof(float);
+  const int n_chunks = max_end / kPoolChunkV;           // only whole chunks are pooled ahead
+  prof_begin(KC_POOL, s);
+  cudaError_t err = cudaSuccess;
+  if (n_chunks > 0) {
+    const dim3 grid(n_chunks, 1);
+    if (nch <= 1)
+      err = launch_pdl(pool_partial_kernel<T, 1, false>, grid, dim3(256), 0, s, phi, nullptr, w_pool, d, isd, n_chunks,
+                       part, 0, nullptr, nullptr, nullptr, nullptr, nullptr, max_end);
+    else if (nch <= 2)
+      err = launch_pdl(pool_partial_kernel<T, 2, false>, grid, dim3(256), 0, s, phi, nullptr, w_pool, d, isd, n_chunks,
+                       part, 0, nullptr, nullptr, nullptr, nullptr, nullptr, max_end);
+    else
+      err = launch_pdl(pool_partial_kernel<T, 4, false>, grid, dim3(256), 0, s, phi, nullptr, w_pool, d, isd, n_chunks,
+                       part, 0, nullptr, nullptr, nullptr, nullptr, nullptr, max_end);
+  }
+  if (err == cudaSuccess) {
+    if (nch <= 1)
+      err = launch_pdl(prefix_finish_kernel<T, 1>, dim3(n_ev), dim3(256), smem, s, phi, w_pool, d, isd, part, g,
+                       ev_off, ev_len, a);
+    else if (nch <= 2)
+      err = launch_pdl(prefix_finish_kernel<T, 2>, dim3(n_ev), dim3(256), smem, s, phi, w_pool, d, isd, part, g,
+                       ev_off, ev_len, a);
+    else
+      err = launch_pdl(prefix_finish_kernel<T, 4>, dim3(n_ev), dim3(256), smem, s, phi, w_pool, d, isd, part, g,
+                       ev_off, ev_len, a);
+  }
+  prof_end(KC_POOL, s);
+  return err;
+}
+
 #define TXS_INST(T)                                                                                                 \
   template cudaError_t launch_pool<T>(const T*, const int*, int, int, const float*, int, int, float*, int, float*, \
                                       float*, float*, float*, int*, cudaStream_t);                                  \
+  template cudaError_t launch_prefix_pool<T>(const T*, const int*, int, int, const float*, int, float*, float*,     \
+                                             int*, int*, cudaStream_t);                                             \
   template cudaError_t launch_anchor_proj<T>(const float*, const T*, const float*, float*, int, int, int,          \
                                              cudaStream_t);                                                         \
   template cudaError_t launch_transpose<T>(const T*, T*, int, int, cudaStream_t);                                  \

@@ -355,8 +355,19 @@ txs_status project_rows(txs_model* m, txs_kv_cache* c, int n_req, const int32_t*
   return TXS_OK;
 }
 
+// What one scoring pass reads of the cache: unit r (a request, or an event of
+// a user) sees rows [off[r], off[r] + len[r]) of every layer's K/V and the
+// anchor projections gkv[l][0|1][r].
+struct KvView {
+  const void* kv;          // [nL][2][cap_total][d]
+  long long cap_total;
+  const int* off;          // device [n]
+  const int* len;          // device [n]
+  const float* gkv;        // device [nL][2][n][d]
+};
+
 template <typename T>
-txs_status score_impl(txs_model* m, const txs_kv_cache* c, int n_req, const int32_t* cand_off, const void* cand_tok,
+txs_status score_impl(txs_model* m, const KvView& c, int n_req, const int32_t* cand_off, const void* cand_tok,
                       const void* ctx_tok, void* ws, float* logits, float* probs, cudaStream_t s) {
   const txs_config& cf = m->cfg;
   const int d = cf.d_model, F = cf.d_ff, H = cf.n_heads, S = cf.n_ctx, k = cf.n_actions;
@@ -377,7 +388,7 @@ txs_status score_impl(txs_model* m, const txs_kv_cache* c, int n_req, const int3
 
   TXS_CK(launch_pack<T>(n_req, cand_off, S, d, k, static_cast<const T*>(cand_tok), static_cast<const T*>(ctx_tok), X,
                         row_req, cand_off_dev, m->weff + size_t(d) * k, m->cdec, xlog, s));
-  const T* kv = static_cast<const T*>(c->kv);
+  const T* kv = static_cast<const T*>(c.kv);
   for (int l = 0; l < cf.n_layers; ++l) {
     const LayerW& W = m->layers[l];
     // serving-stream attention (App. B mask), O-projection + residual + LN1
@@ -403,26 +414,26 @@ txs_status score_impl(txs_model* m, const txs_kv_cache* c, int n_req, const int3
     e.out = QKV;
     e.ldo = d;
     TXS_CK(gemm(m, X1, d, W.Wt_q, e, tmp, s, KC_GEMM_Q));
-    const T* Kc = kv + (size_t(2 * l) * c->cap_total) * d;
-    const T* Vc = kv + (size_t(2 * l + 1) * c->cap_total) * d;
-    const float* Kg = c->gkv + size_t(2 * l) * n_req * d;
-    const float* Vg = c->gkv + size_t(2 * l + 1) * n_req * d;
+    const T* Kc = kv + (size_t(2 * l) * c.cap_total) * d;
+    const T* Vc = kv + (size_t(2 * l + 1) * c.cap_total) * d;
+    const float* Kg = c.gkv + size_t(2 * l) * n_req * d;
+    const float* Vg = c.gkv + size_t(2 * l + 1) * n_req * d;
     cudaError_t lg = cudaErrorNotSupported;
     if (cf.attn_mode == TXS_ATTN_LOCAL_GLOBAL)
       lg = launch_cross_attn_lg<T>(QKV, A, Kc, Vc, cand_off_dev, cand_off, n_req, static_cast<int>(n_cand), S,
-                                   c->d_off, c->d_len, Kg, Vg, cf.l_local, H, d, s);
+                                   c.off, c.len, Kg, Vg, cf.l_local, H, d, s);
     if (lg != cudaErrorNotSupported) {
       if (lg != cudaSuccess) return fail_cuda("cross-attention", lg);
     } else if constexpr (std::is_same<T, __nv_bfloat16>::value) {
-      if (cf.attn_mode == TXS_ATTN_FULL && fa_full_supported(d, H, c->cap_total)) {
-        TXS_CK(launch_fa_full(QKV, A, Kc, Vc, c->cap_total, cand_off_dev, cand_off, c->d_off, c->d_len, n_req,
+      if (cf.attn_mode == TXS_ATTN_FULL && fa_full_supported(d, H, c.cap_total)) {
+        TXS_CK(launch_fa_full(QKV, A, Kc, Vc, c.cap_total, cand_off_dev, cand_off, c.off, c.len, n_req,
                               static_cast<int>(n_cand), S, H, d, m->status, s));
       } else {
-        TXS_CK(launch_cross_attn<T>(QKV, A, Kc, Vc, row_req, static_cast<int>(N), c->d_off, c->d_len, Kg, Vg,
+        TXS_CK(launch_cross_attn<T>(QKV, A, Kc, Vc, row_req, static_cast<int>(N), c.off, c.len, Kg, Vg,
                                     cf.l_local, cf.attn_mode, H, d, s));
       }
     } else {
-      TXS_CK(launch_cross_attn<T>(QKV, A, Kc, Vc, row_req, static_cast<int>(N), c->d_off, c->d_len, Kg, Vg,
+      TXS_CK(launch_cross_attn<T>(QKV, A, Kc, Vc, row_req, static_cast<int>(N), c.off, c.len, Kg, Vg,
                                   cf.l_local, cf.attn_mode, H, d, s));
     }
     e = epi_base(EPI_LN, N, d, d);
@@ -737,10 +748,99 @@ TXS_API txs_status txs_score_candidates(txs_model* m, const txs_kv_cache* c, int
     return TXS_ERR_INVALID_ARG;
   if (workspace_bytes < score_layout(cf, m->es, n_req, n_cand).total) return TXS_ERR_INVALID_ARG;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const KvView v{c->kv, c->cap_total, c->d_off, c->d_len, c->gkv};
   return cf.dtype == TXS_BF16
-             ? score_impl<__nv_bfloat16>(m, c, n_req, cand_offsets, cand_tok, ctx_tok, workspace, out_logits,
+             ? score_impl<__nv_bfloat16>(m, v, n_req, cand_offsets, cand_tok, ctx_tok, workspace, out_logits,
                                          out_probs, s)
-             : score_impl<float>(m, c, n_req, cand_offsets, cand_tok, ctx_tok, workspace, out_logits, out_probs, s);
+             : score_impl<float>(m, v, n_req, cand_offsets, cand_tok, ctx_tok, workspace, out_logits, out_probs, s);
+}
+
+// Streaming events: the score workspace, then per event its cache view
+// (first row, length), pooled anchor g and the anchor's K/V projections.
+struct EventsLayout {
+  size_t score, ev_off, ev_len, g, gkv, part, total;
+};
+EventsLayout events_layout(const txs_config& cf, int es, int n_ev, long long n_cand, int max_end) {
+  EventsLayout L;
+  size_t o = score_layout(cf, es, n_ev, n_cand).total;
+  auto take = [&](size_t bytes) {
+    const size_t at = o;
+    o += (bytes + 255) / 256 * 256;
+    return at;
+  };
+  L.score = 0;
+  L.ev_off = take(sizeof(int) * n_ev);
+  L.ev_len = take(sizeof(int) * n_ev);
+  L.g = take(sizeof(float) * n_ev * cf.d_model);
+  L.gkv = take(sizeof(float) * 2 * cf.n_layers * n_ev * cf.d_model);
+  L.part = take(sizeof(float) * prefix_pool_scratch_floats(max_end, cf.d_model));
+  L.total = o;
+  return L;
+}
+
+TXS_API txs_status txs_events_workspace_size(const txs_model* m, int32_t n_events, int64_t total_cand,
+                                             int32_t max_event_end, size_t* bytes) {
+  if (!m || !bytes || n_events < 0 || total_cand < 0 || max_event_end < 0) return TXS_ERR_INVALID_ARG;
+  *bytes = events_layout(m->cfg, m->es, n_events, total_cand, max_event_end).total;
+  return TXS_OK;
+}
+
+template <typename T>
+txs_status events_impl(txs_model* m, const txs_kv_cache* c, int user, const void* beh_enc, int n_ev,
+                       const int32_t* ends, const int32_t* cand_off, const void* cand_tok, const void* ctx_tok,
+                       void* ws, float* logits, float* probs, cudaStream_t s) {
+  const txs_config& cf = m->cfg;
+  const int d = cf.d_model, nL = cf.n_layers;
+  int max_end = 0;
+  for (int t = 0; t < n_ev; ++t) max_end = std::max(max_end, static_cast<int>(ends[t]));
+  const EventsLayout L = events_layout(cf, sizeof(T), n_ev, cand_off[n_ev], max_end);
+  uint8_t* base = static_cast<uint8_t*>(ws);
+  int* ev_off = reinterpret_cast<int*>(base + L.ev_off);
+  int* ev_len = reinterpret_cast<int*>(base + L.ev_len);
+  float* g = reinterpret_cast<float*>(base + L.g);
+  float* gkv = reinterpret_cast<float*>(base + L.gkv);
+  float* part = reinterpret_cast<float*>(base + L.part);
+  // per-event anchors pooled over each prefix, projected by every layer's W_K, W_V
+  TXS_CK(launch_prefix_pool<T>(static_cast<const T*>(beh_enc), ends, n_ev, c->h_off[user], m->w_pool, d, part, g,
+                               ev_off, ev_len, s));
+  TXS_CK(launch_anchor_proj<T>(g, static_cast<const T*>(m->Wt_kv), m->b_kv, gkv, n_ev, d, nL, s));
+  const KvView v{c->kv, c->cap_total, ev_off, ev_len, gkv};
+  return score_impl<T>(m, v, n_ev, cand_off, cand_tok, ctx_tok, ws, logits, probs, s);
+}
+
+TXS_API txs_status txs_score_events(txs_model* m, const txs_kv_cache* c, int32_t user, const void* beh_enc,
+                                    int32_t n_events, const int32_t* event_ends, const int32_t* cand_offsets,
+                                    const void* cand_tok, const void* ctx_tok, void* workspace,
+                                    size_t workspace_bytes, float* out_logits, float* out_probs, void* stream) {
+  if (!m || !c || !event_ends || !cand_offsets || n_events < 0) return TXS_ERR_INVALID_ARG;
+  if (c->model_hash != m->hash) return TXS_ERR_STALE_CACHE;
+  if (user < 0 || user >= c->n_req) return TXS_ERR_INVALID_ARG;
+  if (n_events == 0) return TXS_OK;
+  if (n_events > kMaxReqParam) return TXS_ERR_UNSUPPORTED;
+  if (!offsets_ok(cand_offsets, n_events, false)) return TXS_ERR_INVALID_ARG;
+  for (int t = 0; t < n_events; ++t) {
+    if (event_ends[t] == 0) return TXS_ERR_COLD_START;
+    if (event_ends[t] < 0 || event_ends[t] > c->h_len[user]) return TXS_ERR_INVALID_ARG;
+  }
+  const txs_config& cf = m->cfg;
+  const long long n_cand = cand_offsets[n_events];
+  if (n_cand + static_cast<long long>(n_events) * cf.n_ctx > 0x7FFFFFFFLL) return TXS_ERR_UNSUPPORTED;
+  if (n_cand == 0) return TXS_OK;
+  if (!beh_enc || !cand_tok || !out_logits || (cf.n_ctx > 0 && !ctx_tok) || !workspace) return TXS_ERR_INVALID_ARG;
+  if (reinterpret_cast<uintptr_t>(workspace) & 255) return TXS_ERR_INVALID_ARG;
+  if ((reinterpret_cast<uintptr_t>(cand_tok) & 15) || (ctx_tok && (reinterpret_cast<uintptr_t>(ctx_tok) & 15)) ||
+      (reinterpret_cast<uintptr_t>(beh_enc) & 15))
+    return TXS_ERR_INVALID_ARG;
+  int max_end = 0;
+  for (int t = 0; t < n_events; ++t) max_end = std::max(max_end, static_cast<int>(event_ends[t]));
+  if (cf.d_model > 512) return TXS_ERR_UNSUPPORTED;
+  if (workspace_bytes < events_layout(cf, m->es, n_events, n_cand, max_end).total) return TXS_ERR_INVALID_ARG;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  return cf.dtype == TXS_BF16
+             ? events_impl<__nv_bfloat16>(m, c, user, beh_enc, n_events, event_ends, cand_offsets, cand_tok, ctx_tok,
+                                          workspace, out_logits, out_probs, s)
+             : events_impl<float>(m, c, user, beh_enc, n_events, event_ends, cand_offsets, cand_tok, ctx_tok,
+                                  workspace, out_logits, out_probs, s);
 }
 
 TXS_API txs_status txs_rank_candidates(int32_t n_req, const int32_t* cand_offsets, const float* probs,

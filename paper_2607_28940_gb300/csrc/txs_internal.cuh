@@ -192,6 +192,14 @@ template <typename T>
 cudaError_t launch_pool(const T* phi, const int* seg_off, int R, int max_rows, const float* w_pool, int d,
                         int max_chunks, float* part, int merge_existing, float* st_m, float* st_s, float* st_acc,
                         float* g, int* counter, cudaStream_t s);
+// Per-event anchors of one user's stream: g[t] = attention pooling of
+// phi[0 .. ends[t]); also writes ev_off[t] = off_user, ev_len[t] = ends[t]
+// (ends: host, at most 4096 events; d <= 512).  `part`: scratch of
+// prefix_pool_scratch_floats(max end, d) floats.
+size_t prefix_pool_scratch_floats(int max_end, int d);
+template <typename T>
+cudaError_t launch_prefix_pool(const T* phi, const int* ends, int n_ev, int off_user, const float* w_pool, int d,
+                               float* part, float* g, int* ev_off, int* ev_len, cudaStream_t s);
 template <typename T>
 cudaError_t launch_anchor_proj(const float* g, const T* Wt_kv, const float* b_kv, float* gkv, int R, int d,
                                int n_layers, cudaStream_t s);

@@ -71,6 +71,8 @@ _SIGS = {
     "txs_score_workspace_size": (_I32, [_P, _I32, ctypes.c_int64, ctypes.POINTER(ctypes.c_size_t)]),
     "txs_score_candidates": (_I32, [_P, _P, _I32, _I32P, _P, _P, _P, ctypes.c_size_t, _P, _P, _P]),
     "txs_rank_candidates": (_I32, [_I32, _I32P, _P, _I32, _I32, _I32, _P, _P]),
+    "txs_events_workspace_size": (_I32, [_P, _I32, ctypes.c_int64, _I32, ctypes.POINTER(ctypes.c_size_t)]),
+    "txs_score_events": (_I32, [_P, _P, _I32, _P, _I32, _I32P, _I32P, _P, _P, _P, ctypes.c_size_t, _P, _P, _P]),
     "txs_device_status": (_I32, [_P]),
     "txs_pool_anchor_static": (_I32, [_P, _I32, _I32P, _P, _P, _P]),
     "txs_profile_enable": (_I32, [_I32]),
@@ -257,6 +259,41 @@ def score(model: Model, cache: KVCache, cand_offsets, cand_tok: torch.Tensor, ct
     _check(lib().txs_score_candidates(model.handle, cache.handle, n_req, p, _ptr(cand_tok), _ptr(ctx_tok),
                                       _ptr(workspace), workspace.numel(), _ptr(out_logits), _ptr(out_probs),
                                       _stream(stream)), "txs_score_candidates")
+    return out_logits, out_probs
+
+
+def events_workspace_bytes(model: Model, n_events: int, total_cand: int, max_event_end: int) -> int:
+    n = ctypes.c_size_t()
+    _check(lib().txs_events_workspace_size(model.handle, n_events, total_cand, max_event_end, ctypes.byref(n)),
+           "events_workspace_size")
+    return int(n.value)
+
+
+def score_events(model: Model, cache: KVCache, user: int, beh_enc: torch.Tensor, event_ends, cand_offsets,
+                 cand_tok: torch.Tensor, ctx_tok: Optional[torch.Tensor], workspace: Optional[torch.Tensor] = None,
+                 out_logits: Optional[torch.Tensor] = None, out_probs: Optional[torch.Tensor] = None,
+                 want_probs: bool = True, stream=None):
+    """Streaming multi-event scores of request ``user`` of ``cache`` (txs_score_events):
+    event t sees the first event_ends[t] rows of the user's stream ``beh_enc``."""
+    ends = np.ascontiguousarray(np.asarray(event_ends, dtype=np.int32))
+    off, p = _offsets(cand_offsets)
+    n_ev = len(off) - 1
+    if len(ends) != n_ev:
+        raise ValueError("one event end per slate")
+    n_cand = int(off[-1])
+    k = model.wl.n_actions
+    if workspace is None:
+        max_end = int(ends.max()) if len(ends) else 0
+        workspace = torch.empty(max(events_workspace_bytes(model, n_ev, n_cand, max_end), 256), dtype=torch.uint8,
+                                device="cuda")
+    if out_logits is None:
+        out_logits = torch.empty((n_cand, k), dtype=torch.float32, device="cuda")
+    if out_probs is None and want_probs:
+        out_probs = torch.empty((n_cand, k), dtype=torch.float32, device="cuda")
+    _check(lib().txs_score_events(model.handle, cache.handle, int(user), _ptr(beh_enc), n_ev,
+                                  ends.ctypes.data_as(_I32P), p, _ptr(cand_tok), _ptr(ctx_tok), _ptr(workspace),
+                                  workspace.numel(), _ptr(out_logits), _ptr(out_probs), _stream(stream)),
+           "txs_score_events")
     return out_logits, out_probs
 
 
