@@ -152,6 +152,30 @@ txs_status txs_cache_read_rows(const txs_kv_cache* cache, int32_t layer, int32_t
  * into dst (device, float, [n_req, d]). */
 txs_status txs_cache_read_anchor(const txs_kv_cache* cache, int32_t layer, int32_t which, float* dst, void* stream);
 
+/*
+ * Cache export / import (App. D cache management: warm start from a
+ * persisted cache; entries versioned by the model identifier and the feature
+ * schema, stale entries never reused).  The host blob holds a header (format
+ * version, model hash, schema_version, sizes), the request lengths, each
+ * layer's cached K and V rows (current lengths only, not spare capacity), the
+ * pooling state and the anchor with its per-layer projections.
+ *
+ * txs_cache_export_size: bytes of the blob of `cache`.
+ * txs_cache_export: writes the blob into host_buf (caller-owned, >= that many
+ *   bytes); synchronises `stream` before returning.
+ * txs_cache_import: builds a new cache from a blob for `model`, with
+ *   capacity_extra spare rows per request; scores, appends and reads of it
+ *   give exactly what the exported cache gave.  Synchronises `stream` (the
+ *   blob may be freed on return).  Errors: TXS_ERR_STALE_CACHE if the blob
+ *   was written for another model hash or schema_version, TXS_ERR_INVALID_ARG
+ *   for a blob that is not one (bad magic or format, truncated, inconsistent).
+ */
+txs_status txs_cache_export_size(const txs_kv_cache* cache, size_t* bytes);
+txs_status txs_cache_export(const txs_kv_cache* cache, uint32_t schema_version, void* host_buf, size_t bytes,
+                            void* stream);
+txs_status txs_cache_import(txs_model* model, uint32_t schema_version, const void* host_buf, size_t bytes,
+                            int32_t capacity_extra, void* stream, txs_kv_cache** out);
+
 /* Current per-request lengths L_r (host int32 [n_req]) and request count. */
 txs_status txs_cache_lengths(const txs_kv_cache* cache, int32_t* out_len);
 int32_t txs_cache_n_req(const txs_kv_cache* cache);

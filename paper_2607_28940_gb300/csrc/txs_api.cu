@@ -554,18 +554,13 @@ TXS_API void txs_model_destroy(txs_model* m) {
 
 TXS_API uint64_t txs_model_hash(const txs_model* m) { return m ? m->hash : 0; }
 
-TXS_API txs_status txs_build_kv_cache(txs_model* m, int32_t n_req, const int32_t* beh_offsets, const void* beh_enc,
-                                      int32_t capacity_extra, void* stream, txs_kv_cache** out) {
-  if (!m || !out || n_req < 1 || capacity_extra < 0 || !beh_offsets) return TXS_ERR_INVALID_ARG;
-  *out = nullptr;
-  if (!offsets_ok(beh_offsets, n_req, false)) return TXS_ERR_INVALID_ARG;
-  for (int r = 0; r < n_req; ++r)
-    if (beh_offsets[r + 1] == beh_offsets[r]) return TXS_ERR_COLD_START;
-  if (!beh_enc) return TXS_ERR_INVALID_ARG;
-  if (n_req > kMaxReqParam) return TXS_ERR_UNSUPPORTED;
+// A cache of n_req requests of the given lengths (each with capacity_extra
+// spare rows), its device arrays allocated and its offsets and lengths
+// uploaded; the K/V rows and pooling state are left for the caller to fill.
+txs_status make_cache(txs_model* m, int n_req, const int* lengths, int capacity_extra, cudaStream_t s,
+                      txs_kv_cache** out) {
   const txs_config& cf = m->cfg;
   const int d = cf.d_model, nL = cf.n_layers;
-  cudaStream_t s = static_cast<cudaStream_t>(stream);
   txs_kv_cache* c = new txs_kv_cache();
   c->n_req = n_req;
   c->n_layers = nL;
@@ -579,7 +574,7 @@ TXS_API txs_status txs_build_kv_cache(txs_model* m, int32_t n_req, const int32_t
   long long tot = 0;
   int max_cap = 0;
   for (int r = 0; r < n_req; ++r) {
-    c->h_len[r] = beh_offsets[r + 1] - beh_offsets[r];
+    c->h_len[r] = lengths[r];
     c->h_cap[r] = c->h_len[r] + capacity_extra;
     max_cap = std::max(max_cap, c->h_cap[r]);
     c->h_off[r] = static_cast<int>(tot);
@@ -629,6 +624,31 @@ TXS_API txs_status txs_build_kv_cache(txs_model* m, int32_t n_req, const int32_t
         (err = stage_upload(c, c->d_len, c->h_len.data(), n_req, s)) != cudaSuccess)
       st = fail_cuda("upload", err);
   }
+  if (st != TXS_OK) {
+    cudaStreamSynchronize(s);
+    txs_cache_destroy(c);
+    return st;
+  }
+  *out = c;
+  return TXS_OK;
+}
+
+TXS_API txs_status txs_build_kv_cache(txs_model* m, int32_t n_req, const int32_t* beh_offsets, const void* beh_enc,
+                                      int32_t capacity_extra, void* stream, txs_kv_cache** out) {
+  if (!m || !out || n_req < 1 || capacity_extra < 0 || !beh_offsets) return TXS_ERR_INVALID_ARG;
+  *out = nullptr;
+  if (!offsets_ok(beh_offsets, n_req, false)) return TXS_ERR_INVALID_ARG;
+  for (int r = 0; r < n_req; ++r)
+    if (beh_offsets[r + 1] == beh_offsets[r]) return TXS_ERR_COLD_START;
+  if (!beh_enc) return TXS_ERR_INVALID_ARG;
+  if (n_req > kMaxReqParam) return TXS_ERR_UNSUPPORTED;
+  const txs_config& cf = m->cfg;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  std::vector<int> lengths(n_req);
+  for (int r = 0; r < n_req; ++r) lengths[r] = beh_offsets[r + 1] - beh_offsets[r];
+  txs_kv_cache* c = nullptr;
+  txs_status st = make_cache(m, n_req, lengths.data(), capacity_extra, s, &c);
+  if (st != TXS_OK) return st;
   if (st == TXS_OK)
     st = cf.dtype == TXS_BF16 ? project_rows<__nv_bfloat16>(m, c, n_req, beh_offsets, beh_enc, false, s)
                               : project_rows<float>(m, c, n_req, beh_offsets, beh_enc, false, s);
@@ -636,6 +656,142 @@ TXS_API txs_status txs_build_kv_cache(txs_model* m, int32_t n_req, const int32_t
     cudaStreamSynchronize(s);
     txs_cache_destroy(c);
     return st;
+  }
+  *out = c;
+  return TXS_OK;
+}
+
+// ------------------------------------------------------------------ cache export / import
+
+// Serialised cache (host memory): header, lengths, each layer's K and V rows
+// of every request (no spare capacity), then the pooling state (m, s, acc),
+// the pooled anchor g and its projections.  Entries are versioned by the
+// model hash and a caller-given feature-schema version (App. D cache
+// management: versioning and consistency).
+namespace {
+constexpr char kCacheMagic[8] = {'T', 'X', 'S', 'C', 'A', 'C', 'H', 'E'};
+constexpr uint32_t kCacheFormat = 1;
+struct CacheHeader {
+  char magic[8];
+  uint32_t format, schema;
+  uint64_t model_hash;
+  int32_t n_req, n_layers, d_model, elem_bytes;
+  int64_t total_rows;
+};
+size_t cache_blob_bytes(int n_req, int nL, int d, int es, long long rows) {
+  return sizeof(CacheHeader) + sizeof(int32_t) * n_req + size_t(nL) * 2 * rows * d * es +
+         sizeof(float) * (2 * size_t(n_req) + size_t(2) * n_req * d + size_t(nL) * 2 * n_req * d);
+}
+}  // namespace
+
+TXS_API txs_status txs_cache_export_size(const txs_kv_cache* c, size_t* bytes) {
+  if (!c || !bytes) return TXS_ERR_INVALID_ARG;
+  long long rows = 0;
+  for (int r = 0; r < c->n_req; ++r) rows += c->h_len[r];
+  *bytes = cache_blob_bytes(c->n_req, c->n_layers, c->d, c->es, rows);
+  return TXS_OK;
+}
+
+TXS_API txs_status txs_cache_export(const txs_kv_cache* c, uint32_t schema_version, void* host_buf, size_t bytes,
+                                    void* stream) {
+  if (!c || !host_buf) return TXS_ERR_INVALID_ARG;
+  size_t need = 0;
+  txs_cache_export_size(c, &need);
+  if (bytes < need) return TXS_ERR_INVALID_ARG;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const int R = c->n_req, nL = c->n_layers, d = c->d, es = c->es;
+  uint8_t* p = static_cast<uint8_t*>(host_buf);
+  CacheHeader h;
+  std::memcpy(h.magic, kCacheMagic, 8);
+  h.format = kCacheFormat;
+  h.schema = schema_version;
+  h.model_hash = c->model_hash;
+  h.n_req = R;
+  h.n_layers = nL;
+  h.d_model = d;
+  h.elem_bytes = es;
+  h.total_rows = 0;
+  for (int r = 0; r < R; ++r) h.total_rows += c->h_len[r];
+  std::memcpy(p, &h, sizeof(h));
+  p += sizeof(h);
+  std::memcpy(p, c->h_len.data(), sizeof(int32_t) * R);
+  p += sizeof(int32_t) * R;
+  cudaError_t err = cudaSuccess;
+  const uint8_t* kv = static_cast<const uint8_t*>(c->kv);
+  for (int l = 0; l < nL && err == cudaSuccess; ++l)
+    for (int w = 0; w < 2 && err == cudaSuccess; ++w)
+      for (int r = 0; r < R && err == cudaSuccess; ++r) {
+        const size_t n = size_t(c->h_len[r]) * d * es;
+        const size_t src = ((size_t(2 * l + w) * c->cap_total) + c->h_off[r]) * d * es;
+        err = cudaMemcpyAsync(p, kv + src, n, cudaMemcpyDeviceToHost, s);
+        p += n;
+      }
+  auto grab = [&](const float* src, size_t n) {
+    if (err == cudaSuccess) err = cudaMemcpyAsync(p, src, sizeof(float) * n, cudaMemcpyDeviceToHost, s);
+    p += sizeof(float) * n;
+  };
+  grab(c->pool_m, R);
+  grab(c->pool_s, R);
+  grab(c->pool_acc, size_t(R) * d);
+  grab(c->g, size_t(R) * d);
+  grab(c->gkv, size_t(nL) * 2 * R * d);
+  if (err == cudaSuccess) err = cudaStreamSynchronize(s);
+  if (err != cudaSuccess) return fail_cuda("cache export", err);
+  return TXS_OK;
+}
+
+TXS_API txs_status txs_cache_import(txs_model* m, uint32_t schema_version, const void* host_buf, size_t bytes,
+                                    int32_t capacity_extra, void* stream, txs_kv_cache** out) {
+  if (!m || !host_buf || !out || capacity_extra < 0) return TXS_ERR_INVALID_ARG;
+  *out = nullptr;
+  if (bytes < sizeof(CacheHeader)) return TXS_ERR_INVALID_ARG;
+  CacheHeader h;
+  std::memcpy(&h, host_buf, sizeof(h));
+  if (std::memcmp(h.magic, kCacheMagic, 8) != 0 || h.format != kCacheFormat) return TXS_ERR_INVALID_ARG;
+  // entries of another model or feature schema are stale, never reinterpreted
+  if (h.model_hash != m->hash || h.schema != schema_version) return TXS_ERR_STALE_CACHE;
+  const txs_config& cf = m->cfg;
+  if (h.n_layers != cf.n_layers || h.d_model != cf.d_model || h.elem_bytes != m->es) return TXS_ERR_STALE_CACHE;
+  if (h.n_req < 1 || h.n_req > kMaxReqParam || h.total_rows < 0) return TXS_ERR_INVALID_ARG;
+  const int R = h.n_req, nL = h.n_layers, d = h.d_model, es = h.elem_bytes;
+  if (bytes < sizeof(h) + sizeof(int32_t) * R) return TXS_ERR_INVALID_ARG;
+  std::vector<int> len(R);
+  std::memcpy(len.data(), static_cast<const uint8_t*>(host_buf) + sizeof(h), sizeof(int32_t) * R);
+  long long rows = 0;
+  for (int r = 0; r < R; ++r) {
+    if (len[r] < 1) return TXS_ERR_INVALID_ARG;
+    rows += len[r];
+  }
+  if (rows != h.total_rows || bytes < cache_blob_bytes(R, nL, d, es, rows)) return TXS_ERR_INVALID_ARG;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  txs_kv_cache* c = nullptr;
+  txs_status st = make_cache(m, R, len.data(), capacity_extra, s, &c);
+  if (st != TXS_OK) return st;
+  const uint8_t* p = static_cast<const uint8_t*>(host_buf) + sizeof(h) + sizeof(int32_t) * R;
+  cudaError_t err = cudaSuccess;
+  uint8_t* kv = static_cast<uint8_t*>(c->kv);
+  for (int l = 0; l < nL && err == cudaSuccess; ++l)
+    for (int w = 0; w < 2 && err == cudaSuccess; ++w)
+      for (int r = 0; r < R && err == cudaSuccess; ++r) {
+        const size_t n = size_t(len[r]) * d * es;
+        const size_t dst = ((size_t(2 * l + w) * c->cap_total) + c->h_off[r]) * d * es;
+        err = cudaMemcpyAsync(kv + dst, p, n, cudaMemcpyHostToDevice, s);
+        p += n;
+      }
+  auto put = [&](float* dst, size_t n) {
+    if (err == cudaSuccess) err = cudaMemcpyAsync(dst, p, sizeof(float) * n, cudaMemcpyHostToDevice, s);
+    p += sizeof(float) * n;
+  };
+  put(c->pool_m, R);
+  put(c->pool_s, R);
+  put(c->pool_acc, size_t(R) * d);
+  put(c->g, size_t(R) * d);
+  put(c->gkv, size_t(nL) * 2 * R * d);
+  // the host buffer may be released as soon as this returns
+  if (err == cudaSuccess) err = cudaStreamSynchronize(s);
+  if (err != cudaSuccess) {
+    txs_cache_destroy(c);
+    return fail_cuda("cache import", err);
   }
   *out = c;
   return TXS_OK;

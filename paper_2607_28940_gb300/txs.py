@@ -67,6 +67,9 @@ _SIGS = {
     "txs_cache_read_rows": (_I32, [_P, _I32, _I32, _I32, _I32, _I32, _P, _P]),
     "txs_cache_read_anchor": (_I32, [_P, _I32, _I32, _P, _P]),
     "txs_cache_lengths": (_I32, [_P, _I32P]),
+    "txs_cache_export_size": (_I32, [_P, ctypes.POINTER(ctypes.c_size_t)]),
+    "txs_cache_export": (_I32, [_P, ctypes.c_uint32, _P, ctypes.c_size_t, _P]),
+    "txs_cache_import": (_I32, [_P, ctypes.c_uint32, _P, ctypes.c_size_t, _I32, _P, ctypes.POINTER(_P)]),
     "txs_cache_n_req": (_I32, [_P]),
     "txs_score_workspace_size": (_I32, [_P, _I32, ctypes.c_int64, ctypes.POINTER(ctypes.c_size_t)]),
     "txs_score_candidates": (_I32, [_P, _P, _I32, _I32P, _P, _P, _P, ctypes.c_size_t, _P, _P, _P]),
@@ -223,6 +226,29 @@ class KVCache:
         _check(lib().txs_cache_read_anchor(self.handle, layer, which, _ptr(out), _stream(stream)),
                "txs_cache_read_anchor")
         return out
+
+    def export(self, schema_version: int = 0, stream=None) -> np.ndarray:
+        """The cache serialised into a host byte array (txs_cache_export)."""
+        n = ctypes.c_size_t()
+        _check(lib().txs_cache_export_size(self.handle, ctypes.byref(n)), "txs_cache_export_size")
+        buf = np.empty(int(n.value), dtype=np.uint8)
+        _check(lib().txs_cache_export(self.handle, int(schema_version), buf.ctypes.data, buf.size, _stream(stream)),
+               "txs_cache_export")
+        return buf
+
+    @classmethod
+    def import_blob(cls, model: Model, blob: np.ndarray, schema_version: int = 0, capacity_extra: int = 0,
+                    stream=None) -> "KVCache":
+        """A cache rebuilt from an exported blob (txs_cache_import)."""
+        blob = np.ascontiguousarray(blob, dtype=np.uint8)
+        h = _P()
+        _check(lib().txs_cache_import(model.handle, int(schema_version), blob.ctypes.data, blob.size,
+                                      int(capacity_extra), _stream(stream), ctypes.byref(h)), "txs_cache_import")
+        self = cls.__new__(cls)
+        self.model = model
+        self.handle = h
+        self.n_req = int(lib().txs_cache_n_req(h))
+        return self
 
     def close(self):
         if getattr(self, "handle", None):
