@@ -15,6 +15,9 @@ What it computes (row-vector convention ``y = x W + b``):
   ``g = alpha^T Phi_b``, projected by each layer's ``W_K``/``W_V``.  The pooling
   state (running max m, running sum s, weighted sum acc) is kept so that an
   incremental append (App. D, incremental-encoding remark) can merge new rows.
+* Grouped K/V heads (the MQA/GQA variants Sec. 4.1.2 cites): the cache may
+  hold n_kv_heads < n_heads key/value heads (W_K, W_V of width n_kv_heads *
+  d_h); query head h attends with key/value head h // (n_heads / n_kv_heads).
 * Key set I_t (Sec. 4.1.2): LOCAL_GLOBAL uses the most recent L_local rows plus
   the global token; FULL ("-sparseAttn", Sec. 5.2) uses all rows and no global
   token.
@@ -72,22 +75,29 @@ def softmax(z: np.ndarray, axis: int = -1) -> np.ndarray:
 
 
 def attention(q: np.ndarray, k: np.ndarray, v: np.ndarray, n_heads: int,
-              allowed: Optional[np.ndarray] = None) -> np.ndarray:
+              allowed: Optional[np.ndarray] = None, n_kv_heads: Optional[int] = None) -> np.ndarray:
     """Multi-head scaled dot-product attention, heads concatenated.
 
-    q [n, d], k/v [m, d]; head h uses columns h*d_h ... (h+1)*d_h - 1.
+    q [n, d], k/v [m, n_kv_heads * d_h]; query head h uses columns
+    h*d_h ... (h+1)*d_h - 1 of q and key/value head h // (n_heads / n_kv_heads)
+    (grouped-query sharing of K/V heads, the MQA/GQA variants Sec. 4.1.2
+    cites; n_kv_heads = n_heads is plain multi-head attention).
     ``allowed`` [n, m] bool restricts the keys of each query row
     (Sec. 4.1.2 sparse cross-attention equation; App. B mask).
     """
     n, d = q.shape
     dh = d // n_heads
+    n_kv = n_heads if n_kv_heads is None else n_kv_heads
+    group = n_heads // n_kv
     out = np.empty((n, d), dtype=np.float64)
     for h in range(n_heads):
         c = slice(h * dh, (h + 1) * dh)
-        s = (q[:, c] @ k[:, c].T) / sqrt(dh)
+        g = h // group
+        ck = slice(g * dh, (g + 1) * dh)
+        s = (q[:, c] @ k[:, ck].T) / sqrt(dh)
         if allowed is not None:
             s = np.where(allowed, s, -np.inf)
-        out[:, c] = softmax(s, axis=-1) @ v[:, c]
+        out[:, c] = softmax(s, axis=-1) @ v[:, ck]
     return out
 
 
@@ -104,12 +114,17 @@ class Model:
     n_actions: int
     l_local: int
     ln_eps: float
+    n_kv_heads: int = 0   # K/V heads of the cache; 0 or n_heads: one per query head
+
+    @property
+    def kv_heads(self) -> int:
+        return self.n_kv_heads or self.n_heads
 
     @staticmethod
     def from_arrays(weights: Dict[str, np.ndarray], wl) -> "Model":
         return Model({k: np.asarray(v, dtype=np.float64) for k, v in weights.items()},
                      wl.n_layers, wl.d_model, wl.n_heads, wl.n_ctx, wl.n_actions,
-                     wl.l_local, wl.ln_eps)
+                     wl.l_local, wl.ln_eps, getattr(wl, "n_kv_heads", 0))
 
 
 @dataclass
@@ -239,7 +254,7 @@ def decoder_layer(model: Model, X: np.ndarray, Kc: np.ndarray, Vc: np.ndarray, l
     X1 = layer_norm(X + a @ w[f"W_os.{l}"] + w[f"b_os.{l}"], w[f"ln1_g.{l}"], w[f"ln1_b.{l}"], eps)
     # multi-query cross-attention against the shared K/V of this request
     qc = X1 @ w[f"W_Q.{l}"] + w[f"b_Q.{l}"]
-    c = attention(qc, Kc, Vc, H)
+    c = attention(qc, Kc, Vc, H, n_kv_heads=model.kv_heads)
     X2 = layer_norm(X1 + c @ w[f"W_oc.{l}"] + w[f"b_oc.{l}"], w[f"ln2_g.{l}"], w[f"ln2_b.{l}"], eps)
     # FFN
     f = gelu(X2 @ w[f"W_1.{l}"] + w[f"b_1.{l}"]) @ w[f"W_2.{l}"] + w[f"b_2.{l}"]

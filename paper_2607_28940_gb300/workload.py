@@ -40,8 +40,8 @@ LAYER_WEIGHTS: Tuple[Tuple[str, str], ...] = (
     # (name, shape code) in draw order; shape codes resolved by _shape()
     ("W_qkv", "d,3d"), ("b_qkv", "3d"), ("W_os", "d,d"), ("b_os", "d"),
     ("ln1_g", "d"), ("ln1_b", "d"),
-    ("W_Q", "d,d"), ("b_Q", "d"), ("W_K", "d,d"), ("b_K", "d"),
-    ("W_V", "d,d"), ("b_V", "d"), ("W_oc", "d,d"), ("b_oc", "d"),
+    ("W_Q", "d,d"), ("b_Q", "d"), ("W_K", "d,dkv"), ("b_K", "dkv"),
+    ("W_V", "d,dkv"), ("b_V", "dkv"), ("W_oc", "d,d"), ("b_oc", "d"),
     ("ln2_g", "d"), ("ln2_b", "d"),
     ("W_1", "d,F"), ("b_1", "F"), ("W_2", "F,d"), ("b_2", "d"),
     ("ln3_g", "d"), ("ln3_b", "d"),
@@ -71,6 +71,7 @@ class Workload:
     ln_eps: float = 1e-5
     dL: SizeSpec = 0        # appended behavior rows per request
     capacity_extra: int = 64
+    n_kv_heads: int = 0     # K/V heads of the cache (0: one per query head)
 
     @property
     def d_head(self) -> int:
@@ -137,8 +138,9 @@ def sizes(wl: Workload) -> Tuple[np.ndarray, np.ndarray, np.ndarray]:
 
 
 def _shape(code: str, wl: Workload) -> Tuple[int, ...]:
+    dkv = (wl.n_kv_heads or wl.n_heads) * (wl.d_model // wl.n_heads)
     env = {"d": wl.d_model, "3d": 3 * wl.d_model, "2d": 2 * wl.d_model,
-           "F": wl.d_ff, "k": wl.n_actions}
+           "F": wl.d_ff, "k": wl.n_actions, "dkv": dkv}
     return tuple(env[c] for c in code.split(","))
 
 

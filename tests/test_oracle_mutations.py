@@ -56,19 +56,19 @@ def _gelu_tanh(x):
     return 0.5 * x * (1 + np.tanh(math.sqrt(2 / math.pi) * (x + 0.044715 * x ** 3)))
 
 
-def _attn_scale_dh(q, k, v, n_heads, allowed=None):
+def _attn_scale_dh(q, k, v, n_heads, allowed=None, n_kv_heads=None):
     dh = q.shape[1] // n_heads
-    return _orig_attn(q / math.sqrt(dh), k, v, n_heads, allowed)   # scale 1/d_h overall
+    return _orig_attn(q / math.sqrt(dh), k, v, n_heads, allowed, n_kv_heads)   # scale 1/d_h overall
 
 
-def _attn_no_mask(q, k, v, n_heads, allowed=None):
-    return _orig_attn(q, k, v, n_heads, None)
+def _attn_no_mask(q, k, v, n_heads, allowed=None, n_kv_heads=None):
+    return _orig_attn(q, k, v, n_heads, None, n_kv_heads)
 
 
-def _attn_heads_interleaved(q, k, v, n_heads, allowed=None):
+def _attn_heads_interleaved(q, k, v, n_heads, allowed=None, n_kv_heads=None):
     n, d = q.shape
     perm = np.arange(d).reshape(d // n_heads, n_heads).T.reshape(-1)
-    out = _orig_attn(q[:, perm], k[:, perm], v[:, perm], n_heads, allowed)
+    out = _orig_attn(q[:, perm], k[:, perm], v[:, perm], n_heads, allowed, n_kv_heads)
     inv = np.argsort(perm)
     return out[:, inv]
 
