@@ -66,6 +66,10 @@ typedef struct {
   int32_t attn_mode; /* txs_attn_mode                                             */
   int32_t dtype;     /* txs_dtype                                                 */
   float ln_eps;      /* LayerNorm epsilon (> 0)                                   */
+  int32_t n_kv_heads;/* K/V heads of the behavior cache (MQA/GQA variants cited in
+                        Sec. 4.1.2): 0 = n_heads; otherwise divides n_heads, and
+                        query head h uses K/V head h / (n_heads / n_kv_heads).  The
+                        cached rows are n_kv_heads * d_head wide.                   */
 } txs_config;
 
 typedef struct txs_model txs_model;       /* opaque */
@@ -81,10 +85,11 @@ typedef struct txs_kv_cache txs_kv_cache; /* opaque */
  *
  * `weights` (host array of device pointers) holds n_layers * 22 + 4 pointers,
  * layer by layer, then the head, in this order and with these shapes
- * (d = d_model, F = d_ff, k = n_actions), all in the config's dtype:
+ * (d = d_model, F = d_ff, k = n_actions, dkv = n_kv_heads * d_head, which is d
+ * when n_kv_heads is 0 or n_heads), all in the config's dtype:
  *   per layer l (Sec. 4.1.2 crossAttend block; App. B serving-stream attention):
  *     0 W_qkv [d,3d]  1 b_qkv [3d]   2 W_os [d,d]  3 b_os [d]  4 ln1_g [d] 5 ln1_b [d]
- *     6 W_Q  [d,d]    7 b_Q  [d]     8 W_K [d,d]   9 b_K [d]  10 W_V [d,d] 11 b_V [d]
+ *     6 W_Q  [d,d]    7 b_Q  [d]     8 W_K [d,dkv] 9 b_K [dkv] 10 W_V [d,dkv] 11 b_V [dkv]
  *    12 W_oc [d,d]   13 b_oc [d]    14 ln2_g [d]  15 ln2_b [d]
  *    16 W_1  [d,F]   17 b_1  [F]    18 W_2 [F,d]  19 b_2 [d]  20 ln3_g [d] 21 ln3_b [d]
  *   head (Sec. 4.1.3; attention pooling Sec. 5.1):
@@ -143,13 +148,13 @@ txs_status txs_append_behavior(txs_model* model, txs_kv_cache* cache, int32_t n_
                                const int32_t* new_offsets, const void* new_enc, void* stream);
 
 /* Copy rows row0 .. row0+n_rows-1 of request `req`'s cached K (which = 0) or
- * V (which = 1) of layer `layer` into dst (device, model dtype, [n_rows, d]),
+ * V (which = 1) of layer `layer` into dst (device, model dtype, [n_rows, dkv]),
  * asynchronously on `stream`.  Rows must be < the request's current length. */
 txs_status txs_cache_read_rows(const txs_kv_cache* cache, int32_t layer, int32_t which, int32_t req, int32_t row0,
                                int32_t n_rows, void* dst, void* stream);
 /* Copy the anchor's projected key (which = 0) or value (which = 1) of `layer`
- * for all requests, or the pooled anchor g itself (which = 2, layer ignored),
- * into dst (device, float, [n_req, d]). */
+ * for all requests (device, float, [n_req, dkv]), or the pooled anchor g
+ * itself (which = 2, layer ignored; [n_req, d]) into dst. */
 txs_status txs_cache_read_anchor(const txs_kv_cache* cache, int32_t layer, int32_t which, float* dst, void* stream);
 
 /*

@@ -126,11 +126,12 @@ struct CrossArgs {
   int n_rows;
   const int* kv_off;    // [R+1] cache row offsets (capacity layout)
   const int* kv_len;    // [R]   current lengths
-  const float* Kg;      // [R, d] anchor key of this layer (LOCAL_GLOBAL), fp32
+  const float* Kg;      // [R, dkv] anchor key of this layer (LOCAL_GLOBAL), fp32
   const float* Vg;
   int l_local;
   int mode;
   int H, d;
+  int dkv, group;       // cached row width; query heads per K/V head
   float scale;
 };
 
@@ -148,8 +149,9 @@ __global__ void __launch_bounds__(256) cross_attn_kernel(const T* __restrict__ q
   if (pair >= static_cast<long long>(a.n_rows) * a.H) return;   // whole group
   const int row = static_cast<int>(pair / a.H);
   const int h = static_cast<int>(pair % a.H);
-  const int col = h * DH + sub * VEC;
-  const int d = a.d;
+  const int col = h * DH + sub * VEC;                         // query / output columns
+  const int ck = (h / a.group) * DH + sub * VEC;              // the same slice of its K/V head
+  const int d = a.d, dkv = a.dkv;
   const unsigned gmask = G::mask();
   float q[VEC], acc[VEC];
   Vec16<T>::load(q_in + static_cast<long long>(row) * d + col, q);
@@ -160,13 +162,13 @@ __global__ void __launch_bounds__(256) cross_attn_kernel(const T* __restrict__ q
   const int len = __ldg(a.kv_len + r);
   const long long base = __ldg(a.kv_off + r);
   const int lo = (a.mode == TXS_ATTN_LOCAL_GLOBAL) ? max(0, len - a.l_local) : 0;
-  attend_rows<T, G>(q, len - lo, col, gmask, a.scale, sm, acc, [&](int t, const T*& kr, const T*& vr) {
-    kr = Kc + (base + lo + t) * d;
-    vr = Vc + (base + lo + t) * d;
+  attend_rows<T, G>(q, len - lo, ck, gmask, a.scale, sm, acc, [&](int t, const T*& kr, const T*& vr) {
+    kr = Kc + (base + lo + t) * dkv;
+    vr = Vc + (base + lo + t) * dkv;
   });
   if (a.mode == TXS_ATTN_LOCAL_GLOBAL) {
-    const float* kg = a.Kg + static_cast<long long>(r) * d + col;
-    const float* vg = a.Vg + static_cast<long long>(r) * d + col;
+    const float* kg = a.Kg + static_cast<long long>(r) * dkv + ck;
+    const float* vg = a.Vg + static_cast<long long>(r) * dkv + ck;
     float dot = 0.f;
 #pragma unroll
     for (int i = 0; i < VEC; ++i) dot = fmaf(q[i], __ldg(kg + i), dot);
@@ -196,9 +198,10 @@ struct CrossLgArgs {
   int n_cand, S;
   const int* kv_off;    // [R+1] cache row offsets
   const int* kv_len;    // [R]
-  const float* Kg;      // [R, d] anchor key / value of this layer, fp32
+  const float* Kg;      // [R, dkv] anchor key / value of this layer, fp32
   const float* Vg;
   int l_local, H, d;
+  int dkv, group;       // cached row width; query heads per K/V head
   float scale_log2;     // log2(e) / sqrt(d_h)
 };
 
@@ -209,11 +212,11 @@ __global__ void __launch_bounds__(256) cross_lg_kernel(const T* __restrict__ q_i
   pdl_launch_dependents();
   pdl_wait();
   extern __shared__ __align__(16) uint8_t smem_lg[];
-  const int d = a.d;
-  T* sK = reinterpret_cast<T*>(smem_lg);                      // [kWin][d]
-  T* sV = sK + kWin * d;                                      // [kWin][d]
-  float* sKg = reinterpret_cast<float*>(sV + kWin * d);       // [d]
-  float* sVg = sKg + d;                                       // [d]
+  const int d = a.d, dkv = a.dkv;
+  T* sK = reinterpret_cast<T*>(smem_lg);                      // [kWin][dkv]
+  T* sV = sK + kWin * dkv;                                    // [kWin][dkv]
+  float* sKg = reinterpret_cast<float*>(sV + kWin * dkv);     // [dkv]
+  float* sVg = sKg + dkv;                                     // [dkv]
   const int r = blockIdx.y;
   const int c0 = __ldg(a.cand_off + r);
   const int M = __ldg(a.cand_off + r + 1) - c0;
@@ -226,15 +229,15 @@ __global__ void __launch_bounds__(256) cross_lg_kernel(const T* __restrict__ q_i
   const long long base = static_cast<long long>(__ldg(a.kv_off + r)) + lo;
   {
     constexpr int VE = Vec16<T>::N;                           // elements per 16 bytes
-    const int per_row = d / VE;
+    const int per_row = dkv / VE;
     for (int i = threadIdx.x; i < W * per_row; i += blockDim.x) {
       const int t = i / per_row, c = (i - t * per_row) * VE;
-      *reinterpret_cast<uint4*>(sK + t * d + c) = *reinterpret_cast<const uint4*>(Kc + (base + t) * d + c);
-      *reinterpret_cast<uint4*>(sV + t * d + c) = *reinterpret_cast<const uint4*>(Vc + (base + t) * d + c);
+      *reinterpret_cast<uint4*>(sK + t * dkv + c) = *reinterpret_cast<const uint4*>(Kc + (base + t) * dkv + c);
+      *reinterpret_cast<uint4*>(sV + t * dkv + c) = *reinterpret_cast<const uint4*>(Vc + (base + t) * dkv + c);
     }
-    for (int i = threadIdx.x; i < d; i += blockDim.x) {
-      sKg[i] = __ldg(a.Kg + static_cast<long long>(r) * d + i);
-      sVg[i] = __ldg(a.Vg + static_cast<long long>(r) * d + i);
+    for (int i = threadIdx.x; i < dkv; i += blockDim.x) {
+      sKg[i] = __ldg(a.Kg + static_cast<long long>(r) * dkv + i);
+      sVg[i] = __ldg(a.Vg + static_cast<long long>(r) * dkv + i);
     }
   }
   __syncthreads();
@@ -244,7 +247,8 @@ __global__ void __launch_bounds__(256) cross_lg_kernel(const T* __restrict__ q_i
   const long long grow = j < M ? static_cast<long long>(c0) + j
                                : a.n_cand + static_cast<long long>(r) * a.S + (j - M);
   for (int h = warp; h < a.H; h += (blockDim.x >> 5)) {
-    const int col = h * DH;
+    const int col = h * DH;                                   // query / output columns
+    const int ck = (h / a.group) * DH;                        // its K/V head
     float q[DH];
     if (valid) {
 #pragma unroll
@@ -265,7 +269,7 @@ __global__ void __launch_bounds__(256) cross_lg_kernel(const T* __restrict__ q_i
 #pragma unroll
         for (int c = 0; c < DH; c += Vec16<T>::N) {
           float k[Vec16<T>::N];
-          Vec16<T>::load(sK + t * d + col + c, k);
+          Vec16<T>::load(sK + t * dkv + ck + c, k);
 #pragma unroll
           for (int i = 0; i < Vec16<T>::N; ++i) dot = fmaf(q[c + i], k[i], dot);
         }
@@ -276,7 +280,7 @@ __global__ void __launch_bounds__(256) cross_lg_kernel(const T* __restrict__ q_i
       float dot = 0.f;
 #pragma unroll
       for (int c = 0; c < DH; c += 4) {
-        const float4 k4 = *reinterpret_cast<const float4*>(sKg + col + c);
+        const float4 k4 = *reinterpret_cast<const float4*>(sKg + ck + c);
         dot = fmaf(q[c], k4.x, dot);
         dot = fmaf(q[c + 1], k4.y, dot);
         dot = fmaf(q[c + 2], k4.z, dot);
@@ -296,7 +300,7 @@ __global__ void __launch_bounds__(256) cross_lg_kernel(const T* __restrict__ q_i
     // weighted values (q reused as the accumulator)
 #pragma unroll
     for (int c = 0; c < DH; c += 4) {
-      const float4 v4 = *reinterpret_cast<const float4*>(sVg + col + c);
+      const float4 v4 = *reinterpret_cast<const float4*>(sVg + ck + c);
       q[c] = sc[kWin] * v4.x;
       q[c + 1] = sc[kWin] * v4.y;
       q[c + 2] = sc[kWin] * v4.z;
@@ -308,7 +312,7 @@ __global__ void __launch_bounds__(256) cross_lg_kernel(const T* __restrict__ q_i
 #pragma unroll
         for (int c = 0; c < DH; c += Vec16<T>::N) {
           float v[Vec16<T>::N];
-          Vec16<T>::load(sV + t * d + col + c, v);
+          Vec16<T>::load(sV + t * dkv + ck + c, v);
 #pragma unroll
           for (int i = 0; i < Vec16<T>::N; ++i) q[c + i] = fmaf(sc[t], v[i], q[c + i]);
         }
@@ -361,9 +365,10 @@ cudaError_t launch_serving_attn(const T* qkv, T* out, const int* row_req, int n_
 template <typename T>
 cudaError_t launch_cross_attn(const T* q, T* out, const T* Kc, const T* Vc, const int* row_req, int n_rows,
                               const int* kv_off, const int* kv_len, const float* Kg, const float* Vg, int l_local,
-                              int mode, int H, int d, cudaStream_t s) {
+                              int mode, int H, int Hkv, int d, cudaStream_t s) {
   if (n_rows == 0) return cudaSuccess;
-  CrossArgs a{row_req, n_rows, kv_off, kv_len, Kg, Vg, l_local, mode, H, d, 0.f};
+  if (Hkv < 1 || H % Hkv) return cudaErrorInvalidValue;
+  CrossArgs a{row_req, n_rows, kv_off, kv_len, Kg, Vg, l_local, mode, H, d, Hkv * (d / H), H / Hkv, 0.f};
   prof_begin(KC_ATTN_CROSS, s);
   cudaError_t err;
   switch (d / H) {
@@ -378,16 +383,18 @@ cudaError_t launch_cross_attn(const T* q, T* out, const T* Kc, const T* Vc, cons
 template <typename T>
 cudaError_t launch_cross_attn_lg(const T* q, T* out, const T* Kc, const T* Vc, const int* cand_off_dev,
                                  const int* cand_off_host, int n_req, int n_cand, int S, const int* kv_off,
-                                 const int* kv_len, const float* Kg, const float* Vg, int l_local, int H, int d,
-                                 cudaStream_t s) {
+                                 const int* kv_len, const float* Kg, const float* Vg, int l_local, int H, int Hkv,
+                                 int d, cudaStream_t s) {
   const int dh = d / H;
   if (l_local > kWin || (dh != 32 && dh != 64) || d % 8 != 0) return cudaErrorNotSupported;
+  if (Hkv < 1 || H % Hkv) return cudaErrorInvalidValue;
+  const int dkv = Hkv * dh;
   int max_q = 0;
   for (int r = 0; r < n_req; ++r) max_q = std::max(max_q, cand_off_host[r + 1] - cand_off_host[r] + S);
   if (max_q == 0 || n_req == 0) return cudaSuccess;
-  CrossLgArgs a{cand_off_dev, n_cand, S, kv_off, kv_len, Kg, Vg, l_local, H, d,
+  CrossLgArgs a{cand_off_dev, n_cand, S, kv_off, kv_len, Kg, Vg, l_local, H, d, dkv, H / Hkv,
                 1.4426950408889634f / sqrtf(static_cast<float>(dh))};
-  const size_t smem = static_cast<size_t>(2 * kWin * d) * sizeof(T) + 2 * d * sizeof(float);
+  const size_t smem = static_cast<size_t>(2 * kWin * dkv) * sizeof(T) + 2 * dkv * sizeof(float);
   const dim3 grid((max_q + 31) / 32, n_req);
   prof_begin(KC_ATTN_CROSS, s);
   cudaError_t err;
@@ -404,20 +411,21 @@ cudaError_t launch_cross_attn_lg(const T* q, T* out, const T* Kc, const T* Vc, c
 
 template cudaError_t launch_cross_attn_lg<float>(const float*, float*, const float*, const float*, const int*,
                                                  const int*, int, int, int, const int*, const int*, const float*,
-                                                 const float*, int, int, int, cudaStream_t);
+                                                 const float*, int, int, int, int, cudaStream_t);
 template cudaError_t launch_cross_attn_lg<__nv_bfloat16>(const __nv_bfloat16*, __nv_bfloat16*, const __nv_bfloat16*,
                                                          const __nv_bfloat16*, const int*, const int*, int, int, int,
                                                          const int*, const int*, const float*, const float*, int,
-                                                         int, int, cudaStream_t);
+                                                         int, int, int, cudaStream_t);
 
 template cudaError_t launch_serving_attn<float>(const float*, float*, const int*, int, int, int, int, int, cudaStream_t);
 template cudaError_t launch_serving_attn<__nv_bfloat16>(const __nv_bfloat16*, __nv_bfloat16*, const int*, int, int,
                                                         int, int, int, cudaStream_t);
 template cudaError_t launch_cross_attn<float>(const float*, float*, const float*, const float*, const int*, int,
                                               const int*, const int*, const float*, const float*, int, int, int, int,
-                                              cudaStream_t);
+                                              int, cudaStream_t);
 template cudaError_t launch_cross_attn<__nv_bfloat16>(const __nv_bfloat16*, __nv_bfloat16*, const __nv_bfloat16*,
                                                       const __nv_bfloat16*, const int*, int, const int*, const int*,
-                                                      const float*, const float*, int, int, int, int, cudaStream_t);
+                                                      const float*, const float*, int, int, int, int, int,
+                                                      cudaStream_t);
 
 }  // namespace txs

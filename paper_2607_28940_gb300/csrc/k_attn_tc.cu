@@ -215,6 +215,7 @@ struct FaArgs {
   const int* kv_off;          // device [R + 1] cache row offsets
   const int* kv_len;          // device [R]
   int n_cand, S, d;
+  int group;                  // query heads per K/V head
   float scale_log2;           // log2(e) / sqrt(d_h)
   int* status;
 };
@@ -298,8 +299,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         const int st = j % STG;
         if (!mbar_wait(kv_empty + st, ((j / STG) & 1) ^ 1, abort_flag)) break;
         mbar_expect_tx(kv_full + st, 2 * Sh::KV_BYTES);
-        tma_load_2d(sK + st * Sh::KV_BYTES, &tmK, kv_full + st, h * DH, kv0 + j * BKV);
-        tma_load_2d(sV + st * Sh::KV_BYTES, &tmV, kv_full + st, h * DH, kv0 + j * BKV);
+        tma_load_2d(sK + st * Sh::KV_BYTES, &tmK, kv_full + st, (h / a.group) * DH, kv0 + j * BKV);
+        tma_load_2d(sV + st * Sh::KV_BYTES, &tmV, kv_full + st, (h / a.group) * DH, kv0 + j * BKV);
         issued = j + 1;
       }
       if (*abort_flag)
@@ -528,7 +529,7 @@ static bool make_kv_map(CUtensorMap* tm, const void* base, long long rows, int d
 
 template <int DH>
 static cudaError_t launch_dh(const FaArgs& a, const void* Kc, const void* Vc, long long cap_total, int n_req,
-                             int max_q_tiles, int H, cudaStream_t s) {
+                             int max_q_tiles, int H, int dkv, cudaStream_t s) {
   using Sh = FaShape<DH>;
   static bool attr = false;
   if (!attr) {
@@ -537,7 +538,7 @@ static cudaError_t launch_dh(const FaArgs& a, const void* Kc, const void* Vc, lo
     attr = true;
   }
   CUtensorMap tk, tv;
-  if (!make_kv_map<DH>(&tk, Kc, cap_total, a.d) || !make_kv_map<DH>(&tv, Vc, cap_total, a.d))
+  if (!make_kv_map<DH>(&tk, Kc, cap_total, dkv) || !make_kv_map<DH>(&tv, Vc, cap_total, dkv))
     return cudaErrorInvalidValue;
   const dim3 grid(max_q_tiles, n_req, H);
   return launch_pdl(fa_full_kernel<DH>, grid, dim3(NUM_THREADS), Sh::SMEM, s, tk, tv, a);
@@ -553,17 +554,18 @@ bool fa_full_supported(int d, int H, long long cap_total) {
 cudaError_t launch_fa_full(const __nv_bfloat16* q, __nv_bfloat16* out, const __nv_bfloat16* Kc,
                            const __nv_bfloat16* Vc, long long cap_total, const int* cand_off_dev,
                            const int* cand_off_host, const int* kv_off, const int* kv_len, int n_req, int n_cand,
-                           int S, int H, int d, int* status, cudaStream_t s) {
+                           int S, int H, int Hkv, int d, int* status, cudaStream_t s) {
   int max_q = 0;
   for (int r = 0; r < n_req; ++r) max_q = std::max(max_q, cand_off_host[r + 1] - cand_off_host[r] + S);
   if (max_q == 0) return cudaSuccess;
+  if (Hkv < 1 || H % Hkv) return cudaErrorInvalidValue;
   const int dh = d / H;
-  fa::FaArgs a{q, out, cand_off_dev, kv_off, kv_len, n_cand, S, d,
+  fa::FaArgs a{q, out, cand_off_dev, kv_off, kv_len, n_cand, S, d, H / Hkv,
                1.4426950408889634f / sqrtf(static_cast<float>(dh)), status};
   const int tiles = (max_q + fa::BQ - 1) / fa::BQ;
   prof_begin(KC_ATTN_CROSS, s);
-  cudaError_t err = dh == 64 ? fa::launch_dh<64>(a, Kc, Vc, cap_total, n_req, tiles, H, s)
-                             : fa::launch_dh<32>(a, Kc, Vc, cap_total, n_req, tiles, H, s);
+  cudaError_t err = dh == 64 ? fa::launch_dh<64>(a, Kc, Vc, cap_total, n_req, tiles, H, Hkv * dh, s)
+                             : fa::launch_dh<32>(a, Kc, Vc, cap_total, n_req, tiles, H, Hkv * dh, s);
   prof_end(KC_ATTN_CROSS, s);
   return err;
 }

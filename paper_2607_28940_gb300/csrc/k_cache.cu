@@ -213,7 +213,7 @@ constexpr int kAnchorReqPerWarp = 8;
 template <typename T, int NCH>
 __global__ void __launch_bounds__(256) anchor_proj_kernel(const float* __restrict__ g, const T* __restrict__ Wt,
                                                           const float* __restrict__ b, float* __restrict__ gkv,
-                                                          int R, int d, int n_total) {
+                                                          int R, int d, int dkv, int n_total) {
   pdl_launch_dependents();
   pdl_wait();
   constexpr int VEC = Vec16<T>::N;
@@ -265,8 +265,8 @@ __global__ void __launch_bounds__(256) anchor_proj_kernel(const float* __restric
 #pragma unroll
     for (int t = 0; t < kAnchorReqPerWarp; ++t)
       if (t == lane) v = dot[t];
-    const int blk = n / d, c = n - blk * d;
-    gkv[(static_cast<long long>(blk) * R + r0 + lane) * d + c] = v + __ldg(b + n);
+    const int blk = n / dkv, c = n - blk * dkv;
+    gkv[(static_cast<long long>(blk) * R + r0 + lane) * dkv + c] = v + __ldg(b + n);
   }
 }
 
@@ -358,18 +358,18 @@ cudaError_t launch_pool(const T* phi, const int* seg_off, int R, int max_rows, c
 }
 
 template <typename T>
-cudaError_t launch_anchor_proj(const float* g, const T* Wt_kv, const float* b_kv, float* gkv, int R, int d,
+cudaError_t launch_anchor_proj(const float* g, const T* Wt_kv, const float* b_kv, float* gkv, int R, int d, int dkv,
                                int n_layers, cudaStream_t s) {
   constexpr int VEC = Vec16<T>::N;
   const int nch = (d + 32 * VEC - 1) / (32 * VEC);
-  const int n_total = 2 * n_layers * d;
+  const int n_total = 2 * n_layers * dkv;
   const long long warps = static_cast<long long>(n_total) * ((R + kAnchorReqPerWarp - 1) / kAnchorReqPerWarp);
   const int blocks = static_cast<int>((warps + 7) / 8);
   prof_begin(KC_GLOBAL_KV, s);
   cudaError_t err;
-  if (nch == 1) err = launch_pdl(anchor_proj_kernel<T, 1>, dim3(blocks), dim3(256), 0, s, g, Wt_kv, b_kv, gkv, R, d, n_total);
-  else if (nch == 2) err = launch_pdl(anchor_proj_kernel<T, 2>, dim3(blocks), dim3(256), 0, s, g, Wt_kv, b_kv, gkv, R, d, n_total);
-  else if (nch <= 4) err = launch_pdl(anchor_proj_kernel<T, 4>, dim3(blocks), dim3(256), 0, s, g, Wt_kv, b_kv, gkv, R, d, n_total);
+  if (nch == 1) err = launch_pdl(anchor_proj_kernel<T, 1>, dim3(blocks), dim3(256), 0, s, g, Wt_kv, b_kv, gkv, R, d, dkv, n_total);
+  else if (nch == 2) err = launch_pdl(anchor_proj_kernel<T, 2>, dim3(blocks), dim3(256), 0, s, g, Wt_kv, b_kv, gkv, R, d, dkv, n_total);
+  else if (nch <= 4) err = launch_pdl(anchor_proj_kernel<T, 4>, dim3(blocks), dim3(256), 0, s, g, Wt_kv, b_kv, gkv, R, d, dkv, n_total);
   else return cudaErrorInvalidValue;
   prof_end(KC_GLOBAL_KV, s);
   return err;
@@ -585,7 +585,7 @@ cudaError_t launch_prefix_pool(const T* phi, const int* ends, int n_ev, int off_
                                       float*, float*, float*, int*, cudaStream_t);                                  \
   template cudaError_t launch_prefix_pool<T>(const T*, const int*, int, int, const float*, int, float*, float*,     \
                                              int*, int*, cudaStream_t);                                             \
-  template cudaError_t launch_anchor_proj<T>(const float*, const T*, const float*, float*, int, int, int,          \
+  template cudaError_t launch_anchor_proj<T>(const float*, const T*, const float*, float*, int, int, int, int,     \
                                              cudaStream_t);                                                         \
   template cudaError_t launch_transpose<T>(const T*, T*, int, int, cudaStream_t);                                  \
   template cudaError_t launch_to_f32<T>(const T*, float*, long long, cudaStream_t);                                \

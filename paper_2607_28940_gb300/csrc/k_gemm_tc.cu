@@ -68,32 +68,41 @@ __device__ __forceinline__ void epilogue(const EpiArgs& e, uint32_t tacc, int ro
   const int lane = threadIdx.x & 31;
   float v[32];
   if constexpr (EPI == EPI_BIAS || EPI == EPI_BIAS_GELU || EPI == EPI_KV) {
-    __nv_bfloat16* out = nullptr;
     // bulk-store coordinates of this warp's 32 rows: plain outputs are a
     // [M, N] tensor (rows past M are dropped by the store); the cache is a
-    // [blocks * cap_total, d] tensor and takes the bulk path only when all 32
-    // rows are valid and belong to one request (consecutive cache rows)
+    // [blocks * cap_total, col_blk] tensor (column blocks of width col_blk,
+    // at least 32, may be narrower than the tile) and takes the bulk path
+    // only when all 32 rows are valid and belong to one request (consecutive
+    // cache rows)
     bool tma_ok = true;
-    int tx = n0 + c0, ty = row - lane;
     long long orow = row;
-    long long ocol = n0 + c0;
-    int r = 0;
+    long long orow0 = row - lane;                // the warp's first row
     if constexpr (EPI == EPI_KV) {
-      const int blk = n0 / e.col_blk;
+      int r = 0;
       if (valid) {
         r = find_seg_gen(seg_off, e.n_seg, row);
         orow = static_cast<long long>(dst_row0[r]) + (row - seg_off[r]);
       }
-      ocol = static_cast<long long>(blk) * e.col_blk_stride + (n0 - blk * e.col_blk) + c0;
       // lane 0 holds the warp's first row: if it is invalid, so are all
       const int r_first = __shfl_sync(0xffffffffu, r, 0);
-      const long long y0 = static_cast<long long>(blk) * (e.col_blk_stride / e.col_blk) + orow;
-      tx = (n0 - blk * e.col_blk) + c0;
-      ty = static_cast<int>(__shfl_sync(0xffffffffu, y0, 0));
+      orow0 = __shfl_sync(0xffffffffu, orow, 0);
       tma_ok = valid && r == r_first;
     }
-    if (valid) out = static_cast<__nv_bfloat16*>(e.out) + orow * e.ldo + ocol;
     tma_ok = __all_sync(0xffffffffu, tma_ok);
+    // stores the 32 columns starting at output column n of this warp's rows
+    auto put = [&](const float* vals, int n) {
+      __nv_bfloat16* out = nullptr;
+      int tx = n, ty = static_cast<int>(orow0);
+      if constexpr (EPI == EPI_KV) {
+        const int blk = n / e.col_blk, xin = n - blk * e.col_blk;
+        if (valid) out = static_cast<__nv_bfloat16*>(e.out) + orow * e.ldo + blk * e.col_blk_stride + xin;
+        tx = xin;
+        ty = static_cast<int>(static_cast<long long>(blk) * (e.col_blk_stride / e.col_blk) + orow0);
+      } else {
+        if (valid) out = static_cast<__nv_bfloat16*>(e.out) + orow * e.ldo + n;
+      }
+      store_chunk(vals, out, valid, tma_ok, tmO, tx, ty, stage, kchunk++, lane);
+    };
     if constexpr (HALF % 64 == 0) {
       // 64 columns per TMEM load (one wait), two bulk-stored chunks
 #pragma unroll 1
@@ -110,7 +119,7 @@ __device__ __forceinline__ void epilogue(const EpiArgs& e, uint32_t tacc, int ro
             if constexpr (EPI == EPI_BIAS_GELU) x = gelu_erf(x);
             w[hh + i] = x;
           }
-          store_chunk(w + hh, out + c + hh, valid, tma_ok, tmO, tx + c + hh, ty, stage, kchunk++, lane);
+          put(w + hh, n0 + c0 + c + hh);
         }
       }
     } else {
@@ -125,7 +134,7 @@ __device__ __forceinline__ void epilogue(const EpiArgs& e, uint32_t tacc, int ro
           if constexpr (EPI == EPI_BIAS_GELU) x = gelu_erf(x);
           v[i] = x;
         }
-        store_chunk(v, out + c, valid, tma_ok, tmO, tx + c, ty, stage, kchunk++, lane);
+        put(v, n0 + c0 + c);
       }
     }
   } else {
@@ -610,7 +619,8 @@ static cudaError_t launch_plain(const __nv_bfloat16* A, long long lda, const __n
   const long long m_tiles = (e.M + BM - 1) / BM;
   auto fits = [&](int bn) {
     if (e.N % bn) return false;
-    if (EPI == EPI_KV && e.col_blk % bn) return false;
+    // cache column blocks: a tile covers whole blocks or lies inside one
+    if (EPI == EPI_KV && e.col_blk % bn != 0 && (e.col_blk % 32 != 0 || bn % e.col_blk != 0)) return false;
     return true;
   };
   // short K and at least two tiles per SM: keep each CTA's B slice resident

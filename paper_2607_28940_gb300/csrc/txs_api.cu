@@ -73,8 +73,8 @@ struct txs_model {
   int es = 0;                    // bytes per stored element
   std::vector<void*> allocs;
   std::vector<txs::LayerW> layers;
-  void* Wt_kv = nullptr;         // [2 nL d, d]: rows (l, K|V, c)
-  float* b_kv = nullptr;         // [2 nL d]
+  void* Wt_kv = nullptr;         // [2 nL dkv, d]: rows (l, K|V, c)
+  float* b_kv = nullptr;         // [2 nL dkv]
   float* w_pool = nullptr;       // [d]
   float* weff = nullptr;         // [2d, k]
   float* cdec = nullptr;         // [k]
@@ -84,6 +84,7 @@ struct txs_model {
 
 struct txs_kv_cache {
   int n_req = 0, n_layers = 0, d = 0, es = 0, cap_extra = 0;
+  int dkv = 0;                           // width of a cached row: n_kv_heads * d_head
   uint64_t model_hash = 0;
   long long cap_total = 0;
   std::vector<int> h_off, h_len, h_cap;  // capacity offsets [R+1], lengths, capacities
@@ -95,9 +96,9 @@ struct txs_kv_cache {
   int* d_len = nullptr;                  // [R]
   int* d_in_off = nullptr;               // [R+1] offsets of the rows being projected
   int* d_dst0 = nullptr;                 // [R]   first cache row they go to
-  void* kv = nullptr;                    // [nL][2][cap_total][d] model dtype
+  void* kv = nullptr;                    // [nL][2][cap_total][dkv] model dtype
   float *pool_m = nullptr, *pool_s = nullptr, *pool_acc = nullptr, *g = nullptr;
-  float* gkv = nullptr;                  // [nL][2][R][d] fp32
+  float* gkv = nullptr;                  // [nL][2][R][dkv] fp32
   float* part = nullptr;                 // pooling chunk states
   int* pool_cnt = nullptr;               // [R] chunk arrivals (zero between calls)
   int max_chunks = 0;
@@ -128,8 +129,12 @@ bool cfg_ok(const txs_config& c, std::string* why) {
   if (c.n_ctx < 0 || c.n_ctx > 8) return bad("n_ctx");
   if (c.l_local < 1) return bad("l_local");
   if (!(c.ln_eps > 0.f) || !std::isfinite(c.ln_eps)) return bad("ln_eps");
+  if (c.n_kv_heads < 0 || (c.n_kv_heads > 0 && c.n_heads % c.n_kv_heads)) return bad("n_kv_heads");
   return true;
 }
+
+// Width of a cached K or V row: n_kv_heads * d_head (d_model for n_kv_heads 0).
+int kv_dim(const txs_config& c) { return (c.n_kv_heads ? c.n_kv_heads : c.n_heads) * (c.d_model / c.n_heads); }
 
 // offsets[0] == 0, non-decreasing (strictly if `strict`), last <= INT32_MAX
 bool offsets_ok(const int32_t* off, int n, bool strict) {
@@ -215,14 +220,14 @@ txs_status fail_cuda(const char* where, cudaError_t e) {
 template <typename T>
 txs_status model_prepare(txs_model* m, const void* const* w, cudaStream_t s) {
   const txs_config& c = m->cfg;
-  const int d = c.d_model, F = c.d_ff, nL = c.n_layers, k = c.n_actions;
+  const int d = c.d_model, F = c.d_ff, nL = c.n_layers, k = c.n_actions, dkv = kv_dim(c);
   cudaError_t err;
   auto wt = [&](int rows, int cols) { return dalloc<T>(m->allocs, size_t(rows) * cols * sizeof(T), &err); };
   auto vf = [&](int n) { return dalloc<float>(m->allocs, size_t(n) * 4, &err); };
   auto W = [&](int l, int i) { return static_cast<const T*>(w[l * TXS_WEIGHTS_PER_LAYER + i]); };
-  m->Wt_kv = wt(2 * nL * d, d);
+  m->Wt_kv = wt(2 * nL * dkv, d);
   if (!m->Wt_kv) return fail_cuda("cudaMalloc", err);
-  m->b_kv = vf(2 * nL * d);
+  m->b_kv = vf(2 * nL * dkv);
   if (!m->b_kv) return fail_cuda("cudaMalloc", err);
   for (int l = 0; l < nL; ++l) {
     LayerW L;
@@ -247,8 +252,8 @@ txs_status model_prepare(txs_model* m, const void* const* w, cudaStream_t s) {
     TXS_CK(launch_transpose<T>(W(l, 18), p, F, d, s));
     L.Wt_2 = p;
     T* kv = static_cast<T*>(m->Wt_kv);
-    TXS_CK(launch_transpose<T>(W(l, 8), kv + size_t(2 * l) * d * d, d, d, s));
-    TXS_CK(launch_transpose<T>(W(l, 10), kv + size_t(2 * l + 1) * d * d, d, d, s));
+    TXS_CK(launch_transpose<T>(W(l, 8), kv + size_t(2 * l) * dkv * d, d, dkv, s));
+    TXS_CK(launch_transpose<T>(W(l, 10), kv + size_t(2 * l + 1) * dkv * d, d, dkv, s));
     // vectors in fp32
     float** dst[] = {&L.b_qkv, &L.b_os, &L.g1, &L.be1, &L.b_q, &L.b_oc, &L.g2, &L.be2,
                      &L.b_1, &L.b_2, &L.g3, &L.be3};
@@ -260,8 +265,8 @@ txs_status model_prepare(txs_model* m, const void* const* w, cudaStream_t s) {
       TXS_CK(launch_to_f32<T>(W(l, idx[i]), v, len[i], s));
       *dst[i] = v;
     }
-    TXS_CK(launch_to_f32<T>(W(l, 9), m->b_kv + size_t(2 * l) * d, d, s));
-    TXS_CK(launch_to_f32<T>(W(l, 11), m->b_kv + size_t(2 * l + 1) * d, d, s));
+    TXS_CK(launch_to_f32<T>(W(l, 9), m->b_kv + size_t(2 * l) * dkv, dkv, s));
+    TXS_CK(launch_to_f32<T>(W(l, 11), m->b_kv + size_t(2 * l + 1) * dkv, dkv, s));
     m->layers.push_back(L);
   }
   const void* const* head = w + nL * TXS_WEIGHTS_PER_LAYER;
@@ -278,8 +283,8 @@ txs_status model_prepare(txs_model* m, const void* const* w, cudaStream_t s) {
   const size_t es = sizeof(T);
   for (int l = 0; l < nL; ++l) {
     const size_t n[TXS_WEIGHTS_PER_LAYER] = {size_t(d) * 3 * d, 3 * size_t(d), size_t(d) * d, size_t(d), size_t(d),
-                                             size_t(d), size_t(d) * d, size_t(d), size_t(d) * d, size_t(d),
-                                             size_t(d) * d, size_t(d), size_t(d) * d, size_t(d), size_t(d), size_t(d),
+                                             size_t(d), size_t(d) * d, size_t(d), size_t(d) * dkv, size_t(dkv),
+                                             size_t(d) * dkv, size_t(dkv), size_t(d) * d, size_t(d), size_t(d), size_t(d),
                                              size_t(d) * F, size_t(F), size_t(F) * d, size_t(d), size_t(d), size_t(d)};
     for (int i = 0; i < TXS_WEIGHTS_PER_LAYER; ++i)
       TXS_CK(launch_hash(W(l, i), static_cast<long long>(n[i] * es), uint64_t(l) * 64 + i + 1, dh, s));
@@ -292,7 +297,7 @@ txs_status model_prepare(txs_model* m, const void* const* w, cudaStream_t s) {
   TXS_CK(cudaStreamSynchronize(s));
   uint64_t h = hv;
   const int32_t cf[] = {c.d_model, c.n_heads, c.d_ff, c.n_layers, c.n_actions, c.n_ctx, c.l_local, c.attn_mode,
-                        c.dtype};
+                        c.dtype, kv_dim(c)};
   for (int32_t v : cf) h = (h ^ static_cast<uint64_t>(static_cast<uint32_t>(v))) * 0x100000001B3ull;
   uint32_t eps_bits;
   std::memcpy(&eps_bits, &c.ln_eps, 4);
@@ -338,20 +343,21 @@ txs_status project_rows(txs_model* m, txs_kv_cache* c, int n_req, const int32_t*
   }
   TXS_CK(stage_upload(c, c->d_in_off, up.data(), 2 * n_req + 1, s));
   if (total > 0) {
-    EpiArgs e = epi_base(EPI_KV, total, 2 * nL * d, d);
+    const int dkv = c->dkv;
+    EpiArgs e = epi_base(EPI_KV, total, 2 * nL * dkv, d);
     e.bias = m->b_kv;
     e.out = c->kv;
-    e.ldo = d;
+    e.ldo = dkv;
     e.seg_off = c->d_in_off;
     e.dst_row0 = c->d_dst0;
     e.n_seg = n_req;
-    e.col_blk = d;
-    e.col_blk_stride = c->cap_total * d;
+    e.col_blk = dkv;
+    e.col_blk_stride = c->cap_total * dkv;
     TXS_CK(gemm(m, rows, d, m->Wt_kv, e, nullptr, s, KC_GEMM_KV));
   }
   TXS_CK(launch_pool<T>(static_cast<const T*>(rows), c->d_in_off, n_req, max_rows, m->w_pool, d, c->max_chunks,
                         c->part, append ? 1 : 0, c->pool_m, c->pool_s, c->pool_acc, c->g, c->pool_cnt, s));
-  TXS_CK(launch_anchor_proj<T>(c->g, static_cast<const T*>(m->Wt_kv), m->b_kv, c->gkv, n_req, d, nL, s));
+  TXS_CK(launch_anchor_proj<T>(c->g, static_cast<const T*>(m->Wt_kv), m->b_kv, c->gkv, n_req, d, c->dkv, nL, s));
   return TXS_OK;
 }
 
@@ -359,11 +365,11 @@ txs_status project_rows(txs_model* m, txs_kv_cache* c, int n_req, const int32_t*
 // a user) sees rows [off[r], off[r] + len[r]) of every layer's K/V and the
 // anchor projections gkv[l][0|1][r].
 struct KvView {
-  const void* kv;          // [nL][2][cap_total][d]
+  const void* kv;          // [nL][2][cap_total][dkv]
   long long cap_total;
   const int* off;          // device [n]
   const int* len;          // device [n]
-  const float* gkv;        // device [nL][2][n][d]
+  const float* gkv;        // device [nL][2][n][dkv]
 };
 
 template <typename T>
@@ -371,6 +377,7 @@ txs_status score_impl(txs_model* m, const KvView& c, int n_req, const int32_t* c
                       const void* ctx_tok, void* ws, float* logits, float* probs, cudaStream_t s) {
   const txs_config& cf = m->cfg;
   const int d = cf.d_model, F = cf.d_ff, H = cf.n_heads, S = cf.n_ctx, k = cf.n_actions;
+  const int dkv = kv_dim(cf), Hkv = dkv / (d / H);
   const long long n_cand = cand_off[n_req];
   const long long N = n_cand + static_cast<long long>(n_req) * S;
   const ScoreLayout L = score_layout(cf, sizeof(T), n_req, n_cand);
@@ -414,27 +421,27 @@ txs_status score_impl(txs_model* m, const KvView& c, int n_req, const int32_t* c
     e.out = QKV;
     e.ldo = d;
     TXS_CK(gemm(m, X1, d, W.Wt_q, e, tmp, s, KC_GEMM_Q));
-    const T* Kc = kv + (size_t(2 * l) * c.cap_total) * d;
-    const T* Vc = kv + (size_t(2 * l + 1) * c.cap_total) * d;
-    const float* Kg = c.gkv + size_t(2 * l) * n_req * d;
-    const float* Vg = c.gkv + size_t(2 * l + 1) * n_req * d;
+    const T* Kc = kv + (size_t(2 * l) * c.cap_total) * dkv;
+    const T* Vc = kv + (size_t(2 * l + 1) * c.cap_total) * dkv;
+    const float* Kg = c.gkv + size_t(2 * l) * n_req * dkv;
+    const float* Vg = c.gkv + size_t(2 * l + 1) * n_req * dkv;
     cudaError_t lg = cudaErrorNotSupported;
     if (cf.attn_mode == TXS_ATTN_LOCAL_GLOBAL)
       lg = launch_cross_attn_lg<T>(QKV, A, Kc, Vc, cand_off_dev, cand_off, n_req, static_cast<int>(n_cand), S,
-                                   c.off, c.len, Kg, Vg, cf.l_local, H, d, s);
+                                   c.off, c.len, Kg, Vg, cf.l_local, H, Hkv, d, s);
     if (lg != cudaErrorNotSupported) {
       if (lg != cudaSuccess) return fail_cuda("cross-attention", lg);
     } else if constexpr (std::is_same<T, __nv_bfloat16>::value) {
       if (cf.attn_mode == TXS_ATTN_FULL && fa_full_supported(d, H, c.cap_total)) {
         TXS_CK(launch_fa_full(QKV, A, Kc, Vc, c.cap_total, cand_off_dev, cand_off, c.off, c.len, n_req,
-                              static_cast<int>(n_cand), S, H, d, m->status, s));
+                              static_cast<int>(n_cand), S, H, Hkv, d, m->status, s));
       } else {
         TXS_CK(launch_cross_attn<T>(QKV, A, Kc, Vc, row_req, static_cast<int>(N), c.off, c.len, Kg, Vg,
-                                    cf.l_local, cf.attn_mode, H, d, s));
+                                    cf.l_local, cf.attn_mode, H, Hkv, d, s));
       }
     } else {
       TXS_CK(launch_cross_attn<T>(QKV, A, Kc, Vc, row_req, static_cast<int>(N), c.off, c.len, Kg, Vg,
-                                  cf.l_local, cf.attn_mode, H, d, s));
+                                  cf.l_local, cf.attn_mode, H, Hkv, d, s));
     }
     e = epi_base(EPI_LN, N, d, d);
     e.bias = W.b_oc;
@@ -565,6 +572,7 @@ txs_status make_cache(txs_model* m, int n_req, const int* lengths, int capacity_
   c->n_req = n_req;
   c->n_layers = nL;
   c->d = d;
+  c->dkv = kv_dim(cf);
   c->es = m->es;
   c->cap_extra = capacity_extra;
   c->model_hash = m->hash;
@@ -595,7 +603,7 @@ txs_status make_cache(txs_model* m, int n_req, const int* lengths, int capacity_
     if (!p) st = fail_cuda("cudaMalloc", err);
     return p;
   };
-  c->kv = A(size_t(nL) * 2 * tot * d * m->es);
+  c->kv = A(size_t(nL) * 2 * tot * c->dkv * m->es);
   c->d_off = static_cast<int*>(A(4 * (n_req + 1)));
   c->d_len = static_cast<int*>(A(4 * n_req));
   c->d_in_off = static_cast<int*>(A(4 * (2 * n_req + 1)));
@@ -604,7 +612,7 @@ txs_status make_cache(txs_model* m, int n_req, const int* lengths, int capacity_
   c->pool_s = static_cast<float*>(A(4 * n_req));
   c->pool_acc = static_cast<float*>(A(size_t(4) * n_req * d));
   c->g = static_cast<float*>(A(size_t(4) * n_req * d));
-  c->gkv = static_cast<float*>(A(size_t(4) * nL * 2 * n_req * d));
+  c->gkv = static_cast<float*>(A(size_t(4) * nL * 2 * n_req * c->dkv));
   c->part = static_cast<float*>(A(size_t(4) * n_req * c->max_chunks * (d + 2)));
   c->pool_cnt = static_cast<int*>(A(size_t(4) * n_req));
   if (st == TXS_OK && (err = cudaMemsetAsync(c->pool_cnt, 0, size_t(4) * n_req, s)) != cudaSuccess)
@@ -675,12 +683,12 @@ struct CacheHeader {
   char magic[8];
   uint32_t format, schema;
   uint64_t model_hash;
-  int32_t n_req, n_layers, d_model, elem_bytes;
+  int32_t n_req, n_layers, d_model, d_kv, elem_bytes, reserved;
   int64_t total_rows;
 };
-size_t cache_blob_bytes(int n_req, int nL, int d, int es, long long rows) {
-  return sizeof(CacheHeader) + sizeof(int32_t) * n_req + size_t(nL) * 2 * rows * d * es +
-         sizeof(float) * (2 * size_t(n_req) + size_t(2) * n_req * d + size_t(nL) * 2 * n_req * d);
+size_t cache_blob_bytes(int n_req, int nL, int d, int dkv, int es, long long rows) {
+  return sizeof(CacheHeader) + sizeof(int32_t) * n_req + size_t(nL) * 2 * rows * dkv * es +
+         sizeof(float) * (2 * size_t(n_req) + size_t(2) * n_req * d + size_t(nL) * 2 * n_req * dkv);
 }
 }  // namespace
 
@@ -688,7 +696,7 @@ TXS_API txs_status txs_cache_export_size(const txs_kv_cache* c, size_t* bytes) {
   if (!c || !bytes) return TXS_ERR_INVALID_ARG;
   long long rows = 0;
   for (int r = 0; r < c->n_req; ++r) rows += c->h_len[r];
-  *bytes = cache_blob_bytes(c->n_req, c->n_layers, c->d, c->es, rows);
+  *bytes = cache_blob_bytes(c->n_req, c->n_layers, c->d, c->dkv, c->es, rows);
   return TXS_OK;
 }
 
@@ -699,7 +707,7 @@ TXS_API txs_status txs_cache_export(const txs_kv_cache* c, uint32_t schema_versi
   txs_cache_export_size(c, &need);
   if (bytes < need) return TXS_ERR_INVALID_ARG;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
-  const int R = c->n_req, nL = c->n_layers, d = c->d, es = c->es;
+  const int R = c->n_req, nL = c->n_layers, d = c->d, dkv = c->dkv, es = c->es;
   uint8_t* p = static_cast<uint8_t*>(host_buf);
   CacheHeader h;
   std::memcpy(h.magic, kCacheMagic, 8);
@@ -709,7 +717,9 @@ TXS_API txs_status txs_cache_export(const txs_kv_cache* c, uint32_t schema_versi
   h.n_req = R;
   h.n_layers = nL;
   h.d_model = d;
+  h.d_kv = dkv;
   h.elem_bytes = es;
+  h.reserved = 0;
   h.total_rows = 0;
   for (int r = 0; r < R; ++r) h.total_rows += c->h_len[r];
   std::memcpy(p, &h, sizeof(h));
@@ -721,8 +731,8 @@ TXS_API txs_status txs_cache_export(const txs_kv_cache* c, uint32_t schema_versi
   for (int l = 0; l < nL && err == cudaSuccess; ++l)
     for (int w = 0; w < 2 && err == cudaSuccess; ++w)
       for (int r = 0; r < R && err == cudaSuccess; ++r) {
-        const size_t n = size_t(c->h_len[r]) * d * es;
-        const size_t src = ((size_t(2 * l + w) * c->cap_total) + c->h_off[r]) * d * es;
+        const size_t n = size_t(c->h_len[r]) * dkv * es;
+        const size_t src = ((size_t(2 * l + w) * c->cap_total) + c->h_off[r]) * dkv * es;
         err = cudaMemcpyAsync(p, kv + src, n, cudaMemcpyDeviceToHost, s);
         p += n;
       }
@@ -734,7 +744,7 @@ TXS_API txs_status txs_cache_export(const txs_kv_cache* c, uint32_t schema_versi
   grab(c->pool_s, R);
   grab(c->pool_acc, size_t(R) * d);
   grab(c->g, size_t(R) * d);
-  grab(c->gkv, size_t(nL) * 2 * R * d);
+  grab(c->gkv, size_t(nL) * 2 * R * dkv);
   if (err == cudaSuccess) err = cudaStreamSynchronize(s);
   if (err != cudaSuccess) return fail_cuda("cache export", err);
   return TXS_OK;
@@ -751,9 +761,10 @@ TXS_API txs_status txs_cache_import(txs_model* m, uint32_t schema_version, const
   // entries of another model or feature schema are stale, never reinterpreted
   if (h.model_hash != m->hash || h.schema != schema_version) return TXS_ERR_STALE_CACHE;
   const txs_config& cf = m->cfg;
-  if (h.n_layers != cf.n_layers || h.d_model != cf.d_model || h.elem_bytes != m->es) return TXS_ERR_STALE_CACHE;
+  if (h.n_layers != cf.n_layers || h.d_model != cf.d_model || h.d_kv != kv_dim(cf) || h.elem_bytes != m->es)
+    return TXS_ERR_STALE_CACHE;
   if (h.n_req < 1 || h.n_req > kMaxReqParam || h.total_rows < 0) return TXS_ERR_INVALID_ARG;
-  const int R = h.n_req, nL = h.n_layers, d = h.d_model, es = h.elem_bytes;
+  const int R = h.n_req, nL = h.n_layers, d = h.d_model, dkv = h.d_kv, es = h.elem_bytes;
   if (bytes < sizeof(h) + sizeof(int32_t) * R) return TXS_ERR_INVALID_ARG;
   std::vector<int> len(R);
   std::memcpy(len.data(), static_cast<const uint8_t*>(host_buf) + sizeof(h), sizeof(int32_t) * R);
@@ -762,7 +773,7 @@ TXS_API txs_status txs_cache_import(txs_model* m, uint32_t schema_version, const
     if (len[r] < 1) return TXS_ERR_INVALID_ARG;
     rows += len[r];
   }
-  if (rows != h.total_rows || bytes < cache_blob_bytes(R, nL, d, es, rows)) return TXS_ERR_INVALID_ARG;
+  if (rows != h.total_rows || bytes < cache_blob_bytes(R, nL, d, dkv, es, rows)) return TXS_ERR_INVALID_ARG;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   txs_kv_cache* c = nullptr;
   txs_status st = make_cache(m, R, len.data(), capacity_extra, s, &c);
@@ -773,8 +784,8 @@ TXS_API txs_status txs_cache_import(txs_model* m, uint32_t schema_version, const
   for (int l = 0; l < nL && err == cudaSuccess; ++l)
     for (int w = 0; w < 2 && err == cudaSuccess; ++w)
       for (int r = 0; r < R && err == cudaSuccess; ++r) {
-        const size_t n = size_t(len[r]) * d * es;
-        const size_t dst = ((size_t(2 * l + w) * c->cap_total) + c->h_off[r]) * d * es;
+        const size_t n = size_t(len[r]) * dkv * es;
+        const size_t dst = ((size_t(2 * l + w) * c->cap_total) + c->h_off[r]) * dkv * es;
         err = cudaMemcpyAsync(kv + dst, p, n, cudaMemcpyHostToDevice, s);
         p += n;
       }
@@ -786,7 +797,7 @@ TXS_API txs_status txs_cache_import(txs_model* m, uint32_t schema_version, const
   put(c->pool_s, R);
   put(c->pool_acc, size_t(R) * d);
   put(c->g, size_t(R) * d);
-  put(c->gkv, size_t(nL) * 2 * R * d);
+  put(c->gkv, size_t(nL) * 2 * R * dkv);
   // the host buffer may be released as soon as this returns
   if (err == cudaSuccess) err = cudaStreamSynchronize(s);
   if (err != cudaSuccess) {
@@ -862,7 +873,7 @@ TXS_API txs_status txs_cache_read_rows(const txs_kv_cache* c, int32_t layer, int
       row0 < 0 || n_rows < 0 || static_cast<long long>(row0) + n_rows > c->h_len[req])
     return TXS_ERR_INVALID_ARG;
   if (n_rows == 0) return TXS_OK;
-  const size_t row_bytes = size_t(c->d) * c->es;
+  const size_t row_bytes = size_t(c->dkv) * c->es;
   const size_t blk = size_t(2 * layer + which) * c->cap_total;
   const uint8_t* src = static_cast<const uint8_t*>(c->kv) + (blk + c->h_off[req] + row0) * row_bytes;
   cudaError_t err = cudaMemcpyAsync(dst, src, n_rows * row_bytes, cudaMemcpyDeviceToDevice,
@@ -874,8 +885,8 @@ TXS_API txs_status txs_cache_read_anchor(const txs_kv_cache* c, int32_t layer, i
                                          void* stream) {
   if (!c || !dst || which < 0 || which > 2 || (which < 2 && (layer < 0 || layer >= c->n_layers)))
     return TXS_ERR_INVALID_ARG;
-  const size_t bytes = size_t(c->n_req) * c->d * 4;
-  const float* src = which == 2 ? c->g : c->gkv + size_t(2 * layer + which) * c->n_req * c->d;
+  const size_t bytes = size_t(c->n_req) * (which == 2 ? c->d : c->dkv) * 4;
+  const float* src = which == 2 ? c->g : c->gkv + size_t(2 * layer + which) * c->n_req * c->dkv;
   cudaError_t err = cudaMemcpyAsync(dst, src, bytes, cudaMemcpyDeviceToDevice, static_cast<cudaStream_t>(stream));
   return err == cudaSuccess ? TXS_OK : fail_cuda("read anchor", err);
 }
@@ -928,7 +939,7 @@ EventsLayout events_layout(const txs_config& cf, int es, int n_ev, long long n_c
   L.ev_off = take(sizeof(int) * n_ev);
   L.ev_len = take(sizeof(int) * n_ev);
   L.g = take(sizeof(float) * n_ev * cf.d_model);
-  L.gkv = take(sizeof(float) * 2 * cf.n_layers * n_ev * cf.d_model);
+  L.gkv = take(sizeof(float) * 2 * cf.n_layers * n_ev * kv_dim(cf));
   L.part = take(sizeof(float) * prefix_pool_scratch_floats(max_end, cf.d_model));
   L.total = o;
   return L;
@@ -959,7 +970,7 @@ txs_status events_impl(txs_model* m, const txs_kv_cache* c, int user, const void
   // per-event anchors pooled over each prefix, projected by every layer's W_K, W_V
   TXS_CK(launch_prefix_pool<T>(static_cast<const T*>(beh_enc), ends, n_ev, c->h_off[user], m->w_pool, d, part, g,
                                ev_off, ev_len, s));
-  TXS_CK(launch_anchor_proj<T>(g, static_cast<const T*>(m->Wt_kv), m->b_kv, gkv, n_ev, d, nL, s));
+  TXS_CK(launch_anchor_proj<T>(g, static_cast<const T*>(m->Wt_kv), m->b_kv, gkv, n_ev, d, c->dkv, nL, s));
   const KvView v{c->kv, c->cap_total, ev_off, ev_len, gkv};
   return score_impl<T>(m, v, n_ev, cand_off, cand_tok, ctx_tok, ws, logits, probs, s);
 }

@@ -172,12 +172,12 @@ cudaError_t launch_serving_attn(const T* qkv, T* out, const int* row_req, int n_
 template <typename T>
 cudaError_t launch_cross_attn_lg(const T* q, T* out, const T* Kc, const T* Vc, const int* cand_off_dev,
                                  const int* cand_off_host, int n_req, int n_cand, int S, const int* kv_off,
-                                 const int* kv_len, const float* Kg, const float* Vg, int l_local, int H, int d,
-                                 cudaStream_t s);
+                                 const int* kv_len, const float* Kg, const float* Vg, int l_local, int H, int Hkv,
+                                 int d, cudaStream_t s);
 template <typename T>
 cudaError_t launch_cross_attn(const T* q, T* out, const T* Kc, const T* Vc, const int* row_req, int n_rows,
                               const int* kv_off, const int* kv_len, const float* Kg, const float* Vg, int l_local,
-                              int mode, int H, int d, cudaStream_t s);
+                              int mode, int H, int Hkv, int d, cudaStream_t s);
 
 // FULL-mode cross-attention on the tensor cores (bf16): one CTA per
 // (128-query tile, request, head).
@@ -185,7 +185,7 @@ bool fa_full_supported(int d, int H, long long cap_total);
 cudaError_t launch_fa_full(const __nv_bfloat16* q, __nv_bfloat16* out, const __nv_bfloat16* Kc,
                            const __nv_bfloat16* Vc, long long cap_total, const int* cand_off_dev,
                            const int* cand_off_host, const int* kv_off, const int* kv_len, int n_req, int n_cand,
-                           int S, int H, int d, int* status, cudaStream_t s);
+                           int S, int H, int Hkv, int d, int* status, cudaStream_t s);
 
 extern const int kPoolChunk;
 template <typename T>
@@ -201,7 +201,7 @@ template <typename T>
 cudaError_t launch_prefix_pool(const T* phi, const int* ends, int n_ev, int off_user, const float* w_pool, int d,
                                float* part, float* g, int* ev_off, int* ev_len, cudaStream_t s);
 template <typename T>
-cudaError_t launch_anchor_proj(const float* g, const T* Wt_kv, const float* b_kv, float* gkv, int R, int d,
+cudaError_t launch_anchor_proj(const float* g, const T* Wt_kv, const float* b_kv, float* gkv, int R, int d, int dkv,
                                int n_layers, cudaStream_t s);
 template <typename T>
 cudaError_t launch_transpose(const T* W, T* Wt, int rows, int cols, cudaStream_t s);

@@ -47,7 +47,7 @@ class txs_config(ctypes.Structure):
     _fields_ = [("d_model", ctypes.c_int32), ("n_heads", ctypes.c_int32), ("d_ff", ctypes.c_int32),
                 ("n_layers", ctypes.c_int32), ("n_actions", ctypes.c_int32), ("n_ctx", ctypes.c_int32),
                 ("l_local", ctypes.c_int32), ("attn_mode", ctypes.c_int32), ("dtype", ctypes.c_int32),
-                ("ln_eps", ctypes.c_float)]
+                ("ln_eps", ctypes.c_float), ("n_kv_heads", ctypes.c_int32)]
 
 
 _lib: Optional[ctypes.CDLL] = None
@@ -140,9 +140,14 @@ def torch_dtype(dtype: str) -> torch.dtype:
     return torch.bfloat16 if dtype == "bf16" else torch.float32
 
 
+def kv_width(wl: W.Workload) -> int:
+    """Width of a cached K or V row: n_kv_heads * d_head."""
+    return (wl.n_kv_heads or wl.n_heads) * (wl.d_model // wl.n_heads)
+
+
 def make_config(wl: W.Workload, mode: int = LOCAL_GLOBAL) -> txs_config:
     return txs_config(wl.d_model, wl.n_heads, wl.d_ff, wl.n_layers, wl.n_actions, wl.n_ctx, wl.l_local, mode,
-                      TXS_BF16 if wl.dtype == "bf16" else TXS_FP32, wl.ln_eps)
+                      TXS_BF16 if wl.dtype == "bf16" else TXS_FP32, wl.ln_eps, wl.n_kv_heads)
 
 
 def weight_order(n_layers: int) -> Sequence[str]:
@@ -216,13 +221,14 @@ class KVCache:
         return out
 
     def read_rows(self, layer: int, which: int, req: int, row0: int, n_rows: int, stream=None) -> torch.Tensor:
-        out = torch.empty((n_rows, self.model.wl.d_model), dtype=self.model.dtype, device="cuda")
+        out = torch.empty((n_rows, kv_width(self.model.wl)), dtype=self.model.dtype, device="cuda")
         _check(lib().txs_cache_read_rows(self.handle, layer, which, req, row0, n_rows, _ptr(out), _stream(stream)),
                "txs_cache_read_rows")
         return out
 
     def read_anchor(self, layer: int, which: int, stream=None) -> torch.Tensor:
-        out = torch.empty((self.n_req, self.model.wl.d_model), dtype=torch.float32, device="cuda")
+        width = self.model.wl.d_model if which == 2 else kv_width(self.model.wl)
+        out = torch.empty((self.n_req, width), dtype=torch.float32, device="cuda")
         _check(lib().txs_cache_read_anchor(self.handle, layer, which, _ptr(out), _stream(stream)),
                "txs_cache_read_anchor")
         return out

@@ -51,7 +51,7 @@ def _cfg(**kw):
 @pytest.mark.parametrize("bad", [
     dict(d_model=96), dict(n_heads=3), dict(n_heads=2), dict(d_ff=100), dict(n_actions=0),
     dict(n_actions=17), dict(n_ctx=9), dict(l_local=0), dict(attn_mode=2), dict(dtype=5),
-    dict(ln_eps=0.0), dict(n_layers=0),
+    dict(ln_eps=0.0), dict(n_layers=0), dict(n_kv_heads=3), dict(n_kv_heads=-1),
 ])
 def test_model_create_rejects_bad_config_on_host(lib, bad):
     cfg = _cfg(**bad)
@@ -70,6 +70,13 @@ def test_null_arguments_rejected(lib):
     assert lib.txs_score_candidates(None, None, 1, None, None, None, None, 0, None, None, None) == \
         txs.TXS_ERR_INVALID_ARG
     assert lib.txs_device_status(None) == txs.TXS_ERR_INVALID_ARG
+    assert lib.txs_score_events(None, None, 0, None, 1, None, None, None, None, None, 0, None, None, None) == \
+        txs.TXS_ERR_INVALID_ARG
+    n = ctypes.c_size_t()
+    assert lib.txs_events_workspace_size(None, 1, 1, 1, ctypes.byref(n)) == txs.TXS_ERR_INVALID_ARG
+    assert lib.txs_cache_export_size(None, ctypes.byref(n)) == txs.TXS_ERR_INVALID_ARG
+    assert lib.txs_cache_export(None, 0, None, 0, None) == txs.TXS_ERR_INVALID_ARG
+    assert lib.txs_cache_import(None, 0, None, 0, 0, None, ctypes.byref(h)) == txs.TXS_ERR_INVALID_ARG
 
 
 def test_rank_rejects_bad_arguments_on_host(lib):
