@@ -28,6 +28,9 @@ What it computes (row-vector convention ``y = x W + b``):
   X2 = LN(X1 + MHA(X1 W_Q + b_Q, K_I, V_I)) (the sparse cross-attention
   equation, scale 1/sqrt(d_h));
   X3 = LN(X2 + GELU(X2 W_1 + b_1) W_2 + b_2).
+* Candidate encoder (Sec. 4.1.2, Phi_candidate "a multi-layer perceptron"):
+  optional, GELU(x W_c1 + b_c1) W_c2 + b_c2 on each candidate token before
+  the decoder; the head still takes the raw token x.
 * Head (Sec. 4.1.3, the action-decoding equation): for candidate rows,
   ``k_dec = [z, x] W_dec + b_dec`` (linear f_dec, Sec. 4.4), logits
   ``= Q_dec k_dec`` (no scale), probabilities ``= softmax(logits)``.
@@ -115,6 +118,7 @@ class Model:
     l_local: int
     ln_eps: float
     n_kv_heads: int = 0   # K/V heads of the cache; 0 or n_heads: one per query head
+    cand_mlp: int = 0     # hidden width of the candidate-to-query MLP; 0: none
 
     @property
     def kv_heads(self) -> int:
@@ -124,7 +128,7 @@ class Model:
     def from_arrays(weights: Dict[str, np.ndarray], wl) -> "Model":
         return Model({k: np.asarray(v, dtype=np.float64) for k, v in weights.items()},
                      wl.n_layers, wl.d_model, wl.n_heads, wl.n_ctx, wl.n_actions,
-                     wl.l_local, wl.ln_eps, getattr(wl, "n_kv_heads", 0))
+                     wl.l_local, wl.ln_eps, getattr(wl, "n_kv_heads", 0), getattr(wl, "cand_mlp", 0))
 
 
 @dataclass
@@ -269,13 +273,23 @@ def head(model: Model, z: np.ndarray, x: np.ndarray):
     return logits, softmax(logits, axis=-1)
 
 
+def candidate_encoder(model: Model, cand: np.ndarray) -> np.ndarray:
+    """Phi_candidate (Sec. 4.1.2): with a candidate MLP, GELU(x W_c1 + b_c1) W_c2
+    + b_c2 per candidate; without one the tokens are already its outputs."""
+    if not model.cand_mlp:
+        return cand
+    w = model.w
+    return gelu(cand @ w["W_c1"] + w["b_c1"]) @ w["W_c2"] + w["b_c2"]
+
+
 def score_request(model: Model, cache: RequestCache, ctx: np.ndarray, cand: np.ndarray,
                   mode: int = LOCAL_GLOBAL, use_global: bool = True):
-    """Scores of one request's candidates: (logits [M, k], probs [M, k])."""
+    """Scores of one request's candidates: (logits [M, k], probs [M, k]).  The
+    decoder sees Phi_candidate(x); the head f_dec(z, x) the raw token x."""
     ctx = np.asarray(ctx, dtype=np.float64).reshape(-1, model.d_model)
     cand = np.asarray(cand, dtype=np.float64)
     S = ctx.shape[0]
-    X = np.concatenate([ctx, cand], axis=0)
+    X = np.concatenate([ctx, candidate_encoder(model, cand)], axis=0)
     for l in range(model.n_layers):
         Kc, Vc = key_set(model, cache, l, mode, use_global)
         X = decoder_layer(model, X, Kc, Vc, l, S)

@@ -49,6 +49,10 @@ LAYER_WEIGHTS: Tuple[Tuple[str, str], ...] = (
 HEAD_WEIGHTS: Tuple[Tuple[str, str], ...] = (
     ("w_pool", "d"), ("W_dec", "2d,d"), ("b_dec", "d"), ("Q_dec", "k,d"),
 )
+# candidate-to-query MLP (drawn after the head, only when cand_mlp > 0)
+CAND_WEIGHTS: Tuple[Tuple[str, str], ...] = (
+    ("W_c1", "d,Fc"), ("b_c1", "Fc"), ("W_c2", "Fc,d"), ("b_c2", "d"),
+)
 
 SizeSpec = Union[int, Tuple[str, int, int], Sequence[int]]
 
@@ -72,6 +76,7 @@ class Workload:
     dL: SizeSpec = 0        # appended behavior rows per request
     capacity_extra: int = 64
     n_kv_heads: int = 0     # K/V heads of the cache (0: one per query head)
+    cand_mlp: int = 0       # hidden width of the candidate-to-query MLP (0: none)
 
     @property
     def d_head(self) -> int:
@@ -140,7 +145,7 @@ def sizes(wl: Workload) -> Tuple[np.ndarray, np.ndarray, np.ndarray]:
 def _shape(code: str, wl: Workload) -> Tuple[int, ...]:
     dkv = (wl.n_kv_heads or wl.n_heads) * (wl.d_model // wl.n_heads)
     env = {"d": wl.d_model, "3d": 3 * wl.d_model, "2d": 2 * wl.d_model,
-           "F": wl.d_ff, "k": wl.n_actions, "dkv": dkv}
+           "F": wl.d_ff, "k": wl.n_actions, "dkv": dkv, "Fc": wl.cand_mlp}
     return tuple(env[c] for c in code.split(","))
 
 
@@ -158,6 +163,9 @@ def weights(wl: Workload) -> Dict[str, np.ndarray]:
             out[f"{name}.{l}"] = _store(wl, x)
     for name, code in HEAD_WEIGHTS:
         out[name] = _store(wl, rng.standard_normal(_shape(code, wl)) * 0.02)
+    if wl.cand_mlp:
+        for name, code in CAND_WEIGHTS:
+            out[name] = _store(wl, rng.standard_normal(_shape(code, wl)) * 0.02)
     return out
 
 

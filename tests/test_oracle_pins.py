@@ -229,9 +229,11 @@ def _torch_layer(model, l):
     return layer
 
 
-def torch_score(model, phi, ctx, cand, mode, use_global=True):
+def torch_score(model, phi, ctx, cand, mode, use_global=True, head_x=None):
     """Independent recompute with PyTorch modules: K/V are projected from Phi_b
-    (and from the pooled g) inside torch's cross-attention, per call."""
+    (and from the pooled g) inside torch's cross-attention, per call.  ``cand``
+    enters the decoder; the head takes ``head_x`` (default: ``cand``)."""
+    head_x = cand if head_x is None else head_x
     S = ctx.shape[0]
     if mode == O.FULL:
         memory = phi
@@ -252,7 +254,7 @@ def torch_score(model, phi, ctx, cand, mode, use_global=True):
         for l in range(model.n_layers):
             X = _torch_layer(model, l)(X, mem, tgt_mask=blocked)
     z = X[0, S:].numpy()
-    kdec = torch.nn.functional.linear(torch.from_numpy(np.concatenate([z, cand], 1)),
+    kdec = torch.nn.functional.linear(torch.from_numpy(np.concatenate([z, head_x], 1)),
                                       torch.from_numpy(model.w["W_dec"].T.copy()),
                                       torch.from_numpy(model.w["b_dec"]))
     logits = kdec @ torch.from_numpy(model.w["Q_dec"]).T
