@@ -70,6 +70,9 @@ typedef struct {
                         Sec. 4.1.2): 0 = n_heads; otherwise divides n_heads, and
                         query head h uses K/V head h / (n_heads / n_kv_heads).  The
                         cached rows are n_kv_heads * d_head wide.                   */
+  int32_t cand_mlp_hidden; /* hidden width Fc of the candidate-to-query MLP
+                        Phi_candidate (Sec. 4.1.2; multiple of 64, <= 16384), or 0
+                        when the candidate tokens already are its outputs       */
 } txs_config;
 
 typedef struct txs_model txs_model;       /* opaque */
@@ -83,7 +86,8 @@ typedef struct txs_kv_cache txs_kv_cache; /* opaque */
 /*
  * txs_model_create — copy the decoder weights into the library's device layout.
  *
- * `weights` (host array of device pointers) holds n_layers * 22 + 4 pointers,
+ * `weights` (host array of device pointers) holds n_layers * 22 + 4 (+ 4)
+ * pointers,
  * layer by layer, then the head, in this order and with these shapes
  * (d = d_model, F = d_ff, k = n_actions, dkv = n_kv_heads * d_head, which is d
  * when n_kv_heads is 0 or n_heads), all in the config's dtype:
@@ -94,6 +98,10 @@ typedef struct txs_kv_cache txs_kv_cache; /* opaque */
  *    16 W_1  [d,F]   17 b_1  [F]    18 W_2 [F,d]  19 b_2 [d]  20 ln3_g [d] 21 ln3_b [d]
  *   head (Sec. 4.1.3; attention pooling Sec. 5.1):
  *     w_pool [d], W_dec [2d,d], b_dec [d], Q_dec [k,d]
+ *   then, when cand_mlp_hidden = Fc > 0, the candidate MLP (4 more pointers):
+ *     W_c1 [d,Fc], b_c1 [Fc], W_c2 [Fc,d], b_c2 [d]
+ *   (the decoder sees GELU(x W_c1 + b_c1) W_c2 + b_c2 for each candidate
+ *   token x; the head's f_dec(z, x) keeps the raw x)
  * The call synchronises the device first (the weights may still be in flight
  * on any stream) and returns after the copies are done; the inputs may be
  * freed afterwards.  The model keeps a 64-bit content hash of config and weights.

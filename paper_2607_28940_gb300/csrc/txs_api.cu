@@ -78,6 +78,8 @@ struct txs_model {
   float* w_pool = nullptr;       // [d]
   float* weff = nullptr;         // [2d, k]
   float* cdec = nullptr;         // [k]
+  void *Wt_c1 = nullptr, *Wt_c2 = nullptr;  // candidate MLP, transposed: [Fc, d], [d, Fc]
+  float *b_c1 = nullptr, *b_c2 = nullptr;
   int* status = nullptr;         // device status word
   uint64_t hash = 0;
 };
@@ -130,6 +132,7 @@ bool cfg_ok(const txs_config& c, std::string* why) {
   if (c.l_local < 1) return bad("l_local");
   if (!(c.ln_eps > 0.f) || !std::isfinite(c.ln_eps)) return bad("ln_eps");
   if (c.n_kv_heads < 0 || (c.n_kv_heads > 0 && c.n_heads % c.n_kv_heads)) return bad("n_kv_heads");
+  if (c.cand_mlp_hidden < 0 || c.cand_mlp_hidden % 64 || c.cand_mlp_hidden > 16384) return bad("cand_mlp_hidden");
   return true;
 }
 
@@ -179,7 +182,7 @@ ScoreLayout score_layout(const txs_config& c, int es, int n_req, long long n_can
   L.A = take(N * d * es);
   L.X1 = take(N * d * es);
   L.X2 = take(N * d * es);
-  L.Hf = take(N * F * es);
+  L.Hf = take(N * std::max(F, static_cast<size_t>(c.cand_mlp_hidden)) * es);
   L.xlog = take(n_cand * c.n_actions * 4);
   L.tmp = take(c.dtype == TXS_FP32 ? N * d * 4 : 0);
   L.total = o;
@@ -276,6 +279,17 @@ txs_status model_prepare(txs_model* m, const void* const* w, cudaStream_t s) {
   if (!(m->cdec = vf(k))) return fail_cuda("cudaMalloc", err);
   TXS_CK(launch_fold_head<T>(static_cast<const T*>(head[1]), static_cast<const T*>(head[2]),
                              static_cast<const T*>(head[3]), m->weff, m->cdec, d, k, s));
+  // candidate-to-query MLP (optional)
+  const int Fc = c.cand_mlp_hidden;
+  const void* const* cm = head + TXS_HEAD_WEIGHTS;
+  if (Fc) {
+    if (!(m->Wt_c1 = wt(Fc, d)) || !(m->Wt_c2 = wt(d, Fc)) || !(m->b_c1 = vf(Fc)) || !(m->b_c2 = vf(d)))
+      return fail_cuda("cudaMalloc", err);
+    TXS_CK(launch_transpose<T>(static_cast<const T*>(cm[0]), static_cast<T*>(m->Wt_c1), d, Fc, s));
+    TXS_CK(launch_transpose<T>(static_cast<const T*>(cm[2]), static_cast<T*>(m->Wt_c2), Fc, d, s));
+    TXS_CK(launch_to_f32<T>(static_cast<const T*>(cm[1]), m->b_c1, Fc, s));
+    TXS_CK(launch_to_f32<T>(static_cast<const T*>(cm[3]), m->b_c2, d, s));
+  }
   // content hash of config and every input tensor
   unsigned long long* dh = dalloc<unsigned long long>(m->allocs, 8, &err);
   if (!dh) return fail_cuda("cudaMalloc", err);
@@ -292,12 +306,16 @@ txs_status model_prepare(txs_model* m, const void* const* w, cudaStream_t s) {
   const size_t nh[TXS_HEAD_WEIGHTS] = {size_t(d), 2 * size_t(d) * d, size_t(d), size_t(k) * d};
   for (int i = 0; i < TXS_HEAD_WEIGHTS; ++i)
     TXS_CK(launch_hash(head[i], static_cast<long long>(nh[i] * es), 100000 + i, dh, s));
+  if (Fc) {
+    const size_t nc[4] = {size_t(d) * Fc, size_t(Fc), size_t(Fc) * d, size_t(d)};
+    for (int i = 0; i < 4; ++i) TXS_CK(launch_hash(cm[i], static_cast<long long>(nc[i] * es), 200000 + i, dh, s));
+  }
   unsigned long long hv = 0;
   TXS_CK(cudaMemcpyAsync(&hv, dh, 8, cudaMemcpyDeviceToHost, s));
   TXS_CK(cudaStreamSynchronize(s));
   uint64_t h = hv;
   const int32_t cf[] = {c.d_model, c.n_heads, c.d_ff, c.n_layers, c.n_actions, c.n_ctx, c.l_local, c.attn_mode,
-                        c.dtype, kv_dim(c)};
+                        c.dtype, kv_dim(c), c.cand_mlp_hidden};
   for (int32_t v : cf) h = (h ^ static_cast<uint64_t>(static_cast<uint32_t>(v))) * 0x100000001B3ull;
   uint32_t eps_bits;
   std::memcpy(&eps_bits, &c.ln_eps, 4);
@@ -395,6 +413,21 @@ txs_status score_impl(txs_model* m, const KvView& c, int n_req, const int32_t* c
 
   TXS_CK(launch_pack<T>(n_req, cand_off, S, d, k, static_cast<const T*>(cand_tok), static_cast<const T*>(ctx_tok), X,
                         row_req, cand_off_dev, m->weff + size_t(d) * k, m->cdec, xlog, s));
+  // Phi_candidate: the candidate rows of X go through the MLP (the head's
+  // x-part above used the raw tokens)
+  if (cf.cand_mlp_hidden && n_cand > 0) {
+    const int Fc = cf.cand_mlp_hidden;
+    EpiArgs e = epi_base(EPI_BIAS_GELU, n_cand, Fc, d);
+    e.bias = m->b_c1;
+    e.out = Hf;
+    e.ldo = Fc;
+    TXS_CK(gemm(m, X, d, m->Wt_c1, e, tmp, s, KC_CAND_MLP));
+    e = epi_base(EPI_BIAS, n_cand, d, Fc);
+    e.bias = m->b_c2;
+    e.out = X;
+    e.ldo = d;
+    TXS_CK(gemm(m, Hf, Fc, m->Wt_c2, e, tmp, s, KC_CAND_MLP));
+  }
   const T* kv = static_cast<const T*>(c.kv);
   for (int l = 0; l < cf.n_layers; ++l) {
     const LayerW& W = m->layers[l];
@@ -523,7 +556,7 @@ TXS_API txs_status txs_model_create(const txs_config* cfg, const void* const* we
     set_error(why.c_str());
     return TXS_ERR_UNSUPPORTED;
   }
-  const int n_w = cfg->n_layers * TXS_WEIGHTS_PER_LAYER + TXS_HEAD_WEIGHTS;
+  const int n_w = cfg->n_layers * TXS_WEIGHTS_PER_LAYER + TXS_HEAD_WEIGHTS + (cfg->cand_mlp_hidden ? 4 : 0);
   for (int i = 0; i < n_w; ++i)
     if (!weights[i]) return TXS_ERR_INVALID_ARG;
   // the weight tensors may still be in flight on any stream of the caller
@@ -1066,7 +1099,7 @@ TXS_API txs_status txs_profile_collect(double* total_ms, int64_t* launches, int3
 TXS_API const char* txs_kernel_class_name(int32_t cls) {
   static const char* names[] = {"pack", "gemm_qkv", "attn_serving", "gemm_oproj_ln", "gemm_q", "attn_cross",
                                 "gemm_ffn1_gelu", "gemm_ffn2_ln", "gemm_kv_build", "pool", "global_kv", "rank",
-                                "misc", "row_ln"};
+                                "misc", "row_ln", "cand_mlp"};
   if (cls < 0 || cls >= KC_COUNT_) return "";
   return names[cls];
 }

@@ -20,7 +20,7 @@ constexpr long long kSpinCycles = 2000000000LL;
 enum KernelClass : int {
   KC_PACK = 0, KC_GEMM_QKV, KC_ATTN_SERVING, KC_GEMM_OPROJ, KC_GEMM_Q, KC_ATTN_CROSS,
   KC_GEMM_FFN1, KC_GEMM_FFN2, KC_GEMM_KV, KC_POOL, KC_GLOBAL_KV, KC_RANK, KC_MISC,
-  KC_ROW_LN, KC_COUNT_
+  KC_ROW_LN, KC_CAND_MLP, KC_COUNT_
 };
 static_assert(KC_COUNT_ <= TXS_N_KERNEL_CLASSES, "profiler classes");
 
