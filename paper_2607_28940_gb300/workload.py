@@ -264,3 +264,115 @@ def events(wl: Workload, L: int, T: int, m: Union[int, Sequence[int]], seed: int
 def with_sizes(wl: Workload, **kw) -> Workload:
     """A copy of ``wl`` with some fields replaced (e.g. a smaller L or M)."""
     return replace(wl, **kw)
+
+
+# ---------------------------------------------------------------- behavior encoder
+
+# Behavior-stream encoder Phi_behavior (Sec. 4.1.1; two causal layers with a
+# relative position bias in Sec. 5.1).  Per encoder layer ``l``, in draw order:
+ENC_LAYER_WEIGHTS: Tuple[Tuple[str, str], ...] = (
+    ("W_qkv", "d,3d"), ("b_qkv", "3d"), ("rel_bias", "H,R"), ("W_o", "d,d"), ("b_o", "d"),
+    ("ln1_g", "d"), ("ln1_b", "d"), ("W_1", "d,F"), ("b_1", "F"), ("W_2", "F,d"), ("b_2", "d"),
+    ("ln2_g", "d"), ("ln2_b", "d"),
+)
+# then, when type_dim > 0, the behavior-type embedding table
+ENC_TYPE_WEIGHTS: Tuple[Tuple[str, str], ...] = (("E_type", "T,dt"),)
+
+
+@dataclass(frozen=True)
+class EncWorkload:
+    """Sizes of an encoder workload.  Each user has L_r earlier behavior tokens
+    and dL_r new ones; a token is a subject row (width d - type_dim) and a
+    behavior-type id in [0, n_types)."""
+    name: str
+    dtype: str
+    n_req: int
+    n_layers: int
+    d_model: int
+    n_heads: int
+    d_ff: int
+    L: SizeSpec
+    dL: SizeSpec
+    type_dim: int
+    n_types: int
+    n_rel: int              # R relative-bias entries per head
+    window: int             # 0: full causal
+    seed: int
+    ln_eps: float = 1e-5
+    capacity_extra: int = 64
+
+    @property
+    def subj_dim(self) -> int:
+        return self.d_model - self.type_dim
+
+
+ENC_WORKLOADS: Dict[str, EncWorkload] = {
+    "enc_tiny_fp32": EncWorkload("enc_tiny_fp32", "fp32", 3, 2, 64, 2, 128, ("uniform", 20, 60),
+                                 ("uniform", 0, 6), 16, 7, 16, 0, 30261),
+    "enc_small_bf16": EncWorkload("enc_small_bf16", "bf16", 32, 2, 256, 8, 1024, 1024, 8, 32, 16, 256, 0, 30262),
+    "enc_mid_bf16": EncWorkload("enc_mid_bf16", "bf16", 64, 2, 512, 8, 2048, 4096, 8, 64, 32, 512, 0, 30263),
+}
+
+
+def enc_weights(ew: EncWorkload) -> Dict[str, np.ndarray]:
+    """Encoder weights: matrices ~ N(0, 1/d_in), biases ~ N(0, 0.02), LN gains
+    1 + N(0, 0.02), relative-bias tables ~ N(0, 1), type table ~ N(0, 1)."""
+    _, s_weights, _ = _streams(ew.seed)
+    rng = np.random.default_rng(s_weights)
+    env = {"d": ew.d_model, "3d": 3 * ew.d_model, "F": ew.d_ff, "H": ew.n_heads, "R": ew.n_rel,
+           "T": ew.n_types, "dt": ew.type_dim}
+    out: Dict[str, np.ndarray] = {}
+    for l in range(ew.n_layers):
+        for name, code in ENC_LAYER_WEIGHTS:
+            shp = tuple(env[c] for c in code.split(","))
+            x = rng.standard_normal(shp)
+            if name.startswith("W_"):
+                x = x / np.sqrt(shp[0])
+            elif name == "rel_bias":
+                pass
+            else:
+                x = x * 0.02
+                if name.endswith("_g"):
+                    x = 1.0 + x
+            out[f"{name}.{l}"] = _store(ew, x)
+    if ew.type_dim:
+        out["E_type"] = _store(ew, rng.standard_normal((ew.n_types, ew.type_dim)))
+    return out
+
+
+@dataclass
+class EncBatch:
+    """Behavior tokens of all users, packed user after user.
+
+    ``subj`` [sum L_r, d - d_t] subject embeddings, ``types`` [sum L_r] int32
+    type ids; ``subj_app``/``types_app`` the dL_r new tokens of each user.
+    """
+    subj: np.ndarray
+    types: np.ndarray
+    off: np.ndarray
+    subj_app: np.ndarray
+    types_app: np.ndarray
+    app_off: np.ndarray
+    L: np.ndarray
+    dL: np.ndarray
+
+
+def enc_batch(ew: EncWorkload) -> EncBatch:
+    """Per user r (own child stream): L_r subject rows ~ N(0, 1), L_r type ids
+    uniform in [0, n_types), then the dL_r new tokens drawn the same way."""
+    s_sizes, _, s_data = _streams(ew.seed)
+    rng = np.random.default_rng(s_sizes)
+    L = _draw_sizes(ew.L, ew.n_req, rng)
+    dL = _draw_sizes(ew.dL, ew.n_req, rng)
+    children = s_data.spawn(ew.n_req)
+    ds, T = ew.subj_dim, max(ew.n_types, 1)
+    subj, types, subj_a, types_a = [], [], [], []
+    for r in range(ew.n_req):
+        g = np.random.default_rng(children[r])
+        subj.append(g.standard_normal((int(L[r]), ds), dtype=np.float32))
+        types.append(g.integers(0, T, size=int(L[r])).astype(np.int32))
+        subj_a.append(g.standard_normal((int(dL[r]), ds), dtype=np.float32))
+        types_a.append(g.integers(0, T, size=int(dL[r])).astype(np.int32))
+    cat = lambda xs: _store(ew, np.concatenate(xs, axis=0))
+    return EncBatch(cat(subj), np.concatenate(types), _offsets(L), cat(subj_a), np.concatenate(types_a),
+                    _offsets(dL), L, dL)
