@@ -103,6 +103,7 @@ def _bias_only(beta, n, window=0):
     v = np.zeros((n, H * dh))
     for h in range(H):
         v[:, h * dh:(h + 1) * dh] = np.eye(n)
+    pos = np.arange(n)
     return E.causal_attention(q, q, v, H, beta, pos, pos, window)
 
 
