@@ -159,8 +159,11 @@ def empty_state(model: EncModel) -> EncState:
 def encode_append(model: EncModel, state: EncState, subj: np.ndarray, types: np.ndarray
                   ) -> Tuple[np.ndarray, EncState]:
     """Encode new tokens of one user after the ones in ``state`` (App. D
-    incremental encoding): returns (Phi_b rows of the new tokens, new state)."""
+    incremental encoding): returns (Phi_b rows of the new tokens, new state).
+    No new tokens leave the state as it is."""
     X = embed(model, subj, types)
+    if X.shape[0] == 0:
+        return np.zeros((0, model.d_model)), state
     K, V = [], []
     for l in range(model.n_layers):
         X, k, v = encoder_layer(model, X, l, state.K[l], state.V[l])

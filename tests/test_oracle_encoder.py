@@ -224,3 +224,16 @@ def test_batch_is_per_user():
     assert np.array_equal(phi[b.off[r]:b.off[r + 1]], own)
     new, _ = E.append_batch(model, states, b.subj_app, b.types_app, b.app_off)
     assert new.shape == (int(b.dL.sum()), ew.d_model)
+
+
+def test_empty_streams():
+    ew, model = _model()
+    subj, types = _tokens(ew, 0, 8)
+    y, st = E.encode(model, subj, types)
+    assert y.shape == (0, ew.d_model) and st.length == 0
+    s2, t2 = _tokens(ew, 6, 8)
+    a, sa = E.encode_append(model, st, s2, t2)
+    b, _ = E.encode(model, s2, t2)
+    assert np.array_equal(a, b)
+    y, sb = E.encode_append(model, sa, subj, types)
+    assert y.shape == (0, ew.d_model) and sb.length == 6
