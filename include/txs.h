@@ -299,6 +299,104 @@ txs_status txs_rank_candidates(int32_t n_req, const int32_t* cand_offsets, const
 txs_status txs_pool_anchor_static(const txs_model* model, int32_t n_req, const int32_t* beh_offsets,
                                   const void* beh_enc, float* out_g, void* stream);
 
+/* ------------------------------------------------------------------ behavior encoder
+ *
+ * The behavior-stream encoder Phi_behavior (Sec. 4.1.1; two layers in the
+ * paper's setup, Sec. 5.1) and its incremental update (App. D,
+ * incremental-encoding remark).  Its outputs are the encoded rows Phi_b that
+ * txs_build_kv_cache / txs_append_behavior take.
+ *
+ * Token of behavior i: x_i = [s_i, E_type[type_i]], s_i the subject
+ * embedding (width d_model - type_dim, given) and E_type the behavior-type
+ * table.  Each layer, post-LN with residuals:
+ *   [q|k|v] = X W_qkv + b_qkv
+ *   a_i (head h) = sum_j softmax_j(q_i.k_j / sqrt(d_h) + beta_h[min(i-j, R-1)]) v_j
+ *     over the visible j: j <= i, and i - j < window when window > 0
+ *   H = LN1(X + A W_o + b_o);  Y = LN2(H + GELU(H W_1 + b_1) W_2 + b_2)
+ * The mask is causal and the bias depends only on i - j, so appending tokens
+ * leaves the earlier outputs unchanged: an append runs the layers for the new
+ * tokens only, against each layer's cached keys/values of the earlier tokens
+ * (the encoder state), and gives the same rows, bit for bit, as encoding the
+ * whole stream at once.
+ */
+typedef struct {
+  int32_t d_model;   /* d; multiple of 64 for TXS_BF16, of 32 for TXS_FP32; <= 512  */
+  int32_t n_heads;   /* H; d_head = d_model / n_heads must be 32 or 64             */
+  int32_t d_ff;      /* F; multiple of 64, <= 16384                                */
+  int32_t n_layers;  /* encoder layers, 1..16                                      */
+  int32_t type_dim;  /* d_t, 0 <= d_t < d_model; subject rows are d_model - d_t wide */
+  int32_t n_types;   /* rows of E_type (>= 1 when type_dim > 0)                    */
+  int32_t n_rel;     /* R relative-bias entries per head, 1..65536                 */
+  int32_t window;    /* 0: every earlier token is visible; w > 0: the w most recent
+                        (the token itself included)                                */
+  int32_t dtype;     /* txs_dtype                                                  */
+  float ln_eps;      /* LayerNorm epsilon (> 0)                                    */
+} txs_enc_config;
+
+typedef struct txs_encoder txs_encoder;     /* opaque */
+typedef struct txs_enc_state txs_enc_state; /* opaque: per-user K/V of every layer */
+
+#define TXS_ENC_WEIGHTS_PER_LAYER 13
+
+/*
+ * txs_encoder_create — copy the encoder weights into the library's layout.
+ * `weights` (host array of device pointers, config dtype) holds, per layer:
+ *    0 W_qkv [d,3d]  1 b_qkv [3d]  2 rel_bias [H,R]  3 W_o [d,d]  4 b_o [d]
+ *    5 ln1_g [d]     6 ln1_b [d]   7 W_1 [d,F]       8 b_1 [F]    9 W_2 [F,d]
+ *   10 b_2 [d]      11 ln2_g [d]  12 ln2_b [d]
+ * then, when type_dim > 0, E_type [n_types, type_dim].  Synchronises the
+ * device first and returns after the copies; keeps a content hash.
+ * Errors: TXS_ERR_INVALID_ARG, TXS_ERR_UNSUPPORTED, TXS_ERR_CUDA.
+ */
+txs_status txs_encoder_create(const txs_enc_config* cfg, const void* const* weights, txs_encoder** out);
+void txs_encoder_destroy(txs_encoder* enc);
+uint64_t txs_encoder_hash(const txs_encoder* enc);
+
+/* Bytes of device scratch one encode call over n_rows tokens needs. */
+txs_status txs_encoder_workspace_size(const txs_encoder* enc, int64_t n_rows, size_t* bytes);
+
+/*
+ * txs_encode_build — encode each user's behavior stream from its first token
+ * and create the encoder state.  User r's tokens are rows offsets[r] ..
+ * offsets[r+1] of `subj` (device, config dtype, [n, d_model - type_dim]) and
+ * `types` (device int32 [n]; may be NULL iff type_dim == 0); `offsets` is a
+ * host int32 array [n_req + 1], non-decreasing from 0 (a user may have no
+ * tokens yet).  Writes Phi_b to phi_out (device, config dtype, [n, d_model])
+ * and keeps every layer's K/V rows, with capacity_extra >= 0 spare rows per
+ * user for appends.  `workspace`: device, >= txs_encoder_workspace_size(n)
+ * bytes, 256-byte aligned, caller-owned.  A type id outside [0, n_types)
+ * latches TXS_ERR_BOUNDS in the encoder's device status.
+ */
+txs_status txs_encode_build(txs_encoder* enc, int32_t n_req, const int32_t* offsets, const void* subj,
+                            const int32_t* types, int32_t capacity_extra, void* workspace, size_t workspace_bytes,
+                            void* phi_out, void* stream, txs_enc_state** out);
+
+/*
+ * txs_encode_append — incremental encoding (App. D remark): user r's new
+ * tokens, rows new_offsets[r] .. new_offsets[r+1] of subj/types (as above;
+ * zero new tokens allowed), are encoded after that user's current tokens;
+ * their Phi_b rows go to phi_out (device, [sum new, d_model]).  Earlier rows
+ * and their K/V are not touched.  n_req must equal the state's.
+ * Errors: TXS_ERR_CAPACITY if a user would exceed its capacity (nothing is
+ * changed), TXS_ERR_STALE_CACHE if the state came from another encoder,
+ * TXS_ERR_INVALID_ARG.
+ */
+txs_status txs_encode_append(txs_encoder* enc, txs_enc_state* state, int32_t n_req, const int32_t* new_offsets,
+                             const void* subj, const int32_t* types, void* workspace, size_t workspace_bytes,
+                             void* phi_out, void* stream);
+
+/* Per-user token counts (host int32 [n_req]) and user count of a state. */
+txs_status txs_enc_state_lengths(const txs_enc_state* state, int32_t* out_len);
+int32_t txs_enc_state_n_req(const txs_enc_state* state);
+/* Copy rows row0 .. row0+n_rows-1 of user `req`'s cached keys (which = 0) or
+ * values (which = 1) of encoder layer `layer` into dst (device, config dtype,
+ * [n_rows, d_model]), asynchronously on `stream`. */
+txs_status txs_enc_state_read_rows(const txs_enc_state* state, int32_t layer, int32_t which, int32_t req,
+                                   int32_t row0, int32_t n_rows, void* dst, void* stream);
+void txs_enc_state_destroy(txs_enc_state* state);
+/* Synchronise the device, read and clear the encoder's latched device status. */
+txs_status txs_encoder_device_status(txs_encoder* enc);
+
 /* Synchronise the device, read and clear the model's latched device status. */
 txs_status txs_device_status(txs_model* model);
 
@@ -308,7 +406,7 @@ txs_status txs_device_status(txs_model* model);
  * milliseconds and launch counts (host arrays of length n >=
  * TXS_N_KERNEL_CLASSES) and clears the record.  Not thread-safe; not for use
  * during CUDA-graph capture. */
-#define TXS_N_KERNEL_CLASSES 16
+#define TXS_N_KERNEL_CLASSES 24
 txs_status txs_profile_enable(int32_t enable);
 txs_status txs_profile_collect(double* total_ms, int64_t* launches, int32_t n);
 const char* txs_kernel_class_name(int32_t cls);

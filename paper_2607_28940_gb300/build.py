@@ -14,7 +14,7 @@ HERE = os.path.dirname(os.path.abspath(__file__))
 CSRC = os.path.join(HERE, "csrc")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libtxs.so")
-SOURCES = ["txs_api.cu", "k_gemm_tc.cu", "k_gemm_ln.cu", "k_simt.cu", "k_attn.cu", "k_attn_tc.cu", "k_cache.cu", "k_score.cu", "k_noalloc.cu"]
+SOURCES = ["txs_api.cu", "k_gemm_tc.cu", "k_gemm_ln.cu", "k_simt.cu", "k_attn.cu", "k_attn_tc.cu", "k_cache.cu", "k_score.cu", "k_noalloc.cu", "k_encoder.cu", "txs_encoder.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC,-fvisibility=hidden", "--expt-relaxed-constexpr"]
 

@@ -1099,7 +1099,7 @@ TXS_API txs_status txs_profile_collect(double* total_ms, int64_t* launches, int3
 TXS_API const char* txs_kernel_class_name(int32_t cls) {
   static const char* names[] = {"pack", "gemm_qkv", "attn_serving", "gemm_oproj_ln", "gemm_q", "attn_cross",
                                 "gemm_ffn1_gelu", "gemm_ffn2_ln", "gemm_kv_build", "pool", "global_kv", "rank",
-                                "misc", "row_ln", "cand_mlp"};
+                                "misc", "row_ln", "cand_mlp", "enc_embed", "enc_gemm", "enc_attn"};
   if (cls < 0 || cls >= KC_COUNT_) return "";
   return names[cls];
 }

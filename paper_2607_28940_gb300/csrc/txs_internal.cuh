@@ -20,7 +20,7 @@ constexpr long long kSpinCycles = 2000000000LL;
 enum KernelClass : int {
   KC_PACK = 0, KC_GEMM_QKV, KC_ATTN_SERVING, KC_GEMM_OPROJ, KC_GEMM_Q, KC_ATTN_CROSS,
   KC_GEMM_FFN1, KC_GEMM_FFN2, KC_GEMM_KV, KC_POOL, KC_GLOBAL_KV, KC_RANK, KC_MISC,
-  KC_ROW_LN, KC_CAND_MLP, KC_COUNT_
+  KC_ROW_LN, KC_CAND_MLP, KC_ENC_EMBED, KC_ENC_GEMM, KC_ENC_ATTN, KC_COUNT_
 };
 static_assert(KC_COUNT_ <= TXS_N_KERNEL_CLASSES, "profiler classes");
 
@@ -219,5 +219,20 @@ cudaError_t launch_pack(int n_req, const int* cand_off_host, int S, int d, int n
                         cudaStream_t s);
 cudaError_t launch_rank(int n_req, const int* cand_off_host, const float* probs, int na, int action, int top_k,
                         int* out, cudaStream_t s);
+
+// Behavior-stream encoder (k_encoder.cu).  Query rows per attention CTA for
+// calls whose users have at most `max_new_rows` new rows each.
+int enc_query_tile(int max_new_rows);
+template <typename T>
+cudaError_t launch_enc_embed(const T* subj, const int* types, const T* E_type, T* X, long long n, int d, int dt,
+                             int n_types, int* status, cudaStream_t s);
+template <typename T>
+cudaError_t launch_enc_rel_prep(const T* beta, float* out, int n, cudaStream_t s);
+template <typename T>
+cudaError_t launch_enc_attn(const T* q, const T* K, const T* V, T* out, const int* in_off, const int* dst0,
+                            const int* slot_off, const int* tile_off, int n_req, int n_tiles, int query_tile,
+                            const float* beta_log2, int n_rel, int window, int H, int d, int* status,
+                            cudaStream_t s);
+void set_last_error(const char* msg);
 
 }  // namespace txs

@@ -31,7 +31,7 @@ TXS_ERR_UNSUPPORTED = 8
 
 TXS_FP32, TXS_BF16 = 0, 1
 LOCAL_GLOBAL, FULL = 0, 1
-N_KERNEL_CLASSES = 16
+N_KERNEL_CLASSES = 24
 
 
 class TxsError(RuntimeError):
@@ -48,6 +48,13 @@ class txs_config(ctypes.Structure):
                 ("n_layers", ctypes.c_int32), ("n_actions", ctypes.c_int32), ("n_ctx", ctypes.c_int32),
                 ("l_local", ctypes.c_int32), ("attn_mode", ctypes.c_int32), ("dtype", ctypes.c_int32),
                 ("ln_eps", ctypes.c_float), ("n_kv_heads", ctypes.c_int32), ("cand_mlp_hidden", ctypes.c_int32)]
+
+
+class txs_enc_config(ctypes.Structure):
+    _fields_ = [("d_model", ctypes.c_int32), ("n_heads", ctypes.c_int32), ("d_ff", ctypes.c_int32),
+                ("n_layers", ctypes.c_int32), ("type_dim", ctypes.c_int32), ("n_types", ctypes.c_int32),
+                ("n_rel", ctypes.c_int32), ("window", ctypes.c_int32), ("dtype", ctypes.c_int32),
+                ("ln_eps", ctypes.c_float)]
 
 
 _lib: Optional[ctypes.CDLL] = None
@@ -77,6 +84,17 @@ _SIGS = {
     "txs_events_workspace_size": (_I32, [_P, _I32, ctypes.c_int64, _I32, ctypes.POINTER(ctypes.c_size_t)]),
     "txs_score_events": (_I32, [_P, _P, _I32, _P, _I32, _I32P, _I32P, _P, _P, _P, ctypes.c_size_t, _P, _P, _P]),
     "txs_device_status": (_I32, [_P]),
+    "txs_encoder_create": (_I32, [ctypes.POINTER(txs_enc_config), ctypes.POINTER(_P), ctypes.POINTER(_P)]),
+    "txs_encoder_destroy": (None, [_P]),
+    "txs_encoder_hash": (ctypes.c_uint64, [_P]),
+    "txs_encoder_workspace_size": (_I32, [_P, ctypes.c_int64, ctypes.POINTER(ctypes.c_size_t)]),
+    "txs_encode_build": (_I32, [_P, _I32, _I32P, _P, _P, _I32, _P, ctypes.c_size_t, _P, _P, ctypes.POINTER(_P)]),
+    "txs_encode_append": (_I32, [_P, _P, _I32, _I32P, _P, _P, _P, ctypes.c_size_t, _P, _P]),
+    "txs_enc_state_lengths": (_I32, [_P, _I32P]),
+    "txs_enc_state_n_req": (_I32, [_P]),
+    "txs_enc_state_read_rows": (_I32, [_P, _I32, _I32, _I32, _I32, _I32, _P, _P]),
+    "txs_enc_state_destroy": (None, [_P]),
+    "txs_encoder_device_status": (_I32, [_P]),
     "txs_pool_anchor_static": (_I32, [_P, _I32, _I32P, _P, _P, _P]),
     "txs_profile_enable": (_I32, [_I32]),
     "txs_profile_collect": (_I32, [ctypes.POINTER(ctypes.c_double), ctypes.POINTER(ctypes.c_int64), _I32]),
@@ -354,6 +372,127 @@ def pool_anchor_static(model: Model, beh_offsets, beh_enc: torch.Tensor, out: Op
     _check(lib().txs_pool_anchor_static(model.handle, n_req, p, _ptr(beh_enc), _ptr(out), _stream(stream)),
            "txs_pool_anchor_static")
     return out
+
+
+# ---------------------------------------------------------------- behavior encoder
+
+def make_enc_config(ew: W.EncWorkload) -> txs_enc_config:
+    return txs_enc_config(ew.d_model, ew.n_heads, ew.d_ff, ew.n_layers, ew.type_dim, ew.n_types, ew.n_rel,
+                          ew.window, TXS_BF16 if ew.dtype == "bf16" else TXS_FP32, ew.ln_eps)
+
+
+def enc_weight_order(ew: W.EncWorkload) -> Sequence[str]:
+    """Names of the encoder weight tensors in the order of txs_encoder_create."""
+    names = [f"{n}.{l}" for l in range(ew.n_layers) for n, _ in W.ENC_LAYER_WEIGHTS]
+    return names + ([n for n, _ in W.ENC_TYPE_WEIGHTS] if ew.type_dim else [])
+
+
+class Encoder:
+    """The behavior-stream encoder on the GPU (txs_encoder)."""
+
+    def __init__(self, ew: W.EncWorkload, weights: Dict[str, np.ndarray], device: str = "cuda"):
+        self.ew = ew
+        self.dtype = torch_dtype(ew.dtype)
+        self.cfg = make_enc_config(ew)
+        dev = [torch.as_tensor(np.asarray(weights[n]), dtype=torch.float32).to(device).to(self.dtype).contiguous()
+               for n in enc_weight_order(ew)]
+        ptrs = (_P * len(dev))(*[t.data_ptr() for t in dev])
+        h = _P()
+        _check(lib().txs_encoder_create(ctypes.byref(self.cfg), ptrs, ctypes.byref(h)), "txs_encoder_create")
+        self.handle = h
+        del dev
+
+    @property
+    def hash(self) -> int:
+        return int(lib().txs_encoder_hash(self.handle))
+
+    def workspace_bytes(self, n_rows: int) -> int:
+        n = ctypes.c_size_t()
+        _check(lib().txs_encoder_workspace_size(self.handle, int(n_rows), ctypes.byref(n)), "workspace_size")
+        return int(n.value)
+
+    def device_status(self) -> int:
+        return int(lib().txs_encoder_device_status(self.handle))
+
+    def close(self):
+        if getattr(self, "handle", None):
+            lib().txs_encoder_destroy(self.handle)
+            self.handle = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+
+def _enc_io(enc: Encoder, off: np.ndarray, workspace, phi_out):
+    n = int(off[-1])
+    if workspace is None:
+        workspace = torch.empty(max(enc.workspace_bytes(n), 256), dtype=torch.uint8, device="cuda")
+    if phi_out is None:
+        phi_out = torch.empty((n, enc.ew.d_model), dtype=enc.dtype, device="cuda")
+    return workspace, phi_out
+
+
+class EncState:
+    """Per-user encoder state: every layer's K/V rows (txs_enc_state)."""
+
+    def __init__(self, enc: Encoder, offsets, subj: torch.Tensor, types: Optional[torch.Tensor],
+                 capacity_extra: int = 0, workspace: Optional[torch.Tensor] = None,
+                 phi_out: Optional[torch.Tensor] = None, stream=None):
+        """Encode each user's stream from its first token (txs_encode_build);
+        the encoded rows are in ``self.phi``."""
+        off, p = _offsets(offsets)
+        self.enc = enc
+        self.n_req = len(off) - 1
+        workspace, phi_out = _enc_io(enc, off, workspace, phi_out)
+        h = _P()
+        _check(lib().txs_encode_build(enc.handle, self.n_req, p, _ptr(subj) if subj.numel() else None,
+                                      _ptr(types) if types is not None and types.numel() else None,
+                                      int(capacity_extra), _ptr(workspace), workspace.numel(),
+                                      _ptr(phi_out) if phi_out.numel() else None, _stream(stream), ctypes.byref(h)),
+               "txs_encode_build")
+        self.handle = h
+        self.phi = phi_out
+
+    def append(self, new_offsets, subj: torch.Tensor, types: Optional[torch.Tensor],
+               workspace: Optional[torch.Tensor] = None, phi_out: Optional[torch.Tensor] = None,
+               stream=None, enc: Optional[Encoder] = None) -> torch.Tensor:
+        """Encode new tokens after each user's current ones (txs_encode_append);
+        returns their encoded rows."""
+        off, p = _offsets(new_offsets)
+        e = enc or self.enc
+        workspace, phi_out = _enc_io(e, off, workspace, phi_out)
+        _check(lib().txs_encode_append(e.handle, self.handle, len(off) - 1, p, _ptr(subj) if subj.numel() else None,
+                                       _ptr(types) if types is not None and types.numel() else None,
+                                       _ptr(workspace), workspace.numel(),
+                                       _ptr(phi_out) if phi_out.numel() else None, _stream(stream)),
+               "txs_encode_append")
+        return phi_out
+
+    def lengths(self) -> np.ndarray:
+        out = np.zeros(self.n_req, dtype=np.int32)
+        _check(lib().txs_enc_state_lengths(self.handle, out.ctypes.data_as(_I32P)), "txs_enc_state_lengths")
+        return out
+
+    def read_rows(self, layer: int, which: int, req: int, row0: int, n_rows: int, stream=None) -> torch.Tensor:
+        out = torch.empty((n_rows, self.enc.ew.d_model), dtype=self.enc.dtype, device="cuda")
+        _check(lib().txs_enc_state_read_rows(self.handle, layer, which, req, row0, n_rows,
+                                             _ptr(out) if n_rows else None, _stream(stream)),
+               "txs_enc_state_read_rows")
+        return out
+
+    def close(self):
+        if getattr(self, "handle", None):
+            lib().txs_enc_state_destroy(self.handle)
+            self.handle = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
 
 
 def profile_enable(on: bool = True):

@@ -96,3 +96,43 @@ def test_rank_rejects_bad_arguments_on_host(lib):
 
 def test_profiler_collect_without_launches(lib):
     assert txs.profile_collect() == {}
+
+
+def _enc_cfg(**kw):
+    base = dict(d_model=256, n_heads=8, d_ff=1024, n_layers=2, type_dim=32, n_types=16, n_rel=128, window=0,
+                dtype=txs.TXS_BF16, ln_eps=1e-5)
+    base.update(kw)
+    return txs.txs_enc_config(**base)
+
+
+@pytest.mark.parametrize("bad", [
+    dict(d_model=96), dict(n_heads=3), dict(n_heads=2), dict(d_ff=100), dict(n_layers=0), dict(n_layers=17),
+    dict(type_dim=256), dict(type_dim=-1), dict(n_types=0), dict(n_rel=0), dict(n_rel=70000), dict(window=-1),
+    dict(ln_eps=0.0),
+])
+def test_encoder_create_rejects_bad_config_on_host(lib, bad):
+    cfg = _enc_cfg(**bad)
+    n = max(cfg.n_layers, 1) * 13 + 1
+    ptrs = (ctypes.c_void_p * n)(*([16] * n))
+    h = ctypes.c_void_p()
+    assert lib.txs_encoder_create(ctypes.byref(cfg), ptrs, ctypes.byref(h)) == txs.TXS_ERR_UNSUPPORTED
+    assert not h.value
+    cfg = _enc_cfg(dtype=7)
+    assert lib.txs_encoder_create(ctypes.byref(cfg), ptrs, ctypes.byref(h)) == txs.TXS_ERR_INVALID_ARG
+
+
+def test_encoder_null_arguments_rejected(lib):
+    h = ctypes.c_void_p()
+    n = ctypes.c_size_t()
+    assert lib.txs_encoder_create(None, None, ctypes.byref(h)) == txs.TXS_ERR_INVALID_ARG
+    assert lib.txs_encoder_workspace_size(None, 1, ctypes.byref(n)) == txs.TXS_ERR_INVALID_ARG
+    assert lib.txs_encode_build(None, 1, None, None, None, 0, None, 0, None, None, ctypes.byref(h)) == \
+        txs.TXS_ERR_INVALID_ARG
+    assert lib.txs_encode_append(None, None, 1, None, None, None, None, 0, None, None) == txs.TXS_ERR_INVALID_ARG
+    assert lib.txs_enc_state_lengths(None, None) == txs.TXS_ERR_INVALID_ARG
+    assert lib.txs_enc_state_read_rows(None, 0, 0, 0, 0, 1, None, None) == txs.TXS_ERR_INVALID_ARG
+    assert lib.txs_encoder_device_status(None) == txs.TXS_ERR_INVALID_ARG
+    assert lib.txs_enc_state_n_req(None) == 0
+    assert lib.txs_encoder_hash(None) == 0
+    lib.txs_encoder_destroy(None)
+    lib.txs_enc_state_destroy(None)
