@@ -324,6 +324,7 @@ def run_txs(args, rank, world):
         if rank == 0:
             out["latency_vs_L"] = latency_sweep(txs, torch)
             out["events"] = events_bench(txs, torch)
+            out["encoder"] = encoder_bench(txs, torch, peaks, peak_src)
             out["cpu_baseline"] = cpu_baseline(args.workload, budget_s=12.0)
     return out
 
@@ -476,6 +477,138 @@ def events_bench(txs, torch):
         cache.close()
         model.close()
     return res
+
+
+ENC_WORKLOAD = "enc_mid_bf16"   # 64 users x 4096 tokens, d = 512, 2 layers, 8 new tokens per user
+ENC_APPENDS, ENC_PROFILED = 24, 8
+# FP32 FMA lanes per SM and the maximum SM clock (nominal): the ALU peak of a
+# SIMT kernel is 152 SMs x 128 lanes x 2 flop x 2070 MHz.
+ALU_FP32_TFLOPS = 152 * 128 * 2 * 2.070e9 / 1e12
+
+
+def encoder_bench(txs, torch, peaks, peak_src):
+    """Behavior encoder (Sec. 4.1.1; App. D incremental encoding) on the
+    64-user x 4096-token workload: the incremental append of 8 new tokens per
+    user (the nearline streaming update) and the full-stream build, with the
+    roofline of each one's attention kernel and the oracle on a sample."""
+    ew = W.ENC_WORKLOADS[ENC_WORKLOAD]
+    w = W.enc_weights(ew)
+    b = W.enc_batch(ew)
+    dt = txs.torch_dtype(ew.dtype)
+    d, es = ew.d_model, 2 if ew.dtype == "bf16" else 4
+    enc = txs.Encoder(ew, w)
+    subj = txs.to_device(b.subj, dt)
+    types = torch.from_numpy(b.types).to("cuda")
+    sa = txs.to_device(b.subj_app, dt)
+    ta = torch.from_numpy(b.types_app).to("cuda")
+    n, na = int(b.off[-1]), int(b.app_off[-1])
+    ws = torch.empty(enc.workspace_bytes(n), dtype=torch.uint8, device="cuda")
+    phi = torch.empty((n, d), dtype=dt, device="cuda")
+    new = torch.empty((na, d), dtype=dt, device="cuda")
+    n_app = 3 + ENC_APPENDS + ENC_PROFILED
+    cap = int(b.dL.max()) * n_app
+    res = {"workload": f"{ENC_WORKLOAD}: {ew.n_req} users x {int(b.L[0])} tokens, d={d}, H={ew.n_heads}, "
+                       f"F={ew.d_ff}, {ew.n_layers} layers, R={ew.n_rel}, full causal; append = "
+                       f"{int(b.dL[0])} new tokens per user", "unit": "tokens/s"}
+
+    def ev_time(fn):
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        e0.record()
+        fn()
+        e1.record()
+        e1.synchronize()
+        return e0.elapsed_time(e1)
+
+    # build (prefill of every stream); the state's allocation is inside the call
+    builds = []
+    for _ in range(2):
+        st = None
+
+        def mk():
+            nonlocal st
+            st = txs.EncState(enc, b.off, subj, types, capacity_extra=cap, workspace=ws, phi_out=phi)
+        builds.append(ev_time(mk))
+        st.close()
+    txs.profile_enable(True)
+    st = txs.EncState(enc, b.off, subj, types, capacity_extra=cap, workspace=ws, phi_out=phi)
+    torch.cuda.synchronize()
+    prof_b = txs.profile_collect()
+    txs.profile_enable(False)
+    # incremental appends against the growing state (inputs far larger than L2)
+    call = lambda: st.append(b.app_off, sa, ta, workspace=ws, phi_out=new)
+    for _ in range(3):
+        call()
+    hist0 = int(st.lengths().mean())
+    times = [ev_time(call) for _ in range(ENC_APPENDS)]
+    txs.profile_enable(True)
+    lens_before = st.lengths().astype(np.int64)
+    for _ in range(ENC_PROFILED):
+        call()
+    torch.cuda.synchronize()
+    prof_a = txs.profile_collect()
+    txs.profile_enable(False)
+    if enc.device_status() != txs.TXS_OK:
+        raise RuntimeError("device status after the encoder measurement")
+    ms_app = statistics.median(times)
+    # attention roofline of the append: each launch (one layer) reads every
+    # visible key and value row once and the new rows' q and writes their output
+    dL = b.dL.astype(np.int64)
+    byts = 0.0
+    for k in range(ENC_PROFILED):
+        L_end = lens_before + (k + 1) * dL
+        byts += ew.n_layers * (2 * float(L_end.sum()) * d * es + 2 * na * d * es)
+    attn_ms, attn_n = prof_a.get("enc_attn", (0.0, 0))
+    ach = byts / (attn_ms / 1e3) / 1e9 if attn_n else None
+    res["append"] = {
+        "ms_per_call": ms_app, "tokens_per_s": na / (ms_app / 1e3), "users_per_s": ew.n_req / (ms_app / 1e3),
+        "history_tokens_per_user": f"{hist0} .. {int(st.lengths().mean())}",
+        "kernels_ms_per_call": {k: v[0] / ENC_PROFILED for k, v in prof_a.items()},
+        "launches_per_call": sum(v[1] for v in prof_a.values()) // ENC_PROFILED,
+        "roofline_attn": {"bound": "hbm", "achieved": ach, "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                          "frac": ach / peaks["hbm_gbs"] if ach else None, "traffic": None,
+                          "kernel": "enc_attn", "peak_source": f"{peak_src} (copy)",
+                          "algorithmic_per_launch_bytes": byts / attn_n if attn_n else None}}
+    # build roofline of the attention: 4 flop per visible (query, key) pair per dim
+    L = b.L.astype(np.int64)
+    pairs = float((L * (L + 1) // 2).sum()) if ew.window == 0 else None
+    fl = ew.n_layers * pairs * 4 * d
+    bms, bn_ = prof_b.get("enc_attn", (0.0, 0))
+    ach_b = fl / (bms / 1e3) / 1e12 if bms else None
+    res["build"] = {
+        "ms_per_call": statistics.median(builds), "tokens_per_s": n / (statistics.median(builds) / 1e3),
+        "note": "includes the state's device allocation (cudaMalloc) inside the call",
+        "kernels_ms": {k: v[0] for k, v in prof_b.items()},
+        "roofline_attn": {"bound": "alu", "achieved": ach_b, "peak": ALU_FP32_TFLOPS, "unit": "TFLOP/s",
+                          "frac": ach_b / ALU_FP32_TFLOPS if ach_b else None, "traffic": None,
+                          "kernel": "enc_attn",
+                          "peak_source": "derived: 152 SMs x 128 FP32 lanes x 2 flop x 2070 MHz",
+                          "algorithmic_flops_per_launch": fl / ew.n_layers}}
+    st.close()
+    enc.close()
+    res["cpu_baseline"] = encoder_cpu_baseline(ew, w, b)
+    return res
+
+
+def encoder_cpu_baseline(ew, w, b, users=(0, 1), reps=20):
+    """The encoder oracle as it stands on the host cores: the same append (8
+    new tokens of a user with 4096 earlier ones) for a sample of users, the
+    users' states built outside the timed region."""
+    from oracle import encoder_oracle as E
+    om = E.EncModel.from_arrays(w, ew)
+    t_tot, toks = 0.0, 0
+    for r in users:
+        sl = slice(b.off[r], b.off[r + 1])
+        _, st = E.encode(om, b.subj[sl], b.types[sl])
+        sa = slice(b.app_off[r], b.app_off[r + 1])
+        for _ in range(reps):
+            t0 = time.perf_counter()
+            E.encode_append(om, st, b.subj_app[sa], b.types_app[sa])
+            t_tot += time.perf_counter() - t0
+            toks += sa.stop - sa.start
+    return {"value": float(toks / t_tot), "unit": "tokens/s", "cores": os.cpu_count(), "kind": "oracle",
+            "sample": f"append of {int(b.dL[0])} tokens for users {list(users)} of {ENC_WORKLOAD}, {reps} times "
+                      f"each (float64 NumPy, {t_tot:.2f} s; the states are built outside the timing)"}
 
 
 # ---------------------------------------------------------------- the oracle (CPU) arm
