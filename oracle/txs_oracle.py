@@ -34,6 +34,8 @@ What it computes (row-vector convention ``y = x W + b``):
 * Head (Sec. 4.1.3, the action-decoding equation): for candidate rows,
   ``k_dec = [z, x] W_dec + b_dec`` (linear f_dec, Sec. 4.4), logits
   ``= Q_dec k_dec`` (no scale), probabilities ``= softmax(logits)``.
+  Optionally the Deep & Wide f_dec (App. B): with x = [x_wide, x_deep],
+  ``k_dec = [x_wide W_w + b_w, GELU([z, x_deep] W_d1 + b_d1) W_d2 + b_d2]``.
 * Ranking: per request, candidates by descending probability of one action,
   ties to the lower candidate index.
 * Streaming multi-event scoring (Sec. 4.2 prefix reuse, Sec. 5.1 per-event
@@ -119,6 +121,9 @@ class Model:
     ln_eps: float
     n_kv_heads: int = 0   # K/V heads of the cache; 0 or n_heads: one per query head
     cand_mlp: int = 0     # hidden width of the candidate-to-query MLP; 0: none
+    dw_hidden: int = 0    # Deep & Wide head: hidden width of the deep FFN; 0: linear head
+    dw_in: int = 0        # width of x_wide (the first dw_in features of x)
+    dw_out: int = 0       # width of the wide part of k_dec
 
     @property
     def kv_heads(self) -> int:
@@ -128,7 +133,8 @@ class Model:
     def from_arrays(weights: Dict[str, np.ndarray], wl) -> "Model":
         return Model({k: np.asarray(v, dtype=np.float64) for k, v in weights.items()},
                      wl.n_layers, wl.d_model, wl.n_heads, wl.n_ctx, wl.n_actions,
-                     wl.l_local, wl.ln_eps, getattr(wl, "n_kv_heads", 0), getattr(wl, "cand_mlp", 0))
+                     wl.l_local, wl.ln_eps, getattr(wl, "n_kv_heads", 0), getattr(wl, "cand_mlp", 0),
+                     getattr(wl, "dw_hidden", 0), getattr(wl, "dw_in", 0), getattr(wl, "dw_out", 0))
 
 
 @dataclass
@@ -265,10 +271,24 @@ def decoder_layer(model: Model, X: np.ndarray, Kc: np.ndarray, Vc: np.ndarray, l
     return layer_norm(X2 + f, w[f"ln3_g.{l}"], w[f"ln3_b.{l}"], eps)
 
 
+def f_dec_deep_wide(model: Model, z: np.ndarray, x: np.ndarray) -> np.ndarray:
+    """Deep & Wide f_dec (App. B): the concatenation of a linear map of the
+    wide features x[:, :dw_in] and an FFN of the cross-attention output z with
+    the deep features x[:, dw_in:]."""
+    w, a = model.w, model.dw_in
+    wide = x[:, :a] @ w["W_w"] + w["b_w"]
+    deep = gelu(np.concatenate([z, x[:, a:]], axis=1) @ w["W_d1"] + w["b_d1"]) @ w["W_d2"] + w["b_d2"]
+    return np.concatenate([wide, deep], axis=1)
+
+
 def head(model: Model, z: np.ndarray, x: np.ndarray):
-    """Query-key softmax action decoder (Sec. 4.1.3): logits = Q_dec k_dec, k_dec linear in [z, x]."""
+    """Query-key softmax action decoder (Sec. 4.1.3): logits = Q_dec k_dec, with
+    k_dec = f_dec(z, x) linear in [z, x], or the Deep & Wide f_dec."""
     w = model.w
-    kdec = np.concatenate([z, x], axis=1) @ w["W_dec"] + w["b_dec"]
+    if model.dw_hidden:
+        kdec = f_dec_deep_wide(model, z, x)
+    else:
+        kdec = np.concatenate([z, x], axis=1) @ w["W_dec"] + w["b_dec"]
     logits = kdec @ w["Q_dec"].T
     return logits, softmax(logits, axis=-1)
 

@@ -54,6 +54,12 @@ CAND_WEIGHTS: Tuple[Tuple[str, str], ...] = (
     ("W_c1", "d,Fc"), ("b_c1", "Fc"), ("W_c2", "Fc,d"), ("b_c2", "d"),
 )
 
+# Deep & Wide head (App. B; drawn last, only when dw_hidden > 0): the wide
+# linear map of x[:, :dw_in] and the deep FFN of [z, x[:, dw_in:]]
+DW_WEIGHTS: Tuple[Tuple[str, str], ...] = (
+    ("W_w", "dwi,dwo"), ("b_w", "dwo"), ("W_d1", "dd,Fh"), ("b_d1", "Fh"), ("W_d2", "Fh,ddo"), ("b_d2", "ddo"),
+)
+
 SizeSpec = Union[int, Tuple[str, int, int], Sequence[int]]
 
 
@@ -77,6 +83,9 @@ class Workload:
     capacity_extra: int = 64
     n_kv_heads: int = 0     # K/V heads of the cache (0: one per query head)
     cand_mlp: int = 0       # hidden width of the candidate-to-query MLP (0: none)
+    dw_hidden: int = 0      # Deep & Wide head: deep FFN hidden width (0: linear head)
+    dw_in: int = 0          # Deep & Wide head: width of the wide features x[:, :dw_in]
+    dw_out: int = 0         # Deep & Wide head: width of the wide part of k_dec
 
     @property
     def d_head(self) -> int:
@@ -145,7 +154,9 @@ def sizes(wl: Workload) -> Tuple[np.ndarray, np.ndarray, np.ndarray]:
 def _shape(code: str, wl: Workload) -> Tuple[int, ...]:
     dkv = (wl.n_kv_heads or wl.n_heads) * (wl.d_model // wl.n_heads)
     env = {"d": wl.d_model, "3d": 3 * wl.d_model, "2d": 2 * wl.d_model,
-           "F": wl.d_ff, "k": wl.n_actions, "dkv": dkv, "Fc": wl.cand_mlp}
+           "F": wl.d_ff, "k": wl.n_actions, "dkv": dkv, "Fc": wl.cand_mlp,
+           "dwi": wl.dw_in, "dwo": wl.dw_out, "dd": 2 * wl.d_model - wl.dw_in, "Fh": wl.dw_hidden,
+           "ddo": wl.d_model - wl.dw_out}
     return tuple(env[c] for c in code.split(","))
 
 
@@ -165,6 +176,9 @@ def weights(wl: Workload) -> Dict[str, np.ndarray]:
         out[name] = _store(wl, rng.standard_normal(_shape(code, wl)) * 0.02)
     if wl.cand_mlp:
         for name, code in CAND_WEIGHTS:
+            out[name] = _store(wl, rng.standard_normal(_shape(code, wl)) * 0.02)
+    if wl.dw_hidden:
+        for name, code in DW_WEIGHTS:
             out[name] = _store(wl, rng.standard_normal(_shape(code, wl)) * 0.02)
     return out
 
