@@ -73,6 +73,13 @@ typedef struct {
   int32_t cand_mlp_hidden; /* hidden width Fc of the candidate-to-query MLP
                         Phi_candidate (Sec. 4.1.2; multiple of 64, <= 16384), or 0
                         when the candidate tokens already are its outputs       */
+  int32_t head_dw_hidden; /* Deep & Wide f_dec (App. B): hidden width Fh of its deep
+                        FFN (multiple of 64, <= 16384), or 0 for the linear f_dec */
+  int32_t head_dw_in;  /* Deep & Wide: the first dw_in features of a candidate token
+                        are its wide (linear) part, the rest its deep part;
+                        0 <= dw_in <= d_model, multiple of 64                    */
+  int32_t head_dw_out; /* Deep & Wide: width of the wide part of k_dec,
+                        0 <= dw_out < d_model (the deep part is the rest)       */
 } txs_config;
 
 typedef struct txs_model txs_model;       /* opaque */
@@ -102,6 +109,12 @@ typedef struct txs_kv_cache txs_kv_cache; /* opaque */
  *     W_c1 [d,Fc], b_c1 [Fc], W_c2 [Fc,d], b_c2 [d]
  *   (the decoder sees GELU(x W_c1 + b_c1) W_c2 + b_c2 for each candidate
  *   token x; the head's f_dec(z, x) keeps the raw x)
+ *   then, when head_dw_hidden = Fh > 0, the Deep & Wide f_dec (6 more;
+ *   a = dw_in, o = dw_out):
+ *     W_w [a,o], b_w [o], W_d1 [2d-a,Fh], b_d1 [Fh], W_d2 [Fh,d-o], b_d2 [d-o]
+ *   with k_dec = [x[:a] W_w + b_w, GELU([z, x[a:]] W_d1 + b_d1) W_d2 + b_d2];
+ *   the head's W_dec and b_dec are then unused and may be NULL, as may
+ *   W_w when a or o is 0 and b_w when o is 0.
  * The call synchronises the device first (the weights may still be in flight
  * on any stream) and returns after the copies are done; the inputs may be
  * freed afterwards.  The model keeps a 64-bit content hash of config and weights.

@@ -310,6 +310,41 @@ __global__ void fold_head_kernel(const T* __restrict__ W_dec, const T* __restric
   else cdec[a] = s;
 }
 
+// Deep & Wide head fold (weights only; App. B f_dec = [x_wide W_w + b_w,
+// FFN([z, x_deep])] with the FFN's last layer W_d2, b_d2).  With Q_w, Q_d the
+// columns of Q_dec against the wide and deep parts of k_dec:
+//   weff_x[j, a] = W_w[j] . Q_w[a] for j < dw_in, 0 for the deep features;
+//   cdec[a]      = b_w . Q_w[a] + b_d2 . Q_d[a];
+//   w2q[f, a]    = W_d2[f] . Q_d[a],
+// so logits = x weff_x + cdec + GELU([z, x_deep] W_d1 + b_d1) w2q.
+template <typename T>
+__global__ void fold_dw_kernel(const T* __restrict__ W_w, const T* __restrict__ b_w, const T* __restrict__ W_d2,
+                               const T* __restrict__ b_d2, const T* __restrict__ Q_dec, float* __restrict__ weff_x,
+                               float* __restrict__ cdec, float* __restrict__ w2q, int d, int dw_in, int dw_out,
+                               int Fh, int k) {
+  const int t = blockIdx.x * 256 + threadIdx.x;
+  if (t >= (d + 1 + Fh) * k) return;
+  const int j = t / k, a = t - j * k;
+  const T* q = Q_dec + static_cast<long long>(a) * d;
+  const int dd = d - dw_out;
+  float s = 0.f;
+  if (j < d) {
+    if (j < dw_in)
+      for (int c = 0; c < dw_out; ++c)
+        s = fmaf(Elem<T>::load(W_w + static_cast<long long>(j) * dw_out + c), Elem<T>::load(q + c), s);
+    weff_x[static_cast<long long>(j) * k + a] = s;
+  } else if (j == d) {
+    for (int c = 0; c < dw_out; ++c) s = fmaf(Elem<T>::load(b_w + c), Elem<T>::load(q + c), s);
+    for (int c = 0; c < dd; ++c) s = fmaf(Elem<T>::load(b_d2 + c), Elem<T>::load(q + dw_out + c), s);
+    cdec[a] = s;
+  } else {
+    const int f = j - d - 1;
+    for (int c = 0; c < dd; ++c)
+      s = fmaf(Elem<T>::load(W_d2 + static_cast<long long>(f) * dd + c), Elem<T>::load(q + dw_out + c), s);
+    w2q[static_cast<long long>(f) * k + a] = s;
+  }
+}
+
 // Order-independent 64-bit content hash: sum over 32-bit words of a
 // splitmix64-style finaliser of (word, index, salt).
 __global__ void hash_kernel(const uint32_t* __restrict__ p, long long n_words, uint64_t salt,
@@ -395,6 +430,15 @@ cudaError_t launch_fold_head(const T* W_dec, const T* b_dec, const T* Q_dec, flo
                              cudaStream_t s) {
   const int n = (2 * d + 1) * k;
   fold_head_kernel<T><<<(n + 255) / 256, 256, 0, s>>>(W_dec, b_dec, Q_dec, weff, cdec, d, k);
+  return cudaGetLastError();
+}
+
+template <typename T>
+cudaError_t launch_fold_dw(const T* W_w, const T* b_w, const T* W_d2, const T* b_d2, const T* Q_dec, float* weff_x,
+                           float* cdec, float* w2q, int d, int dw_in, int dw_out, int Fh, int k, cudaStream_t s) {
+  const int n = (d + 1 + Fh) * k;
+  fold_dw_kernel<T><<<(n + 255) / 256, 256, 0, s>>>(W_w, b_w, W_d2, b_d2, Q_dec, weff_x, cdec, w2q, d, dw_in, dw_out,
+                                                     Fh, k);
   return cudaGetLastError();
 }
 
@@ -589,7 +633,9 @@ cudaError_t launch_prefix_pool(const T* phi, const int* ends, int n_ev, int off_
                                              cudaStream_t);                                                         \
   template cudaError_t launch_transpose<T>(const T*, T*, int, int, cudaStream_t);                                  \
   template cudaError_t launch_to_f32<T>(const T*, float*, long long, cudaStream_t);                                \
-  template cudaError_t launch_fold_head<T>(const T*, const T*, const T*, float*, float*, int, int, cudaStream_t);
+  template cudaError_t launch_fold_head<T>(const T*, const T*, const T*, float*, float*, int, int, cudaStream_t); \
+  template cudaError_t launch_fold_dw<T>(const T*, const T*, const T*, const T*, const T*, float*, float*, float*,   \
+                                         int, int, int, int, int, cudaStream_t);
 TXS_INST(float)
 TXS_INST(__nv_bfloat16)
 #undef TXS_INST

@@ -147,7 +147,104 @@ __global__ void __launch_bounds__(1024) rank_kernel(const __grid_constant__ Rank
     for (int t = M + threadIdx.x; t < a.top_k; t += blockDim.x) out[static_cast<long long>(r) * a.top_k + t] = -1;
 }
 
+// Deep & Wide head input: row i of Z2 = [z_i, x_i[dw_in:]] for the candidate
+// rows (z: the decoder output, x: the raw candidate token).  One warp per row,
+// 16-byte vectors.
+template <typename T>
+__global__ void __launch_bounds__(256) dw_gather_kernel(const T* __restrict__ Z, const T* __restrict__ cand,
+                                                        T* __restrict__ Z2, int n_cand, int d, int dw_in) {
+  pdl_launch_dependents();
+  pdl_wait();
+  constexpr int VEC = Vec16<T>::N;
+  const int row = blockIdx.x * 8 + (threadIdx.x >> 5), lane = threadIdx.x & 31;
+  if (row >= n_cand) return;
+  const int w2 = 2 * d - dw_in;
+  T* dst = Z2 + static_cast<long long>(row) * w2;
+  for (int c = lane * VEC; c < w2; c += 32 * VEC) {
+    float v[VEC];
+    if (c < d) Vec16<T>::load(Z + static_cast<long long>(row) * d + c, v);
+    else Vec16<T>::load(cand + static_cast<long long>(row) * d + dw_in + (c - d), v);
+    Vec16<T>::store(dst + c, v);
+  }
+}
+
+// Deep & Wide head output: logits[i] = xlog[i] + h_i w2q, probs = softmax
+// (h = GELU([z, x_deep] W_d1 + b_d1), w2q = W_d2 Q_deep^T folded).  One warp
+// per candidate row; the fold keeps the Fh x k product in fp32.
+template <typename T>
+__global__ void __launch_bounds__(256) dw_head_kernel(const T* __restrict__ Hd, int Fh, const float* __restrict__ w2q,
+                                                      const float* __restrict__ xlog, int na, int n_cand,
+                                                      float* __restrict__ logits, float* __restrict__ probs) {
+  pdl_launch_dependents();
+  pdl_wait();
+  constexpr int VEC = Vec16<T>::N;
+  const int row = blockIdx.x * 8 + (threadIdx.x >> 5), lane = threadIdx.x & 31;
+  if (row >= n_cand) return;
+  float acc[16];
+#pragma unroll
+  for (int k = 0; k < 16; ++k) acc[k] = 0.f;
+  const T* h = Hd + static_cast<long long>(row) * Fh;
+  for (int f0 = lane * VEC; f0 < Fh; f0 += 32 * VEC) {
+    float v[VEC];
+    Vec16<T>::load(h + f0, v);
+#pragma unroll
+    for (int i = 0; i < VEC; ++i) {
+      const float* w = w2q + static_cast<long long>(f0 + i) * na;
+#pragma unroll
+      for (int k = 0; k < 16; ++k)
+        if (k < na) acc[k] = fmaf(v[i], __ldg(w + k), acc[k]);
+    }
+  }
+  float lg[16], mx = -INFINITY;
+#pragma unroll
+  for (int k = 0; k < 16; ++k) {
+    if (k < na) {
+      float x = acc[k];
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
+      lg[k] = x + xlog[static_cast<long long>(row) * na + k];
+      mx = fmaxf(mx, lg[k]);
+    }
+  }
+  if (lane != 0) return;
+  float sum = 0.f;
+#pragma unroll
+  for (int k = 0; k < 16; ++k)
+    if (k < na) {
+      logits[static_cast<long long>(row) * na + k] = lg[k];
+      sum += __expf(lg[k] - mx);
+    }
+  if (probs) {
+    const float inv = 1.f / sum;
+#pragma unroll
+    for (int k = 0; k < 16; ++k)
+      if (k < na) probs[static_cast<long long>(row) * na + k] = __expf(lg[k] - mx) * inv;
+  }
+}
+
 }  // namespace
+
+template <typename T>
+cudaError_t launch_dw_gather(const T* Z, const T* cand, T* Z2, int n_cand, int d, int dw_in, cudaStream_t s) {
+  if (n_cand == 0) return cudaSuccess;
+  prof_begin(KC_HEAD_DW, s);
+  cudaError_t e = launch_pdl(dw_gather_kernel<T>, dim3((n_cand + 7) / 8), dim3(256), 0, s, Z, cand, Z2, n_cand, d,
+                             dw_in);
+  prof_end(KC_HEAD_DW, s);
+  return e;
+}
+
+template <typename T>
+cudaError_t launch_dw_head(const T* Hd, int Fh, const float* w2q, const float* xlog, int na, int n_cand,
+                           float* logits, float* probs, cudaStream_t s) {
+  if (n_cand == 0) return cudaSuccess;
+  if (na > 16) return cudaErrorInvalidValue;
+  prof_begin(KC_HEAD_DW, s);
+  cudaError_t e = launch_pdl(dw_head_kernel<T>, dim3((n_cand + 7) / 8), dim3(256), 0, s, Hd, Fh, w2q, xlog, na,
+                             n_cand, logits, probs);
+  prof_end(KC_HEAD_DW, s);
+  return e;
+}
 
 template <typename T>
 cudaError_t launch_pack(int n_req, const int* cand_off_host, int S, int d, int na, const T* cand, const T* ctx, T* X,
@@ -205,6 +302,13 @@ cudaError_t launch_rank(int n_req, const int* cand_off_host, const float* probs,
   return err;
 }
 
+template cudaError_t launch_dw_gather<float>(const float*, const float*, float*, int, int, int, cudaStream_t);
+template cudaError_t launch_dw_gather<__nv_bfloat16>(const __nv_bfloat16*, const __nv_bfloat16*, __nv_bfloat16*, int,
+                                                     int, int, cudaStream_t);
+template cudaError_t launch_dw_head<float>(const float*, int, const float*, const float*, int, int, float*, float*,
+                                           cudaStream_t);
+template cudaError_t launch_dw_head<__nv_bfloat16>(const __nv_bfloat16*, int, const float*, const float*, int, int,
+                                                   float*, float*, cudaStream_t);
 template cudaError_t launch_pack<float>(int, const int*, int, int, int, const float*, const float*, float*, int*,
                                         int*, const float*, const float*, float*, cudaStream_t);
 template cudaError_t launch_pack<__nv_bfloat16>(int, const int*, int, int, int, const __nv_bfloat16*,

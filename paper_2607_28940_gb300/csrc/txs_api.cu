@@ -80,6 +80,8 @@ struct txs_model {
   float* cdec = nullptr;         // [k]
   void *Wt_c1 = nullptr, *Wt_c2 = nullptr;  // candidate MLP, transposed: [Fc, d], [d, Fc]
   float *b_c1 = nullptr, *b_c2 = nullptr;
+  void* Wt_d1 = nullptr;         // Deep & Wide deep FFN layer 1, transposed: [Fh, 2d - dw_in]
+  float *b_d1 = nullptr, *w2q = nullptr;  // [Fh], W_d2 Q_deep^T [Fh, k]
   int* status = nullptr;         // device status word
   uint64_t hash = 0;
 };
@@ -133,6 +135,11 @@ bool cfg_ok(const txs_config& c, std::string* why) {
   if (!(c.ln_eps > 0.f) || !std::isfinite(c.ln_eps)) return bad("ln_eps");
   if (c.n_kv_heads < 0 || (c.n_kv_heads > 0 && c.n_heads % c.n_kv_heads)) return bad("n_kv_heads");
   if (c.cand_mlp_hidden < 0 || c.cand_mlp_hidden % 64 || c.cand_mlp_hidden > 16384) return bad("cand_mlp_hidden");
+  if (c.head_dw_hidden < 0 || c.head_dw_hidden % 64 || c.head_dw_hidden > 16384) return bad("head_dw_hidden");
+  if (c.head_dw_hidden > 0) {
+    if (c.head_dw_in < 0 || c.head_dw_in > c.d_model || c.head_dw_in % 64) return bad("head_dw_in");
+    if (c.head_dw_out < 0 || c.head_dw_out >= c.d_model) return bad("head_dw_out");
+  }
   return true;
 }
 
@@ -182,7 +189,7 @@ ScoreLayout score_layout(const txs_config& c, int es, int n_req, long long n_can
   L.A = take(N * d * es);
   L.X1 = take(N * d * es);
   L.X2 = take(N * d * es);
-  L.Hf = take(N * std::max(F, static_cast<size_t>(c.cand_mlp_hidden)) * es);
+  L.Hf = take(N * std::max({F, static_cast<size_t>(c.cand_mlp_hidden), static_cast<size_t>(c.head_dw_hidden)}) * es);
   L.xlog = take(n_cand * c.n_actions * 4);
   L.tmp = take(c.dtype == TXS_FP32 ? N * d * 4 : 0);
   L.total = o;
@@ -277,11 +284,27 @@ txs_status model_prepare(txs_model* m, const void* const* w, cudaStream_t s) {
   TXS_CK(launch_to_f32<T>(static_cast<const T*>(head[0]), m->w_pool, d, s));
   if (!(m->weff = vf(2 * d * k))) return fail_cuda("cudaMalloc", err);
   if (!(m->cdec = vf(k))) return fail_cuda("cudaMalloc", err);
-  TXS_CK(launch_fold_head<T>(static_cast<const T*>(head[1]), static_cast<const T*>(head[2]),
-                             static_cast<const T*>(head[3]), m->weff, m->cdec, d, k, s));
-  // candidate-to-query MLP (optional)
-  const int Fc = c.cand_mlp_hidden;
+  const int Fc = c.cand_mlp_hidden, Fh = c.head_dw_hidden;
   const void* const* cm = head + TXS_HEAD_WEIGHTS;
+  const void* const* dw = cm + (Fc ? 4 : 0);
+  if (!Fh) {
+    TXS_CK(launch_fold_head<T>(static_cast<const T*>(head[1]), static_cast<const T*>(head[2]),
+                               static_cast<const T*>(head[3]), m->weff, m->cdec, d, k, s));
+  } else {
+    // Deep & Wide f_dec: the wide part and both biases fold into the x-part
+    // weights and constant the pack kernel evaluates; W_d2 folds with Q_dec
+    const int a = c.head_dw_in;
+    TXS_CK(cudaMemsetAsync(m->weff, 0, sizeof(float) * d * k, s));
+    if (!(m->w2q = vf(size_t(Fh) * k)) || !(m->b_d1 = vf(Fh)) || !(m->Wt_d1 = wt(Fh, 2 * d - a)))
+      return fail_cuda("cudaMalloc", err);
+    TXS_CK(launch_fold_dw<T>(static_cast<const T*>(dw[0]), static_cast<const T*>(dw[1]),
+                             static_cast<const T*>(dw[4]), static_cast<const T*>(dw[5]),
+                             static_cast<const T*>(head[3]), m->weff + size_t(d) * k, m->cdec, m->w2q, d, a,
+                             c.head_dw_out, Fh, k, s));
+    TXS_CK(launch_transpose<T>(static_cast<const T*>(dw[2]), static_cast<T*>(m->Wt_d1), 2 * d - a, Fh, s));
+    TXS_CK(launch_to_f32<T>(static_cast<const T*>(dw[3]), m->b_d1, Fh, s));
+  }
+  // candidate-to-query MLP (optional)
   if (Fc) {
     if (!(m->Wt_c1 = wt(Fc, d)) || !(m->Wt_c2 = wt(d, Fc)) || !(m->b_c1 = vf(Fc)) || !(m->b_c2 = vf(d)))
       return fail_cuda("cudaMalloc", err);
@@ -305,17 +328,24 @@ txs_status model_prepare(txs_model* m, const void* const* w, cudaStream_t s) {
   }
   const size_t nh[TXS_HEAD_WEIGHTS] = {size_t(d), 2 * size_t(d) * d, size_t(d), size_t(k) * d};
   for (int i = 0; i < TXS_HEAD_WEIGHTS; ++i)
-    TXS_CK(launch_hash(head[i], static_cast<long long>(nh[i] * es), 100000 + i, dh, s));
+    if (!Fh || (i != 1 && i != 2))  // W_dec, b_dec are unused with the Deep & Wide head
+      TXS_CK(launch_hash(head[i], static_cast<long long>(nh[i] * es), 100000 + i, dh, s));
   if (Fc) {
     const size_t nc[4] = {size_t(d) * Fc, size_t(Fc), size_t(Fc) * d, size_t(d)};
     for (int i = 0; i < 4; ++i) TXS_CK(launch_hash(cm[i], static_cast<long long>(nc[i] * es), 200000 + i, dh, s));
+  }
+  if (Fh) {
+    const size_t a = c.head_dw_in, o = c.head_dw_out;
+    const size_t nd[6] = {a * o, o, (2 * size_t(d) - a) * Fh, size_t(Fh), size_t(Fh) * (d - o), size_t(d) - o};
+    for (int i = 0; i < 6; ++i)
+      if (nd[i]) TXS_CK(launch_hash(dw[i], static_cast<long long>(nd[i] * es), 500000 + i, dh, s));
   }
   unsigned long long hv = 0;
   TXS_CK(cudaMemcpyAsync(&hv, dh, 8, cudaMemcpyDeviceToHost, s));
   TXS_CK(cudaStreamSynchronize(s));
   uint64_t h = hv;
   const int32_t cf[] = {c.d_model, c.n_heads, c.d_ff, c.n_layers, c.n_actions, c.n_ctx, c.l_local, c.attn_mode,
-                        c.dtype, kv_dim(c), c.cand_mlp_hidden};
+                        c.dtype, kv_dim(c), c.cand_mlp_hidden, c.head_dw_hidden, c.head_dw_in, c.head_dw_out};
   for (int32_t v : cf) h = (h ^ static_cast<uint64_t>(static_cast<uint32_t>(v))) * 0x100000001B3ull;
   uint32_t eps_bits;
   std::memcpy(&eps_bits, &c.ln_eps, 4);
@@ -492,7 +522,7 @@ txs_status score_impl(txs_model* m, const KvView& c, int n_req, const int32_t* c
     e.out = Hf;
     e.ldo = F;
     TXS_CK(gemm(m, X2, d, W.Wt_1, e, tmp, s, KC_GEMM_FFN1));
-    const bool last = l == cf.n_layers - 1;
+    const bool last = l == cf.n_layers - 1 && !cf.head_dw_hidden;  // fused linear head
     e = epi_base(last ? EPI_LN_HEAD : EPI_LN, N, d, F);
     e.bias = W.b_2;
     e.res = X2;
@@ -511,6 +541,19 @@ txs_status score_impl(txs_model* m, const KvView& c, int n_req, const int32_t* c
       e.probs = probs;
     }
     TXS_CK(gemm(m, Hf, F, W.Wt_2, e, tmp, s, KC_GEMM_FFN2));
+  }
+  // Deep & Wide f_dec (App. B): h = GELU([z, x_deep] W_d1 + b_d1) on the
+  // candidate rows, logits = x weff_x + cdec (from the pack kernel) + h w2q
+  if (cf.head_dw_hidden && n_cand > 0) {
+    const int a = cf.head_dw_in, Fh = cf.head_dw_hidden, w2 = 2 * d - a;
+    T* Z2 = QKV;  // free after the last layer: [n_cand, 2d - dw_in]
+    TXS_CK(launch_dw_gather<T>(X, static_cast<const T*>(cand_tok), Z2, static_cast<int>(n_cand), d, a, s));
+    EpiArgs e = epi_base(EPI_BIAS_GELU, n_cand, Fh, w2);
+    e.bias = m->b_d1;
+    e.out = Hf;
+    e.ldo = Fh;
+    TXS_CK(gemm(m, Z2, w2, m->Wt_d1, e, tmp, s, KC_HEAD_DW));
+    TXS_CK(launch_dw_head<T>(Hf, Fh, m->w2q, xlog, k, static_cast<int>(n_cand), logits, probs, s));
   }
   return TXS_OK;
 }
@@ -556,9 +599,17 @@ TXS_API txs_status txs_model_create(const txs_config* cfg, const void* const* we
     set_error(why.c_str());
     return TXS_ERR_UNSUPPORTED;
   }
-  const int n_w = cfg->n_layers * TXS_WEIGHTS_PER_LAYER + TXS_HEAD_WEIGHTS + (cfg->cand_mlp_hidden ? 4 : 0);
-  for (int i = 0; i < n_w; ++i)
-    if (!weights[i]) return TXS_ERR_INVALID_ARG;
+  const int n_dec = cfg->n_layers * TXS_WEIGHTS_PER_LAYER, n_cm = cfg->cand_mlp_hidden ? 4 : 0;
+  const int n_w = n_dec + TXS_HEAD_WEIGHTS + n_cm + (cfg->head_dw_hidden ? 6 : 0);
+  for (int i = 0; i < n_w; ++i) {
+    if (weights[i]) continue;
+    const int h = i - n_dec, dwi = i - n_dec - TXS_HEAD_WEIGHTS - n_cm;
+    const bool optional = cfg->head_dw_hidden &&
+                          (h == 1 || h == 2 ||  // W_dec, b_dec unused with the Deep & Wide head
+                           (dwi == 0 && (cfg->head_dw_in == 0 || cfg->head_dw_out == 0)) ||
+                           (dwi == 1 && cfg->head_dw_out == 0));
+    if (!optional) return TXS_ERR_INVALID_ARG;
+  }
   // the weight tensors may still be in flight on any stream of the caller
   cudaError_t pre = cudaDeviceSynchronize();
   if (pre != cudaSuccess) return fail_cuda("cudaDeviceSynchronize", pre);
@@ -1099,7 +1150,7 @@ TXS_API txs_status txs_profile_collect(double* total_ms, int64_t* launches, int3
 TXS_API const char* txs_kernel_class_name(int32_t cls) {
   static const char* names[] = {"pack", "gemm_qkv", "attn_serving", "gemm_oproj_ln", "gemm_q", "attn_cross",
                                 "gemm_ffn1_gelu", "gemm_ffn2_ln", "gemm_kv_build", "pool", "global_kv", "rank",
-                                "misc", "row_ln", "cand_mlp", "enc_embed", "enc_gemm", "enc_attn"};
+                                "misc", "row_ln", "cand_mlp", "enc_embed", "enc_gemm", "enc_attn", "head_dw"};
   if (cls < 0 || cls >= KC_COUNT_) return "";
   return names[cls];
 }

@@ -20,7 +20,7 @@ constexpr long long kSpinCycles = 2000000000LL;
 enum KernelClass : int {
   KC_PACK = 0, KC_GEMM_QKV, KC_ATTN_SERVING, KC_GEMM_OPROJ, KC_GEMM_Q, KC_ATTN_CROSS,
   KC_GEMM_FFN1, KC_GEMM_FFN2, KC_GEMM_KV, KC_POOL, KC_GLOBAL_KV, KC_RANK, KC_MISC,
-  KC_ROW_LN, KC_CAND_MLP, KC_ENC_EMBED, KC_ENC_GEMM, KC_ENC_ATTN, KC_COUNT_
+  KC_ROW_LN, KC_CAND_MLP, KC_ENC_EMBED, KC_ENC_GEMM, KC_ENC_ATTN, KC_HEAD_DW, KC_COUNT_
 };
 static_assert(KC_COUNT_ <= TXS_N_KERNEL_CLASSES, "profiler classes");
 
@@ -207,6 +207,14 @@ template <typename T>
 cudaError_t launch_transpose(const T* W, T* Wt, int rows, int cols, cudaStream_t s);
 template <typename T>
 cudaError_t launch_to_f32(const T* src, float* dst, long long n, cudaStream_t s);
+template <typename T>
+cudaError_t launch_fold_dw(const T* W_w, const T* b_w, const T* W_d2, const T* b_d2, const T* Q_dec, float* weff_x,
+                           float* cdec, float* w2q, int d, int dw_in, int dw_out, int Fh, int k, cudaStream_t s);
+template <typename T>
+cudaError_t launch_dw_gather(const T* Z, const T* cand, T* Z2, int n_cand, int d, int dw_in, cudaStream_t s);
+template <typename T>
+cudaError_t launch_dw_head(const T* Hd, int Fh, const float* w2q, const float* xlog, int na, int n_cand,
+                           float* logits, float* probs, cudaStream_t s);
 template <typename T>
 cudaError_t launch_fold_head(const T* W_dec, const T* b_dec, const T* Q_dec, float* weff, float* cdec, int d, int k,
                              cudaStream_t s);

@@ -47,7 +47,8 @@ class txs_config(ctypes.Structure):
     _fields_ = [("d_model", ctypes.c_int32), ("n_heads", ctypes.c_int32), ("d_ff", ctypes.c_int32),
                 ("n_layers", ctypes.c_int32), ("n_actions", ctypes.c_int32), ("n_ctx", ctypes.c_int32),
                 ("l_local", ctypes.c_int32), ("attn_mode", ctypes.c_int32), ("dtype", ctypes.c_int32),
-                ("ln_eps", ctypes.c_float), ("n_kv_heads", ctypes.c_int32), ("cand_mlp_hidden", ctypes.c_int32)]
+                ("ln_eps", ctypes.c_float), ("n_kv_heads", ctypes.c_int32), ("cand_mlp_hidden", ctypes.c_int32),
+                ("head_dw_hidden", ctypes.c_int32), ("head_dw_in", ctypes.c_int32), ("head_dw_out", ctypes.c_int32)]
 
 
 class txs_enc_config(ctypes.Structure):
@@ -165,14 +166,16 @@ def kv_width(wl: W.Workload) -> int:
 
 def make_config(wl: W.Workload, mode: int = LOCAL_GLOBAL) -> txs_config:
     return txs_config(wl.d_model, wl.n_heads, wl.d_ff, wl.n_layers, wl.n_actions, wl.n_ctx, wl.l_local, mode,
-                      TXS_BF16 if wl.dtype == "bf16" else TXS_FP32, wl.ln_eps, wl.n_kv_heads, wl.cand_mlp)
+                      TXS_BF16 if wl.dtype == "bf16" else TXS_FP32, wl.ln_eps, wl.n_kv_heads, wl.cand_mlp,
+                      wl.dw_hidden, wl.dw_in, wl.dw_out)
 
 
-def weight_order(n_layers: int, cand_mlp: int = 0) -> Sequence[str]:
+def weight_order(n_layers: int, cand_mlp: int = 0, dw_hidden: int = 0) -> Sequence[str]:
     """Names of the weight tensors in the order of txs_model_create."""
     names = [f"{n}.{l}" for l in range(n_layers) for n, _ in W.LAYER_WEIGHTS]
     names += [n for n, _ in W.HEAD_WEIGHTS]
-    return names + ([n for n, _ in W.CAND_WEIGHTS] if cand_mlp else [])
+    names += [n for n, _ in W.CAND_WEIGHTS] if cand_mlp else []
+    return names + ([n for n, _ in W.DW_WEIGHTS] if dw_hidden else [])
 
 
 class Model:
@@ -184,9 +187,10 @@ class Model:
         self.mode = mode
         self.dtype = torch_dtype(wl.dtype)
         self.cfg = make_config(wl, mode)
+        names = weight_order(wl.n_layers, wl.cand_mlp, wl.dw_hidden)
         dev = [torch.as_tensor(np.asarray(weights[n]), dtype=torch.float32).to(device).to(self.dtype).contiguous()
-               for n in weight_order(wl.n_layers, wl.cand_mlp)]
-        ptrs = (_P * len(dev))(*[t.data_ptr() for t in dev])
+               if n in weights and np.asarray(weights[n]).size else None for n in names]
+        ptrs = (_P * len(dev))(*[t.data_ptr() if t is not None else None for t in dev])
         h = _P()
         _check(lib().txs_model_create(ctypes.byref(self.cfg), ptrs, ctypes.byref(h)), "txs_model_create")
         self.handle = h
