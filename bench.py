@@ -325,6 +325,7 @@ def run_txs(args, rank, world):
             out["latency_vs_L"] = latency_sweep(txs, torch)
             out["events"] = events_bench(txs, torch)
             out["encoder"] = encoder_bench(txs, torch, peaks, peak_src)
+            out["deep_wide"] = deep_wide_bench(txs, torch)
             out["cpu_baseline"] = cpu_baseline(args.workload, budget_s=12.0)
     return out
 
@@ -474,6 +475,61 @@ def events_bench(txs, torch):
                           "kernels_ms": {k: v[0] for k, v in prof.items()}}
         if model.device_status() != txs.TXS_OK:
             raise RuntimeError("device status after the events measurement")
+        cache.close()
+        model.close()
+    return res
+
+
+DW_FIELDS = dict(dw_in=64, dw_out=32, dw_hidden=256)   # Deep & Wide head on the headline model
+
+
+def deep_wide_bench(txs, torch):
+    """The headline workload's score + rank with the Deep & Wide f_dec (App. B)
+    in place of the linear one, against the same prebuilt caches: candidates/s
+    and the per-class time of one call, next to the linear head's."""
+    wl0 = W.WORKLOADS[HEADLINE]
+    res = {"workload": f"{HEADLINE} with the Deep & Wide head (wide {DW_FIELDS['dw_in']} -> {DW_FIELDS['dw_out']}, "
+                       f"deep FFN [z, x_deep] -> {DW_FIELDS['dw_hidden']} -> d - {DW_FIELDS['dw_out']})",
+           "unit": "candidates/s"}
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device="cuda")
+    for name, wl in (("linear_head", wl0), ("deep_wide_head", W.with_sizes(wl0, **DW_FIELDS))):
+        b = W.batch(wl)
+        dt = txs.torch_dtype(wl.dtype)
+        model = txs.Model(wl, W.weights(wl), txs.LOCAL_GLOBAL)
+        cache = txs.KVCache(model, b.beh_off, txs.to_device(b.beh, dt))
+        cand = txs.to_device(b.cand, dt)
+        ctx = txs.to_device(b.ctx.reshape(-1, wl.d_model), dt)
+        n = int(b.cand_off[-1])
+        ws = torch.empty(txs.workspace_bytes(model, wl.n_req, n), dtype=torch.uint8, device="cuda")
+        lg = torch.empty((n, wl.n_actions), dtype=torch.float32, device="cuda")
+        pr = torch.empty_like(lg)
+        rk = torch.empty(n, dtype=torch.int32, device="cuda")
+
+        def call():
+            txs.score(model, cache, b.cand_off, cand, ctx, workspace=ws, out_logits=lg, out_probs=pr)
+            txs.rank(b.cand_off, pr, wl.n_actions, 0, 0, out=rk)
+        for _ in range(3):
+            call()
+        times = []
+        for _ in range(20):
+            flush.zero_()
+            e0 = torch.cuda.Event(enable_timing=True)
+            e1 = torch.cuda.Event(enable_timing=True)
+            e0.record()
+            call()
+            e1.record()
+            e1.synchronize()
+            times.append(e0.elapsed_time(e1))
+        txs.profile_enable(True)
+        call()
+        torch.cuda.synchronize()
+        prof = txs.profile_collect()
+        txs.profile_enable(False)
+        if model.device_status() != txs.TXS_OK:
+            raise RuntimeError("device status after the Deep & Wide measurement")
+        ms = statistics.median(times)
+        res[name] = {"ms_per_call": ms, "candidates_per_s": n / (ms / 1e3),
+                     "kernels_ms": {k: v[0] for k, v in prof.items()}}
         cache.close()
         model.close()
     return res
