@@ -631,15 +631,18 @@ def encoder_bench(txs, torch, peaks, peak_src):
     fl = ew.n_layers * pairs * 4 * d
     bms, bn_ = prof_b.get("enc_attn", (0.0, 0))
     ach_b = fl / (bms / 1e3) / 1e12 if bms else None
+    if ew.dtype == "bf16":   # enc_fa_kernel: tcgen05 MMAs for Q K^T and P V
+        roof_b = {"bound": "tensor", "peak": peaks["bf16_tflops"], "peak_source": f"{peak_src} (burst)"}
+    else:                    # enc_attn_kernel: FP32 FMAs on the CUDA cores
+        roof_b = {"bound": "alu", "peak": ALU_FP32_TFLOPS,
+                  "peak_source": "derived: 152 SMs x 128 FP32 lanes x 2 flop x 2070 MHz"}
+    roof_b.update({"achieved": ach_b, "unit": "TFLOP/s", "frac": ach_b / roof_b["peak"] if ach_b else None,
+                   "traffic": None, "kernel": "enc_attn", "algorithmic_flops_per_launch": fl / ew.n_layers})
     res["build"] = {
         "ms_per_call": statistics.median(builds), "tokens_per_s": n / (statistics.median(builds) / 1e3),
         "note": "includes the state's device allocation (cudaMalloc) inside the call",
         "kernels_ms": {k: v[0] for k, v in prof_b.items()},
-        "roofline_attn": {"bound": "alu", "achieved": ach_b, "peak": ALU_FP32_TFLOPS, "unit": "TFLOP/s",
-                          "frac": ach_b / ALU_FP32_TFLOPS if ach_b else None, "traffic": None,
-                          "kernel": "enc_attn",
-                          "peak_source": "derived: 152 SMs x 128 FP32 lanes x 2 flop x 2070 MHz",
-                          "algorithmic_flops_per_launch": fl / ew.n_layers}}
+        "roofline_attn": roof_b}
     st.close()
     enc.close()
     res["cpu_baseline"] = encoder_cpu_baseline(ew, w, b)

@@ -494,6 +494,341 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   if (threadIdx.x == 0 && *abort_flag) latch_status(a.status, TXS_ERR_DEVICE_TIMEOUT);
 }
 
+// ------------------------------------------------------------------ encoder self-attention
+
+// Causal self-attention of the behavior encoder (Sec. 4.1.1: causal mask and
+// a relative position bias) for the new rows of each user against that
+// user's cached keys/values of the same layer (App. D incremental encoding;
+// a build is the case "every row is new").  One CTA per (tile of up to 128
+// new rows of one user, head); the same producer / MMA / softmax pipeline as
+// fa_full_kernel, with:
+//   * key tiles of 128 positions aligned to multiples of 128 of the user's
+//     own position axis (tile jj holds positions 128 jj ...), from the tile
+//     of the first row's earliest visible key to the tile of the last row;
+//   * the mask (key position <= row position, inside the window) and the
+//     bias beta_h[min(i - j, R - 1)] (a shared-memory table, log2 units)
+//     applied by the softmax warps;
+//   * the running maximum raised per row (alpha = 1 for the rows that keep
+//     theirs), so that a row's arithmetic depends only on its own position
+//     and the keys: a tile with no visible key leaves the row untouched
+//     (P = 0).  Encoding rows incrementally therefore gives the same bytes as
+//     encoding them all at once.
+// The K/V storage is zero-initialised when the state is created, so key rows
+// of a tile that lie beyond the user's tokens are finite (P = 0 times a
+// finite value).
+struct EncFaArgs {
+  const __nv_bfloat16* q;  // [n, d] queries of the new rows
+  __nv_bfloat16* out;      // [n, d]
+  const int* in_off;       // [R + 1] new rows of user r
+  const int* dst0;         // [R] slot of user r's first new row
+  const int* slot_off;     // [R + 1] slots of user r
+  const int* tile_off;     // [R + 1] 128-row query tiles of user r
+  const float* beta;       // [H][n_rel] relative bias times log2(e)
+  int n_req, n_rel, window, d;
+  float scale_log2;        // log2(e) / sqrt(d_h)
+  int* status;
+};
+
+constexpr int kEncMaxRel = 8192;  // bias table entries staged in shared memory
+
+template <int DH>
+struct EncFaShape {
+  using Sh = FaShape<DH>;
+  static constexpr int BIAS_OFF = 2 * STG * Sh::KV_BYTES;
+  static constexpr int SMEM = BIAS_OFF + kEncMaxRel * 4 + 1024 + 256;
+};
+
+template <int DH>
+__global__ void __launch_bounds__(NUM_THREADS, 1)
+    enc_fa_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV,
+                  const EncFaArgs a) {
+  using Sh = FaShape<DH>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint8_t* sK = smem;
+  uint8_t* sV = sK + STG * Sh::KV_BYTES;
+  float* sB = reinterpret_cast<float*>(smem + EncFaShape<DH>::BIAS_OFF);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(sB + kEncMaxRel);
+  uint64_t* kv_full = bars;
+  uint64_t* kv_empty = kv_full + STG;
+  uint64_t* s_full = kv_empty + STG;
+  uint64_t* s_free = s_full + 2;
+  uint64_t* p_full = s_free + 2;
+  uint64_t* pv_done = p_full + 2;
+  uint64_t* q_ready = pv_done + 2;
+  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(q_ready + 1);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_holder + 1);
+
+  pdl_launch_dependents();
+  pdl_wait();
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int h = blockIdx.y;
+  const int r = find_segment(a.tile_off, a.n_req, blockIdx.x);
+  const int t = blockIdx.x - __ldg(a.tile_off + r);
+  const int row0 = __ldg(a.in_off + r) + t * BQ;
+  const int nrows = min(BQ, __ldg(a.in_off + r + 1) - row0);
+  const int base = __ldg(a.slot_off + r);
+  const int cap = __ldg(a.slot_off + r + 1) - base;
+  const int pos0 = __ldg(a.dst0 + r) - base + t * BQ;
+  if (nrows <= 0) return;                            // uniform
+  if (pos0 < 0 || pos0 + nrows > cap) {              // uniform
+    if (threadIdx.x == 0) latch_status(a.status, TXS_ERR_BOUNDS);
+    return;
+  }
+  const int p_last = pos0 + nrows - 1;
+  const int lo = a.window > 0 ? max(0, pos0 - a.window + 1) : 0;
+  const int jb = lo / BKV;
+  const int nkv = p_last / BKV - jb + 1;
+
+  for (int i = threadIdx.x; i < a.n_rel; i += NUM_THREADS)
+    sB[i] = __ldg(a.beta + static_cast<long long>(h) * a.n_rel + i);
+  if (threadIdx.x == 0) {
+    for (int st = 0; st < STG; ++st) {
+      mbar_init(kv_full + st, 1);
+      mbar_init(kv_empty + st, 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(s_full + b, 1);
+      mbar_init(s_free + b, 4);
+      mbar_init(p_full + b, 4);
+      mbar_init(pv_done + b, 1);
+    }
+    mbar_init(q_ready, 4);
+    *abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == 1) tmem_alloc(tmem_holder, Sh::TMEM_COLS);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_holder;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmK)) : "memory");
+      asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmV)) : "memory");
+      int issued = 0;
+      for (int j = 0; j < nkv; ++j) {
+        const int st = j % STG;
+        if (!mbar_wait(kv_empty + st, ((j / STG) & 1) ^ 1, abort_flag)) break;
+        mbar_expect_tx(kv_full + st, 2 * Sh::KV_BYTES);
+        const int krow = base + (jb + j) * BKV;
+        tma_load_2d(sK + st * Sh::KV_BYTES, &tmK, kv_full + st, h * DH, krow);
+        tma_load_2d(sV + st * Sh::KV_BYTES, &tmV, kv_full + st, h * DH, krow);
+        issued = j + 1;
+      }
+      if (*abort_flag)
+        for (int k = issued > STG ? issued - STG : 0; k < issued; ++k)
+          mbar_wait_plain(kv_full + k % STG, (k / STG) & 1);
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      constexpr uint32_t id_s = idesc_bf16(BQ, BKV, false);
+      constexpr uint32_t id_pv = idesc_bf16(BQ, DH, true);
+      bool ok = mbar_wait(q_ready, 0, abort_flag);
+      tc_fence_after();
+      auto pv = [&](int tt) -> bool {
+        const int bt = tt & 1, st = tt % STG;
+        if (!mbar_wait(p_full + bt, (tt >> 1) & 1, abort_flag)) return false;
+        tc_fence_after();
+        const uint32_t v_addr = smem_u32(sV + st * Sh::KV_BYTES);
+#pragma unroll
+        for (int k = 0; k < BKV / 16; ++k) {
+          const uint64_t vd = sdesc(v_addr + k * 16 * Sh::ROW_BYTES, Sh::ATOM, Sh::ATOM, Sh::SW);
+          mma_bf16_ts(tmem + Sh::T_O, tmem + Sh::T_P + 64 * bt + 8 * k, vd, id_pv, (tt > 0 || k > 0) ? 1u : 0u);
+        }
+        mma_commit(pv_done + bt);
+        mma_commit(kv_empty + st);
+        return true;
+      };
+      for (int j = 0; j < nkv && ok; ++j) {
+        const int st = j % STG, b = j & 1;
+        if (!mbar_wait(kv_full + st, (j / STG) & 1, abort_flag)) break;
+        if (!mbar_wait(s_free + b, ((j >> 1) & 1) ^ 1, abort_flag)) break;
+        tc_fence_after();
+        const uint32_t k_addr = smem_u32(sK + st * Sh::KV_BYTES);
+#pragma unroll
+        for (int k = 0; k < DH / 16; ++k) {
+          const uint64_t kd = sdesc(k_addr + k * 32, 16, Sh::ATOM, Sh::SW);
+          mma_bf16_ts(tmem + Sh::T_S + BKV * b, tmem + Sh::T_Q + 8 * k, kd, id_s, k > 0 ? 1u : 0u);
+        }
+        mma_commit(s_full + b);
+        if (j >= 1) ok = pv(j - 1);
+      }
+      if (ok && !*abort_flag) pv(nkv - 1);
+    }
+  } else {
+    // ---------------- softmax warps: one query row per thread
+    const int qw = warp & 3;
+    const int m = qw * 32 + lane;
+    const bool valid = m < nrows;
+    const int p = pos0 + m;                    // this row's position on the user's axis
+    const uint32_t lane_off = static_cast<uint32_t>(qw * 32) << 16;
+    {
+      uint32_t qv[DH / 2];
+      const uint4* src = reinterpret_cast<const uint4*>(a.q + static_cast<long long>(valid ? row0 + m : row0) * a.d +
+                                                        h * DH);
+#pragma unroll
+      for (int c = 0; c < DH / 8; ++c) {
+        const uint4 v = valid ? src[c] : make_uint4(0, 0, 0, 0);
+        qv[4 * c] = v.x; qv[4 * c + 1] = v.y; qv[4 * c + 2] = v.z; qv[4 * c + 3] = v.w;
+      }
+#pragma unroll
+      for (int c = 0; c < DH / 2; c += 16) tmem_st16(tmem + Sh::T_Q + c + lane_off, qv + c);
+      tmem_wait_st();
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(q_ready);
+    }
+    const uint32_t t_o = tmem + Sh::T_O + lane_off;
+    const int R1 = a.n_rel - 1;
+    const float b_far = sB[R1];
+    // a warp whose 32 rows are all past the tile's last new row only keeps the
+    // barrier protocol: its rows' P, O and sums are never used (each O row
+    // depends on its own P row only)
+    const bool idle = qw * 32 >= nrows;
+    float m_run = -INFINITY, l_run = 0.f;
+    bool ok = true;
+    for (int j = 0; j < nkv && ok; ++j) {
+      const int b = j & 1;
+      ok = mbar_wait(s_full + b, (j >> 1) & 1, abort_flag);
+      ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
+      if (!ok) break;
+      tc_fence_after();
+      if (idle) {
+        __syncwarp();
+        if (lane == 0) mbar_arrive(s_free + b);
+        if (j >= 2) {
+          ok = mbar_wait(pv_done + b, ((j - 2) >> 1) & 1, abort_flag);
+          ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
+          if (!ok) break;
+        }
+        __syncwarp();
+        if (lane == 0) mbar_arrive(p_full + b);
+        continue;
+      }
+      float sv[BKV];
+      tmem_ld128(tmem + Sh::T_S + BKV * b + lane_off, sv);
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(s_free + b);
+      // logits in log2 units: scaled score + bias where visible, -inf
+      // elsewhere.  Rows past the last new row follow the same rule at their
+      // would-be positions (their results are discarded), which keeps the
+      // warp on one path.
+      const int D0 = p - (jb + j) * BKV;       // distance to the tile's first key
+      const bool all_vis = D0 >= BKV - 1 && (a.window <= 0 || D0 < a.window);
+      if (__all_sync(0xffffffffu, all_vis && D0 - (BKV - 1) >= R1)) {
+#pragma unroll
+        for (int i = 0; i < BKV; ++i) sv[i] = fmaf(sv[i], a.scale_log2, b_far);
+      } else {
+#pragma unroll
+        for (int i = 0; i < BKV; ++i) {
+          const int dist = D0 - i;
+          const bool vis = dist >= 0 && (a.window <= 0 || dist < a.window);
+          sv[i] = vis ? fmaf(sv[i], a.scale_log2, sB[min(dist, R1)]) : -INFINITY;
+        }
+      }
+      float mx8[8];
+#pragma unroll
+      for (int i = 0; i < 8; ++i) mx8[i] = sv[i];
+#pragma unroll
+      for (int i = 8; i < BKV; ++i) mx8[i & 7] = fmaxf(mx8[i & 7], sv[i]);
+#pragma unroll
+      for (int w = 4; w >= 1; w >>= 1)
+#pragma unroll
+        for (int i = 0; i < w; ++i) mx8[i] = fmaxf(mx8[i], mx8[i + w]);
+      const float m_tile = mx8[0];
+      const bool need = m_tile > m_run + kRescaleLog2;
+      if (__any_sync(0xffffffffu, need)) {
+        const float m_new = need ? fmaxf(m_run, m_tile) : m_run;
+        const float alpha = need ? ex2(m_run - m_new) : 1.f;   // 0 on a row's first visible tile
+        if (j >= 1) {
+          ok = mbar_wait(pv_done + ((j - 1) & 1), ((j - 1) >> 1) & 1, abort_flag);
+          ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
+          if (!ok) break;
+          tc_fence_after();
+#pragma unroll
+          for (int cc = 0; cc < DH; cc += 32) {
+            float ov[32];
+            tmem_ld32(t_o + cc, ov);
+#pragma unroll
+            for (int i = 0; i < 32; ++i) ov[i] *= alpha;
+            tmem_st32(t_o + cc, ov);
+          }
+        }
+        l_run *= alpha;
+        m_run = m_new;
+      }
+      if (j >= 2) {
+        ok = mbar_wait(pv_done + b, ((j - 2) >> 1) & 1, abort_flag);
+        ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
+        if (!ok) break;
+        tc_fence_after();
+      }
+      // P = 2^(s - m_run); 0 where masked (also while the row has no visible key yet)
+      const uint32_t t_p = tmem + Sh::T_P + 64 * b + lane_off;
+      float ps8[8];
+#pragma unroll
+      for (int i = 0; i < 8; ++i) ps8[i] = 0.f;
+#pragma unroll
+      for (int c32 = 0; c32 < BKV; c32 += 32) {
+        uint32_t pk[16];
+#pragma unroll
+        for (int i = 0; i < 32; i += 2) {
+          const float s0 = sv[c32 + i], s1 = sv[c32 + i + 1];
+          const float p0 = s0 == -INFINITY ? 0.f : ex2(s0 - m_run);
+          const float p1 = s1 == -INFINITY ? 0.f : ex2(s1 - m_run);
+          ps8[i & 7] += p0;
+          ps8[(i + 1) & 7] += p1;
+          __nv_bfloat162 h2 = __floats2bfloat162_rn(p0, p1);
+          pk[i / 2] = *reinterpret_cast<uint32_t*>(&h2);
+        }
+        tmem_st16(t_p + c32 / 2, pk);
+      }
+      tmem_wait_st();
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(p_full + b);
+#pragma unroll
+      for (int w = 4; w >= 1; w >>= 1)
+#pragma unroll
+        for (int i = 0; i < w; ++i) ps8[i] += ps8[i + w];
+      l_run += ps8[0];
+    }
+    if (ok) {
+      ok = mbar_wait(pv_done + ((nkv - 1) & 1), ((nkv - 1) >> 1) & 1, abort_flag);
+      ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
+    }
+    if (ok && !idle) {
+      tc_fence_after();
+      const float inv = valid ? 1.f / l_run : 0.f;
+      __nv_bfloat16* dst = a.out + static_cast<long long>(valid ? row0 + m : row0) * a.d + h * DH;
+#pragma unroll
+      for (int cc = 0; cc < DH; cc += 32) {
+        float ov[32];
+        tmem_ld32(t_o + cc, ov);
+        if (valid) {
+#pragma unroll
+          for (int c = 0; c < 32; c += 8) {
+            float tv[8];
+#pragma unroll
+            for (int i = 0; i < 8; ++i) tv[i] = ov[c + i] * inv;
+            Vec16<__nv_bfloat16>::store(dst + cc + c, tv);
+          }
+        }
+      }
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, Sh::TMEM_COLS);
+  }
+  if (threadIdx.x == 0 && *abort_flag) latch_status(a.status, TXS_ERR_DEVICE_TIMEOUT);
+}
+
 // ------------------------------------------------------------------ host side
 
 typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
@@ -544,7 +879,45 @@ static cudaError_t launch_dh(const FaArgs& a, const void* Kc, const void* Vc, lo
   return launch_pdl(fa_full_kernel<DH>, grid, dim3(NUM_THREADS), Sh::SMEM, s, tk, tv, a);
 }
 
+template <int DH>
+static cudaError_t launch_enc_dh(const EncFaArgs& a, const void* K, const void* V, long long cap_total, int n_tiles,
+                                 int H, cudaStream_t s) {
+  static bool attr = false;
+  if (!attr) {
+    cudaError_t e = cudaFuncSetAttribute(enc_fa_kernel<DH>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         EncFaShape<DH>::SMEM);
+    if (e != cudaSuccess) return e;
+    attr = true;
+  }
+  CUtensorMap tk, tv;
+  if (!make_kv_map<DH>(&tk, K, cap_total, a.d) || !make_kv_map<DH>(&tv, V, cap_total, a.d))
+    return cudaErrorInvalidValue;
+  return launch_pdl(enc_fa_kernel<DH>, dim3(n_tiles, H), dim3(NUM_THREADS), EncFaShape<DH>::SMEM, s, tk, tv, a);
+}
+
 }  // namespace fa
+
+bool enc_attn_tc_supported(int d, int H, int n_rel) {
+  const int dh = d / H;
+  return (dh == 32 || dh == 64) && n_rel >= 1 && n_rel <= fa::kEncMaxRel && d % 8 == 0;
+}
+
+cudaError_t launch_enc_attn_tc(const __nv_bfloat16* q, const __nv_bfloat16* K, const __nv_bfloat16* V,
+                               __nv_bfloat16* out, long long cap_total, const int* in_off, const int* dst0,
+                               const int* slot_off, const int* tile_off, int n_req, int n_tiles,
+                               const float* beta_log2, int n_rel, int window, int H, int d, int* status,
+                               cudaStream_t s) {
+  if (n_tiles == 0) return cudaSuccess;
+  if (!enc_attn_tc_supported(d, H, n_rel)) return cudaErrorNotSupported;
+  const int dh = d / H;
+  fa::EncFaArgs a{q, out, in_off, dst0, slot_off, tile_off, beta_log2, n_req, n_rel, window, d,
+                  1.4426950408889634f / sqrtf(static_cast<float>(dh)), status};
+  prof_begin(KC_ENC_ATTN, s);
+  cudaError_t err = dh == 64 ? fa::launch_enc_dh<64>(a, K, V, cap_total, n_tiles, H, s)
+                             : fa::launch_enc_dh<32>(a, K, V, cap_total, n_tiles, H, s);
+  prof_end(KC_ENC_ATTN, s);
+  return err;
+}
 
 bool fa_full_supported(int d, int H, long long cap_total) {
   const int dh = d / H;

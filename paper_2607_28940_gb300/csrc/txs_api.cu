@@ -688,6 +688,10 @@ txs_status make_cache(txs_model* m, int n_req, const int* lengths, int capacity_
     return p;
   };
   c->kv = A(size_t(nL) * 2 * tot * c->dkv * m->es);
+  // zeroed: a FULL-mode key tile may read rows past a request's length
+  // (masked, P = 0), which must hold finite values
+  if (st == TXS_OK && (err = cudaMemsetAsync(c->kv, 0, size_t(nL) * 2 * tot * c->dkv * m->es, s)) != cudaSuccess)
+    st = fail_cuda("cudaMemsetAsync", err);
   c->d_off = static_cast<int*>(A(4 * (n_req + 1)));
   c->d_len = static_cast<int*>(A(4 * n_req));
   c->d_in_off = static_cast<int*>(A(4 * (2 * n_req + 1)));

@@ -8,6 +8,7 @@
 #include <cmath>
 #include <cstring>
 #include <string>
+#include <type_traits>
 #include <vector>
 
 #include "txs_internal.cuh"
@@ -232,7 +233,10 @@ txs_status encode_impl(txs_encoder* m, txs_enc_state* st, const int32_t* in_off,
   const long long n = in_off[R];
   int max_new = 0;
   for (int r = 0; r < R; ++r) max_new = std::max(max_new, in_off[r + 1] - in_off[r]);
-  const int QT = enc_query_tile(max_new);
+  // bf16: tensor-core attention (128-row tiles) for build and append alike,
+  // which keeps incremental encoding bit-identical to a full encode
+  const bool use_tc = std::is_same<T, __nv_bfloat16>::value && enc_attn_tc_supported(d, H, c.n_rel);
+  const int QT = use_tc ? 128 : enc_query_tile(max_new);
   std::vector<int> up(3 * R + 2);
   int tiles = 0;
   for (int r = 0; r <= R; ++r) up[r] = in_off[r];
@@ -281,8 +285,19 @@ txs_status encode_impl(txs_encoder* m, txs_enc_state* st, const int32_t* in_off,
     e.col_blk_stride = st->cap_total * d;
     ENC_CK(enc_gemm(m, X, d, static_cast<const T*>(W.Wt_qkv) + size_t(d) * d, e, tmp, s));
     // causal attention with the relative position bias
-    ENC_CK(launch_enc_attn<T>(Q, Kl, Vl, A, d_in_off, d_dst0, st->d_off, d_tile_off, R, tiles, QT,
-                              m->rel + size_t(l) * H * c.n_rel, c.n_rel, c.window, H, d, m->status, s));
+    const float* beta = m->rel + size_t(l) * H * c.n_rel;
+    if constexpr (std::is_same<T, __nv_bfloat16>::value) {
+      if (use_tc) {
+        ENC_CK(launch_enc_attn_tc(Q, Kl, Vl, A, st->cap_total, d_in_off, d_dst0, st->d_off, d_tile_off, R, tiles,
+                                  beta, c.n_rel, c.window, H, d, m->status, s));
+      } else {
+        ENC_CK(launch_enc_attn<T>(Q, Kl, Vl, A, d_in_off, d_dst0, st->d_off, d_tile_off, R, tiles, QT, beta,
+                                  c.n_rel, c.window, H, d, m->status, s));
+      }
+    } else {
+      ENC_CK(launch_enc_attn<T>(Q, Kl, Vl, A, d_in_off, d_dst0, st->d_off, d_tile_off, R, tiles, QT, beta,
+                                c.n_rel, c.window, H, d, m->status, s));
+    }
     // H = LN1(X + A W_o + b_o)
     e = enc_epi(EPI_LN, n, d, d);
     e.bias = W.b_o;
@@ -435,6 +450,11 @@ TXS_API txs_status txs_encode_build(txs_encoder* m, int32_t n_req, const int32_t
     return p;
   };
   st->kv = A(size_t(c.n_layers) * 2 * tot * c.d_model * m->es);
+  // zeroed: attention tiles may read key rows past a user's tokens (masked,
+  // P = 0), which must hold finite values
+  if (rc == TXS_OK && (err = cudaMemsetAsync(st->kv, 0, size_t(c.n_layers) * 2 * tot * c.d_model * m->es, s)) !=
+                          cudaSuccess)
+    rc = enc_fail("cudaMemsetAsync", err);
   st->d_off = static_cast<int*>(A(4 * size_t(n_req + 1)));
   st->d_call = static_cast<int*>(A(4 * size_t(3 * n_req + 2)));
   if (rc == TXS_OK) {

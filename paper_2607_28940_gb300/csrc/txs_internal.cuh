@@ -241,6 +241,15 @@ cudaError_t launch_enc_attn(const T* q, const T* K, const T* V, T* out, const in
                             const int* slot_off, const int* tile_off, int n_req, int n_tiles, int query_tile,
                             const float* beta_log2, int n_rel, int window, int H, int d, int* status,
                             cudaStream_t s);
+// The same on the tensor cores (bf16; 128-row query tiles, 128-key tiles
+// aligned on each user's position axis); cudaErrorNotSupported unless d_h is
+// 32 or 64 and n_rel <= 8192.
+bool enc_attn_tc_supported(int d, int H, int n_rel);
+cudaError_t launch_enc_attn_tc(const __nv_bfloat16* q, const __nv_bfloat16* K, const __nv_bfloat16* V,
+                               __nv_bfloat16* out, long long cap_total, const int* in_off, const int* dst0,
+                               const int* slot_off, const int* tile_off, int n_req, int n_tiles,
+                               const float* beta_log2, int n_rel, int window, int H, int d, int* status,
+                               cudaStream_t s);
 void set_last_error(const char* msg);
 
 }  // namespace txs
