@@ -48,7 +48,7 @@ FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0}
 # one --set full capture of that class's kernel on that workload.
 NCU_TRAFFIC = {
     ("small_bf16", "local_global", "gemm_oproj_ln"): (8.62e6, "19df9b0ee59c"),
-    ("mid_bf16", "full", "attn_cross"): (830.4e6, "5e48154e4f63"),
+    ("mid_bf16", "full", "attn_cross"): (825.0e6, "a39aec35cabd"),
 }
 
 
@@ -61,6 +61,10 @@ def parse():
     p.add_argument("--workload", default=HEADLINE, choices=sorted(W.WORKLOADS))
     p.add_argument("--mode", default="local_global", choices=["local_global", "full"])
     p.add_argument("--no-extras", action="store_true", help="skip latency sweep, e2e and CPU baseline")
+    p.add_argument("--section", choices=["encoder", "deep_wide", "events"],
+                   help="run only this extra section (one JSON object) and exit")
+    p.add_argument("--enc-len", type=int, default=0,
+                   help="tokens per user of the encoder section (default: the workload's)")
     return p.parse_args()
 
 
@@ -542,12 +546,14 @@ ENC_APPENDS, ENC_PROFILED = 24, 8
 ALU_FP32_TFLOPS = 152 * 128 * 2 * 2.070e9 / 1e12
 
 
-def encoder_bench(txs, torch, peaks, peak_src):
+def encoder_bench(txs, torch, peaks, peak_src, tokens=0):
     """Behavior encoder (Sec. 4.1.1; App. D incremental encoding) on the
     64-user x 4096-token workload: the incremental append of 8 new tokens per
     user (the nearline streaming update) and the full-stream build, with the
     roofline of each one's attention kernel and the oracle on a sample."""
     ew = W.ENC_WORKLOADS[ENC_WORKLOAD]
+    if tokens:
+        ew = W.with_sizes(ew, L=tokens)
     w = W.enc_weights(ew)
     b = W.enc_batch(ew)
     dt = txs.torch_dtype(ew.dtype)
@@ -736,6 +742,17 @@ def main():
     if args.impl == "reference":
         if rank == 0:
             print(json.dumps(run_reference(args, rank, world)), flush=True)
+        return
+    if args.section:
+        import torch
+        from paper_2607_28940_gb300 import build as B
+        from paper_2607_28940_gb300 import txs
+        B.build()
+        peaks, peak_src = load_peaks()
+        fn = {"encoder": lambda: encoder_bench(txs, torch, peaks, peak_src, args.enc_len),
+              "deep_wide": lambda: deep_wide_bench(txs, torch),
+              "events": lambda: events_bench(txs, torch)}[args.section]
+        print(json.dumps({args.section: fn()}, default=float), flush=True)
         return
     if world > 1:
         import torch
