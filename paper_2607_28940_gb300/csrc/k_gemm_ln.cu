@@ -167,15 +167,23 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     for (int i = 0; i < my_tiles; ++i) {
       const int buf = i & 1, pb = i & 1;
       const uint32_t use = static_cast<uint32_t>(i >> 1) & 1;
+      const int m0 = (cid + i * ncl) * BM;
+      const int row = m0 + trow;
+      const bool valid = row < e.M;
+      // the residual row does not depend on the product: fetch it before
+      // waiting for the accumulator, so its DRAM latency overlaps the MMAs
+      uint4 rres[8];
+      {
+        const uint4* rp = reinterpret_cast<const uint4*>(static_cast<const __nv_bfloat16*>(e.res) +
+                                                         (valid ? row : 0) * e.ldr + n0 + c0);
+#pragma unroll
+        for (int k = 0; k < 8; ++k) rres[k] = valid ? __ldg(rp + k) : make_uint4(0, 0, 0, 0);
+      }
       bool go = mbar_wait(acc_full + buf, use, abort_flag);
       go = __shfl_sync(0xffffffffu, go ? 1 : 0, 0) != 0;
       if (!go) break;
       tc_fence_after();
-      const int m0 = (cid + i * ncl) * BM;
-      const int row = m0 + trow;
-      const bool valid = row < e.M;
       const uint32_t tacc = tmem + buf * BN + (static_cast<uint32_t>(q * 32) << 16) + c0;
-      const __nv_bfloat16* res = valid ? static_cast<const __nv_bfloat16*>(e.res) + row * e.ldr + n0 + c0 : nullptr;
       // pass 1: v = acc + bias + residual, written back to TMEM
       float sum = 0.f;
 #pragma unroll
@@ -183,10 +191,15 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         tmem_ld32(tacc + c, v);
         float b[32], r[32];
         load_f32x32(e.bias + n0 + c0 + c, b);
-        if (valid) load_bf16x32(res + c, r);
-        else {
 #pragma unroll
-          for (int k = 0; k < 32; ++k) r[k] = 0.f;
+        for (int k = 0; k < 4; ++k) {
+          const __nv_bfloat162* h2 = reinterpret_cast<const __nv_bfloat162*>(&rres[c / 8 + k]);
+#pragma unroll
+          for (int t = 0; t < 4; ++t) {
+            const float2 f = __bfloat1622float2(h2[t]);
+            r[8 * k + 2 * t] = f.x;
+            r[8 * k + 2 * t + 1] = f.y;
+          }
         }
 #pragma unroll
         for (int k = 0; k < 32; ++k) {
