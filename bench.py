@@ -61,7 +61,7 @@ def parse():
     p.add_argument("--workload", default=HEADLINE, choices=sorted(W.WORKLOADS))
     p.add_argument("--mode", default="local_global", choices=["local_global", "full"])
     p.add_argument("--no-extras", action="store_true", help="skip latency sweep, e2e and CPU baseline")
-    p.add_argument("--section", choices=["encoder", "deep_wide", "events"],
+    p.add_argument("--section", choices=["encoder", "deep_wide", "events", "sweep"],
                    help="run only this extra section (one JSON object) and exit")
     p.add_argument("--enc-len", type=int, default=0,
                    help="tokens per user of the encoder section (default: the workload's)")
@@ -330,6 +330,7 @@ def run_txs(args, rank, world):
             out["events"] = events_bench(txs, torch)
             out["encoder"] = encoder_bench(txs, torch, peaks, peak_src)
             out["deep_wide"] = deep_wide_bench(txs, torch)
+            out["sweep"] = sweep_bench(txs, torch, peaks, peak_src)
             out["cpu_baseline"] = cpu_baseline(args.workload, budget_s=12.0)
     return out
 
@@ -481,6 +482,112 @@ def events_bench(txs, torch):
             raise RuntimeError("device status after the events measurement")
         cache.close()
         model.close()
+    return res
+
+
+SWEEP_WORKLOAD = "sweep_bf16"   # R = 16 requests x 8192 behavior rows, d = 512, 4 layers
+SWEEP_M = (64, 256, 1024, 4096)
+SWEEP_DL = (1, 2, 4, 8, 16, 32, 64)
+
+
+def sweep_bench(txs, torch, peaks, peak_src):
+    """The sweep configuration: score + rank latency and candidates/s for
+    M in SWEEP_M candidates per request against one prebuilt cache (both
+    key-set modes; FULL with the roofline of its cross-attention), and the
+    incremental append of dL in SWEEP_DL rows per request against a full
+    rebuild of the cache (App. D: an append scales with the new rows)."""
+    base = W.WORKLOADS[SWEEP_WORKLOAD]
+    weights = W.weights(base)
+    dt = txs.torch_dtype(base.dtype)
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device="cuda")
+    b0 = W.batch(base, M_override=SWEEP_M[0])
+    beh = txs.to_device(b0.beh, dt)
+    L = int(b0.L[0])
+    d, nL = base.d_model, base.n_layers
+    res = {"workload": f"{SWEEP_WORKLOAD}: R={base.n_req} requests x L={L} rows, d={d}, {nL} layers; "
+                       f"M per request in {list(SWEEP_M)}; appends of dL rows per request in {list(SWEEP_DL)}",
+           "unit": "ms"}
+
+    def timed(fn, reps, flush_l2=True):
+        for _ in range(3):
+            fn()
+        times = []
+        for _ in range(reps):
+            if flush_l2:
+                flush.zero_()
+            e0 = torch.cuda.Event(enable_timing=True)
+            e1 = torch.cuda.Event(enable_timing=True)
+            e0.record()
+            fn()
+            e1.record()
+            e1.synchronize()
+            times.append(e0.elapsed_time(e1))
+        return statistics.median(times)
+
+    for mode_name, mode in (("local_global", txs.LOCAL_GLOBAL), ("full", txs.FULL)):
+        model = txs.Model(base, weights, mode)
+        cache = txs.KVCache(model, b0.beh_off, beh)
+        rows = {}
+        for M in SWEEP_M:
+            b = W.batch(base, M_override=M)
+            cand = txs.to_device(b.cand, dt)
+            ctx = txs.to_device(b.ctx.reshape(-1, d), dt)
+            n = int(b.cand_off[-1])
+            ws = torch.empty(txs.workspace_bytes(model, base.n_req, n), dtype=torch.uint8, device="cuda")
+            lg = torch.empty((n, base.n_actions), dtype=torch.float32, device="cuda")
+            pr = torch.empty_like(lg)
+            rk = torch.empty(n, dtype=torch.int32, device="cuda")
+
+            def call():
+                txs.score(model, cache, b.cand_off, cand, ctx, workspace=ws, out_logits=lg, out_probs=pr)
+                txs.rank(b.cand_off, pr, base.n_actions, 0, 0, out=rk)
+            ms = timed(call, 10)
+            row = {"ms_per_call": ms, "candidates_per_s": n / (ms / 1e3)}
+            if mode == txs.FULL:
+                txs.profile_enable(True)
+                call()
+                torch.cuda.synchronize()
+                prof = txs.profile_collect()
+                txs.profile_enable(False)
+                a_ms = prof.get("attn_cross", (0.0, 0))[0]
+                fl = 4.0 * n * L * d * nL          # candidate rows only
+                by = 2.0 * nL * (2 * base.n_req * L * d + 2 * n * d)
+                t_t, t_h = fl / (peaks["bf16_tflops"] * 1e12), by / (peaks["hbm_gbs"] * 1e9)
+                if t_t >= t_h:
+                    ach = fl / (a_ms / 1e3) / 1e12
+                    row["roofline_attn_cross"] = {"bound": "tensor", "achieved": ach, "peak": peaks["bf16_tflops"],
+                                                  "unit": "TFLOP/s", "frac": ach / peaks["bf16_tflops"]}
+                else:
+                    ach = by / (a_ms / 1e3) / 1e9
+                    row["roofline_attn_cross"] = {"bound": "hbm", "achieved": ach, "peak": peaks["hbm_gbs"],
+                                                  "unit": "GB/s", "frac": ach / peaks["hbm_gbs"]}
+                row["roofline_attn_cross"].update({"kernel": "attn_cross", "ms": a_ms,
+                                                   "peak_source": f"{peak_src} ({'burst' if t_t >= t_h else 'copy'})"})
+            rows[str(M)] = row
+        res[mode_name] = rows
+        if model.device_status() != txs.TXS_OK:
+            raise RuntimeError("device status after the sweep")
+        cache.close()
+        model.close()
+    # appends of dL rows per request against the rebuild of all L rows
+    model = txs.Model(base, weights, txs.LOCAL_GLOBAL)
+    reps = 5
+    cache = txs.KVCache(model, b0.beh_off, beh, capacity_extra=sum(SWEEP_DL) * (reps + 3))
+    rng = np.random.default_rng(20268)
+    app = {}
+    for dL in SWEEP_DL:
+        new = txs.to_device(W.round_bf16(rng.standard_normal((base.n_req * dL, d), dtype=np.float32)), dt)
+        off = np.arange(base.n_req + 1, dtype=np.int32) * dL
+        app[str(dL)] = timed(lambda: cache.append(off, new), reps, flush_l2=False)
+    rebuild = timed(lambda: cache.rebuild(b0.beh_off, beh), 5)
+    res["append_ms"] = app
+    res["rebuild_ms"] = rebuild
+    res["append_note"] = ("append: K/V projection of the new rows into their slots, pooling-state merge, anchor "
+                          "re-projection; rebuild: the same for all L rows of every request (L2 flushed first)")
+    if model.device_status() != txs.TXS_OK:
+        raise RuntimeError("device status after the append sweep")
+    cache.close()
+    model.close()
     return res
 
 
@@ -751,6 +858,7 @@ def main():
         peaks, peak_src = load_peaks()
         fn = {"encoder": lambda: encoder_bench(txs, torch, peaks, peak_src, args.enc_len),
               "deep_wide": lambda: deep_wide_bench(txs, torch),
+              "sweep": lambda: sweep_bench(txs, torch, peaks, peak_src),
               "events": lambda: events_bench(txs, torch)}[args.section]
         print(json.dumps({args.section: fn()}, default=float), flush=True)
         return

@@ -208,8 +208,14 @@ __global__ void __launch_bounds__(256) pool_partial_kernel(const T* __restrict__
 // n = blk * d + c, blk = 2 l + {0: K, 1: V}.  One warp per (column n, group of
 // 8 requests): the weight row is read once per warp (coalesced), the 8 dot
 // products are reduced with shuffles.
-constexpr int kAnchorReqPerWarp = 8;
+constexpr int kAnchorReq = 16;        // anchors staged per CTA (grid.y covers the rest)
+constexpr int kAnchorRowsPerWarp = 1;  // weight rows per warp
 
+// Anchor projections gkv[blk][r][c] = g_r . Wt[n] + b[n] for the 2 nL dkv
+// rows n of the transposed K/V weights (n = blk dkv + c).  One CTA per
+// (32 weight rows, 16 requests): the 16 fp32 anchors are staged in shared
+// memory once, each warp reads its weight row once (16-byte vectors) and
+// dots it with all 16 anchors.
 template <typename T, int NCH>
 __global__ void __launch_bounds__(256) anchor_proj_kernel(const float* __restrict__ g, const T* __restrict__ Wt,
                                                           const float* __restrict__ b, float* __restrict__ gkv,
@@ -217,56 +223,77 @@ __global__ void __launch_bounds__(256) anchor_proj_kernel(const float* __restric
   pdl_launch_dependents();
   pdl_wait();
   constexpr int VEC = Vec16<T>::N;
+  extern __shared__ float sg[];                    // [kAnchorReq][d]
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const long long wid = static_cast<long long>(blockIdx.x) * 8 + warp;
-  const int r_groups = (R + kAnchorReqPerWarp - 1) / kAnchorReqPerWarp;
-  if (wid >= static_cast<long long>(n_total) * r_groups) return;
-  const int n = static_cast<int>(wid / r_groups);
-  const int r0 = static_cast<int>(wid % r_groups) * kAnchorReqPerWarp;
-  float w[NCH][VEC];
+  const int r0 = blockIdx.y * kAnchorReq;
+  const int nr = min(kAnchorReq, R - r0);
+  // all weight loads of this warp's rows, then the anchors (every load issued
+  // before the first use)
+  float w[kAnchorRowsPerWarp][NCH][VEC];
+  const int nw0 = (blockIdx.x * 8 + warp) * kAnchorRowsPerWarp;
 #pragma unroll
-  for (int j = 0; j < NCH; ++j) {
-    const int col = (j * 32 + lane) * VEC;
-    if (col < d) Vec16<T>::load(Wt + static_cast<long long>(n) * d + col, w[j]);
-    else {
+  for (int k = 0; k < kAnchorRowsPerWarp; ++k)
 #pragma unroll
-      for (int q = 0; q < VEC; ++q) w[j][q] = 0.f;
+    for (int j = 0; j < NCH; ++j) {
+      const int col = (j * 32 + lane) * VEC;
+      if (nw0 + k < n_total && col < d) Vec16<T>::load(Wt + static_cast<long long>(nw0 + k) * d + col, w[k][j]);
+      else {
+#pragma unroll
+        for (int q = 0; q < VEC; ++q) w[k][j][q] = 0.f;
+      }
     }
+  constexpr int kStage = kAnchorReq * 512 / 4 / 256;   // float4 per thread (d <= 512)
+  float4 st[kStage];
+  const float4* gsrc = reinterpret_cast<const float4*>(g + static_cast<long long>(r0) * d);
+#pragma unroll
+  for (int u = 0; u < kStage; ++u) {
+    const int i = threadIdx.x + u * 256;
+    if (i * 4 < nr * d) st[u] = __ldg(gsrc + i);
   }
-  float dot[kAnchorReqPerWarp];
 #pragma unroll
-  for (int t = 0; t < kAnchorReqPerWarp; ++t) {
-    dot[t] = 0.f;
-    const int r = r0 + t;
-    if (r < R) {
+  for (int u = 0; u < kStage; ++u) {
+    const int i = threadIdx.x + u * 256;
+    if (i * 4 < nr * d) reinterpret_cast<float4*>(sg)[i] = st[u];
+  }
+  __syncthreads();
 #pragma unroll
-      for (int j = 0; j < NCH; ++j) {
-        const int col = (j * 32 + lane) * VEC;
-        if (col < d) {
-          const float4* gp = reinterpret_cast<const float4*>(g + static_cast<long long>(r) * d + col);
+  for (int k = 0; k < kAnchorRowsPerWarp; ++k) {
+    const int n = nw0 + k;
+    if (n >= n_total) break;
+    float dot[kAnchorReq];
 #pragma unroll
-          for (int q4 = 0; q4 < VEC / 4; ++q4) {
-            const float4 x = __ldg(gp + q4);
-            dot[t] = fmaf(w[j][4 * q4], x.x, dot[t]);
-            dot[t] = fmaf(w[j][4 * q4 + 1], x.y, dot[t]);
-            dot[t] = fmaf(w[j][4 * q4 + 2], x.z, dot[t]);
-            dot[t] = fmaf(w[j][4 * q4 + 3], x.w, dot[t]);
+    for (int t = 0; t < kAnchorReq; ++t) {
+      dot[t] = 0.f;
+      if (t < nr) {
+#pragma unroll
+        for (int j = 0; j < NCH; ++j) {
+          const int col = (j * 32 + lane) * VEC;
+          if (col < d) {
+            const float4* gp = reinterpret_cast<const float4*>(sg + t * d + col);
+#pragma unroll
+            for (int q4 = 0; q4 < VEC / 4; ++q4) {
+              const float4 x = gp[q4];
+              dot[t] = fmaf(w[k][j][4 * q4], x.x, dot[t]);
+              dot[t] = fmaf(w[k][j][4 * q4 + 1], x.y, dot[t]);
+              dot[t] = fmaf(w[k][j][4 * q4 + 2], x.z, dot[t]);
+              dot[t] = fmaf(w[k][j][4 * q4 + 3], x.w, dot[t]);
+            }
           }
         }
       }
     }
-  }
 #pragma unroll
-  for (int t = 0; t < kAnchorReqPerWarp; ++t)
+    for (int t = 0; t < kAnchorReq; ++t)
 #pragma unroll
-    for (int o = 16; o > 0; o >>= 1) dot[t] += __shfl_xor_sync(0xffffffffu, dot[t], o);
-  if (lane < kAnchorReqPerWarp && r0 + lane < R) {
-    float v = 0.f;
+      for (int o = 16; o > 0; o >>= 1) dot[t] += __shfl_xor_sync(0xffffffffu, dot[t], o);
+    if (lane < nr) {
+      float v = 0.f;
 #pragma unroll
-    for (int t = 0; t < kAnchorReqPerWarp; ++t)
-      if (t == lane) v = dot[t];
-    const int blk = n / dkv, c = n - blk * dkv;
-    gkv[(static_cast<long long>(blk) * R + r0 + lane) * dkv + c] = v + __ldg(b + n);
+      for (int t = 0; t < kAnchorReq; ++t)
+        if (t == lane) v = dot[t];
+      const int blk = n / dkv, c = n - blk * dkv;
+      gkv[(static_cast<long long>(blk) * R + r0 + lane) * dkv + c] = v + __ldg(b + n);
+    }
   }
 }
 
@@ -397,14 +424,17 @@ cudaError_t launch_anchor_proj(const float* g, const T* Wt_kv, const float* b_kv
                                int n_layers, cudaStream_t s) {
   constexpr int VEC = Vec16<T>::N;
   const int nch = (d + 32 * VEC - 1) / (32 * VEC);
+  if (R <= 0) return cudaSuccess;
+  if (d % 4 || d > 512) return cudaErrorInvalidValue;
   const int n_total = 2 * n_layers * dkv;
-  const long long warps = static_cast<long long>(n_total) * ((R + kAnchorReqPerWarp - 1) / kAnchorReqPerWarp);
-  const int blocks = static_cast<int>((warps + 7) / 8);
+  const dim3 grid((n_total + 8 * kAnchorRowsPerWarp - 1) / (8 * kAnchorRowsPerWarp),
+                  (R + kAnchorReq - 1) / kAnchorReq);
+  const size_t smem = sizeof(float) * kAnchorReq * d;   // <= 32 KB for d <= 512
   prof_begin(KC_GLOBAL_KV, s);
   cudaError_t err;
-  if (nch == 1) err = launch_pdl(anchor_proj_kernel<T, 1>, dim3(blocks), dim3(256), 0, s, g, Wt_kv, b_kv, gkv, R, d, dkv, n_total);
-  else if (nch == 2) err = launch_pdl(anchor_proj_kernel<T, 2>, dim3(blocks), dim3(256), 0, s, g, Wt_kv, b_kv, gkv, R, d, dkv, n_total);
-  else if (nch <= 4) err = launch_pdl(anchor_proj_kernel<T, 4>, dim3(blocks), dim3(256), 0, s, g, Wt_kv, b_kv, gkv, R, d, dkv, n_total);
+  if (nch == 1) err = launch_pdl(anchor_proj_kernel<T, 1>, grid, dim3(256), smem, s, g, Wt_kv, b_kv, gkv, R, d, dkv, n_total);
+  else if (nch == 2) err = launch_pdl(anchor_proj_kernel<T, 2>, grid, dim3(256), smem, s, g, Wt_kv, b_kv, gkv, R, d, dkv, n_total);
+  else if (nch <= 4) err = launch_pdl(anchor_proj_kernel<T, 4>, grid, dim3(256), smem, s, g, Wt_kv, b_kv, gkv, R, d, dkv, n_total);
   else return cudaErrorInvalidValue;
   prof_end(KC_GLOBAL_KV, s);
   return err;
