@@ -24,6 +24,14 @@
  *   create/build time and free it in the matching destroy call.
  * - Calls on the same handle must be ordered by the caller (same stream, or
  *   events); the library does not lock.
+ * - CUDA graphs: txs_rebuild_kv_cache, txs_append_behavior,
+ *   txs_score_candidates, txs_rank_candidates and txs_encode_append can be
+ *   captured (stream capture) when their host offset
+ *   arrays hold at most 8000 ints in all per call (they travel as kernel
+ *   parameters).  A replay repeats the captured device work, the uploads of
+ *   the offsets and lengths computed at capture included, but not the host
+ *   bookkeeping: host-side lengths (txs_cache_lengths, capacity checks) stay
+ *   those of the last direct call.
  */
 #ifndef TXS_H
 #define TXS_H

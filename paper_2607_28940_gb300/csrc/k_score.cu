@@ -147,6 +147,29 @@ __global__ void __launch_bounds__(1024) rank_kernel(const __grid_constant__ Rank
     for (int t = M + threadIdx.x; t < a.top_k; t += blockDim.x) out[static_cast<long long>(r) * a.top_k + t] = -1;
 }
 
+// Small host int arrays reach the device as kernel parameters (copied by
+// value at launch: no copy-engine transfer, nothing left behind in host
+// memory, so the call can be captured into a CUDA graph).  Two segments, a
+// then b, in one launch; it waits for the preceding kernel first, which may
+// still be reading the old values.
+template <int N>
+struct UploadArgs {
+  int* dst_a;
+  int* dst_b;
+  int n_a, n_b;
+  int v[N];
+};
+
+template <int N>
+__global__ void __launch_bounds__(256) upload_kernel(const __grid_constant__ UploadArgs<N> a) {
+  pdl_launch_dependents();
+  pdl_wait();
+  for (int i = blockIdx.x * 256 + threadIdx.x; i < a.n_a + a.n_b; i += gridDim.x * 256) {
+    if (i < a.n_a) a.dst_a[i] = a.v[i];
+    else a.dst_b[i - a.n_a] = a.v[i];
+  }
+}
+
 // Deep & Wide head input: row i of Z2 = [z_i, x_i[dw_in:]] for the candidate
 // rows (z: the decoder output, x: the raw candidate token).  One warp per row,
 // 16-byte vectors.
@@ -223,6 +246,30 @@ __global__ void __launch_bounds__(256) dw_head_kernel(const T* __restrict__ Hd, 
 }
 
 }  // namespace
+
+template <int N>
+static cudaError_t upload_n(int* dst_a, const int* src_a, int n_a, int* dst_b, const int* src_b, int n_b,
+                            cudaStream_t s) {
+  UploadArgs<N> a;
+  a.dst_a = dst_a;
+  a.dst_b = dst_b;
+  a.n_a = n_a;
+  a.n_b = n_b;
+  for (int i = 0; i < n_a; ++i) a.v[i] = src_a[i];
+  for (int i = 0; i < n_b; ++i) a.v[n_a + i] = src_b[i];
+  const int blocks = (n_a + n_b + 255) / 256;
+  return launch_pdl(upload_kernel<N>, dim3(blocks > 0 ? blocks : 1), dim3(256), 0, s, a);
+}
+
+const int kUploadParamInts = 8000;
+
+cudaError_t launch_upload_ints(int* dst_a, const int* src_a, int n_a, int* dst_b, const int* src_b, int n_b,
+                               cudaStream_t s) {
+  if (n_a < 0 || n_b < 0) return cudaErrorInvalidValue;
+  if (n_a + n_b > kUploadParamInts) return cudaErrorNotSupported;
+  if (n_a + n_b <= 1000) return upload_n<1000>(dst_a, src_a, n_a, dst_b, src_b, n_b, s);
+  return upload_n<8000>(dst_a, src_a, n_a, dst_b, src_b, n_b, s);
+}
 
 template <typename T>
 cudaError_t launch_dw_gather(const T* Z, const T* cand, T* Z2, int n_cand, int d, int dw_in, cudaStream_t s) {

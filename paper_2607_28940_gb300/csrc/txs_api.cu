@@ -375,21 +375,32 @@ cudaError_t stage_upload(txs_kv_cache* c, int* dst, const int* src, int n, cudaS
   return cudaEventRecord(*ev, s);
 }
 
+// Upload [in_off (R+1) | dst0 (R)] and the lengths after the call (R): by
+// kernel parameters when they fit (capturable), else through pinned memory.
+cudaError_t upload_call(txs_kv_cache* c, const std::vector<int>& up, const std::vector<int>& len, cudaStream_t s) {
+  const int n_req = c->n_req;
+  cudaError_t err = launch_upload_ints(c->d_in_off, up.data(), 2 * n_req + 1, c->d_len, len.data(), n_req, s);
+  if (err != cudaErrorNotSupported) return err;
+  if ((err = stage_upload(c, c->d_in_off, up.data(), 2 * n_req + 1, s)) != cudaSuccess) return err;
+  return stage_upload(c, c->d_len, len.data(), n_req, s);
+}
+
 template <typename T>
 txs_status project_rows(txs_model* m, txs_kv_cache* c, int n_req, const int32_t* in_off, const void* rows,
                         bool append, cudaStream_t s) {
   const txs_config& cf = m->cfg;
   const int d = cf.d_model, nL = cf.n_layers;
   const long long total = in_off[n_req];
-  // [in_off (R+1) | dst0 (R)] in one upload
-  std::vector<int> up(2 * n_req + 1);
+  // [in_off (R+1) | dst0 (R)] and the new lengths in one upload
+  std::vector<int> up(2 * n_req + 1), len(n_req);
   int max_rows = 0;
   for (int r = 0; r <= n_req; ++r) up[r] = in_off[r];
   for (int r = 0; r < n_req; ++r) {
     up[n_req + 1 + r] = c->h_off[r] + (append ? c->h_len[r] : 0);
+    len[r] = (append ? c->h_len[r] : 0) + in_off[r + 1] - in_off[r];
     max_rows = std::max(max_rows, in_off[r + 1] - in_off[r]);
   }
-  TXS_CK(stage_upload(c, c->d_in_off, up.data(), 2 * n_req + 1, s));
+  TXS_CK(upload_call(c, up, len, s));
   if (total > 0) {
     const int dkv = c->dkv;
     EpiArgs e = epi_base(EPI_KV, total, 2 * nL * dkv, d);
@@ -922,8 +933,6 @@ TXS_API txs_status txs_rebuild_kv_cache(txs_model* m, txs_kv_cache* c, int32_t n
                                            : project_rows<float>(m, c, n_req, beh_offsets, beh_enc, false, s);
   if (st != TXS_OK) return st;
   for (int r = 0; r < n_req; ++r) c->h_len[r] = beh_offsets[r + 1] - beh_offsets[r];
-  cudaError_t err = stage_upload(c, c->d_len, c->h_len.data(), n_req, s);
-  if (err != cudaSuccess) return fail_cuda("upload lengths", err);
   return TXS_OK;
 }
 
@@ -942,8 +951,6 @@ TXS_API txs_status txs_append_behavior(txs_model* m, txs_kv_cache* c, int32_t n_
                                            : project_rows<float>(m, c, n_req, new_offsets, new_enc, true, s);
   if (st != TXS_OK) return st;
   for (int r = 0; r < n_req; ++r) c->h_len[r] += new_offsets[r + 1] - new_offsets[r];
-  cudaError_t err = stage_upload(c, c->d_len, c->h_len.data(), n_req, s);
-  if (err != cudaSuccess) return fail_cuda("upload lengths", err);
   return TXS_OK;
 }
 

@@ -247,7 +247,12 @@ txs_status encode_impl(txs_encoder* m, txs_enc_state* st, const int32_t* in_off,
   }
   up[3 * R + 1] = tiles;
   if (n == 0) return TXS_OK;
-  ENC_CK(enc_upload(st, st->d_call, up.data(), 3 * R + 2, s));
+  {
+    // kernel parameters when they fit (capturable), else the pinned ring
+    cudaError_t err = launch_upload_ints(st->d_call, up.data(), 3 * R + 2, nullptr, nullptr, 0, s);
+    if (err == cudaErrorNotSupported) err = enc_upload(st, st->d_call, up.data(), 3 * R + 2, s);
+    if (err != cudaSuccess) return enc_fail("upload", err);
+  }
   const int* d_in_off = st->d_call;
   const int* d_dst0 = st->d_call + R + 1;
   const int* d_tile_off = st->d_call + 2 * R + 1;

@@ -221,6 +221,12 @@ cudaError_t launch_fold_head(const T* W_dec, const T* b_dec, const T* Q_dec, flo
 cudaError_t launch_hash(const void* p, long long bytes, uint64_t salt, unsigned long long* out, cudaStream_t s);
 
 extern const int kMaxReqParam;
+// dst_a[0..n_a) = src_a, dst_b[0..n_b) = src_b (host arrays) by one kernel
+// whose parameters carry the values; cudaErrorNotSupported above
+// kUploadParamInts ints in all (the caller then copies through pinned memory).
+extern const int kUploadParamInts;
+cudaError_t launch_upload_ints(int* dst_a, const int* src_a, int n_a, int* dst_b, const int* src_b, int n_b,
+                               cudaStream_t s);
 template <typename T>
 cudaError_t launch_pack(int n_req, const int* cand_off_host, int S, int d, int na, const T* cand, const T* ctx, T* X,
                         int* row_req, int* cand_off_dev, const float* weff_x, const float* cdec, float* xlog,
