@@ -179,6 +179,19 @@ __device__ __forceinline__ void tmem_ld128(uint32_t taddr, float* v) {
   for (int i = 0; i < 128; ++i) v[i] = __uint_as_float(r[i]);
 }
 
+// 64 consecutive columns of this warp's 32 lanes: one load, one wait.
+__device__ __forceinline__ void tmem_ld64(uint32_t taddr, float* v) {
+  uint32_t r[64];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x64.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,%32,%33,%34,%35,%36,%37,%38,%39,%40,%41,%42,%43,%44,%45,%46,%47,%48,%49,%50,%51,%52,%53,%54,%55,%56,%57,%58,%59,%60,%61,%62,%63}, [%64];\n\t"
+      "tcgen05.wait::ld.sync.aligned;"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31]), "=r"(r[32]), "=r"(r[33]), "=r"(r[34]), "=r"(r[35]), "=r"(r[36]), "=r"(r[37]), "=r"(r[38]), "=r"(r[39]), "=r"(r[40]), "=r"(r[41]), "=r"(r[42]), "=r"(r[43]), "=r"(r[44]), "=r"(r[45]), "=r"(r[46]), "=r"(r[47]), "=r"(r[48]), "=r"(r[49]), "=r"(r[50]), "=r"(r[51]), "=r"(r[52]), "=r"(r[53]), "=r"(r[54]), "=r"(r[55]), "=r"(r[56]), "=r"(r[57]), "=r"(r[58]), "=r"(r[59]), "=r"(r[60]), "=r"(r[61]), "=r"(r[62]), "=r"(r[63])
+      : "r"(taddr)
+      : "memory");
+#pragma unroll
+  for (int i = 0; i < 64; ++i) v[i] = __uint_as_float(r[i]);
+}
+
 // 2^x on the special-function unit (PTX ex2.approx, flush-to-zero).
 __device__ __forceinline__ float ex2(float x) {
   float y;
@@ -485,6 +498,306 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       }
     }
   }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, Sh::TMEM_COLS);
+  }
+  if (threadIdx.x == 0 && *abort_flag) latch_status(a.status, TXS_ERR_DEVICE_TIMEOUT);
+}
+
+// ------------------------------------------------------------------ two query tiles per CTA
+
+// FULL cross-attention with two 128-row query tiles (A, B) of one request and
+// head per CTA.  Both tiles use each staged K/V tile, and two softmax warp
+// groups (warps 2-5: tile A, warps 6-9: tile B) take turns with the tensor
+// core: the MMA warp issues S_A(j), S_B(j), then, as each group hands over
+// its P(j), that group's P V(j) immediately followed by its S(j+1), so one
+// group computes exponentials while the other's products run.
+// TMEM per tile: S (128 columns fp32; P, bf16, is written over its first 64
+// columns once S has been read: the next S of the tile is issued after the P V
+// that reads P, and one thread's MMAs run in issue order), O (d_h columns),
+// Q (d_h / 2 columns).  A CTA whose second tile would be empty (the last of
+// an odd number) runs the first alone.  The softmax reads a score row in two
+// halves of 64 keys (max over both, then exponentials half by half) to stay
+// within the register file at 320 threads.  Online softmax with the
+// stale-maximum rule of fa_full_kernel.
+constexpr int PAIR_THREADS = 320;
+
+template <int DH>
+struct PairShape {
+  static constexpr int ROW_BYTES = DH * 2;
+  static constexpr uint32_t SW = DH == 64 ? 2u : 4u;
+  static constexpr int ATOM = 8 * ROW_BYTES;
+  static constexpr int KV_BYTES = BKV * ROW_BYTES;
+  static constexpr int SMEM = 2 * STG * KV_BYTES + 1024 + 256;
+  static constexpr uint32_t T_S = 0, T_O = 256, T_Q = 256 + 2 * 64;
+  static constexpr int TMEM_COLS = 512;
+  static_assert(T_Q + 2 * (DH / 2) <= TMEM_COLS, "TMEM columns");
+};
+
+template <int DH>
+__global__ void __launch_bounds__(PAIR_THREADS, 1)
+    fa_pair_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV, const FaArgs a) {
+  using Sh = PairShape<DH>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint8_t* sK = smem;
+  uint8_t* sV = sK + STG * Sh::KV_BYTES;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(sV + STG * Sh::KV_BYTES);
+  uint64_t* kv_full = bars;
+  uint64_t* kv_empty = kv_full + STG;
+  uint64_t* s_full = kv_empty + STG;     // [2] S_t(j) in TMEM (P V_t(j-1) complete too)
+  uint64_t* p_full = s_full + 2;         // [2] P_t(j) written
+  uint64_t* o_done = p_full + 2;         // [2] the last P V_t complete
+  uint64_t* q_ready = o_done + 2;
+  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(q_ready + 1);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_holder + 1);
+
+  pdl_launch_dependents();
+  pdl_wait();
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int qp = blockIdx.x, r = blockIdx.y, h = blockIdx.z;
+  const int c0 = a.cand_off[r];
+  const int M = a.cand_off[r + 1] - c0;
+  const int n_q = M + a.S;
+  if (qp * 2 * BQ >= n_q) return;                   // uniform: no tile here
+  const int n_t = (qp * 2 + 1) * BQ < n_q ? 2 : 1;  // tiles of this CTA (uniform)
+  const int len = a.kv_len[r];
+  const int kv0 = a.kv_off[r];
+  const int nkv = (len + BKV - 1) / BKV;
+  if (nkv <= 0) {
+    if (threadIdx.x == 0) latch_status(a.status, TXS_ERR_BOUNDS);
+    return;
+  }
+
+  if (threadIdx.x == 0) {
+    for (int st = 0; st < STG; ++st) {
+      mbar_init(kv_full + st, 1);
+      mbar_init(kv_empty + st, 1);
+    }
+    for (int t = 0; t < 2; ++t) {
+      mbar_init(s_full + t, 1);
+      mbar_init(p_full + t, 4);
+      mbar_init(o_done + t, 1);
+    }
+    mbar_init(q_ready, 4 * n_t);
+    *abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == 1) tmem_alloc(tmem_holder, Sh::TMEM_COLS);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_holder;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmK)) : "memory");
+      asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmV)) : "memory");
+      int issued = 0;
+      for (int j = 0; j < nkv; ++j) {
+        const int st = j % STG;
+        if (!mbar_wait(kv_empty + st, ((j / STG) & 1) ^ 1, abort_flag)) break;
+        mbar_expect_tx(kv_full + st, 2 * Sh::KV_BYTES);
+        tma_load_2d(sK + st * Sh::KV_BYTES, &tmK, kv_full + st, (h / a.group) * DH, kv0 + j * BKV);
+        tma_load_2d(sV + st * Sh::KV_BYTES, &tmV, kv_full + st, (h / a.group) * DH, kv0 + j * BKV);
+        issued = j + 1;
+      }
+      if (*abort_flag)
+        for (int k = issued > STG ? issued - STG : 0; k < issued; ++k)
+          mbar_wait_plain(kv_full + k % STG, (k / STG) & 1);
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      constexpr uint32_t id_s = idesc_bf16(BQ, BKV, false);
+      constexpr uint32_t id_pv = idesc_bf16(BQ, DH, true);
+      auto qk = [&](int t, int j) {
+        const uint32_t k_addr = smem_u32(sK + (j % STG) * Sh::KV_BYTES);
+#pragma unroll
+        for (int k = 0; k < DH / 16; ++k) {
+          const uint64_t kd = sdesc(k_addr + k * 32, 16, Sh::ATOM, Sh::SW);
+          mma_bf16_ts(tmem + Sh::T_S + BKV * t, tmem + Sh::T_Q + (DH / 2) * t + 8 * k, kd, id_s, k > 0 ? 1u : 0u);
+        }
+        mma_commit(s_full + t);
+      };
+      auto pv = [&](int t, int j) {
+        const uint32_t v_addr = smem_u32(sV + (j % STG) * Sh::KV_BYTES);
+#pragma unroll
+        for (int k = 0; k < BKV / 16; ++k) {
+          const uint64_t vd = sdesc(v_addr + k * 16 * Sh::ROW_BYTES, Sh::ATOM, Sh::ATOM, Sh::SW);
+          mma_bf16_ts(tmem + Sh::T_O + 64 * t, tmem + Sh::T_S + BKV * t + 8 * k, vd, id_pv,
+                      (j > 0 || k > 0) ? 1u : 0u);
+        }
+      };
+      bool ok = mbar_wait(q_ready, 0, abort_flag);
+      ok = ok && mbar_wait(kv_full, 0, abort_flag);
+      if (ok) {
+        tc_fence_after();
+        for (int t = 0; t < n_t; ++t) qk(t, 0);
+      }
+      for (int j = 0; j < nkv && ok; ++j) {
+        const bool more = j + 1 < nkv;
+        for (int t = 0; t < n_t && ok; ++t) {
+          if (!mbar_wait(p_full + t, j & 1, abort_flag)) { ok = false; break; }
+          tc_fence_after();
+          pv(t, j);
+          if (t == n_t - 1) mma_commit(kv_empty + j % STG);   // every P V of key tile j issued
+          if (more) {
+            if (t == 0 && !mbar_wait(kv_full + (j + 1) % STG, ((j + 1) / STG) & 1, abort_flag)) { ok = false; break; }
+            tc_fence_after();
+            qk(t, j + 1);
+          } else {
+            mma_commit(o_done + t);
+          }
+        }
+      }
+    }
+  } else {
+    // ---------------- softmax: warps 2-5 tile A, warps 6-9 tile B; one query row per thread
+    const int t = (warp - 2) >> 2;
+    if (t >= n_t) goto done;                  // no second tile in this CTA (uniform per group)
+    {
+    const int qw = warp & 3;                  // TMEM lane quarter
+    const int m = qw * 32 + lane;
+    const int j_q = (qp * 2 + t) * BQ + m;     // query index within the request
+    const bool valid = j_q < n_q;
+    const long long grow = j_q < M ? static_cast<long long>(c0) + j_q
+                                   : a.n_cand + static_cast<long long>(r) * a.S + (j_q - M);
+    const uint32_t lane_off = static_cast<uint32_t>(qw * 32) << 16;
+    {
+      uint32_t qv[DH / 2];
+      const uint4* src = reinterpret_cast<const uint4*>(a.q + (valid ? grow : 0) * a.d + h * DH);
+#pragma unroll
+      for (int c = 0; c < DH / 8; ++c) {
+        const uint4 v = valid ? src[c] : make_uint4(0, 0, 0, 0);
+        qv[4 * c] = v.x; qv[4 * c + 1] = v.y; qv[4 * c + 2] = v.z; qv[4 * c + 3] = v.w;
+      }
+#pragma unroll
+      for (int c = 0; c < DH / 2; c += 16) tmem_st16(tmem + Sh::T_Q + (DH / 2) * t + c + lane_off, qv + c);
+      tmem_wait_st();
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(q_ready);
+    }
+    const uint32_t t_s = tmem + Sh::T_S + BKV * t + lane_off;
+    const uint32_t t_o = tmem + Sh::T_O + 64 * t + lane_off;
+    float m_run = -INFINITY, l_run = 0.f;
+    bool ok = true;
+    for (int j = 0; j < nkv && ok; ++j) {
+      ok = mbar_wait(s_full + t, j & 1, abort_flag);
+      ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
+      if (!ok) break;
+      tc_fence_after();
+      const int kbase = j * BKV;
+      const bool ragged = kbase + BKV > len;     // uniform
+      // row max over both halves of 64 keys (a half at a time keeps the
+      // register count within the file at 320 threads)
+      float mx = -INFINITY;
+#pragma unroll
+      for (int half = 0; half < 2; ++half) {
+        float sv[64];
+        tmem_ld64(t_s + 64 * half, sv);
+        if (ragged) {
+#pragma unroll
+          for (int i = 0; i < 64; ++i)
+            if (kbase + 64 * half + i >= len) sv[i] = -INFINITY;
+        }
+        float mx8[8];
+#pragma unroll
+        for (int i = 0; i < 8; ++i) mx8[i] = sv[i];
+#pragma unroll
+        for (int i = 8; i < 64; ++i) mx8[i & 7] = fmaxf(mx8[i & 7], sv[i]);
+#pragma unroll
+        for (int w = 4; w >= 1; w >>= 1)
+#pragma unroll
+          for (int i = 0; i < w; ++i) mx8[i] = fmaxf(mx8[i], mx8[i + w]);
+        mx = fmaxf(mx, mx8[0]);
+      }
+      const float m_tile = mx * a.scale_log2;
+      if (__any_sync(0xffffffffu, m_tile > m_run + kRescaleLog2)) {
+        const float m_new = fmaxf(m_run, m_tile);
+        const float alpha = ex2(m_run - m_new);   // 0 on the first tile
+        if (j >= 1) {                              // O holds P V up to j - 1 (complete: S_t(j) is)
+#pragma unroll
+          for (int cc = 0; cc < DH; cc += 32) {
+            float ov[32];
+            tmem_ld32(t_o + cc, ov);
+#pragma unroll
+            for (int i = 0; i < 32; ++i) ov[i] *= alpha;
+            tmem_st32(t_o + cc, ov);
+          }
+        }
+        l_run *= alpha;
+        m_run = m_new;
+      }
+      // P half by half over the first 64 columns of S: half 0 (keys 0-63)
+      // lands on columns 0-31, read already; half 1 is read before its P
+      // lands on columns 32-63
+      float ps8[8];
+#pragma unroll
+      for (int i = 0; i < 8; ++i) ps8[i] = 0.f;
+#pragma unroll
+      for (int half = 0; half < 2; ++half) {
+        float sv[64];
+        tmem_ld64(t_s + 64 * half, sv);
+        if (ragged) {
+#pragma unroll
+          for (int i = 0; i < 64; ++i)
+            if (kbase + 64 * half + i >= len) sv[i] = -INFINITY;
+        }
+#pragma unroll
+        for (int c32 = 0; c32 < 64; c32 += 32) {
+          uint32_t pk[16];
+#pragma unroll
+          for (int i = 0; i < 32; i += 2) {
+            const float p0 = ex2(fmaf(sv[c32 + i], a.scale_log2, -m_run));
+            const float p1 = ex2(fmaf(sv[c32 + i + 1], a.scale_log2, -m_run));
+            ps8[i & 7] += p0;
+            ps8[(i + 1) & 7] += p1;
+            __nv_bfloat162 h2 = __floats2bfloat162_rn(p0, p1);
+            pk[i / 2] = *reinterpret_cast<uint32_t*>(&h2);
+          }
+          tmem_st16(t_s + 32 * half + c32 / 2, pk);
+        }
+      }
+      tmem_wait_st();
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(p_full + t);
+#pragma unroll
+      for (int w = 4; w >= 1; w >>= 1)
+#pragma unroll
+        for (int i = 0; i < w; ++i) ps8[i] += ps8[i + w];
+      l_run += ps8[0];
+    }
+    if (ok) {
+      ok = mbar_wait(o_done + t, 0, abort_flag);
+      ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
+    }
+    if (ok) {
+      tc_fence_after();
+      const float inv = 1.f / l_run;
+      __nv_bfloat16* dst = a.out + grow * a.d + h * DH;
+#pragma unroll
+      for (int cc = 0; cc < DH; cc += 32) {
+        float ov[32];
+        tmem_ld32(t_o + cc, ov);
+        if (valid) {
+#pragma unroll
+          for (int c = 0; c < 32; c += 8) {
+            float tv[8];
+#pragma unroll
+            for (int i = 0; i < 8; ++i) tv[i] = ov[c + i] * inv;
+            Vec16<__nv_bfloat16>::store(dst + cc + c, tv);
+          }
+        }
+      }
+    }
+    }
+  }
+done:
   tc_fence_before();
   __syncthreads();
   if (warp == 1) {
@@ -880,6 +1193,22 @@ static cudaError_t launch_dh(const FaArgs& a, const void* Kc, const void* Vc, lo
 }
 
 template <int DH>
+static cudaError_t launch_pair_dh(const FaArgs& a, const void* Kc, const void* Vc, long long cap_total, int n_req,
+                                  int max_q_pairs, int H, int dkv, cudaStream_t s) {
+  using Sh = PairShape<DH>;
+  static bool attr = false;
+  if (!attr) {
+    cudaError_t e = cudaFuncSetAttribute(fa_pair_kernel<DH>, cudaFuncAttributeMaxDynamicSharedMemorySize, Sh::SMEM);
+    if (e != cudaSuccess) return e;
+    attr = true;
+  }
+  CUtensorMap tk, tv;
+  if (!make_kv_map<DH>(&tk, Kc, cap_total, dkv) || !make_kv_map<DH>(&tv, Vc, cap_total, dkv))
+    return cudaErrorInvalidValue;
+  return launch_pdl(fa_pair_kernel<DH>, dim3(max_q_pairs, n_req, H), dim3(PAIR_THREADS), Sh::SMEM, s, tk, tv, a);
+}
+
+template <int DH>
 static cudaError_t launch_enc_dh(const EncFaArgs& a, const void* K, const void* V, long long cap_total, int n_tiles,
                                  int H, cudaStream_t s) {
   static bool attr = false;
@@ -937,8 +1266,15 @@ cudaError_t launch_fa_full(const __nv_bfloat16* q, __nv_bfloat16* out, const __n
                1.4426950408889634f / sqrtf(static_cast<float>(dh)), status};
   const int tiles = (max_q + fa::BQ - 1) / fa::BQ;
   prof_begin(KC_ATTN_CROSS, s);
-  cudaError_t err = dh == 64 ? fa::launch_dh<64>(a, Kc, Vc, cap_total, n_req, tiles, H, Hkv * dh, s)
-                             : fa::launch_dh<32>(a, Kc, Vc, cap_total, n_req, tiles, H, Hkv * dh, s);
+  cudaError_t err;
+  if (tiles >= 2) {   // two query tiles per CTA share each K/V tile
+    const int pairs = (tiles + 1) / 2;
+    err = dh == 64 ? fa::launch_pair_dh<64>(a, Kc, Vc, cap_total, n_req, pairs, H, Hkv * dh, s)
+                   : fa::launch_pair_dh<32>(a, Kc, Vc, cap_total, n_req, pairs, H, Hkv * dh, s);
+  } else {
+    err = dh == 64 ? fa::launch_dh<64>(a, Kc, Vc, cap_total, n_req, tiles, H, Hkv * dh, s)
+                   : fa::launch_dh<32>(a, Kc, Vc, cap_total, n_req, tiles, H, Hkv * dh, s);
+  }
   prof_end(KC_ATTN_CROSS, s);
   return err;
 }
