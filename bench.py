@@ -61,7 +61,7 @@ def parse():
     p.add_argument("--workload", default=HEADLINE, choices=sorted(W.WORKLOADS))
     p.add_argument("--mode", default="local_global", choices=["local_global", "full"])
     p.add_argument("--no-extras", action="store_true", help="skip latency sweep, e2e and CPU baseline")
-    p.add_argument("--section", choices=["encoder", "deep_wide", "events", "sweep"],
+    p.add_argument("--section", choices=["encoder", "deep_wide", "events", "sweep", "latency"],
                    help="run only this extra section (one JSON object) and exit")
     p.add_argument("--enc-len", type=int, default=0,
                    help="tokens per user of the encoder section (default: the workload's)")
@@ -859,6 +859,7 @@ def main():
         fn = {"encoder": lambda: encoder_bench(txs, torch, peaks, peak_src, args.enc_len),
               "deep_wide": lambda: deep_wide_bench(txs, torch),
               "sweep": lambda: sweep_bench(txs, torch, peaks, peak_src),
+              "latency": lambda: latency_sweep(txs, torch),
               "events": lambda: events_bench(txs, torch)}[args.section]
         print(json.dumps({args.section: fn()}, default=float), flush=True)
         return

@@ -1267,7 +1267,17 @@ cudaError_t launch_fa_full(const __nv_bfloat16* q, __nv_bfloat16* out, const __n
   const int tiles = (max_q + fa::BQ - 1) / fa::BQ;
   prof_begin(KC_ATTN_CROSS, s);
   cudaError_t err;
-  if (tiles >= 2) {   // two query tiles per CTA share each K/V tile
+  // two query tiles per CTA share each K/V tile, when the pairs still fill
+  // the GPU (a single request would otherwise leave most SMs idle)
+  static int sms = 0;
+  if (!sms) {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || sms <= 0)
+      sms = 152;
+  }
+  const long long pair_ctas = static_cast<long long>((tiles + 1) / 2) * n_req * H;
+  if (tiles >= 2 && pair_ctas >= 2LL * sms) {
     const int pairs = (tiles + 1) / 2;
     err = dh == 64 ? fa::launch_pair_dh<64>(a, Kc, Vc, cap_total, n_req, pairs, H, Hkv * dh, s)
                    : fa::launch_pair_dh<32>(a, Kc, Vc, cap_total, n_req, pairs, H, Hkv * dh, s);

@@ -258,7 +258,10 @@ static cudaError_t upload_n(int* dst_a, const int* src_a, int n_a, int* dst_b, c
   for (int i = 0; i < n_a; ++i) a.v[i] = src_a[i];
   for (int i = 0; i < n_b; ++i) a.v[n_a + i] = src_b[i];
   const int blocks = (n_a + n_b + 255) / 256;
-  return launch_pdl(upload_kernel<N>, dim3(blocks > 0 ? blocks : 1), dim3(256), 0, s, a);
+  prof_begin(KC_MISC, s);
+  const cudaError_t err = launch_pdl(upload_kernel<N>, dim3(blocks > 0 ? blocks : 1), dim3(256), 0, s, a);
+  prof_end(KC_MISC, s);
+  return err;
 }
 
 const int kUploadParamInts = 8000;
