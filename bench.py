@@ -393,10 +393,12 @@ def latency_sweep(txs, torch):
     base = W.WORKLOADS[LAT_WORKLOAD]
     weights = W.weights(base)
     res = {"model": f"{LAT_WORKLOAD} layers/width (d={base.d_model}, {base.n_layers} layers), R=1, M={LAT_M}",
-           "unit": "ms", "note": "CUDA events, weights L2-warm as in steady serving"}
+           "unit": "ms", "note": "CUDA events, weights L2-warm as in steady serving; *_graph_replay: the same "
+                                 "score + rank captured into a CUDA graph once per length and replayed"}
+    side = torch.cuda.Stream()
     for mode_name, mode in (("local_global", txs.LOCAL_GLOBAL), ("full", txs.FULL)):
         model = txs.Model(base, weights, mode)
-        p50 = {}
+        p50, p50_graph = {}, {}
         for L in LAT_LENGTHS:
             wl = W.with_sizes(base, n_req=1, L=L, M=LAT_M, dL=0)
             b = W.batch(wl)
@@ -408,20 +410,34 @@ def latency_sweep(txs, torch):
             lg = torch.empty((LAT_M, wl.n_actions), dtype=torch.float32, device="cuda")
             pr = torch.empty_like(lg)
             rk = torch.empty(LAT_M, dtype=torch.int32, device="cuda")
-            times = []
-            for i in range(40):
-                e0 = torch.cuda.Event(enable_timing=True)
-                e1 = torch.cuda.Event(enable_timing=True)
-                e0.record()
+            def call():
                 txs.score(model, cache, b.cand_off, cand, ctx, workspace=ws, out_logits=lg, out_probs=pr)
                 txs.rank(b.cand_off, pr, wl.n_actions, 0, 0, out=rk)
-                e1.record()
-                e1.synchronize()
-                if i >= 10:
-                    times.append(e0.elapsed_time(e1))
-            p50[str(L)] = statistics.median(times)
+
+            def p50_of(fn):
+                times = []
+                with torch.cuda.stream(side):
+                    for i in range(40):
+                        e0 = torch.cuda.Event(enable_timing=True)
+                        e1 = torch.cuda.Event(enable_timing=True)
+                        e0.record()
+                        fn()
+                        e1.record()
+                        e1.synchronize()
+                        if i >= 10:
+                            times.append(e0.elapsed_time(e1))
+                return statistics.median(times)
+            p50[str(L)] = p50_of(call)
+            # the same call captured once into a CUDA graph and replayed (a
+            # server keeps one graph per slate shape)
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g, stream=side):
+                call()
+            p50_graph[str(L)] = p50_of(g.replay)
+            del g
             cache.close()
         res[mode_name] = p50
+        res[f"{mode_name}_graph_replay"] = p50_graph
         res[f"{mode_name}_ratio_16384_over_1024"] = p50["16384"] / p50["1024"]
         model.close()
     return res
