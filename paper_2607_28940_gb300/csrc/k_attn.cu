@@ -213,9 +213,9 @@ __global__ void __launch_bounds__(256) cross_lg_kernel(const T* __restrict__ q_i
   pdl_wait();
   extern __shared__ __align__(16) uint8_t smem_lg[];
   const int d = a.d, dkv = a.dkv;
-  T* sK = reinterpret_cast<T*>(smem_lg);                      // [kWin][dkv]
-  T* sV = sK + kWin * dkv;                                    // [kWin][dkv]
-  float* sKg = reinterpret_cast<float*>(sV + kWin * dkv);     // [dkv]
+  float* sK = reinterpret_cast<float*>(smem_lg);              // [kWin][dkv], fp32
+  float* sV = sK + kWin * dkv;                                // [kWin][dkv]
+  float* sKg = sV + kWin * dkv;                               // [dkv]
   float* sVg = sKg + dkv;                                     // [dkv]
   const int r = blockIdx.y;
   const int c0 = __ldg(a.cand_off + r);
@@ -232,8 +232,15 @@ __global__ void __launch_bounds__(256) cross_lg_kernel(const T* __restrict__ q_i
     const int per_row = dkv / VE;
     for (int i = threadIdx.x; i < W * per_row; i += blockDim.x) {
       const int t = i / per_row, c = (i - t * per_row) * VE;
-      *reinterpret_cast<uint4*>(sK + t * dkv + c) = *reinterpret_cast<const uint4*>(Kc + (base + t) * dkv + c);
-      *reinterpret_cast<uint4*>(sV + t * dkv + c) = *reinterpret_cast<const uint4*>(Vc + (base + t) * dkv + c);
+      // converted once here: every lane (query row) reads every element
+      float kf[VE], vf[VE];
+      Vec16<T>::load(Kc + (base + t) * dkv + c, kf);
+      Vec16<T>::load(Vc + (base + t) * dkv + c, vf);
+#pragma unroll
+      for (int e = 0; e < VE; e += 4) {
+        *reinterpret_cast<float4*>(sK + t * dkv + c + e) = make_float4(kf[e], kf[e + 1], kf[e + 2], kf[e + 3]);
+        *reinterpret_cast<float4*>(sV + t * dkv + c + e) = make_float4(vf[e], vf[e + 1], vf[e + 2], vf[e + 3]);
+      }
     }
     for (int i = threadIdx.x; i < dkv; i += blockDim.x) {
       sKg[i] = __ldg(a.Kg + static_cast<long long>(r) * dkv + i);
@@ -267,11 +274,12 @@ __global__ void __launch_bounds__(256) cross_lg_kernel(const T* __restrict__ q_i
       if (t < W) {
         dot = 0.f;
 #pragma unroll
-        for (int c = 0; c < DH; c += Vec16<T>::N) {
-          float k[Vec16<T>::N];
-          Vec16<T>::load(sK + t * dkv + ck + c, k);
-#pragma unroll
-          for (int i = 0; i < Vec16<T>::N; ++i) dot = fmaf(q[c + i], k[i], dot);
+        for (int c = 0; c < DH; c += 4) {
+          const float4 k4 = *reinterpret_cast<const float4*>(sK + t * dkv + ck + c);
+          dot = fmaf(q[c], k4.x, dot);
+          dot = fmaf(q[c + 1], k4.y, dot);
+          dot = fmaf(q[c + 2], k4.z, dot);
+          dot = fmaf(q[c + 3], k4.w, dot);
         }
       }
       sc[t] = dot;
@@ -310,11 +318,12 @@ __global__ void __launch_bounds__(256) cross_lg_kernel(const T* __restrict__ q_i
     for (int t = 0; t < kWin; ++t) {
       if (t < W) {
 #pragma unroll
-        for (int c = 0; c < DH; c += Vec16<T>::N) {
-          float v[Vec16<T>::N];
-          Vec16<T>::load(sV + t * dkv + ck + c, v);
-#pragma unroll
-          for (int i = 0; i < Vec16<T>::N; ++i) q[c + i] = fmaf(sc[t], v[i], q[c + i]);
+        for (int c = 0; c < DH; c += 4) {
+          const float4 v4 = *reinterpret_cast<const float4*>(sV + t * dkv + ck + c);
+          q[c] = fmaf(sc[t], v4.x, q[c]);
+          q[c + 1] = fmaf(sc[t], v4.y, q[c + 1]);
+          q[c + 2] = fmaf(sc[t], v4.z, q[c + 2]);
+          q[c + 3] = fmaf(sc[t], v4.w, q[c + 3]);
         }
       }
     }
@@ -394,7 +403,7 @@ cudaError_t launch_cross_attn_lg(const T* q, T* out, const T* Kc, const T* Vc, c
   if (max_q == 0 || n_req == 0) return cudaSuccess;
   CrossLgArgs a{cand_off_dev, n_cand, S, kv_off, kv_len, Kg, Vg, l_local, H, d, dkv, H / Hkv,
                 1.4426950408889634f / sqrtf(static_cast<float>(dh))};
-  const size_t smem = static_cast<size_t>(2 * kWin * dkv) * sizeof(T) + 2 * dkv * sizeof(float);
+  const size_t smem = static_cast<size_t>(2 * kWin * dkv) * sizeof(float) + 2 * dkv * sizeof(float);
   const dim3 grid((max_q + 31) / 32, n_req);
   prof_begin(KC_ATTN_CROSS, s);
   cudaError_t err;
