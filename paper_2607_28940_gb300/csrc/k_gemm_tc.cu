@@ -16,6 +16,8 @@
 // buffer.  All waits are bounded; a timeout latches TXS_ERR_DEVICE_TIMEOUT.
 #include <cstdio>
 
+#include <type_traits>
+
 #include "tc_ptx.cuh"
 
 namespace txs {
@@ -293,10 +295,23 @@ struct Shape {
 // blocks; warp 1: MMA issuer, accumulating tile i into TMEM buffer i % 2;
 // warps 2..9: epilogue, releasing the buffer as soon as its last TMEM read is
 // done so the next tile's MMAs overlap this tile's stores.
+// Request offsets of a cache projection carried by value (EPI_KV only):
+// [in_off (n+1) | dst0 (n) | lengths (n)]; n_seg < 0: not carried.
+struct KvParams {
+  int n_seg;
+  int v[3 * kKvParamReq + 1];
+};
+struct NoParams {
+  int n_seg;
+};
+template <int EPI>
+using ParamsFor = typename std::conditional<EPI == EPI_KV, KvParams, NoParams>::type;
+
 template <int BN, int EPI, int NAP, bool BRES>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
-                   const __grid_constant__ CUtensorMap tmO, const EpiArgs e) {
+                   const __grid_constant__ CUtensorMap tmO, const EpiArgs e,
+                   const __grid_constant__ ParamsFor<EPI> kp) {
   using S = Shape<BN, EPI, NAP, BRES>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -373,7 +388,19 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       bias = s_bias;
     }
     if constexpr (EPI == EPI_KV) {
-      if (e.n_seg <= kStageSeg) {
+      if (kp.n_seg >= 0) {
+        // offsets carried by value: stage them, and CTA 0 publishes them
+        // (with the new lengths) for the kernels that follow
+        const int n = kp.n_seg;
+        for (int i = threadIdx.x; i <= n; i += NUM_THREADS) s_seg[i] = kp.v[i];
+        for (int i = threadIdx.x; i < n; i += NUM_THREADS) s_dst[i] = kp.v[n + 1 + i];
+        if (blockIdx.x == 0) {
+          for (int i = threadIdx.x; i < 2 * n + 1; i += NUM_THREADS) e.kv_dev_up[i] = kp.v[i];
+          for (int i = threadIdx.x; i < n; i += NUM_THREADS) e.kv_dev_len[i] = kp.v[2 * n + 1 + i];
+        }
+        seg_off = s_seg;
+        dst_row0 = s_dst;
+      } else if (e.n_seg <= kStageSeg) {
         for (int i = threadIdx.x; i <= e.n_seg; i += NUM_THREADS) s_seg[i] = e.seg_off[i];
         for (int i = threadIdx.x; i < e.n_seg; i += NUM_THREADS) s_dst[i] = e.dst_row0[i];
         seg_off = s_seg;
@@ -598,9 +625,19 @@ static cudaError_t launch_bn(const __nv_bfloat16* A, long long lda, const __nv_b
   }
   const long long tiles = static_cast<long long>((e.M + BM - 1) / BM) * (e.N / BN);
   const int grid = static_cast<int>(tiles < num_sms() ? tiles : num_sms());
+  ParamsFor<EPI> kp;
+  kp.n_seg = -1;
+  if constexpr (EPI == EPI_KV) {
+    if (e.kv_host_up && e.kv_host_len && e.n_seg <= kKvParamReq && e.n_seg <= kStageSeg) {
+      const int n = e.n_seg;
+      kp.n_seg = n;
+      for (int i = 0; i < 2 * n + 1; ++i) kp.v[i] = e.kv_host_up[i];
+      for (int i = 0; i < n; ++i) kp.v[2 * n + 1 + i] = e.kv_host_len[i];
+    }
+  }
   prof_begin(cls, s);
-  cudaError_t err =
-      launch_pdl(gemm_tc_kernel<BN, EPI, NAP, BRES>, dim3(grid), dim3(NUM_THREADS), Sh::SMEM_BYTES, s, ta, tb, to, e);
+  cudaError_t err = launch_pdl(gemm_tc_kernel<BN, EPI, NAP, BRES>, dim3(grid), dim3(NUM_THREADS), Sh::SMEM_BYTES,
+                               s, ta, tb, to, e, kp);
   prof_end(cls, s);
   return err;
 }

@@ -400,10 +400,19 @@ txs_status project_rows(txs_model* m, txs_kv_cache* c, int n_req, const int32_t*
     len[r] = (append ? c->h_len[r] : 0) + in_off[r + 1] - in_off[r];
     max_rows = std::max(max_rows, in_off[r + 1] - in_off[r]);
   }
-  TXS_CK(upload_call(c, up, len, s));
+  // the tensor-core projection carries the offsets by value and publishes
+  // them; otherwise a separate upload comes first
+  const bool by_value = std::is_same<T, __nv_bfloat16>::value && total > 0 && n_req <= kKvParamReq;
+  if (!by_value) TXS_CK(upload_call(c, up, len, s));
   if (total > 0) {
     const int dkv = c->dkv;
     EpiArgs e = epi_base(EPI_KV, total, 2 * nL * dkv, d);
+    if (by_value) {
+      e.kv_host_up = up.data();
+      e.kv_host_len = len.data();
+      e.kv_dev_up = c->d_in_off;
+      e.kv_dev_len = c->d_len;
+    }
     e.bias = m->b_kv;
     e.out = c->kv;
     e.ldo = dkv;

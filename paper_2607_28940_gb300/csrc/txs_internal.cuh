@@ -153,7 +153,18 @@ struct EpiArgs {
   float* logits;
   float* probs;
   int* status;
+  // EPI_KV on the tensor cores: when kv_host_up is set (host [in_off (R+1) |
+  // dst0 (R)] and kv_host_len [R]) and n_seg fits the kernel's parameter
+  // block, the launch carries these values by value; the kernel uses them for
+  // its row remap and writes them to kv_dev_up / kv_dev_len (seg_off and the
+  // lengths the later kernels read), so no separate upload is needed.
+  const int* kv_host_up;
+  const int* kv_host_len;
+  int* kv_dev_up;
+  int* kv_dev_len;
 };
+// Largest request count whose offsets an EPI_KV launch carries by value.
+constexpr int kKvParamReq = 1000;
 
 // Launchers (return cudaError_t of the launch).
 // fp32 A; B float or bf16; fp32 output (EPI_KV with seg_off == nullptr keeps rows)
