@@ -83,3 +83,18 @@ def test_deep_wide_events():
     rl, rp = O.score_events(O.Model.from_arrays(w, wl), ev.beh, ev.ends, ev.ctx, ev.cand, ev.cand_off, O.FULL)
     assert_scores_close(lg.cpu().numpy(), rl, "bf16", "event logits")
     assert_scores_close(pr.cpu().numpy(), rp, "bf16", "event probs")
+
+
+def test_full_size_sampled_requests():
+    """The benchmark's Deep & Wide configuration: the whole small_bf16 batch
+    (32 requests x 256 candidates) scored on the GPU; requests 0 and 31
+    against the oracle."""
+    wl = W.with_sizes(W.WORKLOADS["small_bf16"], dw_in=64, dw_out=32, dw_hidden=256)
+    w = _weights(wl, 1.0)
+    g = run_gpu(wl, O.LOCAL_GLOBAL, append=True, weights=w)
+    assert np.isfinite(g.logits).all()
+    for r in (0, wl.n_req - 1):
+        lg, pr, _, _ = oracle_scores(wl, O.LOCAL_GLOBAL, requests=[r], append=True, weights=w)
+        sl = slice(g.batch.cand_off[r], g.batch.cand_off[r + 1])
+        assert_scores_close(g.logits[sl], lg, "bf16", f"logits request {r}")
+        assert_scores_close(g.probs[sl], pr, "bf16", f"probs request {r}")

@@ -125,3 +125,31 @@ def test_event_errors():
         txs.score_events(model, cache, 1, beh, np.ones(4097, np.int32), big, cand, ctx)
     assert e.value.status == txs.TXS_ERR_UNSUPPORTED
     assert model.device_status() == txs.TXS_OK
+
+
+@pytest.mark.parametrize("mode", [O.LOCAL_GLOBAL, O.FULL])
+def test_benchmark_configuration_sampled_events(mode):
+    """The benchmark's streaming configuration: one 8192-row stream of the
+    mid_bf16 model, 64 events at sorted prefix ends with 256 candidates each,
+    scored in one call; the first, a middle and the last event against the
+    oracle."""
+    wl = W.with_sizes(W.WORKLOADS["mid_bf16"], n_req=1, L=8192, M=1, dL=0)
+    weights = W.weights(wl)
+    model = txs.Model(wl, weights, mode)
+    ev = W.events(wl, 8192, 64, 256, 20267)
+    dt = txs.torch_dtype(wl.dtype)
+    beh = txs.to_device(ev.beh, dt)
+    cache = txs.KVCache(model, np.array([0, 8192], np.int32), beh)
+    lg, pr = txs.score_events(model, cache, 0, beh, ev.ends, ev.cand_off, txs.to_device(ev.cand, dt),
+                              txs.to_device(ev.ctx.reshape(-1, wl.d_model), dt))
+    torch.cuda.synchronize()
+    assert model.device_status() == txs.TXS_OK
+    lg, pr = lg.cpu().numpy(), pr.cpu().numpy()
+    assert np.isfinite(lg).all()
+    om = O.Model.from_arrays(weights, wl)
+    for t in (0, 31, 63):
+        sl = slice(ev.cand_off[t], ev.cand_off[t + 1])
+        rl, rp = O.score_events(om, ev.beh, ev.ends[t:t + 1], ev.ctx[t:t + 1], ev.cand[sl],
+                                np.array([0, sl.stop - sl.start]), mode)
+        assert_scores_close(lg[sl], rl, "bf16", f"event {t} logits")
+        assert_scores_close(pr[sl], rp, "bf16", f"event {t} probs")
