@@ -245,6 +245,24 @@ txs_status txs_score_candidates(txs_model* model, const txs_kv_cache* cache, int
                                 float* out_logits, float* out_probs, void* stream);
 
 /*
+ * txs_score_candidates_after — txs_score_candidates for a cache that may still
+ * be being written (rebuilt or appended) on another stream.  The work that
+ * does not read the cache (packing, and in the first layer the serving-stream
+ * attention, its output projection and the query projection) is enqueued on
+ * `stream` at once; `stream` then waits on `cache_ready` (a cudaEvent_t
+ * recorded on the writing stream after its last cache call, passed as void*)
+ * before the first cross-attention, so that prefix overlaps the cache write.
+ * cache_ready == NULL gives txs_score_candidates.  The host-side cache state
+ * (lengths) must already be that of the writes the event covers, i.e. the
+ * cache calls are issued first.  The caller also orders any later write of
+ * the cache after this call's reads (an event recorded on `stream`).
+ */
+txs_status txs_score_candidates_after(txs_model* model, const txs_kv_cache* cache, int32_t n_req,
+                                      const int32_t* cand_offsets, const void* cand_tok, const void* ctx_tok,
+                                      void* workspace, size_t workspace_bytes, float* out_logits,
+                                      float* out_probs, void* cache_ready, void* stream);
+
+/*
  * txs_events_workspace_size — bytes of device scratch txs_score_events needs
  * for n_events events with total_cand candidates in all, the longest event
  * prefix being max_event_end rows.

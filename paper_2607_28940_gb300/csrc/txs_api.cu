@@ -438,6 +438,7 @@ struct KvView {
   const int* off;          // device [n]
   const int* len;          // device [n]
   const float* gkv;        // device [nL][2][n][dkv]
+  cudaEvent_t ready = nullptr;  // recorded after the cache's last write (may be null)
 };
 
 template <typename T>
@@ -504,6 +505,9 @@ txs_status score_impl(txs_model* m, const KvView& c, int n_req, const int32_t* c
     e.out = QKV;
     e.ldo = d;
     TXS_CK(gemm(m, X1, d, W.Wt_q, e, tmp, s, KC_GEMM_Q));
+    // the first read of the cache: a caller that is still writing it on
+    // another stream made everything above overlap with that write
+    if (l == 0 && c.ready) TXS_CK(cudaStreamWaitEvent(s, c.ready, 0));
     const T* Kc = kv + (size_t(2 * l) * c.cap_total) * dkv;
     const T* Vc = kv + (size_t(2 * l + 1) * c.cap_total) * dkv;
     const float* Kg = c.gkv + size_t(2 * l) * n_req * dkv;
@@ -1001,10 +1005,11 @@ TXS_API txs_status txs_score_workspace_size(const txs_model* m, int32_t n_req, i
   return TXS_OK;
 }
 
-TXS_API txs_status txs_score_candidates(txs_model* m, const txs_kv_cache* c, int32_t n_req,
-                                        const int32_t* cand_offsets, const void* cand_tok, const void* ctx_tok,
-                                        void* workspace, size_t workspace_bytes, float* out_logits, float* out_probs,
-                                        void* stream) {
+namespace txs {
+namespace {
+txs_status score_entry(txs_model* m, const txs_kv_cache* c, int32_t n_req, const int32_t* cand_offsets,
+                       const void* cand_tok, const void* ctx_tok, void* workspace, size_t workspace_bytes,
+                       float* out_logits, float* out_probs, cudaEvent_t cache_ready, void* stream) {
   if (!m || !c || !cand_offsets) return TXS_ERR_INVALID_ARG;
   if (c->model_hash != m->hash) return TXS_ERR_STALE_CACHE;
   if (n_req != c->n_req || !offsets_ok(cand_offsets, n_req, false)) return TXS_ERR_INVALID_ARG;
@@ -1019,11 +1024,30 @@ TXS_API txs_status txs_score_candidates(txs_model* m, const txs_kv_cache* c, int
     return TXS_ERR_INVALID_ARG;
   if (workspace_bytes < score_layout(cf, m->es, n_req, n_cand).total) return TXS_ERR_INVALID_ARG;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
-  const KvView v{c->kv, c->cap_total, c->d_off, c->d_len, c->gkv};
+  const KvView v{c->kv, c->cap_total, c->d_off, c->d_len, c->gkv, cache_ready};
   return cf.dtype == TXS_BF16
              ? score_impl<__nv_bfloat16>(m, v, n_req, cand_offsets, cand_tok, ctx_tok, workspace, out_logits,
                                          out_probs, s)
              : score_impl<float>(m, v, n_req, cand_offsets, cand_tok, ctx_tok, workspace, out_logits, out_probs, s);
+}
+}  // namespace
+}  // namespace txs
+
+TXS_API txs_status txs_score_candidates(txs_model* m, const txs_kv_cache* c, int32_t n_req,
+                                        const int32_t* cand_offsets, const void* cand_tok, const void* ctx_tok,
+                                        void* workspace, size_t workspace_bytes, float* out_logits, float* out_probs,
+                                        void* stream) {
+  return score_entry(m, c, n_req, cand_offsets, cand_tok, ctx_tok, workspace, workspace_bytes, out_logits,
+                     out_probs, nullptr, stream);
+}
+
+TXS_API txs_status txs_score_candidates_after(txs_model* m, const txs_kv_cache* c, int32_t n_req,
+                                              const int32_t* cand_offsets, const void* cand_tok,
+                                              const void* ctx_tok, void* workspace, size_t workspace_bytes,
+                                              float* out_logits, float* out_probs, void* cache_ready,
+                                              void* stream) {
+  return score_entry(m, c, n_req, cand_offsets, cand_tok, ctx_tok, workspace, workspace_bytes, out_logits,
+                     out_probs, static_cast<cudaEvent_t>(cache_ready), stream);
 }
 
 // Streaming events: the score workspace, then per event its cache view

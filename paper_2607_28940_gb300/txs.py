@@ -81,6 +81,7 @@ _SIGS = {
     "txs_cache_n_req": (_I32, [_P]),
     "txs_score_workspace_size": (_I32, [_P, _I32, ctypes.c_int64, ctypes.POINTER(ctypes.c_size_t)]),
     "txs_score_candidates": (_I32, [_P, _P, _I32, _I32P, _P, _P, _P, ctypes.c_size_t, _P, _P, _P]),
+    "txs_score_candidates_after": (_I32, [_P, _P, _I32, _I32P, _P, _P, _P, ctypes.c_size_t, _P, _P, _P, _P]),
     "txs_rank_candidates": (_I32, [_I32, _I32P, _P, _I32, _I32, _I32, _P, _P]),
     "txs_events_workspace_size": (_I32, [_P, _I32, ctypes.c_int64, _I32, ctypes.POINTER(ctypes.c_size_t)]),
     "txs_score_events": (_I32, [_P, _P, _I32, _P, _I32, _I32P, _I32P, _P, _P, _P, ctypes.c_size_t, _P, _P, _P]),
@@ -299,8 +300,12 @@ def workspace_bytes(model: Model, n_req: int, total_cand: int) -> int:
 
 def score(model: Model, cache: KVCache, cand_offsets, cand_tok: torch.Tensor, ctx_tok: Optional[torch.Tensor],
           workspace: Optional[torch.Tensor] = None, out_logits: Optional[torch.Tensor] = None,
-          out_probs: Optional[torch.Tensor] = None, want_probs: bool = True, stream=None):
-    """Scores of all candidates: (logits, probs) as [sum M, k] float32 CUDA tensors."""
+          out_probs: Optional[torch.Tensor] = None, want_probs: bool = True, stream=None,
+          cache_ready: Optional[torch.cuda.Event] = None):
+    """Scores of all candidates: (logits, probs) as [sum M, k] float32 CUDA tensors.
+    With ``cache_ready`` (an event recorded after the cache's last write on
+    another stream), the work that does not read the cache starts at once
+    (txs_score_candidates_after)."""
     off, p = _offsets(cand_offsets)
     n_req = len(off) - 1
     n_cand = int(off[-1])
@@ -311,9 +316,15 @@ def score(model: Model, cache: KVCache, cand_offsets, cand_tok: torch.Tensor, ct
         out_logits = torch.empty((n_cand, k), dtype=torch.float32, device="cuda")
     if out_probs is None and want_probs:
         out_probs = torch.empty((n_cand, k), dtype=torch.float32, device="cuda")
-    _check(lib().txs_score_candidates(model.handle, cache.handle, n_req, p, _ptr(cand_tok), _ptr(ctx_tok),
-                                      _ptr(workspace), workspace.numel(), _ptr(out_logits), _ptr(out_probs),
-                                      _stream(stream)), "txs_score_candidates")
+    if cache_ready is not None:
+        _check(lib().txs_score_candidates_after(model.handle, cache.handle, n_req, p, _ptr(cand_tok), _ptr(ctx_tok),
+                                                _ptr(workspace), workspace.numel(), _ptr(out_logits),
+                                                _ptr(out_probs), cache_ready.cuda_event, _stream(stream)),
+               "txs_score_candidates_after")
+    else:
+        _check(lib().txs_score_candidates(model.handle, cache.handle, n_req, p, _ptr(cand_tok), _ptr(ctx_tok),
+                                          _ptr(workspace), workspace.numel(), _ptr(out_logits), _ptr(out_probs),
+                                          _stream(stream)), "txs_score_candidates")
     return out_logits, out_probs
 
 

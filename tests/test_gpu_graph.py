@@ -82,3 +82,38 @@ def test_encoder_append_replays_from_a_graph():
     torch.cuda.synchronize()
     assert torch.equal(out, ref)
     assert enc.device_status() == txs.TXS_OK
+
+
+@pytest.mark.parametrize("mode", [txs.LOCAL_GLOBAL, txs.FULL])
+def test_score_after_cache_event_matches_sequential(mode):
+    """txs_score_candidates_after: the cache refreshed on a side stream while
+    the part of scoring that does not read it runs on the main stream gives
+    the same bytes as the calls issued one after the other."""
+    wl = W.with_sizes(W.WORKLOADS["small_bf16"], n_req=4, L=[30, 300, 5, 77], M=[9, 1, 40, 0], dL=[3, 0, 8, 1])
+    b = W.batch(wl)
+    dt = txs.torch_dtype(wl.dtype)
+    model = txs.Model(wl, W.weights(wl), mode)
+    beh, cand, app = txs.to_device(b.beh, dt), txs.to_device(b.cand, dt), txs.to_device(b.app, dt)
+    ctx = txs.to_device(b.ctx.reshape(-1, wl.d_model), dt)
+    cache = txs.KVCache(model, b.beh_off, beh, capacity_extra=wl.capacity_extra)
+    n = int(b.cand_off[-1])
+    ws = torch.empty(txs.workspace_bytes(model, wl.n_req, n), dtype=torch.uint8, device="cuda")
+    lg = torch.empty((n, wl.n_actions), dtype=torch.float32, device="cuda")
+    pr = torch.empty_like(lg)
+    cache.rebuild(b.beh_off, beh)
+    cache.append(b.app_off, app)
+    txs.score(model, cache, b.cand_off, cand, ctx, workspace=ws, out_logits=lg, out_probs=pr)
+    torch.cuda.synchronize()
+    ref = (lg.clone(), pr.clone())
+    main, side, ready = torch.cuda.current_stream(), torch.cuda.Stream(), torch.cuda.Event()
+    for _ in range(3):
+        lg.zero_(); pr.zero_()
+        side.wait_stream(main)
+        with torch.cuda.stream(side):
+            cache.rebuild(b.beh_off, beh)
+            cache.append(b.app_off, app)
+            ready.record(side)
+        txs.score(model, cache, b.cand_off, cand, ctx, workspace=ws, out_logits=lg, out_probs=pr, cache_ready=ready)
+        torch.cuda.synchronize()
+        assert torch.equal(lg, ref[0]) and torch.equal(pr, ref[1])
+    assert model.device_status() == txs.TXS_OK
