@@ -221,8 +221,7 @@ def run_txs(args, rank, world):
     stream = torch.cuda.current_stream()
 
     def step(start_ev=None, beh_t=beh, app_t=app, cand_t=cand, ctx_t=ctx):
-        cache.rebuild(full_off, beh_t)
-        cache.append(b.app_off, app_t)
+        cache.rebuild_append(full_off, beh_t, b.app_off, app_t)
         txs.score(model, cache, b.cand_off, cand_t, ctx_t, workspace=ws, out_logits=logits, out_probs=probs)
         txs.rank(b.cand_off, probs, wl.n_actions, 0, 0, out=ranks)
 
@@ -237,8 +236,7 @@ def run_txs(args, rank, world):
     def step_overlap(start_ev):
         side.wait_event(start_ev)
         with torch.cuda.stream(side):
-            cache.rebuild(full_off, beh)
-            cache.append(b.app_off, app)
+            cache.rebuild_append(full_off, beh, b.app_off, app)
             ready.record(side)
         txs.score(model, cache, b.cand_off, cand, ctx, workspace=ws, out_logits=logits, out_probs=probs,
                   cache_ready=ready)
@@ -296,8 +294,8 @@ def run_txs(args, rank, world):
            "data": "synthetic (seeded N(0,1) inputs, N(0,0.02) weights; shapes of the paper's serving setting)"}
     out["config"] = {"workload": describe(wl, args.mode), "global_batch": n_cand * world,
                      "requests_per_gpu": wl.n_req, "seq_len": int(b.L.max()),
-                     "step": "in-place cache rebuild + append (side stream) + score + rank; the part of "
-                             "scoring that does not read the cache overlaps the refresh",
+                     "step": "in-place cache rebuild + append (one call, side stream) + score + rank; the part "
+                             "of scoring that does not read the cache overlaps the refresh",
                      "l2": "flushed before every timed step (256 MiB device write, untimed)",
                      "parallelism": f"request-sharded replicas x{world} (no data-path collective)"}
     out["wall_s_timed_region"] = wall
@@ -391,8 +389,7 @@ def e2e(txs, torch, model, cache, b, wl, args, dt, logits, probs, ranks, ws, wor
         with torch.cuda.stream(side):
             d_beh.copy_(h_beh, non_blocking=True)
             d_app.copy_(h_app, non_blocking=True)
-            cache.rebuild(b.beh_off, d_beh)
-            cache.append(b.app_off, d_app)
+            cache.rebuild_append(b.beh_off, d_beh, b.app_off, d_app)
             ready.record(side)
         d_cand.copy_(h_cand, non_blocking=True)
         if d_ctx is not None:

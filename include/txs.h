@@ -176,6 +176,18 @@ txs_status txs_rebuild_kv_cache(txs_model* model, txs_kv_cache* cache, int32_t n
 txs_status txs_append_behavior(txs_model* model, txs_kv_cache* cache, int32_t n_req,
                                const int32_t* new_offsets, const void* new_enc, void* stream);
 
+/*
+ * txs_rebuild_append_kv_cache — txs_rebuild_kv_cache from beh_offsets /
+ * beh_enc followed by txs_append_behavior of new_offsets / new_enc, in one
+ * call (App. D: the batch re-encode and the streamed tail since it).  The
+ * result is exactly that of the two calls; the anchor's projections are
+ * computed once, after the append.  Capacity is checked for the sum before
+ * anything is enqueued.
+ */
+txs_status txs_rebuild_append_kv_cache(txs_model* model, txs_kv_cache* cache, int32_t n_req,
+                                       const int32_t* beh_offsets, const void* beh_enc,
+                                       const int32_t* new_offsets, const void* new_enc, void* stream);
+
 /* Copy rows row0 .. row0+n_rows-1 of request `req`'s cached K (which = 0) or
  * V (which = 1) of layer `layer` into dst (device, model dtype, [n_rows, dkv]),
  * asynchronously on `stream`.  Rows must be < the request's current length. */

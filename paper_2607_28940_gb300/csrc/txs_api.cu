@@ -387,7 +387,7 @@ cudaError_t upload_call(txs_kv_cache* c, const std::vector<int>& up, const std::
 
 template <typename T>
 txs_status project_rows(txs_model* m, txs_kv_cache* c, int n_req, const int32_t* in_off, const void* rows,
-                        bool append, cudaStream_t s) {
+                        bool append, cudaStream_t s, bool project_anchor = true) {
   const txs_config& cf = m->cfg;
   const int d = cf.d_model, nL = cf.n_layers;
   const long long total = in_off[n_req];
@@ -425,7 +425,8 @@ txs_status project_rows(txs_model* m, txs_kv_cache* c, int n_req, const int32_t*
   }
   TXS_CK(launch_pool<T>(static_cast<const T*>(rows), c->d_in_off, n_req, max_rows, m->w_pool, d, c->max_chunks,
                         c->part, append ? 1 : 0, c->pool_m, c->pool_s, c->pool_acc, c->g, c->pool_cnt, s));
-  TXS_CK(launch_anchor_proj<T>(c->g, static_cast<const T*>(m->Wt_kv), m->b_kv, c->gkv, n_req, d, c->dkv, nL, s));
+  if (project_anchor)
+    TXS_CK(launch_anchor_proj<T>(c->g, static_cast<const T*>(m->Wt_kv), m->b_kv, c->gkv, n_req, d, c->dkv, nL, s));
   return TXS_OK;
 }
 
@@ -946,6 +947,36 @@ TXS_API txs_status txs_rebuild_kv_cache(txs_model* m, txs_kv_cache* c, int32_t n
                                            : project_rows<float>(m, c, n_req, beh_offsets, beh_enc, false, s);
   if (st != TXS_OK) return st;
   for (int r = 0; r < n_req; ++r) c->h_len[r] = beh_offsets[r + 1] - beh_offsets[r];
+  return TXS_OK;
+}
+
+TXS_API txs_status txs_rebuild_append_kv_cache(txs_model* m, txs_kv_cache* c, int32_t n_req,
+                                               const int32_t* beh_offsets, const void* beh_enc,
+                                               const int32_t* new_offsets, const void* new_enc, void* stream) {
+  if (!m || !c || !beh_offsets || !new_offsets) return TXS_ERR_INVALID_ARG;
+  if (c->model_hash != m->hash) return TXS_ERR_STALE_CACHE;
+  if (n_req != c->n_req || !offsets_ok(beh_offsets, n_req, false) || !offsets_ok(new_offsets, n_req, false))
+    return TXS_ERR_INVALID_ARG;
+  for (int r = 0; r < n_req; ++r) {
+    if (beh_offsets[r + 1] == beh_offsets[r]) return TXS_ERR_COLD_START;
+    if (static_cast<long long>(beh_offsets[r + 1] - beh_offsets[r]) + (new_offsets[r + 1] - new_offsets[r]) >
+        c->h_cap[r])
+      return TXS_ERR_CAPACITY;
+  }
+  if (!beh_enc || (new_offsets[n_req] > 0 && !new_enc)) return TXS_ERR_INVALID_ARG;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const bool bf16 = m->cfg.dtype == TXS_BF16;
+  const bool any_new = new_offsets[n_req] > 0;
+  // the rebuild's anchor would be replaced at once: project it only after the append
+  txs_status st = bf16 ? project_rows<__nv_bfloat16>(m, c, n_req, beh_offsets, beh_enc, false, s, !any_new)
+                       : project_rows<float>(m, c, n_req, beh_offsets, beh_enc, false, s, !any_new);
+  if (st != TXS_OK) return st;
+  for (int r = 0; r < n_req; ++r) c->h_len[r] = beh_offsets[r + 1] - beh_offsets[r];
+  if (!any_new) return TXS_OK;
+  st = bf16 ? project_rows<__nv_bfloat16>(m, c, n_req, new_offsets, new_enc, true, s)
+            : project_rows<float>(m, c, n_req, new_offsets, new_enc, true, s);
+  if (st != TXS_OK) return st;
+  for (int r = 0; r < n_req; ++r) c->h_len[r] += new_offsets[r + 1] - new_offsets[r];
   return TXS_OK;
 }
 

@@ -72,6 +72,7 @@ _SIGS = {
     "txs_cache_destroy": (None, [_P]),
     "txs_rebuild_kv_cache": (_I32, [_P, _P, _I32, _I32P, _P, _P]),
     "txs_append_behavior": (_I32, [_P, _P, _I32, _I32P, _P, _P]),
+    "txs_rebuild_append_kv_cache": (_I32, [_P, _P, _I32, _I32P, _P, _I32P, _P, _P]),
     "txs_cache_read_rows": (_I32, [_P, _I32, _I32, _I32, _I32, _I32, _P, _P]),
     "txs_cache_read_anchor": (_I32, [_P, _I32, _I32, _P, _P]),
     "txs_cache_lengths": (_I32, [_P, _I32P]),
@@ -232,6 +233,16 @@ class KVCache:
         off, p = _offsets(beh_offsets)
         _check(lib().txs_rebuild_kv_cache(self.model.handle, self.handle, len(off) - 1, p, _ptr(beh_enc),
                                           _stream(stream)), "txs_rebuild_kv_cache")
+
+    def rebuild_append(self, beh_offsets, beh_enc: torch.Tensor, new_offsets, new_enc: Optional[torch.Tensor],
+                       stream=None):
+        """rebuild(beh_offsets, beh_enc) then append(new_offsets, new_enc) in one
+        call (txs_rebuild_append_kv_cache)."""
+        off, p = _offsets(beh_offsets)
+        noff, np_ = _offsets(new_offsets)
+        _check(lib().txs_rebuild_append_kv_cache(self.model.handle, self.handle, len(off) - 1, p, _ptr(beh_enc), np_,
+                                                 _ptr(new_enc) if new_enc is not None and new_enc.numel() else None,
+                                                 _stream(stream)), "txs_rebuild_append_kv_cache")
 
     def append(self, new_offsets, new_enc: Optional[torch.Tensor], stream=None, model: Optional[Model] = None):
         off, p = _offsets(new_offsets)

@@ -256,3 +256,38 @@ def test_window_covering_history_both_modes():
     ref_f, _, _, _ = oracle_scores(wl, txs.FULL)
     assert_scores_close(lg_l, ref_l, "bf16")
     assert_scores_close(lg_f, ref_f, "bf16")
+
+
+@pytest.mark.parametrize("name", ["tiny_fp32", "small_bf16"])
+def test_rebuild_append_equals_the_two_calls(name):
+    """txs_rebuild_append_kv_cache gives the bytes of txs_rebuild_kv_cache
+    followed by txs_append_behavior: cached rows, anchor and scores."""
+    wl = W.with_sizes(W.WORKLOADS[name], n_req=3, L=[20, 300, 7], M=[5, 40, 1], dL=[4, 0, 9])
+    b = W.batch(wl)
+    dt = txs.torch_dtype(wl.dtype)
+    model = txs.Model(wl, W.weights(wl), O.LOCAL_GLOBAL)
+    beh, app = txs.to_device(b.beh, dt), txs.to_device(b.app, dt)
+    cand, ctx = txs.to_device(b.cand, dt), txs.to_device(b.ctx.reshape(-1, wl.d_model), dt)
+    c1 = txs.KVCache(model, b.beh_off, beh, capacity_extra=16)
+    c2 = txs.KVCache(model, b.beh_off, beh, capacity_extra=16)
+    c1.rebuild(b.beh_off, beh)
+    c1.append(b.app_off, app)
+    c2.rebuild_append(b.beh_off, beh, b.app_off, app)
+    torch.cuda.synchronize()
+    assert np.array_equal(c1.lengths(), c2.lengths())
+    for r in range(wl.n_req):
+        n = int(c1.lengths()[r])
+        for l in range(wl.n_layers):
+            for which in (0, 1):
+                assert torch.equal(c1.read_rows(l, which, r, 0, n), c2.read_rows(l, which, r, 0, n))
+    for which in (0, 1, 2):
+        assert torch.equal(c1.read_anchor(0, which), c2.read_anchor(0, which))
+    s1 = txs.score(model, c1, b.cand_off, cand, ctx)
+    s2 = txs.score(model, c2, b.cand_off, cand, ctx)
+    assert torch.equal(s1[0], s2[0]) and torch.equal(s1[1], s2[1])
+    # capacity is checked for the sum, before anything runs
+    big = np.array([0, 20, 20, 20], np.int32)
+    with pytest.raises(txs.TxsError) as e:
+        c2.rebuild_append(b.beh_off, beh, big, txs.to_device(np.zeros((20, wl.d_model), np.float32), dt))
+    assert e.value.status == txs.TXS_ERR_CAPACITY
+    assert np.array_equal(c2.lengths(), c1.lengths())
