@@ -96,6 +96,16 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   const uint32_t tmem = *tmem_holder;
   cluster_sync();                     // every CTA's barriers exist before any peer arrives
   pdl_launch_dependents();
+  // the weights are not written by the preceding kernels: the weight part of
+  // the first k-blocks is fetched before the wait (overlapping the
+  // predecessor's tail); the activations only after it
+  const int n_pre = my_tiles > 0 ? (num_kb < S::STAGES ? num_kb : S::STAGES) : 0;
+  if (warp == 0 && lane == 0) {
+    for (int kb = 0; kb < n_pre; ++kb) {   // fresh ring: these stages are free
+      mbar_expect_tx(full + kb, S::STAGE_BYTES);
+      tma_load_2d(sB + kb * S::B_STAGE_BYTES, &tmB, full + kb, kb * BK, n0);
+    }
+  }
   pdl_wait();
   if constexpr (HEAD) {
     for (int i = threadIdx.x; i < BN * NAP; i += NUM_THREADS) {
@@ -115,6 +125,10 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         const int m0 = (cid + i * ncl) * BM;
         for (int kb = 0; kb < num_kb; ++kb, ++it) {
           const int s = it % S::STAGES;
+          if (it < n_pre) {     // weights in flight since before the wait
+            tma_load_2d(sA + s * A_STAGE_BYTES, &tmA, full + s, kb * BK, m0);
+            continue;
+          }
           if (!mbar_wait(empty + s, ((it / S::STAGES) & 1) ^ 1, abort_flag)) {
             ok = false;
             break;

@@ -369,6 +369,29 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   const uint32_t tmem = *tmem_holder;
   // the set-up above overlaps the previous kernel's tail; its outputs are read below
   pdl_launch_dependents();
+  // The weights are not written by the kernels before this one: the
+  // producer issues the weight part of its first k-blocks (or the resident
+  // weight slice) before waiting, so that fetch overlaps the predecessor's
+  // tail.  The activations (A) are loaded only after the wait.
+  int n_pre = 0;                      // leading k-blocks whose weights are in flight
+  if (warp == 0 && lane == 0 && t_lo < t_hi) {
+    const int n0 = tile_n(t_lo) * BN;
+    if constexpr (BRES) {
+      mbar_expect_tx(b_full, BN * e.K * 2);
+      for (int kb = 0; kb < num_kb; ++kb)
+#pragma unroll
+        for (int j = 0; j < BN; j += S::B_BOX)
+          tma_load_2d(sBres + kb * (BN * BK * 2) + j * (BK * 2), &tmB, b_full, kb * BK, n0 + j);
+    } else {
+      n_pre = num_kb < S::STAGES ? num_kb : S::STAGES;
+      for (int kb = 0; kb < n_pre; ++kb) {   // fresh ring: these stages are free
+        mbar_expect_tx(full + kb, S::STAGE_BYTES);
+#pragma unroll
+        for (int j = 0; j < BN; j += S::B_BOX)
+          tma_load_2d(sB + kb * S::B_STAGE_BYTES + j * (BK * 2), &tmB, full + kb, kb * BK, n0 + j);
+      }
+    }
+  }
   pdl_wait();
   if constexpr (EPI == EPI_LN_HEAD) {
     for (int i = threadIdx.x; i < e.N * NAP; i += NUM_THREADS) {
@@ -416,6 +439,10 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmB)) : "memory");
       int it = 0;  // global k-block counter (ring position)
       int nb = 0, cur_n = -1;   // resident B slices loaded, current slice
+      if (BRES && t_lo < t_hi) {   // the first slice was issued before the wait
+        nb = 1;
+        cur_n = tile_n(t_lo) * BN;
+      }
       bool ok = true;
       for (int t = t_lo; t < t_hi && ok; t += t_step) {
         const int m0 = tile_m(t) * BM, n0 = tile_n(t) * BN;
@@ -434,6 +461,10 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         for (int kb = 0; kb < num_kb; ++kb, ++it) {
           const int s = it % S::STAGES;
           const uint32_t ph = (it / S::STAGES) & 1;
+          if (it < n_pre) {       // weights already in flight, bytes already expected
+            tma_load_2d(sA + s * A_STAGE_BYTES, &tmA, full + s, kb * BK, m0);
+            continue;
+          }
           if (!mbar_wait(empty + s, ph ^ 1, abort_flag)) {
             ok = false;
             break;
