@@ -199,6 +199,35 @@ __device__ __forceinline__ float ex2(float x) {
   return y;
 }
 
+// max(a, b, c) in one instruction (three-source max.f32, sm_100 and later).
+__device__ __forceinline__ float fmax3(float a, float b, float c) {
+  float r;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(r) : "f"(a), "f"(b), "f"(c));
+  return r;
+}
+// Lane-wise a * b + c and a + b on a pair of fp32 values in one instruction
+// (f32x2 arithmetic, sm_100 and later); each lane rounds like fmaf / fadd.
+__device__ __forceinline__ float2 ffma2(float2 a, float2 b, float2 c) {
+  uint64_t r;
+  asm("{\n\t.reg .b64 x, y, z;\n\t"
+      "mov.b64 x, {%1, %2};\n\tmov.b64 y, {%3, %4};\n\tmov.b64 z, {%5, %6};\n\t"
+      "fma.rn.f32x2 %0, x, y, z;\n\t}"
+      : "=l"(r) : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y), "f"(c.x), "f"(c.y));
+  float2 o;
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(o.x), "=f"(o.y) : "l"(r));
+  return o;
+}
+__device__ __forceinline__ float2 fadd2(float2 a, float2 b) {
+  uint64_t r;
+  asm("{\n\t.reg .b64 x, y;\n\t"
+      "mov.b64 x, {%1, %2};\n\tmov.b64 y, {%3, %4};\n\t"
+      "add.rn.f32x2 %0, x, y;\n\t}"
+      : "=l"(r) : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y));
+  float2 o;
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(o.x), "=f"(o.y) : "l"(r));
+  return o;
+}
+
 // Shared-memory matrix descriptor (tcgen05): start address, leading/stride
 // byte offsets, descriptor version 1, layout code (2 = 128-byte swizzle,
 // 4 = 64-byte swizzle).
@@ -231,6 +260,7 @@ struct FaArgs {
   int group;                  // query heads per K/V head
   float scale_log2;           // log2(e) / sqrt(d_h)
   int* status;
+  int tiles_per_cta;          // fa_pair_kernel: 2 (query-tile pairs) or 1 (every tile splits its keys)
 };
 
 template <int DH>
@@ -519,10 +549,15 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
 // columns once S has been read: the next S of the tile is issued after the P V
 // that reads P, and one thread's MMAs run in issue order), O (d_h columns),
 // Q (d_h / 2 columns).  A CTA whose second tile would be empty (the last of
-// an odd number) runs the first alone.  The softmax reads a score row in two
-// halves of 64 keys (max over both, then exponentials half by half) to stay
-// within the register file at 320 threads.  Online softmax with the
-// stale-maximum rule of fa_full_kernel.
+// an odd number, often only the S context rows) splits its key range
+// instead: group A takes the first ceil(nkv / 2) key tiles and group B the
+// rest, both for the same query rows, and group A merges the two partial
+// softmax states (O, running max, row sum) at the end through shared memory
+// (a two-part form of the same online softmax).  The softmax holds a whole score row
+// (128 keys) in registers after one TMEM load, takes its maximum with
+// three-source max and forms the exponent arguments and row sums two lanes at
+// a time (f32x2 arithmetic).  Online softmax with the stale-maximum rule of
+// fa_full_kernel.
 constexpr int PAIR_THREADS = 320;
 
 template <int DH>
@@ -531,7 +566,9 @@ struct PairShape {
   static constexpr uint32_t SW = DH == 64 ? 2u : 4u;
   static constexpr int ATOM = 8 * ROW_BYTES;
   static constexpr int KV_BYTES = BKV * ROW_BYTES;
-  static constexpr int SMEM = 2 * STG * KV_BYTES + 1024 + 256;
+  static constexpr int XSTRIDE = DH + 1;                   // floats per exchange row (padded)
+  static constexpr int XCHG = BQ * (XSTRIDE + 2) * 4;       // O rows, running max, row sum of group B
+  static constexpr int SMEM = 2 * STG * KV_BYTES + 256 + XCHG + 1024;
   static constexpr uint32_t T_S = 0, T_O = 256, T_Q = 256 + 2 * 64;
   static constexpr int TMEM_COLS = 512;
   static_assert(T_Q + 2 * (DH / 2) <= TMEM_COLS, "TMEM columns");
@@ -554,6 +591,9 @@ __global__ void __launch_bounds__(PAIR_THREADS, 1)
   uint64_t* q_ready = o_done + 2;
   uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(q_ready + 1);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_holder + 1);
+  float* xo = reinterpret_cast<float*>(bars + 32);   // [BQ][XSTRIDE] O of group B (split keys)
+  float* xm = xo + BQ * Sh::XSTRIDE;                 // [BQ] running max of group B
+  float* xl = xm + BQ;                               // [BQ] row sum of group B
 
   pdl_launch_dependents();
   pdl_wait();
@@ -562,8 +602,8 @@ __global__ void __launch_bounds__(PAIR_THREADS, 1)
   const int c0 = a.cand_off[r];
   const int M = a.cand_off[r + 1] - c0;
   const int n_q = M + a.S;
-  if (qp * 2 * BQ >= n_q) return;                   // uniform: no tile here
-  const int n_t = (qp * 2 + 1) * BQ < n_q ? 2 : 1;  // tiles of this CTA (uniform)
+  const int tile0 = qp * a.tiles_per_cta;           // first query tile of this CTA
+  if (tile0 * BQ >= n_q) return;                    // uniform: no tile here
   const int len = a.kv_len[r];
   const int kv0 = a.kv_off[r];
   const int nkv = (len + BKV - 1) / BKV;
@@ -571,6 +611,17 @@ __global__ void __launch_bounds__(PAIR_THREADS, 1)
     if (threadIdx.x == 0) latch_status(a.status, TXS_ERR_BOUNDS);
     return;
   }
+  // a lone query tile with at least two key tiles splits its keys over the
+  // two groups; otherwise each group has a query tile and sees every key tile
+  const bool lone = a.tiles_per_cta == 1 || (tile0 + 1) * BQ >= n_q;
+  const bool split = lone && nkv >= 2;
+  const int n_t = lone && !split ? 1 : 2;            // softmax groups in use (uniform)
+  const int n_a = split ? (nkv + 1) / 2 : nkv;       // key tiles of group A
+  // key-tile sequence of the ring: pairs, u = i (both groups read it); split
+  // keys, u = 2 i + t (group t's i-th key tile; A: tile i, B: tile n_a + i)
+  auto iters = [&](int t) { return split ? (t == 0 ? n_a : nkv - n_a) : nkv; };
+  auto seq = [&](int t, int i) { return split ? 2 * i + t : i; };
+  auto key_tile = [&](int t, int i) { return split && t == 1 ? n_a + i : i; };
 
   if (threadIdx.x == 0) {
     for (int st = 0; st < STG; ++st) {
@@ -601,8 +652,9 @@ __global__ void __launch_bounds__(PAIR_THREADS, 1)
         const int st = j % STG;
         if (!mbar_wait(kv_empty + st, ((j / STG) & 1) ^ 1, abort_flag)) break;
         mbar_expect_tx(kv_full + st, 2 * Sh::KV_BYTES);
-        tma_load_2d(sK + st * Sh::KV_BYTES, &tmK, kv_full + st, (h / a.group) * DH, kv0 + j * BKV);
-        tma_load_2d(sV + st * Sh::KV_BYTES, &tmV, kv_full + st, (h / a.group) * DH, kv0 + j * BKV);
+        const int kt = split ? ((j & 1) ? n_a + (j >> 1) : (j >> 1)) : j;   // j-th tile of the sequence
+        tma_load_2d(sK + st * Sh::KV_BYTES, &tmK, kv_full + st, (h / a.group) * DH, kv0 + kt * BKV);
+        tma_load_2d(sV + st * Sh::KV_BYTES, &tmV, kv_full + st, (h / a.group) * DH, kv0 + kt * BKV);
         issued = j + 1;
       }
       if (*abort_flag)
@@ -613,8 +665,8 @@ __global__ void __launch_bounds__(PAIR_THREADS, 1)
     if (lane == 0) {
       constexpr uint32_t id_s = idesc_bf16(BQ, BKV, false);
       constexpr uint32_t id_pv = idesc_bf16(BQ, DH, true);
-      auto qk = [&](int t, int j) {
-        const uint32_t k_addr = smem_u32(sK + (j % STG) * Sh::KV_BYTES);
+      auto qk = [&](int t, int u) {
+        const uint32_t k_addr = smem_u32(sK + (u % STG) * Sh::KV_BYTES);
 #pragma unroll
         for (int k = 0; k < DH / 16; ++k) {
           const uint64_t kd = sdesc(k_addr + k * 32, 16, Sh::ATOM, Sh::SW);
@@ -622,32 +674,42 @@ __global__ void __launch_bounds__(PAIR_THREADS, 1)
         }
         mma_commit(s_full + t);
       };
-      auto pv = [&](int t, int j) {
-        const uint32_t v_addr = smem_u32(sV + (j % STG) * Sh::KV_BYTES);
+      auto pv = [&](int t, int u, bool acc) {
+        const uint32_t v_addr = smem_u32(sV + (u % STG) * Sh::KV_BYTES);
 #pragma unroll
         for (int k = 0; k < BKV / 16; ++k) {
           const uint64_t vd = sdesc(v_addr + k * 16 * Sh::ROW_BYTES, Sh::ATOM, Sh::ATOM, Sh::SW);
           mma_bf16_ts(tmem + Sh::T_O + 64 * t, tmem + Sh::T_S + BKV * t + 8 * k, vd, id_pv,
-                      (j > 0 || k > 0) ? 1u : 0u);
+                      (acc || k > 0) ? 1u : 0u);
         }
       };
       bool ok = mbar_wait(q_ready, 0, abort_flag);
-      ok = ok && mbar_wait(kv_full, 0, abort_flag);
-      if (ok) {
-        tc_fence_after();
-        for (int t = 0; t < n_t; ++t) qk(t, 0);
-      }
-      for (int j = 0; j < nkv && ok; ++j) {
-        const bool more = j + 1 < nkv;
-        for (int t = 0; t < n_t && ok; ++t) {
-          if (!mbar_wait(p_full + t, j & 1, abort_flag)) { ok = false; break; }
+      for (int t = 0; t < n_t && ok; ++t) {
+        const int u = seq(t, 0);
+        if (t == 0 || split) ok = mbar_wait(kv_full + u % STG, (u / STG) & 1, abort_flag);
+        if (ok) {
           tc_fence_after();
-          pv(t, j);
-          if (t == n_t - 1) mma_commit(kv_empty + j % STG);   // every P V of key tile j issued
-          if (more) {
-            if (t == 0 && !mbar_wait(kv_full + (j + 1) % STG, ((j + 1) / STG) & 1, abort_flag)) { ok = false; break; }
+          qk(t, u);
+        }
+      }
+      const int n_it = iters(0);               // group A has at least as many key tiles as B
+      for (int i = 0; i < n_it && ok; ++i) {
+        for (int t = 0; t < n_t && ok; ++t) {
+          if (i >= iters(t)) continue;
+          const int u = seq(t, i);
+          if (!mbar_wait(p_full + t, i & 1, abort_flag)) { ok = false; break; }
+          tc_fence_after();
+          pv(t, u, i > 0);
+          // a key tile is released once every product that reads it is issued
+          if (split || t == n_t - 1) mma_commit(kv_empty + u % STG);
+          if (i + 1 < iters(t)) {
+            const int un = seq(t, i + 1);
+            if ((t == 0 || split) && !mbar_wait(kv_full + un % STG, (un / STG) & 1, abort_flag)) {
+              ok = false;
+              break;
+            }
             tc_fence_after();
-            qk(t, j + 1);
+            qk(t, un);
           } else {
             mma_commit(o_done + t);
           }
@@ -661,7 +723,7 @@ __global__ void __launch_bounds__(PAIR_THREADS, 1)
     {
     const int qw = warp & 3;                  // TMEM lane quarter
     const int m = qw * 32 + lane;
-    const int j_q = (qp * 2 + t) * BQ + m;     // query index within the request
+    const int j_q = (tile0 + (split ? 0 : t)) * BQ + m;   // query index within the request
     const bool valid = j_q < n_q;
     const long long grow = j_q < M ? static_cast<long long>(c0) + j_q
                                    : a.n_cand + static_cast<long long>(r) * a.S + (j_q - M);
@@ -685,40 +747,57 @@ __global__ void __launch_bounds__(PAIR_THREADS, 1)
     const uint32_t t_o = tmem + Sh::T_O + 64 * t + lane_off;
     float m_run = -INFINITY, l_run = 0.f;
     bool ok = true;
-    for (int j = 0; j < nkv && ok; ++j) {
+    const int n_it = iters(t);
+    for (int j = 0; j < n_it && ok; ++j) {
       ok = mbar_wait(s_full + t, j & 1, abort_flag);
       ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
       if (!ok) break;
       tc_fence_after();
-      const int kbase = j * BKV;
+      const int kbase = key_tile(t, j) * BKV;
       const bool ragged = kbase + BKV > len;     // uniform
-      // row max over both halves of 64 keys (a half at a time keeps the
-      // register count within the file at 320 threads)
-      float mx = -INFINITY;
+      // the whole score row in registers: one TMEM load, one wait
+      float sv[BKV];
+      tmem_ld128(t_s, sv);
+      if (ragged) {
 #pragma unroll
-      for (int half = 0; half < 2; ++half) {
-        float sv[64];
-        tmem_ld64(t_s + 64 * half, sv);
-        if (ragged) {
-#pragma unroll
-          for (int i = 0; i < 64; ++i)
-            if (kbase + 64 * half + i >= len) sv[i] = -INFINITY;
-        }
-        float mx8[8];
-#pragma unroll
-        for (int i = 0; i < 8; ++i) mx8[i] = sv[i];
-#pragma unroll
-        for (int i = 8; i < 64; ++i) mx8[i & 7] = fmaxf(mx8[i & 7], sv[i]);
-#pragma unroll
-        for (int w = 4; w >= 1; w >>= 1)
-#pragma unroll
-          for (int i = 0; i < w; ++i) mx8[i] = fmaxf(mx8[i], mx8[i + w]);
-        mx = fmaxf(mx, mx8[0]);
+        for (int i = 0; i < BKV; ++i)
+          if (kbase + i >= len) sv[i] = -INFINITY;
       }
-      const float m_tile = mx * a.scale_log2;
-      if (__any_sync(0xffffffffu, m_tile > m_run + kRescaleLog2)) {
+      float mx4[4] = {sv[0], sv[1], sv[2], sv[3]};
+#pragma unroll
+      for (int i = 4; i < BKV; i += 2) mx4[(i >> 1) & 3] = fmax3(mx4[(i >> 1) & 3], sv[i], sv[i + 1]);
+      const float m_tile = fmax3(fmax3(mx4[0], mx4[1], mx4[2]), mx4[3], -INFINITY) * a.scale_log2;
+      const bool rescale = __any_sync(0xffffffffu, m_tile > m_run + kRescaleLog2);
+      float alpha = 1.f;
+      if (rescale) {
         const float m_new = fmaxf(m_run, m_tile);
-        const float alpha = ex2(m_run - m_new);   // 0 on the first tile
+        alpha = ex2(m_run - m_new);                // 0 on the first tile
+        m_run = m_new;
+      }
+      // P (bf16 pairs) over the first 64 columns of S, which is wholly in
+      // registers by now; scale-and-shift and the row sum two lanes at a time.
+      // Partial sums by key index mod 8, reduced as a fixed tree.  O is
+      // rescaled after P is formed (the score registers are free by then);
+      // P V(j) waits for p_full, which follows both.
+      const float2 sc2 = make_float2(a.scale_log2, a.scale_log2);
+      const float2 nm2 = make_float2(-m_run, -m_run);
+      float2 ps[4];
+#pragma unroll
+      for (int i = 0; i < 4; ++i) ps[i] = make_float2(0.f, 0.f);
+#pragma unroll
+      for (int c32 = 0; c32 < BKV; c32 += 32) {
+        uint32_t pk[16];
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+          const float2 x = ffma2(make_float2(sv[c32 + 2 * i], sv[c32 + 2 * i + 1]), sc2, nm2);
+          const float2 p = make_float2(ex2(x.x), ex2(x.y));
+          ps[i & 3] = fadd2(ps[i & 3], p);
+          __nv_bfloat162 h2 = __floats2bfloat162_rn(p.x, p.y);
+          pk[i] = *reinterpret_cast<uint32_t*>(&h2);
+        }
+        tmem_st16(t_s + c32 / 2, pk);
+      }
+      if (rescale) {
         if (j >= 1) {                              // O holds P V up to j - 1 (complete: S_t(j) is)
 #pragma unroll
           for (int cc = 0; cc < DH; cc += 32) {
@@ -730,51 +809,52 @@ __global__ void __launch_bounds__(PAIR_THREADS, 1)
           }
         }
         l_run *= alpha;
-        m_run = m_new;
-      }
-      // P half by half over the first 64 columns of S: half 0 (keys 0-63)
-      // lands on columns 0-31, read already; half 1 is read before its P
-      // lands on columns 32-63
-      float ps8[8];
-#pragma unroll
-      for (int i = 0; i < 8; ++i) ps8[i] = 0.f;
-#pragma unroll
-      for (int half = 0; half < 2; ++half) {
-        float sv[64];
-        tmem_ld64(t_s + 64 * half, sv);
-        if (ragged) {
-#pragma unroll
-          for (int i = 0; i < 64; ++i)
-            if (kbase + 64 * half + i >= len) sv[i] = -INFINITY;
-        }
-#pragma unroll
-        for (int c32 = 0; c32 < 64; c32 += 32) {
-          uint32_t pk[16];
-#pragma unroll
-          for (int i = 0; i < 32; i += 2) {
-            const float p0 = ex2(fmaf(sv[c32 + i], a.scale_log2, -m_run));
-            const float p1 = ex2(fmaf(sv[c32 + i + 1], a.scale_log2, -m_run));
-            ps8[i & 7] += p0;
-            ps8[(i + 1) & 7] += p1;
-            __nv_bfloat162 h2 = __floats2bfloat162_rn(p0, p1);
-            pk[i / 2] = *reinterpret_cast<uint32_t*>(&h2);
-          }
-          tmem_st16(t_s + 32 * half + c32 / 2, pk);
-        }
       }
       tmem_wait_st();
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(p_full + t);
-#pragma unroll
-      for (int w = 4; w >= 1; w >>= 1)
-#pragma unroll
-        for (int i = 0; i < w; ++i) ps8[i] += ps8[i + w];
-      l_run += ps8[0];
+      ps[0] = fadd2(ps[0], ps[2]);
+      ps[1] = fadd2(ps[1], ps[3]);
+      ps[0] = fadd2(ps[0], ps[1]);
+      l_run += ps[0].x + ps[0].y;
     }
     if (ok) {
       ok = mbar_wait(o_done + t, 0, abort_flag);
       ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
+    }
+    // split keys: group B hands its partial state (O, running max, row sum)
+    // to group A, which merges the two.  Both groups reach the named barrier
+    // on every path, failed waits included.
+    float f_a = 1.f, f_b = 0.f;
+    if (split) {
+      if (t == 1) {
+        if (ok) {
+          tc_fence_after();
+#pragma unroll
+          for (int cc = 0; cc < DH; cc += 32) {
+            float ov[32];
+            tmem_ld32(t_o + cc, ov);
+#pragma unroll
+            for (int i = 0; i < 32; ++i) xo[m * Sh::XSTRIDE + cc + i] = ov[i];
+          }
+          xm[m] = m_run;
+          xl[m] = l_run;
+        } else {
+          xl[m] = -1.f;                      // no partial state: group A stores nothing
+        }
+      }
+      asm volatile("bar.sync 1, 256;" ::: "memory");
+      if (t == 1) goto done;
+      ok = ok && xl[m] >= 0.f;
+      ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
+      if (ok) {
+        const float m_b = xm[m];
+        const float m_all = fmaxf(m_run, m_b);
+        f_a = ex2(m_run - m_all);
+        f_b = ex2(m_b - m_all);
+        l_run = l_run * f_a + xl[m] * f_b;
+      }
     }
     if (ok) {
       tc_fence_after();
@@ -784,6 +864,10 @@ __global__ void __launch_bounds__(PAIR_THREADS, 1)
       for (int cc = 0; cc < DH; cc += 32) {
         float ov[32];
         tmem_ld32(t_o + cc, ov);
+        if (split) {
+#pragma unroll
+          for (int i = 0; i < 32; ++i) ov[i] = ov[i] * f_a + xo[m * Sh::XSTRIDE + cc + i] * f_b;
+        }
         if (valid) {
 #pragma unroll
           for (int c = 0; c < 32; c += 8) {
@@ -1263,12 +1347,13 @@ cudaError_t launch_fa_full(const __nv_bfloat16* q, __nv_bfloat16* out, const __n
   if (Hkv < 1 || H % Hkv) return cudaErrorInvalidValue;
   const int dh = d / H;
   fa::FaArgs a{q, out, cand_off_dev, kv_off, kv_len, n_cand, S, d, H / Hkv,
-               1.4426950408889634f / sqrtf(static_cast<float>(dh)), status};
+               1.4426950408889634f / sqrtf(static_cast<float>(dh)), status, 2};
   const int tiles = (max_q + fa::BQ - 1) / fa::BQ;
   prof_begin(KC_ATTN_CROSS, s);
   cudaError_t err;
-  // two query tiles per CTA share each K/V tile, when the pairs still fill
-  // the GPU (a single request would otherwise leave most SMs idle)
+  // two query tiles per CTA share each K/V tile when the pairs still fill
+  // the GPU; otherwise (few requests: a single request would leave most SMs
+  // idle) one query tile per CTA, its key tiles split over the two groups
   static int sms = 0;
   if (!sms) {
     int dev = 0;
@@ -1277,14 +1362,10 @@ cudaError_t launch_fa_full(const __nv_bfloat16* q, __nv_bfloat16* out, const __n
       sms = 152;
   }
   const long long pair_ctas = static_cast<long long>((tiles + 1) / 2) * n_req * H;
-  if (tiles >= 2 && pair_ctas >= 2LL * sms) {
-    const int pairs = (tiles + 1) / 2;
-    err = dh == 64 ? fa::launch_pair_dh<64>(a, Kc, Vc, cap_total, n_req, pairs, H, Hkv * dh, s)
-                   : fa::launch_pair_dh<32>(a, Kc, Vc, cap_total, n_req, pairs, H, Hkv * dh, s);
-  } else {
-    err = dh == 64 ? fa::launch_dh<64>(a, Kc, Vc, cap_total, n_req, tiles, H, Hkv * dh, s)
-                   : fa::launch_dh<32>(a, Kc, Vc, cap_total, n_req, tiles, H, Hkv * dh, s);
-  }
+  a.tiles_per_cta = tiles >= 2 && pair_ctas >= 2LL * sms ? 2 : 1;
+  const int grid_x = (tiles + a.tiles_per_cta - 1) / a.tiles_per_cta;
+  err = dh == 64 ? fa::launch_pair_dh<64>(a, Kc, Vc, cap_total, n_req, grid_x, H, Hkv * dh, s)
+                 : fa::launch_pair_dh<32>(a, Kc, Vc, cap_total, n_req, grid_x, H, Hkv * dh, s);
   prof_end(KC_ATTN_CROSS, s);
   return err;
 }

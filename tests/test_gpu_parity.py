@@ -87,6 +87,22 @@ def test_full_size_sampled_requests(name, mode):
     np.testing.assert_allclose(g.probs.sum(1), 1.0, atol=1e-5)
 
 
+@pytest.mark.parametrize("name", ["small_bf16", "mid_bf16"])
+def test_full_attention_lone_query_tiles(name):
+    # FULL mode with enough requests for two query tiles per CTA: slates of
+    # 252..259 candidates (+ 2 context rows) leave the last query tile of
+    # most requests alone in its CTA, which then splits the request's key
+    # tiles over its two softmax groups and merges them; histories of one key
+    # tile (no split), two, an odd number and ragged last tiles
+    L = [100, 129, 300, 1000, 257, 128, 640, 385] * 3
+    M = [252 + (r % 8) for r in range(24)]
+    wl = W.with_sizes(W.WORKLOADS[name], n_req=24, n_layers=1, L=L, M=M)
+    g = run_gpu(wl, txs.FULL)
+    lg, pr, _, _ = oracle_scores(wl, txs.FULL)
+    assert_scores_close(g.logits, lg, wl.dtype, f"{name} logits")
+    assert_scores_close(g.probs, pr, wl.dtype, f"{name} probs")
+
+
 @pytest.mark.parametrize("M", [64, 256, 1024, 4096])
 def test_sweep_candidate_counts(M):
     wl = W.WORKLOADS["sweep_bf16"]
