@@ -1,21 +1,21 @@
-// Multi-query cross-attention over all cached rows of a request on the tensor
-// cores (FULL key set: the -sparseAttn variant of Sec. 5.2; sparse
-// cross-attention equation of Sec. 4.1.2 with I = every behavior row).
-//
-// One CTA per (query tile of 128 rows, request r, head h).  All M_r + S query
-// rows of request r share the request's K/V (Sec. 4.1.2 multi-query
-// formulation), so each 128-key K/V tile is staged once per CTA by TMA and
-// serves all 128 queries:
-//   warp 0     TMA producer: K_j, V_j tiles of the request (head h columns)
-//              into a STG-deep shared-memory ring;
-//   warp 1     MMA issuer: S_j = Q K_j^T into one of two TMEM buffers, then
-//              O += P_j V_j into the TMEM output tile.  Q and P are the A
-//              operands and are read from TMEM, so the tensor core reads only
-//              K and V from shared memory (V used MN-major: no transpose);
-//   warps 2-5  softmax: one query row per thread straight out of TMEM (row
-//              max, exp2, row sum need no shuffles); P_j (bf16) goes back to
-//              one of two TMEM buffers, so the exponentials of tile j overlap
-//              the PV product of tile j - 1.
+// Attention on the tensor cores (tcgen05, TMA, TMEM):
+//   fa_pair_kernel  multi-query cross-attention over all cached rows of a
+//                   request (FULL key set: the -sparseAttn variant of
+//                   Sec. 5.2; sparse cross-attention equation of Sec. 4.1.2
+//                   with I = every behavior row);
+//   enc_fa_kernel   causal self-attention of the behavior encoder with a
+//                   relative position bias (Sec. 4.1.1, App. D).
+// Both follow one pipeline.  All query rows of a request (or of a user)
+// share its K/V (Sec. 4.1.2 multi-query formulation), so each 128-key K/V
+// tile is staged once per CTA and serves every query row of the CTA:
+//   warp 0     TMA producer: K_j, V_j tiles (one head's columns) into a
+//              STG-deep shared-memory ring;
+//   warp 1     MMA issuer: S_j = Q K_j^T into TMEM, then O += P_j V_j into
+//              the TMEM output tile.  Q and P are the A operands and are read
+//              from TMEM, so the tensor core reads only K and V from shared
+//              memory (V used MN-major: no transpose);
+//   softmax    one query row per thread straight out of TMEM (row max,
+//              exp2, row sum need no shuffles); P_j (bf16) goes back to TMEM.
 // The running maximum is raised only when a tile's maximum exceeds it by more
 // than 2^8 (then O and the row sum are rescaled in place); otherwise the
 // stale maximum is kept, P stays below 256 and no rescale is needed.  Exact
@@ -260,9 +260,11 @@ struct FaArgs {
   int group;                  // query heads per K/V head
   float scale_log2;           // log2(e) / sqrt(d_h)
   int* status;
-  int tiles_per_cta;          // fa_pair_kernel: 2 (query-tile pairs) or 1 (every tile splits its keys)
+  int tiles_per_cta;          // 2 (query-tile pairs) or 1 (every tile splits its keys)
 };
 
+// Shared-memory ring and TMEM layout of enc_fa_kernel (one 128-row query tile
+// per CTA, two S and two P buffers).
 template <int DH>
 struct FaShape {
   static constexpr int ROW_BYTES = DH * 2;                  // 64 or 128: one swizzle row
@@ -276,266 +278,6 @@ struct FaShape {
   static constexpr int TMEM_COLS = 512;
   static_assert(T_O + DH <= T_P && T_Q + DH / 2 <= TMEM_COLS, "TMEM columns");
 };
-
-template <int DH>
-__global__ void __launch_bounds__(NUM_THREADS, 1)
-    fa_full_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV, const FaArgs a) {
-  using Sh = FaShape<DH>;
-  extern __shared__ uint8_t smem_raw[];
-  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  uint8_t* sK = smem;
-  uint8_t* sV = sK + STG * Sh::KV_BYTES;
-  uint64_t* bars = reinterpret_cast<uint64_t*>(sV + STG * Sh::KV_BYTES);
-  uint64_t* kv_full = bars;
-  uint64_t* kv_empty = kv_full + STG;
-  uint64_t* s_full = kv_empty + STG;    // [2] S_j in TMEM buffer j % 2
-  uint64_t* s_free = s_full + 2;        // [2] the softmax warps have read it
-  uint64_t* p_full = s_free + 2;        // [2] P_j in TMEM buffer j % 2
-  uint64_t* pv_done = p_full + 2;       // [2] O += P_j V_j complete
-  uint64_t* q_ready = pv_done + 2;
-  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(q_ready + 1);
-  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_holder + 1);
-
-  pdl_launch_dependents();
-  pdl_wait();
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int qt = blockIdx.x, r = blockIdx.y, h = blockIdx.z;
-  const int c0 = a.cand_off[r];
-  const int M = a.cand_off[r + 1] - c0;
-  const int n_q = M + a.S;
-  if (qt * BQ >= n_q) return;                       // uniform: no tile here
-  const int len = a.kv_len[r];
-  const int kv0 = a.kv_off[r];
-  const int nkv = (len + BKV - 1) / BKV;
-  if (nkv <= 0) {                                   // a built cache never has an empty request
-    if (threadIdx.x == 0) latch_status(a.status, TXS_ERR_BOUNDS);
-    return;
-  }
-
-  if (threadIdx.x == 0) {
-    for (int s = 0; s < STG; ++s) {
-      mbar_init(kv_full + s, 1);
-      mbar_init(kv_empty + s, 1);
-    }
-    for (int b = 0; b < 2; ++b) {
-      mbar_init(s_full + b, 1);
-      mbar_init(s_free + b, 4);
-      mbar_init(p_full + b, 4);
-      mbar_init(pv_done + b, 1);
-    }
-    mbar_init(q_ready, 4);
-    *abort_flag = 0;
-    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-  }
-  if (warp == 1) tmem_alloc(tmem_holder, Sh::TMEM_COLS);
-  tc_fence_before();
-  __syncthreads();
-  tc_fence_after();
-  const uint32_t tmem = *tmem_holder;
-
-  if (warp == 0) {
-    if (lane == 0) {
-      asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmK)) : "memory");
-      asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmV)) : "memory");
-      int issued = 0;
-      for (int j = 0; j < nkv; ++j) {
-        const int st = j % STG;
-        if (!mbar_wait(kv_empty + st, ((j / STG) & 1) ^ 1, abort_flag)) break;
-        mbar_expect_tx(kv_full + st, 2 * Sh::KV_BYTES);
-        tma_load_2d(sK + st * Sh::KV_BYTES, &tmK, kv_full + st, (h / a.group) * DH, kv0 + j * BKV);
-        tma_load_2d(sV + st * Sh::KV_BYTES, &tmV, kv_full + st, (h / a.group) * DH, kv0 + j * BKV);
-        issued = j + 1;
-      }
-      if (*abort_flag)
-        for (int k = issued > STG ? issued - STG : 0; k < issued; ++k)
-          mbar_wait_plain(kv_full + k % STG, (k / STG) & 1);
-    }
-  } else if (warp == 1) {
-    if (lane == 0) {
-      constexpr uint32_t id_s = idesc_bf16(BQ, BKV, false);
-      constexpr uint32_t id_pv = idesc_bf16(BQ, DH, true);
-      bool ok = mbar_wait(q_ready, 0, abort_flag);
-      tc_fence_after();
-      // O += P_t V_t, after the softmax warps have written P_t (and rescaled O
-      // if they had to)
-      auto pv = [&](int t) -> bool {
-        const int bt = t & 1, st = t % STG;
-        if (!mbar_wait(p_full + bt, (t >> 1) & 1, abort_flag)) return false;
-        tc_fence_after();
-        const uint32_t v_addr = smem_u32(sV + st * Sh::KV_BYTES);
-#pragma unroll
-        for (int k = 0; k < BKV / 16; ++k) {
-          // V (MN-major): 16 keys = two 8-row atoms of the tile
-          const uint64_t vd = sdesc(v_addr + k * 16 * Sh::ROW_BYTES, Sh::ATOM, Sh::ATOM, Sh::SW);
-          mma_bf16_ts(tmem + Sh::T_O, tmem + Sh::T_P + 64 * bt + 8 * k, vd, id_pv, (t > 0 || k > 0) ? 1u : 0u);
-        }
-        mma_commit(pv_done + bt);
-        mma_commit(kv_empty + st);
-        return true;
-      };
-      for (int j = 0; j < nkv && ok; ++j) {
-        const int st = j % STG, b = j & 1;
-        if (!mbar_wait(kv_full + st, (j / STG) & 1, abort_flag)) break;
-        if (!mbar_wait(s_free + b, ((j >> 1) & 1) ^ 1, abort_flag)) break;
-        tc_fence_after();
-        const uint32_t k_addr = smem_u32(sK + st * Sh::KV_BYTES);
-#pragma unroll
-        for (int k = 0; k < DH / 16; ++k) {
-          const uint64_t kd = sdesc(k_addr + k * 32, 16, Sh::ATOM, Sh::SW);
-          mma_bf16_ts(tmem + Sh::T_S + BKV * b, tmem + Sh::T_Q + 8 * k, kd, id_s, k > 0 ? 1u : 0u);
-        }
-        mma_commit(s_full + b);
-        if (j >= 1) ok = pv(j - 1);
-      }
-      if (ok && !*abort_flag) pv(nkv - 1);
-    }
-  } else {
-    // ---------------- softmax warps: one query row per thread
-    const int qw = warp & 3;                  // TMEM lane quarter
-    const int m = qw * 32 + lane;             // row of the tile
-    const int j_q = qt * BQ + m;              // query index within the request
-    const bool valid = j_q < n_q;
-    const long long grow = j_q < M ? static_cast<long long>(c0) + j_q
-                                   : a.n_cand + static_cast<long long>(r) * a.S + (j_q - M);
-    const uint32_t lane_off = static_cast<uint32_t>(qw * 32) << 16;
-    // this row's head slice of Q into TMEM (bf16 pairs)
-    {
-      uint32_t qv[DH / 2];
-      const uint4* src = reinterpret_cast<const uint4*>(a.q + (valid ? grow : 0) * a.d + h * DH);
-#pragma unroll
-      for (int c = 0; c < DH / 8; ++c) {
-        const uint4 v = valid ? src[c] : make_uint4(0, 0, 0, 0);
-        qv[4 * c] = v.x; qv[4 * c + 1] = v.y; qv[4 * c + 2] = v.z; qv[4 * c + 3] = v.w;
-      }
-#pragma unroll
-      for (int c = 0; c < DH / 2; c += 16) tmem_st16(tmem + Sh::T_Q + c + lane_off, qv + c);
-      tmem_wait_st();
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(q_ready);
-    }
-    const uint32_t t_o = tmem + Sh::T_O + lane_off;
-    float m_run = -INFINITY, l_run = 0.f;     // running max (log2 units, scaled), row sum
-    bool ok = true;
-    for (int j = 0; j < nkv && ok; ++j) {
-      const int b = j & 1;
-      ok = mbar_wait(s_full + b, (j >> 1) & 1, abort_flag);
-      ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
-      if (!ok) break;
-      tc_fence_after();
-      // the whole score row of this tile in one TMEM load; the buffer is free
-      // for S_{j+2} as soon as it is in registers
-      float sv[BKV];
-      tmem_ld128(tmem + Sh::T_S + BKV * b + lane_off, sv);
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(s_free + b);
-      const int kbase = j * BKV;
-      if (kbase + BKV > len) {                   // ragged last tile (uniform)
-#pragma unroll
-        for (int i = 0; i < BKV; ++i)
-          if (kbase + i >= len) sv[i] = -INFINITY;
-      }
-      // row max in 8 independent chains
-      float mx8[8];
-#pragma unroll
-      for (int i = 0; i < 8; ++i) mx8[i] = sv[i];
-#pragma unroll
-      for (int i = 8; i < BKV; ++i) mx8[i & 7] = fmaxf(mx8[i & 7], sv[i]);
-#pragma unroll
-      for (int w = 4; w >= 1; w >>= 1)
-#pragma unroll
-        for (int i = 0; i < w; ++i) mx8[i] = fmaxf(mx8[i], mx8[i + w]);
-      const float m_tile = mx8[0] * a.scale_log2;
-      if (__any_sync(0xffffffffu, m_tile > m_run + kRescaleLog2)) {
-        const float m_new = fmaxf(m_run, m_tile);
-        const float alpha = ex2(m_run - m_new);  // 0 on the first tile
-        if (j >= 1) {
-          // O holds P_0..P_{j-1} V: rescale it once PV(j-1) is complete
-          ok = mbar_wait(pv_done + ((j - 1) & 1), ((j - 1) >> 1) & 1, abort_flag);
-          ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
-          if (!ok) break;
-          tc_fence_after();
-#pragma unroll
-          for (int cc = 0; cc < DH; cc += 32) {
-            float ov[32];
-            tmem_ld32(t_o + cc, ov);
-#pragma unroll
-            for (int i = 0; i < 32; ++i) ov[i] *= alpha;
-            tmem_st32(t_o + cc, ov);
-          }
-        }
-        l_run *= alpha;
-        m_run = m_new;
-      }
-      // P buffer b was last read by PV(j - 2)
-      if (j >= 2) {
-        ok = mbar_wait(pv_done + b, ((j - 2) >> 1) & 1, abort_flag);
-        ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
-        if (!ok) break;
-        tc_fence_after();
-      }
-      // P = 2^(s * scale - m_run) as bf16 pairs into TMEM buffer b, row sum
-      const uint32_t t_p = tmem + Sh::T_P + 64 * b + lane_off;
-      float ps8[8];
-#pragma unroll
-      for (int i = 0; i < 8; ++i) ps8[i] = 0.f;
-#pragma unroll
-      for (int c32 = 0; c32 < BKV; c32 += 32) {
-        uint32_t pk[16];
-#pragma unroll
-        for (int i = 0; i < 32; i += 2) {
-          const float p0 = ex2(fmaf(sv[c32 + i], a.scale_log2, -m_run));
-          const float p1 = ex2(fmaf(sv[c32 + i + 1], a.scale_log2, -m_run));
-          ps8[i & 7] += p0;
-          ps8[(i + 1) & 7] += p1;
-          __nv_bfloat162 h2 = __floats2bfloat162_rn(p0, p1);      // lower key in the low half
-          pk[i / 2] = *reinterpret_cast<uint32_t*>(&h2);
-        }
-        tmem_st16(t_p + c32 / 2, pk);
-      }
-      tmem_wait_st();
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(p_full + b);
-#pragma unroll
-      for (int w = 4; w >= 1; w >>= 1)
-#pragma unroll
-        for (int i = 0; i < w; ++i) ps8[i] += ps8[i + w];
-      l_run += ps8[0];
-    }
-    if (ok) {
-      ok = mbar_wait(pv_done + ((nkv - 1) & 1), ((nkv - 1) >> 1) & 1, abort_flag);
-      ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
-    }
-    if (ok) {
-      tc_fence_after();
-      const float inv = 1.f / l_run;
-      __nv_bfloat16* dst = a.out + grow * a.d + h * DH;
-#pragma unroll
-      for (int cc = 0; cc < DH; cc += 32) {
-        float ov[32];
-        tmem_ld32(t_o + cc, ov);
-        if (valid) {
-#pragma unroll
-          for (int c = 0; c < 32; c += 8) {
-            float t[8];
-#pragma unroll
-            for (int i = 0; i < 8; ++i) t[i] = ov[c + i] * inv;
-            Vec16<__nv_bfloat16>::store(dst + cc + c, t);
-          }
-        }
-      }
-    }
-  }
-  tc_fence_before();
-  __syncthreads();
-  if (warp == 1) {
-    tc_fence_after();
-    tmem_dealloc(tmem, Sh::TMEM_COLS);
-  }
-  if (threadIdx.x == 0 && *abort_flag) latch_status(a.status, TXS_ERR_DEVICE_TIMEOUT);
-}
 
 // ------------------------------------------------------------------ two query tiles per CTA
 
@@ -556,8 +298,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
 // (a two-part form of the same online softmax).  The softmax holds a whole score row
 // (128 keys) in registers after one TMEM load, takes its maximum with
 // three-source max and forms the exponent arguments and row sums two lanes at
-// a time (f32x2 arithmetic).  Online softmax with the stale-maximum rule of
-// fa_full_kernel.
+// a time (f32x2 arithmetic).  Online softmax with the stale-maximum rule
+// described at the top of this file.
 constexpr int PAIR_THREADS = 320;
 
 template <int DH>
@@ -897,8 +639,9 @@ done:
 // a relative position bias) for the new rows of each user against that
 // user's cached keys/values of the same layer (App. D incremental encoding;
 // a build is the case "every row is new").  One CTA per (tile of up to 128
-// new rows of one user, head); the same producer / MMA / softmax pipeline as
-// fa_full_kernel, with:
+// new rows of one user, head); the pipeline described at the top of this
+// file with 4 softmax warps, two S buffers and two P buffers in TMEM (the
+// exponentials of key tile j overlap the products of tile j + 1), and:
 //   * key tiles of 128 positions aligned to multiples of 128 of the user's
 //     own position axis (tile jj holds positions 128 jj ...), from the tile
 //     of the first row's earliest visible key to the tile of the last row;
@@ -1257,23 +1000,6 @@ static bool make_kv_map(CUtensorMap* tm, const void* base, long long rows, int d
   return fn(tm, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
             CU_TENSOR_MAP_INTERLEAVE_NONE, DH == 64 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_64B,
             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
-}
-
-template <int DH>
-static cudaError_t launch_dh(const FaArgs& a, const void* Kc, const void* Vc, long long cap_total, int n_req,
-                             int max_q_tiles, int H, int dkv, cudaStream_t s) {
-  using Sh = FaShape<DH>;
-  static bool attr = false;
-  if (!attr) {
-    cudaError_t e = cudaFuncSetAttribute(fa_full_kernel<DH>, cudaFuncAttributeMaxDynamicSharedMemorySize, Sh::SMEM);
-    if (e != cudaSuccess) return e;
-    attr = true;
-  }
-  CUtensorMap tk, tv;
-  if (!make_kv_map<DH>(&tk, Kc, cap_total, dkv) || !make_kv_map<DH>(&tv, Vc, cap_total, dkv))
-    return cudaErrorInvalidValue;
-  const dim3 grid(max_q_tiles, n_req, H);
-  return launch_pdl(fa_full_kernel<DH>, grid, dim3(NUM_THREADS), Sh::SMEM, s, tk, tv, a);
 }
 
 template <int DH>
