@@ -39,10 +39,36 @@ __device__ __forceinline__ int find_segment_param(const int* off, int n, int row
 
 constexpr int kPackRowsPerWarp = 2;
 
-// 8 warps per CTA, kPackRowsPerWarp rows per warp.  W_eff_x is staged once per
-// CTA in shared memory as [action][column] so that a lane's 16-byte slice of a
-// row meets contiguous weights.
-template <typename T>
+// Sum of NA per-lane values over the 32 lanes of a warp, scattered: on return
+// every lane holds the total of value lane / (32 / NA).  Each halving step
+// exchanges half of the remaining values with the partner lane (NA - 1
+// shuffles in all), then the lanes that share a value finish with a butterfly.
+template <int NA>
+__device__ __forceinline__ float warp_reduce_scatter(float (&v)[NA], int lane) {
+#pragma unroll
+  for (int h = NA / 2, o = 16; h >= 1; h >>= 1, o >>= 1) {
+    const bool upper = (lane & o) != 0;
+#pragma unroll
+    for (int i = 0; i < h; ++i) {
+      const float send = upper ? v[i] : v[i + h];
+      const float keep = upper ? v[i + h] : v[i];
+      v[i] = keep + __shfl_xor_sync(0xffffffffu, send, o);
+    }
+  }
+  float x = v[0];
+#pragma unroll
+  for (int o = 16 / NA; o >= 1; o >>= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
+  return x;
+}
+
+// 8 warps per CTA, kPackRowsPerWarp consecutive rows per warp (all of a
+// warp's row loads are issued before its arithmetic); CH 16-byte chunks per
+// lane and row cover d.  The x-part of the
+// logits takes NA >= na actions (the actions na..NA-1 have zero weights and
+// are not written); a lane's head weights for its columns are loaded once, to
+// registers when NA <= 4, else staged per CTA in shared memory as
+// [action][column].
+template <typename T, int NA, int CH>
 __global__ void __launch_bounds__(256) pack_kernel(const __grid_constant__ PackArgs a, const T* __restrict__ cand,
                                                    const T* __restrict__ ctx, T* __restrict__ X,
                                                    int* __restrict__ row_req, int* __restrict__ cand_off_dev,
@@ -51,64 +77,95 @@ __global__ void __launch_bounds__(256) pack_kernel(const __grid_constant__ PackA
   pdl_launch_dependents();
   pdl_wait();
   constexpr int VEC = Vec16<T>::N;
-  extern __shared__ float sw[];                 // [na][d]
+  constexpr int MAXCH = CH;
+  constexpr bool kRegW = NA <= 4;
+  extern __shared__ float sw[];                 // [NA][d] when !kRegW
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int d = a.d, na = a.na;
   if (blockIdx.x == 0)
     for (int i = threadIdx.x; i <= a.n_req; i += 256) cand_off_dev[i] = a.cand_off[i];
-  for (int i = threadIdx.x; i < d * na; i += 256) {
-    const int c = i / na, k = i - c * na;       // weff_x is [d][na]
-    sw[k * d + c] = weff_x[i];
-  }
-  __syncthreads();
   const long long n_rows = a.n_cand + static_cast<long long>(a.n_req) * a.S;
   const long long p0 = (static_cast<long long>(blockIdx.x) * 8 + warp) * kPackRowsPerWarp;
+  uint4 raw[kPackRowsPerWarp][MAXCH];
+#pragma unroll
   for (int t = 0; t < kPackRowsPerWarp; ++t) {
     const long long p = p0 + t;
-    if (p >= n_rows) return;
-    int r;
-    const T* src;
-    const bool is_cand = p < a.n_cand;
-    if (is_cand) {
-      r = find_segment_param(a.cand_off, a.n_req, static_cast<int>(p));
-      src = cand + p * d;
-    } else {
-      const long long q = p - a.n_cand;
-      r = static_cast<int>(q / a.S);
-      src = ctx + q * d;
+    const T* src = p < a.n_cand ? cand + p * d : (p < n_rows ? ctx + (p - a.n_cand) * d : cand);
+#pragma unroll
+    for (int j = 0; j < MAXCH; ++j) {
+      const int col = (j * 32 + lane) * VEC;
+      raw[t][j] = (p < n_rows && col < d) ? *reinterpret_cast<const uint4*>(src + col) : make_uint4(0, 0, 0, 0);
     }
+  }
+  // head weights after the row loads are in flight: a lane's columns
+  // col..col+VEC-1 hold VEC * na consecutive floats of weff_x ([d][na])
+  float wr[kRegW ? MAXCH : 1][kRegW ? VEC : 1][NA];
+  if constexpr (kRegW) {
+#pragma unroll
+    for (int j = 0; j < MAXCH; ++j) {
+      const int col = (j * 32 + lane) * VEC;
+      if (na == NA && col < d) {
+        const float4* w4 = reinterpret_cast<const float4*>(weff_x + static_cast<long long>(col) * NA);
+#pragma unroll
+        for (int q = 0; q < VEC * NA / 4; ++q) {
+          const float4 f = __ldg(w4 + q);
+          const float e[4] = {f.x, f.y, f.z, f.w};
+#pragma unroll
+          for (int u = 0; u < 4; ++u) wr[j][(4 * q + u) / NA][(4 * q + u) % NA] = e[u];
+        }
+      } else {
+#pragma unroll
+        for (int i = 0; i < VEC; ++i)
+#pragma unroll
+          for (int k = 0; k < NA; ++k)
+            wr[j][i][k] = (col < d && k < na) ? __ldg(weff_x + static_cast<long long>(col + i) * na + k) : 0.f;
+      }
+    }
+  } else {
+    for (int c = threadIdx.x; c < d; c += 256)
+#pragma unroll
+      for (int k = 0; k < NA; ++k) sw[k * d + c] = k < na ? weff_x[static_cast<long long>(c) * na + k] : 0.f;
+    __syncthreads();
+  }
+#pragma unroll
+  for (int t = 0; t < kPackRowsPerWarp; ++t) {
+    const long long p = p0 + t;
+    if (p >= n_rows) break;                     // uniform over the warp
+    const bool is_cand = p < a.n_cand;
     T* dst = X + p * d;
-    float lg[16];
 #pragma unroll
-    for (int k = 0; k < 16; ++k) lg[k] = 0.f;
-    for (int c = lane * VEC; c < d; c += 32 * VEC) {
-      float v[VEC];
-      Vec16<T>::load(src + c, v);
-      Vec16<T>::store(dst + c, v);
-      if (is_cand) {
+    for (int j = 0; j < MAXCH; ++j) {
+      const int col = (j * 32 + lane) * VEC;
+      if (col < d) *reinterpret_cast<uint4*>(dst + col) = raw[t][j];
+    }
+    if (lane == 0)
+      row_req[p] = is_cand ? find_segment_param(a.cand_off, a.n_req, static_cast<int>(p))
+                           : static_cast<int>((p - a.n_cand) / a.S);
+    if (is_cand) {
+      float lg[NA];
 #pragma unroll
-        for (int k = 0; k < 16; ++k) {
-          if (k < na) {
-            const float* w = sw + k * d + c;
+      for (int k = 0; k < NA; ++k) lg[k] = 0.f;
+#pragma unroll
+      for (int j = 0; j < MAXCH; ++j) {
+        const int col = (j * 32 + lane) * VEC;
+        if (col < d) {
+          float v[VEC];
+          Vec16<T>::load(reinterpret_cast<const T*>(&raw[t][j]), v);
+#pragma unroll
+          for (int k = 0; k < NA; ++k) {
             float acc = 0.f;
 #pragma unroll
-            for (int i = 0; i < VEC; ++i) acc = fmaf(v[i], w[i], acc);
+            for (int i = 0; i < VEC; ++i) {
+              if constexpr (kRegW) acc = fmaf(v[i], wr[j][i][k], acc);
+              else acc = fmaf(v[i], sw[k * d + col + i], acc);
+            }
             lg[k] += acc;
           }
         }
       }
-    }
-    if (lane == 0) row_req[p] = r;
-    if (is_cand) {
-#pragma unroll
-      for (int k = 0; k < 16; ++k) {
-        if (k < na) {
-          float x = lg[k];
-#pragma unroll
-          for (int o = 16; o > 0; o >>= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
-          if (lane == 0) xlog[p * na + k] = x + __ldg(cdec + k);
-        }
-      }
+      const float x = warp_reduce_scatter<NA>(lg, lane);
+      const int k = lane / (32 / NA);
+      if ((lane & (32 / NA - 1)) == 0 && k < na) xlog[p * na + k] = x + __ldg(cdec + k);
     }
   }
 }
@@ -133,15 +190,41 @@ __global__ void __launch_bounds__(1024) rank_kernel(const __grid_constant__ Rank
   for (int i = threadIdx.x; i < M; i += blockDim.x)
     keys[i] = order_key(probs[static_cast<long long>(c0 + i) * a.na + a.action]);
   __syncthreads();
-  for (int i = threadIdx.x; i < M; i += blockDim.x) {
-    const uint32_t ki = keys[i];
+  // tpc consecutive lanes share a candidate (short slates leave threads to
+  // spare), each counting every tpc-th key with four independent counters;
+  // the group adds its counts with shuffles.  Every lane runs the same number
+  // of rounds, so the shuffles see full warps.
+  int tpc = 1;
+  while (tpc < 32 && tpc * 2 * M <= static_cast<int>(blockDim.x)) tpc *= 2;
+  const int per_round = blockDim.x / tpc;
+  const int sub = threadIdx.x & (tpc - 1);
+  const int rounds = (M + per_round - 1) / per_round;
+  for (int round = 0; round < rounds; ++round) {
+    const int i = round * per_round + static_cast<int>(threadIdx.x) / tpc;
     int rank = 0;
-    for (int j = 0; j < M; ++j) {
-      const uint32_t kj = keys[j];
-      rank += (kj > ki) | ((kj == ki) & (j < i));
+    if (i < M) {
+      const uint32_t ki = keys[i];
+      int c[4] = {0, 0, 0, 0};
+      int j = sub;
+      for (; j + 3 * tpc < M; j += 4 * tpc) {
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+          const int jj = j + u * tpc;
+          const uint32_t kj = keys[jj];
+          c[u] += (kj > ki) | ((kj == ki) & (jj < i));
+        }
+      }
+      for (; j < M; j += tpc) {
+        const uint32_t kj = keys[j];
+        c[0] += (kj > ki) | ((kj == ki) & (j < i));
+      }
+      rank = (c[0] + c[1]) + (c[2] + c[3]);
     }
-    if (a.top_k == 0) out[c0 + rank] = i;
-    else if (rank < a.top_k) out[static_cast<long long>(r) * a.top_k + rank] = i;
+    for (int o = tpc >> 1; o >= 1; o >>= 1) rank += __shfl_xor_sync(0xffffffffu, rank, o);
+    if (i < M && sub == 0) {
+      if (a.top_k == 0) out[c0 + rank] = i;
+      else if (rank < a.top_k) out[static_cast<long long>(r) * a.top_k + rank] = i;
+    }
   }
   if (a.top_k > 0)
     for (int t = M + threadIdx.x; t < a.top_k; t += blockDim.x) out[static_cast<long long>(r) * a.top_k + t] = -1;
@@ -296,6 +379,27 @@ cudaError_t launch_dw_head(const T* Hd, int Fh, const float* w2q, const float* x
   return e;
 }
 
+template <typename T, int CH>
+static cudaError_t pack_launch_ch(int na, dim3 grid, cudaStream_t s, const PackArgs& a, const T* cand, const T* ctx,
+                                  T* X, int* row_req, int* cand_off_dev, const float* weff_x, const float* cdec,
+                                  float* xlog) {
+  const int d = a.d;
+  if (na <= 1)
+    return launch_pdl(pack_kernel<T, 1, CH>, grid, dim3(256), 0, s, a, cand, ctx, X, row_req, cand_off_dev, weff_x,
+                      cdec, xlog);
+  if (na <= 2)
+    return launch_pdl(pack_kernel<T, 2, CH>, grid, dim3(256), 0, s, a, cand, ctx, X, row_req, cand_off_dev, weff_x,
+                      cdec, xlog);
+  if (na <= 4)
+    return launch_pdl(pack_kernel<T, 4, CH>, grid, dim3(256), 0, s, a, cand, ctx, X, row_req, cand_off_dev, weff_x,
+                      cdec, xlog);
+  if (na <= 8)
+    return launch_pdl(pack_kernel<T, 8, CH>, grid, dim3(256), sizeof(float) * 8 * d, s, a, cand, ctx, X, row_req,
+                      cand_off_dev, weff_x, cdec, xlog);
+  return launch_pdl(pack_kernel<T, 16, CH>, grid, dim3(256), sizeof(float) * 16 * d, s, a, cand, ctx, X, row_req,
+                    cand_off_dev, weff_x, cdec, xlog);
+}
+
 template <typename T>
 cudaError_t launch_pack(int n_req, const int* cand_off_host, int S, int d, int na, const T* cand, const T* ctx, T* X,
                         int* row_req, int* cand_off_dev, const float* weff_x, const float* cdec, float* xlog,
@@ -310,17 +414,14 @@ cudaError_t launch_pack(int n_req, const int* cand_off_host, int S, int d, int n
   for (int i = 0; i <= n_req; ++i) a.cand_off[i] = cand_off_host[i];
   const long long n_rows = a.n_cand + static_cast<long long>(n_req) * S;
   if (n_rows == 0) return cudaSuccess;
-  const size_t smem = sizeof(float) * d * na;
-  static bool attr = false;
-  if (!attr) {
-    cudaError_t e = cudaFuncSetAttribute(pack_kernel<T>, cudaFuncAttributeMaxDynamicSharedMemorySize, 512 * 16 * 4);
-    if (e != cudaSuccess) return e;
-    attr = true;
-  }
   const long long rows_per_cta = 8LL * kPackRowsPerWarp;
+  const dim3 grid(static_cast<unsigned>((n_rows + rows_per_cta - 1) / rows_per_cta));
+  const int ch = (d + 32 * Vec16<T>::N - 1) / (32 * Vec16<T>::N);   // 1, 2 or 4 (d <= 512)
   prof_begin(KC_PACK, s);
-  cudaError_t err = launch_pdl(pack_kernel<T>, dim3(static_cast<int>((n_rows + rows_per_cta - 1) / rows_per_cta)),
-                               dim3(256), smem, s, a, cand, ctx, X, row_req, cand_off_dev, weff_x, cdec, xlog);
+  cudaError_t err;
+  if (ch == 1) err = pack_launch_ch<T, 1>(na, grid, s, a, cand, ctx, X, row_req, cand_off_dev, weff_x, cdec, xlog);
+  else if (ch == 2) err = pack_launch_ch<T, 2>(na, grid, s, a, cand, ctx, X, row_req, cand_off_dev, weff_x, cdec, xlog);
+  else err = pack_launch_ch<T, 4>(na, grid, s, a, cand, ctx, X, row_req, cand_off_dev, weff_x, cdec, xlog);
   prof_end(KC_PACK, s);
   return err;
 }
