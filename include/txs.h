@@ -451,6 +451,14 @@ txs_status txs_encoder_device_status(txs_encoder* enc);
 /* Synchronise the device, read and clear the model's latched device status. */
 txs_status txs_device_status(txs_model* model);
 
+/* The GELU of the FFN epilogues, element-wise on device float arrays x -> y
+ * of n elements, for tests of its accuracy (no paper counterpart; the
+ * activation is the exact erf form 0.5 x (1 + erf(x / sqrt 2))).  variant 0:
+ * the bf16 tensor-core epilogues' evaluation (erf by Abramowitz & Stegun
+ * 7.1.26, absolute error <= 1.5e-7); variant 1: the fp32 path's (erff).
+ * Asynchronous on `stream`.  Errors: TXS_ERR_INVALID_ARG, TXS_ERR_CUDA. */
+txs_status txs_gelu_eval(const float* x, float* y, int64_t n, int32_t variant, void* stream);
+
 /* Process-wide per-kernel-class timing with CUDA events on the launching
  * stream (off by default).  While enabled, every library launch is bracketed
  * by two events; txs_profile_collect synchronises, writes per-class total

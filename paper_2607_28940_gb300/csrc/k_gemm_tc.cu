@@ -118,7 +118,7 @@ __device__ __forceinline__ void epilogue(const EpiArgs& e, uint32_t tacc, int ro
 #pragma unroll
           for (int i = 0; i < 32; ++i) {
             float x = w[hh + i] + b[i];
-            if constexpr (EPI == EPI_BIAS_GELU) x = gelu_erf(x);
+            if constexpr (EPI == EPI_BIAS_GELU) x = gelu_erf_as(x);
             w[hh + i] = x;
           }
           put(w + hh, n0 + c0 + c + hh);
@@ -133,7 +133,7 @@ __device__ __forceinline__ void epilogue(const EpiArgs& e, uint32_t tacc, int ro
 #pragma unroll
         for (int i = 0; i < 32; ++i) {
           float x = v[i] + b[i];
-          if constexpr (EPI == EPI_BIAS_GELU) x = gelu_erf(x);
+          if constexpr (EPI == EPI_BIAS_GELU) x = gelu_erf_as(x);
           v[i] = x;
         }
         put(v, n0 + c0 + c);
@@ -620,6 +620,22 @@ bool make_tmap_out(CUtensorMap* tm, const void* base, long long rows, long long 
             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// Element-wise GELU of the epilogues, for tests: variant 0 is the bf16
+// tensor-core epilogue's (gelu_erf_as), 1 the fp32 path's (gelu_erf).
+__global__ void __launch_bounds__(256) gelu_eval_kernel(const float* __restrict__ x, float* __restrict__ y, long long n,
+                                                        int variant) {
+  for (long long i = static_cast<long long>(blockIdx.x) * 256 + threadIdx.x; i < n;
+       i += static_cast<long long>(gridDim.x) * 256)
+    y[i] = variant == 0 ? gelu_erf_as(x[i]) : gelu_erf(x[i]);
+}
+
+cudaError_t launch_gelu_eval(const float* x, float* y, long long n, int variant, cudaStream_t s) {
+  if (n <= 0) return cudaSuccess;
+  const long long blocks = std::min<long long>((n + 255) / 256, 4096);
+  gelu_eval_kernel<<<static_cast<unsigned>(blocks), 256, 0, s>>>(x, y, n, variant);
+  return cudaGetLastError();
+}
+
 int num_sms() {
   static int n = 0;
   if (!n) {
@@ -749,5 +765,8 @@ cudaError_t launch_gemm_tc(const __nv_bfloat16* A, long long lda, const __nv_bfl
   return tc::launch_gemm_tc(A, lda, B, e, s, cls);
 }
 bool tc_gemm_supported(int N, int K, int epi) { return tc::tc_gemm_supported(N, K, epi); }
+cudaError_t launch_gelu_eval(const float* x, float* y, long long n, int variant, cudaStream_t s) {
+  return tc::launch_gelu_eval(x, y, n, variant, s);
+}
 
 }  // namespace txs

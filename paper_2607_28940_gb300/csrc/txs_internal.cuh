@@ -82,6 +82,25 @@ __device__ __forceinline__ float gelu_erf(float x) {
   return 0.5f * x * (1.0f + erff(x * 0.70710678118654752f));
 }
 
+// The same GELU with erf from the rational approximation of Abramowitz &
+// Stegun, Handbook of Mathematical Functions (1964), formula 7.1.26:
+// erf(z) = 1 - t (a1 + t (a2 + t (a3 + t (a4 + t a5)))) exp(-z^2),
+// t = 1 / (1 + p z) for z >= 0, odd in z; the approximation's absolute error
+// is at most 1.5e-7, and with fp32 arithmetic and the hardware exp2 and
+// reciprocal the result stays within a few 1e-7 of erf, against bf16
+// outputs with a relative step of 2^-8.  The bf16 tensor-core epilogues use
+// it (fewer instructions per output element than erff).
+__device__ __forceinline__ float gelu_erf_as(float x) {
+  const float z = fabsf(x) * 0.70710678118654752f;
+  const float t = __fdividef(1.0f, fmaf(0.3275911f, z, 1.0f));
+  const float poly =
+      t * fmaf(t, fmaf(t, fmaf(t, fmaf(t, 1.061405429f, -1.453152027f), 1.421413741f), -0.284496736f),
+               0.254829592f);
+  const float e = exp2f(-z * z * 1.4426950408889634f);
+  const float erf_abs = 1.0f - poly * e;
+  return 0.5f * x * (1.0f + copysignf(erf_abs, x));
+}
+
 // Index of the segment that contains `row` in an exclusive-offset array
 // off[0..n] (off[0] == 0, non-decreasing): largest r with off[r] <= row.
 __device__ __forceinline__ int find_segment(const int* off, int n, int row) {
@@ -171,6 +190,9 @@ constexpr int kKvParamReq = 1000;
 template <typename TB>
 cudaError_t launch_gemm_simt(const float* A, long long lda, const TB* B, const EpiArgs& e,
                              float* tmp, cudaStream_t s, int cls);
+// GELU of the GEMM epilogues on device float arrays (variant 0: bf16
+// tensor-core epilogue, 1: fp32 path), for tests.
+cudaError_t launch_gelu_eval(const float* x, float* y, long long n, int variant, cudaStream_t s);
 cudaError_t launch_gemm_tc(const __nv_bfloat16* A, long long lda, const __nv_bfloat16* B,
                            const EpiArgs& e, cudaStream_t s, int cls);
 bool tc_gemm_supported(int N, int K, int epi);

@@ -99,6 +99,7 @@ _SIGS = {
     "txs_enc_state_destroy": (None, [_P]),
     "txs_encoder_device_status": (_I32, [_P]),
     "txs_pool_anchor_static": (_I32, [_P, _I32, _I32P, _P, _P, _P]),
+    "txs_gelu_eval": (_I32, [_P, _P, ctypes.c_int64, _I32, _P]),
     "txs_profile_enable": (_I32, [_I32]),
     "txs_profile_collect": (_I32, [ctypes.POINTER(ctypes.c_double), ctypes.POINTER(ctypes.c_int64), _I32]),
     "txs_kernel_class_name": (ctypes.c_char_p, [_I32]),
@@ -519,6 +520,16 @@ class EncState:
             self.close()
         except Exception:
             pass
+
+
+def gelu_eval(x: torch.Tensor, variant: int = 0) -> torch.Tensor:
+    """The FFN epilogues' GELU on a device float32 tensor (variant 0: bf16
+    tensor-core epilogue, 1: fp32 path)."""
+    assert x.is_cuda and x.dtype == torch.float32 and x.is_contiguous()
+    y = torch.empty_like(x)
+    _check(lib().txs_gelu_eval(ctypes.c_void_p(x.data_ptr()), ctypes.c_void_p(y.data_ptr()), x.numel(), variant,
+                               _stream(None)), "txs_gelu_eval")
+    return y
 
 
 def profile_enable(on: bool = True):
