@@ -171,24 +171,50 @@ __global__ void __launch_bounds__(256) pool_partial_kernel(const T* __restrict__
   if (!is_last) return;
   __threadfence();
   const float* pr = part + static_cast<long long>(r) * max_chunks * (d + 2);
+  // chunk maxima and weighted sums as block reductions (thread t takes
+  // chunks t, t + 256, ...), then each column's sum over the chunks with its
+  // loads issued ahead of the multiply-adds; the order is fixed, so the
+  // result is deterministic
   __shared__ float ch_scale[512];
+  __shared__ float red[kPoolWarps];
   const float old_m = merge_existing ? st_m[r] : -INFINITY;
   const float old_s = merge_existing ? st_s[r] : 0.f;
+  float mloc = -INFINITY;
+  for (int ch = tid; ch < nch_r; ch += 256) mloc = fmaxf(mloc, __ldcg(pr + static_cast<long long>(ch) * (d + 2)));
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) mloc = fmaxf(mloc, __shfl_xor_sync(0xffffffffu, mloc, o));
+  if (lane == 0) red[warp] = mloc;
+  __syncthreads();
   float Mr = old_m;
-  for (int ch = 0; ch < nch_r; ++ch) Mr = fmaxf(Mr, __ldcg(pr + static_cast<long long>(ch) * (d + 2)));
+#pragma unroll
+  for (int w8 = 0; w8 < kPoolWarps; ++w8) Mr = fmaxf(Mr, red[w8]);
   const float w_old = merge_existing ? expf(old_m - Mr) : 0.f;
-  for (int ch = tid; ch < nch_r && ch < 512; ch += 256)
-    ch_scale[ch] = expf(__ldcg(pr + static_cast<long long>(ch) * (d + 2)) - Mr);
+  __syncthreads();                                  // red is reused below
+  float sloc = 0.f;
+  for (int ch = tid; ch < nch_r; ch += 256) {
+    const float* pc = pr + static_cast<long long>(ch) * (d + 2);
+    const float sc = expf(__ldcg(pc) - Mr);
+    if (ch < 512) ch_scale[ch] = sc;
+    sloc = fmaf(__ldcg(pc + 1), sc, sloc);
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) sloc += __shfl_xor_sync(0xffffffffu, sloc, o);
+  if (lane == 0) red[warp] = sloc;
   __syncthreads();
   float Sr = old_s * w_old;
-  for (int ch = 0; ch < nch_r; ++ch) {
-    const float* pc = pr + static_cast<long long>(ch) * (d + 2);
-    const float sc = ch < 512 ? ch_scale[ch] : expf(__ldcg(pc) - Mr);
-    Sr += __ldcg(pc + 1) * sc;
-  }
+#pragma unroll
+  for (int w8 = 0; w8 < kPoolWarps; ++w8) Sr += red[w8];
   for (int k = tid; k < d; k += 256) {
     float a = merge_existing ? st_acc[static_cast<long long>(r) * d + k] * w_old : 0.f;
-    for (int ch = 0; ch < nch_r; ++ch) {
+    int ch = 0;
+    for (; ch + 8 <= nch_r && ch + 8 <= 512; ch += 8) {
+      float pv[8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u) pv[u] = __ldcg(pr + static_cast<long long>(ch + u) * (d + 2) + 2 + k);
+#pragma unroll
+      for (int u = 0; u < 8; ++u) a = fmaf(pv[u], ch_scale[ch + u], a);
+    }
+    for (; ch < nch_r; ++ch) {
       const float* pc = pr + static_cast<long long>(ch) * (d + 2);
       const float sc = ch < 512 ? ch_scale[ch] : expf(__ldcg(pc) - Mr);
       a = fmaf(__ldcg(pc + 2 + k), sc, a);
