@@ -149,11 +149,45 @@ __global__ void __launch_bounds__(256) pool_partial_kernel(const T* __restrict__
     scale[w8] = sm_s[w8] > 0.f ? expf(sm_m[w8] - M) : 0.f;
     S += sm_s[w8] * scale[w8];
   }
-  for (int k = tid; k < d; k += 256) {
-    float a = 0.f;
+  // one chunk per request (every request's rows fit one chunk, as in an
+  // append of up to kPoolChunkV rows): merge with the stored state right
+  // here, with the arithmetic of the general merge below
+  const bool single = MERGE && gridDim.x == 1;
+  float a_k[2];                                      // this thread's columns tid, tid + 256 (d <= 512)
 #pragma unroll
-    for (int w8 = 0; w8 < kPoolWarps; ++w8) a = fmaf(sm_acc[w8][k], scale[w8], a);
-    out[2 + k] = a;
+  for (int kk = 0; kk < 2; ++kk) {
+    const int k = tid + 256 * kk;
+    float a = 0.f;
+    if (k < d) {
+#pragma unroll
+      for (int w8 = 0; w8 < kPoolWarps; ++w8) a = fmaf(sm_acc[w8][k], scale[w8], a);
+      if (!single) out[2 + k] = a;
+    }
+    a_k[kk] = a;
+  }
+  if (single) {
+    const float old_m = merge_existing ? st_m[r] : -INFINITY;
+    const float old_s = merge_existing ? st_s[r] : 0.f;
+    const float Mr = fmaxf(old_m, M);
+    const float w_old = merge_existing ? expf(old_m - Mr) : 0.f;
+    const float sc = expf(M - Mr);
+    const float Sr = __fadd_rn(__fmul_rn(old_s, w_old), fmaf(S, sc, 0.f));
+#pragma unroll
+    for (int kk = 0; kk < 2; ++kk) {
+      const int k = tid + 256 * kk;
+      if (k < d) {
+        const float a0 = merge_existing ? __fmul_rn(st_acc[static_cast<long long>(r) * d + k], w_old) : 0.f;
+        const float a = fmaf(a_k[kk], sc, a0);
+        st_acc[static_cast<long long>(r) * d + k] = a;
+        g[static_cast<long long>(r) * d + k] = a / Sr;
+      }
+    }
+    __syncthreads();                                 // every thread has read st_m / st_s
+    if (tid == 0) {
+      st_m[r] = Mr;
+      st_s[r] = Sr;
+    }
+    return;
   }
   if (tid == 0) {
     out[0] = M;
@@ -201,11 +235,11 @@ __global__ void __launch_bounds__(256) pool_partial_kernel(const T* __restrict__
   for (int o = 16; o > 0; o >>= 1) sloc += __shfl_xor_sync(0xffffffffu, sloc, o);
   if (lane == 0) red[warp] = sloc;
   __syncthreads();
-  float Sr = old_s * w_old;
+  float Sr = __fmul_rn(old_s, w_old);
 #pragma unroll
-  for (int w8 = 0; w8 < kPoolWarps; ++w8) Sr += red[w8];
+  for (int w8 = 0; w8 < kPoolWarps; ++w8) Sr = __fadd_rn(Sr, red[w8]);
   for (int k = tid; k < d; k += 256) {
-    float a = merge_existing ? st_acc[static_cast<long long>(r) * d + k] * w_old : 0.f;
+    float a = merge_existing ? __fmul_rn(st_acc[static_cast<long long>(r) * d + k], w_old) : 0.f;
     int ch = 0;
     for (; ch + 8 <= nch_r && ch + 8 <= 512; ch += 8) {
       float pv[8];
