@@ -48,7 +48,7 @@ FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0}
 # one --set full capture of that class's kernel on that workload.
 NCU_TRAFFIC = {
     ("small_bf16", "local_global", "gemm_oproj_ln"): (8.62e6, "0298cec9094e"),
-    ("mid_bf16", "full", "attn_cross"): (855.2e6, "0cb06472b837"),
+    ("mid_bf16", "full", "attn_cross"): (855.2e6, "a3d03e1da489"),
 }
 
 

@@ -199,35 +199,6 @@ __device__ __forceinline__ float ex2(float x) {
   return y;
 }
 
-// max(a, b, c) in one instruction (three-source max.f32, sm_100 and later).
-__device__ __forceinline__ float fmax3(float a, float b, float c) {
-  float r;
-  asm("max.f32 %0, %1, %2, %3;" : "=f"(r) : "f"(a), "f"(b), "f"(c));
-  return r;
-}
-// Lane-wise a * b + c and a + b on a pair of fp32 values in one instruction
-// (f32x2 arithmetic, sm_100 and later); each lane rounds like fmaf / fadd.
-__device__ __forceinline__ float2 ffma2(float2 a, float2 b, float2 c) {
-  uint64_t r;
-  asm("{\n\t.reg .b64 x, y, z;\n\t"
-      "mov.b64 x, {%1, %2};\n\tmov.b64 y, {%3, %4};\n\tmov.b64 z, {%5, %6};\n\t"
-      "fma.rn.f32x2 %0, x, y, z;\n\t}"
-      : "=l"(r) : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y), "f"(c.x), "f"(c.y));
-  float2 o;
-  asm("mov.b64 {%0, %1}, %2;" : "=f"(o.x), "=f"(o.y) : "l"(r));
-  return o;
-}
-__device__ __forceinline__ float2 fadd2(float2 a, float2 b) {
-  uint64_t r;
-  asm("{\n\t.reg .b64 x, y;\n\t"
-      "mov.b64 x, {%1, %2};\n\tmov.b64 y, {%3, %4};\n\t"
-      "add.rn.f32x2 %0, x, y;\n\t}"
-      : "=l"(r) : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y));
-  float2 o;
-  asm("mov.b64 {%0, %1}, %2;" : "=f"(o.x), "=f"(o.y) : "l"(r));
-  return o;
-}
-
 // Shared-memory matrix descriptor (tcgen05): start address, leading/stride
 // byte offsets, descriptor version 1, layout code (2 = 128-byte swizzle,
 // 4 = 64-byte swizzle).

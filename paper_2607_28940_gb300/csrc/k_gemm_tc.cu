@@ -116,10 +116,11 @@ __device__ __forceinline__ void epilogue(const EpiArgs& e, uint32_t tacc, int ro
           float b[32];
           load_f32x32_gen(bias + n0 + c0 + c + hh, b);
 #pragma unroll
-          for (int i = 0; i < 32; ++i) {
-            float x = w[hh + i] + b[i];
-            if constexpr (EPI == EPI_BIAS_GELU) x = gelu_erf_as(x);
-            w[hh + i] = x;
+          for (int i = 0; i < 32; i += 2) {
+            float2 x = fadd2(make_float2(w[hh + i], w[hh + i + 1]), make_float2(b[i], b[i + 1]));
+            if constexpr (EPI == EPI_BIAS_GELU) x = gelu_erf_as2(x);
+            w[hh + i] = x.x;
+            w[hh + i + 1] = x.y;
           }
           put(w + hh, n0 + c0 + c + hh);
         }
@@ -131,10 +132,11 @@ __device__ __forceinline__ void epilogue(const EpiArgs& e, uint32_t tacc, int ro
         float b[32];
         load_f32x32_gen(bias + n0 + c0 + c, b);
 #pragma unroll
-        for (int i = 0; i < 32; ++i) {
-          float x = v[i] + b[i];
-          if constexpr (EPI == EPI_BIAS_GELU) x = gelu_erf_as(x);
-          v[i] = x;
+        for (int i = 0; i < 32; i += 2) {
+          float2 x = fadd2(make_float2(v[i], v[i + 1]), make_float2(b[i], b[i + 1]));
+          if constexpr (EPI == EPI_BIAS_GELU) x = gelu_erf_as2(x);
+          v[i] = x.x;
+          v[i + 1] = x.y;
         }
         put(v, n0 + c0 + c);
       }
@@ -621,17 +623,27 @@ bool make_tmap_out(CUtensorMap* tm, const void* base, long long rows, long long 
 }
 
 // Element-wise GELU of the epilogues, for tests: variant 0 is the bf16
-// tensor-core epilogue's (gelu_erf_as), 1 the fp32 path's (gelu_erf).
+// tensor-core epilogue's (gelu_erf_as2, on pairs), 1 the fp32 path's
+// (gelu_erf).
 __global__ void __launch_bounds__(256) gelu_eval_kernel(const float* __restrict__ x, float* __restrict__ y, long long n,
                                                         int variant) {
-  for (long long i = static_cast<long long>(blockIdx.x) * 256 + threadIdx.x; i < n;
-       i += static_cast<long long>(gridDim.x) * 256)
-    y[i] = variant == 0 ? gelu_erf_as(x[i]) : gelu_erf(x[i]);
+  for (long long i = (static_cast<long long>(blockIdx.x) * 256 + threadIdx.x) * 2; i < n;
+       i += static_cast<long long>(gridDim.x) * 512) {
+    const bool two = i + 1 < n;
+    if (variant == 0) {
+      const float2 r = gelu_erf_as2(make_float2(x[i], two ? x[i + 1] : 0.f));
+      y[i] = r.x;
+      if (two) y[i + 1] = r.y;
+    } else {
+      y[i] = gelu_erf(x[i]);
+      if (two) y[i + 1] = gelu_erf(x[i + 1]);
+    }
+  }
 }
 
 cudaError_t launch_gelu_eval(const float* x, float* y, long long n, int variant, cudaStream_t s) {
   if (n <= 0) return cudaSuccess;
-  const long long blocks = std::min<long long>((n + 255) / 256, 4096);
+  const long long blocks = std::min<long long>((n + 511) / 512, 4096);
   gelu_eval_kernel<<<static_cast<unsigned>(blocks), 256, 0, s>>>(x, y, n, variant);
   return cudaGetLastError();
 }

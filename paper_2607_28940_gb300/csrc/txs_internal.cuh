@@ -82,6 +82,45 @@ __device__ __forceinline__ float gelu_erf(float x) {
   return 0.5f * x * (1.0f + erff(x * 0.70710678118654752f));
 }
 
+// max(a, b, c) in one instruction (three-source max.f32, sm_100 and later).
+__device__ __forceinline__ float fmax3(float a, float b, float c) {
+  float r;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(r) : "f"(a), "f"(b), "f"(c));
+  return r;
+}
+// Lane-wise a * b + c and a + b on a pair of fp32 values in one instruction
+// (f32x2 arithmetic, sm_100 and later); each lane rounds like fmaf / fadd.
+__device__ __forceinline__ float2 ffma2(float2 a, float2 b, float2 c) {
+  uint64_t r;
+  asm("{\n\t.reg .b64 x, y, z;\n\t"
+      "mov.b64 x, {%1, %2};\n\tmov.b64 y, {%3, %4};\n\tmov.b64 z, {%5, %6};\n\t"
+      "fma.rn.f32x2 %0, x, y, z;\n\t}"
+      : "=l"(r) : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y), "f"(c.x), "f"(c.y));
+  float2 o;
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(o.x), "=f"(o.y) : "l"(r));
+  return o;
+}
+__device__ __forceinline__ float2 fmul2(float2 a, float2 b) {
+  uint64_t r;
+  asm("{\n\t.reg .b64 x, y;\n\t"
+      "mov.b64 x, {%1, %2};\n\tmov.b64 y, {%3, %4};\n\t"
+      "mul.rn.f32x2 %0, x, y;\n\t}"
+      : "=l"(r) : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y));
+  float2 o;
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(o.x), "=f"(o.y) : "l"(r));
+  return o;
+}
+__device__ __forceinline__ float2 fadd2(float2 a, float2 b) {
+  uint64_t r;
+  asm("{\n\t.reg .b64 x, y;\n\t"
+      "mov.b64 x, {%1, %2};\n\tmov.b64 y, {%3, %4};\n\t"
+      "add.rn.f32x2 %0, x, y;\n\t}"
+      : "=l"(r) : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y));
+  float2 o;
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(o.x), "=f"(o.y) : "l"(r));
+  return o;
+}
+
 // The same GELU with erf from the rational approximation of Abramowitz &
 // Stegun, Handbook of Mathematical Functions (1964), formula 7.1.26:
 // erf(z) = 1 - t (a1 + t (a2 + t (a3 + t (a4 + t a5)))) exp(-z^2),
@@ -89,16 +128,22 @@ __device__ __forceinline__ float gelu_erf(float x) {
 // is at most 1.5e-7, and with fp32 arithmetic and the hardware exp2 and
 // reciprocal the result stays within a few 1e-7 of erf, against bf16
 // outputs with a relative step of 2^-8.  The bf16 tensor-core epilogues use
-// it (fewer instructions per output element than erff).
-__device__ __forceinline__ float gelu_erf_as(float x) {
-  const float z = fabsf(x) * 0.70710678118654752f;
-  const float t = __fdividef(1.0f, fmaf(0.3275911f, z, 1.0f));
-  const float poly =
-      t * fmaf(t, fmaf(t, fmaf(t, fmaf(t, 1.061405429f, -1.453152027f), 1.421413741f), -0.284496736f),
-               0.254829592f);
-  const float e = exp2f(-z * z * 1.4426950408889634f);
-  const float erf_abs = 1.0f - poly * e;
-  return 0.5f * x * (1.0f + copysignf(erf_abs, x));
+// it (fewer instructions per output element than erff), on two values at
+// once: the multiplies and multiply-adds run as f32x2 instructions.
+__device__ __forceinline__ float2 gelu_erf_as2(float2 x) {
+  const float2 z = fmul2(make_float2(fabsf(x.x), fabsf(x.y)), make_float2(0.70710678118654752f, 0.70710678118654752f));
+  const float2 den = ffma2(make_float2(0.3275911f, 0.3275911f), z, make_float2(1.0f, 1.0f));
+  const float2 t = make_float2(__fdividef(1.0f, den.x), __fdividef(1.0f, den.y));
+  float2 q = ffma2(t, make_float2(1.061405429f, 1.061405429f), make_float2(-1.453152027f, -1.453152027f));
+  q = ffma2(t, q, make_float2(1.421413741f, 1.421413741f));
+  q = ffma2(t, q, make_float2(-0.284496736f, -0.284496736f));
+  q = ffma2(t, q, make_float2(0.254829592f, 0.254829592f));
+  const float2 poly = fmul2(t, q);
+  const float2 zz = fmul2(fmul2(make_float2(-z.x, -z.y), z), make_float2(1.4426950408889634f, 1.4426950408889634f));
+  const float2 e = make_float2(exp2f(zz.x), exp2f(zz.y));
+  const float2 ea = ffma2(make_float2(-poly.x, -poly.y), e, make_float2(1.0f, 1.0f));
+  const float2 onep = make_float2(1.0f + copysignf(ea.x, x.x), 1.0f + copysignf(ea.y, x.y));
+  return fmul2(fmul2(make_float2(0.5f, 0.5f), x), onep);
 }
 
 // Index of the segment that contains `row` in an exclusive-offset array
