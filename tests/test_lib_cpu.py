@@ -94,6 +94,13 @@ def test_rank_rejects_bad_arguments_on_host(lib):
     assert lib.txs_rank_candidates(0, p, None, 4, 0, 0, None, None) == txs.TXS_OK
 
 
+def test_gelu_eval_rejects_bad_arguments_on_host(lib):
+    assert lib.txs_gelu_eval(None, None, 4, 0, None) == txs.TXS_ERR_INVALID_ARG       # null arrays
+    assert lib.txs_gelu_eval(16, 16, -1, 0, None) == txs.TXS_ERR_INVALID_ARG          # negative size
+    assert lib.txs_gelu_eval(16, 16, 4, 2, None) == txs.TXS_ERR_INVALID_ARG           # unknown variant
+    assert lib.txs_gelu_eval(None, None, 0, 1, None) == txs.TXS_OK                    # nothing to do
+
+
 def test_profiler_collect_without_launches(lib):
     assert txs.profile_collect() == {}
 
