@@ -121,7 +121,7 @@ __device__ __forceinline__ float2 fadd2(float2 a, float2 b) {
   return o;
 }
 
-// The same GELU with erf from the rational approximation of Abramowitz &
+// gelu_erf (above the f32x2 helpers) with erf from the rational approximation of Abramowitz &
 // Stegun, Handbook of Mathematical Functions (1964), formula 7.1.26:
 // erf(z) = 1 - t (a1 + t (a2 + t (a3 + t (a4 + t a5)))) exp(-z^2),
 // t = 1 / (1 + p z) for z >= 0, odd in z; the approximation's absolute error
