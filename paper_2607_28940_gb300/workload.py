@@ -183,6 +183,51 @@ def weights(wl: Workload) -> Dict[str, np.ndarray]:
     return out
 
 
+def sharp_gains(wl: Workload) -> Dict[str, float]:
+    """Power-of-two gains of ``sharp_weights`` for this workload's width.
+
+    ``att``  on the query and key projections of both attentions (scores of
+             standard deviation ~1.6 at d = 256, ~3.3 at d = 512, so the
+             softmax over the keys is far from uniform);
+    ``oc``   on the cross-attention output projection (the attended values
+             move the residual stream);
+    ``head`` on W_dec (logits of standard deviation ~0.3; with N(0, 0.02)
+             weights it is about 0.0004 * sqrt(2) * d; larger logits make
+             the bf16 rounding of the activations through four decoder
+             layers exceed the mean tolerance of 2e-3 on their own);
+    ``pool`` on w_pool (pooling logits of standard deviation ~2.6, so the
+             anchor is a weighted mix of a few rows, not the mean).
+    """
+    d = wl.d_model
+    head = 2.0 ** max(0, int(round(np.log2(0.3 / (0.0004 * np.sqrt(2.0) * d)))))
+    return {"att": 4.0, "oc": 4.0, "head": head, "pool": 128.0}
+
+
+def sharp_weights(wl: Workload, base: Optional[Dict[str, np.ndarray]] = None) -> Dict[str, np.ndarray]:
+    """The workload's weights with the gains of ``sharp_gains`` applied.
+
+    The gains are powers of two, so bf16-stored weights stay exactly
+    representable and both sides of a parity test still see identical
+    values.  With the plain N(0, 0.02) draws every attention softmax is
+    nearly uniform and logits have a standard deviation of ~0.14, which hides
+    errors in which keys an attention reads; these weights make such errors
+    move the scores by far more than the bf16 tolerances.
+    """
+    w = dict(weights(wl) if base is None else base)
+    gn = sharp_gains(wl)
+    d = wl.d_model
+    for l in range(wl.n_layers):
+        qkv = np.array(w[f"W_qkv.{l}"], dtype=np.float32, copy=True)
+        qkv[:, :2 * d] *= gn["att"]
+        w[f"W_qkv.{l}"] = qkv
+        w[f"W_Q.{l}"] = np.asarray(w[f"W_Q.{l}"], np.float32) * np.float32(gn["att"])
+        w[f"W_K.{l}"] = np.asarray(w[f"W_K.{l}"], np.float32) * np.float32(gn["att"])
+        w[f"W_oc.{l}"] = np.asarray(w[f"W_oc.{l}"], np.float32) * np.float32(gn["oc"])
+    w["W_dec"] = np.asarray(w["W_dec"], np.float32) * np.float32(gn["head"])
+    w["w_pool"] = np.asarray(w["w_pool"], np.float32) * np.float32(gn["pool"])
+    return w
+
+
 @dataclass
 class Batch:
     """One synthetic serving batch, packed request after request.

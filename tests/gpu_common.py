@@ -2,6 +2,7 @@
 and the fp64 oracle on the same seeded inputs, and compare."""
 from __future__ import annotations
 
+import os
 from dataclasses import dataclass
 from typing import Dict, List, Optional, Sequence
 
@@ -25,6 +26,8 @@ def assert_scores_close(gpu: np.ndarray, ref: np.ndarray, dtype: str, what: str 
     err = np.abs(gpu - ref)
     if err.size == 0:
         return
+    if os.environ.get("TXS_PRINT_ERRORS"):
+        print(f"[scores] {what}: max|d| {err.max():.3e} mean|d| {err.mean():.3e}")
     if dtype == "bf16":
         assert err.max() <= BF16_MAX and err.mean() <= BF16_MEAN, \
             f"{what}: max|d| {err.max():.3g} mean|d| {err.mean():.3g}"
@@ -80,3 +83,24 @@ def oracle_scores(wl: W.Workload, mode: int, requests: Optional[Sequence[int]] =
 def rows_of(b: W.Batch, requests: Sequence[int], arr: np.ndarray) -> np.ndarray:
     """Concatenate the candidate rows of `requests` from a full-batch output."""
     return np.concatenate([arr[b.cand_off[r]:b.cand_off[r + 1]] for r in requests], axis=0)
+
+
+def score_errors(gpu: np.ndarray, ref: np.ndarray):
+    """(max|d|, mean|d|) of two score arrays, for reports."""
+    e = np.abs(np.asarray(gpu, np.float64) - np.asarray(ref, np.float64))
+    return (float(e.max()), float(e.mean())) if e.size else (0.0, 0.0)
+
+
+def oracle_candidate_subset(wl: W.Workload, mode: int, r: int, cand_idx: Sequence[int],
+                            weights: Dict[str, np.ndarray], M_override: Optional[int] = None, append: bool = False):
+    """Oracle logits/probs of some candidates of request r.  Candidates are
+    scored independently of each other (a candidate row attends to the context
+    rows and itself only, App. B mask), so a subset of the slate gives the same
+    values as the whole slate; the oracle pins this invariance."""
+    model = O.Model.from_arrays(weights, wl)
+    b = W.batch(wl, requests=[r], M_override=M_override)
+    cache = O.build_cache(model, b.beh)
+    if append:
+        cache = O.append_cache(model, cache, b.app)
+    cand = b.cand[np.asarray(cand_idx, dtype=np.int64)]
+    return O.score_request(model, cache, b.ctx[0], cand, mode)
