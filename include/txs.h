@@ -339,13 +339,14 @@ txs_status txs_rank_candidates(int32_t n_req, const int32_t* cand_offsets, const
  *
  * Scratch: a 4 MiB file-scope device array of the library (held on every GPU
  * that loads it until the process exits) — n_req * 16 * (d_model + 2) floats
- * must fit in 1,048,576 (d_model = 512: up to 127 requests), and n_req <= 1024;
- * larger calls return TXS_ERR_UNSUPPORTED (txs_last_error says why) before
- * anything is enqueued.  Every call overwrites all scratch it reads, and all
- * calls share that one array: calls that overlap on the GPU (other streams,
- * other threads) race and must be serialised by the caller.  The first call
- * on each device looks up the array's device address with that device
- * current; make that first call before any stream capture.
+ * must fit in 1,048,576 (d_model = 512: up to 127 requests), n_req <= 1024 and
+ * d_model <= 512; larger calls return TXS_ERR_UNSUPPORTED (txs_last_error says
+ * why) before anything is enqueued.  Every call overwrites all scratch it
+ * reads, and all calls share that one array: calls that overlap on the GPU
+ * (other streams, other threads) race and must be serialised by the caller.
+ * Each call looks up the array's device address in the current device's
+ * context (cudaGetSymbolAddress, which allocates nothing); make the first call
+ * on a device before any stream capture.
  */
 txs_status txs_pool_anchor_static(const txs_model* model, int32_t n_req, const int32_t* beh_offsets,
                                   const void* beh_enc, float* out_g, void* stream);

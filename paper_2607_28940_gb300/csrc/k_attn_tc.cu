@@ -23,10 +23,12 @@
 // All waits are bounded; a timeout latches TXS_ERR_DEVICE_TIMEOUT.
 #include <algorithm>
 
-#include "txs_internal.cuh"
+#include "tc_ptx.cuh"
 
 namespace txs {
 namespace fa {
+
+using namespace tc;
 
 constexpr int BQ = 128;            // queries per CTA (TMEM lanes)
 constexpr int BKV = 128;           // keys per K/V tile
@@ -35,75 +37,11 @@ constexpr int NUM_THREADS = 192;   // producer, MMA, 4 softmax warps
 constexpr float kRescaleLog2 = 8.f;  // raise the running max only past this (log2 units)
 
 // ------------------------------------------------------------------ PTX wrappers
+//
+// The common tcgen05 / TMA / mbarrier wrappers come from tc_ptx.cuh; the
+// attention's waits poll without the suspend-time hint (mbar_wait<false>).
+// Below: the TMEM-operand MMA and the wider TMEM loads only this file uses.
 
-__device__ __forceinline__ uint32_t smem_u32(const void* p) {
-  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
-}
-__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
-  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count) : "memory");
-}
-__device__ __forceinline__ void mbar_expect_tx(uint64_t* bar, uint32_t bytes) {
-  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)), "r"(bytes)
-               : "memory");
-}
-__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
-  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
-}
-__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
-  uint32_t ok;
-  asm volatile(
-      "{\n\t.reg .pred p;\n\t"
-      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
-      "selp.u32 %0, 1, 0, p;\n\t}"
-      : "=r"(ok)
-      : "r"(smem_u32(bar)), "r"(parity)
-      : "memory");
-  return ok != 0;
-}
-__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort) {
-  const long long t0 = clock64();
-  while (!mbar_try_wait(bar, parity)) {
-    if (*abort) return false;
-    if (clock64() - t0 > kSpinCycles) {
-      *abort = 1;
-      return false;
-    }
-  }
-  return true;
-}
-__device__ __forceinline__ bool mbar_wait_plain(uint64_t* bar, uint32_t parity) {
-  const long long t0 = clock64();
-  while (!mbar_try_wait(bar, parity))
-    if (clock64() - t0 > kSpinCycles) return false;
-  return true;
-}
-__device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* tm, uint64_t* bar, int x, int y) {
-  asm volatile(
-      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%3, %4}], [%2];" ::"r"(
-          smem_u32(dst)),
-      "l"(reinterpret_cast<uint64_t>(tm)), "r"(smem_u32(bar)), "r"(x), "r"(y)
-      : "memory");
-}
-__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
-__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
-__device__ __forceinline__ void fence_async_smem() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
-__device__ __forceinline__ void tmem_alloc(uint32_t* holder, uint32_t ncols) {
-  asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(holder)), "r"(ncols)
-               : "memory");
-  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
-}
-__device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
-  asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols) : "memory");
-}
-__device__ __forceinline__ void mma_bf16(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
-                                         uint32_t accumulate) {
-  asm volatile(
-      "{\n\t.reg .pred p;\n\t"
-      "setp.ne.b32 p, %4, 0;\n\t"
-      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
-      "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
-      : "memory");
-}
 // Same, with the A operand (M x 16 bf16, K-major: lane = row, two elements
 // per 32-bit column) read from TMEM at a_tmem.
 __device__ __forceinline__ void mma_bf16_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t bdesc, uint32_t idesc,
@@ -125,47 +63,6 @@ __device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint32_t* v) {
       : "memory");
 }
 __device__ __forceinline__ void tmem_wait_st() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
-__device__ __forceinline__ void mma_commit(uint64_t* bar) {
-  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(smem_u32(bar))
-               : "memory");
-}
-__device__ __forceinline__ void tmem_ld32(uint32_t taddr, float* v) {
-  uint32_t r[32];
-  asm volatile(
-      "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
-      "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
-      "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];\n\t"
-      "tcgen05.wait::ld.sync.aligned;"
-      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
-        "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]),
-        "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]),
-        "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
-      : "r"(taddr)
-      : "memory");
-#pragma unroll
-  for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
-}
-
-__device__ __forceinline__ void tmem_st32(uint32_t taddr, const float* v) {
-  asm volatile(
-      "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], "
-      "{%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,"
-      "%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,%32};\n\t"
-      "tcgen05.wait::st.sync.aligned;" ::"r"(taddr),
-      "r"(__float_as_uint(v[0])), "r"(__float_as_uint(v[1])), "r"(__float_as_uint(v[2])),
-      "r"(__float_as_uint(v[3])), "r"(__float_as_uint(v[4])), "r"(__float_as_uint(v[5])),
-      "r"(__float_as_uint(v[6])), "r"(__float_as_uint(v[7])), "r"(__float_as_uint(v[8])),
-      "r"(__float_as_uint(v[9])), "r"(__float_as_uint(v[10])), "r"(__float_as_uint(v[11])),
-      "r"(__float_as_uint(v[12])), "r"(__float_as_uint(v[13])), "r"(__float_as_uint(v[14])),
-      "r"(__float_as_uint(v[15])), "r"(__float_as_uint(v[16])), "r"(__float_as_uint(v[17])),
-      "r"(__float_as_uint(v[18])), "r"(__float_as_uint(v[19])), "r"(__float_as_uint(v[20])),
-      "r"(__float_as_uint(v[21])), "r"(__float_as_uint(v[22])), "r"(__float_as_uint(v[23])),
-      "r"(__float_as_uint(v[24])), "r"(__float_as_uint(v[25])), "r"(__float_as_uint(v[26])),
-      "r"(__float_as_uint(v[27])), "r"(__float_as_uint(v[28])), "r"(__float_as_uint(v[29])),
-      "r"(__float_as_uint(v[30])), "r"(__float_as_uint(v[31]))
-      : "memory");
-}
-
 // 128 consecutive columns of this warp's 32 lanes: one load, one wait.
 __device__ __forceinline__ void tmem_ld128(uint32_t taddr, float* v) {
   uint32_t r[128];
@@ -177,19 +74,6 @@ __device__ __forceinline__ void tmem_ld128(uint32_t taddr, float* v) {
       : "memory");
 #pragma unroll
   for (int i = 0; i < 128; ++i) v[i] = __uint_as_float(r[i]);
-}
-
-// 64 consecutive columns of this warp's 32 lanes: one load, one wait.
-__device__ __forceinline__ void tmem_ld64(uint32_t taddr, float* v) {
-  uint32_t r[64];
-  asm volatile(
-      "tcgen05.ld.sync.aligned.32x32b.x64.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,%32,%33,%34,%35,%36,%37,%38,%39,%40,%41,%42,%43,%44,%45,%46,%47,%48,%49,%50,%51,%52,%53,%54,%55,%56,%57,%58,%59,%60,%61,%62,%63}, [%64];\n\t"
-      "tcgen05.wait::ld.sync.aligned;"
-      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31]), "=r"(r[32]), "=r"(r[33]), "=r"(r[34]), "=r"(r[35]), "=r"(r[36]), "=r"(r[37]), "=r"(r[38]), "=r"(r[39]), "=r"(r[40]), "=r"(r[41]), "=r"(r[42]), "=r"(r[43]), "=r"(r[44]), "=r"(r[45]), "=r"(r[46]), "=r"(r[47]), "=r"(r[48]), "=r"(r[49]), "=r"(r[50]), "=r"(r[51]), "=r"(r[52]), "=r"(r[53]), "=r"(r[54]), "=r"(r[55]), "=r"(r[56]), "=r"(r[57]), "=r"(r[58]), "=r"(r[59]), "=r"(r[60]), "=r"(r[61]), "=r"(r[62]), "=r"(r[63])
-      : "r"(taddr)
-      : "memory");
-#pragma unroll
-  for (int i = 0; i < 64; ++i) v[i] = __uint_as_float(r[i]);
 }
 
 // 2^x on the special-function unit (PTX ex2.approx, flush-to-zero).
@@ -363,7 +247,7 @@ __global__ void __launch_bounds__(PAIR_THREADS, 1)
       int issued = 0;
       for (int j = 0; j < nkv; ++j) {
         const int st = j % STG;
-        if (!mbar_wait(kv_empty + st, ((j / STG) & 1) ^ 1, abort_flag)) break;
+        if (!mbar_wait<false>(kv_empty + st, ((j / STG) & 1) ^ 1, abort_flag)) break;
         mbar_expect_tx(kv_full + st, 2 * Sh::KV_BYTES);
         const int kt = split ? ((j & 1) ? n_a + (j >> 1) : (j >> 1)) : j;   // j-th tile of the sequence
         tma_load_2d(sK + st * Sh::KV_BYTES, &tmK, kv_full + st, (h / a.group) * DH, kv0 + kt * BKV);
@@ -372,7 +256,7 @@ __global__ void __launch_bounds__(PAIR_THREADS, 1)
       }
       if (*abort_flag)
         for (int k = issued > STG ? issued - STG : 0; k < issued; ++k)
-          mbar_wait_plain(kv_full + k % STG, (k / STG) & 1);
+          mbar_wait_plain<false>(kv_full + k % STG, (k / STG) & 1);
     }
   } else if (warp == 1) {
     if (lane == 0) {
@@ -396,10 +280,10 @@ __global__ void __launch_bounds__(PAIR_THREADS, 1)
                       (acc || k > 0) ? 1u : 0u);
         }
       };
-      bool ok = mbar_wait(q_ready, 0, abort_flag);
+      bool ok = mbar_wait<false>(q_ready, 0, abort_flag);
       for (int t = 0; t < n_t && ok; ++t) {
         const int u = seq(t, 0);
-        if (t == 0 || split) ok = mbar_wait(kv_full + u % STG, (u / STG) & 1, abort_flag);
+        if (t == 0 || split) ok = mbar_wait<false>(kv_full + u % STG, (u / STG) & 1, abort_flag);
         if (ok) {
           tc_fence_after();
           qk(t, u);
@@ -410,14 +294,14 @@ __global__ void __launch_bounds__(PAIR_THREADS, 1)
         for (int t = 0; t < n_t && ok; ++t) {
           if (i >= iters(t)) continue;
           const int u = seq(t, i);
-          if (!mbar_wait(p_full + t, i & 1, abort_flag)) { ok = false; break; }
+          if (!mbar_wait<false>(p_full + t, i & 1, abort_flag)) { ok = false; break; }
           tc_fence_after();
           pv(t, u, i > 0);
           // a key tile is released once every product that reads it is issued
           if (split || t == n_t - 1) mma_commit(kv_empty + u % STG);
           if (i + 1 < iters(t)) {
             const int un = seq(t, i + 1);
-            if ((t == 0 || split) && !mbar_wait(kv_full + un % STG, (un / STG) & 1, abort_flag)) {
+            if ((t == 0 || split) && !mbar_wait<false>(kv_full + un % STG, (un / STG) & 1, abort_flag)) {
               ok = false;
               break;
             }
@@ -462,7 +346,7 @@ __global__ void __launch_bounds__(PAIR_THREADS, 1)
     bool ok = true;
     const int n_it = iters(t);
     for (int j = 0; j < n_it && ok; ++j) {
-      ok = mbar_wait(s_full + t, j & 1, abort_flag);
+      ok = mbar_wait<false>(s_full + t, j & 1, abort_flag);
       ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
       if (!ok) break;
       tc_fence_after();
@@ -533,7 +417,7 @@ __global__ void __launch_bounds__(PAIR_THREADS, 1)
       l_run += ps[0].x + ps[0].y;
     }
     if (ok) {
-      ok = mbar_wait(o_done + t, 0, abort_flag);
+      ok = mbar_wait<false>(o_done + t, 0, abort_flag);
       ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
     }
     // split keys: group B hands its partial state (O, running max, row sum)
@@ -721,7 +605,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       int issued = 0;
       for (int j = 0; j < nkv; ++j) {
         const int st = j % STG;
-        if (!mbar_wait(kv_empty + st, ((j / STG) & 1) ^ 1, abort_flag)) break;
+        if (!mbar_wait<false>(kv_empty + st, ((j / STG) & 1) ^ 1, abort_flag)) break;
         mbar_expect_tx(kv_full + st, 2 * Sh::KV_BYTES);
         const int krow = base + (jb + j) * BKV;
         tma_load_2d(sK + st * Sh::KV_BYTES, &tmK, kv_full + st, h * DH, krow);
@@ -730,17 +614,17 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       }
       if (*abort_flag)
         for (int k = issued > STG ? issued - STG : 0; k < issued; ++k)
-          mbar_wait_plain(kv_full + k % STG, (k / STG) & 1);
+          mbar_wait_plain<false>(kv_full + k % STG, (k / STG) & 1);
     }
   } else if (warp == 1) {
     if (lane == 0) {
       constexpr uint32_t id_s = idesc_bf16(BQ, BKV, false);
       constexpr uint32_t id_pv = idesc_bf16(BQ, DH, true);
-      bool ok = mbar_wait(q_ready, 0, abort_flag);
+      bool ok = mbar_wait<false>(q_ready, 0, abort_flag);
       tc_fence_after();
       auto pv = [&](int tt) -> bool {
         const int bt = tt & 1, st = tt % STG;
-        if (!mbar_wait(p_full + bt, (tt >> 1) & 1, abort_flag)) return false;
+        if (!mbar_wait<false>(p_full + bt, (tt >> 1) & 1, abort_flag)) return false;
         tc_fence_after();
         const uint32_t v_addr = smem_u32(sV + st * Sh::KV_BYTES);
 #pragma unroll
@@ -754,8 +638,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       };
       for (int j = 0; j < nkv && ok; ++j) {
         const int st = j % STG, b = j & 1;
-        if (!mbar_wait(kv_full + st, (j / STG) & 1, abort_flag)) break;
-        if (!mbar_wait(s_free + b, ((j >> 1) & 1) ^ 1, abort_flag)) break;
+        if (!mbar_wait<false>(kv_full + st, (j / STG) & 1, abort_flag)) break;
+        if (!mbar_wait<false>(s_free + b, ((j >> 1) & 1) ^ 1, abort_flag)) break;
         tc_fence_after();
         const uint32_t k_addr = smem_u32(sK + st * Sh::KV_BYTES);
 #pragma unroll
@@ -802,7 +686,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     bool ok = true;
     for (int j = 0; j < nkv && ok; ++j) {
       const int b = j & 1;
-      ok = mbar_wait(s_full + b, (j >> 1) & 1, abort_flag);
+      ok = mbar_wait<false>(s_full + b, (j >> 1) & 1, abort_flag);
       ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
       if (!ok) break;
       tc_fence_after();
@@ -810,7 +694,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         __syncwarp();
         if (lane == 0) mbar_arrive(s_free + b);
         if (j >= 2) {
-          ok = mbar_wait(pv_done + b, ((j - 2) >> 1) & 1, abort_flag);
+          ok = mbar_wait<false>(pv_done + b, ((j - 2) >> 1) & 1, abort_flag);
           ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
           if (!ok) break;
         }
@@ -855,7 +739,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         const float m_new = need ? fmaxf(m_run, m_tile) : m_run;
         const float alpha = need ? ex2(m_run - m_new) : 1.f;   // 0 on a row's first visible tile
         if (j >= 1) {
-          ok = mbar_wait(pv_done + ((j - 1) & 1), ((j - 1) >> 1) & 1, abort_flag);
+          ok = mbar_wait<false>(pv_done + ((j - 1) & 1), ((j - 1) >> 1) & 1, abort_flag);
           ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
           if (!ok) break;
           tc_fence_after();
@@ -872,7 +756,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         m_run = m_new;
       }
       if (j >= 2) {
-        ok = mbar_wait(pv_done + b, ((j - 2) >> 1) & 1, abort_flag);
+        ok = mbar_wait<false>(pv_done + b, ((j - 2) >> 1) & 1, abort_flag);
         ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
         if (!ok) break;
         tc_fence_after();
@@ -908,7 +792,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       l_run += ps8[0];
     }
     if (ok) {
-      ok = mbar_wait(pv_done + ((nkv - 1) & 1), ((nkv - 1) >> 1) & 1, abort_flag);
+      ok = mbar_wait<false>(pv_done + ((nkv - 1) & 1), ((nkv - 1) >> 1) & 1, abort_flag);
       ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
     }
     if (ok && !idle) {

@@ -1,8 +1,8 @@
 // Cache-side kernels: attention pooling of the global anchor, its per-layer
 // K/V projection, and the one-time weight preparation of txs_model_create.
 //
-// Attention pooling (Sec. 4.1.2 local-global set: "attention-pooled global
-// representation"; Sec. 5.1 "attention pooling to generate the global token"):
+// Attention pooling (Sec. 4.1.2, the global token of the local-global key set;
+// Sec. 5.1, where pooling produces that token):
 // alpha = softmax_i(phi_i . w_pool / sqrt(d)), g = sum_i alpha_i phi_i.  It is
 // kept as an online-softmax state (m = max logit, s = sum exp(logit - m),
 // acc = sum exp(logit - m) phi) so that an append (App. D incremental-encoding

@@ -11,7 +11,6 @@
 //
 // The caller still passes the behavior rows and the output buffer.  The
 // library never calls cudaMalloc, cudaFree or any allocating routine here.
-#include <mutex>
 #include <string>
 
 #include "txs_internal.cuh"
@@ -26,7 +25,7 @@ constexpr int kSlots = 16;                        // slices per request
 constexpr int kPiece = 128;                       // rows per online-softmax piece
 constexpr long long kScratchFloats = 1 << 20;     // 4 MiB of static scratch
 constexpr int kMaxReq = 1024;                     // offsets passed by value
-constexpr int kMaxDevices = 64;
+constexpr int kMaxD = 512;                        // two accumulator columns per thread of 256
 
 static __device__ __align__(256) float g_anchor_scratch[kScratchFloats];
 
@@ -56,7 +55,7 @@ __global__ void __launch_bounds__(256) pool_slices_static_kernel(const __grid_co
   const int end = min(re, beg + span);
   float* out = scratch + (static_cast<long long>(r) * kSlots + slot) * (d + 2);
   float m_run = -INFINITY, s_run = 0.f;
-  float acc[2] = {0.f, 0.f};   // columns tid and tid + 256 (d <= 512)
+  float acc[2] = {0.f, 0.f};   // columns tid and tid + 256 (d <= kMaxD)
   for (int p0 = beg; p0 < end; p0 += kPiece) {
     const int n = min(kPiece, end - p0);
     for (int i = warp; i < n; i += 8) {
@@ -131,26 +130,17 @@ __global__ void __launch_bounds__(256) pool_finish_static_kernel(const __grid_co
   }
 }
 
-std::mutex g_setup_mu;
-float* g_scratch_dev[kMaxDevices] = {};
-
-// Device address of the static scratch on the current device, looked up once
-// per device with that device current (a failed lookup is retried on the next
-// call).  In host code `g_anchor_scratch` names only a host-side stand-in,
-// never the device memory, so kernels get this address instead.
+// Device address of the static scratch in the current device's context,
+// looked up on every call with that device current.  In host code
+// `g_anchor_scratch` names only a host-side stand-in, never the device memory,
+// so kernels get this address instead.  The lookup allocates nothing; doing it
+// per call (instead of caching it per device index) keeps the address right
+// after the context has been torn down and created again.
 cudaError_t scratch_on_current_device(float** ptr) {
-  int dev = 0;
-  cudaError_t e = cudaGetDevice(&dev);
+  void* p = nullptr;
+  const cudaError_t e = cudaGetSymbolAddress(&p, g_anchor_scratch);
   if (e != cudaSuccess) return e;
-  if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
-  std::lock_guard<std::mutex> lock(g_setup_mu);
-  if (!g_scratch_dev[dev]) {
-    void* p = nullptr;
-    e = cudaGetSymbolAddress(&p, g_anchor_scratch);
-    if (e != cudaSuccess) return e;
-    g_scratch_dev[dev] = static_cast<float*>(p);
-  }
-  *ptr = g_scratch_dev[dev];
+  *ptr = static_cast<float*>(p);
   return cudaSuccess;
 }
 
@@ -174,6 +164,12 @@ TXS_API txs_status txs_pool_anchor_static(const txs_model* model, int32_t n_req,
     if (beh_offsets[r + 1] == beh_offsets[r]) return TXS_ERR_COLD_START;
   }
   const int d = model_d(model);
+  if (d > kMaxD) {
+    const std::string msg = "txs_pool_anchor_static: d_model " + std::to_string(d) + " is above the limit of " +
+                            std::to_string(kMaxD);
+    set_last_error(msg.c_str());
+    return TXS_ERR_UNSUPPORTED;
+  }
   const long long need = static_cast<long long>(n_req) * kSlots * (d + 2);
   if (n_req > kMaxReq || need > kScratchFloats) {
     const std::string msg = "txs_pool_anchor_static: " + std::to_string(n_req) + " requests of width " +

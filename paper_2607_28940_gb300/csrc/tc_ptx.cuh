@@ -26,26 +26,40 @@ __device__ __forceinline__ void mbar_expect_tx(uint64_t* bar, uint32_t bytes) {
 
 // A waiting thread is suspended until the phase completes or kSuspendNs
 // passes, so a wait loop costs a few instructions per phase instead of
-// keeping the load/store pipe busy while the producer needs it.
+// keeping the load/store pipe busy while the producer needs it.  kSuspend =
+// false polls without the time hint (the attention pipelines, whose waits are
+// short and on the critical path of every key tile).
 constexpr uint32_t kSuspendNs = 1000000;
 
+template <bool kSuspend = true>
 __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
   uint32_t ok;
-  asm volatile(
-      "{\n\t.reg .pred p;\n\t"
-      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
-      "selp.u32 %0, 1, 0, p;\n\t}"
-      : "=r"(ok)
-      : "r"(smem_u32(bar)), "r"(parity), "r"(kSuspendNs)
-      : "memory");
+  if constexpr (kSuspend) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(smem_u32(bar)), "r"(parity), "r"(kSuspendNs)
+        : "memory");
+  } else {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(smem_u32(bar)), "r"(parity)
+        : "memory");
+  }
   return ok != 0;
 }
 
 // Wait for the phase of `parity` to complete; gives up (returning false) when
 // another role raised *abort or after kSpinCycles, raising *abort itself.
+template <bool kSuspend = true>
 __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort) {
   const long long t0 = clock64();
-  while (!mbar_try_wait(bar, parity)) {
+  while (!mbar_try_wait<kSuspend>(bar, parity)) {
     if (*abort) return false;
     if (clock64() - t0 > kSpinCycles) {
       *abort = 1;
@@ -55,9 +69,10 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volati
   return true;
 }
 
+template <bool kSuspend = true>
 __device__ __forceinline__ bool mbar_wait_plain(uint64_t* bar, uint32_t parity) {
   const long long t0 = clock64();
-  while (!mbar_try_wait(bar, parity))
+  while (!mbar_try_wait<kSuspend>(bar, parity))
     if (clock64() - t0 > kSpinCycles) return false;
   return true;
 }

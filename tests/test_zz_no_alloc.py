@@ -8,7 +8,9 @@ cudaFree imply.  Its scratch is a fixed array inside the library, shared by
 every call, so the test checks two calls in a row: the second must not see
 anything the first left behind.  Both are compared with the pooled anchor
 that the cache build (txs_build_kv_cache, read back with
-txs_cache_read_anchor) computes for the same rows.
+txs_cache_read_anchor) computes for the same rows, and with the fp64
+oracle's attention pooling of each request's rows (alpha = softmax(phi .
+w_pool / sqrt(d)), g = alpha^T phi; Sec. 4.1.2 global token, Sec. 5.1).
 
 The file name makes pytest collect it last, so a run that stops at the first
 failure has run every other test before this one.
@@ -17,6 +19,7 @@ import numpy as np
 import pytest
 import torch
 
+from oracle import txs_oracle as O
 from paper_2607_28940_gb300 import txs
 from paper_2607_28940_gb300 import workload as W
 
@@ -56,6 +59,9 @@ def test_static_pooling_matches_cache_build_on_two_calls_in_a_row(dtype):
         got = got.cpu().numpy()
         ref = _anchor_from_cache_build(model, b, beh)
         np.testing.assert_allclose(got, ref, atol=ATOL, rtol=RTOL)
+        om = O.Model.from_arrays(weights, wl)
+        g64 = np.stack([O.pool_direct(om, b.beh[b.beh_off[r]:b.beh_off[r + 1]]).g for r in range(wl.n_req)])
+        np.testing.assert_allclose(got, g64, atol=ATOL, rtol=RTOL)
         results.append(got)
     assert model.device_status() == txs.TXS_OK
     # the first batch again gives the same values as its first call
