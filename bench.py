@@ -105,10 +105,12 @@ def load_peaks():
 
 # ---------------------------------------------------------------- algorithmic work per class
 
-def algorithmic(wl: W.Workload, mode: int, L: np.ndarray, M: np.ndarray, dL: np.ndarray):
+def algorithmic(wl: W.Workload, mode: int, L: np.ndarray, M: np.ndarray, dL: np.ndarray, fused_lg: bool = False):
     """Per-step algorithmic (flops, bytes) of each kernel class: what the method
     must compute and move (bf16 operands, fp32 vectors), independent of how the
-    kernels tile it."""
+    kernels tile it.  fused_lg: the LOCAL_GLOBAL attention of the candidate
+    rows runs inside the query projection (class gemm_q_attn_lg) and only the
+    context-token rows go through a separate attention launch (attn_cross)."""
     es = 2 if wl.dtype == "bf16" else 4
     d, F, nL, H, S, k = wl.d_model, wl.d_ff, wl.n_layers, wl.n_heads, wl.n_ctx, wl.n_actions
     R = wl.n_req
@@ -139,9 +141,17 @@ def algorithmic(wl: W.Workload, mode: int, L: np.ndarray, M: np.ndarray, dL: np.
         add("gemm_qkv", gemm(N, 3 * d, d))
         add("attn_serving", (4.0 * d * (n_cand * (S + 1) + R * S * S), es * (N * 3 * d + N * d)))
         add("gemm_oproj_ln", gemm(N, d, d, res=True))
-        add("gemm_q", gemm(N, d, d))
         kv_bytes = float((W_keys * 2 * d * es).sum())
-        add("attn_cross", (float((4.0 * d * rows_per_req * W_keys).sum()), es * 2 * N * d + kv_bytes))
+        if fused_lg:
+            # query projection and the candidate rows' attention in one kernel
+            # (the query of a candidate row never goes to memory); the context
+            # rows' queries go out and their attention runs separately
+            qf, qb = gemm(N, d, d)
+            add("gemm_q_attn_lg", (qf + float((4.0 * d * M * W_keys).sum()), qb + kv_bytes))
+            add("attn_cross", (float((4.0 * d * S * W_keys).sum()), es * 3 * R * S * d + kv_bytes))
+        else:
+            add("gemm_q", gemm(N, d, d))
+            add("attn_cross", (float((4.0 * d * rows_per_req * W_keys).sum()), es * 2 * N * d + kv_bytes))
         add("gemm_oproj_ln", gemm(N, d, d, res=True))
         add("gemm_ffn1_gelu", gemm(N, F, d))
         add("gemm_ffn2_ln", gemm(N, d, F, res=True))
@@ -316,7 +326,7 @@ def run_txs(args, rank, world):
     out["clocks"] = clocks.summary()
 
     peaks, peak_src = load_peaks()
-    alg = algorithmic(wl, mode, b.L, b.M, b.dL)
+    alg = algorithmic(wl, mode, b.L, b.M, b.dL, fused_lg="gemm_q_attn_lg" in prof)
     kern = {}
     for name, (tot, cnt) in prof.items():
         per_step_ms = tot / args.steps

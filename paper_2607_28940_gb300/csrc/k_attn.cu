@@ -418,6 +418,105 @@ cudaError_t launch_cross_attn_lg(const T* q, T* out, const T* Kc, const T* Vc, c
   return err;
 }
 
+// LOCAL_GLOBAL cross-attention of the S context-token rows of every request
+// (rows n_cand + r S + j of the packed layout), whose q the fused query
+// projection left in `q`: one warp per (row, head).  Lane t < W scores the
+// request's window row t, lane W its anchor (Sec. 4.1.2 sparse
+// cross-attention equation, scale 1/sqrt(d_h)); the softmax runs across the
+// lanes; lane c then sums the weighted values of output columns c, c + 32.
+struct CtxAttnArgs {
+  int n_req, n_cand, S, H, d, dkv, group, l_local;
+  const int* kv_off;
+  const int* kv_len;
+  const float* Kg;
+  const float* Vg;
+  float scale_log2;
+};
+
+template <int DH>
+__global__ void __launch_bounds__(256) ctx_attn_kernel(const __nv_bfloat16* __restrict__ q,
+                                                       __nv_bfloat16* __restrict__ out,
+                                                       const __nv_bfloat16* __restrict__ Kc,
+                                                       const __nv_bfloat16* __restrict__ Vc, const CtxAttnArgs a) {
+  pdl_launch_dependents();
+  pdl_wait();
+  const int lane = threadIdx.x & 31;
+  const int gw = blockIdx.x * 8 + (threadIdx.x >> 5);
+  if (gw >= a.n_req * a.S * a.H) return;                     // uniform per warp
+  const int i = gw / a.H, h = gw - i * a.H;
+  const int r = i / a.S;
+  const long long row = static_cast<long long>(a.n_cand) + i;
+  const int kcol = (h / a.group) * DH;
+  const int len = __ldg(a.kv_len + r);
+  const int lo = len > a.l_local ? len - a.l_local : 0;
+  const int W = len - lo;
+  const long long base = static_cast<long long>(__ldg(a.kv_off + r)) + lo;
+  // this lane's key: window row `lane` or (lane W) the anchor
+  float s = -INFINITY;
+  if (lane <= W) {
+    float qv[DH], kv[DH];
+#pragma unroll
+    for (int c = 0; c < DH; c += 8) Vec16<__nv_bfloat16>::load(q + row * a.d + h * DH + c, qv + c);
+    if (lane < W) {
+#pragma unroll
+      for (int c = 0; c < DH; c += 8) Vec16<__nv_bfloat16>::load(Kc + (base + lane) * a.dkv + kcol + c, kv + c);
+    } else {
+#pragma unroll
+      for (int c = 0; c < DH; c += 4) {
+        const float4 g4 = __ldg(reinterpret_cast<const float4*>(a.Kg + static_cast<long long>(r) * a.dkv + kcol + c));
+        kv[c] = g4.x; kv[c + 1] = g4.y; kv[c + 2] = g4.z; kv[c + 3] = g4.w;
+      }
+    }
+    float acc[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+    for (int c = 0; c < DH; ++c) acc[c & 3] = fmaf(qv[c], kv[c], acc[c & 3]);
+    s = ((acc[0] + acc[1]) + (acc[2] + acc[3])) * a.scale_log2;
+  }
+  float mx = s;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+  const float p = lane <= W ? exp2f(s - mx) : 0.f;
+  float sum = p;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
+  // output columns lane, lane + 32 (DH = 64) of this head
+  float o0 = 0.f, o1 = 0.f;
+  for (int t = 0; t <= W; ++t) {
+    const float pt = __shfl_sync(0xffffffffu, p, t);
+    if (t < W) {
+      const __nv_bfloat16* vr = Vc + (base + t) * a.dkv + kcol;
+      o0 = fmaf(pt, __bfloat162float(vr[lane]), o0);
+      if (DH == 64) o1 = fmaf(pt, __bfloat162float(vr[lane + 32]), o1);
+    } else {
+      const float* vg = a.Vg + static_cast<long long>(r) * a.dkv + kcol;
+      o0 = fmaf(pt, __ldg(vg + lane), o0);
+      if (DH == 64) o1 = fmaf(pt, __ldg(vg + lane + 32), o1);
+    }
+  }
+  const float inv = 1.f / sum;
+  __nv_bfloat16* dst = out + row * a.d + h * DH;
+  dst[lane] = __float2bfloat16_rn(o0 * inv);
+  if (DH == 64) dst[lane + 32] = __float2bfloat16_rn(o1 * inv);
+}
+
+cudaError_t launch_ctx_attn_lg(const __nv_bfloat16* q, __nv_bfloat16* out, const __nv_bfloat16* Kc,
+                               const __nv_bfloat16* Vc, int n_req, int n_cand, int S, const int* kv_off,
+                               const int* kv_len, const float* Kg, const float* Vg, int l_local, int H, int Hkv,
+                               int d, cudaStream_t s) {
+  const int dh = d / H;
+  if ((dh != 32 && dh != 64) || l_local > 31 || Hkv < 1 || H % Hkv) return cudaErrorInvalidValue;
+  const long long warps = static_cast<long long>(n_req) * S * H;
+  if (warps == 0) return cudaSuccess;
+  CtxAttnArgs a{n_req, n_cand, S, H, d, Hkv * dh, H / Hkv, l_local, kv_off, kv_len, Kg, Vg,
+                1.4426950408889634f / sqrtf(static_cast<float>(dh))};
+  const dim3 grid(static_cast<unsigned>((warps + 7) / 8));
+  prof_begin(KC_ATTN_CROSS, s);
+  const cudaError_t err = dh == 64 ? launch_pdl(ctx_attn_kernel<64>, grid, dim3(256), 0, s, q, out, Kc, Vc, a)
+                                   : launch_pdl(ctx_attn_kernel<32>, grid, dim3(256), 0, s, q, out, Kc, Vc, a);
+  prof_end(KC_ATTN_CROSS, s);
+  return err;
+}
+
 template cudaError_t launch_cross_attn_lg<float>(const float*, float*, const float*, const float*, const int*,
                                                  const int*, int, int, int, const int*, const int*, const float*,
                                                  const float*, int, int, int, int, cudaStream_t);

@@ -53,6 +53,18 @@ constexpr int kStageSeg = 1024;   // request offsets staged in shared memory (ca
 
 
 
+constexpr int kStageNAtt = 512;   // bias entries staged with the fused attention (N = d <= 512)
+
+// Fused LOCAL_GLOBAL cross-attention (EPI_ATTN_LG): each epilogue warp owns
+// 64 query columns (one head of 64 or two of 32) of 32 rows.  Per request
+// among its rows it stages the K/V columns its heads read as 16 key slots of
+// bf16: slots 0 .. W-1 the window rows, W .. 14 zero, 15 the anchor.
+constexpr int kAttKeys = 16;                  // key slots: window (at most 15 rows) + anchor
+constexpr int kAttAnchor = kAttKeys - 1;
+constexpr int kAttWinMax = kAttKeys - 1;      // longest window the fused path takes
+constexpr int kAttCols = 64;                  // query columns per epilogue warp
+constexpr int kAttKvBytes = kAttKeys * kAttCols * 2;   // one of K, V staged for one warp
+
 constexpr int kEpiWarps = 8;                  // two warps per TMEM lane quarter
 constexpr int NUM_THREADS = 64 + 32 * kEpiWarps;
 constexpr int kRedStride = 17;                // per-row exchange slots: sum + 16 logits
@@ -250,10 +262,386 @@ __device__ __forceinline__ void epilogue(const EpiArgs& e, uint32_t tacc, int ro
   }
 }
 
+// ------------------------------------------------------------------ fused LOCAL_GLOBAL attention
+
+// The attention of one warp's 32 query rows against one request's 16 key
+// slots is two small matrix products per head, S = Q K^T (32 x 16, inner
+// dimension d_h) and O = P V (32 x d_h, inner dimension 16).  They run as
+// warp-level bf16 MMAs (m16n8k16, fp32 accumulation) on shared-memory tiles
+// of this warp; the softmax runs on the S fragments in registers, and the P
+// fragments are the A operand of the second product (the S accumulator
+// layout of two 8-key tiles is the A layout of one 16-key step).  The
+// tcgen05 MMAs of the projection are issued by one thread for the whole
+// 128-row tile; these products belong to each warp's own rows and keys.
+
+__device__ __forceinline__ void mma_16816(float* d, const uint32_t* a, const uint32_t* b) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
+      "{%0,%1,%2,%3};"
+      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b[0]), "r"(b[1]));
+}
+__device__ __forceinline__ void ldsm_x4(uint32_t* r, uint32_t addr) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];"
+               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+               : "r"(addr));
+}
+__device__ __forceinline__ void ldsm_x4_t(uint32_t* r, uint32_t addr) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];"
+               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+               : "r"(addr));
+}
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
+  __nv_bfloat162 h = __floats2bfloat162_rn(lo, hi);
+  return *reinterpret_cast<uint32_t*>(&h);
+}
+// Byte offset of 16-byte unit u of row r in a [rows][64] bf16 tile (128-byte
+// rows; units XOR-swizzled by the row so that eight rows read as an 8 x 8
+// matrix hit distinct banks).
+__device__ __forceinline__ uint32_t tile_off(int r, int u) {
+  return static_cast<uint32_t>(r * 128 + ((u ^ (r & 7)) << 4));
+}
+
+// Row tile of tile t in the fused-attention kernel: the row tiles are
+// rotated so that the last one (the context-token rows of every request,
+// whose warps attend to many requests each) is processed in the first round
+// by the last CTAs, which have no extra tile in the last round.
+__device__ __forceinline__ int att_tile_m(int t, int n_tiles, int m_tiles) {
+  const int shift = static_cast<int>(gridDim.x) / n_tiles - 1;   // first-round position of the last row tile
+  return (t / n_tiles + m_tiles - 1 + (m_tiles - shift % m_tiles)) % m_tiles;
+}
+
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src, uint32_t src_bytes) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src), "r"(src_bytes) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+__device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_all;" ::: "memory"); }
+
+// Shared memory of one epilogue warp for the fused attention: two K/V
+// buffers (16 key slots x 64 columns bf16 each for K and V) and two fp32
+// anchor rows (K then V, 64 columns each); q and the outputs use the warp's
+// bulk-store staging buffers.
+constexpr int kAttBufBytes = 2 * kAttKvBytes + 2 * kAttCols * 4;
+constexpr int kAttWarpBytes = 2 * kAttBufBytes;
+
+// This lane's row: its request, that request's window rows and first window
+// row in the cache (W = 0 for a row past M).
+struct AttRow {
+  int r;
+  int W;
+  long long base;
+};
+__device__ __forceinline__ void att_row_meta(const EpiArgs& e, AttRow& a) {
+  a.W = 0;
+  a.base = 0;
+  if (a.r >= 0) {
+    const int len = __ldg(e.att_kv_len + a.r);
+    const int lo = len > e.att_l_local ? len - e.att_l_local : 0;
+    a.W = len - lo;                                           // <= kAttWinMax (checked on the host)
+    a.base = static_cast<long long>(__ldg(e.att_kv_off + a.r)) + lo;
+  }
+}
+
+// K/V columns [kc0, kc0 + kvw) read by the heads of query columns
+// [col0, col0 + 64): kvw <= 64, a whole number of heads.
+__device__ __forceinline__ void att_kv_cols(const EpiArgs& e, int col0, int& kc0, int& kvw) {
+  const int dh = e.att_dh, grp = e.att_group;
+  kc0 = (col0 / dh) / grp * dh;
+  kvw = ((col0 + kAttCols - 1) / dh) / grp * dh + dh - kc0;
+}
+
+// Starts the asynchronous copies of request rc's key slots into buffer `buf`:
+// window rows 0 .. W-1 of the K and V columns [kc0, kc0 + kvw), zero-filled
+// slots W .. 14, and the fp32 anchor columns; one commit group.
+__device__ __forceinline__ void att_issue(const EpiArgs& e, int rc, int W, long long base, int kc0, int kvw,
+                                          uint8_t* buf, int lane) {
+  const __nv_bfloat16* Kc = static_cast<const __nv_bfloat16*>(e.att_k);
+  const __nv_bfloat16* Vc = static_cast<const __nv_bfloat16*>(e.att_v);
+  const uint32_t sK = smem_u32(buf), sV = sK + kAttKvBytes, sA = sV + kAttKvBytes;
+  const int per_row = kvw / 8;
+  const long long dkv = e.att_dkv;
+  for (int idx = lane; idx < kAttWinMax * per_row; idx += 32) {
+    const int t = idx / per_row, u = idx - t * per_row;
+    const bool in = t < W;
+    const long long src = (base + (in ? t : 0)) * dkv + kc0 + 8 * u;   // a valid row when zero-filling
+    cp_async16(sK + tile_off(t, u), Kc + src, in ? 16u : 0u);
+    cp_async16(sV + tile_off(t, u), Vc + src, in ? 16u : 0u);
+  }
+  const int q4 = kvw / 4;
+  for (int i = lane; i < 2 * q4; i += 32) {
+    const bool isv = i >= q4;
+    const int c = 4 * (isv ? i - q4 : i);
+    cp_async16(sA + (isv ? kAttCols * 4 : 0) + 4 * c, (isv ? e.att_vg : e.att_kg) + rc * dkv + kc0 + c, 16u);
+  }
+  cp_async_commit();
+}
+
+// After the copies into `buf` have landed: the anchor (fp32) into key slot
+// 15 of the K and V tiles as bf16.
+__device__ __forceinline__ void att_anchor_slot(uint8_t* buf, int kvw, int lane) {
+  uint8_t* sK = buf;
+  uint8_t* sV = buf + kAttKvBytes;
+  const float* sA = reinterpret_cast<const float*>(buf + 2 * kAttKvBytes);
+  for (int c = lane; c < kvw; c += 32) {
+    const uint32_t off = tile_off(kAttAnchor, c >> 3) + (c & 7) * 2;
+    *reinterpret_cast<__nv_bfloat16*>(sK + off) = __float2bfloat16_rn(sA[c]);
+    *reinterpret_cast<__nv_bfloat16*>(sV + off) = __float2bfloat16_rn(sA[kAttCols + c]);
+  }
+}
+
+// Starts the copies for the request of the first lane in `lanes` (if any).
+__device__ __forceinline__ void att_issue_first(const EpiArgs& e, const AttRow& a, unsigned lanes, int kc0, int kvw,
+                                                uint8_t* buf, int lane) {
+  if (!lanes) return;
+  const int l = __ffs(lanes) - 1;
+  const int rc = __shfl_sync(0xffffffffu, a.r, l);
+  const int W = __shfl_sync(0xffffffffu, a.W, l);
+  const long long base = __shfl_sync(0xffffffffu, a.base, l);
+  att_issue(e, rc, W, base, kc0, kvw, buf, lane);
+}
+
+// The heads (DH = 64: one, 32: two) of one warp's 32 query rows (q in sQ,
+// bf16, 128-byte swizzled rows) against the key slots of each request among
+// its rows (rows of other requests get p = 0), one request after another;
+// the copies for the next request are started before each request's
+// products, those for the next tile's first request (its rows are `nxt`)
+// after the last request's products.  Writes the normalised attention output (bf16) into
+// the two staging buffers at `stage` (over sQ, once every read of q is done).
+template <int DH>
+__device__ __forceinline__ void att_tile(const EpiArgs& e, const AttRow& cur, const AttRow& nxt, bool has_next,
+                                         int lane, int col0, int kc0, int kvw, int kn0, int kvwn, uint8_t* sQ,
+                                         uint8_t* att, int& buf, uint8_t* stage) {
+  const int g = lane >> 2, tq = lane & 3;                     // MMA fragment row group / column pair
+  const int grp = e.att_group;
+  // rows of the fragment slots s = 2 mt + hf (m-tile mt, half hf): 8 s + g
+  int rreq[4];
+#pragma unroll
+  for (int s = 0; s < 4; ++s) rreq[s] = __shfl_sync(0xffffffffu, cur.r, 8 * s + g);
+  const uint32_t aQ = smem_u32(sQ);
+  const int mi = lane >> 3, rr = lane & 7;                     // ldmatrix: matrix index, row within it
+  const float sc = e.att_scale_log2;
+  constexpr int hpw = kAttCols / DH;                           // heads of this warp (1 or 2)
+  float o[2][8][4];                                            // [m-tile][8-column tile][fragment]
+  float lsum[2][2][2];                                         // row sums [head][m-tile][half]
+#pragma unroll
+  for (int mt = 0; mt < 2; ++mt) {
+#pragma unroll
+    for (int hl = 0; hl < 2; ++hl) lsum[hl][mt][0] = lsum[hl][mt][1] = 0.f;
+#pragma unroll
+    for (int n = 0; n < 8; ++n) o[mt][n][0] = o[mt][n][1] = o[mt][n][2] = o[mt][n][3] = 0.f;
+  }
+  unsigned pending = __ballot_sync(0xffffffffu, cur.r >= 0);
+  while (pending) {
+    const int leader = __ffs(pending) - 1;
+    const int rc = __shfl_sync(0xffffffffu, cur.r, leader);
+    const int W = __shfl_sync(0xffffffffu, cur.W, leader);
+    pending &= ~__ballot_sync(0xffffffffu, cur.r == rc);
+    uint8_t* cb = att + buf * kAttBufBytes;
+    cp_async_wait_all();                                      // this request's slots have landed
+    __syncwarp();
+    att_anchor_slot(cb, kvw, lane);
+    // the next copies go to the other buffer, whose last readers (the
+    // products of the previous request) are done
+    uint8_t* nb = att + (buf ^ 1) * kAttBufBytes;
+    if (pending) att_issue_first(e, cur, pending, kc0, kvw, nb, lane);
+    __syncwarp();
+    const uint32_t aK = smem_u32(cb), aV = aK + kAttKvBytes;
+#pragma unroll
+    for (int hl = 0; hl < 2; ++hl) {
+      if (hl >= hpw) break;
+      const int ku = (((col0 + hl * DH) / DH) / grp * DH - kc0) / 8;   // this head's first K/V unit
+      const int qu = hl * DH / 8;                                      // its first query unit
+      constexpr int nks = DH / 16;                                     // k-steps of S
+      // S = Q K^T: [m-tile][key tile][fragment]
+      float sfr[2][2][4];
+#pragma unroll
+      for (int mt = 0; mt < 2; ++mt)
+#pragma unroll
+        for (int nt = 0; nt < 2; ++nt) sfr[mt][nt][0] = sfr[mt][nt][1] = sfr[mt][nt][2] = sfr[mt][nt][3] = 0.f;
+#pragma unroll
+      for (int ks = 0; ks < nks; ++ks) {
+        uint32_t kb[4];   // key tile 0 (dims lo, hi), key tile 1 (dims lo, hi)
+        ldsm_x4(kb, aK + tile_off((mi >> 1) * 8 + rr, ku + 2 * ks + (mi & 1)));
+#pragma unroll
+        for (int mt = 0; mt < 2; ++mt) {
+          uint32_t qa[4];
+          ldsm_x4(qa, aQ + tile_off(16 * mt + (mi & 1) * 8 + rr, qu + 2 * ks + (mi >> 1)));
+          mma_16816(sfr[mt][0], qa, kb);
+          mma_16816(sfr[mt][1], qa, kb + 2);
+        }
+      }
+      // softmax of each row over its valid slots (window rows below W and
+      // the anchor), exp2 of log2-scaled scores; P as the A fragment
+      uint32_t pa[2][4];
+#pragma unroll
+      for (int mt = 0; mt < 2; ++mt) {
+#pragma unroll
+        for (int hf = 0; hf < 2; ++hf) {
+          const bool mine = rreq[2 * mt + hf] == rc;
+          float x[4];
+#pragma unroll
+          for (int i = 0; i < 4; ++i) {
+            const int key = (i >> 1) * 8 + 2 * tq + (i & 1);
+            x[i] = key < W || key == kAttAnchor ? sfr[mt][i >> 1][2 * hf + (i & 1)] * sc : -INFINITY;
+          }
+          float mx = fmaxf(fmaxf(x[0], x[1]), fmaxf(x[2], x[3]));
+          mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 1));
+          mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 2));
+          float sum = 0.f;
+#pragma unroll
+          for (int i = 0; i < 4; ++i) {
+            x[i] = mine ? exp2f(x[i] - mx) : 0.f;
+            sum += x[i];
+          }
+          sum += __shfl_xor_sync(0xffffffffu, sum, 1);
+          sum += __shfl_xor_sync(0xffffffffu, sum, 2);
+          if (mine) lsum[hl][mt][hf] = sum;
+          pa[mt][hf] = pack_bf16x2(x[0], x[1]);                  // slots 2 tq, 2 tq + 1
+          pa[mt][2 + hf] = pack_bf16x2(x[2], x[3]);              // slots 8 + 2 tq, 9 + 2 tq
+        }
+      }
+      // O += P V over this head's 8-column tiles (two per transposed load)
+#pragma unroll
+      for (int j = 0; j < DH / 8; j += 2) {
+        uint32_t vb[4];   // column tile j (slots 0-7, 8-15), column tile j + 1 (slots 0-7, 8-15)
+        ldsm_x4_t(vb, aV + tile_off((mi & 1) * 8 + rr, ku + j + (mi >> 1)));
+#pragma unroll
+        for (int mt = 0; mt < 2; ++mt) {
+          mma_16816(o[mt][qu + j], pa[mt], vb);
+          mma_16816(o[mt][qu + j + 1], pa[mt], vb + 2);
+        }
+      }
+    }
+    // after the tile's last request: the next tile's first request (its
+    // window was looked up during this tile)
+    if (!pending && has_next) att_issue_first(e, nxt, __ballot_sync(0xffffffffu, nxt.r >= 0), kn0, kvwn, nb, lane);
+    buf ^= 1;
+  }
+  // no request among this warp's rows (all past M): the next tile's copies
+  // (nothing is in flight for this tile)
+  if (!__ballot_sync(0xffffffffu, cur.r >= 0) && has_next)
+    att_issue_first(e, nxt, __ballot_sync(0xffffffffu, nxt.r >= 0), kn0, kvwn, att + buf * kAttBufBytes, lane);
+  // normalise and store: output column 8 n + 2 tq (+1) of rows 16 mt + g and
+  // 16 mt + 8 + g into the staging buffers (over q, whose reads are done)
+  __syncwarp();
+#pragma unroll
+  for (int mt = 0; mt < 2; ++mt) {
+#pragma unroll
+    for (int hf = 0; hf < 2; ++hf) {
+      const int orow = 16 * mt + 8 * hf + g;
+#pragma unroll
+      for (int n = 0; n < 8; ++n) {
+        const float l = lsum[(8 * n) / DH][mt][hf];
+        const float inv = l > 0.f ? 1.f / l : 0.f;
+        const int col = 8 * n + 2 * tq;
+        const int cc = col & 31, u = cc >> 3;
+        uint8_t* sb = stage + (col >> 5) * 2048;
+        *reinterpret_cast<uint32_t*>(sb + orow * 64 + ((u ^ ((orow >> 1) & 3)) << 4) + (cc & 7) * 2) =
+            pack_bf16x2(o[mt][n][2 * hf] * inv, o[mt][n][2 * hf + 1] * inv);
+      }
+    }
+  }
+}
+
+// The fused epilogue of EPI_ATTN_LG for one epilogue warp over all its tiles
+// (TMEM lane quarter q, column half h): per tile, q = acc + b_Q rounded to
+// bf16 (the accumulator is released as soon as it has been read), then per
+// head the softmax over the request's window rows and anchor of
+// q . k / sqrt(d_h) and the weighted values (Sec. 4.1.2 sparse
+// cross-attention equation with the local-global key set), stored where q
+// would have gone.  The key slots of each tile's first request are copied
+// while the previous tile computes; this lane's row request for the next
+// tile is read at the start of the current one.
+__device__ __forceinline__ void attn_epilogue_warp(const EpiArgs& e, uint32_t tmem_q, uint64_t* acc_full,
+                                                   uint64_t* acc_empty, volatile int* abort_flag, int t_lo, int t_hi,
+                                                   int t_step, int n_tiles, int m_tiles, int q, int h,
+                                                   const float* bias, const CUtensorMap* tmO, uint8_t* stage,
+                                                   uint8_t* att) {
+  constexpr int BNA = 2 * kAttCols;
+  const int lane = threadIdx.x & 31;
+  auto row_of = [&](int t) { return att_tile_m(t, n_tiles, m_tiles) * BM + q * 32 + lane; };
+  auto col_of = [&](int t) { return (t % n_tiles) * BNA + h * kAttCols; };
+  // request attended by this lane's row of tile t (-1: past M, or a
+  // context-token row, attended by a separate launch)
+  auto req_of = [&](int t) {
+    return t < t_hi && row_of(t) < e.att_n_cand ? __ldg(e.att_row_req + row_of(t)) : -1;
+  };
+  // this lane's row in the current tile (cur) and the next (nxt, window
+  // looked up during the current tile), and the request of its row two tiles
+  // ahead (r2, read during the current tile)
+  AttRow cur, nxt;
+  int buf = 0;
+  if (t_lo < t_hi) {
+    cur.r = req_of(t_lo);
+    att_row_meta(e, cur);
+    int kc0, kvw;
+    att_kv_cols(e, col_of(t_lo), kc0, kvw);
+    att_issue_first(e, cur, __ballot_sync(0xffffffffu, cur.r >= 0), kc0, kvw, att, lane);
+    nxt.r = req_of(t_lo + t_step);
+  }
+  int i = 0;
+  for (int t = t_lo; t < t_hi; t += t_step, ++i) {
+    const int b = i & 1;
+    const bool has_next = t + t_step < t_hi;
+    const int row = row_of(t), col0 = col_of(t);
+    const int r2 = req_of(t + 2 * t_step);
+    att_row_meta(e, nxt);
+    bool go = mbar_wait(acc_full + b, (i >> 1) & 1, abort_flag);
+    go = __shfl_sync(0xffffffffu, go ? 1 : 0, 0) != 0;
+    if (!go) break;
+    tc_fence_after();
+    // q = acc + b_Q (bf16) into the staging buffers, free of earlier stores
+    if (lane == 0) bulk_wait_read<0>();
+    __syncwarp();
+    uint8_t* sQ = stage;
+    {
+      float w[kAttCols];
+      tmem_ld64(tmem_q + b * BNA + h * kAttCols, w);
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(acc_empty + b);              // the accumulator may be reused
+#pragma unroll
+      for (int u = 0; u < kAttCols / 8; ++u) {
+        uint4 pk;
+        pk.x = pack_bf16x2(w[8 * u] + bias[col0 + 8 * u], w[8 * u + 1] + bias[col0 + 8 * u + 1]);
+        pk.y = pack_bf16x2(w[8 * u + 2] + bias[col0 + 8 * u + 2], w[8 * u + 3] + bias[col0 + 8 * u + 3]);
+        pk.z = pack_bf16x2(w[8 * u + 4] + bias[col0 + 8 * u + 4], w[8 * u + 5] + bias[col0 + 8 * u + 5]);
+        pk.w = pack_bf16x2(w[8 * u + 6] + bias[col0 + 8 * u + 6], w[8 * u + 7] + bias[col0 + 8 * u + 7]);
+        *reinterpret_cast<uint4*>(sQ + tile_off(lane, u)) = pk;
+        if (row >= e.att_n_cand && row < e.M)   // a context-token row: its q for the separate launch
+          *reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(e.att_q_ctx) + static_cast<long long>(row) * e.ldo +
+                                    col0 + 8 * u) = pk;
+      }
+    }
+    __syncwarp();
+    int kc0, kvw, kn0 = 0, kvwn = 0;
+    att_kv_cols(e, col0, kc0, kvw);
+    if (has_next) att_kv_cols(e, col_of(t + t_step), kn0, kvwn);
+    if (e.att_dh == 64)
+      att_tile<64>(e, cur, nxt, has_next, lane, col0, kc0, kvw, kn0, kvwn, sQ, att, buf, stage);
+    else
+      att_tile<32>(e, cur, nxt, has_next, lane, col0, kc0, kvw, kn0, kvwn, sQ, att, buf, stage);
+    // rows past M hold stale values; the bulk stores of the [M, N] output
+    // drop those rows
+    fence_async_smem();
+    __syncwarp();
+    if (lane == 0) {
+      tma_store_2d(tmO, stage, col0, row - lane);
+      tma_store_2d(tmO, stage + 2048, col0 + 32, row - lane);
+      bulk_commit();
+    }
+    cur = nxt;
+    nxt.r = r2;
+  }
+  cp_async_wait_all();                                        // no copy outlives the kernel's shared memory
+  if (lane == 0) bulk_wait_all();
+}
+
 // ------------------------------------------------------------------ kernel
 
 // BRES: the CTA's whole B slice (BN x K, K <= KRES) stays resident in shared
-// memory and only A streams through the ring.
+// memory and only A streams through the ring.  NAP: head actions padded
+// (EPI_LN_HEAD).
 template <int BN, int EPI, int NAP = 4, bool BRES = false>
 struct Shape {
   static constexpr int BN_MMA = BN < 256 ? BN : 256;     // N of one tcgen05.mma
@@ -268,12 +656,15 @@ struct Shape {
   // bias [kStageN] floats ([kStageNRes] with BRES), then (cache-row remap) offsets and
   // first rows; rounded to 1 KB so that the staging buffers after it start on
   // a swizzle-atom boundary
+  static constexpr bool ATT = EPI == EPI_ATTN_LG;
+  static constexpr int STAGE_N = BRES ? kStageNRes : ATT ? kStageNAtt : kStageN;
   static constexpr int AUX_BYTES =
-      LN ? 0
-         : (((BRES ? kStageNRes * 4 : kStageN * 4) + (EPI == EPI_KV ? (2 * kStageSeg + 1) * 4 : 0) + 1023) / 1024) * 1024;
+      LN ? 0 : (((STAGE_N * 4) + (EPI == EPI_KV ? (2 * kStageSeg + 1) * 4 : 0) + 1023) / 1024) * 1024;
+  // fused attention: each epilogue warp's staged window and anchor (fp32)
+  static constexpr int ATT_BYTES = ATT ? kEpiWarps * kAttWarpBytes : 0;
   // bulk-store staging: two 2 KB buffers per epilogue warp (bf16 outputs)
   static constexpr int STG_BYTES = EPI == EPI_LN_HEAD ? 0 : kEpiWarps * 2 * 2048;
-  static constexpr int EXTRA = BRES_BYTES + RED_BYTES + WEFF_BYTES + AUX_BYTES + STG_BYTES + 1024 + 256;
+  static constexpr int EXTRA = BRES_BYTES + RED_BYTES + WEFF_BYTES + AUX_BYTES + STG_BYTES + ATT_BYTES + 1024 + 256;
   static constexpr int STAGES_FIT = (227 * 1024 - EXTRA) / STAGE_BYTES;
   static constexpr int STAGES = STAGES_FIT > 8 ? 8 : STAGES_FIT;
   static constexpr int ACC_BUFS = BN <= 256 ? 2 : 1;      // TMEM double buffer
@@ -283,7 +674,9 @@ struct Shape {
   static_assert(!(BRES && LN), "resident B only for the plain epilogues");
   static_assert((RED_BYTES + WEFF_BYTES + AUX_BYTES) % 1024 == 0 || STG_BYTES == 0,
                 "staging buffers need 512-byte alignment (64-byte swizzle atoms)");
-  static_assert((RED_BYTES + WEFF_BYTES + AUX_BYTES + STG_BYTES) % 16 == 0, "mbarriers must stay 8-byte aligned");
+  static_assert((RED_BYTES + WEFF_BYTES + AUX_BYTES + STG_BYTES + ATT_BYTES) % 16 == 0,
+                "mbarriers must stay 8-byte aligned");
+  static_assert(!ATT || (BN == 2 * kAttCols && !BRES), "fused attention: 128-column tiles");
   static_assert(SMEM_BYTES <= 232448, "shared memory");
   static_assert((TMEM_COLS & (TMEM_COLS - 1)) == 0 && TMEM_COLS <= 512, "TMEM columns");
 };
@@ -323,10 +716,11 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   float* red = reinterpret_cast<float*>(sBres + S::BRES_BYTES);
   float* s_weff = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(red) + S::RED_BYTES);
   float* s_bias = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(s_weff) + S::WEFF_BYTES);
-  int* s_seg = reinterpret_cast<int*>(s_bias + (BRES ? kStageNRes : kStageN));
+  int* s_seg = reinterpret_cast<int*>(s_bias + S::STAGE_N);
   int* s_dst = s_seg + kStageSeg + 1;
   uint8_t* s_stage = reinterpret_cast<uint8_t*>(s_bias) + S::AUX_BYTES;
-  uint64_t* full = reinterpret_cast<uint64_t*>(s_stage + S::STG_BYTES);
+  uint8_t* s_att = s_stage + S::STG_BYTES;
+  uint64_t* full = reinterpret_cast<uint64_t*>(s_att + S::ATT_BYTES);
   uint64_t* empty = full + S::STAGES;
   uint64_t* acc_full = empty + S::STAGES;
   uint64_t* acc_empty = acc_full + 2;
@@ -348,7 +742,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     t_step = 1;
   }
   auto tile_n = [&](int t) { return BRES ? t / m_tiles : t % n_tiles; };
-  auto tile_m = [&](int t) { return BRES ? t % m_tiles : t / n_tiles; };
+  auto tile_m = [&](int t) { return BRES ? t % m_tiles : S::ATT ? att_tile_m(t, n_tiles, m_tiles) : t / n_tiles; };
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < S::STAGES; ++s) {
@@ -408,7 +802,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   const int* seg_off = e.seg_off;
   const int* dst_row0 = e.dst_row0;
   if constexpr (!S::LN) {
-    if (e.N <= (BRES ? kStageNRes : kStageN)) {
+    if (e.N <= S::STAGE_N) {
       for (int i = threadIdx.x; i < e.N; i += NUM_THREADS) s_bias[i] = e.bias[i];
       bias = s_bias;
     }
@@ -543,27 +937,32 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     const int q = warp & 3;           // TMEM lane quarter this warp may access
     const int h = ew / 4;             // column half
     uint8_t* stage = s_stage + ew * 4096;
-    int kchunk = 0;
-    int i = 0;
-    for (int t = t_lo; t < t_hi; t += t_step, ++i) {
-      const int buf = i % S::ACC_BUFS;
-      const uint32_t use = i / S::ACC_BUFS;
-      // Go on exactly when the accumulator is complete: both warps of a lane
-      // quarter see the same barrier phase, so they agree (they meet at named
-      // barriers inside the LayerNorm epilogues).  Warp-uniform because
-      // tcgen05.ld is .sync.aligned.
-      bool go = mbar_wait(acc_full + buf, use & 1, abort_flag);
-      go = __shfl_sync(0xffffffffu, go ? 1 : 0, 0) != 0;
-      if (!go) break;
-      tc_fence_after();
-      const int m0 = tile_m(t) * BM, n0 = tile_n(t) * BN;
-      epilogue<BN, EPI, NAP>(e, tmem + buf * BN + (static_cast<uint32_t>(q * 32) << 16), m0 + q * 32 + lane, n0,
-                             h * (BN / 2), q, h, red, s_weff, bias, seg_off, dst_row0, &tmO, stage, kchunk);
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(acc_empty + buf);
+    if constexpr (S::ATT) {
+      attn_epilogue_warp(e, tmem + (static_cast<uint32_t>(q * 32) << 16), acc_full, acc_empty, abort_flag, t_lo,
+                         t_hi, t_step, n_tiles, m_tiles, q, h, bias, &tmO, stage, s_att + ew * kAttWarpBytes);
+    } else {
+      int kchunk = 0;
+      int i = 0;
+      for (int t = t_lo; t < t_hi; t += t_step, ++i) {
+        const int buf = i % S::ACC_BUFS;
+        const uint32_t use = i / S::ACC_BUFS;
+        // Go on exactly when the accumulator is complete: both warps of a lane
+        // quarter see the same barrier phase, so they agree (they meet at named
+        // barriers inside the LayerNorm epilogues).  Warp-uniform because
+        // tcgen05.ld is .sync.aligned.
+        bool go = mbar_wait(acc_full + buf, use & 1, abort_flag);
+        go = __shfl_sync(0xffffffffu, go ? 1 : 0, 0) != 0;
+        if (!go) break;
+        tc_fence_after();
+        const int m0 = tile_m(t) * BM, n0 = tile_n(t) * BN;
+        epilogue<BN, EPI, NAP>(e, tmem + buf * BN + (static_cast<uint32_t>(q * 32) << 16), m0 + q * 32 + lane, n0,
+                               h * (BN / 2), q, h, red, s_weff, bias, seg_off, dst_row0, &tmO, stage, kchunk);
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(acc_empty + buf);
+      }
+      if (lane == 0) bulk_wait_all();   // this warp's bulk stores are complete before exit
     }
-    if (lane == 0) bulk_wait_all();   // this warp's bulk stores are complete before exit
   }
   tc_fence_before();
   __syncthreads();
@@ -704,6 +1103,7 @@ static cudaError_t launch_bn(const __nv_bfloat16* A, long long lda, const __nv_b
 bool tc_gemm_supported(int N, int K, int epi) {
   if (K <= 0 || K % BK != 0 || N <= 0) return false;
   if (epi == EPI_LN || epi == EPI_LN_HEAD) return N == 64 || N == 128 || N == 256 || N == 512;
+  if (epi == EPI_ATTN_LG) return N % 128 == 0 && N <= kStageNAtt;
   return N % 64 == 0;
 }
 
@@ -766,6 +1166,11 @@ cudaError_t launch_gemm_tc(const __nv_bfloat16* A, long long lda, const __nv_bfl
     case EPI_BIAS: return launch_plain<EPI_BIAS>(A, lda, B, e, s, cls);
     case EPI_BIAS_GELU: return launch_plain<EPI_BIAS_GELU>(A, lda, B, e, s, cls);
     case EPI_KV: return launch_plain<EPI_KV>(A, lda, B, e, s, cls);
+    case EPI_ATTN_LG:
+      if ((e.att_dh != 32 && e.att_dh != 64) || e.att_l_local < 0 || e.att_l_local > kAttWinMax ||
+          e.att_group < 1 || e.att_dkv % 8 != 0)
+        return cudaErrorNotSupported;
+      return launch_bn<128, EPI_ATTN_LG>(A, lda, B, e, s, cls);
     default: return cudaErrorInvalidValue;
   }
 }

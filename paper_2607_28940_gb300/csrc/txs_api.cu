@@ -481,6 +481,11 @@ txs_status score_impl(txs_model* m, const KvView& c, int n_req, const int32_t* c
     TXS_CK(gemm(m, Hf, Fc, m->Wt_c2, e, tmp, s, KC_CAND_MLP));
   }
   const T* kv = static_cast<const T*>(c.kv);
+  // LOCAL_GLOBAL attention fused into the query projection (bf16; heads of
+  // 32 or 64 columns, 128-column query tiles, windows of at most 16 rows)
+  const int dh = d / H;
+  const bool lg_fused = std::is_same<T, __nv_bfloat16>::value && cf.attn_mode == TXS_ATTN_LOCAL_GLOBAL &&
+                        (dh == 32 || dh == 64) && d % 128 == 0 && d <= 512 && cf.l_local <= 16 && dkv % 8 == 0;
   for (int l = 0; l < cf.n_layers; ++l) {
     const LayerW& W = m->layers[l];
     // serving-stream attention (App. B mask), O-projection + residual + LN1
@@ -501,6 +506,45 @@ txs_status score_impl(txs_model* m, const KvView& c, int n_req, const int32_t* c
     e.ldo = d;
     TXS_CK(gemm(m, A, d, W.Wt_os, e, tmp, s, KC_GEMM_OPROJ));
     // multi-query cross-attention against the shared cache (Sec. 4.1.2)
+    const T* Kc = kv + (size_t(2 * l) * c.cap_total) * dkv;
+    const T* Vc = kv + (size_t(2 * l + 1) * c.cap_total) * dkv;
+    const float* Kg = c.gkv + size_t(2 * l) * n_req * dkv;
+    const float* Vg = c.gkv + size_t(2 * l + 1) * n_req * dkv;
+    if (lg_fused) {
+      // LOCAL_GLOBAL, bf16: the query projection's epilogue attends to each
+      // row's window and anchor and writes the attention output (the query
+      // never goes to memory).  It reads the cache, so a caller that is still
+      // writing the cache on another stream is waited for here.
+      if (l == 0 && c.ready) TXS_CK(cudaStreamWaitEvent(s, c.ready, 0));
+      e = epi_base(EPI_ATTN_LG, N, d, d);
+      e.bias = W.b_q;
+      e.out = A;
+      e.ldo = d;
+      e.att_k = Kc;
+      e.att_v = Vc;
+      e.att_kg = Kg;
+      e.att_vg = Vg;
+      e.att_row_req = row_req;
+      e.att_kv_off = c.off;
+      e.att_kv_len = c.len;
+      e.att_dkv = dkv;
+      e.att_group = H / Hkv;
+      e.att_dh = d / H;
+      e.att_l_local = cf.l_local;
+      e.att_scale_log2 = 1.4426950408889634f / sqrtf(static_cast<float>(d / H));
+      e.att_n_cand = static_cast<int>(n_cand);
+      e.att_q_ctx = QKV;   // free here: the serving attention has read it
+      TXS_CK(gemm(m, X1, d, W.Wt_q, e, tmp, s, KC_GEMM_Q_ATTN));
+      // the context-token rows (S per request, rows n_cand + r S + j): q from
+      // QKV, attention output over their rows of A
+      if (S > 0) {
+        const cudaError_t err = launch_ctx_attn_lg(
+            reinterpret_cast<const __nv_bfloat16*>(QKV), reinterpret_cast<__nv_bfloat16*>(A),
+            reinterpret_cast<const __nv_bfloat16*>(Kc), reinterpret_cast<const __nv_bfloat16*>(Vc), n_req,
+            static_cast<int>(n_cand), S, c.off, c.len, Kg, Vg, cf.l_local, H, Hkv, d, s);
+        if (err != cudaSuccess) return fail_cuda("context-row cross-attention", err);
+      }
+    } else {
     e = epi_base(EPI_BIAS, N, d, d);
     e.bias = W.b_q;
     e.out = QKV;
@@ -509,10 +553,6 @@ txs_status score_impl(txs_model* m, const KvView& c, int n_req, const int32_t* c
     // the first read of the cache: a caller that is still writing it on
     // another stream made everything above overlap with that write
     if (l == 0 && c.ready) TXS_CK(cudaStreamWaitEvent(s, c.ready, 0));
-    const T* Kc = kv + (size_t(2 * l) * c.cap_total) * dkv;
-    const T* Vc = kv + (size_t(2 * l + 1) * c.cap_total) * dkv;
-    const float* Kg = c.gkv + size_t(2 * l) * n_req * dkv;
-    const float* Vg = c.gkv + size_t(2 * l + 1) * n_req * dkv;
     cudaError_t lg = cudaErrorNotSupported;
     if (cf.attn_mode == TXS_ATTN_LOCAL_GLOBAL)
       lg = launch_cross_attn_lg<T>(QKV, A, Kc, Vc, cand_off_dev, cand_off, n_req, static_cast<int>(n_cand), S,
@@ -530,6 +570,7 @@ txs_status score_impl(txs_model* m, const KvView& c, int n_req, const int32_t* c
     } else {
       TXS_CK(launch_cross_attn<T>(QKV, A, Kc, Vc, row_req, static_cast<int>(N), c.off, c.len, Kg, Vg,
                                   cf.l_local, cf.attn_mode, H, Hkv, d, s));
+    }
     }
     e = epi_base(EPI_LN, N, d, d);
     e.bias = W.b_oc;
@@ -1231,7 +1272,8 @@ TXS_API txs_status txs_profile_collect(double* total_ms, int64_t* launches, int3
 TXS_API const char* txs_kernel_class_name(int32_t cls) {
   static const char* names[] = {"pack", "gemm_qkv", "attn_serving", "gemm_oproj_ln", "gemm_q", "attn_cross",
                                 "gemm_ffn1_gelu", "gemm_ffn2_ln", "gemm_kv_build", "pool", "global_kv", "rank",
-                                "misc", "row_ln", "cand_mlp", "enc_embed", "enc_gemm", "enc_attn", "head_dw"};
+                                "misc", "row_ln", "cand_mlp", "enc_embed", "enc_gemm", "enc_attn", "head_dw",
+                                "gemm_q_attn_lg"};
   if (cls < 0 || cls >= KC_COUNT_) return "";
   return names[cls];
 }

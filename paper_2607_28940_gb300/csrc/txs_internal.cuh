@@ -20,7 +20,7 @@ constexpr long long kSpinCycles = 2000000000LL;
 enum KernelClass : int {
   KC_PACK = 0, KC_GEMM_QKV, KC_ATTN_SERVING, KC_GEMM_OPROJ, KC_GEMM_Q, KC_ATTN_CROSS,
   KC_GEMM_FFN1, KC_GEMM_FFN2, KC_GEMM_KV, KC_POOL, KC_GLOBAL_KV, KC_RANK, KC_MISC,
-  KC_ROW_LN, KC_CAND_MLP, KC_ENC_EMBED, KC_ENC_GEMM, KC_ENC_ATTN, KC_HEAD_DW, KC_COUNT_
+  KC_ROW_LN, KC_CAND_MLP, KC_ENC_EMBED, KC_ENC_GEMM, KC_ENC_ATTN, KC_HEAD_DW, KC_GEMM_Q_ATTN, KC_COUNT_
 };
 static_assert(KC_COUNT_ <= TXS_N_KERNEL_CLASSES, "profiler classes");
 
@@ -187,6 +187,7 @@ enum Epi : int {
   EPI_KV = 2,         // out = acc + bias, rows remapped into the cache, cols into [l][K|V]
   EPI_LN = 3,         // out = LN(acc + bias + res) over the full row (N == d)
   EPI_LN_HEAD = 4,    // z = LN(...); logits = z Weff_z + xlog; probs = softmax(logits)
+  EPI_ATTN_LG = 5,    // q = acc + bias; out = LOCAL_GLOBAL cross-attention of q (tensor cores, bf16)
 };
 
 // Arguments of every GEMM epilogue; unused fields are ignored.
@@ -226,6 +227,27 @@ struct EpiArgs {
   const int* kv_host_len;
   int* kv_dev_up;
   int* kv_dev_len;
+  // EPI_ATTN_LG: the accumulator row is a query q = acc + bias of packed row
+  // `row` (request att_row_req[row]); the epilogue writes, per head, the
+  // softmax-weighted values of that request's last att_l_local cached rows
+  // (att_k / att_v: the layer's cache, [cap_total][att_dkv] bf16, request r
+  // at row att_kv_off[r], att_kv_len[r] rows) and of its anchor
+  // (att_kg / att_vg [R][att_dkv] fp32); query head h reads K/V head
+  // h / att_group.
+  const void* att_k;
+  const void* att_v;
+  const float* att_kg;
+  const float* att_vg;
+  const int* att_row_req;
+  const int* att_kv_off;
+  const int* att_kv_len;
+  int att_dkv, att_group, att_dh, att_l_local;
+  float att_scale_log2;   // log2(e) / sqrt(d_h)
+  // rows at or past att_n_cand (the context tokens, several requests per
+  // warp) are not attended here: their q (bf16) goes to att_q_ctx at the
+  // same row and column, for a separate launch over those rows
+  int att_n_cand;
+  void* att_q_ctx;
 };
 // Largest request count whose offsets an EPI_KV launch carries by value.
 constexpr int kKvParamReq = 1000;
@@ -252,6 +274,13 @@ cudaError_t launch_cross_attn_lg(const T* q, T* out, const T* Kc, const T* Vc, c
                                  const int* cand_off_host, int n_req, int n_cand, int S, const int* kv_off,
                                  const int* kv_len, const float* Kg, const float* Vg, int l_local, int H, int Hkv,
                                  int d, cudaStream_t s);
+// LOCAL_GLOBAL cross-attention of the context-token rows only (rows n_cand +
+// r S + j), one warp per (row, head), for the fused query projection that
+// leaves those rows' q in `q` (row stride d).
+cudaError_t launch_ctx_attn_lg(const __nv_bfloat16* q, __nv_bfloat16* out, const __nv_bfloat16* Kc,
+                               const __nv_bfloat16* Vc, int n_req, int n_cand, int S, const int* kv_off,
+                               const int* kv_len, const float* Kg, const float* Vg, int l_local, int H, int Hkv,
+                               int d, cudaStream_t s);
 template <typename T>
 cudaError_t launch_cross_attn(const T* q, T* out, const T* Kc, const T* Vc, const int* row_req, int n_rows,
                               const int* kv_off, const int* kv_len, const float* Kg, const float* Vg, int l_local,
