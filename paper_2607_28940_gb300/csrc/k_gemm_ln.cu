@@ -8,11 +8,14 @@
 // double buffer, persistent over the cluster's row tiles) and the row
 // statistics are combined across the cluster through distributed shared
 // memory: every epilogue warp publishes the mean and the sum of squared
-// deviations of its 64 columns to all CTAs of the cluster, and each row merges
-// the 2 CS partial results (pairwise-update formula for equal counts).  With
-// the head, each CTA's partial logits z . W_eff_z go to rank 0, which adds the
-// x part, applies the softmax and writes logits and probabilities
-// (Sec. 4.1.3 action-decoding equation).
+// deviations of its 128 columns to all CTAs of the cluster, and each row
+// merges the CS partial results (pairwise-update formula for equal counts).
+// The epilogue warps form two groups that take alternate tiles (group g the
+// tiles of TMEM buffer g), so one tile's normalisation runs while the other
+// group waits for its cluster's statistics.  With the head, each CTA's
+// partial logits z . W_eff_z go to rank 0, which adds the x part, applies the
+// softmax and writes logits and probabilities (Sec. 4.1.3 action-decoding
+// equation).
 #include "tc_ptx.cuh"
 
 namespace txs {
@@ -21,20 +24,22 @@ namespace tcln {
 using namespace tc;
 
 constexpr int BN = 128;                 // columns per CTA
-constexpr int kWarps = 8;               // epilogue warps: two per TMEM lane quarter
+constexpr int kWarps = 8;               // epilogue warps: two groups of one per TMEM lane quarter
+constexpr int kGroupWarps = kWarps / 2;
 constexpr int NUM_THREADS = 64 + 32 * kWarps;
 
 template <int CS, bool HEAD>
 struct LnShape {
   static constexpr int NAP = 4;                                    // head actions padded to 4
-  static constexpr int P = 2 * CS;                                 // partials per row
+  static constexpr int P = CS;                                     // partials per row (one per CTA)
   static constexpr int B_STAGE_BYTES = BN * BK * 2;                // 16 KB
   static constexpr int STAGE_BYTES = A_STAGE_BYTES + B_STAGE_BYTES;
   static constexpr int STG_BYTES = HEAD ? 0 : kWarps * 2 * 2048;   // bulk-store staging
   static constexpr int XBUF_BYTES = 2 * P * 128 * 8;               // (mean, M2), two parities
   static constexpr int HBUF_BYTES = HEAD ? 2 * P * 128 * NAP * 4 : 0;
   static constexpr int WEFF_BYTES = HEAD ? BN * NAP * 4 : 0;
-  static constexpr int EXTRA = STG_BYTES + XBUF_BYTES + HBUF_BYTES + WEFF_BYTES + 1024 + 512;
+  static constexpr int PAR_BYTES = 3 * BN * 4;                      // bias, gamma, beta of the slice
+  static constexpr int EXTRA = STG_BYTES + XBUF_BYTES + HBUF_BYTES + WEFF_BYTES + PAR_BYTES + 1024 + 512;
   static constexpr int STAGES_FIT = (227 * 1024 - EXTRA) / STAGE_BYTES;
   static constexpr int STAGES = STAGES_FIT > 6 ? 6 : STAGES_FIT;
   static constexpr int SMEM_BYTES = STAGES * STAGE_BYTES + EXTRA;
@@ -56,7 +61,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   float2* xbuf = reinterpret_cast<float2*>(s_stage + S::STG_BYTES);                 // [2][P][128]
   float* hbuf = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(xbuf) + S::XBUF_BYTES);  // [2][P][128][NAP]
   float* s_weff = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(hbuf) + S::HBUF_BYTES);
-  uint64_t* full = reinterpret_cast<uint64_t*>(reinterpret_cast<uint8_t*>(s_weff) + S::WEFF_BYTES);
+  float* s_par = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(s_weff) + S::WEFF_BYTES);   // [3][BN]
+  uint64_t* full = reinterpret_cast<uint64_t*>(reinterpret_cast<uint8_t*>(s_par) + S::PAR_BYTES);
   uint64_t* empty = full + S::STAGES;
   uint64_t* acc_full = empty + S::STAGES;
   uint64_t* acc_empty = acc_full + 2;
@@ -80,7 +86,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(acc_full + b, 1);
-      mbar_init(acc_empty + b, kWarps);
+      mbar_init(acc_empty + b, kGroupWarps);
     }
     for (int i = 0; i < 8; ++i) {
       mbar_init(xfull + i, P * 32);
@@ -112,8 +118,13 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       const int c = i / NAP, a = i - c * NAP;
       s_weff[i] = a < e.n_act ? e.weff_z[static_cast<long long>(n0 + c) * e.n_act + a] : 0.f;
     }
-    __syncthreads();
   }
+  for (int i = threadIdx.x; i < BN; i += NUM_THREADS) {
+    s_par[i] = e.bias[n0 + i];
+    s_par[BN + i] = e.gamma[n0 + i];
+    s_par[2 * BN + i] = e.beta[n0 + i];
+  }
+  __syncthreads();
 
   if (warp == 0) {
     if (lane == 0) {
@@ -170,72 +181,80 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     }
   } else {
     const int ew = warp - 2;
+    const int grp = ew / kGroupWarps;  // tiles i with i % 2 == grp, TMEM buffer grp
     const int q = warp & 3;            // TMEM lane quarter
-    const int h = ew / 4;              // 64-column half of this CTA's slice
-    const int c0 = h * 64;
-    const int slot = static_cast<int>(rk) * 2 + h;
     const int trow = q * 32 + lane;
     uint8_t* stage = s_stage + ew * 4096;
+    const float* s_bias = s_par;
+    const float* s_gamma = s_par + BN;
+    const float* s_beta = s_par + 2 * BN;
     int kchunk = 0;
     float v[32];
-    for (int i = 0; i < my_tiles; ++i) {
-      const int buf = i & 1, pb = i & 1;
+    for (int i = grp; i < my_tiles; i += 2) {
+      const int buf = grp, pb = grp;
       const uint32_t use = static_cast<uint32_t>(i >> 1) & 1;
       const int m0 = (cid + i * ncl) * BM;
       const int row = m0 + trow;
       const bool valid = row < e.M;
-      // the residual row does not depend on the product: fetch it before
-      // waiting for the accumulator, so its DRAM latency overlaps the MMAs
+      // the residual does not depend on the product: its first 64 columns are
+      // fetched before waiting for the accumulator, the rest one chunk ahead
+      const uint4* rp = reinterpret_cast<const uint4*>(static_cast<const __nv_bfloat16*>(e.res) +
+                                                       (valid ? row : 0) * e.ldr + n0);
       uint4 rres[8];
-      {
-        const uint4* rp = reinterpret_cast<const uint4*>(static_cast<const __nv_bfloat16*>(e.res) +
-                                                         (valid ? row : 0) * e.ldr + n0 + c0);
 #pragma unroll
-        for (int k = 0; k < 8; ++k) rres[k] = valid ? __ldg(rp + k) : make_uint4(0, 0, 0, 0);
-      }
+      for (int k = 0; k < 8; ++k) rres[k] = valid ? __ldg(rp + k) : make_uint4(0, 0, 0, 0);
       bool go = mbar_wait(acc_full + buf, use, abort_flag);
       go = __shfl_sync(0xffffffffu, go ? 1 : 0, 0) != 0;
       if (!go) break;
       tc_fence_after();
-      const uint32_t tacc = tmem + buf * BN + (static_cast<uint32_t>(q * 32) << 16) + c0;
-      // pass 1: v = acc + bias + residual, written back to TMEM
-      float sum = 0.f;
+      const uint32_t tacc = tmem + buf * BN + (static_cast<uint32_t>(q * 32) << 16);
+      // pass 1: v = acc + bias + residual, written back to TMEM; per chunk of
+      // 32 columns its mean and squared deviations, merged over the chunks
+      // (pairwise update; equal chunk sizes)
+      float mean_p = 0.f, m2 = 0.f;
 #pragma unroll
-      for (int c = 0; c < 64; c += 32) {
+      for (int c = 0; c < BN; c += 32) {
         tmem_ld32(tacc + c, v);
-        float b[32], r[32];
-        load_f32x32(e.bias + n0 + c0 + c, b);
+        const int rb = (c / 8) & 7;            // residual registers of this chunk
+        float sum = 0.f;
 #pragma unroll
         for (int k = 0; k < 4; ++k) {
-          const __nv_bfloat162* h2 = reinterpret_cast<const __nv_bfloat162*>(&rres[c / 8 + k]);
+          const __nv_bfloat162* h2 = reinterpret_cast<const __nv_bfloat162*>(&rres[rb + k]);
 #pragma unroll
           for (int t = 0; t < 4; ++t) {
             const float2 f = __bfloat1622float2(h2[t]);
-            r[8 * k + 2 * t] = f.x;
-            r[8 * k + 2 * t + 1] = f.y;
+            const int j = 8 * k + 2 * t;
+            v[j] += s_bias[c + j] + f.x;
+            v[j + 1] += s_bias[c + j + 1] + f.y;
+            sum += v[j] + v[j + 1];
           }
         }
+        if (c + 64 < BN) {                     // this chunk's registers now hold chunk c + 64
+#pragma unroll
+          for (int k = 0; k < 4; ++k) rres[rb + k] = valid ? __ldg(rp + (c + 64) / 8 + k) : make_uint4(0, 0, 0, 0);
+        }
+        const float mc = sum * (1.f / 32.f);
+        float m2c = 0.f;
 #pragma unroll
         for (int k = 0; k < 32; ++k) {
-          v[k] += b[k] + r[k];
-          sum += v[k];
+          const float t = v[k] - mc;
+          m2c = fmaf(t, t, m2c);
         }
         tmem_st32(tacc + c, v);
-      }
-      const float mean_p = sum * (1.f / 64.f);
-      float m2 = 0.f;
-#pragma unroll
-      for (int c = 0; c < 64; c += 32) {
-        tmem_ld32(tacc + c, v);
-#pragma unroll
-        for (int k = 0; k < 32; ++k) {
-          const float t = v[k] - mean_p;
-          m2 = fmaf(t, t, m2);
+        if (c == 0) {
+          mean_p = mc;
+          m2 = m2c;
+        } else {
+          // merge n_a = c columns (mean_p, m2) with 32 (mc, m2c)
+          const float na = static_cast<float>(c), nt = na + 32.f;
+          const float dlt = mc - mean_p;
+          mean_p = fmaf(dlt, 32.f / nt, mean_p);
+          m2 = m2 + m2c + dlt * dlt * (na * 32.f / nt);
         }
       }
-      // publish (mean, M2) of these 64 columns to every CTA of the cluster
+      // publish (mean, M2) of these 128 columns to every CTA of the cluster
       {
-        float2* mine = xbuf + (pb * P + slot) * 128 + trow;
+        float2* mine = xbuf + (pb * P + static_cast<int>(rk)) * 128 + trow;
 #pragma unroll
         for (int pr = 0; pr < CS; ++pr) {
           st_peer_f32x2(map_peer(mine, pr), mean_p, m2);
@@ -258,26 +277,23 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
 #pragma unroll
       for (int p = 0; p < P; ++p) {
         const float t = mp[p] - mean;
-        m2 = fmaf(64.f * t, t, m2);
+        m2 = fmaf(static_cast<float>(BN) * t, t, m2);
       }
       const float rstd = rsqrtf(m2 / static_cast<float>(BN * CS) + e.ln_eps);
-      // pass 3: normalise; store, or the head's partial logits
+      // pass 2: normalise; store, or the head's partial logits
       float lg[NAP];
 #pragma unroll
       for (int a = 0; a < NAP; ++a) lg[a] = 0.f;
 #pragma unroll
-      for (int c = 0; c < 64; c += 32) {
+      for (int c = 0; c < BN; c += 32) {
         tmem_ld32(tacc + c, v);
-        float g[32], bt[32];
-        load_f32x32(e.gamma + n0 + c0 + c, g);
-        load_f32x32(e.beta + n0 + c0 + c, bt);
 #pragma unroll
-        for (int k = 0; k < 32; ++k) v[k] = (v[k] - mean) * rstd * g[k] + bt[k];
+        for (int k = 0; k < 32; ++k) v[k] = (v[k] - mean) * rstd * s_gamma[c + k] + s_beta[c + k];
         if constexpr (!HEAD) {
-          __nv_bfloat16* out = valid ? static_cast<__nv_bfloat16*>(e.out) + row * e.ldo + n0 + c0 + c : nullptr;
-          store_chunk(v, out, valid, true, &tmO, n0 + c0 + c, m0 + q * 32, stage, kchunk++, lane);
+          __nv_bfloat16* out = valid ? static_cast<__nv_bfloat16*>(e.out) + row * e.ldo + n0 + c : nullptr;
+          store_chunk(v, out, valid, true, &tmO, n0 + c, m0 + q * 32, stage, kchunk++, lane);
         } else {
-          const float4* w4 = reinterpret_cast<const float4*>(s_weff + (c0 + c) * NAP);
+          const float4* w4 = reinterpret_cast<const float4*>(s_weff + c * NAP);
 #pragma unroll
           for (int k = 0; k < 32; ++k) {
             const float4 w = w4[k];
@@ -288,12 +304,16 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           }
         }
       }
+      // every read of this accumulator is done
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(acc_empty + buf);
       if constexpr (HEAD) {
-        // partial logits of these 64 columns -> rank 0
-        float* mine = hbuf + ((pb * P + slot) * 128 + trow) * NAP;
+        // partial logits of these 128 columns -> rank 0
+        float* mine = hbuf + ((pb * P + static_cast<int>(rk)) * 128 + trow) * NAP;
         st_peer_f32x4(map_peer(mine, 0), lg[0], lg[1], lg[2], lg[3]);
         mbar_arrive_peer(map_peer(hfull + pb * 4 + q, 0));
-        if (rk == 0 && h == 0) {
+        if (rk == 0) {
           ok = mbar_wait_cluster(hfull + pb * 4 + q, use, abort_flag);
           ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
           if (!ok) break;
@@ -330,9 +350,6 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           }
         }
       }
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(acc_empty + buf);
     }
     if (lane == 0) bulk_wait_all();
   }
