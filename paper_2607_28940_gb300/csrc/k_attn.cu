@@ -433,6 +433,8 @@ struct CtxAttnArgs {
   float scale_log2;
 };
 
+constexpr int kCtxKeys = 16;   // window rows (at most 15) + anchor
+
 template <int DH>
 __global__ void __launch_bounds__(256) ctx_attn_kernel(const __nv_bfloat16* __restrict__ q,
                                                        __nv_bfloat16* __restrict__ out,
@@ -451,22 +453,39 @@ __global__ void __launch_bounds__(256) ctx_attn_kernel(const __nv_bfloat16* __re
   const int lo = len > a.l_local ? len - a.l_local : 0;
   const int W = len - lo;
   const long long base = static_cast<long long>(__ldg(a.kv_off + r)) + lo;
-  // this lane's key: window row `lane` or (lane W) the anchor
+  // every load up front (one round of latency): q (all lanes), this lane's
+  // key (window row `lane`, or the anchor for lane W), and this lane's value
+  // columns (lane, lane + 32) of every key
+  float qv[DH], kv[DH];
+  float v0[kCtxKeys], v1[kCtxKeys];
+#pragma unroll
+  for (int c = 0; c < DH; c += 8) Vec16<__nv_bfloat16>::load(q + row * a.d + h * DH + c, qv + c);
+  if (lane < W) {
+#pragma unroll
+    for (int c = 0; c < DH; c += 8) Vec16<__nv_bfloat16>::load(Kc + (base + lane) * a.dkv + kcol + c, kv + c);
+  } else {
+    const float* kg = a.Kg + static_cast<long long>(r) * a.dkv + kcol;
+#pragma unroll
+    for (int c = 0; c < DH; c += 4) {
+      const float4 g4 = __ldg(reinterpret_cast<const float4*>(kg + c));
+      kv[c] = g4.x; kv[c + 1] = g4.y; kv[c + 2] = g4.z; kv[c + 3] = g4.w;
+    }
+  }
+  const float* vg = a.Vg + static_cast<long long>(r) * a.dkv + kcol;
+#pragma unroll
+  for (int t = 0; t < kCtxKeys; ++t) {
+    v0[t] = v1[t] = 0.f;
+    if (t < W) {
+      const __nv_bfloat16* vr = Vc + (base + t) * a.dkv + kcol;
+      v0[t] = __bfloat162float(vr[lane]);
+      if (DH == 64) v1[t] = __bfloat162float(vr[lane + 32]);
+    } else if (t == W) {
+      v0[t] = __ldg(vg + lane);
+      if (DH == 64) v1[t] = __ldg(vg + lane + 32);
+    }
+  }
   float s = -INFINITY;
   if (lane <= W) {
-    float qv[DH], kv[DH];
-#pragma unroll
-    for (int c = 0; c < DH; c += 8) Vec16<__nv_bfloat16>::load(q + row * a.d + h * DH + c, qv + c);
-    if (lane < W) {
-#pragma unroll
-      for (int c = 0; c < DH; c += 8) Vec16<__nv_bfloat16>::load(Kc + (base + lane) * a.dkv + kcol + c, kv + c);
-    } else {
-#pragma unroll
-      for (int c = 0; c < DH; c += 4) {
-        const float4 g4 = __ldg(reinterpret_cast<const float4*>(a.Kg + static_cast<long long>(r) * a.dkv + kcol + c));
-        kv[c] = g4.x; kv[c + 1] = g4.y; kv[c + 2] = g4.z; kv[c + 3] = g4.w;
-      }
-    }
     float acc[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
     for (int c = 0; c < DH; ++c) acc[c & 3] = fmaf(qv[c], kv[c], acc[c & 3]);
@@ -481,17 +500,11 @@ __global__ void __launch_bounds__(256) ctx_attn_kernel(const __nv_bfloat16* __re
   for (int o = 16; o > 0; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
   // output columns lane, lane + 32 (DH = 64) of this head
   float o0 = 0.f, o1 = 0.f;
-  for (int t = 0; t <= W; ++t) {
-    const float pt = __shfl_sync(0xffffffffu, p, t);
-    if (t < W) {
-      const __nv_bfloat16* vr = Vc + (base + t) * a.dkv + kcol;
-      o0 = fmaf(pt, __bfloat162float(vr[lane]), o0);
-      if (DH == 64) o1 = fmaf(pt, __bfloat162float(vr[lane + 32]), o1);
-    } else {
-      const float* vg = a.Vg + static_cast<long long>(r) * a.dkv + kcol;
-      o0 = fmaf(pt, __ldg(vg + lane), o0);
-      if (DH == 64) o1 = fmaf(pt, __ldg(vg + lane + 32), o1);
-    }
+#pragma unroll
+  for (int t = 0; t < kCtxKeys; ++t) {
+    const float pt = __shfl_sync(0xffffffffu, p, t);   // 0 past the anchor
+    o0 = fmaf(pt, v0[t], o0);
+    if (DH == 64) o1 = fmaf(pt, v1[t], o1);
   }
   const float inv = 1.f / sum;
   __nv_bfloat16* dst = out + row * a.d + h * DH;
@@ -504,7 +517,7 @@ cudaError_t launch_ctx_attn_lg(const __nv_bfloat16* q, __nv_bfloat16* out, const
                                const int* kv_len, const float* Kg, const float* Vg, int l_local, int H, int Hkv,
                                int d, cudaStream_t s) {
   const int dh = d / H;
-  if ((dh != 32 && dh != 64) || l_local > 31 || Hkv < 1 || H % Hkv) return cudaErrorInvalidValue;
+  if ((dh != 32 && dh != 64) || l_local >= kCtxKeys || Hkv < 1 || H % Hkv) return cudaErrorInvalidValue;
   const long long warps = static_cast<long long>(n_req) * S * H;
   if (warps == 0) return cudaSuccess;
   CtxAttnArgs a{n_req, n_cand, S, H, d, Hkv * dh, H / Hkv, l_local, kv_off, kv_len, Kg, Vg,

@@ -264,18 +264,14 @@ __global__ void __launch_bounds__(256) pool_partial_kernel(const T* __restrict__
   }
 }
 
-// Anchor projections of every layer: gkv[blk][r][c] = g[r] . Wt[n] + b[n] with
-// n = blk * d + c, blk = 2 l + {0: K, 1: V}.  One warp per (column n, group of
-// 8 requests): the weight row is read once per warp (coalesced), the 8 dot
-// products are reduced with shuffles.
 constexpr int kAnchorReq = 16;        // anchors staged per CTA (grid.y covers the rest)
-constexpr int kAnchorRowsPerWarp = 1;  // weight rows per warp
+constexpr int kAnchorRowsPerWarp = 4;  // weight rows per warp (each staged anchor value read once for all four)
 
 // Anchor projections gkv[blk][r][c] = g_r . Wt[n] + b[n] for the 2 nL dkv
 // rows n of the transposed K/V weights (n = blk dkv + c).  One CTA per
-// (32 weight rows, 16 requests): the 16 fp32 anchors are staged in shared
-// memory once, each warp reads its weight row once (16-byte vectors) and
-// dots it with all 16 anchors.
+// (8 kAnchorRowsPerWarp weight rows, 16 requests): the 16 fp32 anchors are
+// staged in shared memory once, each warp reads its weight rows once
+// (16-byte vectors) and dots them with all 16 anchors.
 template <typename T, int NCH>
 __global__ void __launch_bounds__(256) anchor_proj_kernel(const float* __restrict__ g, const T* __restrict__ Wt,
                                                           const float* __restrict__ b, float* __restrict__ gkv,
@@ -316,41 +312,49 @@ __global__ void __launch_bounds__(256) anchor_proj_kernel(const float* __restric
     if (i * 4 < nr * d) reinterpret_cast<float4*>(sg)[i] = st[u];
   }
   __syncthreads();
+  // dot[k][t] = Wt[nw0 + k] . g[r0 + t]: each anchor value from shared
+  // memory serves the warp's kAnchorRowsPerWarp weight rows
+  float dot[kAnchorRowsPerWarp][kAnchorReq];
 #pragma unroll
-  for (int k = 0; k < kAnchorRowsPerWarp; ++k) {
-    const int n = nw0 + k;
-    if (n >= n_total) break;
-    float dot[kAnchorReq];
+  for (int k = 0; k < kAnchorRowsPerWarp; ++k)
 #pragma unroll
-    for (int t = 0; t < kAnchorReq; ++t) {
-      dot[t] = 0.f;
-      if (t < nr) {
+    for (int t = 0; t < kAnchorReq; ++t) dot[k][t] = 0.f;
 #pragma unroll
-        for (int j = 0; j < NCH; ++j) {
-          const int col = (j * 32 + lane) * VEC;
-          if (col < d) {
-            const float4* gp = reinterpret_cast<const float4*>(sg + t * d + col);
+  for (int t = 0; t < kAnchorReq; ++t) {
+    if (t < nr) {
 #pragma unroll
-            for (int q4 = 0; q4 < VEC / 4; ++q4) {
-              const float4 x = gp[q4];
-              dot[t] = fmaf(w[k][j][4 * q4], x.x, dot[t]);
-              dot[t] = fmaf(w[k][j][4 * q4 + 1], x.y, dot[t]);
-              dot[t] = fmaf(w[k][j][4 * q4 + 2], x.z, dot[t]);
-              dot[t] = fmaf(w[k][j][4 * q4 + 3], x.w, dot[t]);
+      for (int j = 0; j < NCH; ++j) {
+        const int col = (j * 32 + lane) * VEC;
+        if (col < d) {
+          const float4* gp = reinterpret_cast<const float4*>(sg + t * d + col);
+#pragma unroll
+          for (int q4 = 0; q4 < VEC / 4; ++q4) {
+            const float4 x = gp[q4];
+#pragma unroll
+            for (int k = 0; k < kAnchorRowsPerWarp; ++k) {
+              dot[k][t] = fmaf(w[k][j][4 * q4], x.x, dot[k][t]);
+              dot[k][t] = fmaf(w[k][j][4 * q4 + 1], x.y, dot[k][t]);
+              dot[k][t] = fmaf(w[k][j][4 * q4 + 2], x.z, dot[k][t]);
+              dot[k][t] = fmaf(w[k][j][4 * q4 + 3], x.w, dot[k][t]);
             }
           }
         }
       }
     }
+  }
+#pragma unroll
+  for (int k = 0; k < kAnchorRowsPerWarp; ++k) {
+    const int n = nw0 + k;
+    if (n >= n_total) break;
 #pragma unroll
     for (int t = 0; t < kAnchorReq; ++t)
 #pragma unroll
-      for (int o = 16; o > 0; o >>= 1) dot[t] += __shfl_xor_sync(0xffffffffu, dot[t], o);
+      for (int o = 16; o > 0; o >>= 1) dot[k][t] += __shfl_xor_sync(0xffffffffu, dot[k][t], o);
     if (lane < nr) {
       float v = 0.f;
 #pragma unroll
       for (int t = 0; t < kAnchorReq; ++t)
-        if (t == lane) v = dot[t];
+        if (t == lane) v = dot[k][t];
       const int blk = n / dkv, c = n - blk * dkv;
       gkv[(static_cast<long long>(blk) * R + r0 + lane) * dkv + c] = v + __ldg(b + n);
     }

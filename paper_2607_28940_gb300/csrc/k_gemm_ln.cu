@@ -28,10 +28,10 @@ constexpr int kWarps = 8;               // epilogue warps: two groups of one per
 constexpr int kGroupWarps = kWarps / 2;
 constexpr int NUM_THREADS = 64 + 32 * kWarps;
 
-template <int CS, bool HEAD>
+template <int CS, bool HEAD, bool PING>
 struct LnShape {
   static constexpr int NAP = 4;                                    // head actions padded to 4
-  static constexpr int P = CS;                                     // partials per row (one per CTA)
+  static constexpr int P = PING ? CS : 2 * CS;                     // partials per row (per CTA or half)
   static constexpr int B_STAGE_BYTES = BN * BK * 2;                // 16 KB
   static constexpr int STAGE_BYTES = A_STAGE_BYTES + B_STAGE_BYTES;
   static constexpr int STG_BYTES = HEAD ? 0 : kWarps * 2 * 2048;   // bulk-store staging
@@ -47,11 +47,11 @@ struct LnShape {
   static_assert(STAGES >= 2 && SMEM_BYTES <= 232448, "shared memory");
 };
 
-template <int CS, bool HEAD>
+template <int CS, bool HEAD, bool PING>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
     gemm_ln_cluster_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                            const __grid_constant__ CUtensorMap tmO, const EpiArgs e) {
-  using S = LnShape<CS, HEAD>;
+  using S = LnShape<CS, HEAD, PING>;
   constexpr int NAP = S::NAP, P = S::P;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -86,7 +86,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(acc_full + b, 1);
-      mbar_init(acc_empty + b, kGroupWarps);
+      mbar_init(acc_empty + b, PING ? kGroupWarps : kWarps);
     }
     for (int i = 0; i < 8; ++i) {
       mbar_init(xfull + i, P * 32);
@@ -179,7 +179,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         mma_commit(acc_full + buf);
       }
     }
-  } else {
+  } else if constexpr (PING) {
     const int ew = warp - 2;
     const int grp = ew / kGroupWarps;  // tiles i with i % 2 == grp, TMEM buffer grp
     const int q = warp & 3;            // TMEM lane quarter
@@ -352,6 +352,173 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       }
     }
     if (lane == 0) bulk_wait_all();
+  } else {
+    // few tiles per cluster: all eight warps on each tile, two per lane
+    // quarter, each 64 of the CTA's 128 columns
+    const int ew = warp - 2;
+    const int q = warp & 3;            // TMEM lane quarter
+    const int h = ew / 4;              // 64-column half of this CTA's slice
+    const int c0 = h * 64;
+    const int slot = static_cast<int>(rk) * 2 + h;
+    const int trow = q * 32 + lane;
+    uint8_t* stage = s_stage + ew * 4096;
+    int kchunk = 0;
+    float v[32];
+    for (int i = 0; i < my_tiles; ++i) {
+      const int buf = i & 1, pb = i & 1;
+      const uint32_t use = static_cast<uint32_t>(i >> 1) & 1;
+      const int m0 = (cid + i * ncl) * BM;
+      const int row = m0 + trow;
+      const bool valid = row < e.M;
+      // the residual row does not depend on the product: fetch it before
+      // waiting for the accumulator, so its DRAM latency overlaps the MMAs
+      uint4 rres[8];
+      {
+        const uint4* rp = reinterpret_cast<const uint4*>(static_cast<const __nv_bfloat16*>(e.res) +
+                                                         (valid ? row : 0) * e.ldr + n0 + c0);
+#pragma unroll
+        for (int k = 0; k < 8; ++k) rres[k] = valid ? __ldg(rp + k) : make_uint4(0, 0, 0, 0);
+      }
+      bool go = mbar_wait(acc_full + buf, use, abort_flag);
+      go = __shfl_sync(0xffffffffu, go ? 1 : 0, 0) != 0;
+      if (!go) break;
+      tc_fence_after();
+      const uint32_t tacc = tmem + buf * BN + (static_cast<uint32_t>(q * 32) << 16) + c0;
+      // pass 1: v = acc + bias + residual, written back to TMEM
+      float sum = 0.f;
+#pragma unroll
+      for (int c = 0; c < 64; c += 32) {
+        tmem_ld32(tacc + c, v);
+        float b[32], r[32];
+#pragma unroll
+        for (int k = 0; k < 32; ++k) b[k] = s_par[c0 + c + k];
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+          const __nv_bfloat162* h2 = reinterpret_cast<const __nv_bfloat162*>(&rres[c / 8 + k]);
+#pragma unroll
+          for (int t = 0; t < 4; ++t) {
+            const float2 f = __bfloat1622float2(h2[t]);
+            r[8 * k + 2 * t] = f.x;
+            r[8 * k + 2 * t + 1] = f.y;
+          }
+        }
+#pragma unroll
+        for (int k = 0; k < 32; ++k) {
+          v[k] += b[k] + r[k];
+          sum += v[k];
+        }
+        tmem_st32(tacc + c, v);
+      }
+      const float mean_p = sum * (1.f / 64.f);
+      float m2 = 0.f;
+#pragma unroll
+      for (int c = 0; c < 64; c += 32) {
+        tmem_ld32(tacc + c, v);
+#pragma unroll
+        for (int k = 0; k < 32; ++k) {
+          const float t = v[k] - mean_p;
+          m2 = fmaf(t, t, m2);
+        }
+      }
+      // publish (mean, M2) of these 64 columns to every CTA of the cluster
+      {
+        float2* mine = xbuf + (pb * P + slot) * 128 + trow;
+#pragma unroll
+        for (int pr = 0; pr < CS; ++pr) {
+          st_peer_f32x2(map_peer(mine, pr), mean_p, m2);
+          mbar_arrive_peer(map_peer(xfull + pb * 4 + q, pr));
+        }
+      }
+      bool ok = mbar_wait_cluster(xfull + pb * 4 + q, use, abort_flag);
+      ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
+      if (!ok) break;
+      float mp[P];
+      float mean = 0.f;
+#pragma unroll
+      for (int p = 0; p < P; ++p) {
+        const float2 x = xbuf[(pb * P + p) * 128 + trow];
+        mp[p] = x.x;
+        mean += x.x;
+        m2 = p == 0 ? x.y : m2 + x.y;
+      }
+      mean *= 1.f / P;
+#pragma unroll
+      for (int p = 0; p < P; ++p) {
+        const float t = mp[p] - mean;
+        m2 = fmaf(64.f * t, t, m2);
+      }
+      const float rstd = rsqrtf(m2 / static_cast<float>(BN * CS) + e.ln_eps);
+      // pass 3: normalise; store, or the head's partial logits
+      float lg[NAP];
+#pragma unroll
+      for (int a = 0; a < NAP; ++a) lg[a] = 0.f;
+#pragma unroll
+      for (int c = 0; c < 64; c += 32) {
+        tmem_ld32(tacc + c, v);
+#pragma unroll
+        for (int k = 0; k < 32; ++k) v[k] = (v[k] - mean) * rstd * s_par[BN + c0 + c + k] + s_par[2 * BN + c0 + c + k];
+        if constexpr (!HEAD) {
+          __nv_bfloat16* out = valid ? static_cast<__nv_bfloat16*>(e.out) + row * e.ldo + n0 + c0 + c : nullptr;
+          store_chunk(v, out, valid, true, &tmO, n0 + c0 + c, m0 + q * 32, stage, kchunk++, lane);
+        } else {
+          const float4* w4 = reinterpret_cast<const float4*>(s_weff + (c0 + c) * NAP);
+#pragma unroll
+          for (int k = 0; k < 32; ++k) {
+            const float4 w = w4[k];
+            lg[0] = fmaf(v[k], w.x, lg[0]);
+            lg[1] = fmaf(v[k], w.y, lg[1]);
+            lg[2] = fmaf(v[k], w.z, lg[2]);
+            lg[3] = fmaf(v[k], w.w, lg[3]);
+          }
+        }
+      }
+      if constexpr (HEAD) {
+        // partial logits of these 64 columns -> rank 0
+        float* mine = hbuf + ((pb * P + slot) * 128 + trow) * NAP;
+        st_peer_f32x4(map_peer(mine, 0), lg[0], lg[1], lg[2], lg[3]);
+        mbar_arrive_peer(map_peer(hfull + pb * 4 + q, 0));
+        if (rk == 0 && h == 0) {
+          ok = mbar_wait_cluster(hfull + pb * 4 + q, use, abort_flag);
+          ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
+          if (!ok) break;
+          if (valid && row < e.n_cand_rows) {
+            const int na = e.n_act;
+            float t[NAP];
+#pragma unroll
+            for (int a = 0; a < NAP; ++a) t[a] = 0.f;
+#pragma unroll
+            for (int p = 0; p < P; ++p) {
+              const float4 x = *reinterpret_cast<const float4*>(hbuf + ((pb * P + p) * 128 + trow) * NAP);
+              t[0] += x.x; t[1] += x.y; t[2] += x.z; t[3] += x.w;
+            }
+            float mx = -INFINITY;
+#pragma unroll
+            for (int a = 0; a < NAP; ++a)
+              if (a < na) {
+                t[a] += __ldg(e.xlog + static_cast<long long>(row) * na + a);
+                mx = fmaxf(mx, t[a]);
+              }
+            float ssum = 0.f, pe[NAP];
+#pragma unroll
+            for (int a = 0; a < NAP; ++a) {
+              pe[a] = a < na ? expf(t[a] - mx) : 0.f;
+              ssum += pe[a];
+            }
+            const float inv = 1.f / ssum;
+#pragma unroll
+            for (int a = 0; a < NAP; ++a)
+              if (a < na) {
+                e.logits[static_cast<long long>(row) * na + a] = t[a];
+                if (e.probs) e.probs[static_cast<long long>(row) * na + a] = pe[a] * inv;
+              }
+          }
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(acc_empty + buf);
+    }
+    if (lane == 0) bulk_wait_all();
   }
   tc_fence_before();
   __syncthreads();
@@ -363,11 +530,11 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   if (threadIdx.x == 0 && *abort_flag) latch_status(e.status, TXS_ERR_DEVICE_TIMEOUT);
 }
 
-template <int CS, bool HEAD>
+template <int CS, bool HEAD, bool PING>
 static cudaError_t launch_cs(const __nv_bfloat16* A, long long lda, const __nv_bfloat16* B, const EpiArgs& e,
                              cudaStream_t s, int cls) {
-  using Sh = LnShape<CS, HEAD>;
-  auto kern = gemm_ln_cluster_kernel<CS, HEAD>;
+  using Sh = LnShape<CS, HEAD, PING>;
+  auto kern = gemm_ln_cluster_kernel<CS, HEAD, PING>;
   cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeClusterDimension;
   attr[0].val.clusterDim.x = CS;
@@ -418,9 +585,20 @@ cudaError_t launch_gemm_ln_cluster(const __nv_bfloat16* A, long long lda, const 
   if (e.epi == EPI_LN_HEAD && (e.n_act < 1 || e.n_act > 4)) return cudaErrorNotSupported;
   if (e.epi != EPI_LN && e.epi != EPI_LN_HEAD) return cudaErrorNotSupported;
   const bool head = e.epi == EPI_LN_HEAD;
+  // the two epilogue groups pay off once each cluster has several row tiles
+  const int m_tiles = (e.M + tc::BM - 1) / tc::BM;
+  const bool ping = m_tiles >= 4 * (num_sms() / (e.N / tcln::BN));
   switch (e.N) {
-    case 256: return head ? tcln::launch_cs<2, true>(A, lda, B, e, s, cls) : tcln::launch_cs<2, false>(A, lda, B, e, s, cls);
-    case 512: return head ? tcln::launch_cs<4, true>(A, lda, B, e, s, cls) : tcln::launch_cs<4, false>(A, lda, B, e, s, cls);
+    case 256:
+      if (ping) return head ? tcln::launch_cs<2, true, true>(A, lda, B, e, s, cls)
+                            : tcln::launch_cs<2, false, true>(A, lda, B, e, s, cls);
+      return head ? tcln::launch_cs<2, true, false>(A, lda, B, e, s, cls)
+                  : tcln::launch_cs<2, false, false>(A, lda, B, e, s, cls);
+    case 512:
+      if (ping) return head ? tcln::launch_cs<4, true, true>(A, lda, B, e, s, cls)
+                            : tcln::launch_cs<4, false, true>(A, lda, B, e, s, cls);
+      return head ? tcln::launch_cs<4, true, false>(A, lda, B, e, s, cls)
+                  : tcln::launch_cs<4, false, false>(A, lda, B, e, s, cls);
     default: return cudaErrorNotSupported;
   }
 }

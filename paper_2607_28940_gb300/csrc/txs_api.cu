@@ -482,10 +482,14 @@ txs_status score_impl(txs_model* m, const KvView& c, int n_req, const int32_t* c
   }
   const T* kv = static_cast<const T*>(c.kv);
   // LOCAL_GLOBAL attention fused into the query projection (bf16; heads of
-  // 32 or 64 columns, 128-column query tiles, windows of at most 16 rows)
+  // 32 or 64 columns, 128-column query tiles, windows of at most 15 rows),
+  // when there are at least two 128 x 128 tiles per SM to pipeline; smaller
+  // batches take the separate query projection and window kernel
   const int dh = d / H;
+  const long long q_tiles = (N + 127) / 128 * (d / 128);
   const bool lg_fused = std::is_same<T, __nv_bfloat16>::value && cf.attn_mode == TXS_ATTN_LOCAL_GLOBAL &&
-                        (dh == 32 || dh == 64) && d % 128 == 0 && d <= 512 && cf.l_local <= 16 && dkv % 8 == 0;
+                        (dh == 32 || dh == 64) && d % 128 == 0 && d <= 512 && cf.l_local <= 15 && dkv % 8 == 0 &&
+                        q_tiles >= 2LL * tc::num_sms();
   for (int l = 0; l < cf.n_layers; ++l) {
     const LayerW& W = m->layers[l];
     // serving-stream attention (App. B mask), O-projection + residual + LN1

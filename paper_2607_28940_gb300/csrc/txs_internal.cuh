@@ -263,6 +263,9 @@ cudaError_t launch_gelu_eval(const float* x, float* y, long long n, int variant,
 cudaError_t launch_gemm_tc(const __nv_bfloat16* A, long long lda, const __nv_bfloat16* B,
                            const EpiArgs& e, cudaStream_t s, int cls);
 bool tc_gemm_supported(int N, int K, int epi);
+namespace tc {
+int num_sms();   // streaming multiprocessors of the current device
+}
 
 template <typename T>
 cudaError_t launch_serving_attn(const T* qkv, T* out, const int* row_req, int n_rows, int n_cand_rows, int S, int H,
