@@ -72,7 +72,7 @@ constexpr int kRedStride = 17;                // per-row exchange slots: sum + 1
 // Epilogue of one 128 x BN tile for one warp: TMEM lanes `tlane` (32 rows of
 // the tile), columns [c0, c0 + BN/2) of the accumulator.  The two warps that
 // share a lane quarter exchange row sums (and head logits) through `red`.
-template <int BN, int EPI, int NAP>
+template <int BN, int EPI, int NAP, int SB>
 __device__ __forceinline__ void epilogue(const EpiArgs& e, uint32_t tacc, int row, int n0, int c0, int q, int h,
                                          float* red, const float* s_weff, const float* bias,
                                          const int* seg_off, const int* dst_row0, const CUtensorMap* tmO,
@@ -115,7 +115,7 @@ __device__ __forceinline__ void epilogue(const EpiArgs& e, uint32_t tacc, int ro
       } else {
         if (valid) out = static_cast<__nv_bfloat16*>(e.out) + orow * e.ldo + n;
       }
-      store_chunk(vals, out, valid, tma_ok, tmO, tx, ty, stage, kchunk++, lane);
+      store_chunk<SB>(vals, out, valid, tma_ok, tmO, tx, ty, stage, kchunk++, lane);
     };
     if constexpr (HALF % 64 == 0) {
       // 64 columns per TMEM load (one wait), two bulk-stored chunks
@@ -212,7 +212,7 @@ __device__ __forceinline__ void epilogue(const EpiArgs& e, uint32_t tacc, int ro
 #pragma unroll
       for (int i = 0; i < 32; ++i) v[i] = (v[i] - mean) * rstd * g[i] + bt[i];
       if constexpr (EPI == EPI_LN) {
-        store_chunk(v, out + c, valid, true, tmO, c0 + c, ty, stage, kchunk++, lane);
+        store_chunk<SB>(v, out + c, valid, true, tmO, c0 + c, ty, stage, kchunk++, lane);
       } else {
         // head: z . W_eff_z, weights zero-padded to NAP actions in shared memory
         const float4* w4 = reinterpret_cast<const float4*>(s_weff + (c0 + c) * NAP);
@@ -657,13 +657,18 @@ struct Shape {
   // first rows; rounded to 1 KB so that the staging buffers after it start on
   // a swizzle-atom boundary
   static constexpr bool ATT = EPI == EPI_ATTN_LG;
-  static constexpr int STAGE_N = BRES ? kStageNRes : ATT ? kStageNAtt : kStageN;
+  // 256-column tiles streaming both operands (the K/V build, the QKV and FFN
+  // projections at d = 512): one bulk-store staging buffer per warp and the
+  // bias read through L1 leave room for a fourth operand stage
+  static constexpr bool LEAN = !BRES && !LN && !ATT && BN == 256;
+  static constexpr int SBUF = LEAN ? 1 : 2;               // bulk-store staging buffers per warp
+  static constexpr int STAGE_N = BRES ? kStageNRes : (ATT || LEAN) ? kStageNAtt : kStageN;
   static constexpr int AUX_BYTES =
       LN ? 0 : (((STAGE_N * 4) + (EPI == EPI_KV ? (2 * kStageSeg + 1) * 4 : 0) + 1023) / 1024) * 1024;
   // fused attention: each epilogue warp's staged window and anchor (fp32)
   static constexpr int ATT_BYTES = ATT ? kEpiWarps * kAttWarpBytes : 0;
   // bulk-store staging: two 2 KB buffers per epilogue warp (bf16 outputs)
-  static constexpr int STG_BYTES = EPI == EPI_LN_HEAD ? 0 : kEpiWarps * 2 * 2048;
+  static constexpr int STG_BYTES = EPI == EPI_LN_HEAD ? 0 : kEpiWarps * SBUF * 2048;
   static constexpr int EXTRA = BRES_BYTES + RED_BYTES + WEFF_BYTES + AUX_BYTES + STG_BYTES + ATT_BYTES + 1024 + 256;
   static constexpr int STAGES_FIT = (227 * 1024 - EXTRA) / STAGE_BYTES;
   static constexpr int STAGES = STAGES_FIT > 8 ? 8 : STAGES_FIT;
@@ -936,7 +941,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     const int ew = warp - 2;
     const int q = warp & 3;           // TMEM lane quarter this warp may access
     const int h = ew / 4;             // column half
-    uint8_t* stage = s_stage + ew * 4096;
+    uint8_t* stage = s_stage + ew * S::SBUF * 2048;
     if constexpr (S::ATT) {
       attn_epilogue_warp(e, tmem + (static_cast<uint32_t>(q * 32) << 16), acc_full, acc_empty, abort_flag, t_lo,
                          t_hi, t_step, n_tiles, m_tiles, q, h, bias, &tmO, stage, s_att + ew * kAttWarpBytes);
@@ -955,7 +960,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         if (!go) break;
         tc_fence_after();
         const int m0 = tile_m(t) * BM, n0 = tile_n(t) * BN;
-        epilogue<BN, EPI, NAP>(e, tmem + buf * BN + (static_cast<uint32_t>(q * 32) << 16), m0 + q * 32 + lane, n0,
+        epilogue<BN, EPI, NAP, S::SBUF>(e, tmem + buf * BN + (static_cast<uint32_t>(q * 32) << 16), m0 + q * 32 + lane, n0,
                                h * (BN / 2), q, h, red, s_weff, bias, seg_off, dst_row0, &tmO, stage, kchunk);
         tc_fence_before();
         __syncwarp();

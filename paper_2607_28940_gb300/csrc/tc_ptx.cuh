@@ -231,12 +231,14 @@ __device__ __forceinline__ void store_bf16x32(__nv_bfloat16* p, const float* v) 
 // tensor map) and lane 0 issues one bulk tensor store at (x, y): full 32-byte
 // sectors instead of 32 row-strided 16-byte stores.  Otherwise each valid lane
 // stores its own 64 bytes at `direct`.  `k` counts the warp's chunks so that
-// each of the two staging buffers is reused only after its store has read it.
+// each of the NB (1 or 2) staging buffers is reused only after its store has
+// read it.
+template <int NB = 2>
 __device__ __forceinline__ void store_chunk(const float* v, __nv_bfloat16* direct, bool valid, bool tma_ok,
                                             const CUtensorMap* tmO, int x, int y, uint8_t* stage, int k, int lane) {
   if (tma_ok) {
-    uint8_t* buf = stage + (k & 1) * 2048;
-    if (lane == 0) bulk_wait_read<1>();
+    uint8_t* buf = stage + (NB == 2 ? (k & 1) * 2048 : 0);
+    if (lane == 0) bulk_wait_read<NB - 1>();
     __syncwarp();
 #pragma unroll
     for (int c = 0; c < 4; ++c) {
