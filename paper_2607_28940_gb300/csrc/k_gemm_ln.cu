@@ -10,9 +10,12 @@
 // memory: every epilogue warp publishes the mean and the sum of squared
 // deviations of its 128 columns to all CTAs of the cluster, and each row
 // merges the CS partial results (pairwise-update formula for equal counts).
-// The epilogue warps form two groups that take alternate tiles (group g the
-// tiles of TMEM buffer g), so one tile's normalisation runs while the other
-// group waits for its cluster's statistics.  With the head, each CTA's
+// The CTAs of a cluster read the same activation rows: each loads 1 / CS of
+// every activation stage and multicasts it into the stage of all CTAs (a stage
+// is reloaded once every CTA's MMAs have released it).  The epilogue warps
+// form two groups that take alternate tiles (group g the tiles of TMEM buffer
+// g) when each cluster has several row tiles, so one tile's normalisation
+// runs while the other group waits for its cluster's statistics.  With the head, each CTA's
 // partial logits z . W_eff_z go to rank 0, which adds the x part, applies the
 // softmax and writes logits and probabilities (Sec. 4.1.3 action-decoding
 // equation).
@@ -78,11 +81,12 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   const int my_tiles = m_tiles > cid ? (m_tiles - 1 - cid) / ncl + 1 : 0;   // equal within a cluster
   const int n0 = static_cast<int>(rk) * BN;
   const int num_kb = e.K / BK;
+  constexpr uint16_t kAllCtas = static_cast<uint16_t>((1u << CS) - 1);
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < S::STAGES; ++s) {
       mbar_init(full + s, 1);
-      mbar_init(empty + s, 1);
+      mbar_init(empty + s, CS);          // released by the MMAs of every CTA of the cluster
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(acc_full + b, 1);
@@ -134,18 +138,23 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       bool ok = true;
       for (int i = 0; i < my_tiles && ok; ++i) {
         const int m0 = (cid + i * ncl) * BM;
+        // every CTA of the cluster reads the same activation rows: each loads
+        // BM / CS of them into the stage of all CTAs (multicast)
+        const int a_rows = m0 + static_cast<int>(rk) * (BM / CS);
+        uint8_t* a_dst = sA + static_cast<int>(rk) * (A_STAGE_BYTES / CS);
         for (int kb = 0; kb < num_kb; ++kb, ++it) {
           const int s = it % S::STAGES;
           if (it < n_pre) {     // weights in flight since before the wait
-            tma_load_2d(sA + s * A_STAGE_BYTES, &tmA, full + s, kb * BK, m0);
+            tma_load_2d_mc(a_dst + s * A_STAGE_BYTES, &tmA, full + s, kb * BK, a_rows, kAllCtas);
             continue;
           }
+          // the stage is free in every CTA of the cluster
           if (!mbar_wait(empty + s, ((it / S::STAGES) & 1) ^ 1, abort_flag)) {
             ok = false;
             break;
           }
           mbar_expect_tx(full + s, S::STAGE_BYTES);
-          tma_load_2d(sA + s * A_STAGE_BYTES, &tmA, full + s, kb * BK, m0);
+          tma_load_2d_mc(a_dst + s * A_STAGE_BYTES, &tmA, full + s, kb * BK, a_rows, kAllCtas);
           tma_load_2d(sB + s * S::B_STAGE_BYTES, &tmB, full + s, kb * BK, n0);
         }
       }
@@ -174,7 +183,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
 #pragma unroll
           for (int k = 0; k < BK / 16; ++k)
             mma_bf16(tmem + buf * BN, adesc + 2 * k, bdesc + 2 * k, idesc, (kb > 0 || k > 0) ? 1u : 0u);
-          mma_commit(empty + s);
+          mma_commit_mc(empty + s, kAllCtas);   // this CTA's reads of the stage are done, in every CTA
         }
         mma_commit(acc_full + buf);
       }
@@ -562,7 +571,8 @@ static cudaError_t launch_cs(const __nv_bfloat16* A, long long lda, const __nv_b
     max_clusters = n;
   }
   CUtensorMap ta, tb, to;
-  if (!make_tmap(&ta, A, e.M, e.K, lda, BM)) return cudaErrorInvalidValue;
+  // activation boxes of BM / CS rows: each CTA multicasts its share of a tile
+  if (!make_tmap(&ta, A, e.M, e.K, lda, BM / CS)) return cudaErrorInvalidValue;
   if (!make_tmap(&tb, B, e.N, e.K, e.K, BN)) return cudaErrorInvalidValue;
   if (HEAD) to = ta;   // unused
   else if (!make_tmap_out(&to, e.out, e.M, e.N, e.ldo)) return cudaErrorInvalidValue;
