@@ -45,7 +45,7 @@ def test_static_pooling_matches_cache_build_on_two_calls_in_a_row(dtype):
     else:
         base = W.WORKLOADS["tiny_fp32"]
     weights = W.weights(base)
-    weights["w_pool"] = weights["w_pool"] * 30.0    # uneven pooling weights
+    weights["w_pool"] = weights["w_pool"] * 32.0    # uneven pooling weights (a power of two: still exact in bf16)
     model = txs.Model(base, weights)
     dt = txs.torch_dtype(base.dtype)
     first = W.with_sizes(base, n_req=6, L=[1, 127, 128, 129, 2000, 5000], M=1, seed=101)
