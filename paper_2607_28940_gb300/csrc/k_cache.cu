@@ -10,7 +10,7 @@
 // chunks of kPoolChunk (one CTA each); chunk states are merged per request.
 #include <algorithm>
 
-#include "txs_internal.cuh"
+#include "tc_ptx.cuh"
 
 namespace txs {
 
@@ -21,6 +21,79 @@ namespace {
 
 constexpr int kPoolWarps = 8;
 constexpr int kPoolRowsPerWarp = kPoolChunkV / kPoolWarps;
+
+// The last chunk CTA of request r to finish merges the request's nch_r chunk
+// states part_r[c] = (m, s, acc[d]) (and, for an append, the stored state)
+// into the pooling state and writes g = acc / s.  Called by every thread of
+// a 256-thread CTA once its own chunk state is in part_r.
+__device__ __forceinline__ void pool_merge_if_last(const float* pr, int nch_r, int d, int r, int merge_existing,
+                                                   float* st_m, float* st_s, float* st_acc, float* g, int* counter) {
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  __shared__ int is_last;
+  __threadfence();
+  __syncthreads();
+  if (tid == 0) is_last = atomicAdd(counter + r, 1) == nch_r - 1;
+  __syncthreads();
+  if (!is_last) return;
+  __threadfence();
+  // chunk maxima and weighted sums as block reductions (thread t takes
+  // chunks t, t + 256, ...), then each column's sum over the chunks with its
+  // loads issued ahead of the multiply-adds; the order is fixed, so the
+  // result is deterministic
+  __shared__ float ch_scale[512];
+  __shared__ float red[kPoolWarps];
+  const float old_m = merge_existing ? st_m[r] : -INFINITY;
+  const float old_s = merge_existing ? st_s[r] : 0.f;
+  float mloc = -INFINITY;
+  for (int ch = tid; ch < nch_r; ch += 256) mloc = fmaxf(mloc, __ldcg(pr + static_cast<long long>(ch) * (d + 2)));
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) mloc = fmaxf(mloc, __shfl_xor_sync(0xffffffffu, mloc, o));
+  if (lane == 0) red[warp] = mloc;
+  __syncthreads();
+  float Mr = old_m;
+#pragma unroll
+  for (int w8 = 0; w8 < kPoolWarps; ++w8) Mr = fmaxf(Mr, red[w8]);
+  const float w_old = merge_existing ? expf(old_m - Mr) : 0.f;
+  __syncthreads();                                  // red is reused below
+  float sloc = 0.f;
+  for (int ch = tid; ch < nch_r; ch += 256) {
+    const float* pc = pr + static_cast<long long>(ch) * (d + 2);
+    const float sc = expf(__ldcg(pc) - Mr);
+    if (ch < 512) ch_scale[ch] = sc;
+    sloc = fmaf(__ldcg(pc + 1), sc, sloc);
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) sloc += __shfl_xor_sync(0xffffffffu, sloc, o);
+  if (lane == 0) red[warp] = sloc;
+  __syncthreads();
+  float Sr = __fmul_rn(old_s, w_old);
+#pragma unroll
+  for (int w8 = 0; w8 < kPoolWarps; ++w8) Sr = __fadd_rn(Sr, red[w8]);
+  for (int k = tid; k < d; k += 256) {
+    float a = merge_existing ? __fmul_rn(st_acc[static_cast<long long>(r) * d + k], w_old) : 0.f;
+    int ch = 0;
+    for (; ch + 8 <= nch_r && ch + 8 <= 512; ch += 8) {
+      float pv[8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u) pv[u] = __ldcg(pr + static_cast<long long>(ch + u) * (d + 2) + 2 + k);
+#pragma unroll
+      for (int u = 0; u < 8; ++u) a = fmaf(pv[u], ch_scale[ch + u], a);
+    }
+    for (; ch < nch_r; ++ch) {
+      const float* pc = pr + static_cast<long long>(ch) * (d + 2);
+      const float sc = ch < 512 ? ch_scale[ch] : expf(__ldcg(pc) - Mr);
+      a = fmaf(__ldcg(pc + 2 + k), sc, a);
+    }
+    st_acc[static_cast<long long>(r) * d + k] = a;
+    g[static_cast<long long>(r) * d + k] = a / Sr;
+  }
+  __syncthreads();
+  if (tid == 0) {
+    st_m[r] = Mr;
+    st_s[r] = Sr;
+    counter[r] = 0;   // ready for the next call
+  }
+}
 
 // One CTA per (chunk of kPoolChunk rows, request).  Each warp loads its rows
 // (all loads issued before any arithmetic), computes the pooling logits with a
@@ -194,74 +267,185 @@ __global__ void __launch_bounds__(256) pool_partial_kernel(const T* __restrict__
     out[1] = S;
   }
   if constexpr (!MERGE) return;
-  // The last chunk CTA of request r to finish merges the request's chunk states
-  // (and, for an append, the stored state) and writes g = acc / s.
-  __shared__ int is_last;
-  __threadfence();
-  __syncthreads();
-  const int nch_r = (seg_end - seg_beg + kPoolChunkV - 1) / kPoolChunkV;
-  if (tid == 0) is_last = atomicAdd(counter + r, 1) == nch_r - 1;
-  __syncthreads();
-  if (!is_last) return;
-  __threadfence();
-  const float* pr = part + static_cast<long long>(r) * max_chunks * (d + 2);
-  // chunk maxima and weighted sums as block reductions (thread t takes
-  // chunks t, t + 256, ...), then each column's sum over the chunks with its
-  // loads issued ahead of the multiply-adds; the order is fixed, so the
-  // result is deterministic
-  __shared__ float ch_scale[512];
-  __shared__ float red[kPoolWarps];
-  const float old_m = merge_existing ? st_m[r] : -INFINITY;
-  const float old_s = merge_existing ? st_s[r] : 0.f;
-  float mloc = -INFINITY;
-  for (int ch = tid; ch < nch_r; ch += 256) mloc = fmaxf(mloc, __ldcg(pr + static_cast<long long>(ch) * (d + 2)));
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) mloc = fmaxf(mloc, __shfl_xor_sync(0xffffffffu, mloc, o));
-  if (lane == 0) red[warp] = mloc;
-  __syncthreads();
-  float Mr = old_m;
-#pragma unroll
-  for (int w8 = 0; w8 < kPoolWarps; ++w8) Mr = fmaxf(Mr, red[w8]);
-  const float w_old = merge_existing ? expf(old_m - Mr) : 0.f;
-  __syncthreads();                                  // red is reused below
-  float sloc = 0.f;
-  for (int ch = tid; ch < nch_r; ch += 256) {
-    const float* pc = pr + static_cast<long long>(ch) * (d + 2);
-    const float sc = expf(__ldcg(pc) - Mr);
-    if (ch < 512) ch_scale[ch] = sc;
-    sloc = fmaf(__ldcg(pc + 1), sc, sloc);
-  }
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) sloc += __shfl_xor_sync(0xffffffffu, sloc, o);
-  if (lane == 0) red[warp] = sloc;
-  __syncthreads();
-  float Sr = __fmul_rn(old_s, w_old);
-#pragma unroll
-  for (int w8 = 0; w8 < kPoolWarps; ++w8) Sr = __fadd_rn(Sr, red[w8]);
-  for (int k = tid; k < d; k += 256) {
-    float a = merge_existing ? __fmul_rn(st_acc[static_cast<long long>(r) * d + k], w_old) : 0.f;
-    int ch = 0;
-    for (; ch + 8 <= nch_r && ch + 8 <= 512; ch += 8) {
-      float pv[8];
-#pragma unroll
-      for (int u = 0; u < 8; ++u) pv[u] = __ldcg(pr + static_cast<long long>(ch + u) * (d + 2) + 2 + k);
-#pragma unroll
-      for (int u = 0; u < 8; ++u) a = fmaf(pv[u], ch_scale[ch + u], a);
-    }
-    for (; ch < nch_r; ++ch) {
-      const float* pc = pr + static_cast<long long>(ch) * (d + 2);
-      const float sc = ch < 512 ? ch_scale[ch] : expf(__ldcg(pc) - Mr);
-      a = fmaf(__ldcg(pc + 2 + k), sc, a);
-    }
-    st_acc[static_cast<long long>(r) * d + k] = a;
-    g[static_cast<long long>(r) * d + k] = a / Sr;
-  }
-  __syncthreads();
+  pool_merge_if_last(part + static_cast<long long>(r) * max_chunks * (d + 2),
+                     (seg_end - seg_beg + kPoolChunkV - 1) / kPoolChunkV, d, r, merge_existing, st_m, st_s, st_acc,
+                     g, counter);
+}
+
+constexpr int kPoolStages = 4;
+constexpr int kPoolStageBytes = 16384;
+constexpr int kPoolStreamCtasPerSm = 3;   // 64 KB ring each
+
+// Rebuild pooling of long histories.  One CTA per (chunk of chunk_rows rows,
+// request).  A request's rows are contiguous, so a stage of SR = 8 RW rows is
+// one untiled bulk copy; thread 0 keeps kPoolStages of them in flight
+// through a shared-memory ring (64 KB per CTA in flight, independent of the
+// register count), and each warp folds RW rows of every stage into its
+// online-softmax state.  The CTA's chunk state goes to part and the last
+// CTA of the request merges (pool_merge_if_last).
+template <typename T, int MAXC, int RW>
+__global__ void __launch_bounds__(256) pool_stream_kernel(const T* __restrict__ phi, const int* __restrict__ seg_off,
+                                                          const float* __restrict__ w_pool, int d, float inv_sqrt_d,
+                                                          int chunk_rows, int max_chunks, float* __restrict__ part,
+                                                          int merge_existing, float* st_m, float* st_s, float* st_acc,
+                                                          float* __restrict__ g, int* counter, int* status) {
+  constexpr int VEC = Vec16<T>::N;
+  constexpr int SR = kPoolWarps * RW;
+  extern __shared__ __align__(128) uint8_t pool_ring[];
+  __shared__ __align__(8) uint64_t full[kPoolStages];
+  __shared__ float sm_m[kPoolWarps], sm_s[kPoolWarps];
+  __shared__ int abort_flag;
+  const int r = blockIdx.y, c = blockIdx.x;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   if (tid == 0) {
-    st_m[r] = Mr;
-    st_s[r] = Sr;
-    counter[r] = 0;   // ready for the next call
+#pragma unroll
+    for (int i = 0; i < kPoolStages; ++i) tc::mbar_init(&full[i], 1);
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    abort_flag = 0;
   }
+  pdl_launch_dependents();
+  pdl_wait();
+  const int seg_beg = seg_off[r], seg_end = seg_off[r + 1];
+  const int beg = seg_beg + c * chunk_rows;
+  const int nrows = min(seg_end - beg, chunk_rows);
+  if (nrows <= 0) return;                           // past the request's rows (uniform over the CTA)
+  const int n_st = (nrows + SR - 1) / SR;
+  const uint32_t row_bytes = static_cast<uint32_t>(d) * sizeof(T);
+  const T* src0 = phi + static_cast<long long>(beg) * d;
+  __syncthreads();                                  // barriers initialised
+  if (tid == 0) {
+    for (int j = 0; j < min(n_st, kPoolStages); ++j) {
+      const uint32_t bytes = static_cast<uint32_t>(min(SR, nrows - j * SR)) * row_bytes;
+      tc::mbar_expect_tx(&full[j], bytes);
+      tc::bulk_load(pool_ring + j * kPoolStageBytes, src0 + static_cast<long long>(j) * SR * d, bytes, &full[j]);
+    }
+  }
+  float w[MAXC][VEC], acc[MAXC][VEC];
+#pragma unroll
+  for (int j = 0; j < MAXC; ++j) {
+    const int col = (j * 32 + lane) * VEC;
+#pragma unroll
+    for (int i = 0; i < VEC; ++i) {
+      w[j][i] = col + i < d ? __ldg(w_pool + col + i) : 0.f;
+      acc[j][i] = 0.f;
+    }
+  }
+  float m = -INFINITY, ssum = 0.f;
+  int j = 0;
+  for (; j < n_st; ++j) {
+    const int slot = j % kPoolStages;
+    if (!tc::mbar_wait_plain(&full[slot], (j / kPoolStages) & 1)) abort_flag = 1;
+    const T* st = reinterpret_cast<const T*>(pool_ring + slot * kPoolStageBytes);
+    const int nr = min(SR, nrows - j * SR);
+    float v[RW][MAXC][VEC];
+#pragma unroll
+    for (int t = 0; t < RW; ++t) {
+      const int i = warp + kPoolWarps * t;
+#pragma unroll
+      for (int q = 0; q < MAXC; ++q) {
+        const int col = (q * 32 + lane) * VEC;
+        if (i < nr && col < d) Vec16<T>::load(st + i * d + col, v[t][q]);
+        else {
+#pragma unroll
+          for (int e = 0; e < VEC; ++e) v[t][q][e] = 0.f;
+        }
+      }
+    }
+    float z[RW];
+#pragma unroll
+    for (int t = 0; t < RW; ++t) {
+      float dot = 0.f;
+#pragma unroll
+      for (int q = 0; q < MAXC; ++q)
+#pragma unroll
+        for (int e = 0; e < VEC; ++e) dot = fmaf(v[t][q][e], w[q][e], dot);
+      z[t] = dot;
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1)
+#pragma unroll
+      for (int t = 0; t < RW; ++t) z[t] += __shfl_xor_sync(0xffffffffu, z[t], o);
+    float mb = m;
+#pragma unroll
+    for (int t = 0; t < RW; ++t) {
+      z[t] *= inv_sqrt_d;
+      if (warp + kPoolWarps * t < nr) mb = fmaxf(mb, z[t]);
+    }
+    const float corr = mb == -INFINITY ? 1.f : expf(m - mb);
+    ssum *= corr;
+#pragma unroll
+    for (int q = 0; q < MAXC; ++q)
+#pragma unroll
+      for (int e = 0; e < VEC; ++e) acc[q][e] *= corr;
+#pragma unroll
+    for (int t = 0; t < RW; ++t) {
+      if (warp + kPoolWarps * t < nr) {
+        const float e = expf(z[t] - mb);
+        ssum += e;
+#pragma unroll
+        for (int q = 0; q < MAXC; ++q)
+#pragma unroll
+          for (int u = 0; u < VEC; ++u) acc[q][u] = fmaf(e, v[t][q][u], acc[q][u]);
+      }
+    }
+    m = mb;
+    __syncthreads();                                // every warp is done with this slot
+    if (abort_flag) break;
+    if (tid == 0 && j + kPoolStages < n_st) {
+      const int jn = j + kPoolStages;
+      const uint32_t bytes = static_cast<uint32_t>(min(SR, nrows - jn * SR)) * row_bytes;
+      tc::mbar_expect_tx(&full[slot], bytes);
+      tc::bulk_load(pool_ring + slot * kPoolStageBytes, src0 + static_cast<long long>(jn) * SR * d, bytes,
+                    &full[slot]);
+    }
+  }
+  if (abort_flag) {
+    // let the copies still in flight land (bounded) before the CTA exits
+    if (tid == 0) {
+      latch_status(status, TXS_ERR_DEVICE_TIMEOUT);
+      for (int jj = j; jj < min(n_st, j + kPoolStages); ++jj)
+        tc::mbar_wait_plain(&full[jj % kPoolStages], (jj / kPoolStages) & 1);
+    }
+    return;
+  }
+  // combine the warps' states; the ring is free now and holds acc[8][512]
+  float* sm_acc = reinterpret_cast<float*>(pool_ring);
+#pragma unroll
+  for (int q = 0; q < MAXC; ++q) {
+    const int col = (q * 32 + lane) * VEC;
+#pragma unroll
+    for (int e = 0; e < VEC; ++e)
+      if (col + e < d) sm_acc[warp * 512 + col + e] = acc[q][e];
+  }
+  if (lane == 0) {
+    sm_m[warp] = m;
+    sm_s[warp] = ssum;
+  }
+  __syncthreads();
+  float M = -INFINITY;
+#pragma unroll
+  for (int w8 = 0; w8 < kPoolWarps; ++w8) M = fmaxf(M, sm_m[w8]);
+  float scale[kPoolWarps];
+  float S = 0.f;
+#pragma unroll
+  for (int w8 = 0; w8 < kPoolWarps; ++w8) {
+    scale[w8] = sm_s[w8] > 0.f ? expf(sm_m[w8] - M) : 0.f;
+    S += sm_s[w8] * scale[w8];
+  }
+  float* out = part + (static_cast<long long>(r) * max_chunks + c) * (d + 2);
+  for (int k = tid; k < d; k += 256) {
+    float a = 0.f;
+#pragma unroll
+    for (int w8 = 0; w8 < kPoolWarps; ++w8) a = fmaf(sm_acc[w8 * 512 + k], scale[w8], a);
+    out[2 + k] = a;
+  }
+  if (tid == 0) {
+    out[0] = M;
+    out[1] = S;
+  }
+  pool_merge_if_last(part + static_cast<long long>(r) * max_chunks * (d + 2),
+                     (seg_end - seg_beg + chunk_rows - 1) / chunk_rows, d, r, merge_existing, st_m, st_s, st_acc, g,
+                     counter);
 }
 
 constexpr int kAnchorReq = 16;        // anchors staged per CTA (grid.y covers the rest)
@@ -454,30 +638,85 @@ __global__ void hash_kernel(const uint32_t* __restrict__ p, long long n_words, u
 
 }  // namespace
 
+template <typename T, int MAXC, int RW>
+cudaError_t launch_pool_stream(const T* phi, const int* seg_off, int R, int chunks, int chunk_rows, const float* w_pool,
+                               int d, float isd, int max_chunks, float* part, int merge_existing, float* st_m,
+                               float* st_s, float* st_acc, float* g, int* counter, int* status, cudaStream_t s) {
+  constexpr int kSmem = kPoolStages * kPoolStageBytes;
+  static bool attr = false;
+  if (!attr) {
+    cudaError_t e = cudaFuncSetAttribute(pool_stream_kernel<T, MAXC, RW>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         kSmem);
+    if (e != cudaSuccess) return e;
+    attr = true;
+  }
+  return launch_pdl(pool_stream_kernel<T, MAXC, RW>, dim3(chunks, R), dim3(256), kSmem, s, phi, seg_off, w_pool, d,
+                    isd, chunk_rows, max_chunks, part, merge_existing, st_m, st_s, st_acc, g, counter, status);
+}
+
+template <typename T, int RW>
+cudaError_t launch_pool_stream_c(int nch, const T* phi, const int* seg_off, int R, int chunks, int chunk_rows,
+                                 const float* w_pool, int d, float isd, int max_chunks, float* part, int merge_existing,
+                                 float* st_m, float* st_s, float* st_acc, float* g, int* counter, int* status,
+                                 cudaStream_t s) {
+  if (nch == 1)
+    return launch_pool_stream<T, 1, RW>(phi, seg_off, R, chunks, chunk_rows, w_pool, d, isd, max_chunks, part,
+                                        merge_existing, st_m, st_s, st_acc, g, counter, status, s);
+  if (nch == 2)
+    return launch_pool_stream<T, 2, RW>(phi, seg_off, R, chunks, chunk_rows, w_pool, d, isd, max_chunks, part,
+                                        merge_existing, st_m, st_s, st_acc, g, counter, status, s);
+  return launch_pool_stream<T, 4, RW>(phi, seg_off, R, chunks, chunk_rows, w_pool, d, isd, max_chunks, part,
+                                      merge_existing, st_m, st_s, st_acc, g, counter, status, s);
+}
+
+// Chunks of more than kPoolChunkV rows go through the streaming kernel (rows
+// 16-byte aligned); an append of at most kPoolChunkV rows per request keeps
+// the one-chunk kernel, which merges in the CTA.
 template <typename T>
 cudaError_t launch_pool(const T* phi, const int* seg_off, int R, int max_rows, const float* w_pool, int d,
                         int max_chunks, float* part, int merge_existing, float* st_m, float* st_s, float* st_acc,
-                        float* g, int* counter, cudaStream_t s) {
+                        float* g, int* counter, int* status, cudaStream_t s) {
   const int chunks = (max_rows + kPoolChunkV - 1) / kPoolChunkV;
   if (chunks > max_chunks) return cudaErrorInvalidValue;
   if (chunks == 0) return cudaSuccess;   // no new rows: the stored state and g stay as they are
   constexpr int VEC = Vec16<T>::N;
   const int nch = (d + 32 * VEC - 1) / (32 * VEC);
+  if (nch > 4 || d > 512) return cudaErrorInvalidValue;
   const float isd = 1.0f / sqrtf(static_cast<float>(d));
-  const dim3 grid(chunks, R);
+  const int row_bytes = d * static_cast<int>(sizeof(T));
+  const bool stream = max_rows > kPoolChunkV && row_bytes % 16 == 0 && reinterpret_cast<uintptr_t>(phi) % 16 == 0;
   cudaError_t err0 = cudaSuccess;
   prof_begin(KC_POOL, s);
-  if (nch == 1)
-    err0 = launch_pdl(pool_partial_kernel<T, 1>, grid, dim3(256), 0, s, phi, seg_off, w_pool, d, isd, max_chunks,
-                      part, merge_existing, st_m, st_s, st_acc, g, counter, 0);
-  else if (nch == 2)
-    err0 = launch_pdl(pool_partial_kernel<T, 2>, grid, dim3(256), 0, s, phi, seg_off, w_pool, d, isd, max_chunks,
-                      part, merge_existing, st_m, st_s, st_acc, g, counter, 0);
-  else if (nch <= 4)
-    err0 = launch_pdl(pool_partial_kernel<T, 4>, grid, dim3(256), 0, s, phi, seg_off, w_pool, d, isd, max_chunks,
-                      part, merge_existing, st_m, st_s, st_acc, g, counter, 0);
-  else
-    return cudaErrorInvalidValue;
+  if (stream) {
+    // the longest chunk that still gives every SM its resident CTAs twice over
+    int chunk_rows = 256;
+    while (chunk_rows > kPoolChunkV &&
+           static_cast<long long>(R) * ((max_rows + chunk_rows - 1) / chunk_rows) <
+               2LL * kPoolStreamCtasPerSm * tc::num_sms())
+      chunk_rows /= 2;
+    const int n_chunks = (max_rows + chunk_rows - 1) / chunk_rows;
+    const int rw = kPoolStageBytes / (kPoolWarps * row_bytes);   // rows per warp and stage
+    if (rw >= 4)
+      err0 = launch_pool_stream_c<T, 4>(nch, phi, seg_off, R, n_chunks, chunk_rows, w_pool, d, isd, max_chunks, part,
+                                        merge_existing, st_m, st_s, st_acc, g, counter, status, s);
+    else if (rw >= 2)
+      err0 = launch_pool_stream_c<T, 2>(nch, phi, seg_off, R, n_chunks, chunk_rows, w_pool, d, isd, max_chunks, part,
+                                        merge_existing, st_m, st_s, st_acc, g, counter, status, s);
+    else
+      err0 = launch_pool_stream_c<T, 1>(nch, phi, seg_off, R, n_chunks, chunk_rows, w_pool, d, isd, max_chunks, part,
+                                        merge_existing, st_m, st_s, st_acc, g, counter, status, s);
+  } else {
+    const dim3 grid(chunks, R);
+    if (nch == 1)
+      err0 = launch_pdl(pool_partial_kernel<T, 1>, grid, dim3(256), 0, s, phi, seg_off, w_pool, d, isd, max_chunks,
+                        part, merge_existing, st_m, st_s, st_acc, g, counter, 0);
+    else if (nch == 2)
+      err0 = launch_pdl(pool_partial_kernel<T, 2>, grid, dim3(256), 0, s, phi, seg_off, w_pool, d, isd, max_chunks,
+                        part, merge_existing, st_m, st_s, st_acc, g, counter, 0);
+    else
+      err0 = launch_pdl(pool_partial_kernel<T, 4>, grid, dim3(256), 0, s, phi, seg_off, w_pool, d, isd, max_chunks,
+                        part, merge_existing, st_m, st_s, st_acc, g, counter, 0);
+  }
   cudaError_t err = err0 != cudaSuccess ? err0 : cudaGetLastError();
   prof_end(KC_POOL, s);
   return err;
@@ -720,7 +959,7 @@ cudaError_t launch_prefix_pool(const T* phi, const int* ends, int n_ev, int off_
 
 #define TXS_INST(T)                                                                                                 \
   template cudaError_t launch_pool<T>(const T*, const int*, int, int, const float*, int, int, float*, int, float*, \
-                                      float*, float*, float*, int*, cudaStream_t);                                  \
+                                      float*, float*, float*, int*, int*, cudaStream_t);                            \
   template cudaError_t launch_prefix_pool<T>(const T*, const int*, int, int, const float*, int, float*, float*,     \
                                              int*, int*, cudaStream_t);                                             \
   template cudaError_t launch_anchor_proj<T>(const float*, const T*, const float*, float*, int, int, int, int,     \

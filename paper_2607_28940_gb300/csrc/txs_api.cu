@@ -424,7 +424,7 @@ txs_status project_rows(txs_model* m, txs_kv_cache* c, int n_req, const int32_t*
     TXS_CK(gemm(m, rows, d, m->Wt_kv, e, nullptr, s, KC_GEMM_KV));
   }
   TXS_CK(launch_pool<T>(static_cast<const T*>(rows), c->d_in_off, n_req, max_rows, m->w_pool, d, c->max_chunks,
-                        c->part, append ? 1 : 0, c->pool_m, c->pool_s, c->pool_acc, c->g, c->pool_cnt, s));
+                        c->part, append ? 1 : 0, c->pool_m, c->pool_s, c->pool_acc, c->g, c->pool_cnt, m->status, s));
   if (project_anchor)
     TXS_CK(launch_anchor_proj<T>(c->g, static_cast<const T*>(m->Wt_kv), m->b_kv, c->gkv, n_req, d, c->dkv, nL, s));
   return TXS_OK;

@@ -301,7 +301,7 @@ extern const int kPoolChunk;
 template <typename T>
 cudaError_t launch_pool(const T* phi, const int* seg_off, int R, int max_rows, const float* w_pool, int d,
                         int max_chunks, float* part, int merge_existing, float* st_m, float* st_s, float* st_acc,
-                        float* g, int* counter, cudaStream_t s);
+                        float* g, int* counter, int* status, cudaStream_t s);
 // Per-event anchors of one user's stream: g[t] = attention pooling of
 // phi[0 .. ends[t]); also writes ev_off[t] = off_user, ev_len[t] = ends[t]
 // (ends: host, at most 4096 events; d <= 512).  `part`: scratch of
