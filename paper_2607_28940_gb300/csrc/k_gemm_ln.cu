@@ -93,7 +93,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       mbar_init(acc_empty + b, PING ? kGroupWarps : kWarps);
     }
     for (int i = 0; i < 8; ++i) {
-      mbar_init(xfull + i, P * 32);
+      // PING: the waiting warp's expect_tx is the one arrival; the peers'
+      // statistics complete as transaction bytes
+      mbar_init(xfull + i, PING ? 1 : P * 32);
       mbar_init(hfull + i, P * 32);
     }
     *abort_flag = 0;
@@ -261,15 +263,18 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           m2 = m2 + m2c + dlt * dlt * (na * 32.f / nt);
         }
       }
-      // publish (mean, M2) of these 128 columns to every CTA of the cluster
+      // publish (mean, M2) of these 128 columns to every CTA of the cluster:
+      // this CTA's slot by a plain store (read back by this thread), the
+      // peers' by asynchronous stores counted on their barriers
       {
         float2* mine = xbuf + (pb * P + static_cast<int>(rk)) * 128 + trow;
+        *mine = make_float2(mean_p, m2);
 #pragma unroll
-        for (int pr = 0; pr < CS; ++pr) {
-          st_peer_f32x2(map_peer(mine, pr), mean_p, m2);
-          mbar_arrive_peer(map_peer(xfull + pb * 4 + q, pr));
-        }
+        for (int pr = 0; pr < CS; ++pr)
+          if (pr != static_cast<int>(rk))
+            st_async_f32x2(map_peer(mine, pr), mean_p, m2, map_peer(xfull + pb * 4 + q, pr));
       }
+      if (lane == 0) mbar_expect_tx(xfull + pb * 4 + q, (CS - 1) * 32 * 8);
       bool ok = mbar_wait_cluster(xfull + pb * 4 + q, use, abort_flag);
       ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
       if (!ok) break;

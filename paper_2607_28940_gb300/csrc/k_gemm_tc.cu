@@ -641,14 +641,19 @@ __device__ __forceinline__ void attn_epilogue_warp(const EpiArgs& e, uint32_t tm
 
 // BRES: the CTA's whole B slice (BN x K, K <= KRES) stays resident in shared
 // memory and only A streams through the ring.  NAP: head actions padded
-// (EPI_LN_HEAD).
-template <int BN, int EPI, int NAP = 4, bool BRES = false>
+// (EPI_LN_HEAD).  PAIR: a cluster of two CTAs computes a 256 x BN tile with
+// M = 256 MMAs (cta_group::2): each CTA stages its 128 rows of A and half of
+// the BN rows of B, so a stage carries half the weight bytes per MMA flop of
+// a one-CTA tile.
+template <int BN, int EPI, int NAP = 4, bool BRES = false, bool PAIR = false>
 struct Shape {
   static constexpr int BN_MMA = BN < 256 ? BN : 256;     // N of one tcgen05.mma
-  static constexpr int B_BOX = BN_MMA;                    // rows of one TMA box of B
+  static constexpr int B_ROWS = PAIR ? BN / 2 : BN;       // rows of B this CTA stages
+  static constexpr int B_BOX = PAIR ? B_ROWS : BN_MMA;    // rows of one TMA box of B
+  static constexpr int TM = PAIR ? 2 * BM : BM;           // rows of a tile
   static constexpr int KRES = 256;
   static constexpr int BRES_BYTES = BRES ? BN * KRES * 2 : 0;
-  static constexpr int B_STAGE_BYTES = BRES ? 0 : BN * BK * 2;
+  static constexpr int B_STAGE_BYTES = BRES ? 0 : B_ROWS * BK * 2;
   static constexpr int STAGE_BYTES = A_STAGE_BYTES + B_STAGE_BYTES;
   static constexpr bool LN = EPI == EPI_LN || EPI == EPI_LN_HEAD;
   static constexpr int RED_BYTES = LN ? 2 * 128 * kRedStride * 4 : 0;
@@ -682,6 +687,7 @@ struct Shape {
   static_assert((RED_BYTES + WEFF_BYTES + AUX_BYTES + STG_BYTES + ATT_BYTES) % 16 == 0,
                 "mbarriers must stay 8-byte aligned");
   static_assert(!ATT || (BN == 2 * kAttCols && !BRES), "fused attention: 128-column tiles");
+  static_assert(!PAIR || (LEAN && BN == 256), "CTA pairs: 256-column streaming tiles");
   static_assert(SMEM_BYTES <= 232448, "shared memory");
   static_assert((TMEM_COLS & (TMEM_COLS - 1)) == 0 && TMEM_COLS <= 512, "TMEM columns");
 };
@@ -707,12 +713,12 @@ struct NoParams {
 template <int EPI>
 using ParamsFor = typename std::conditional<EPI == EPI_KV, KvParams, NoParams>::type;
 
-template <int BN, int EPI, int NAP, bool BRES>
+template <int BN, int EPI, int NAP, bool BRES, bool PAIR>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                    const __grid_constant__ CUtensorMap tmO, const EpiArgs e,
                    const __grid_constant__ ParamsFor<EPI> kp) {
-  using S = Shape<BN, EPI, NAP, BRES>;
+  using S = Shape<BN, EPI, NAP, BRES, PAIR>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* sA = smem;
@@ -735,12 +741,15 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_holder + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  // PAIR: rank 1 holds rows [128, 256) of every tile; rank 0 issues the MMAs
+  // and owns the barriers that gate them (full, acc_empty)
+  const uint32_t rank = PAIR ? cluster_rank() : 0;
   const int n_tiles = e.N / BN;
-  const int num_tiles = ((e.M + BM - 1) / BM) * n_tiles;
+  const int m_tiles = (e.M + S::TM - 1) / S::TM;
+  const int num_tiles = m_tiles * n_tiles;
   const int num_kb = e.K / BK;
-  const int m_tiles = (e.M + BM - 1) / BM;
-  // this CTA's tiles: t_lo, t_lo + t_step, ... < t_hi
-  int t_lo = blockIdx.x, t_hi = num_tiles, t_step = gridDim.x;
+  // this CTA's tiles: t_lo, t_lo + t_step, ... < t_hi (the same for both CTAs of a pair)
+  int t_lo = PAIR ? blockIdx.x / 2 : blockIdx.x, t_hi = num_tiles, t_step = PAIR ? gridDim.x / 2 : gridDim.x;
   if constexpr (BRES) {
     t_lo = static_cast<int>(static_cast<long long>(blockIdx.x) * num_tiles / gridDim.x);
     t_hi = static_cast<int>(static_cast<long long>(blockIdx.x + 1) * num_tiles / gridDim.x);
@@ -756,18 +765,41 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(acc_full + b, 1);
-      mbar_init(acc_empty + b, kEpiWarps);
+      mbar_init(acc_empty + b, PAIR ? 2 * kEpiWarps : kEpiWarps);   // rank 0's: both CTAs' epilogues
     }
     mbar_init(b_full, 1);
     mbar_init(b_empty, 1);
     *abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
-  if (warp == 1) tmem_alloc(tmem_holder, S::TMEM_COLS);
+  if (warp == 1) {
+    if constexpr (PAIR) tmem_alloc_pair(tmem_holder, S::TMEM_COLS);
+    else tmem_alloc(tmem_holder, S::TMEM_COLS);
+  }
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_holder;
+  if constexpr (PAIR) cluster_sync();   // both CTAs' barriers exist before any crosses the pair
+  // shared::cluster address of rank 0's copy of a barrier (PAIR)
+  auto lead = [&](uint64_t* bar) { return PAIR ? map_peer(bar, 0) : smem_u32(bar); };
+  // bytes that complete one stage: both CTAs' loads count on rank 0's barrier
+  constexpr uint32_t kFullBytes = (PAIR ? 2 : 1) * S::STAGE_BYTES;
+  const bool expects = !PAIR || rank == 0;
+  auto load_a = [&](int s, int kb, int m0) {
+    if constexpr (PAIR) tma_load_2d_pair(sA + s * A_STAGE_BYTES, &tmA, lead(full + s), kb * BK, m0);
+    else tma_load_2d(sA + s * A_STAGE_BYTES, &tmA, full + s, kb * BK, m0);
+  };
+  auto load_b = [&](int s, int kb, int n0) {
+#pragma unroll
+    for (int j = 0; j < S::B_ROWS; j += S::B_BOX) {
+      if constexpr (PAIR)
+        tma_load_2d_pair(sB + s * S::B_STAGE_BYTES + j * (BK * 2), &tmB, lead(full + s), kb * BK,
+                         n0 + static_cast<int>(rank) * S::B_ROWS + j);
+      else
+        tma_load_2d(sB + s * S::B_STAGE_BYTES + j * (BK * 2), &tmB, full + s, kb * BK, n0 + j);
+    }
+  };
   // the set-up above overlaps the previous kernel's tail; its outputs are read below
   pdl_launch_dependents();
   // The weights are not written by the kernels before this one: the
@@ -786,10 +818,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     } else {
       n_pre = num_kb < S::STAGES ? num_kb : S::STAGES;
       for (int kb = 0; kb < n_pre; ++kb) {   // fresh ring: these stages are free
-        mbar_expect_tx(full + kb, S::STAGE_BYTES);
-#pragma unroll
-        for (int j = 0; j < BN; j += S::B_BOX)
-          tma_load_2d(sB + kb * S::B_STAGE_BYTES + j * (BK * 2), &tmB, full + kb, kb * BK, n0 + j);
+        if (expects) mbar_expect_tx(full + kb, kFullBytes);
+        load_b(kb, kb, n0);
       }
     }
   }
@@ -846,7 +876,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       }
       bool ok = true;
       for (int t = t_lo; t < t_hi && ok; t += t_step) {
-        const int m0 = tile_m(t) * BM, n0 = tile_n(t) * BN;
+        const int m0 = tile_m(t) * S::TM + static_cast<int>(rank) * BM, n0 = tile_n(t) * BN;
         if constexpr (BRES) {
           if (n0 != cur_n) {
             if (nb > 0 && !mbar_wait(b_empty, (nb - 1) & 1, abort_flag)) break;
@@ -863,23 +893,25 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           const int s = it % S::STAGES;
           const uint32_t ph = (it / S::STAGES) & 1;
           if (it < n_pre) {       // weights already in flight, bytes already expected
-            tma_load_2d(sA + s * A_STAGE_BYTES, &tmA, full + s, kb * BK, m0);
+            load_a(s, kb, m0);
             continue;
           }
           if (!mbar_wait(empty + s, ph ^ 1, abort_flag)) {
             ok = false;
             break;
           }
-          mbar_expect_tx(full + s, S::STAGE_BYTES);
-          tma_load_2d(sA + s * A_STAGE_BYTES, &tmA, full + s, kb * BK, m0);
-          if constexpr (!BRES) {
-#pragma unroll
-            for (int j = 0; j < BN; j += S::B_BOX)
-              tma_load_2d(sB + s * S::B_STAGE_BYTES + j * (BK * 2), &tmB, full + s, kb * BK, n0 + j);
-          }
+          if (expects) mbar_expect_tx(full + s, kFullBytes);
+          load_a(s, kb, m0);
+          if constexpr (!BRES) load_b(s, kb, n0);
         }
       }
-      if (*abort_flag) {
+      if constexpr (PAIR) {
+        // rank 0's MMAs release this CTA's stages by multicast commits: take
+        // the last ones before the CTA may exit
+        for (int k = it > S::STAGES ? it - S::STAGES : 0; k < it && !*abort_flag; ++k)
+          mbar_wait(empty + k % S::STAGES, (k / S::STAGES) & 1, abort_flag);
+      }
+      if (*abort_flag && expects) {
         // let the copies already in flight land before shared memory is released
         for (int k = it > S::STAGES ? it - S::STAGES : 0; k < it; ++k)
           mbar_wait_plain(full + k % S::STAGES, (k / S::STAGES) & 1);
@@ -887,8 +919,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       }
     }
   } else if (warp == 1) {
-    if (lane == 0) {
-      constexpr uint32_t idesc = idesc_bf16(BM, S::BN_MMA);
+    if (lane == 0 && (!PAIR || rank == 0)) {
+      constexpr uint32_t idesc = idesc_bf16(S::TM, S::BN_MMA);
       int it = 0, i = 0;
       int nb = 0, cur_n = -1;
       bool ok = true;
@@ -924,13 +956,20 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
               // 32 bytes along K per step inside the swizzle row; N halves are
               // S::BN_MMA rows (x 128 bytes) apart
               const uint64_t boff = static_cast<uint64_t>((j * S::BN_MMA * BK * 2) >> 4);
-              mma_bf16(dacc + j * S::BN_MMA, adesc + 2 * k, bdesc + boff + 2 * k, idesc,
-                       (kb > 0 || k > 0) ? 1u : 0u);
+              if constexpr (PAIR)
+                mma_bf16_pair(dacc + j * S::BN_MMA, adesc + 2 * k, bdesc + boff + 2 * k, idesc,
+                              (kb > 0 || k > 0) ? 1u : 0u);
+              else
+                mma_bf16(dacc + j * S::BN_MMA, adesc + 2 * k, bdesc + boff + 2 * k, idesc,
+                         (kb > 0 || k > 0) ? 1u : 0u);
             }
           }
-          mma_commit(empty + s);
+          if constexpr (PAIR) mma_commit_pair(empty + s, 3);
+          else mma_commit(empty + s);
         }
-        mma_commit(acc_full + buf);   // also on abort: the epilogue waits on every issued MMA
+        // also on abort: the epilogue waits on every issued MMA
+        if constexpr (PAIR) mma_commit_pair(acc_full + buf, 3);
+        else mma_commit(acc_full + buf);
         if constexpr (BRES) {
           // the resident slice is free once this tile's MMAs are done
           if (t + 1 >= t_hi || tile_n(t + 1) != nt) mma_commit(b_empty);
@@ -959,21 +998,28 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         go = __shfl_sync(0xffffffffu, go ? 1 : 0, 0) != 0;
         if (!go) break;
         tc_fence_after();
-        const int m0 = tile_m(t) * BM, n0 = tile_n(t) * BN;
+        const int m0 = tile_m(t) * S::TM + static_cast<int>(rank) * BM, n0 = tile_n(t) * BN;
         epilogue<BN, EPI, NAP, S::SBUF>(e, tmem + buf * BN + (static_cast<uint32_t>(q * 32) << 16), m0 + q * 32 + lane, n0,
                                h * (BN / 2), q, h, red, s_weff, bias, seg_off, dst_row0, &tmO, stage, kchunk);
         tc_fence_before();
         __syncwarp();
-        if (lane == 0) mbar_arrive(acc_empty + buf);
+        if (lane == 0) {
+          if constexpr (PAIR) mbar_arrive_peer_signal(lead(acc_empty + buf));
+          else mbar_arrive(acc_empty + buf);
+        }
       }
       if (lane == 0) bulk_wait_all();   // this warp's bulk stores are complete before exit
     }
   }
   tc_fence_before();
   __syncthreads();
+  // PAIR: rank 1's epilogue arrivals on rank 0 have landed and neither CTA
+  // frees its TMEM before the other is done with the pair's accumulators
+  if constexpr (PAIR) cluster_sync();
   if (warp == 1) {
     tc_fence_after();
-    tmem_dealloc(tmem, S::TMEM_COLS);
+    if constexpr (PAIR) tmem_dealloc_pair(tmem, S::TMEM_COLS);
+    else tmem_dealloc(tmem, S::TMEM_COLS);
   }
   if (threadIdx.x == 0 && *abort_flag) latch_status(e.status, TXS_ERR_DEVICE_TIMEOUT);
 }
@@ -1062,17 +1108,37 @@ int num_sms() {
   return n;
 }
 
-template <int BN, int EPI, int NAP = 4, bool BRES = false>
+template <int BN, int EPI, int NAP = 4, bool BRES = false, bool PAIR = false>
 static cudaError_t launch_bn(const __nv_bfloat16* A, long long lda, const __nv_bfloat16* B, const EpiArgs& e,
                              cudaStream_t s, int cls) {
-  using Sh = Shape<BN, EPI, NAP, BRES>;
+  using Sh = Shape<BN, EPI, NAP, BRES, PAIR>;
+  auto kern = gemm_tc_kernel<BN, EPI, NAP, BRES, PAIR>;
   if (BRES && e.K > Sh::KRES) return cudaErrorInvalidValue;
-  static bool attr_set = false;
-  if (!attr_set) {
-    cudaError_t err = cudaFuncSetAttribute(gemm_tc_kernel<BN, EPI, NAP, BRES>,
-                                           cudaFuncAttributeMaxDynamicSharedMemorySize, Sh::SMEM_BYTES);
+  static int max_ctas = 0;   // CTAs resident at once (whole pairs with PAIR)
+  if (!max_ctas) {
+    cudaError_t err = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, Sh::SMEM_BYTES);
     if (err != cudaSuccess) return err;
-    attr_set = true;
+    int n = num_sms();
+    if (PAIR) {
+      cudaLaunchAttribute at[1];
+      at[0].id = cudaLaunchAttributeClusterDimension;
+      at[0].val.clusterDim.x = 2;
+      at[0].val.clusterDim.y = 1;
+      at[0].val.clusterDim.z = 1;
+      cudaLaunchConfig_t q = {};
+      q.gridDim = dim3((num_sms() / 2) * 2);
+      q.blockDim = dim3(NUM_THREADS);
+      q.dynamicSmemBytes = Sh::SMEM_BYTES;
+      q.attrs = at;
+      q.numAttrs = 1;
+      int c = 0;
+      if (cudaOccupancyMaxActiveClusters(&c, kern, &q) != cudaSuccess || c <= 0) {
+        (void)cudaGetLastError();
+        c = num_sms() / 2;
+      }
+      n = 2 * c;
+    }
+    max_ctas = n;
   }
   CUtensorMap ta, tb, to;
   if (!make_tmap(&ta, A, e.M, e.K, lda, BM)) return cudaErrorInvalidValue;
@@ -1086,8 +1152,9 @@ static cudaError_t launch_bn(const __nv_bfloat16* A, long long lda, const __nv_b
   } else {
     if (!make_tmap_out(&to, e.out, e.M, e.N, e.ldo)) return cudaErrorInvalidValue;
   }
-  const long long tiles = static_cast<long long>((e.M + BM - 1) / BM) * (e.N / BN);
-  const int grid = static_cast<int>(tiles < num_sms() ? tiles : num_sms());
+  const long long tiles = static_cast<long long>((e.M + Sh::TM - 1) / Sh::TM) * (e.N / BN);
+  const int per_tile = PAIR ? 2 : 1;
+  const int grid = static_cast<int>(tiles * per_tile < max_ctas ? tiles * per_tile : (max_ctas / per_tile) * per_tile);
   ParamsFor<EPI> kp;
   kp.n_seg = -1;
   if constexpr (EPI == EPI_KV) {
@@ -1099,8 +1166,26 @@ static cudaError_t launch_bn(const __nv_bfloat16* A, long long lda, const __nv_b
     }
   }
   prof_begin(cls, s);
-  cudaError_t err = launch_pdl(gemm_tc_kernel<BN, EPI, NAP, BRES>, dim3(grid), dim3(NUM_THREADS), Sh::SMEM_BYTES,
-                               s, ta, tb, to, e, kp);
+  cudaError_t err;
+  if constexpr (PAIR) {
+    cudaLaunchAttribute at[2];
+    at[0].id = cudaLaunchAttributeClusterDimension;
+    at[0].val.clusterDim.x = 2;
+    at[0].val.clusterDim.y = 1;
+    at[0].val.clusterDim.z = 1;
+    at[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    at[1].val.programmaticStreamSerializationAllowed = 1;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(grid);
+    cfg.blockDim = dim3(NUM_THREADS);
+    cfg.dynamicSmemBytes = Sh::SMEM_BYTES;
+    cfg.stream = s;
+    cfg.attrs = at;
+    cfg.numAttrs = 2;
+    err = cudaLaunchKernelEx(&cfg, kern, ta, tb, to, e, kp);
+  } else {
+    err = launch_pdl(kern, dim3(grid), dim3(NUM_THREADS), Sh::SMEM_BYTES, s, ta, tb, to, e, kp);
+  }
   prof_end(cls, s);
   return err;
 }
@@ -1127,6 +1212,9 @@ static cudaError_t launch_plain(const __nv_bfloat16* A, long long lda, const __n
   // short K and at least two tiles per SM: keep each CTA's B slice resident
   if (fits(256) && e.K <= Shape<256, EPI, 4, true>::KRES && m_tiles * (e.N / 256) >= 2 * num_sms())
     return launch_bn<256, EPI, 4, true>(A, lda, B, e, s, cls);
+  // long streams of 256-column tiles: CTA pairs with M = 256 MMAs
+  if (fits(256) && ((e.M + 255) / 256) * (e.N / 256) >= num_sms())
+    return launch_bn<256, EPI, 4, false, true>(A, lda, B, e, s, cls);
   if (fits(256) && m_tiles * (e.N / 256) >= num_sms()) return launch_bn<256, EPI>(A, lda, B, e, s, cls);
   if (fits(128)) return launch_bn<128, EPI>(A, lda, B, e, s, cls);
   if (fits(64)) return launch_bn<64, EPI>(A, lda, B, e, s, cls);

@@ -370,6 +370,19 @@ __device__ __forceinline__ void st_peer_f32x4(uint32_t addr, float a, float b, f
 __device__ __forceinline__ void mbar_arrive_peer(uint32_t addr) {
   asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(addr) : "memory");
 }
+// Asynchronous store of two floats into a peer CTA's shared memory; its 8
+// bytes complete on that CTA's mbarrier at bar_cl (no fence, no arrival).
+__device__ __forceinline__ void st_async_f32x2(uint32_t addr, float a, float b, uint32_t bar_cl) {
+  asm volatile("st.async.shared::cluster.mbarrier::complete_tx::bytes.v2.f32 [%0], {%1, %2}, [%3];" ::"r"(addr),
+               "f"(a), "f"(b), "r"(bar_cl)
+               : "memory");
+}
+// arrive on a barrier of a peer CTA with CTA-scope release: no cluster-wide
+// memory fence, for signals that publish no memory (a TMEM buffer read out,
+// ordered by tcgen05.fence::before_thread_sync)
+__device__ __forceinline__ void mbar_arrive_peer_signal(uint32_t addr) {
+  asm volatile("mbarrier.arrive.shared::cluster.b64 _, [%0];" ::"r"(addr) : "memory");
+}
 __device__ __forceinline__ bool mbar_try_wait_cluster(uint64_t* bar, uint32_t parity) {
   uint32_t ok;
   asm volatile(
