@@ -544,6 +544,342 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   if (threadIdx.x == 0 && *abort_flag) latch_status(e.status, TXS_ERR_DEVICE_TIMEOUT);
 }
 
+// ------------------------------------------------------------------ CTA pairs
+
+// Rows of d = 256 NP columns on clusters of NP CTA pairs (no action head):
+// pair p computes columns [256 p, 256 p + 256) of a 256-row tile with
+// M = 256 MMAs (cta_group::2), issued by its even CTA; CTA 2 p + r holds rows
+// [128 r, 128 r + 128) of the tile in its TMEM (two 256-column buffers).
+// Each CTA stages its 128 activation rows and 128 of its pair's 256 weight
+// rows (32 KB per stage).  The row statistics of a CTA's 256 columns go to
+// the CTA of the other pair that holds the same rows (st.async, counted on
+// its barrier); with NP = 1 the row is whole in one CTA.  The eight epilogue
+// warps form two groups taking alternate tiles, as in the cluster kernel.
+constexpr int PBN = 256;               // columns per CTA (and per pair)
+
+template <int NP>
+struct PairShape {
+  static constexpr int CS = 2 * NP;
+  static constexpr int B_STAGE_BYTES = 128 * BK * 2;                // 16 KB
+  static constexpr int STAGE_BYTES = A_STAGE_BYTES + B_STAGE_BYTES;
+  static constexpr int STG_BYTES = kWarps * 2048;                   // one bulk-store buffer per warp
+  static constexpr int XBUF_BYTES = 2 * NP * 128 * 8;               // (mean, M2) per column block, two parities
+  static constexpr int PAR_BYTES = 3 * PBN * 4;
+  static constexpr int EXTRA = STG_BYTES + XBUF_BYTES + PAR_BYTES + 1024 + 512;
+  static constexpr int STAGES_FIT = (227 * 1024 - EXTRA) / STAGE_BYTES;
+  static constexpr int STAGES = STAGES_FIT > 8 ? 8 : STAGES_FIT;
+  static constexpr int SMEM_BYTES = STAGES * STAGE_BYTES + EXTRA;
+  static constexpr int TMEM_COLS = 2 * PBN;
+  static_assert(STAGES >= 4 && SMEM_BYTES <= 232448, "shared memory");
+};
+
+template <int NP>
+__global__ void __launch_bounds__(NUM_THREADS, 1)
+    gemm_ln_pair_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                        const __grid_constant__ CUtensorMap tmO, const EpiArgs e) {
+  using S = PairShape<NP>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint8_t* sA = smem;
+  uint8_t* sB = sA + S::STAGES * A_STAGE_BYTES;
+  uint8_t* s_stage = sB + S::STAGES * S::B_STAGE_BYTES;
+  float2* xbuf = reinterpret_cast<float2*>(s_stage + S::STG_BYTES);                 // [2][NP][128]
+  float* s_par = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(xbuf) + S::XBUF_BYTES);   // [3][PBN]
+  uint64_t* full = reinterpret_cast<uint64_t*>(reinterpret_cast<uint8_t*>(s_par) + S::PAR_BYTES);
+  uint64_t* empty = full + S::STAGES;
+  uint64_t* acc_full = empty + S::STAGES;
+  uint64_t* acc_empty = acc_full + 2;
+  uint64_t* xfull = acc_empty + 2;    // [2][4]: the other pair's statistics of lane quarter q
+  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(xfull + 8);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_holder + 1);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint32_t rk = cluster_rank();
+  const int pr = static_cast<int>(rk) >> 1, half = static_cast<int>(rk) & 1;
+  const uint32_t lead_rank = rk & ~1u;
+  const uint16_t pair_mask = static_cast<uint16_t>(3u << (2 * pr));
+  const int cid = blockIdx.x / S::CS, ncl = gridDim.x / S::CS;
+  const int m_tiles = (e.M + 2 * BM - 1) / (2 * BM);
+  const int my_tiles = m_tiles > cid ? (m_tiles - 1 - cid) / ncl + 1 : 0;   // equal within a cluster
+  const int n0 = pr * PBN;                      // this pair's columns
+  const int nb0 = n0 + half * 128;              // this CTA's weight rows
+  const int num_kb = e.K / BK;
+  constexpr uint32_t kFullBytes = 2 * S::STAGE_BYTES;   // both CTAs' loads, on the even CTA's barrier
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < S::STAGES; ++s) {
+      mbar_init(full + s, 1);
+      mbar_init(empty + s, 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(acc_full + b, 1);
+      mbar_init(acc_empty + b, 2 * kGroupWarps);     // the even CTA's: both CTAs' group
+    }
+    for (int i = 0; i < 8; ++i) mbar_init(xfull + i, 1);
+    *abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == 1) tmem_alloc_pair(tmem_holder, S::TMEM_COLS);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_holder;
+  cluster_sync();                     // every CTA's barriers exist before any peer signals them
+  pdl_launch_dependents();
+  auto lead = [&](uint64_t* bar) { return map_peer(bar, lead_rank); };
+  const int n_pre = my_tiles > 0 ? (num_kb < S::STAGES ? num_kb : S::STAGES) : 0;
+  if (warp == 0 && lane == 0) {
+    for (int kb = 0; kb < n_pre; ++kb) {   // weights: not written by the preceding kernels
+      if (half == 0) mbar_expect_tx(full + kb, kFullBytes);
+      tma_load_2d_pair(sB + kb * S::B_STAGE_BYTES, &tmB, lead(full + kb), kb * BK, nb0);
+    }
+  }
+  pdl_wait();
+  for (int i = threadIdx.x; i < PBN; i += NUM_THREADS) {
+    s_par[i] = e.bias[n0 + i];
+    s_par[PBN + i] = e.gamma[n0 + i];
+    s_par[2 * PBN + i] = e.beta[n0 + i];
+  }
+  __syncthreads();
+
+  if (warp == 0) {
+    if (lane == 0) {
+      asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmA)) : "memory");
+      asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmB)) : "memory");
+      int it = 0;
+      bool ok = true;
+      for (int i = 0; i < my_tiles && ok; ++i) {
+        const int a_rows = (cid + i * ncl) * 2 * BM + half * BM;
+        for (int kb = 0; kb < num_kb; ++kb, ++it) {
+          const int s = it % S::STAGES;
+          if (it < n_pre) {     // weights in flight since before the wait
+            tma_load_2d_pair(sA + s * A_STAGE_BYTES, &tmA, lead(full + s), kb * BK, a_rows);
+            continue;
+          }
+          if (!mbar_wait(empty + s, ((it / S::STAGES) & 1) ^ 1, abort_flag)) {
+            ok = false;
+            break;
+          }
+          if (half == 0) mbar_expect_tx(full + s, kFullBytes);
+          tma_load_2d_pair(sA + s * A_STAGE_BYTES, &tmA, lead(full + s), kb * BK, a_rows);
+          tma_load_2d_pair(sB + s * S::B_STAGE_BYTES, &tmB, lead(full + s), kb * BK, nb0);
+        }
+      }
+      // the pair's MMAs release this CTA's stages by multicast commits: take
+      // the last ones before the CTA may exit
+      for (int k = it > S::STAGES ? it - S::STAGES : 0; k < it && !*abort_flag; ++k)
+        mbar_wait(empty + k % S::STAGES, (k / S::STAGES) & 1, abort_flag);
+      if (*abort_flag && half == 0)
+        for (int k = it > S::STAGES ? it - S::STAGES : 0; k < it; ++k)
+          mbar_wait_plain(full + k % S::STAGES, (k / S::STAGES) & 1);
+    }
+  } else if (warp == 1) {
+    if (lane == 0 && half == 0) {
+      constexpr uint32_t idesc = idesc_bf16(2 * BM, PBN);
+      int it = 0;
+      bool ok = true;
+      for (int i = 0; i < my_tiles && ok; ++i) {
+        const int buf = i & 1;
+        if (!mbar_wait(acc_empty + buf, ((i >> 1) & 1) ^ 1, abort_flag)) break;
+        tc_fence_after();
+        for (int kb = 0; kb < num_kb; ++kb, ++it) {
+          const int s = it % S::STAGES;
+          if (!mbar_wait(full + s, (it / S::STAGES) & 1, abort_flag)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint64_t adesc = sdesc_sw128(smem_u32(sA + s * A_STAGE_BYTES));
+          const uint64_t bdesc = sdesc_sw128(smem_u32(sB + s * S::B_STAGE_BYTES));
+#pragma unroll
+          for (int k = 0; k < BK / 16; ++k)
+            mma_bf16_pair(tmem + buf * PBN, adesc + 2 * k, bdesc + 2 * k, idesc, (kb > 0 || k > 0) ? 1u : 0u);
+          mma_commit_pair(empty + s, pair_mask);
+        }
+        mma_commit_pair(acc_full + buf, pair_mask);   // also on abort: the epilogues wait on every issued MMA
+      }
+    }
+  } else {
+    const int ew = warp - 2;
+    const int grp = ew / kGroupWarps;  // tiles i with i % 2 == grp, TMEM buffer grp
+    const int q = warp & 3;            // TMEM lane quarter
+    const int trow = q * 32 + lane;
+    uint8_t* stage = s_stage + ew * 2048;
+    const float* s_bias = s_par;
+    const float* s_gamma = s_par + PBN;
+    const float* s_beta = s_par + 2 * PBN;
+    int kchunk = 0;
+    float v[32];
+    for (int i = grp; i < my_tiles; i += 2) {
+      const int buf = grp, pb = grp;
+      const uint32_t use = static_cast<uint32_t>(i >> 1) & 1;
+      const int m0 = (cid + i * ncl) * 2 * BM + half * BM;   // this CTA's rows
+      const int row = m0 + trow;
+      const bool valid = row < e.M;
+      // the residual's first 64 columns are fetched before the wait, the rest
+      // one chunk ahead
+      const uint4* rp = reinterpret_cast<const uint4*>(static_cast<const __nv_bfloat16*>(e.res) +
+                                                       static_cast<long long>(valid ? row : 0) * e.ldr + n0);
+      uint4 rres[8];
+#pragma unroll
+      for (int k = 0; k < 8; ++k) rres[k] = valid ? __ldg(rp + k) : make_uint4(0, 0, 0, 0);
+      bool go = mbar_wait(acc_full + buf, use, abort_flag);
+      go = __shfl_sync(0xffffffffu, go ? 1 : 0, 0) != 0;
+      if (!go) break;
+      tc_fence_after();
+      const uint32_t tacc = tmem + buf * PBN + (static_cast<uint32_t>(q * 32) << 16);
+      // pass 1: v = acc + bias + residual, written back to TMEM; per chunk of
+      // 32 columns its mean and squared deviations, merged pairwise
+      float mean_p = 0.f, m2 = 0.f;
+      // 64 columns per iteration: chunk h of 32 uses residual registers
+      // rres[4 h .. 4 h + 3] (static indices), then refills them for c + 64
+#pragma unroll 1
+      for (int c64 = 0; c64 < PBN; c64 += 64) {
+#pragma unroll
+        for (int hh = 0; hh < 2; ++hh) {
+          const int c = c64 + 32 * hh;
+          tmem_ld32(tacc + c, v);
+          float sum = 0.f;
+#pragma unroll
+          for (int k = 0; k < 4; ++k) {
+            const __nv_bfloat162* h2 = reinterpret_cast<const __nv_bfloat162*>(&rres[4 * hh + k]);
+#pragma unroll
+            for (int t = 0; t < 4; ++t) {
+              const float2 f = __bfloat1622float2(h2[t]);
+              const int j = 8 * k + 2 * t;
+              v[j] += s_bias[c + j] + f.x;
+              v[j + 1] += s_bias[c + j + 1] + f.y;
+              sum += v[j] + v[j + 1];
+            }
+          }
+          if (c + 64 < PBN) {
+#pragma unroll
+            for (int k = 0; k < 4; ++k)
+              rres[4 * hh + k] = valid ? __ldg(rp + (c + 64) / 8 + k) : make_uint4(0, 0, 0, 0);
+          }
+          const float mc = sum * (1.f / 32.f);
+          float m2c = 0.f;
+#pragma unroll
+          for (int k = 0; k < 32; ++k) {
+            const float t = v[k] - mc;
+            m2c = fmaf(t, t, m2c);
+          }
+          tmem_st32(tacc + c, v);
+          if (c == 0) {
+            mean_p = mc;
+            m2 = m2c;
+          } else {
+            const float na = static_cast<float>(c), nt = na + 32.f;
+            const float dlt = mc - mean_p;
+            mean_p = fmaf(dlt, 32.f / nt, mean_p);
+            m2 = m2 + m2c + dlt * dlt * (na * 32.f / nt);
+          }
+        }
+      }
+      float mean = mean_p;
+      if constexpr (NP > 1) {
+        // (mean, M2) of these 256 columns to the CTAs of the other pairs that
+        // hold the same rows; this CTA's own slot by a plain store
+        float2* mine = xbuf + (pb * NP + pr) * 128 + trow;
+        *mine = make_float2(mean_p, m2);
+#pragma unroll
+        for (int o = 0; o < NP; ++o)
+          if (o != pr) {
+            const uint32_t peer = static_cast<uint32_t>(2 * o + half);
+            st_async_f32x2(map_peer(mine, peer), mean_p, m2, map_peer(xfull + pb * 4 + q, peer));
+          }
+        if (lane == 0) mbar_expect_tx(xfull + pb * 4 + q, (NP - 1) * 32 * 8);
+        bool ok = mbar_wait_cluster(xfull + pb * 4 + q, use, abort_flag);
+        ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
+        if (!ok) break;
+        float mp[NP];
+        mean = 0.f;
+#pragma unroll
+        for (int o = 0; o < NP; ++o) {
+          const float2 x = xbuf[(pb * NP + o) * 128 + trow];
+          mp[o] = x.x;
+          mean += x.x;
+          m2 = o == 0 ? x.y : m2 + x.y;
+        }
+        mean *= 1.f / NP;
+#pragma unroll
+        for (int o = 0; o < NP; ++o) {
+          const float t = mp[o] - mean;
+          m2 = fmaf(static_cast<float>(PBN) * t, t, m2);
+        }
+      }
+      const float rstd = rsqrtf(m2 / static_cast<float>(PBN * NP) + e.ln_eps);
+      // pass 2: normalise and store
+#pragma unroll 1
+      for (int c = 0; c < PBN; c += 32) {
+        tmem_ld32(tacc + c, v);
+#pragma unroll
+        for (int k = 0; k < 32; ++k) v[k] = (v[k] - mean) * rstd * s_gamma[c + k] + s_beta[c + k];
+        __nv_bfloat16* out =
+            valid ? static_cast<__nv_bfloat16*>(e.out) + static_cast<long long>(row) * e.ldo + n0 + c : nullptr;
+        store_chunk<1>(v, out, valid, true, &tmO, n0 + c, m0 + q * 32, stage, kchunk++, lane);
+      }
+      // every read of this accumulator is done: release it on the even CTA
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive_peer_signal(lead(acc_empty + buf));
+    }
+    if (lane == 0) bulk_wait_all();
+  }
+  tc_fence_before();
+  __syncthreads();
+  cluster_sync();                     // no CTA leaves while a peer may still signal or write into it
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc_pair(tmem, S::TMEM_COLS);
+  }
+  if (threadIdx.x == 0 && *abort_flag) latch_status(e.status, TXS_ERR_DEVICE_TIMEOUT);
+}
+
+template <int NP>
+static cudaError_t launch_pair(const __nv_bfloat16* A, long long lda, const __nv_bfloat16* B, const EpiArgs& e,
+                               cudaStream_t s, int cls) {
+  using Sh = PairShape<NP>;
+  auto kern = gemm_ln_pair_kernel<NP>;
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = Sh::CS;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
+  cudaLaunchConfig_t cfg = {};
+  cfg.blockDim = dim3(NUM_THREADS);
+  cfg.dynamicSmemBytes = Sh::SMEM_BYTES;
+  cfg.stream = s;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  static int max_clusters = 0;
+  if (!max_clusters) {
+    cudaError_t err = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, Sh::SMEM_BYTES);
+    if (err != cudaSuccess) return err;
+    cfg.gridDim = dim3((num_sms() / Sh::CS) * Sh::CS);
+    int n = 0;
+    if (cudaOccupancyMaxActiveClusters(&n, kern, &cfg) != cudaSuccess || n <= 0) {
+      (void)cudaGetLastError();
+      n = num_sms() / Sh::CS;
+    }
+    max_clusters = n;
+  }
+  CUtensorMap ta, tb, to;
+  if (!make_tmap(&ta, A, e.M, e.K, lda, BM)) return cudaErrorInvalidValue;
+  if (!make_tmap(&tb, B, e.N, e.K, e.K, 128)) return cudaErrorInvalidValue;
+  if (!make_tmap_out(&to, e.out, e.M, e.N, e.ldo)) return cudaErrorInvalidValue;
+  const int m_tiles = (e.M + 2 * BM - 1) / (2 * BM);
+  const int ncl = m_tiles < max_clusters ? m_tiles : max_clusters;
+  cfg.gridDim = dim3(ncl * Sh::CS);
+  cfg.numAttrs = 2;
+  prof_begin(cls, s);
+  cudaError_t err = cudaLaunchKernelEx(&cfg, kern, ta, tb, to, e);
+  prof_end(cls, s);
+  return err;
+}
+
 template <int CS, bool HEAD, bool PING>
 static cudaError_t launch_cs(const __nv_bfloat16* A, long long lda, const __nv_bfloat16* B, const EpiArgs& e,
                              cudaStream_t s, int cls) {
@@ -600,6 +936,12 @@ cudaError_t launch_gemm_ln_cluster(const __nv_bfloat16* A, long long lda, const 
   if (e.epi == EPI_LN_HEAD && (e.n_act < 1 || e.n_act > 4)) return cudaErrorNotSupported;
   if (e.epi != EPI_LN && e.epi != EPI_LN_HEAD) return cudaErrorNotSupported;
   const bool head = e.epi == EPI_LN_HEAD;
+  // CTA pairs (256 columns per CTA) once every cluster gets two 256-row tiles
+  if (!head && (e.N == 256 || e.N == 512)) {
+    const int ncs = e.N / 128;   // CTAs per cluster either way
+    if ((e.M + 2 * tc::BM - 1) / (2 * tc::BM) >= 2 * (num_sms() / ncs))
+      return e.N == 256 ? tcln::launch_pair<1>(A, lda, B, e, s, cls) : tcln::launch_pair<2>(A, lda, B, e, s, cls);
+  }
   // the two epilogue groups pay off once each cluster has several row tiles
   const int m_tiles = (e.M + tc::BM - 1) / tc::BM;
   const bool ping = m_tiles >= 4 * (num_sms() / (e.N / tcln::BN));
