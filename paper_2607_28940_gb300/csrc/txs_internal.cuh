@@ -121,29 +121,48 @@ __device__ __forceinline__ float2 fadd2(float2 a, float2 b) {
   return o;
 }
 
-// gelu_erf (above the f32x2 helpers) with erf from the rational approximation of Abramowitz &
-// Stegun, Handbook of Mathematical Functions (1964), formula 7.1.26:
-// erf(z) = 1 - t (a1 + t (a2 + t (a3 + t (a4 + t a5)))) exp(-z^2),
-// t = 1 / (1 + p z) for z >= 0, odd in z; the approximation's absolute error
-// is at most 1.5e-7, and with fp32 arithmetic and the hardware exp2 and
-// reciprocal the result stays within a few 1e-7 of erf, against bf16
-// outputs with a relative step of 2^-8.  The bf16 tensor-core epilogues use
-// it (fewer instructions per output element than erff), on two values at
-// once: the multiplies and multiply-adds run as f32x2 instructions.
+// Hardware approximations (PTX): reciprocal and 2^x, subnormal results
+// flushed to zero.
+__device__ __forceinline__ float rcp_approx(float x) {
+  float r;
+  asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(r) : "f"(x));
+  return r;
+}
+__device__ __forceinline__ float ex2_approx(float x) {
+  float r;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(r) : "f"(x));
+  return r;
+}
+
+// gelu_erf (above the f32x2 helpers) with erf from the rational approximation
+// of Abramowitz & Stegun, Handbook of Mathematical Functions (1964), formula
+// 7.1.26: for z >= 0, 1 - erf(z) = t P(t) exp(-z^2) with t = 1 / (1 + p z),
+// P(t) = a1 + t (a2 + t (a3 + t (a4 + t a5))), absolute error at most 1.5e-7.
+// Since erf is odd, with a = |x| and z = a / sqrt 2 both signs reduce to
+//   GELU(x) = 0.5 x (1 + erf(x / sqrt 2)) = max(x, 0) - 0.5 a t P(t) exp(-a^2 / 2),
+// which needs no sign handling and never forms 1 - (1 - small).  The bf16
+// tensor-core epilogues use it on two values at once (f32x2 multiplies and
+// multiply-adds; the 0.5 and 1 / sqrt 2 are folded into the constants), with
+// the hardware reciprocal and 2^x; in fp32 the result stays within a few
+// 1e-7 of 0.5 |x| of the exact GELU, against bf16 outputs with a relative
+// step of 2^-8.
 __device__ __forceinline__ float2 gelu_erf_as2(float2 x) {
-  const float2 z = fmul2(make_float2(fabsf(x.x), fabsf(x.y)), make_float2(0.70710678118654752f, 0.70710678118654752f));
-  const float2 den = ffma2(make_float2(0.3275911f, 0.3275911f), z, make_float2(1.0f, 1.0f));
-  const float2 t = make_float2(__fdividef(1.0f, den.x), __fdividef(1.0f, den.y));
-  float2 q = ffma2(t, make_float2(1.061405429f, 1.061405429f), make_float2(-1.453152027f, -1.453152027f));
-  q = ffma2(t, q, make_float2(1.421413741f, 1.421413741f));
-  q = ffma2(t, q, make_float2(-0.284496736f, -0.284496736f));
-  q = ffma2(t, q, make_float2(0.254829592f, 0.254829592f));
-  const float2 poly = fmul2(t, q);
-  const float2 zz = fmul2(fmul2(make_float2(-z.x, -z.y), z), make_float2(1.4426950408889634f, 1.4426950408889634f));
-  const float2 e = make_float2(exp2f(zz.x), exp2f(zz.y));
-  const float2 ea = ffma2(make_float2(-poly.x, -poly.y), e, make_float2(1.0f, 1.0f));
-  const float2 onep = make_float2(1.0f + copysignf(ea.x, x.x), 1.0f + copysignf(ea.y, x.y));
-  return fmul2(fmul2(make_float2(0.5f, 0.5f), x), onep);
+  const float2 a = make_float2(fabsf(x.x), fabsf(x.y));
+  constexpr float kP = 0.3275911f * 0.70710678118654752f;        // p / sqrt 2
+  const float2 den = ffma2(a, make_float2(kP, kP), make_float2(1.0f, 1.0f));
+  const float2 t = make_float2(rcp_approx(den.x), rcp_approx(den.y));
+  // 0.5 P(t)
+  float2 q = ffma2(t, make_float2(0.5f * 1.061405429f, 0.5f * 1.061405429f),
+                   make_float2(0.5f * -1.453152027f, 0.5f * -1.453152027f));
+  q = ffma2(t, q, make_float2(0.5f * 1.421413741f, 0.5f * 1.421413741f));
+  q = ffma2(t, q, make_float2(0.5f * -0.284496736f, 0.5f * -0.284496736f));
+  q = ffma2(t, q, make_float2(0.5f * 0.254829592f, 0.5f * 0.254829592f));
+  // exp(-a^2 / 2) = 2^(-a^2 log2(e) / 2)
+  constexpr float kE = -0.5f * 1.4426950408889634f;
+  const float2 zz = fmul2(a, fmul2(a, make_float2(kE, kE)));
+  const float2 e = make_float2(ex2_approx(zz.x), ex2_approx(zz.y));
+  const float2 g = fmul2(fmul2(fmul2(a, t), q), e);
+  return fadd2(make_float2(fmaxf(x.x, 0.0f), fmaxf(x.y, 0.0f)), make_float2(-g.x, -g.y));
 }
 
 // Index of the segment that contains `row` in an exclusive-offset array
