@@ -8,8 +8,8 @@ reading the wrong keys moves the scores by less than the bf16 tolerances
 power-of-two gains (exact in bf16) to the attention projections, the
 cross-attention output, the head and the pooling vector.
 
-Each case below plants one error of the kind a cross-attention kernel can
-make into a copy of the oracle (a patched function, on the CPU; no kernel is
+Each case below plants one error of the kind a cross-attention or serving-
+stream attention kernel can make into a copy of the oracle (a patched function, on the CPU; no kernel is
 touched) and checks that, at the sharp weights and the shapes of the small
 (d = 256, d_h = 32) and mid (d = 512, d_h = 64) workloads, the scores move by
 more than the bf16 tolerances.  A GPU parity test at these weights therefore
@@ -72,7 +72,37 @@ def _next_kv_head(q, k, v, n_heads, allowed=None, n_kv_heads=None):
     return _attention(q, np.roll(k, -dh, axis=1), np.roll(v, -dh, axis=1), n_heads, allowed, n_kv_heads)
 
 
+_serving_mask = O.serving_mask
+
+
+def _serving_self_dropped(n_ctx, n_cand):
+    # a candidate sees the context rows but not itself
+    m = _serving_mask(n_ctx, n_cand)
+    m[np.arange(n_ctx, n_ctx + n_cand), np.arange(n_ctx, n_ctx + n_cand)] = False
+    return m
+
+
+def _serving_last_context_row_dropped(n_ctx, n_cand):
+    m = _serving_mask(n_ctx, n_cand)
+    if n_ctx > 1:
+        m[n_ctx:, n_ctx - 1] = False
+    return m
+
+
+def _serving_context_rows_of_other_request(n_ctx, n_cand):
+    # a candidate reads the context keys at the wrong rows: its own row and
+    # the next candidate instead of the context rows
+    m = _serving_mask(n_ctx, n_cand)
+    rows = np.arange(n_ctx, n_ctx + n_cand)
+    m[rows, :n_ctx] = False
+    m[rows, n_ctx + (rows - n_ctx + 1) % n_cand] = True
+    return m
+
+
 SLIPS = {
+    "serving_self_key_dropped": ("serving_mask", _serving_self_dropped, O.LOCAL_GLOBAL),
+    "serving_last_context_row_dropped": ("serving_mask", _serving_last_context_row_dropped, O.LOCAL_GLOBAL),
+    "serving_wrong_context_keys": ("serving_mask", _serving_context_rows_of_other_request, O.LOCAL_GLOBAL),
     "full_last_key_tile_dropped": ("key_set", _full_last_tile_dropped, O.FULL),
     "full_half_of_keys_dropped": ("key_set", _full_second_half_dropped, O.FULL),
     "full_query_head_reads_next_kv_head": ("attention", _next_kv_head, O.FULL),
