@@ -54,6 +54,9 @@ constexpr int kStageSeg = 1024;   // request offsets staged in shared memory (ca
 
 
 constexpr int kStageNAtt = 512;   // bias entries staged with the fused attention (N = d <= 512)
+constexpr int kStageNSrv = 1536;  // bias entries staged with the fused serving attention (N = 3 d <= 1536)
+constexpr int kSrvMaxS = 8;       // context rows per request the fused serving attention takes
+constexpr int kSrvSlots = kSrvMaxS + 1;
 
 // Fused LOCAL_GLOBAL cross-attention (EPI_ATTN_LG): each epilogue warp owns
 // 64 query columns (one head of 64 or two of 32) of 32 rows.  Per request
@@ -637,6 +640,108 @@ __device__ __forceinline__ void attn_epilogue_warp(const EpiArgs& e, uint32_t tm
   if (lane == 0) bulk_wait_all();
 }
 
+// ------------------------------------------------------------------ fused serving attention
+
+// Serving-stream attention of one head for the 32 rows of one warp
+// (EPI_SERVE; App. B mask): a candidate row attends to the S context rows of
+// its request and to itself.  The tile's accumulator holds q | k | v of the
+// head (DH columns each; bias in `bias` at the tile's columns n0 ..); this
+// warp takes dims [32 h2, 32 h2 + 32) of each.  The two warps of a lane
+// quarter add their partial scores through `red` (slots per row: S context
+// keys and the row's own key; `par` alternates the buffer by tile), then
+// each forms its 32 output dims: the softmax-weighted context values (bf16,
+// from srv_ctx) and the row's own value.
+template <int DH>
+__device__ __forceinline__ void serve_tile(const EpiArgs& e, uint32_t tacc, int m0, int n0, int head, int h2, int q,
+                                           int lane, int par, int r, const float* bias, float* red,
+                                           const CUtensorMap* tmO, uint8_t* stage, int& kchunk) {
+  const int trow = q * 32 + lane;
+  const int row = m0 + trow;
+  const bool valid = row < e.M;
+  const int S = e.srv_S, d = e.srv_d;
+  const int col = 32 * h2;
+  const long long ld = 3LL * d;
+  const __nv_bfloat16* ctx = static_cast<const __nv_bfloat16*>(e.srv_ctx) + static_cast<long long>(r) * S * ld +
+                             head * DH + col;   // q of context row 0; k at + d, v at + 2 d
+  float qv[32], kv[32];
+  tmem_ld32x2(tacc + col, tacc + DH + col, qv, kv);
+  float self = 0.f;
+#pragma unroll
+  for (int i = 0; i < 32; ++i) {
+    qv[i] += bias[n0 + col + i];
+    kv[i] += bias[n0 + DH + col + i];
+    self = fmaf(qv[i], kv[i], self);
+  }
+  float part[kSrvSlots];
+#pragma unroll
+  for (int t = 0; t < kSrvMaxS; ++t) {
+    part[t] = 0.f;
+    if (t < S) {
+      float kc[32];
+      load_bf16x32(ctx + t * ld + d, kc);
+#pragma unroll
+      for (int i = 0; i < 32; ++i) part[t] = fmaf(qv[i], kc[i], part[t]);
+    }
+  }
+  part[kSrvMaxS] = self;
+  float* mine = red + ((par * 2 + h2) * 128 + trow) * kSrvSlots;
+  const float* other = red + ((par * 2 + (1 - h2)) * 128 + trow) * kSrvSlots;
+#pragma unroll
+  for (int t = 0; t < kSrvSlots; ++t) mine[t] = part[t];
+  named_bar(1 + q, 64);
+  float mx = -INFINITY;
+#pragma unroll
+  for (int t = 0; t < kSrvSlots; ++t) {
+    part[t] = (part[t] + other[t]) * e.srv_scale_log2;   // log2-domain scores
+    if (t < S || t == kSrvMaxS) mx = fmaxf(mx, part[t]);
+  }
+  float sum = 0.f;
+#pragma unroll
+  for (int t = 0; t < kSrvSlots; ++t) {
+    part[t] = (t < S || t == kSrvMaxS) ? ex2_approx(part[t] - mx) : 0.f;
+    sum += part[t];
+  }
+  const float inv = 1.f / sum;
+  float o[32];
+  tmem_ld32(tacc + 2 * DH + col, o);
+#pragma unroll
+  for (int i = 0; i < 32; ++i) o[i] = (o[i] + bias[n0 + 2 * DH + col + i]) * part[kSrvMaxS];
+#pragma unroll
+  for (int t = 0; t < kSrvMaxS; ++t) {
+    if (t < S) {
+      float vc[32];
+      load_bf16x32(ctx + t * ld + 2 * d, vc);
+#pragma unroll
+      for (int i = 0; i < 32; ++i) o[i] = fmaf(part[t], vc[i], o[i]);
+    }
+  }
+#pragma unroll
+  for (int i = 0; i < 32; ++i) o[i] *= inv;
+  __nv_bfloat16* out =
+      valid ? static_cast<__nv_bfloat16*>(e.out) + static_cast<long long>(row) * e.ldo + head * DH + col : nullptr;
+  store_chunk<1>(o, out, valid, true, tmO, head * DH + col, m0 + q * 32, stage, kchunk++, lane);
+}
+
+// Request of this lane's row of the tile at rows m0.. (0 past M).
+__device__ __forceinline__ int serve_req(const EpiArgs& e, int m0, int q, int lane) {
+  const int row = m0 + q * 32 + lane;
+  return row < e.M ? __ldg(e.srv_row_req + row) : 0;
+}
+
+// L1 prefetch of the context keys and values of request r that serve_tile
+// reads (head `head`, dims [32 h2, 32 h2 + 32)).
+template <int DH>
+__device__ __forceinline__ void serve_prefetch(const EpiArgs& e, int r, int head, int h2) {
+  const int S = e.srv_S, d = e.srv_d;
+  const long long ld = 3LL * d;
+  const __nv_bfloat16* ctx =
+      static_cast<const __nv_bfloat16*>(e.srv_ctx) + static_cast<long long>(r) * S * ld + head * DH + 32 * h2;
+  for (int t = 0; t < S; ++t) {
+    prefetch_l1(ctx + t * ld + d);
+    prefetch_l1(ctx + t * ld + 2 * d);
+  }
+}
+
 // ------------------------------------------------------------------ kernel
 
 // BRES: the CTA's whole B slice (BN x K, K <= KRES) stays resident in shared
@@ -648,6 +753,7 @@ __device__ __forceinline__ void attn_epilogue_warp(const EpiArgs& e, uint32_t tm
 template <int BN, int EPI, int NAP = 4, bool BRES = false, bool PAIR = false>
 struct Shape {
   static constexpr int BN_MMA = BN < 256 ? BN : 256;     // N of one tcgen05.mma
+  static constexpr bool SERVE = EPI == EPI_SERVE;
   static constexpr int B_ROWS = PAIR ? BN / 2 : BN;       // rows of B this CTA stages
   static constexpr int B_BOX = PAIR ? B_ROWS : BN_MMA;    // rows of one TMA box of B
   static constexpr int TM = PAIR ? 2 * BM : BM;           // rows of a tile
@@ -656,7 +762,7 @@ struct Shape {
   static constexpr int B_STAGE_BYTES = BRES ? 0 : B_ROWS * BK * 2;
   static constexpr int STAGE_BYTES = A_STAGE_BYTES + B_STAGE_BYTES;
   static constexpr bool LN = EPI == EPI_LN || EPI == EPI_LN_HEAD;
-  static constexpr int RED_BYTES = LN ? 2 * 128 * kRedStride * 4 : 0;
+  static constexpr int RED_BYTES = LN ? 2 * 128 * kRedStride * 4 : SERVE ? 2 * 2 * 128 * kSrvSlots * 4 : 0;
   static constexpr int WEFF_BYTES = EPI == EPI_LN_HEAD ? BN * NAP * 4 : 0;
   // bias [kStageN] floats ([kStageNRes] with BRES), then (cache-row remap) offsets and
   // first rows; rounded to 1 KB so that the staging buffers after it start on
@@ -666,8 +772,8 @@ struct Shape {
   // projections at d = 512): one bulk-store staging buffer per warp and the
   // bias read through L1 leave room for a fourth operand stage
   static constexpr bool LEAN = !BRES && !LN && !ATT && BN == 256;
-  static constexpr int SBUF = LEAN ? 1 : 2;               // bulk-store staging buffers per warp
-  static constexpr int STAGE_N = BRES ? kStageNRes : (ATT || LEAN) ? kStageNAtt : kStageN;
+  static constexpr int SBUF = (LEAN || SERVE) ? 1 : 2;    // bulk-store staging buffers per warp
+  static constexpr int STAGE_N = BRES ? kStageNRes : SERVE ? kStageNSrv : (ATT || LEAN) ? kStageNAtt : kStageN;
   static constexpr int AUX_BYTES =
       LN ? 0 : (((STAGE_N * 4) + (EPI == EPI_KV ? (2 * kStageSeg + 1) * 4 : 0) + 1023) / 1024) * 1024;
   // fused attention: each epilogue warp's staged window and anchor (fp32)
@@ -678,7 +784,9 @@ struct Shape {
   static constexpr int STAGES_FIT = (227 * 1024 - EXTRA) / STAGE_BYTES;
   static constexpr int STAGES = STAGES_FIT > 8 ? 8 : STAGES_FIT;
   static constexpr int ACC_BUFS = BN <= 256 ? 2 : 1;      // TMEM double buffer
-  static constexpr int TMEM_COLS = BN * ACC_BUFS < 32 ? 32 : BN * ACC_BUFS;
+  static constexpr int TMEM_USED = BN * ACC_BUFS;
+  static constexpr int TMEM_COLS = TMEM_USED <= 32 ? 32 : TMEM_USED <= 64 ? 64 : TMEM_USED <= 128 ? 128
+                                   : TMEM_USED <= 256 ? 256 : 512;   // a power of two
   static constexpr int SMEM_BYTES = STAGES * STAGE_BYTES + EXTRA;
   static_assert(STAGES >= 2, "pipeline depth");
   static_assert(!(BRES && LN), "resident B only for the plain epilogues");
@@ -687,7 +795,8 @@ struct Shape {
   static_assert((RED_BYTES + WEFF_BYTES + AUX_BYTES + STG_BYTES + ATT_BYTES) % 16 == 0,
                 "mbarriers must stay 8-byte aligned");
   static_assert(!ATT || (BN == 2 * kAttCols && !BRES), "fused attention: 128-column tiles");
-  static_assert(!PAIR || (LEAN && BN == 256), "CTA pairs: 256-column streaming tiles");
+  static_assert(!PAIR || (LEAN && BN == 256) || (SERVE && BN == 192), "CTA pairs: 256-column streaming tiles");
+  static_assert(!SERVE || PAIR, "fused serving attention: CTA pairs");
   static_assert(SMEM_BYTES <= 232448, "shared memory");
   static_assert((TMEM_COLS & (TMEM_COLS - 1)) == 0 && TMEM_COLS <= 512, "TMEM columns");
 };
@@ -984,6 +1093,35 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     if constexpr (S::ATT) {
       attn_epilogue_warp(e, tmem + (static_cast<uint32_t>(q * 32) << 16), acc_full, acc_empty, abort_flag, t_lo,
                          t_hi, t_step, n_tiles, m_tiles, q, h, bias, &tmO, stage, s_att + ew * kAttWarpBytes);
+    } else if constexpr (S::SERVE) {
+      int kchunk = 0;
+      int i = 0;
+      // Each tile's row requests are read two tiles ahead and its context
+      // rows prefetched into L1 one tile ahead, so no tile waits on a chain
+      // of dependent global loads.
+      auto rows_of = [&](int t) { return tile_m(t) * S::TM + static_cast<int>(rank) * BM; };
+      int r_cur = t_lo < t_hi ? serve_req(e, rows_of(t_lo), q, lane) : 0;
+      int r_next = t_lo + t_step < t_hi ? serve_req(e, rows_of(t_lo + t_step), q, lane) : 0;
+      if (t_lo < t_hi) serve_prefetch<BN / 3>(e, r_cur, tile_n(t_lo), h);
+      for (int t = t_lo; t < t_hi; t += t_step, ++i) {
+        const int buf = i % S::ACC_BUFS;
+        const uint32_t use = i / S::ACC_BUFS;
+        const int r = r_cur;
+        r_cur = r_next;
+        r_next = t + 2 * t_step < t_hi ? serve_req(e, rows_of(t + 2 * t_step), q, lane) : 0;
+        if (t + t_step < t_hi) serve_prefetch<BN / 3>(e, r_cur, tile_n(t + t_step), h);
+        bool go = mbar_wait(acc_full + buf, use & 1, abort_flag);
+        go = __shfl_sync(0xffffffffu, go ? 1 : 0, 0) != 0;
+        if (!go) break;
+        tc_fence_after();
+        const int m0 = rows_of(t), hd = tile_n(t);
+        serve_tile<BN / 3>(e, tmem + buf * BN + (static_cast<uint32_t>(q * 32) << 16), m0, hd * BN, hd, h, q, lane,
+                           i & 1, r, bias, red, &tmO, stage, kchunk);
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive_peer_signal(lead(acc_empty + buf));
+      }
+      if (lane == 0) bulk_wait_all();
     } else {
       int kchunk = 0;
       int i = 0;
@@ -1149,6 +1287,8 @@ static cudaError_t launch_bn(const __nv_bfloat16* A, long long lda, const __nv_b
     // the cache viewed as [(N / col_blk) * cap_total rows, col_blk] bf16
     const long long rows = static_cast<long long>(e.N / e.col_blk) * (e.col_blk_stride / e.col_blk);
     if (!make_tmap_out(&to, e.out, rows, e.col_blk, e.ldo)) return cudaErrorInvalidValue;
+  } else if (EPI == EPI_SERVE) {
+    if (!make_tmap_out(&to, e.out, e.M, e.N / 3, e.ldo)) return cudaErrorInvalidValue;   // one head's d_h per tile
   } else {
     if (!make_tmap_out(&to, e.out, e.M, e.N, e.ldo)) return cudaErrorInvalidValue;
   }
@@ -1194,6 +1334,7 @@ bool tc_gemm_supported(int N, int K, int epi) {
   if (K <= 0 || K % BK != 0 || N <= 0) return false;
   if (epi == EPI_LN || epi == EPI_LN_HEAD) return N == 64 || N == 128 || N == 256 || N == 512;
   if (epi == EPI_ATTN_LG) return N % 128 == 0 && N <= kStageNAtt;
+  if (epi == EPI_SERVE) return N % 192 == 0 && N <= kStageNSrv;
   return N % 64 == 0;
 }
 
@@ -1264,6 +1405,9 @@ cudaError_t launch_gemm_tc(const __nv_bfloat16* A, long long lda, const __nv_bfl
           e.att_group < 1 || e.att_dkv % 8 != 0)
         return cudaErrorNotSupported;
       return launch_bn<128, EPI_ATTN_LG>(A, lda, B, e, s, cls);
+    case EPI_SERVE:
+      if (e.srv_S < 0 || e.srv_S > kSrvMaxS || e.N != 3 * e.srv_d) return cudaErrorNotSupported;
+      return launch_bn<192, EPI_SERVE, 4, false, true>(A, lda, B, e, s, cls);
     default: return cudaErrorInvalidValue;
   }
 }

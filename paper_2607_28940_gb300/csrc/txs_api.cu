@@ -64,6 +64,10 @@ void prof_end(int cls, cudaStream_t s) {
 struct LayerW {
   void *Wt_qkv, *Wt_os, *Wt_q, *Wt_oc, *Wt_1, *Wt_2;  // transposed weights [d_out, d_in]
   float *b_qkv, *b_os, *g1, *be1, *b_q, *b_oc, *g2, *be2, *b_1, *b_2, *g3, *be3;
+  // the QKV projection with its output columns grouped per head, [q_h | k_h | v_h]
+  // (bf16 models with d_h = 64; null otherwise): the fused serving attention
+  void* Wt_qkv_h = nullptr;
+  float* b_qkv_h = nullptr;
 };
 
 }  // namespace txs
@@ -277,6 +281,22 @@ txs_status model_prepare(txs_model* m, const void* const* w, cudaStream_t s) {
     }
     TXS_CK(launch_to_f32<T>(W(l, 9), m->b_kv + size_t(2 * l) * dkv, dkv, s));
     TXS_CK(launch_to_f32<T>(W(l, 11), m->b_kv + size_t(2 * l + 1) * dkv, dkv, s));
+    if (std::is_same<T, __nv_bfloat16>::value && d / c.n_heads == 64 && 3 * d <= 1536) {
+      // rows (h, j, i) of the per-head copy = rows (j d + h 64 + i) of Wt_qkv
+      const int H = c.n_heads, dh = 64;
+      T* ph = wt(3 * d, d);
+      float* bh = vf(3 * d);
+      if (!ph || !bh) return fail_cuda("cudaMalloc", err);
+      for (int h = 0; h < H; ++h)
+        for (int j = 0; j < 3; ++j) {
+          TXS_CK(cudaMemcpyAsync(ph + size_t(h * 3 * dh + j * dh) * d, static_cast<T*>(L.Wt_qkv) + size_t(j * d + h * dh) * d,
+                                 size_t(dh) * d * sizeof(T), cudaMemcpyDeviceToDevice, s));
+          TXS_CK(cudaMemcpyAsync(bh + h * 3 * dh + j * dh, L.b_qkv + j * d + h * dh, dh * sizeof(float),
+                                 cudaMemcpyDeviceToDevice, s));
+        }
+      L.Wt_qkv_h = ph;
+      L.b_qkv_h = bh;
+    }
     m->layers.push_back(L);
   }
   const void* const* head = w + nL * TXS_WEIGHTS_PER_LAYER;
@@ -490,15 +510,45 @@ txs_status score_impl(txs_model* m, const KvView& c, int n_req, const int32_t* c
   const bool lg_fused = std::is_same<T, __nv_bfloat16>::value && cf.attn_mode == TXS_ATTN_LOCAL_GLOBAL &&
                         (dh == 32 || dh == 64) && d % 128 == 0 && d <= 512 && cf.l_local <= 15 && dkv % 8 == 0 &&
                         q_tiles >= 2LL * tc::num_sms();
+  // serving-stream attention fused into the candidate rows' QKV projection
+  // (bf16, d_h = 64, at most 8 context rows, when the 256-row x one-head
+  // tiles fill the GPU): the context rows are projected and attended first,
+  // then each candidate tile's epilogue attends to them and to its own row
+  const bool serve_fused = std::is_same<T, __nv_bfloat16>::value && m->layers[0].Wt_qkv_h != nullptr && S <= 8 &&
+                           n_cand > 0 && (n_cand + 255) / 256 * H >= tc::num_sms();
   for (int l = 0; l < cf.n_layers; ++l) {
     const LayerW& W = m->layers[l];
     // serving-stream attention (App. B mask), O-projection + residual + LN1
-    EpiArgs e = epi_base(EPI_BIAS, N, 3 * d, d);
-    e.bias = W.b_qkv;
-    e.out = QKV;
-    e.ldo = 3 * d;
-    TXS_CK(gemm(m, X, d, W.Wt_qkv, e, tmp, s, KC_GEMM_QKV));
-    TXS_CK(launch_serving_attn<T>(QKV, A, row_req, static_cast<int>(N), static_cast<int>(n_cand), S, H, d, s));
+    EpiArgs e;
+    if (serve_fused) {
+      const long long n_ctx_rows = N - n_cand;   // R S
+      if (n_ctx_rows > 0) {
+        e = epi_base(EPI_BIAS, n_ctx_rows, 3 * d, d);
+        e.bias = W.b_qkv;
+        e.out = QKV + n_cand * 3 * d;
+        e.ldo = 3 * d;
+        TXS_CK(gemm(m, X + n_cand * d, d, W.Wt_qkv, e, tmp, s, KC_GEMM_QKV));
+        TXS_CK(launch_serving_attn<T>(QKV + n_cand * 3 * d, A + n_cand * d, row_req + n_cand,
+                                      static_cast<int>(n_ctx_rows), 0, S, H, d, s));
+      }
+      e = epi_base(EPI_SERVE, n_cand, 3 * d, d);
+      e.bias = W.b_qkv_h;
+      e.out = A;
+      e.ldo = d;
+      e.srv_ctx = QKV + n_cand * 3 * d;
+      e.srv_row_req = row_req;
+      e.srv_S = S;
+      e.srv_d = d;
+      e.srv_scale_log2 = 1.4426950408889634f / sqrtf(static_cast<float>(d / H));
+      TXS_CK(gemm(m, X, d, W.Wt_qkv_h, e, tmp, s, KC_GEMM_QKV));
+    } else {
+      e = epi_base(EPI_BIAS, N, 3 * d, d);
+      e.bias = W.b_qkv;
+      e.out = QKV;
+      e.ldo = 3 * d;
+      TXS_CK(gemm(m, X, d, W.Wt_qkv, e, tmp, s, KC_GEMM_QKV));
+      TXS_CK(launch_serving_attn<T>(QKV, A, row_req, static_cast<int>(N), static_cast<int>(n_cand), S, H, d, s));
+    }
     e = epi_base(EPI_LN, N, d, d);
     e.bias = W.b_os;
     e.res = X;

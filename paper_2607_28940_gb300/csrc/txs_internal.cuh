@@ -207,6 +207,7 @@ enum Epi : int {
   EPI_LN = 3,         // out = LN(acc + bias + res) over the full row (N == d)
   EPI_LN_HEAD = 4,    // z = LN(...); logits = z Weff_z + xlog; probs = softmax(logits)
   EPI_ATTN_LG = 5,    // q = acc + bias; out = LOCAL_GLOBAL cross-attention of q (tensor cores, bf16)
+  EPI_SERVE = 6,      // q, k, v = acc + bias of one head; out = serving-stream attention (tensor cores, bf16)
 };
 
 // Arguments of every GEMM epilogue; unused fields are ignored.
@@ -267,6 +268,16 @@ struct EpiArgs {
   // same row and column, for a separate launch over those rows
   int att_n_cand;
   void* att_q_ctx;
+  // EPI_SERVE: tile n holds q, k, v (d_h columns each, the weights' output
+  // columns permuted per head) of head n for candidate row `row` (request
+  // srv_row_req[row]); the epilogue writes that head's serving-stream
+  // attention output (App. B mask: the request's srv_S context rows and the
+  // row itself) to out[row][n d_h ...].  The context rows' k and v are rows
+  // r srv_S + t of srv_ctx ([R S][3 srv_d] bf16, columns [q | k | v]).
+  const void* srv_ctx;
+  const int* srv_row_req;
+  int srv_S, srv_d;
+  float srv_scale_log2;   // log2(e) / sqrt(d_h)
 };
 // Largest request count whose offsets an EPI_KV launch carries by value.
 constexpr int kKvParamReq = 1000;

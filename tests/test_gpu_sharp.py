@@ -169,3 +169,18 @@ def test_sharp_cache_rows_and_anchor(name):
             got = g.cache.read_anchor(l, which).cpu().numpy()
             scale = np.sqrt((ref ** 2).mean())
             np.testing.assert_allclose(got / scale, ref / scale, atol=2e-2)
+
+
+@pytest.mark.parametrize("S", [0, 1, 2, 8])
+def test_sharp_fused_serving_attention(S):
+    # batches large enough for the serving-stream attention fused into the
+    # candidate rows' QKV projection (bf16, d_h = 64, a 256-row x one-head
+    # tile per SM): 0, 1, 2 and 8 context rows per request (the fused path
+    # takes up to 8), ragged slates incl. a single candidate, every candidate
+    # compared; the attention gain makes the serving softmax decide the scores
+    wl = W.Workload(f"serve{S}", seed=880 + S, dtype="bf16", n_req=6, n_layers=1, d_model=512, n_heads=8,
+                    d_ff=512, L=[40, 3, 12, 90, 1, 25], M=[1100, 900, 1000, 1300, 1, 1000], n_ctx=S)
+    w = W.sharp_weights(wl)
+    g = run_gpu(wl, txs.LOCAL_GLOBAL, weights=w)
+    lg, pr, _, _ = oracle_scores(wl, txs.LOCAL_GLOBAL, weights=w)
+    _check(g.logits, g.probs, lg, pr, wl.dtype, f"fused serving S={S}")
