@@ -546,7 +546,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
 
 // ------------------------------------------------------------------ CTA pairs
 
-// Rows of d = 256 NP columns on clusters of NP CTA pairs (no action head):
+// Rows of d = 256 NP columns on clusters of NP CTA pairs (HEAD: the last
+// layer, whose LN output goes into the action head instead of memory):
 // pair p computes columns [256 p, 256 p + 256) of a 256-row tile with
 // M = 256 MMAs (cta_group::2), issued by its even CTA; CTA 2 p + r holds rows
 // [128 r, 128 r + 128) of the tile in its TMEM (two 256-column buffers).
@@ -555,17 +556,23 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
 // the CTA of the other pair that holds the same rows (st.async, counted on
 // its barrier); with NP = 1 the row is whole in one CTA.  The eight epilogue
 // warps form two groups taking alternate tiles, as in the cluster kernel.
+// With HEAD each CTA forms the partial logits z . W_eff_z of its 256 columns
+// (at most 4 actions) and sends them to the CTA of pair 0 with the same rows,
+// which adds the x part and writes logits and probabilities.
 constexpr int PBN = 256;               // columns per CTA (and per pair)
 
-template <int NP>
+template <int NP, bool HEAD>
 struct PairShape {
   static constexpr int CS = 2 * NP;
+  static constexpr int NAP = 4;                                     // head actions padded to 4
   static constexpr int B_STAGE_BYTES = 128 * BK * 2;                // 16 KB
   static constexpr int STAGE_BYTES = A_STAGE_BYTES + B_STAGE_BYTES;
-  static constexpr int STG_BYTES = kWarps * 2048;                   // one bulk-store buffer per warp
+  static constexpr int STG_BYTES = HEAD ? 0 : kWarps * 2048;        // one bulk-store buffer per warp
   static constexpr int XBUF_BYTES = 2 * NP * 128 * 8;               // (mean, M2) per column block, two parities
+  static constexpr int HBUF_BYTES = HEAD ? 2 * NP * 128 * NAP * 4 : 0;   // partial logits per column block
+  static constexpr int WEFF_BYTES = HEAD ? PBN * NAP * 4 : 0;
   static constexpr int PAR_BYTES = 3 * PBN * 4;
-  static constexpr int EXTRA = STG_BYTES + XBUF_BYTES + PAR_BYTES + 1024 + 512;
+  static constexpr int EXTRA = STG_BYTES + XBUF_BYTES + HBUF_BYTES + WEFF_BYTES + PAR_BYTES + 1024 + 512;
   static constexpr int STAGES_FIT = (227 * 1024 - EXTRA) / STAGE_BYTES;
   static constexpr int STAGES = STAGES_FIT > 8 ? 8 : STAGES_FIT;
   static constexpr int SMEM_BYTES = STAGES * STAGE_BYTES + EXTRA;
@@ -573,24 +580,28 @@ struct PairShape {
   static_assert(STAGES >= 4 && SMEM_BYTES <= 232448, "shared memory");
 };
 
-template <int NP>
+template <int NP, bool HEAD>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
     gemm_ln_pair_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                         const __grid_constant__ CUtensorMap tmO, const EpiArgs e) {
-  using S = PairShape<NP>;
+  using S = PairShape<NP, HEAD>;
+  constexpr int NAP = S::NAP;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* sA = smem;
   uint8_t* sB = sA + S::STAGES * A_STAGE_BYTES;
   uint8_t* s_stage = sB + S::STAGES * S::B_STAGE_BYTES;
   float2* xbuf = reinterpret_cast<float2*>(s_stage + S::STG_BYTES);                 // [2][NP][128]
-  float* s_par = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(xbuf) + S::XBUF_BYTES);   // [3][PBN]
+  float* hbuf = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(xbuf) + S::XBUF_BYTES);     // [2][NP][128][NAP]
+  float* s_weff = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(hbuf) + S::HBUF_BYTES);  // [PBN][NAP]
+  float* s_par = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(s_weff) + S::WEFF_BYTES);  // [3][PBN]
   uint64_t* full = reinterpret_cast<uint64_t*>(reinterpret_cast<uint8_t*>(s_par) + S::PAR_BYTES);
   uint64_t* empty = full + S::STAGES;
   uint64_t* acc_full = empty + S::STAGES;
   uint64_t* acc_empty = acc_full + 2;
   uint64_t* xfull = acc_empty + 2;    // [2][4]: the other pair's statistics of lane quarter q
-  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(xfull + 8);
+  uint64_t* hfull = xfull + 8;        // [2][4]: the other pairs' partial logits (pair 0, HEAD)
+  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(hfull + 8);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_holder + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -615,7 +626,10 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       mbar_init(acc_full + b, 1);
       mbar_init(acc_empty + b, 2 * kGroupWarps);     // the even CTA's: both CTAs' group
     }
-    for (int i = 0; i < 8; ++i) mbar_init(xfull + i, 1);
+    for (int i = 0; i < 8; ++i) {
+      mbar_init(xfull + i, 1);
+      mbar_init(hfull + i, 1);
+    }
     *abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
@@ -639,6 +653,12 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     s_par[i] = e.bias[n0 + i];
     s_par[PBN + i] = e.gamma[n0 + i];
     s_par[2 * PBN + i] = e.beta[n0 + i];
+  }
+  if constexpr (HEAD) {
+    for (int i = threadIdx.x; i < PBN * NAP; i += NUM_THREADS) {
+      const int c = i / NAP, a = i - c * NAP;
+      s_weff[i] = a < e.n_act ? e.weff_z[static_cast<long long>(n0 + c) * e.n_act + a] : 0.f;
+    }
   }
   __syncthreads();
 
@@ -809,20 +829,84 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         }
       }
       const float rstd = rsqrtf(m2 / static_cast<float>(PBN * NP) + e.ln_eps);
-      // pass 2: normalise and store
+      // pass 2: normalise and store, or the head's partial logits
+      float lg[NAP];
+#pragma unroll
+      for (int a = 0; a < NAP; ++a) lg[a] = 0.f;
 #pragma unroll 1
       for (int c = 0; c < PBN; c += 32) {
         tmem_ld32(tacc + c, v);
 #pragma unroll
         for (int k = 0; k < 32; ++k) v[k] = (v[k] - mean) * rstd * s_gamma[c + k] + s_beta[c + k];
-        __nv_bfloat16* out =
-            valid ? static_cast<__nv_bfloat16*>(e.out) + static_cast<long long>(row) * e.ldo + n0 + c : nullptr;
-        store_chunk<1>(v, out, valid, true, &tmO, n0 + c, m0 + q * 32, stage, kchunk++, lane);
+        if constexpr (!HEAD) {
+          __nv_bfloat16* out =
+              valid ? static_cast<__nv_bfloat16*>(e.out) + static_cast<long long>(row) * e.ldo + n0 + c : nullptr;
+          store_chunk<1>(v, out, valid, true, &tmO, n0 + c, m0 + q * 32, stage, kchunk++, lane);
+        } else {
+          const float4* w4 = reinterpret_cast<const float4*>(s_weff + c * NAP);
+#pragma unroll
+          for (int k = 0; k < 32; ++k) {
+            const float4 w = w4[k];
+            lg[0] = fmaf(v[k], w.x, lg[0]);
+            lg[1] = fmaf(v[k], w.y, lg[1]);
+            lg[2] = fmaf(v[k], w.z, lg[2]);
+            lg[3] = fmaf(v[k], w.w, lg[3]);
+          }
+        }
       }
       // every read of this accumulator is done: release it on the even CTA
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive_peer_signal(lead(acc_empty + buf));
+      if constexpr (HEAD) {
+        // partial logits of these 256 columns -> the CTA of pair 0 with the same rows
+        float* mine = hbuf + ((pb * NP + pr) * 128 + trow) * NAP;
+        if (pr == 0) {
+          *reinterpret_cast<float4*>(mine) = make_float4(lg[0], lg[1], lg[2], lg[3]);
+        } else {
+          const uint32_t owner = static_cast<uint32_t>(half);
+          st_async_f32x4(map_peer(mine, owner), lg[0], lg[1], lg[2], lg[3], map_peer(hfull + pb * 4 + q, owner));
+        }
+        if (pr == 0) {
+          if constexpr (NP > 1) {
+            if (lane == 0) mbar_expect_tx(hfull + pb * 4 + q, (NP - 1) * 32 * NAP * 4);
+            bool ok = mbar_wait_cluster(hfull + pb * 4 + q, use, abort_flag);
+            ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
+            if (!ok) break;
+          }
+          if (valid && row < e.n_cand_rows) {
+            const int na = e.n_act;
+            float t[NAP];
+#pragma unroll
+            for (int a = 0; a < NAP; ++a) t[a] = 0.f;
+#pragma unroll
+            for (int o = 0; o < NP; ++o) {
+              const float4 x = *reinterpret_cast<const float4*>(hbuf + ((pb * NP + o) * 128 + trow) * NAP);
+              t[0] += x.x; t[1] += x.y; t[2] += x.z; t[3] += x.w;
+            }
+            float mx = -INFINITY;
+#pragma unroll
+            for (int a = 0; a < NAP; ++a)
+              if (a < na) {
+                t[a] += __ldg(e.xlog + static_cast<long long>(row) * na + a);
+                mx = fmaxf(mx, t[a]);
+              }
+            float ssum = 0.f, pe[NAP];
+#pragma unroll
+            for (int a = 0; a < NAP; ++a) {
+              pe[a] = a < na ? expf(t[a] - mx) : 0.f;
+              ssum += pe[a];
+            }
+            const float inv = 1.f / ssum;
+#pragma unroll
+            for (int a = 0; a < NAP; ++a)
+              if (a < na) {
+                e.logits[static_cast<long long>(row) * na + a] = t[a];
+                if (e.probs) e.probs[static_cast<long long>(row) * na + a] = pe[a] * inv;
+              }
+          }
+        }
+      }
     }
     if (lane == 0) bulk_wait_all();
   }
@@ -836,11 +920,11 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   if (threadIdx.x == 0 && *abort_flag) latch_status(e.status, TXS_ERR_DEVICE_TIMEOUT);
 }
 
-template <int NP>
+template <int NP, bool HEAD>
 static cudaError_t launch_pair(const __nv_bfloat16* A, long long lda, const __nv_bfloat16* B, const EpiArgs& e,
                                cudaStream_t s, int cls) {
-  using Sh = PairShape<NP>;
-  auto kern = gemm_ln_pair_kernel<NP>;
+  using Sh = PairShape<NP, HEAD>;
+  auto kern = gemm_ln_pair_kernel<NP, HEAD>;
   cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeClusterDimension;
   attr[0].val.clusterDim.x = Sh::CS;
@@ -869,7 +953,8 @@ static cudaError_t launch_pair(const __nv_bfloat16* A, long long lda, const __nv
   CUtensorMap ta, tb, to;
   if (!make_tmap(&ta, A, e.M, e.K, lda, BM)) return cudaErrorInvalidValue;
   if (!make_tmap(&tb, B, e.N, e.K, e.K, 128)) return cudaErrorInvalidValue;
-  if (!make_tmap_out(&to, e.out, e.M, e.N, e.ldo)) return cudaErrorInvalidValue;
+  if (HEAD) to = ta;   // unused
+  else if (!make_tmap_out(&to, e.out, e.M, e.N, e.ldo)) return cudaErrorInvalidValue;
   const int m_tiles = (e.M + 2 * BM - 1) / (2 * BM);
   const int ncl = m_tiles < max_clusters ? m_tiles : max_clusters;
   cfg.gridDim = dim3(ncl * Sh::CS);
@@ -937,10 +1022,15 @@ cudaError_t launch_gemm_ln_cluster(const __nv_bfloat16* A, long long lda, const 
   if (e.epi != EPI_LN && e.epi != EPI_LN_HEAD) return cudaErrorNotSupported;
   const bool head = e.epi == EPI_LN_HEAD;
   // CTA pairs (256 columns per CTA) once every cluster gets two 256-row tiles
-  if (!head && (e.N == 256 || e.N == 512)) {
+  if ((e.N == 256 || e.N == 512) && (!head || e.n_act <= 4)) {
     const int ncs = e.N / 128;   // CTAs per cluster either way
-    if ((e.M + 2 * tc::BM - 1) / (2 * tc::BM) >= 2 * (num_sms() / ncs))
-      return e.N == 256 ? tcln::launch_pair<1>(A, lda, B, e, s, cls) : tcln::launch_pair<2>(A, lda, B, e, s, cls);
+    if ((e.M + 2 * tc::BM - 1) / (2 * tc::BM) >= 2 * (num_sms() / ncs)) {
+      if (head)
+        return e.N == 256 ? tcln::launch_pair<1, true>(A, lda, B, e, s, cls)
+                          : tcln::launch_pair<2, true>(A, lda, B, e, s, cls);
+      return e.N == 256 ? tcln::launch_pair<1, false>(A, lda, B, e, s, cls)
+                        : tcln::launch_pair<2, false>(A, lda, B, e, s, cls);
+    }
   }
   // the two epilogue groups pay off once each cluster has several row tiles
   const int m_tiles = (e.M + tc::BM - 1) / tc::BM;

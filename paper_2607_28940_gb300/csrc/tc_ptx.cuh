@@ -399,6 +399,12 @@ __device__ __forceinline__ void st_async_f32x2(uint32_t addr, float a, float b, 
                "f"(a), "f"(b), "r"(bar_cl)
                : "memory");
 }
+__device__ __forceinline__ void st_async_f32x4(uint32_t addr, float a, float b, float c, float d, uint32_t bar_cl) {
+  asm volatile("st.async.shared::cluster.mbarrier::complete_tx::bytes.v4.f32 [%0], {%1, %2, %3, %4}, [%5];" ::"r"(
+                   addr),
+               "f"(a), "f"(b), "f"(c), "f"(d), "r"(bar_cl)
+               : "memory");
+}
 // arrive on a barrier of a peer CTA with CTA-scope release: no cluster-wide
 // memory fence, for signals that publish no memory (a TMEM buffer read out,
 // ordered by tcgen05.fence::before_thread_sync)
