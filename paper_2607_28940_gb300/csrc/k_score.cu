@@ -37,7 +37,7 @@ __device__ __forceinline__ int find_segment_param(const int* off, int n, int row
   return lo;
 }
 
-constexpr int kPackRowsPerWarp = 2;
+constexpr int kPackRowsPerWarp = 4;
 
 // Sum of NA per-lane values over the 32 lanes of a warp, scattered: on return
 // every lane holds the total of value lane / (32 / NA).  Each halving step
@@ -63,11 +63,11 @@ __device__ __forceinline__ float warp_reduce_scatter(float (&v)[NA], int lane) {
 
 // 8 warps per CTA, kPackRowsPerWarp consecutive rows per warp (all of a
 // warp's row loads are issued before its arithmetic); CH 16-byte chunks per
-// lane and row cover d.  The x-part of the
-// logits takes NA >= na actions (the actions na..NA-1 have zero weights and
-// are not written); a lane's head weights for its columns are loaded once, to
-// registers when NA <= 4, else staged per CTA in shared memory as
-// [action][column].
+// lane and row cover d.  The x-part of the logits takes NA >= na actions (the
+// actions na..NA-1 have zero weights and are not written); the head weights
+// are staged per CTA in shared memory as [action][column] and read as float4
+// runs, which keeps the register count low enough for four CTAs per SM and
+// so many rows in flight.
 template <typename T, int NA, int CH>
 __global__ void __launch_bounds__(256) pack_kernel(const __grid_constant__ PackArgs a, const T* __restrict__ cand,
                                                    const T* __restrict__ ctx, T* __restrict__ X,
@@ -78,8 +78,8 @@ __global__ void __launch_bounds__(256) pack_kernel(const __grid_constant__ PackA
   pdl_wait();
   constexpr int VEC = Vec16<T>::N;
   constexpr int MAXCH = CH;
-  constexpr bool kRegW = NA <= 4;
-  extern __shared__ float sw[];                 // [NA][d] when !kRegW
+  extern __shared__ float4 sw4[];
+  float* sw = reinterpret_cast<float*>(sw4);    // [NA][d]
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int d = a.d, na = a.na;
   if (blockIdx.x == 0)
@@ -97,36 +97,11 @@ __global__ void __launch_bounds__(256) pack_kernel(const __grid_constant__ PackA
       raw[t][j] = (p < n_rows && col < d) ? *reinterpret_cast<const uint4*>(src + col) : make_uint4(0, 0, 0, 0);
     }
   }
-  // head weights after the row loads are in flight: a lane's columns
-  // col..col+VEC-1 hold VEC * na consecutive floats of weff_x ([d][na])
-  float wr[kRegW ? MAXCH : 1][kRegW ? VEC : 1][NA];
-  if constexpr (kRegW) {
+  // head weights, staged after the row loads are in flight
+  for (int c = threadIdx.x; c < d; c += 256)
 #pragma unroll
-    for (int j = 0; j < MAXCH; ++j) {
-      const int col = (j * 32 + lane) * VEC;
-      if (na == NA && col < d) {
-        const float4* w4 = reinterpret_cast<const float4*>(weff_x + static_cast<long long>(col) * NA);
-#pragma unroll
-        for (int q = 0; q < VEC * NA / 4; ++q) {
-          const float4 f = __ldg(w4 + q);
-          const float e[4] = {f.x, f.y, f.z, f.w};
-#pragma unroll
-          for (int u = 0; u < 4; ++u) wr[j][(4 * q + u) / NA][(4 * q + u) % NA] = e[u];
-        }
-      } else {
-#pragma unroll
-        for (int i = 0; i < VEC; ++i)
-#pragma unroll
-          for (int k = 0; k < NA; ++k)
-            wr[j][i][k] = (col < d && k < na) ? __ldg(weff_x + static_cast<long long>(col + i) * na + k) : 0.f;
-      }
-    }
-  } else {
-    for (int c = threadIdx.x; c < d; c += 256)
-#pragma unroll
-      for (int k = 0; k < NA; ++k) sw[k * d + c] = k < na ? weff_x[static_cast<long long>(c) * na + k] : 0.f;
-    __syncthreads();
-  }
+    for (int k = 0; k < NA; ++k) sw[k * d + c] = k < na ? weff_x[static_cast<long long>(c) * na + k] : 0.f;
+  __syncthreads();
 #pragma unroll
   for (int t = 0; t < kPackRowsPerWarp; ++t) {
     const long long p = p0 + t;
@@ -153,11 +128,15 @@ __global__ void __launch_bounds__(256) pack_kernel(const __grid_constant__ PackA
           Vec16<T>::load(reinterpret_cast<const T*>(&raw[t][j]), v);
 #pragma unroll
           for (int k = 0; k < NA; ++k) {
+            const float4* w4 = reinterpret_cast<const float4*>(sw + k * d + col);
             float acc = 0.f;
 #pragma unroll
-            for (int i = 0; i < VEC; ++i) {
-              if constexpr (kRegW) acc = fmaf(v[i], wr[j][i][k], acc);
-              else acc = fmaf(v[i], sw[k * d + col + i], acc);
+            for (int qq = 0; qq < VEC / 4; ++qq) {
+              const float4 w = w4[qq];
+              acc = fmaf(v[4 * qq], w.x, acc);
+              acc = fmaf(v[4 * qq + 1], w.y, acc);
+              acc = fmaf(v[4 * qq + 2], w.z, acc);
+              acc = fmaf(v[4 * qq + 3], w.w, acc);
             }
             lg[k] += acc;
           }
@@ -190,19 +169,24 @@ __global__ void __launch_bounds__(1024) rank_kernel(const __grid_constant__ Rank
   for (int i = threadIdx.x; i < M; i += blockDim.x)
     keys[i] = order_key(probs[static_cast<long long>(c0 + i) * a.na + a.action]);
   __syncthreads();
+  // CTA y of the request ranks candidates [i0, i1) against all M keys
+  const int per = (M + static_cast<int>(gridDim.y) - 1) / static_cast<int>(gridDim.y);
+  const int i0 = static_cast<int>(blockIdx.y) * per;
+  const int i1 = min(M, i0 + per);
+  const int n_i = i1 > i0 ? i1 - i0 : 0;
   // tpc consecutive lanes share a candidate (short slates leave threads to
   // spare), each counting every tpc-th key with four independent counters;
   // the group adds its counts with shuffles.  Every lane runs the same number
   // of rounds, so the shuffles see full warps.
   int tpc = 1;
-  while (tpc < 32 && tpc * 2 * M <= static_cast<int>(blockDim.x)) tpc *= 2;
+  while (tpc < 32 && tpc * 2 * n_i <= static_cast<int>(blockDim.x)) tpc *= 2;
   const int per_round = blockDim.x / tpc;
   const int sub = threadIdx.x & (tpc - 1);
-  const int rounds = (M + per_round - 1) / per_round;
+  const int rounds = (n_i + per_round - 1) / per_round;
   for (int round = 0; round < rounds; ++round) {
-    const int i = round * per_round + static_cast<int>(threadIdx.x) / tpc;
+    const int i = i0 + round * per_round + static_cast<int>(threadIdx.x) / tpc;
     int rank = 0;
-    if (i < M) {
+    if (i < i1) {
       const uint32_t ki = keys[i];
       int c[4] = {0, 0, 0, 0};
       int j = sub;
@@ -221,12 +205,12 @@ __global__ void __launch_bounds__(1024) rank_kernel(const __grid_constant__ Rank
       rank = (c[0] + c[1]) + (c[2] + c[3]);
     }
     for (int o = tpc >> 1; o >= 1; o >>= 1) rank += __shfl_xor_sync(0xffffffffu, rank, o);
-    if (i < M && sub == 0) {
+    if (i < i1 && sub == 0) {
       if (a.top_k == 0) out[c0 + rank] = i;
       else if (rank < a.top_k) out[static_cast<long long>(r) * a.top_k + rank] = i;
     }
   }
-  if (a.top_k > 0)
+  if (a.top_k > 0 && blockIdx.y == 0)
     for (int t = M + threadIdx.x; t < a.top_k; t += blockDim.x) out[static_cast<long long>(r) * a.top_k + t] = -1;
 }
 
@@ -385,14 +369,14 @@ static cudaError_t pack_launch_ch(int na, dim3 grid, cudaStream_t s, const PackA
                                   float* xlog) {
   const int d = a.d;
   if (na <= 1)
-    return launch_pdl(pack_kernel<T, 1, CH>, grid, dim3(256), 0, s, a, cand, ctx, X, row_req, cand_off_dev, weff_x,
-                      cdec, xlog);
+    return launch_pdl(pack_kernel<T, 1, CH>, grid, dim3(256), sizeof(float) * 1 * d, s, a, cand, ctx, X, row_req,
+                      cand_off_dev, weff_x, cdec, xlog);
   if (na <= 2)
-    return launch_pdl(pack_kernel<T, 2, CH>, grid, dim3(256), 0, s, a, cand, ctx, X, row_req, cand_off_dev, weff_x,
-                      cdec, xlog);
+    return launch_pdl(pack_kernel<T, 2, CH>, grid, dim3(256), sizeof(float) * 2 * d, s, a, cand, ctx, X, row_req,
+                      cand_off_dev, weff_x, cdec, xlog);
   if (na <= 4)
-    return launch_pdl(pack_kernel<T, 4, CH>, grid, dim3(256), 0, s, a, cand, ctx, X, row_req, cand_off_dev, weff_x,
-                      cdec, xlog);
+    return launch_pdl(pack_kernel<T, 4, CH>, grid, dim3(256), sizeof(float) * 4 * d, s, a, cand, ctx, X, row_req,
+                      cand_off_dev, weff_x, cdec, xlog);
   if (na <= 8)
     return launch_pdl(pack_kernel<T, 8, CH>, grid, dim3(256), sizeof(float) * 8 * d, s, a, cand, ctx, X, row_req,
                       cand_off_dev, weff_x, cdec, xlog);
@@ -447,8 +431,13 @@ cudaError_t launch_rank(int n_req, const int* cand_off_host, const float* probs,
     if (e != cudaSuccess) return e;
     attr = true;
   }
+  // up to 8 CTAs per request (each ranks a slice of its slate against all of
+  // it), so that the launch covers the GPU when there are few requests
+  int splits = 1;
+  while (splits < 8 && static_cast<long long>(splits) * n_req < tc::num_sms() && max_m / (2 * splits) >= 128)
+    splits *= 2;
   prof_begin(KC_RANK, s);
-  cudaError_t err = launch_pdl(rank_kernel, dim3(n_req), dim3(1024), smem, s, a, probs, out);
+  cudaError_t err = launch_pdl(rank_kernel, dim3(n_req, splits), dim3(1024), smem, s, a, probs, out);
   prof_end(KC_RANK, s);
   return err;
 }
