@@ -55,6 +55,7 @@ NCU_TRAFFIC = {
     # (4.8 MB + 43.0 MB), averaged over the two launches of a step
     ("ragged_bf16", "local_global", "gemm_kv_build"): (2.395e+09, "9b7cd1c6e33a"),
     ("mid_bf16", "full", "attn_cross"): (873.9e6, "db3c1a34b26e"),
+    ("sweep_bf16", "full", "attn_cross"): (317.1e6, "db3c1a34b26e"),
 }
 
 
