@@ -452,6 +452,15 @@ txs_status txs_encoder_device_status(txs_encoder* enc);
 /* Synchronise the device, read and clear the model's latched device status. */
 txs_status txs_device_status(txs_model* model);
 
+/* Self-test of the device-side failure path (no paper counterpart): enqueue
+ * on `stream` one kernel whose bounded wait, the same wait every pipeline
+ * of the library uses, runs out (about a second: nothing ever arrives at
+ * its barrier).  The kernel then latches TXS_ERR_DEVICE_TIMEOUT into the
+ * model's status word and returns; no fault, the context stays usable.  A
+ * following txs_device_status(model) returns TXS_ERR_DEVICE_TIMEOUT and
+ * clears the word.  Errors: TXS_ERR_INVALID_ARG (null model), TXS_ERR_CUDA. */
+txs_status txs_selftest_wait_timeout(txs_model* model, void* stream);
+
 /* The GELU of the FFN epilogues, element-wise on device float arrays x -> y
  * of n elements, for tests of its accuracy (no paper counterpart; the
  * activation is the exact erf form 0.5 x (1 + erf(x / sqrt 2))).  variant 0:

@@ -784,6 +784,27 @@ cudaError_t launch_hash(const void* p, long long bytes, uint64_t salt, unsigned 
   return cudaGetLastError();
 }
 
+// Self-test of the bounded waits every pipeline of this library uses: one
+// thread waits (tc::mbar_wait, kSpinCycles) on an mbarrier nothing arrives
+// at; when the wait gives up the kernel latches TXS_ERR_DEVICE_TIMEOUT into
+// the status word and returns, leaving the context usable.
+__global__ void wait_timeout_probe_kernel(int* status) {
+  __shared__ __align__(8) uint64_t bar;
+  __shared__ int abort_flag;
+  if (threadIdx.x == 0) {
+    tc::mbar_init(&bar, 1);
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    abort_flag = 0;
+  }
+  __syncthreads();
+  if (threadIdx.x == 0 && !tc::mbar_wait(&bar, 0, &abort_flag)) latch_status(status, TXS_ERR_DEVICE_TIMEOUT);
+}
+
+cudaError_t launch_wait_timeout_probe(int* status, cudaStream_t s) {
+  wait_timeout_probe_kernel<<<1, 32, 0, s>>>(status);
+  return cudaGetLastError();
+}
+
 // ------------------------------------------------------------------ prefix pooling
 
 // Streaming events (Sec. 4.2 prefix reuse; Sec. 5.1 a global token for each

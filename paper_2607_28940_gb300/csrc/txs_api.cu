@@ -1292,6 +1292,12 @@ TXS_API txs_status txs_device_status(txs_model* m) {
   return static_cast<txs_status>(v);
 }
 
+TXS_API txs_status txs_selftest_wait_timeout(txs_model* m, void* stream) {
+  if (!m) return TXS_ERR_INVALID_ARG;
+  const cudaError_t e = launch_wait_timeout_probe(m->status, static_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? TXS_OK : fail_cuda("wait_timeout_probe", e);
+}
+
 TXS_API txs_status txs_gelu_eval(const float* x, float* y, int64_t n, int32_t variant, void* stream) {
   if (n < 0 || (n > 0 && (!x || !y)) || (variant != 0 && variant != 1)) return TXS_ERR_INVALID_ARG;
   const cudaError_t e = launch_gelu_eval(x, y, n, variant, static_cast<cudaStream_t>(stream));

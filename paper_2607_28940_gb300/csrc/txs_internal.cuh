@@ -290,6 +290,8 @@ cudaError_t launch_gemm_simt(const float* A, long long lda, const TB* B, const E
 // GELU of the GEMM epilogues on device float arrays (variant 0: bf16
 // tensor-core epilogue, 1: fp32 path), for tests.
 cudaError_t launch_gelu_eval(const float* x, float* y, long long n, int variant, cudaStream_t s);
+// One bounded wait that runs out (about a second), latching TXS_ERR_DEVICE_TIMEOUT.
+cudaError_t launch_wait_timeout_probe(int* status, cudaStream_t s);
 cudaError_t launch_gemm_tc(const __nv_bfloat16* A, long long lda, const __nv_bfloat16* B,
                            const EpiArgs& e, cudaStream_t s, int cls);
 bool tc_gemm_supported(int N, int K, int epi);

@@ -100,6 +100,7 @@ _SIGS = {
     "txs_encoder_device_status": (_I32, [_P]),
     "txs_pool_anchor_static": (_I32, [_P, _I32, _I32P, _P, _P, _P]),
     "txs_gelu_eval": (_I32, [_P, _P, ctypes.c_int64, _I32, _P]),
+    "txs_selftest_wait_timeout": (_I32, [_P, _P]),
     "txs_profile_enable": (_I32, [_I32]),
     "txs_profile_collect": (_I32, [ctypes.POINTER(ctypes.c_double), ctypes.POINTER(ctypes.c_int64), _I32]),
     "txs_kernel_class_name": (ctypes.c_char_p, [_I32]),
@@ -205,6 +206,10 @@ class Model:
 
     def device_status(self) -> int:
         return int(lib().txs_device_status(self.handle))
+
+    def selftest_wait_timeout(self) -> None:
+        """Enqueue the bounded-wait self-test; device_status() then reports the timeout."""
+        _check(lib().txs_selftest_wait_timeout(self.handle, _stream(None)), "txs_selftest_wait_timeout")
 
     def close(self):
         if getattr(self, "handle", None):
