@@ -157,6 +157,7 @@ using namespace txs;
 
 TXS_API txs_status txs_pool_anchor_static(const txs_model* model, int32_t n_req, const int32_t* beh_offsets,
                                           const void* beh_enc, float* out_g, void* stream) {
+  TXS_TRACE();
   if (!model || !beh_offsets || !beh_enc || !out_g || n_req < 1) return TXS_ERR_INVALID_ARG;
   if (beh_offsets[0] != 0) return TXS_ERR_INVALID_ARG;
   for (int r = 0; r < n_req; ++r) {

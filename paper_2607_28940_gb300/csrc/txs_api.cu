@@ -688,6 +688,7 @@ using namespace txs;
 TXS_API const char* txs_version(void) { return "txs 0.1 (sm_103a)"; }
 
 TXS_API const char* txs_status_string(txs_status s) {
+  TXS_TRACE();
   switch (s) {
     case TXS_OK: return "ok";
     case TXS_ERR_INVALID_ARG: return "invalid argument";
@@ -712,6 +713,7 @@ const float* model_w_pool(const txs_model* m) { return m->w_pool; }
 }  // namespace txs
 
 TXS_API txs_status txs_model_create(const txs_config* cfg, const void* const* weights, txs_model** out) {
+  TXS_TRACE();
   if (!cfg || !weights || !out) return TXS_ERR_INVALID_ARG;
   *out = nullptr;
   std::string why;
@@ -758,6 +760,7 @@ TXS_API txs_status txs_model_create(const txs_config* cfg, const void* const* we
 }
 
 TXS_API void txs_model_destroy(txs_model* m) {
+  TXS_TRACE();
   if (!m) return;
   for (void* p : m->allocs) cudaFree(p);
   delete m;
@@ -851,6 +854,7 @@ txs_status make_cache(txs_model* m, int n_req, const int* lengths, int capacity_
 
 TXS_API txs_status txs_build_kv_cache(txs_model* m, int32_t n_req, const int32_t* beh_offsets, const void* beh_enc,
                                       int32_t capacity_extra, void* stream, txs_kv_cache** out) {
+  TXS_TRACE();
   if (!m || !out || n_req < 1 || capacity_extra < 0 || !beh_offsets) return TXS_ERR_INVALID_ARG;
   *out = nullptr;
   if (!offsets_ok(beh_offsets, n_req, false)) return TXS_ERR_INVALID_ARG;
@@ -901,6 +905,7 @@ size_t cache_blob_bytes(int n_req, int nL, int d, int dkv, int es, long long row
 }  // namespace
 
 TXS_API txs_status txs_cache_export_size(const txs_kv_cache* c, size_t* bytes) {
+  TXS_TRACE();
   if (!c || !bytes) return TXS_ERR_INVALID_ARG;
   long long rows = 0;
   for (int r = 0; r < c->n_req; ++r) rows += c->h_len[r];
@@ -910,6 +915,7 @@ TXS_API txs_status txs_cache_export_size(const txs_kv_cache* c, size_t* bytes) {
 
 TXS_API txs_status txs_cache_export(const txs_kv_cache* c, uint32_t schema_version, void* host_buf, size_t bytes,
                                     void* stream) {
+  TXS_TRACE();
   if (!c || !host_buf) return TXS_ERR_INVALID_ARG;
   size_t need = 0;
   txs_cache_export_size(c, &need);
@@ -960,6 +966,7 @@ TXS_API txs_status txs_cache_export(const txs_kv_cache* c, uint32_t schema_versi
 
 TXS_API txs_status txs_cache_import(txs_model* m, uint32_t schema_version, const void* host_buf, size_t bytes,
                                     int32_t capacity_extra, void* stream, txs_kv_cache** out) {
+  TXS_TRACE();
   if (!m || !host_buf || !out || capacity_extra < 0) return TXS_ERR_INVALID_ARG;
   *out = nullptr;
   if (bytes < sizeof(CacheHeader)) return TXS_ERR_INVALID_ARG;
@@ -1017,6 +1024,7 @@ TXS_API txs_status txs_cache_import(txs_model* m, uint32_t schema_version, const
 }
 
 TXS_API void txs_cache_destroy(txs_kv_cache* c) {
+  TXS_TRACE();
   if (!c) return;
   for (cudaEvent_t e : c->stage_ev)
     if (e) cudaEventSynchronize(e);
@@ -1029,6 +1037,7 @@ TXS_API void txs_cache_destroy(txs_kv_cache* c) {
 
 TXS_API txs_status txs_rebuild_kv_cache(txs_model* m, txs_kv_cache* c, int32_t n_req, const int32_t* beh_offsets,
                                         const void* beh_enc, void* stream) {
+  TXS_TRACE();
   if (!m || !c || !beh_offsets) return TXS_ERR_INVALID_ARG;
   if (c->model_hash != m->hash) return TXS_ERR_STALE_CACHE;
   if (n_req != c->n_req || !offsets_ok(beh_offsets, n_req, false)) return TXS_ERR_INVALID_ARG;
@@ -1048,6 +1057,7 @@ TXS_API txs_status txs_rebuild_kv_cache(txs_model* m, txs_kv_cache* c, int32_t n
 TXS_API txs_status txs_rebuild_append_kv_cache(txs_model* m, txs_kv_cache* c, int32_t n_req,
                                                const int32_t* beh_offsets, const void* beh_enc,
                                                const int32_t* new_offsets, const void* new_enc, void* stream) {
+  TXS_TRACE();
   if (!m || !c || !beh_offsets || !new_offsets) return TXS_ERR_INVALID_ARG;
   if (c->model_hash != m->hash) return TXS_ERR_STALE_CACHE;
   if (n_req != c->n_req || !offsets_ok(beh_offsets, n_req, false) || !offsets_ok(new_offsets, n_req, false))
@@ -1077,6 +1087,7 @@ TXS_API txs_status txs_rebuild_append_kv_cache(txs_model* m, txs_kv_cache* c, in
 
 TXS_API txs_status txs_append_behavior(txs_model* m, txs_kv_cache* c, int32_t n_req, const int32_t* new_offsets,
                                        const void* new_enc, void* stream) {
+  TXS_TRACE();
   if (!m || !c || !new_offsets) return TXS_ERR_INVALID_ARG;
   if (c->model_hash != m->hash) return TXS_ERR_STALE_CACHE;
   if (n_req != c->n_req || !offsets_ok(new_offsets, n_req, false)) return TXS_ERR_INVALID_ARG;
@@ -1094,6 +1105,7 @@ TXS_API txs_status txs_append_behavior(txs_model* m, txs_kv_cache* c, int32_t n_
 }
 
 TXS_API txs_status txs_cache_lengths(const txs_kv_cache* c, int32_t* out_len) {
+  TXS_TRACE();
   if (!c || !out_len) return TXS_ERR_INVALID_ARG;
   for (int r = 0; r < c->n_req; ++r) out_len[r] = c->h_len[r];
   return TXS_OK;
@@ -1103,6 +1115,7 @@ TXS_API int32_t txs_cache_n_req(const txs_kv_cache* c) { return c ? c->n_req : 0
 
 TXS_API txs_status txs_cache_read_rows(const txs_kv_cache* c, int32_t layer, int32_t which, int32_t req, int32_t row0,
                                        int32_t n_rows, void* dst, void* stream) {
+  TXS_TRACE();
   if (!c || !dst || layer < 0 || layer >= c->n_layers || which < 0 || which > 1 || req < 0 || req >= c->n_req ||
       row0 < 0 || n_rows < 0 || static_cast<long long>(row0) + n_rows > c->h_len[req])
     return TXS_ERR_INVALID_ARG;
@@ -1117,6 +1130,7 @@ TXS_API txs_status txs_cache_read_rows(const txs_kv_cache* c, int32_t layer, int
 
 TXS_API txs_status txs_cache_read_anchor(const txs_kv_cache* c, int32_t layer, int32_t which, float* dst,
                                          void* stream) {
+  TXS_TRACE();
   if (!c || !dst || which < 0 || which > 2 || (which < 2 && (layer < 0 || layer >= c->n_layers)))
     return TXS_ERR_INVALID_ARG;
   const size_t bytes = size_t(c->n_req) * (which == 2 ? c->d : c->dkv) * 4;
@@ -1126,6 +1140,7 @@ TXS_API txs_status txs_cache_read_anchor(const txs_kv_cache* c, int32_t layer, i
 }
 
 TXS_API txs_status txs_score_workspace_size(const txs_model* m, int32_t n_req, int64_t total_cand, size_t* bytes) {
+  TXS_TRACE();
   if (!m || !bytes || n_req < 0 || total_cand < 0) return TXS_ERR_INVALID_ARG;
   *bytes = score_layout(m->cfg, m->es, n_req, total_cand).total;
   return TXS_OK;
@@ -1163,6 +1178,7 @@ TXS_API txs_status txs_score_candidates(txs_model* m, const txs_kv_cache* c, int
                                         const int32_t* cand_offsets, const void* cand_tok, const void* ctx_tok,
                                         void* workspace, size_t workspace_bytes, float* out_logits, float* out_probs,
                                         void* stream) {
+  TXS_TRACE();
   return score_entry(m, c, n_req, cand_offsets, cand_tok, ctx_tok, workspace, workspace_bytes, out_logits,
                      out_probs, nullptr, stream);
 }
@@ -1172,6 +1188,7 @@ TXS_API txs_status txs_score_candidates_after(txs_model* m, const txs_kv_cache* 
                                               const void* ctx_tok, void* workspace, size_t workspace_bytes,
                                               float* out_logits, float* out_probs, void* cache_ready,
                                               void* stream) {
+  TXS_TRACE();
   return score_entry(m, c, n_req, cand_offsets, cand_tok, ctx_tok, workspace, workspace_bytes, out_logits,
                      out_probs, static_cast<cudaEvent_t>(cache_ready), stream);
 }
@@ -1201,6 +1218,7 @@ EventsLayout events_layout(const txs_config& cf, int es, int n_ev, long long n_c
 
 TXS_API txs_status txs_events_workspace_size(const txs_model* m, int32_t n_events, int64_t total_cand,
                                              int32_t max_event_end, size_t* bytes) {
+  TXS_TRACE();
   if (!m || !bytes || n_events < 0 || total_cand < 0 || max_event_end < 0) return TXS_ERR_INVALID_ARG;
   *bytes = events_layout(m->cfg, m->es, n_events, total_cand, max_event_end).total;
   return TXS_OK;
@@ -1233,6 +1251,7 @@ TXS_API txs_status txs_score_events(txs_model* m, const txs_kv_cache* c, int32_t
                                     int32_t n_events, const int32_t* event_ends, const int32_t* cand_offsets,
                                     const void* cand_tok, const void* ctx_tok, void* workspace,
                                     size_t workspace_bytes, float* out_logits, float* out_probs, void* stream) {
+  TXS_TRACE();
   if (!m || !c || !event_ends || !cand_offsets || n_events < 0) return TXS_ERR_INVALID_ARG;
   if (c->model_hash != m->hash) return TXS_ERR_STALE_CACHE;
   if (user < 0 || user >= c->n_req) return TXS_ERR_INVALID_ARG;
@@ -1267,6 +1286,7 @@ TXS_API txs_status txs_score_events(txs_model* m, const txs_kv_cache* c, int32_t
 TXS_API txs_status txs_rank_candidates(int32_t n_req, const int32_t* cand_offsets, const float* probs,
                                        int32_t n_actions, int32_t action, int32_t top_k, int32_t* out_idx,
                                        void* stream) {
+  TXS_TRACE();
   if (n_req < 0 || !cand_offsets || n_actions < 1 || action < 0 || action >= n_actions || top_k < 0)
     return TXS_ERR_INVALID_ARG;
   if (n_req == 0) return TXS_OK;
@@ -1283,6 +1303,7 @@ TXS_API txs_status txs_rank_candidates(int32_t n_req, const int32_t* cand_offset
 }
 
 TXS_API txs_status txs_device_status(txs_model* m) {
+  TXS_TRACE();
   if (!m) return TXS_ERR_INVALID_ARG;
   cudaError_t err = cudaDeviceSynchronize();
   if (err != cudaSuccess) return fail_cuda("cudaDeviceSynchronize", err);
@@ -1293,23 +1314,27 @@ TXS_API txs_status txs_device_status(txs_model* m) {
 }
 
 TXS_API txs_status txs_selftest_wait_timeout(txs_model* m, void* stream) {
+  TXS_TRACE();
   if (!m) return TXS_ERR_INVALID_ARG;
   const cudaError_t e = launch_wait_timeout_probe(m->status, static_cast<cudaStream_t>(stream));
   return e == cudaSuccess ? TXS_OK : fail_cuda("wait_timeout_probe", e);
 }
 
 TXS_API txs_status txs_gelu_eval(const float* x, float* y, int64_t n, int32_t variant, void* stream) {
+  TXS_TRACE();
   if (n < 0 || (n > 0 && (!x || !y)) || (variant != 0 && variant != 1)) return TXS_ERR_INVALID_ARG;
   const cudaError_t e = launch_gelu_eval(x, y, n, variant, static_cast<cudaStream_t>(stream));
   return e == cudaSuccess ? TXS_OK : fail_cuda("gelu_eval", e);
 }
 
 TXS_API txs_status txs_profile_enable(int32_t enable) {
+  TXS_TRACE();
   g_prof.on = enable != 0;
   return TXS_OK;
 }
 
 TXS_API txs_status txs_profile_collect(double* total_ms, int64_t* launches, int32_t n) {
+  TXS_TRACE();
   if (!total_ms || !launches || n < TXS_N_KERNEL_CLASSES) return TXS_ERR_INVALID_ARG;
   for (int i = 0; i < n; ++i) {
     total_ms[i] = 0;
@@ -1330,6 +1355,7 @@ TXS_API txs_status txs_profile_collect(double* total_ms, int64_t* launches, int3
 }
 
 TXS_API const char* txs_kernel_class_name(int32_t cls) {
+  TXS_TRACE();
   static const char* names[] = {"pack", "gemm_qkv", "attn_serving", "gemm_oproj_ln", "gemm_q", "attn_cross",
                                 "gemm_ffn1_gelu", "gemm_ffn2_ln", "gemm_kv_build", "pool", "global_kv", "rank",
                                 "misc", "row_ln", "cand_mlp", "enc_embed", "enc_gemm", "enc_attn", "head_dw",

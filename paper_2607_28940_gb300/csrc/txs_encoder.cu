@@ -356,6 +356,7 @@ void state_free(txs_enc_state* st) {
 using namespace txs;
 
 TXS_API txs_status txs_encoder_create(const txs_enc_config* cfg, const void* const* weights, txs_encoder** out) {
+  TXS_TRACE();
   if (!cfg || !weights || !out) return TXS_ERR_INVALID_ARG;
   *out = nullptr;
   std::string why;
@@ -388,6 +389,7 @@ TXS_API txs_status txs_encoder_create(const txs_enc_config* cfg, const void* con
 }
 
 TXS_API void txs_encoder_destroy(txs_encoder* m) {
+  TXS_TRACE();
   if (!m) return;
   for (void* p : m->allocs) cudaFree(p);
   delete m;
@@ -396,6 +398,7 @@ TXS_API void txs_encoder_destroy(txs_encoder* m) {
 TXS_API uint64_t txs_encoder_hash(const txs_encoder* m) { return m ? m->hash : 0; }
 
 TXS_API txs_status txs_encoder_workspace_size(const txs_encoder* m, int64_t n_rows, size_t* bytes) {
+  TXS_TRACE();
   if (!m || !bytes || n_rows < 0) return TXS_ERR_INVALID_ARG;
   *bytes = enc_ws_layout(m->cfg, m->es, n_rows).total;
   return TXS_OK;
@@ -421,6 +424,7 @@ txs_status check_call(const txs_encoder* m, int n_req, const int32_t* off, const
 TXS_API txs_status txs_encode_build(txs_encoder* m, int32_t n_req, const int32_t* offsets, const void* subj,
                                     const int32_t* types, int32_t capacity_extra, void* workspace,
                                     size_t workspace_bytes, void* phi_out, void* stream, txs_enc_state** out) {
+  TXS_TRACE();
   if (!m || !out || n_req < 1 || capacity_extra < 0 || !offsets) return TXS_ERR_INVALID_ARG;
   *out = nullptr;
   txs_status chk = check_call(m, n_req, offsets, subj, types, workspace, workspace_bytes, phi_out);
@@ -491,6 +495,7 @@ TXS_API txs_status txs_encode_build(txs_encoder* m, int32_t n_req, const int32_t
 TXS_API txs_status txs_encode_append(txs_encoder* m, txs_enc_state* st, int32_t n_req, const int32_t* new_offsets,
                                      const void* subj, const int32_t* types, void* workspace,
                                      size_t workspace_bytes, void* phi_out, void* stream) {
+  TXS_TRACE();
   if (!m || !st || !new_offsets) return TXS_ERR_INVALID_ARG;
   if (n_req != st->n_req) return TXS_ERR_INVALID_ARG;
   if (st->enc_hash != m->hash) return TXS_ERR_STALE_CACHE;
@@ -511,6 +516,7 @@ TXS_API txs_status txs_encode_append(txs_encoder* m, txs_enc_state* st, int32_t 
 }
 
 TXS_API txs_status txs_enc_state_lengths(const txs_enc_state* st, int32_t* out_len) {
+  TXS_TRACE();
   if (!st || !out_len) return TXS_ERR_INVALID_ARG;
   std::copy(st->h_len.begin(), st->h_len.end(), out_len);
   return TXS_OK;
@@ -520,6 +526,7 @@ TXS_API int32_t txs_enc_state_n_req(const txs_enc_state* st) { return st ? st->n
 
 TXS_API txs_status txs_enc_state_read_rows(const txs_enc_state* st, int32_t layer, int32_t which, int32_t req,
                                            int32_t row0, int32_t n_rows, void* dst, void* stream) {
+  TXS_TRACE();
   if (!st || !dst || layer < 0 || layer >= st->n_layers || which < 0 || which > 1 || req < 0 || req >= st->n_req ||
       row0 < 0 || n_rows < 0 || static_cast<long long>(row0) + n_rows > st->h_len[req])
     return TXS_ERR_INVALID_ARG;
@@ -533,12 +540,14 @@ TXS_API txs_status txs_enc_state_read_rows(const txs_enc_state* st, int32_t laye
 }
 
 TXS_API void txs_enc_state_destroy(txs_enc_state* st) {
+  TXS_TRACE();
   if (!st) return;
   cudaDeviceSynchronize();
   state_free(st);
 }
 
 TXS_API txs_status txs_encoder_device_status(txs_encoder* m) {
+  TXS_TRACE();
   if (!m) return TXS_ERR_INVALID_ARG;
   cudaError_t err = cudaDeviceSynchronize();
   if (err != cudaSuccess) return enc_fail("cudaDeviceSynchronize", err);

@@ -2,6 +2,7 @@
 #pragma once
 
 #include <cuda.h>
+#include <nvtx3/nvToolsExt.h>
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
@@ -11,6 +12,17 @@
 #define TXS_API extern "C" __attribute__((visibility("default")))
 
 namespace txs {
+
+// NVTX range around a public call (named after the function): it shows in a
+// profiler's timeline; without a tool attached it costs a pointer check.
+struct NvtxRange {
+  explicit NvtxRange(const char* name) { nvtxRangePushA(name); }
+  ~NvtxRange() { nvtxRangePop(); }
+  NvtxRange(const NvtxRange&) = delete;
+  NvtxRange& operator=(const NvtxRange&) = delete;
+};
+#define TXS_TRACE() ::txs::NvtxRange txs_trace_range_(__func__)
+
 
 // Device-side bounded waits give up after this many SM clock cycles (~1 s at
 // 2 GHz), latch TXS_ERR_DEVICE_TIMEOUT and let the kernel wind down.
