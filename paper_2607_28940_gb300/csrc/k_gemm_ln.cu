@@ -559,9 +559,17 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
 // With HEAD each CTA forms the partial logits z . W_eff_z of its 256 columns
 // (at most 4 actions) and sends them to the CTA of pair 0 with the same rows,
 // which adds the x part and writes logits and probabilities.
+// With RS the residual rows come through shared memory: the epilogue warp of
+// lane quarter q owns four 32-row x 64-column boxes (128-byte swizzle), and
+// after adding box c of its tile it loads box c of the CTA's next tile (TMA),
+// which the other group's warp of the same quarter reads; so every tile's
+// residual is in flight while the previous tile's epilogue runs, at the
+// price of two operand stages.
 constexpr int PBN = 256;               // columns per CTA (and per pair)
+constexpr int kResBox = 32 * 64 * 2;   // one residual box: 32 rows x 64 bf16 columns
+constexpr int kResStagedMaxK = 1024;   // longest K that takes the shared-memory residual
 
-template <int NP, bool HEAD>
+template <int NP, bool HEAD, bool RS>
 struct PairShape {
   static constexpr int CS = 2 * NP;
   static constexpr int NAP = 4;                                     // head actions padded to 4
@@ -572,7 +580,9 @@ struct PairShape {
   static constexpr int HBUF_BYTES = HEAD ? 2 * NP * 128 * NAP * 4 : 0;   // partial logits per column block
   static constexpr int WEFF_BYTES = HEAD ? PBN * NAP * 4 : 0;
   static constexpr int PAR_BYTES = 3 * PBN * 4;
-  static constexpr int EXTRA = STG_BYTES + XBUF_BYTES + HBUF_BYTES + WEFF_BYTES + PAR_BYTES + 1024 + 512;
+  static constexpr int RES_BYTES = RS ? 4 * (PBN / 64) * kResBox : 0;   // [quarter][box]
+  static constexpr int EXTRA =
+      RES_BYTES + STG_BYTES + XBUF_BYTES + HBUF_BYTES + WEFF_BYTES + PAR_BYTES + 1024 + 640;
   static constexpr int STAGES_FIT = (227 * 1024 - EXTRA) / STAGE_BYTES;
   static constexpr int STAGES = STAGES_FIT > 8 ? 8 : STAGES_FIT;
   static constexpr int SMEM_BYTES = STAGES * STAGE_BYTES + EXTRA;
@@ -580,17 +590,19 @@ struct PairShape {
   static_assert(STAGES >= 4 && SMEM_BYTES <= 232448, "shared memory");
 };
 
-template <int NP, bool HEAD>
+template <int NP, bool HEAD, bool RS>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
     gemm_ln_pair_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
-                        const __grid_constant__ CUtensorMap tmO, const EpiArgs e) {
-  using S = PairShape<NP, HEAD>;
+                        const __grid_constant__ CUtensorMap tmO, const __grid_constant__ CUtensorMap tmR,
+                        const EpiArgs e) {
+  using S = PairShape<NP, HEAD, RS>;
   constexpr int NAP = S::NAP;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* sA = smem;
   uint8_t* sB = sA + S::STAGES * A_STAGE_BYTES;
-  uint8_t* s_stage = sB + S::STAGES * S::B_STAGE_BYTES;
+  uint8_t* s_res = sB + S::STAGES * S::B_STAGE_BYTES;                                 // [4][PBN / 64] boxes
+  uint8_t* s_stage = s_res + S::RES_BYTES;
   float2* xbuf = reinterpret_cast<float2*>(s_stage + S::STG_BYTES);                 // [2][NP][128]
   float* hbuf = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(xbuf) + S::XBUF_BYTES);     // [2][NP][128][NAP]
   float* s_weff = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(hbuf) + S::HBUF_BYTES);  // [PBN][NAP]
@@ -601,7 +613,10 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   uint64_t* acc_empty = acc_full + 2;
   uint64_t* xfull = acc_empty + 2;    // [2][4]: the other pair's statistics of lane quarter q
   uint64_t* hfull = xfull + 8;        // [2][4]: the other pairs' partial logits (pair 0, HEAD)
-  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(hfull + 8);
+  uint64_t* res_full = hfull + 8;     // [4][PBN / 64]: residual box landed (RS)
+  int* res_iss = reinterpret_cast<int*>(res_full + 16);    // per box: last tile whose load was issued
+  int* res_seen = res_iss + 16;                            // per box: last tile whose load was waited for
+  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(res_seen + 16);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_holder + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -629,6 +644,10 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     for (int i = 0; i < 8; ++i) {
       mbar_init(xfull + i, 1);
       mbar_init(hfull + i, 1);
+    }
+    for (int i = 0; i < 16; ++i) {
+      mbar_init(res_full + i, 1);
+      res_iss[i] = res_seen[i] = -1;
     }
     *abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
@@ -730,19 +749,36 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     const float* s_beta = s_par + 2 * PBN;
     int kchunk = 0;
     float v[32];
+    // RS: this quarter's residual boxes; lane 0 loads box c of the rows of
+    // this CTA's tile j (rows past M read as zeros)
+    constexpr int kBoxes = PBN / 64;
+    uint8_t* res_q = s_res + q * kBoxes * kResBox;
+    uint64_t* res_bar = res_full + q * kBoxes;
+    auto res_issue = [&](int j, int c) {
+      mbar_expect_tx(res_bar + c, kResBox);
+      tma_load_2d(res_q + c * kResBox, &tmR, res_bar + c, n0 + 64 * c, (cid + j * ncl) * 2 * BM + half * BM + q * 32);
+      res_iss[q * kBoxes + c] = j;
+    };
+    if constexpr (RS) {
+      // the first tile's boxes; later ones are loaded by the previous tile's warp
+      if (grp == 0 && lane == 0 && my_tiles > 0)
+        for (int c = 0; c < kBoxes; ++c) res_issue(0, c);
+    }
     for (int i = grp; i < my_tiles; i += 2) {
       const int buf = grp, pb = grp;
       const uint32_t use = static_cast<uint32_t>(i >> 1) & 1;
       const int m0 = (cid + i * ncl) * 2 * BM + half * BM;   // this CTA's rows
       const int row = m0 + trow;
       const bool valid = row < e.M;
-      // the residual's first 64 columns are fetched before the wait, the rest
-      // one chunk ahead
+      // without RS the residual's first 64 columns are fetched before the
+      // wait, the rest one chunk ahead
       const uint4* rp = reinterpret_cast<const uint4*>(static_cast<const __nv_bfloat16*>(e.res) +
                                                        static_cast<long long>(valid ? row : 0) * e.ldr + n0);
       uint4 rres[8];
+      if constexpr (!RS) {
 #pragma unroll
-      for (int k = 0; k < 8; ++k) rres[k] = valid ? __ldg(rp + k) : make_uint4(0, 0, 0, 0);
+        for (int k = 0; k < 8; ++k) rres[k] = valid ? __ldg(rp + k) : make_uint4(0, 0, 0, 0);
+      }
       bool go = mbar_wait(acc_full + buf, use, abort_flag);
       go = __shfl_sync(0xffffffffu, go ? 1 : 0, 0) != 0;
       if (!go) break;
@@ -753,26 +789,41 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       float mean_p = 0.f, m2 = 0.f;
       // 64 columns per iteration: chunk h of 32 uses residual registers
       // rres[4 h .. 4 h + 3] (static indices), then refills them for c + 64
+      // (RS: box c64 / 64 read from shared memory when it has landed)
+      bool res_ok = true;
 #pragma unroll 1
       for (int c64 = 0; c64 < PBN; c64 += 64) {
+        if constexpr (RS) {
+          const int cb = c64 / 64;
+          res_ok = mbar_wait(res_bar + cb, static_cast<uint32_t>(i) & 1, abort_flag);
+          res_ok = __shfl_sync(0xffffffffu, res_ok ? 1 : 0, 0) != 0;
+          if (!res_ok) break;
+          if (lane == 0) res_seen[q * kBoxes + cb] = i;
+          const uint8_t* bx = res_q + cb * kResBox + lane * 128;
+#pragma unroll
+          for (int k = 0; k < 8; ++k) rres[k] = *reinterpret_cast<const uint4*>(bx + ((k ^ (lane & 7)) << 4));
+        }
 #pragma unroll
         for (int hh = 0; hh < 2; ++hh) {
           const int c = c64 + 32 * hh;
           tmem_ld32(tacc + c, v);
           float sum = 0.f;
+          const float4* b4 = reinterpret_cast<const float4*>(s_bias + c);   // broadcast 16-byte reads
 #pragma unroll
           for (int k = 0; k < 4; ++k) {
             const __nv_bfloat162* h2 = reinterpret_cast<const __nv_bfloat162*>(&rres[4 * hh + k]);
+            const float4 bl = b4[2 * k], bh = b4[2 * k + 1];
+            const float bk[8] = {bl.x, bl.y, bl.z, bl.w, bh.x, bh.y, bh.z, bh.w};
 #pragma unroll
             for (int t = 0; t < 4; ++t) {
               const float2 f = __bfloat1622float2(h2[t]);
               const int j = 8 * k + 2 * t;
-              v[j] += s_bias[c + j] + f.x;
-              v[j + 1] += s_bias[c + j + 1] + f.y;
+              v[j] += bk[2 * t] + f.x;
+              v[j + 1] += bk[2 * t + 1] + f.y;
               sum += v[j] + v[j + 1];
             }
           }
-          if (c + 64 < PBN) {
+          if (!RS && c + 64 < PBN) {
 #pragma unroll
             for (int k = 0; k < 4; ++k)
               rres[4 * hh + k] = valid ? __ldg(rp + (c + 64) / 8 + k) : make_uint4(0, 0, 0, 0);
@@ -795,7 +846,14 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             m2 = m2 + m2c + dlt * dlt * (na * 32.f / nt);
           }
         }
+        if constexpr (RS) {
+          // every lane has consumed the box: the next tile's rows go into it
+          fence_async_smem();
+          __syncwarp();
+          if (lane == 0 && i + 1 < my_tiles) res_issue(i + 1, c64 / 64);
+        }
       }
+      if (!res_ok) break;
       float mean = mean_p;
       if constexpr (NP > 1) {
         // (mean, M2) of these 256 columns to the CTAs of the other pairs that
@@ -836,8 +894,16 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
 #pragma unroll 1
       for (int c = 0; c < PBN; c += 32) {
         tmem_ld32(tacc + c, v);
+        const float4* g4 = reinterpret_cast<const float4*>(s_gamma + c);
+        const float4* e4 = reinterpret_cast<const float4*>(s_beta + c);
 #pragma unroll
-        for (int k = 0; k < 32; ++k) v[k] = (v[k] - mean) * rstd * s_gamma[c + k] + s_beta[c + k];
+        for (int k = 0; k < 8; ++k) {
+          const float4 g = g4[k], b = e4[k];
+          v[4 * k] = (v[4 * k] - mean) * rstd * g.x + b.x;
+          v[4 * k + 1] = (v[4 * k + 1] - mean) * rstd * g.y + b.y;
+          v[4 * k + 2] = (v[4 * k + 2] - mean) * rstd * g.z + b.z;
+          v[4 * k + 3] = (v[4 * k + 3] - mean) * rstd * g.w + b.w;
+        }
         if constexpr (!HEAD) {
           __nv_bfloat16* out =
               valid ? static_cast<__nv_bfloat16*>(e.out) + static_cast<long long>(row) * e.ldo + n0 + c : nullptr;
@@ -912,6 +978,13 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   }
   tc_fence_before();
   __syncthreads();
+  if constexpr (RS) {
+    // after an abort: a residual box whose load was issued but never waited
+    // for lands before the CTA exits
+    if (threadIdx.x < 16 && *abort_flag && res_iss[threadIdx.x] > res_seen[threadIdx.x])
+      mbar_wait_plain(res_full + threadIdx.x, static_cast<uint32_t>(res_iss[threadIdx.x]) & 1);
+    __syncthreads();
+  }
   cluster_sync();                     // no CTA leaves while a peer may still signal or write into it
   if (warp == 1) {
     tc_fence_after();
@@ -920,11 +993,11 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   if (threadIdx.x == 0 && *abort_flag) latch_status(e.status, TXS_ERR_DEVICE_TIMEOUT);
 }
 
-template <int NP, bool HEAD>
+template <int NP, bool HEAD, bool RS>
 static cudaError_t launch_pair(const __nv_bfloat16* A, long long lda, const __nv_bfloat16* B, const EpiArgs& e,
                                cudaStream_t s, int cls) {
-  using Sh = PairShape<NP, HEAD>;
-  auto kern = gemm_ln_pair_kernel<NP, HEAD>;
+  using Sh = PairShape<NP, HEAD, RS>;
+  auto kern = gemm_ln_pair_kernel<NP, HEAD, RS>;
   cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeClusterDimension;
   attr[0].val.clusterDim.x = Sh::CS;
@@ -950,17 +1023,20 @@ static cudaError_t launch_pair(const __nv_bfloat16* A, long long lda, const __nv
     }
     max_clusters = n;
   }
-  CUtensorMap ta, tb, to;
+  CUtensorMap ta, tb, to, tr;
   if (!make_tmap(&ta, A, e.M, e.K, lda, BM)) return cudaErrorInvalidValue;
   if (!make_tmap(&tb, B, e.N, e.K, e.K, 128)) return cudaErrorInvalidValue;
   if (HEAD) to = ta;   // unused
   else if (!make_tmap_out(&to, e.out, e.M, e.N, e.ldo)) return cudaErrorInvalidValue;
+  // residual boxes of 32 rows x 64 columns (RS)
+  if (!RS) tr = ta;   // unused
+  else if (!make_tmap(&tr, e.res, e.M, e.N, e.ldr, 32)) return cudaErrorInvalidValue;
   const int m_tiles = (e.M + 2 * BM - 1) / (2 * BM);
   const int ncl = m_tiles < max_clusters ? m_tiles : max_clusters;
   cfg.gridDim = dim3(ncl * Sh::CS);
   cfg.numAttrs = 2;
   prof_begin(cls, s);
-  cudaError_t err = cudaLaunchKernelEx(&cfg, kern, ta, tb, to, e);
+  cudaError_t err = cudaLaunchKernelEx(&cfg, kern, ta, tb, to, tr, e);
   prof_end(cls, s);
   return err;
 }
@@ -1026,10 +1102,15 @@ cudaError_t launch_gemm_ln_cluster(const __nv_bfloat16* A, long long lda, const 
     const int ncs = e.N / 128;   // CTAs per cluster either way
     if ((e.M + 2 * tc::BM - 1) / (2 * tc::BM) >= 2 * (num_sms() / ncs)) {
       if (head)
-        return e.N == 256 ? tcln::launch_pair<1, true>(A, lda, B, e, s, cls)
-                          : tcln::launch_pair<2, true>(A, lda, B, e, s, cls);
-      return e.N == 256 ? tcln::launch_pair<1, false>(A, lda, B, e, s, cls)
-                        : tcln::launch_pair<2, false>(A, lda, B, e, s, cls);
+        return e.N == 256 ? tcln::launch_pair<1, true, false>(A, lda, B, e, s, cls)
+                          : tcln::launch_pair<2, true, false>(A, lda, B, e, s, cls);
+      // short K: the residual through shared memory (the mainloop keeps
+      // up with four operand stages); long K keeps six stages
+      if (e.K <= tcln::kResStagedMaxK)
+        return e.N == 256 ? tcln::launch_pair<1, false, true>(A, lda, B, e, s, cls)
+                          : tcln::launch_pair<2, false, true>(A, lda, B, e, s, cls);
+      return e.N == 256 ? tcln::launch_pair<1, false, false>(A, lda, B, e, s, cls)
+                        : tcln::launch_pair<2, false, false>(A, lda, B, e, s, cls);
     }
   }
   // the two epilogue groups pay off once each cluster has several row tiles

@@ -308,9 +308,10 @@ __device__ __forceinline__ uint32_t tile_off(int r, int u) {
 // Row tile of tile t in the fused-attention kernel: the row tiles are
 // rotated so that the last one (the context-token rows of every request,
 // whose warps attend to many requests each) is processed in the first round
-// by the last CTAs, which have no extra tile in the last round.
-__device__ __forceinline__ int att_tile_m(int t, int n_tiles, int m_tiles) {
-  const int shift = static_cast<int>(gridDim.x) / n_tiles - 1;   // first-round position of the last row tile
+// by the last CTAs (or pairs: `slots` tiles run at once), which have no
+// extra tile in the last round.
+__device__ __forceinline__ int att_tile_m(int t, int n_tiles, int m_tiles, int slots) {
+  const int shift = slots / n_tiles - 1;   // first-round position of the last row tile
   return (t / n_tiles + m_tiles - 1 + (m_tiles - shift % m_tiles)) % m_tiles;
 }
 
@@ -554,15 +555,19 @@ __device__ __forceinline__ void att_tile(const EpiArgs& e, const AttRow& cur, co
 // cross-attention equation with the local-global key set), stored where q
 // would have gone.  The key slots of each tile's first request are copied
 // while the previous tile computes; this lane's row request for the next
-// tile is read at the start of the current one.
+// tile is read at the start of the current one.  PAIR: tiles of 256 rows on
+// a CTA pair, this CTA's 128 rows starting at rank * 128; the accumulator
+// is released on rank 0's barrier.
+template <bool PAIR>
 __device__ __forceinline__ void attn_epilogue_warp(const EpiArgs& e, uint32_t tmem_q, uint64_t* acc_full,
                                                    uint64_t* acc_empty, volatile int* abort_flag, int t_lo, int t_hi,
                                                    int t_step, int n_tiles, int m_tiles, int q, int h,
                                                    const float* bias, const CUtensorMap* tmO, uint8_t* stage,
-                                                   uint8_t* att) {
+                                                   uint8_t* att, int rank) {
   constexpr int BNA = 2 * kAttCols;
+  constexpr int TM = PAIR ? 2 * BM : BM;
   const int lane = threadIdx.x & 31;
-  auto row_of = [&](int t) { return att_tile_m(t, n_tiles, m_tiles) * BM + q * 32 + lane; };
+  auto row_of = [&](int t) { return att_tile_m(t, n_tiles, m_tiles, t_step) * TM + rank * BM + q * 32 + lane; };
   auto col_of = [&](int t) { return (t % n_tiles) * BNA + h * kAttCols; };
   // request attended by this lane's row of tile t (-1: past M, or a
   // context-token row, attended by a separate launch)
@@ -602,7 +607,10 @@ __device__ __forceinline__ void attn_epilogue_warp(const EpiArgs& e, uint32_t tm
       tmem_ld64(tmem_q + b * BNA + h * kAttCols, w);
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(acc_empty + b);              // the accumulator may be reused
+      if (lane == 0) {                                        // the accumulator may be reused
+        if constexpr (PAIR) mbar_arrive_peer_signal(map_peer(acc_empty + b, 0));
+        else mbar_arrive(acc_empty + b);
+      }
 #pragma unroll
       for (int u = 0; u < kAttCols / 8; ++u) {
         uint4 pk;
@@ -773,7 +781,10 @@ struct Shape {
   // bias read through L1 leave room for a fourth operand stage
   static constexpr bool LEAN = !BRES && !LN && !ATT && BN == 256;
   static constexpr int SBUF = (LEAN || SERVE) ? 1 : 2;    // bulk-store staging buffers per warp
-  static constexpr int STAGE_N = BRES ? kStageNRes : SERVE ? kStageNSrv : (ATT || LEAN) ? kStageNAtt : kStageN;
+  // (the fused attention on pairs reads its bias through L1: the room is a
+  // fifth operand stage)
+  static constexpr int STAGE_N = BRES ? kStageNRes : SERVE ? kStageNSrv : (ATT && PAIR) ? 0
+                                 : (ATT || LEAN) ? kStageNAtt : kStageN;
   static constexpr int AUX_BYTES =
       LN ? 0 : (((STAGE_N * 4) + (EPI == EPI_KV ? (2 * kStageSeg + 1) * 4 : 0) + 1023) / 1024) * 1024;
   // fused attention: each epilogue warp's staged window and anchor (fp32)
@@ -795,7 +806,8 @@ struct Shape {
   static_assert((RED_BYTES + WEFF_BYTES + AUX_BYTES + STG_BYTES + ATT_BYTES) % 16 == 0,
                 "mbarriers must stay 8-byte aligned");
   static_assert(!ATT || (BN == 2 * kAttCols && !BRES), "fused attention: 128-column tiles");
-  static_assert(!PAIR || (LEAN && BN == 256) || (SERVE && BN == 192), "CTA pairs: 256-column streaming tiles");
+  static_assert(!PAIR || (LEAN && BN == 256) || (SERVE && BN == 192) || (ATT && BN == 128),
+                "CTA pairs: 256-column streaming tiles and the fused attentions");
   static_assert(!SERVE || PAIR, "fused serving attention: CTA pairs");
   static_assert(SMEM_BYTES <= 232448, "shared memory");
   static_assert((TMEM_COLS & (TMEM_COLS - 1)) == 0 && TMEM_COLS <= 512, "TMEM columns");
@@ -865,7 +877,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     t_step = 1;
   }
   auto tile_n = [&](int t) { return BRES ? t / m_tiles : t % n_tiles; };
-  auto tile_m = [&](int t) { return BRES ? t % m_tiles : S::ATT ? att_tile_m(t, n_tiles, m_tiles) : t / n_tiles; };
+  auto tile_m = [&](int t) {
+    return BRES ? t % m_tiles : S::ATT ? att_tile_m(t, n_tiles, m_tiles, t_step) : t / n_tiles;
+  };
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < S::STAGES; ++s) {
@@ -1091,8 +1105,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     const int h = ew / 4;             // column half
     uint8_t* stage = s_stage + ew * S::SBUF * 2048;
     if constexpr (S::ATT) {
-      attn_epilogue_warp(e, tmem + (static_cast<uint32_t>(q * 32) << 16), acc_full, acc_empty, abort_flag, t_lo,
-                         t_hi, t_step, n_tiles, m_tiles, q, h, bias, &tmO, stage, s_att + ew * kAttWarpBytes);
+      attn_epilogue_warp<PAIR>(e, tmem + (static_cast<uint32_t>(q * 32) << 16), acc_full, acc_empty, abort_flag,
+                               t_lo, t_hi, t_step, n_tiles, m_tiles, q, h, bias, &tmO, stage,
+                               s_att + ew * kAttWarpBytes, static_cast<int>(rank));
     } else if constexpr (S::SERVE) {
       int kchunk = 0;
       int i = 0;
@@ -1404,6 +1419,10 @@ cudaError_t launch_gemm_tc(const __nv_bfloat16* A, long long lda, const __nv_bfl
       if ((e.att_dh != 32 && e.att_dh != 64) || e.att_l_local < 0 || e.att_l_local > kAttWinMax ||
           e.att_group < 1 || e.att_dkv % 8 != 0)
         return cudaErrorNotSupported;
+      // long streams of row tiles: CTA pairs (M = 256 MMAs, half the weight
+      // bytes per CTA, five operand stages)
+      if (((e.M + 255) / 256) * (e.N / 128) >= num_sms())
+        return launch_bn<128, EPI_ATTN_LG, 4, false, true>(A, lda, B, e, s, cls);
       return launch_bn<128, EPI_ATTN_LG>(A, lda, B, e, s, cls);
     case EPI_SERVE:
       if (e.srv_S < 0 || e.srv_S > kSrvMaxS || e.N != 3 * e.srv_d) return cudaErrorNotSupported;
