@@ -347,11 +347,14 @@ __device__ __forceinline__ void att_row_meta(const EpiArgs& e, AttRow& a) {
 }
 
 // K/V columns [kc0, kc0 + kvw) read by the heads of query columns
-// [col0, col0 + 64): kvw <= 64, a whole number of heads.
+// [col0, col0 + 64): kvw is 32 or 64, a whole number of heads (d_h = 32 or
+// 64, so the head index is a shift).
 __device__ __forceinline__ void att_kv_cols(const EpiArgs& e, int col0, int& kc0, int& kvw) {
-  const int dh = e.att_dh, grp = e.att_group;
-  kc0 = (col0 / dh) / grp * dh;
-  kvw = ((col0 + kAttCols - 1) / dh) / grp * dh + dh - kc0;
+  const int lg = e.att_dh == 64 ? 6 : 5, grp = e.att_group;
+  const int h0 = col0 >> lg, h1 = (col0 + kAttCols - 1) >> lg;
+  const int g0 = grp == 1 ? h0 : h0 / grp, g1 = grp == 1 ? h1 : h1 / grp;
+  kc0 = g0 << lg;
+  kvw = ((g1 - g0) << lg) + e.att_dh;
 }
 
 // Starts the asynchronous copies of request rc's key slots into buffer `buf`:
@@ -362,10 +365,10 @@ __device__ __forceinline__ void att_issue(const EpiArgs& e, int rc, int W, long 
   const __nv_bfloat16* Kc = static_cast<const __nv_bfloat16*>(e.att_k);
   const __nv_bfloat16* Vc = static_cast<const __nv_bfloat16*>(e.att_v);
   const uint32_t sK = smem_u32(buf), sV = sK + kAttKvBytes, sA = sV + kAttKvBytes;
-  const int per_row = kvw / 8;
+  const int sh = kvw == 64 ? 3 : 2;                        // 16-byte units per row: 8 or 4
   const long long dkv = e.att_dkv;
-  for (int idx = lane; idx < kAttWinMax * per_row; idx += 32) {
-    const int t = idx / per_row, u = idx - t * per_row;
+  for (int idx = lane; idx < (kAttWinMax << sh); idx += 32) {
+    const int t = idx >> sh, u = idx & ((1 << sh) - 1);
     const bool in = t < W;
     const long long src = (base + (in ? t : 0)) * dkv + kc0 + 8 * u;   // a valid row when zero-filling
     cp_async16(sK + tile_off(t, u), Kc + src, in ? 16u : 0u);
@@ -453,7 +456,8 @@ __device__ __forceinline__ void att_tile(const EpiArgs& e, const AttRow& cur, co
 #pragma unroll
     for (int hl = 0; hl < 2; ++hl) {
       if (hl >= hpw) break;
-      const int ku = (((col0 + hl * DH) / DH) / grp * DH - kc0) / 8;   // this head's first K/V unit
+      const int hq = (col0 + hl * DH) / DH;                            // this head (DH: a power of two)
+      const int ku = ((grp == 1 ? hq : hq / grp) * DH - kc0) / 8;      // its first K/V unit
       const int qu = hl * DH / 8;                                      // its first query unit
       constexpr int nks = DH / 16;                                     // k-steps of S
       // S = Q K^T: [m-tile][key tile][fragment]
@@ -611,17 +615,25 @@ __device__ __forceinline__ void attn_epilogue_warp(const EpiArgs& e, uint32_t tm
         if constexpr (PAIR) mbar_arrive_peer_signal(map_peer(acc_empty + b, 0));
         else mbar_arrive(acc_empty + b);
       }
+      // every bias read (16-byte aligned columns) before the first store, so
+      // the reads are not ordered behind the shared-memory stores
+      uint4 pk[kAttCols / 8];
+      const float4* b4 = reinterpret_cast<const float4*>(bias + col0);
 #pragma unroll
       for (int u = 0; u < kAttCols / 8; ++u) {
-        uint4 pk;
-        pk.x = pack_bf16x2(w[8 * u] + bias[col0 + 8 * u], w[8 * u + 1] + bias[col0 + 8 * u + 1]);
-        pk.y = pack_bf16x2(w[8 * u + 2] + bias[col0 + 8 * u + 2], w[8 * u + 3] + bias[col0 + 8 * u + 3]);
-        pk.z = pack_bf16x2(w[8 * u + 4] + bias[col0 + 8 * u + 4], w[8 * u + 5] + bias[col0 + 8 * u + 5]);
-        pk.w = pack_bf16x2(w[8 * u + 6] + bias[col0 + 8 * u + 6], w[8 * u + 7] + bias[col0 + 8 * u + 7]);
-        *reinterpret_cast<uint4*>(sQ + tile_off(lane, u)) = pk;
-        if (row >= e.att_n_cand && row < e.M)   // a context-token row: its q for the separate launch
-          *reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(e.att_q_ctx) + static_cast<long long>(row) * e.ldo +
-                                    col0 + 8 * u) = pk;
+        const float4 bl = b4[2 * u], bh = b4[2 * u + 1];
+        pk[u].x = pack_bf16x2(w[8 * u] + bl.x, w[8 * u + 1] + bl.y);
+        pk[u].y = pack_bf16x2(w[8 * u + 2] + bl.z, w[8 * u + 3] + bl.w);
+        pk[u].z = pack_bf16x2(w[8 * u + 4] + bh.x, w[8 * u + 5] + bh.y);
+        pk[u].w = pack_bf16x2(w[8 * u + 6] + bh.z, w[8 * u + 7] + bh.w);
+      }
+#pragma unroll
+      for (int u = 0; u < kAttCols / 8; ++u) *reinterpret_cast<uint4*>(sQ + tile_off(lane, u)) = pk[u];
+      if (row >= e.att_n_cand && row < e.M) {   // a context-token row: its q for the separate launch
+        uint4* qc = reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(e.att_q_ctx) +
+                                             static_cast<long long>(row) * e.ldo + col0);
+#pragma unroll
+        for (int u = 0; u < kAttCols / 8; ++u) qc[u] = pk[u];
       }
     }
     __syncwarp();
