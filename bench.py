@@ -50,10 +50,10 @@ FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0}
 # (workload, mode, class) -> (bytes per launch, source sha256[:12]), each from
 # one --set full capture of that class's kernel on that workload.
 NCU_TRAFFIC = {
-    # rebuild of the 262,144 rows of mid_bf16 (274.9 MB read + 2.093 GB written)
+    # rebuild of the 262,144 rows of mid_bf16 (272.7 MB read + 2.092 GB written)
     # scaled by rows to the 525,811 of ragged_bf16, plus the 512-row append
     # (4.8 MB + 0.04 MB), averaged over the two launches of a step
-    ("ragged_bf16", "local_global", "gemm_kv_build"): (2.377e+09, "e2011ec9952c"),
+    ("ragged_bf16", "local_global", "gemm_kv_build"): (2.374e+09, "d7e79a9337e8"),
     ("mid_bf16", "full", "attn_cross"): (873.9e6, "db3c1a34b26e"),
     ("sweep_bf16", "full", "attn_cross"): (317.1e6, "db3c1a34b26e"),
 }
